@@ -1,0 +1,191 @@
+"""Python binding of the fp64 CPU oracle (oracle/luna_oracle.c).
+
+TEST INFRASTRUCTURE ONLY: imported by the tests, by the graft smoke check and
+by the CPU-baseline leg of the benchmark, never by the library path.  It shares
+no code with the CUDA path; both sides only share the seeded input generator
+in `synth`.
+
+Parity pins (tests/test_oracle_pins.py): hand-computed feature maps
+(tests/golden/phi_hand.json), brute-force quadratic form of Eq. (kernel-attn),
+constant-channel closed form, Gram matrix PSD (Prop. 1), permutation/padding/
+linearity invariances, normalised weights summing to 1, causal = masked
+quadratic form, and central finite differences of every gradient.
+"""
+from __future__ import annotations
+
+import ctypes
+import os
+import subprocess
+import threading
+
+import numpy as np
+
+_HERE = os.path.dirname(os.path.abspath(__file__))
+_SRC = os.path.join(_HERE, "luna_oracle.c")
+_BUILD_DIR = os.path.join(_HERE, "_build")
+_SO = os.path.join(_BUILD_DIR, "libluna_oracle.so")
+_lock = threading.Lock()
+_lib = None
+
+
+def build(force: bool = False) -> str:
+    """Compile the oracle shared library with gcc (OpenMP when available)."""
+    os.makedirs(_BUILD_DIR, exist_ok=True)
+    if not force and os.path.exists(_SO) and os.path.getmtime(_SO) >= os.path.getmtime(_SRC):
+        return _SO
+    base = ["gcc", "-O2", "-std=c99", "-fPIC", "-shared", "-ffp-contract=off", _SRC, "-lm"]
+    tmp = _SO + f".tmp{os.getpid()}"
+    try:
+        subprocess.run(base[:-1] + ["-fopenmp", "-o", tmp, "-lm"], check=True, capture_output=True)
+    except subprocess.CalledProcessError:
+        subprocess.run(base + ["-o", tmp], check=True)
+    os.replace(tmp, _SO)
+    return _SO
+
+
+class _Phi(ctypes.Structure):
+    _fields_ = [("d", ctypes.c_int), ("M", ctypes.c_int), ("L", ctypes.c_int), ("hid", ctypes.c_int)] + [
+        (k, ctypes.c_void_p) for k in ("W", "b", "w1", "b1", "w2", "b2")
+    ]
+
+
+_P = ctypes.c_void_p
+_I = ctypes.c_int
+_D = ctypes.c_double
+_I64 = ctypes.c_int64
+
+
+def lib():
+    global _lib
+    with _lock:
+        if _lib is None:
+            so = build()
+            L = ctypes.CDLL(so)
+            phi = ctypes.POINTER(_Phi)
+            L.oracle_featmap.argtypes = [phi, _P, _I64, _P]
+            L.oracle_kink_margin.argtypes = [phi, _P, _I64, _P]
+            L.oracle_psi.argtypes = [phi, _I, _D]
+            L.oracle_psi.restype = _D
+            L.oracle_attn_fwd.argtypes = [phi, _I, _I, _I, _I, _I, _D, _P, _P, _P, _P, _P]
+            L.oracle_attn_quadratic.argtypes = [phi, _I, _I, _I, _I, _I, _D, _P, _P, _P, _P, _P]
+            L.oracle_attn_bwd.argtypes = [phi, _I, _I, _I, _I, _I, _D, _P, _P, _P, _P, _P, _P, _P, _P] + [_P] * 6
+            L.oracle_max_threads.restype = _I
+            L.oracle_set_threads.argtypes = [_I]
+            _lib = L
+    return _lib
+
+
+def max_threads() -> int:
+    return lib().oracle_max_threads()
+
+
+def set_threads(t: int) -> None:
+    lib().oracle_set_threads(int(t))
+
+
+def _f64(a) -> np.ndarray:
+    return np.ascontiguousarray(a, dtype=np.float64)
+
+
+class PhiParams:
+    """fp64 copies of the feature-map parameters (W, b, w1, b1, w2, b2)."""
+
+    def __init__(self, params: dict):
+        self.arrays = {k: _f64(params[k]) for k in ("W", "b", "w1", "b1", "w2", "b2")}
+        W = self.arrays["W"]
+        self.M, self.d = W.shape
+        self.L, self.hid = self.arrays["w1"].shape
+        assert self.arrays["b"].shape == (self.M,)
+        assert self.arrays["b1"].shape == self.arrays["w2"].shape == (self.L, self.hid)
+        assert self.arrays["b2"].shape == (self.L,)
+        self.struct = _Phi(self.d, self.M, self.L, self.hid,
+                           *[self.arrays[k].ctypes.data for k in ("W", "b", "w1", "b1", "w2", "b2")])
+
+    @property
+    def D(self) -> int:
+        return self.M * self.L
+
+    def ref(self):
+        return ctypes.byref(self.struct)
+
+
+def _as_params(params) -> PhiParams:
+    return params if isinstance(params, PhiParams) else PhiParams(params)
+
+
+def featmap(params, X) -> np.ndarray:
+    """phi(X) for rows of X (..., d) -> (..., M*L), feature index i*L + l."""
+    p = _as_params(params)
+    X = _f64(X)
+    rows = X.size // p.d
+    out = np.empty(X.shape[:-1] + (p.D,), dtype=np.float64)
+    lib().oracle_featmap(p.ref(), X.ctypes.data, rows, out.ctypes.data)
+    return out
+
+
+def kink_margin(params, X) -> np.ndarray:
+    p = _as_params(params)
+    X = _f64(X)
+    out = np.empty(X.shape[:-1], dtype=np.float64)
+    lib().oracle_kink_margin(p.ref(), X.ctypes.data, X.size // p.d, out.ctypes.data)
+    return out
+
+
+def psi(params, l: int, u: float) -> float:
+    p = _as_params(params)
+    return lib().oracle_psi(p.ref(), int(l), float(u))
+
+
+def _lens(lengths, B):
+    if lengths is None:
+        return None, 0
+    a = np.ascontiguousarray(lengths, dtype=np.int32)
+    assert a.shape == (B,)
+    return a, a.ctypes.data
+
+
+def attn_fwd(params, Q, K, V, lengths=None, causal=False, eps=1e-6) -> np.ndarray:
+    """Linear (sufficient statistics) form; Q, K (B,H,n,d), V (B,H,n,dv)."""
+    p = _as_params(params)
+    Q, K, V = _f64(Q), _f64(K), _f64(V)
+    B, H, n, d = Q.shape
+    dv = V.shape[-1]
+    assert d == p.d and K.shape == Q.shape and V.shape[:3] == Q.shape[:3]
+    la, lp = _lens(lengths, B)
+    O = np.empty(V.shape, dtype=np.float64)
+    lib().oracle_attn_fwd(p.ref(), B, H, n, dv, int(bool(causal)), float(eps),
+                          Q.ctypes.data, K.ctypes.data, V.ctypes.data, lp, O.ctypes.data)
+    return O
+
+
+def attn_quadratic(params, Q, K, V, lengths=None, causal=False, eps=1e-6) -> np.ndarray:
+    """Brute force: O_i = sum_j k(q_i,k_j) v_j / (sum_j k(q_i,k_j) + eps)."""
+    p = _as_params(params)
+    Q, K, V = _f64(Q), _f64(K), _f64(V)
+    B, H, n, d = Q.shape
+    dv = V.shape[-1]
+    la, lp = _lens(lengths, B)
+    O = np.empty(V.shape, dtype=np.float64)
+    lib().oracle_attn_quadratic(p.ref(), B, H, n, dv, int(bool(causal)), float(eps),
+                                Q.ctypes.data, K.ctypes.data, V.ctypes.data, lp, O.ctypes.data)
+    return O
+
+
+def attn_bwd(params, Q, K, V, dO, lengths=None, causal=False, eps=1e-6) -> dict:
+    """Gradients of sum(O * dO) w.r.t. Q, K, V and every feature-map parameter."""
+    p = _as_params(params)
+    Q, K, V, dO = _f64(Q), _f64(K), _f64(V), _f64(dO)
+    B, H, n, d = Q.shape
+    dv = V.shape[-1]
+    la, lp = _lens(lengths, B)
+    out = {
+        "dQ": np.empty(Q.shape), "dK": np.empty(K.shape), "dV": np.empty(V.shape),
+        "dW": np.empty((p.M, p.d)), "db": np.empty((p.M,)),
+        "dw1": np.empty((p.L, p.hid)), "db1": np.empty((p.L, p.hid)),
+        "dw2": np.empty((p.L, p.hid)), "db2": np.empty((p.L,)),
+    }
+    lib().oracle_attn_bwd(p.ref(), B, H, n, dv, int(bool(causal)), float(eps),
+                          Q.ctypes.data, K.ctypes.data, V.ctypes.data, dO.ctypes.data, lp,
+                          out["dQ"].ctypes.data, out["dK"].ctypes.data, out["dV"].ctypes.data,
+                          *[out[k].ctypes.data for k in ("dW", "db", "dw1", "db1", "dw2", "db2")])
+    return out

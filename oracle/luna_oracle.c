@@ -1,0 +1,408 @@
+/*
+ * LUNA oracle: a plain, slow fp64 CPU restatement of the method.
+ *
+ * TEST INFRASTRUCTURE ONLY.  Nothing in the library path may call, link or
+ * execute this file; only the tests, the graft smoke check and the CPU
+ * baseline leg of the benchmark use it.  It shares no code, header, table or
+ * constant with the CUDA path.
+ *
+ * What it computes (paper: "LUNA: Linear Universal Neural Attention", arXiv
+ * 2512.08061):
+ *   - the feature map of Eq. (phi-def-scalarenv) with the default "no gate"
+ *     envelope h = 1 of Sec. 5.4 / Table 5, scale 1/sqrt(M), projection bias b
+ *     and per-channel scalar MLPs psi_l(u) = relu(fc2(relu(fc1(u)))) as in the
+ *     appendix listing (TaskSpecificProjections, ScalarMLP, MLPLearnable-
+ *     FeatureMap).  Feature index i*L + l (projection-major).
+ *   - kernelized linear attention, Eq. (kernel-attn):
+ *       O_i = phi(q_i)^T S / (phi(q_i)^T z + eps),  S = sum_j phi(k_j) v_j^T,
+ *       z = sum_j phi(k_j); rows/keys at or beyond a sequence's valid length
+ *       are excluded (keys) and produce 0 (queries).
+ *   - the streaming (causal) form named in the abstract and Sec. 3.2: the same
+ *     with the sums over j <= i, evaluated as a sequential prefix recurrence.
+ *   - the brute-force quadratic form sum_j k(q_i,k_j) v_j / (sum_j k + eps)
+ *     with k(x,y) = phi(x)^T phi(y) (Eq. kernel-attn read right to left).
+ *   - the backward pass by the direct chain rule, sample by sample through
+ *     every hidden unit of every channel MLP (ReLU'(0) taken as 0).
+ *
+ * Parity pinned by the CPU tests: hand-computed feature maps, the brute-force
+ * quadratic form, closed-form special cases (constant channels give a plain
+ * mean), the positive semi-definite Gram matrix of Prop. 1, invariances, and
+ * central finite differences of the backward pass.
+ */
+#include <math.h>
+#include <stdint.h>
+#include <stdlib.h>
+#include <string.h>
+#ifdef _OPENMP
+#include <omp.h>
+#endif
+
+typedef struct {
+    int d;            /* width of a query/key row                        */
+    int M;            /* number of projections (rows of W)               */
+    int L;            /* number of channel functions psi_l               */
+    int hid;          /* hidden width of each channel MLP                */
+    const double *W;  /* M x d                                           */
+    const double *b;  /* M                                               */
+    const double *w1; /* L x hid, fc1 weight of channel l (fan-in 1)     */
+    const double *b1; /* L x hid                                         */
+    const double *w2; /* L x hid, fc2 weight of channel l (fan-out 1)    */
+    const double *b2; /* L                                               */
+} oracle_phi;
+
+typedef struct {
+    double *dW, *db, *dw1, *db1, *dw2, *db2;
+} oracle_grads;
+
+static double relu(double x) { return x > 0.0 ? x : 0.0; }
+
+int oracle_max_threads(void) {
+#ifdef _OPENMP
+    return omp_get_max_threads();
+#else
+    return 1;
+#endif
+}
+
+void oracle_set_threads(int t) {
+#ifdef _OPENMP
+    if (t > 0) omp_set_num_threads(t);
+#else
+    (void)t;
+#endif
+}
+
+/* u_i = w_i^T x + b_i  (listing: TaskSpecificProjections.forward) */
+static double project(const oracle_phi *p, int i, const double *x) {
+    double u = p->b[i];
+    for (int c = 0; c < p->d; ++c) u += p->W[(size_t)i * p->d + c] * x[c];
+    return u;
+}
+
+/* y_l(u) = fc2(relu(fc1(u))) before the non-negativity ReLU (listing: ScalarMLP) */
+static double channel_pre(const oracle_phi *p, int l, double u) {
+    const double *w1 = p->w1 + (size_t)l * p->hid;
+    const double *b1 = p->b1 + (size_t)l * p->hid;
+    const double *w2 = p->w2 + (size_t)l * p->hid;
+    double y = p->b2[l];
+    for (int k = 0; k < p->hid; ++k) y += w2[k] * relu(w1[k] * u + b1[k]);
+    return y;
+}
+
+double oracle_psi(const oracle_phi *p, int l, double u) { return relu(channel_pre(p, l, u)); }
+
+/* phi(x) = (1/sqrt(M)) [psi_l(w_i^T x + b_i)]_{i,l},  index i*L + l */
+static void phi_row(const oracle_phi *p, const double *x, double *out) {
+    const double s = 1.0 / sqrt((double)p->M);
+    for (int i = 0; i < p->M; ++i) {
+        double u = project(p, i, x);
+        for (int l = 0; l < p->L; ++l) out[i * p->L + l] = s * relu(channel_pre(p, l, u));
+    }
+}
+
+void oracle_featmap(const oracle_phi *p, const double *X, int64_t rows, double *Phi) {
+    const int D = p->M * p->L;
+#pragma omp parallel for schedule(static)
+    for (int64_t r = 0; r < rows; ++r) phi_row(p, X + r * p->d, Phi + r * D);
+}
+
+/* Smallest relative distance of any ReLU argument of the feature map of a row
+ * from its kink (inner hidden units and outer non-negativity ReLU).  Where it
+ * is at rounding level the gradient of that row is not unique. */
+void oracle_kink_margin(const oracle_phi *p, const double *X, int64_t rows, double *margin) {
+#pragma omp parallel for schedule(static)
+    for (int64_t r = 0; r < rows; ++r) {
+        const double *x = X + r * p->d;
+        double m = INFINITY;
+        for (int i = 0; i < p->M; ++i) {
+            double u = project(p, i, x);
+            for (int l = 0; l < p->L; ++l) {
+                const double *w1 = p->w1 + (size_t)l * p->hid;
+                const double *b1 = p->b1 + (size_t)l * p->hid;
+                const double *w2 = p->w2 + (size_t)l * p->hid;
+                double y = p->b2[l], ysc = fabs(p->b2[l]);
+                for (int k = 0; k < p->hid; ++k) {
+                    double a = w1[k] * u + b1[k];
+                    double sc = fabs(w1[k] * u) + fabs(b1[k]);
+                    if (w1[k] != 0.0 && sc > 0.0) {
+                        double rel = fabs(a) / sc;
+                        if (rel < m) m = rel;
+                    }
+                    y += w2[k] * relu(a);
+                    ysc += fabs(w2[k] * relu(a));
+                }
+                if (ysc > 0.0) {
+                    double rel = fabs(y) / ysc;
+                    if (rel < m) m = rel;
+                }
+            }
+        }
+        margin[r] = m;
+    }
+}
+
+/* Backward of phi for `rows` rows: given dPhi, writes dX and accumulates the
+ * parameter gradients into g, by the chain rule through every hidden unit. */
+static void phi_rows_backward(const oracle_phi *p, const double *X, int64_t rows, const double *dPhi,
+                              double *dX, oracle_grads *g) {
+    const int D = p->M * p->L, d = p->d;
+    const double s = 1.0 / sqrt((double)p->M);
+    for (int64_t r = 0; r < rows; ++r) {
+        const double *x = X + r * d;
+        double *dx = dX + r * d;
+        for (int c = 0; c < d; ++c) dx[c] = 0.0;
+        for (int i = 0; i < p->M; ++i) {
+            double u = project(p, i, x);
+            double du = 0.0;
+            for (int l = 0; l < p->L; ++l) {
+                double y = channel_pre(p, l, u);
+                if (!(y > 0.0)) continue; /* outer ReLU inactive */
+                double dy = dPhi[r * D + i * p->L + l] * s;
+                if (dy == 0.0) continue;
+                const double *w1 = p->w1 + (size_t)l * p->hid;
+                const double *b1 = p->b1 + (size_t)l * p->hid;
+                const double *w2 = p->w2 + (size_t)l * p->hid;
+                g->db2[l] += dy;
+                for (int k = 0; k < p->hid; ++k) {
+                    double a = w1[k] * u + b1[k];
+                    if (!(a > 0.0)) continue;
+                    g->dw2[(size_t)l * p->hid + k] += dy * a;
+                    double dh = dy * w2[k];
+                    g->dw1[(size_t)l * p->hid + k] += dh * u;
+                    g->db1[(size_t)l * p->hid + k] += dh;
+                    du += dh * w1[k];
+                }
+            }
+            g->db[i] += du;
+            for (int c = 0; c < d; ++c) {
+                g->dW[(size_t)i * d + c] += du * x[c];
+                dx[c] += du * p->W[(size_t)i * d + c];
+            }
+        }
+    }
+}
+
+static int head_len(const int32_t *lengths, int b, int n) {
+    if (!lengths) return n;
+    int len = lengths[b];
+    if (len < 0) len = 0;
+    if (len > n) len = n;
+    return len;
+}
+
+/* ------------------------------------------------------------------------ */
+/* forward, linear (sufficient-statistics) form                              */
+
+static void attn_fwd_head(const oracle_phi *p, int n, int dv, int causal, double eps, const double *Q,
+                          const double *K, const double *V, int len, double *O) {
+    const int D = p->M * p->L, d = p->d;
+    double *phq = (double *)malloc(sizeof(double) * D);
+    double *phk = (double *)malloc(sizeof(double) * D);
+    double *S = (double *)calloc((size_t)D * dv, sizeof(double));
+    double *z = (double *)calloc((size_t)D, sizeof(double));
+    memset(O, 0, sizeof(double) * (size_t)n * dv);
+    if (!causal) {
+        for (int j = 0; j < len; ++j) {
+            phi_row(p, K + (size_t)j * d, phk);
+            for (int f = 0; f < D; ++f) {
+                z[f] += phk[f];
+                for (int c = 0; c < dv; ++c) S[(size_t)f * dv + c] += phk[f] * V[(size_t)j * dv + c];
+            }
+        }
+    }
+    for (int i = 0; i < len; ++i) {
+        if (causal) { /* S_i = S_{i-1} + phi(k_i) v_i^T, z_i likewise */
+            phi_row(p, K + (size_t)i * d, phk);
+            for (int f = 0; f < D; ++f) {
+                z[f] += phk[f];
+                for (int c = 0; c < dv; ++c) S[(size_t)f * dv + c] += phk[f] * V[(size_t)i * dv + c];
+            }
+        }
+        phi_row(p, Q + (size_t)i * d, phq);
+        double den = eps;
+        for (int f = 0; f < D; ++f) den += phq[f] * z[f];
+        if (den == 0.0) continue;
+        for (int c = 0; c < dv; ++c) {
+            double num = 0.0;
+            for (int f = 0; f < D; ++f) num += phq[f] * S[(size_t)f * dv + c];
+            O[(size_t)i * dv + c] = num / den;
+        }
+    }
+    free(phq); free(phk); free(S); free(z);
+}
+
+void oracle_attn_fwd(const oracle_phi *p, int B, int H, int n, int dv, int causal, double eps, const double *Q,
+                     const double *K, const double *V, const int32_t *lengths, double *O) {
+    const int d = p->d;
+#pragma omp parallel for schedule(dynamic, 1)
+    for (int bh = 0; bh < B * H; ++bh) {
+        int b = bh / H;
+        size_t qo = (size_t)bh * n * d, vo = (size_t)bh * n * dv;
+        attn_fwd_head(p, n, dv, causal, eps, Q + qo, K + qo, V + vo, head_len(lengths, b, n), O + vo);
+    }
+}
+
+/* ------------------------------------------------------------------------ */
+/* forward, brute-force quadratic form                                        */
+
+void oracle_attn_quadratic(const oracle_phi *p, int B, int H, int n, int dv, int causal, double eps,
+                           const double *Q, const double *K, const double *V, const int32_t *lengths,
+                           double *O) {
+    const int D = p->M * p->L, d = p->d;
+#pragma omp parallel for schedule(dynamic, 1)
+    for (int bh = 0; bh < B * H; ++bh) {
+        int len = head_len(lengths, bh / H, n);
+        const double *q = Q + (size_t)bh * n * d, *k = K + (size_t)bh * n * d, *v = V + (size_t)bh * n * dv;
+        double *o = O + (size_t)bh * n * dv;
+        double *PQ = (double *)malloc(sizeof(double) * (size_t)(len > 0 ? len : 1) * D);
+        double *PK = (double *)malloc(sizeof(double) * (size_t)(len > 0 ? len : 1) * D);
+        for (int i = 0; i < len; ++i) {
+            phi_row(p, q + (size_t)i * d, PQ + (size_t)i * D);
+            phi_row(p, k + (size_t)i * d, PK + (size_t)i * D);
+        }
+        memset(o, 0, sizeof(double) * (size_t)n * dv);
+        for (int i = 0; i < len; ++i) {
+            double den = eps;
+            int jmax = causal ? i + 1 : len;
+            double *acc = o + (size_t)i * dv;
+            for (int j = 0; j < jmax; ++j) {
+                double kij = 0.0; /* k(q_i, k_j) = phi(q_i)^T phi(k_j) */
+                for (int f = 0; f < D; ++f) kij += PQ[(size_t)i * D + f] * PK[(size_t)j * D + f];
+                den += kij;
+                for (int c = 0; c < dv; ++c) acc[c] += kij * v[(size_t)j * dv + c];
+            }
+            if (den == 0.0) {
+                for (int c = 0; c < dv; ++c) acc[c] = 0.0;
+            } else {
+                for (int c = 0; c < dv; ++c) acc[c] /= den;
+            }
+        }
+        free(PQ); free(PK);
+    }
+}
+
+/* ------------------------------------------------------------------------ */
+/* backward                                                                  */
+
+static void attn_bwd_head(const oracle_phi *p, int n, int dv, int causal, double eps, const double *Q,
+                          const double *K, const double *V, const double *dO, int len, double *dQ, double *dK,
+                          double *dV, oracle_grads *g) {
+    const int D = p->M * p->L, d = p->d;
+    size_t nl = (size_t)(len > 0 ? len : 1);
+    double *PQ = (double *)malloc(sizeof(double) * nl * D);
+    double *PK = (double *)malloc(sizeof(double) * nl * D);
+    double *dPQ = (double *)calloc(nl * D, sizeof(double));
+    double *dPK = (double *)calloc(nl * D, sizeof(double));
+    double *dnum = (double *)calloc(nl * dv, sizeof(double));
+    double *dden = (double *)calloc(nl, sizeof(double));
+    double *S = (double *)calloc((size_t)D * dv, sizeof(double));
+    double *z = (double *)calloc((size_t)D, sizeof(double));
+    double *o = (double *)malloc(sizeof(double) * dv);
+    memset(dQ, 0, sizeof(double) * (size_t)n * d);
+    memset(dK, 0, sizeof(double) * (size_t)n * d);
+    memset(dV, 0, sizeof(double) * (size_t)n * dv);
+    for (int i = 0; i < len; ++i) {
+        phi_row(p, Q + (size_t)i * d, PQ + (size_t)i * D);
+        phi_row(p, K + (size_t)i * d, PK + (size_t)i * D);
+    }
+    if (!causal) {
+        for (int j = 0; j < len; ++j)
+            for (int f = 0; f < D; ++f) {
+                z[f] += PK[(size_t)j * D + f];
+                for (int c = 0; c < dv; ++c) S[(size_t)f * dv + c] += PK[(size_t)j * D + f] * V[(size_t)j * dv + c];
+            }
+    }
+    /* query side: o_i, dnum_i = do_i/den_i, dden_i = -(do_i . o_i)/den_i,
+     * dphi(q_i) = S_i dnum_i + z_i dden_i */
+    for (int i = 0; i < len; ++i) {
+        if (causal)
+            for (int f = 0; f < D; ++f) {
+                z[f] += PK[(size_t)i * D + f];
+                for (int c = 0; c < dv; ++c) S[(size_t)f * dv + c] += PK[(size_t)i * D + f] * V[(size_t)i * dv + c];
+            }
+        const double *pq = PQ + (size_t)i * D;
+        double den = eps;
+        for (int f = 0; f < D; ++f) den += pq[f] * z[f];
+        if (den == 0.0) continue;
+        double dot = 0.0;
+        for (int c = 0; c < dv; ++c) {
+            double num = 0.0;
+            for (int f = 0; f < D; ++f) num += pq[f] * S[(size_t)f * dv + c];
+            o[c] = num / den;
+            dot += dO[(size_t)i * dv + c] * o[c];
+        }
+        dden[i] = -dot / den;
+        for (int c = 0; c < dv; ++c) dnum[(size_t)i * dv + c] = dO[(size_t)i * dv + c] / den;
+        for (int f = 0; f < D; ++f) {
+            double acc = z[f] * dden[i];
+            for (int c = 0; c < dv; ++c) acc += S[(size_t)f * dv + c] * dnum[(size_t)i * dv + c];
+            dPQ[(size_t)i * D + f] = acc;
+        }
+    }
+    /* key side: G_j = sum_{i >= j (or all i)} phi(q_i) dnum_i^T, g_j likewise with dden;
+     * dv_j = G_j^T phi(k_j), dphi(k_j) = G_j v_j + g_j */
+    double *G = S, *gz = z; /* reuse storage */
+    memset(G, 0, sizeof(double) * (size_t)D * dv);
+    memset(gz, 0, sizeof(double) * (size_t)D);
+    if (!causal) {
+        for (int i = 0; i < len; ++i)
+            for (int f = 0; f < D; ++f) {
+                gz[f] += PQ[(size_t)i * D + f] * dden[i];
+                for (int c = 0; c < dv; ++c) G[(size_t)f * dv + c] += PQ[(size_t)i * D + f] * dnum[(size_t)i * dv + c];
+            }
+    }
+    for (int j = len - 1; j >= 0; --j) {
+        if (causal)
+            for (int f = 0; f < D; ++f) {
+                gz[f] += PQ[(size_t)j * D + f] * dden[j];
+                for (int c = 0; c < dv; ++c) G[(size_t)f * dv + c] += PQ[(size_t)j * D + f] * dnum[(size_t)j * dv + c];
+            }
+        const double *pk = PK + (size_t)j * D;
+        for (int c = 0; c < dv; ++c) {
+            double acc = 0.0;
+            for (int f = 0; f < D; ++f) acc += G[(size_t)f * dv + c] * pk[f];
+            dV[(size_t)j * dv + c] = acc;
+        }
+        for (int f = 0; f < D; ++f) {
+            double acc = gz[f];
+            for (int c = 0; c < dv; ++c) acc += G[(size_t)f * dv + c] * V[(size_t)j * dv + c];
+            dPK[(size_t)j * D + f] = acc;
+        }
+    }
+    phi_rows_backward(p, Q, len, dPQ, dQ, g);
+    phi_rows_backward(p, K, len, dPK, dK, g);
+    free(PQ); free(PK); free(dPQ); free(dPK); free(dnum); free(dden); free(S); free(z); free(o);
+}
+
+void oracle_attn_bwd(const oracle_phi *p, int B, int H, int n, int dv, int causal, double eps, const double *Q,
+                     const double *K, const double *V, const double *dO, const int32_t *lengths, double *dQ,
+                     double *dK, double *dV, double *dW, double *db, double *dw1, double *db1, double *dw2,
+                     double *db2) {
+    const int d = p->d, M = p->M, L = p->L, hid = p->hid;
+    const size_t nW = (size_t)M * d, nb = M, nh = (size_t)L * hid, nb2 = L;
+    const size_t per = nW + nb + 3 * nh + nb2;
+    const int BH = B * H;
+    double *part = (double *)calloc((size_t)BH * per, sizeof(double));
+#pragma omp parallel for schedule(dynamic, 1)
+    for (int bh = 0; bh < BH; ++bh) {
+        double *base = part + (size_t)bh * per;
+        oracle_grads g = {base, base + nW, base + nW + nb, base + nW + nb + nh, base + nW + nb + 2 * nh,
+                          base + nW + nb + 3 * nh};
+        size_t qo = (size_t)bh * n * d, vo = (size_t)bh * n * dv;
+        attn_bwd_head(p, n, dv, causal, eps, Q + qo, K + qo, V + vo, dO + vo, head_len(lengths, bh / H, n),
+                      dQ + qo, dK + qo, dV + vo, &g);
+    }
+    /* ordered reduction over heads */
+    double *outs[6] = {dW, db, dw1, db1, dw2, db2};
+    size_t sizes[6] = {nW, nb, nh, nh, nh, nb2};
+    size_t off = 0;
+    for (int t = 0; t < 6; ++t) {
+        for (size_t e = 0; e < sizes[t]; ++e) {
+            double acc = 0.0;
+            for (int bh = 0; bh < BH; ++bh) acc += part[(size_t)bh * per + off + e];
+            outs[t][e] = acc;
+        }
+        off += sizes[t];
+    }
+    free(part);
+}

@@ -1,0 +1,44 @@
+"""The oracle pins are sensitive: plausible mistakes planted in a temporary
+copy of the oracle source (on the CPU) make at least one pin fail."""
+import os
+import shutil
+import subprocess
+import sys
+
+import pytest
+
+ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+
+MUTANTS = {
+    "dropped 1/sqrt(M) scale": (
+        "const double s = 1.0 / sqrt((double)p->M);\n    for (int i = 0; i < p->M; ++i) {\n        double u = project(p, i, x);",
+        "const double s = 1.0;\n    for (int i = 0; i < p->M; ++i) {\n        double u = project(p, i, x);"),
+    "dropped projection bias": ("double u = p->b[i];", "double u = 0.0;"),
+    "channel-major feature order": ("out[i * p->L + l]", "out[l * p->M + i]"),
+    "wrong sign of d(den)": ("dden[i] = -dot / den;", "dden[i] = dot / den;"),
+    "exclusive causal mask": ("int jmax = causal ? i + 1 : len;", "int jmax = causal ? i : len;"),
+    "fc2 weight gradient without activation": (
+        "g->dw2[(size_t)l * p->hid + k] += dy * a;", "g->dw2[(size_t)l * p->hid + k] += dy;"),
+    "eps dropped from the linear form": (
+        "double den = eps;\n        for (int f = 0; f < D; ++f) den += phq[f] * z[f];",
+        "double den = 0;\n        for (int f = 0; f < D; ++f) den += phq[f] * z[f];"),
+    "transposed state index": (
+        "for (int f = 0; f < D; ++f) num += phq[f] * S[(size_t)f * dv + c];",
+        "for (int f = 0; f < D; ++f) num += phq[f] * S[(size_t)c * D + f];"),
+    "inner ReLU mask dropped in backward": ("if (!(a > 0.0)) continue;\n                    g->dw2", "g->dw2"),
+}
+
+
+@pytest.mark.parametrize("name", sorted(MUTANTS))
+def test_planted_mistake_is_caught(name, tmp_path):
+    src = open(os.path.join(ROOT, "oracle", "luna_oracle.c")).read()
+    a, b = MUTANTS[name]
+    assert a in src, f"mutation site for {name!r} not found"
+    work = tmp_path / "w"
+    shutil.copytree(os.path.join(ROOT, "oracle"), work / "oracle", ignore=shutil.ignore_patterns("_build", "__pycache__"))
+    shutil.copytree(os.path.join(ROOT, "synth"), work / "synth", ignore=shutil.ignore_patterns("__pycache__"))
+    shutil.copytree(os.path.join(ROOT, "tests"), work / "tests", ignore=shutil.ignore_patterns("__pycache__"))
+    (work / "oracle" / "luna_oracle.c").write_text(src.replace(a, b, 1))
+    r = subprocess.run([sys.executable, "-m", "pytest", "-q", "-x", "-p", "no:cacheprovider",
+                        "tests/test_oracle_pins.py"], cwd=str(work), capture_output=True, text=True, timeout=600)
+    assert r.returncode != 0, f"mutant {name!r} survived the pins:\n{r.stdout[-2000:]}"
