@@ -1,0 +1,424 @@
+#!/usr/bin/env python3
+"""Throughput of the LUNA attention hot path on GB300 (one JSON line on stdout).
+
+A step is one pass of the whole path over one batch of synthetic input: the
+feature-map table is prepared from the parameters, the forward pass runs
+(saving the key statistics) and the backward pass produces dQ, dK, dV and the
+parameter gradients.  The default workload is the Long-Range-Arena-shaped
+encoder attention (B=32, H=4, n=4096, d=32, D=64, bf16 I/O, valid lengths
+uniform in [2048, 4096]).  Tokens per step = B * n.
+
+  python bench.py [--gpus N] [--steps K] [--warmup W] [--workload NAME] [--impl reference]
+
+Multi-GPU (torchrun): every rank runs an independent replica of the workload
+(the (batch, head) units are independent; there is no data-path collective),
+so scaling is weak and value = all ranks' tokens / max-over-ranks time.
+`--impl reference` times the fp64 CPU oracle instead (rank 0 only), on a
+bounded sample of the same workload.
+"""
+from __future__ import annotations
+
+import argparse
+import json
+import math
+import os
+import statistics
+import subprocess
+import sys
+import tempfile
+import time
+
+import numpy as np
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+sys.path.insert(0, ROOT)
+
+import synth  # noqa: E402
+from synth.workloads import WORKLOADS  # noqa: E402
+
+METRIC = "LUNA attn tokens/sec fwd & fwd+bwd on 1 GB300; % of HBM/tensor roofline"
+L2_BYTES = 129 * 1024 * 1024
+
+
+def parse():
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=100)
+    ap.add_argument("--warmup", type=int, default=5)
+    ap.add_argument("--workload", default="lra", choices=sorted(WORKLOADS))
+    ap.add_argument("--impl", default="gb300", choices=["gb300", "reference"])
+    ap.add_argument("--no-e2e", action="store_true")
+    ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--cpu-seconds", type=float, default=12.0, help="target CPU work of the oracle sample")
+    return ap.parse_args()
+
+
+def dist_env():
+    return int(os.environ.get("RANK", 0)), int(os.environ.get("LOCAL_RANK", 0)), int(os.environ.get("WORLD_SIZE", 1))
+
+
+def peaks():
+    try:
+        with open(os.path.join(ROOT, "MEASURED_PEAKS.json")) as f:
+            p = json.load(f)
+        return float(p["hbm_gbs"]), float(p["bf16_tflops"]), "measured"
+    except Exception:
+        return 6800.0, 1900.0, "fallback"
+
+
+# --------------------------------------------------------------------------
+# algorithmic bytes and flops ("Roofline accounting")
+
+def row_counts(w, lengths):
+    valid = int(np.sum(lengths)) * w.H if lengths is not None else w.B * w.H * w.n
+    return valid, w.B * w.H * w.n
+
+
+def kernel_bytes(w, lengths, kernel: str) -> float:
+    """Algorithmic HBM bytes of one launch of a kernel: every valid input row
+    read once, every output row written once (padded output rows are written
+    as zeros), the (D x dv + D) fp32 statistics per head read or written once."""
+    eb = 4 if w.io == "f32" else 2
+    valid, total = row_counts(w, lengths)
+    stats = w.B * w.H * (w.D * w.dv + w.D) * 4
+    rd, rv = w.d * eb, w.dv * eb
+    table = {
+        "keystats": valid * (rd + rv) + stats,
+        "query": valid * rd + total * rv + stats,
+        "bwd_query": valid * (rd + rv) + total * rd + 2 * stats,
+        "bwd_key": valid * (rd + rv) + total * (rd + rv) + stats,
+        "causal_out": valid * (2 * rd + rv) + total * rv,
+    }
+    return float(table.get(kernel, 0.0))
+
+
+def step_bytes(w, lengths) -> float:
+    eb = 4 if w.io == "f32" else 2
+    valid, total = row_counts(w, lengths)
+    fwd = valid * (2 * w.d + w.dv) * eb + total * w.dv * eb
+    bwd = valid * (2 * w.d + 2 * w.dv) * eb + total * (2 * w.d + w.dv) * eb
+    return float(fwd + bwd) if w.backward else float(fwd)
+
+
+def step_flops(w, lengths) -> float:
+    """Tensor-core flops of the recurrent minimum per valid row (Sec. 4 runtime
+    model): forward 4Md + 4Dd + 4D, backward 12Md + 10Dd + 6D (both sides)."""
+    valid, _ = row_counts(w, lengths)
+    f = 4 * w.M * w.d + 4 * w.D * w.dv + 4 * w.D
+    b = 12 * w.M * w.d + 10 * w.D * w.dv + 6 * w.D
+    return float(valid * (f + (b if w.backward else 0)))
+
+
+# --------------------------------------------------------------------------
+# clocks during the timed region
+
+class ClockSampler:
+    FIELDS = ("clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,clocks_event_reasons.hw_slowdown,"
+              "clocks_event_reasons.hw_thermal_slowdown,clocks_event_reasons.sw_thermal_slowdown,"
+              "clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, gpu_index: str):
+        self.proc = None
+        self.path = None
+        try:
+            fd, self.path = tempfile.mkstemp(suffix=".csv")
+            os.close(fd)
+            self.fh = open(self.path, "w")
+            self.proc = subprocess.Popen(["nvidia-smi", f"--query-gpu={self.FIELDS}", "--format=csv,noheader,nounits",
+                                          "-i", gpu_index, "-lms", "50"], stdout=self.fh,
+                                         stderr=subprocess.DEVNULL)
+        except Exception:
+            self.proc = None
+
+    def stop(self):
+        if self.proc is None:
+            return None
+        self.proc.terminate()
+        try:
+            self.proc.wait(timeout=5)
+        except Exception:
+            self.proc.kill()
+        self.fh.close()
+        rows = []
+        for line in open(self.path):
+            parts = [p.strip() for p in line.split(",")]
+            if len(parts) == 8:
+                rows.append(parts)
+        os.unlink(self.path)
+        if not rows:
+            return None
+        sm = [float(r[0]) for r in rows if r[0].replace(".", "").isdigit()]
+        smax = [float(r[1]) for r in rows if r[1].replace(".", "").isdigit()]
+        names = ("hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap")
+        reasons = sorted({names[i] for r in rows for i in range(4) if r[4 + i].lower().startswith("active")})
+        return {"sm_mhz": statistics.median(sm) if sm else None, "sm_max_mhz": max(smax) if smax else None,
+                "reasons": reasons, "samples": len(rows)}
+
+
+# --------------------------------------------------------------------------
+# the GPU arm
+
+def host_inputs(w):
+    inp = synth.attn_inputs(w.seed, w.B, w.H, w.n, w.d, w.dv, w.io, w.qkv_scale, w.len_range, with_grad=w.backward)
+    params = synth.phi_params(w.seed, w.d, w.M, w.L, w.hidden)
+    return inp, params
+
+
+def run_gpu(args, w):
+    import torch
+    import torch.distributed as tdist
+
+    rank, local_rank, world = dist_env()
+    torch.cuda.set_device(local_rank)
+    if world > 1:
+        tdist.init_process_group("nccl", device_id=torch.device("cuda", local_rank))
+    from paper_2512_08061_gb300 import build
+    if rank == 0 or world == 1:
+        build.build()
+    if world > 1:
+        tdist.barrier()
+    import paper_2512_08061_gb300.luna as L
+
+    dev = torch.device("cuda", local_rank)
+    inp, params = host_inputs(w)
+    io_dtype = torch.float32 if w.io == "f32" else torch.bfloat16
+
+    def pinned(t):
+        if t.io == "f32":
+            h = torch.from_numpy(np.ascontiguousarray(t.raw))
+        else:
+            h = torch.from_numpy(np.ascontiguousarray(t.raw).view(np.int16)).view(torch.bfloat16)
+        return h.pin_memory()
+
+    host = {k: pinned(inp[k]) for k in ("Q", "K", "V", "dO") if k in inp}
+    lengths_h = None if inp["lengths"] is None else torch.from_numpy(inp["lengths"]).pin_memory()
+    devt = {k: v.to(dev, non_blocking=True) for k, v in host.items()}
+    lengths_d = None if lengths_h is None else lengths_h.to(dev)
+    params_d = {k: torch.from_numpy(v).to(dev) for k, v in params.items()}
+    lu = L.Luna(w.B, w.H, w.n, w.d, w.dv, w.M, w.L, w.hidden, w.causal, w.eps, io_dtype, w.chunk, dev)
+    O = torch.empty_like(devt["V"])
+    grads = None
+    if w.backward:
+        f32 = dict(dtype=torch.float32, device=dev)
+        grads = {"dQ": torch.empty_like(devt["Q"]), "dK": torch.empty_like(devt["K"]), "dV": torch.empty_like(devt["V"]),
+                 "dW": torch.empty(w.M, w.d, **f32), "db": torch.empty(w.M, **f32),
+                 "dw1": torch.empty(w.L, w.hidden, **f32), "db1": torch.empty(w.L, w.hidden, **f32),
+                 "dw2": torch.empty(w.L, w.hidden, **f32), "db2": torch.empty(w.L, **f32)}
+    flush = torch.empty(2 * L2_BYTES, dtype=torch.uint8, device=dev)
+    stream = torch.cuda.current_stream()
+
+    def step(t, backward=w.backward):
+        lu.prepare(params_d)
+        lu.forward(t["Q"], t["K"], t["V"], lengths_d, O=O, save_state=True)
+        if backward:
+            lu.backward(t["Q"], t["K"], t["V"], t["dO"], lengths_d, use_state=True, out=grads)
+
+    def timed(n_steps, fn):
+        """Per-step CUDA-event times with an L2 flush (outside the events) before each step."""
+        evs = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)) for _ in range(n_steps)]
+        for s0, s1 in evs:
+            flush.zero_()
+            s0.record(stream)
+            fn()
+            s1.record(stream)
+        torch.cuda.synchronize()
+        return sum(s0.elapsed_time(s1) for s0, s1 in evs)
+
+    for _ in range(max(args.warmup, 3)):
+        step(devt)
+    torch.cuda.synchronize()
+
+    # dominant kernel: the library kernel with the largest device time in one step
+    kernels = ["phi_prepare", "keystats", "query", "bwd_query", "bwd_key", "grad_sum", "mlp_grads",
+               "causal_out", "causal_bwd_seg", "causal_dq", "causal_dkv"] + L.TC_KERNELS
+    per_kernel = {}
+    for k in kernels:
+        L.luna_profile_start(k)
+        step(devt)
+        ms, n = L.luna_profile_stop()
+        if n:
+            per_kernel[k] = ms / n
+    dominant = max(per_kernel, key=per_kernel.get) if per_kernel else None
+
+    # timed region
+    if world > 1:
+        tdist.barrier()
+    torch.cuda.synchronize()
+    uuid = str(getattr(torch.cuda.get_device_properties(local_rank), "uuid", "") or "")
+    clocks = ClockSampler(("GPU-" + uuid if uuid and not uuid.startswith("GPU-") else uuid) or str(local_rank))
+    if dominant:
+        L.luna_profile_start(dominant)
+    n0 = L.luna_launch_count()
+    ms_total = timed(args.steps, lambda: step(devt))
+    launches = L.luna_launch_count() - n0
+    dom_ms, dom_n = L.luna_profile_stop() if dominant else (0.0, 0)
+    clk = clocks.stop()
+    torch.cuda.synchronize()
+    ms_step = ms_total / args.steps
+    if world > 1:
+        t = torch.tensor([ms_step], device=dev)
+        tdist.all_reduce(t, op=tdist.ReduceOp.MAX)
+        ms_step = float(t.item())
+
+    # forward-only throughput (same flush discipline)
+    fwd_ms = timed(args.steps, lambda: step(devt, backward=False)) / args.steps
+    if world > 1:
+        t = torch.tensor([fwd_ms], device=dev)
+        tdist.all_reduce(t, op=tdist.ReduceOp.MAX)
+        fwd_ms = float(t.item())
+
+    # end to end through the public API with host buffers
+    e2e = None
+    if not args.no_e2e:
+        out_host = {"O": torch.empty(O.shape, dtype=O.dtype).pin_memory()}
+        if grads:
+            for k, v in grads.items():
+                out_host[k] = torch.empty(v.shape, dtype=v.dtype).pin_memory()
+        bi = sum(v.numel() * v.element_size() for v in host.values()) + (
+            lengths_h.numel() * 4 if lengths_h is not None else 0)
+        bo = sum(v.numel() * v.element_size() for v in out_host.values())
+
+        def e2e_step():
+            t = {k: host[k].to(dev, non_blocking=True) for k in host}
+            if lengths_h is not None:
+                lengths_d.copy_(lengths_h, non_blocking=True)
+            step(t)
+            out_host["O"].copy_(O, non_blocking=True)
+            if grads:
+                for k, v in grads.items():
+                    out_host[k].copy_(v, non_blocking=True)
+
+        for _ in range(2):
+            e2e_step()
+        torch.cuda.synchronize()
+        e2e_ms = timed(max(3, args.steps // 4), e2e_step) / max(3, args.steps // 4)
+        if world > 1:
+            t = torch.tensor([e2e_ms], device=dev)
+            tdist.all_reduce(t, op=tdist.ReduceOp.MAX)
+            e2e_ms = float(t.item())
+        e2e = {"value": w.tokens * world / (e2e_ms * 1e-3), "unit": "tokens/s", "h2d_bytes_per_step": int(bi),
+               "d2h_bytes_per_step": int(bo), "ms_per_step": e2e_ms}
+
+    hbm, tflops, peak_src = peaks()
+    lengths = inp["lengths"]
+    roof = None
+    if dominant and dom_n:
+        byts = kernel_bytes(w, lengths, dominant)
+        dur = dom_ms / dom_n * 1e-3
+        achieved = byts / dur / 1e9 if byts else None
+        roof = {"bound": "hbm", "kernel": dominant, "achieved": achieved, "peak": hbm, "unit": "GB/s",
+                "frac": (achieved / hbm) if achieved else None, "traffic": None, "peak_source": peak_src,
+                "algorithmic_bytes": byts, "launch_ms": dom_ms / dom_n, "launches": dom_n}
+    sb, sf = step_bytes(w, lengths), step_flops(w, lengths)
+    t_roof = max(sb / (hbm * 1e9), sf / (tflops * 1e12))
+    result = {
+        "metric": METRIC,
+        "value": w.tokens * world / (ms_step * 1e-3),
+        "unit": "tokens/s",
+        "n_gpus": world,
+        "steps": args.steps,
+        "warmup": args.warmup,
+        "ms_per_step": ms_step,
+        "higher_is_better": True,
+        "scaling": "weak",
+        "vs_baseline": None,
+        "dtype": w.io,
+        "data": "synthetic",
+        "config": {"workload": f"{w.name}: B={w.B} H={w.H} n={w.n} d={w.d} D={w.D} (M={w.M}, L={w.L}), "
+                               f"{w.io}, {'causal' if w.causal else 'non-causal'}, "
+                               f"{'fwd+bwd' if w.backward else 'fwd'}"
+                               + (f", lengths U[{w.len_range[0]},{w.len_range[1]}]" if w.len_range else ""),
+                   "global_batch": w.B * world, "seq_len": w.n, "parallelism": f"replicas{world}",
+                   "l2": "flushed before every timed step (2x L2 buffer written outside the events)"},
+        "fwd": {"value": w.tokens * world / (fwd_ms * 1e-3), "unit": "tokens/s", "ms_per_step": fwd_ms},
+        "step_roofline": {"bytes": sb, "tensor_flops": sf, "time_ms": t_roof * 1e3,
+                          "frac": t_roof * 1e3 / ms_step},
+        "roofline": roof,
+        "per_kernel_ms": per_kernel,
+        "e2e": e2e,
+        "gpu_launches": int(launches),
+        "clocks": clk,
+    }
+    if rank == 0 and world == 1 and not args.no_cpu_baseline:
+        result["cpu_baseline"] = cpu_baseline(w, args.cpu_seconds)
+    if world > 1:
+        tdist.destroy_process_group()
+    return result if rank == 0 else None
+
+
+# --------------------------------------------------------------------------
+# the CPU oracle (reported baseline, and the --impl reference arm)
+
+def oracle_run(w, units: int) -> float:
+    """Runs the fp64 oracle (fwd, and bwd for training workloads) on the first
+    `units` (batch, head) units of the workload's own input streams; returns
+    the wall time in seconds."""
+    import oracle
+    ln = None
+    if w.len_range is not None:
+        ln = synth.randint(w.seed, "attn.lengths", (w.B,), w.len_range[0], w.len_range[1]).astype(np.int32)
+    # (units, 1, n, d) has the same flat order as the first `units` heads of (B, H, n, d)
+    shape = (units, 1, w.n, w.d)
+    Q = synth.IOTensor(synth.normal(w.seed, "attn.Q", shape) * w.qkv_scale, w.io).value
+    K = synth.IOTensor(synth.normal(w.seed, "attn.K", shape) * w.qkv_scale, w.io).value
+    V = synth.IOTensor(synth.normal(w.seed, "attn.V", (units, 1, w.n, w.dv)) * w.qkv_scale, w.io).value
+    dO = synth.IOTensor(synth.normal(w.seed, "attn.dO", (units, 1, w.n, w.dv)), w.io).value if w.backward else None
+    lengths = None if ln is None else np.array([ln[(u // w.H) % w.B] for u in range(units)], dtype=np.int32)
+    p = oracle.PhiParams(synth.phi_params(w.seed, w.d, w.M, w.L, w.hidden))
+    t0 = time.perf_counter()
+    oracle.attn_fwd(p, Q, K, V, lengths, w.causal, w.eps)
+    if w.backward:
+        oracle.attn_bwd(p, Q, K, V, dO, lengths, w.causal, w.eps)
+    return time.perf_counter() - t0
+
+
+def tokens_per_s(w, units, seconds) -> float:
+    # one step = B*H units = B*n tokens
+    return w.n / (w.H * seconds / units)
+
+
+def cpu_baseline(w, target_s):
+    import oracle
+    threads = oracle.max_threads()
+    t1 = oracle_run(w, threads)
+    units = int(min(max(threads, threads * round(target_s / max(t1, 1e-3))), 4 * w.B * w.H))
+    t = oracle_run(w, units) if units != threads else t1
+    return {"value": tokens_per_s(w, units, t), "unit": "tokens/s", "cores": threads, "kind": "oracle",
+            "sample": f"{units} (batch, head) units of {w.n} tokens, fwd{'+bwd' if w.backward else ''}, "
+                      f"{t:.1f} s on {threads} threads, scaled to B*H={w.B * w.H} units per step"}
+
+
+def run_reference(args, w):
+    rank, _, world = dist_env()
+    if rank != 0:
+        return None
+    import oracle
+    threads = oracle.max_threads()
+    if args.warmup > 0:
+        oracle_run(w, 1)
+    per = []
+    for _ in range(args.steps):
+        t = oracle_run(w, threads)
+        per.append(tokens_per_s(w, threads, t))
+    value = statistics.median(per)
+    sample = f"{threads} (batch, head) units of {w.n} tokens per step on {threads} threads"
+    return {"metric": METRIC, "value": value, "unit": "tokens/s", "n_gpus": world, "steps": args.steps,
+            "warmup": args.warmup, "ms_per_step": w.tokens / value * 1e3, "higher_is_better": True,
+            "scaling": "weak", "vs_baseline": None, "dtype": "f64", "data": "synthetic", "impl": "reference",
+            "config": {"workload": f"{w.name}: B={w.B} H={w.H} n={w.n} d={w.d} D={w.D}, fp64 CPU oracle",
+                       "global_batch": w.B, "seq_len": w.n, "parallelism": "cpu"},
+            "cpu_baseline": {"value": value, "unit": "tokens/s", "cores": threads, "kind": "oracle",
+                             "sample": sample},
+            "e2e": {"value": value, "unit": "tokens/s", "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}}
+
+
+def main():
+    args = parse()
+    w = WORKLOADS[args.workload]
+    res = run_reference(args, w) if args.impl == "reference" else run_gpu(args, w)
+    if res is not None:
+        print(json.dumps(res), flush=True)
+
+
+if __name__ == "__main__":
+    main()

@@ -1,0 +1,191 @@
+/*
+ * luna.h — C ABI of the GB300 (sm_103a) LUNA attention library.
+ *
+ * LUNA (arXiv 2512.08061) is kernelized linear attention with a learned
+ * feature map
+ *
+ *     phi(x) = (1/sqrt(M)) [ psi_l(w_i^T x + b_i) ]_{i<M, l<L}  in R^{D},  D = M*L
+ *
+ * (Eq. phi-def-scalarenv with the default envelope h = 1 of Sec. 5.4 /
+ * Table 5; projection bias b and feature index i*L + l as in the appendix
+ * listing), where each channel function is a scalar ReLU MLP
+ *
+ *     psi_l(u) = relu( sum_k w2[l,k] relu(w1[l,k] u + b1[l,k]) + b2[l] )
+ *
+ * (listing: ScalarMLP with hidden width `hidden`, act = ReLU, nonneg = True,
+ * one MLP per channel).  Attention is Eq. (kernel-attn):
+ *
+ *     O_i = phi(q_i)^T S / (phi(q_i)^T z + eps),  S = sum_j phi(k_j) v_j^T,  z = sum_j phi(k_j)
+ *
+ * with the sums over all valid keys (non-causal) or over j <= i (the streaming
+ * form named in the abstract and Sec. 3.2).  S and z are the key-side
+ * sufficient statistics S_KV and S_K1 of Sec. 4.
+ *
+ * Conventions for every entry point:
+ *   - All tensor pointers are DEVICE pointers owned by the caller.  The
+ *     library never allocates device memory and keeps no state between calls
+ *     except a per-process cache of the driver entry point it needs for TMA.
+ *   - Q, K, dQ, dK are contiguous (B, H, n, d); V, O, dO, dV are contiguous
+ *     (B, H, n, dv), element type `io` (fp32 or bf16).  Row-major, C order.
+ *   - `lengths` is NULL (every sequence has n valid tokens) or a device array
+ *     of B int32 valid lengths (right padding).  Values are clamped to [0, n].
+ *     Keys at or beyond the length do not enter S and z; query rows at or
+ *     beyond it produce O = 0 and receive dQ = dK = dV = 0.
+ *   - `stream` is a cudaStream_t passed as void* (NULL = legacy default stream).
+ *     Every call only enqueues work on it and returns without synchronising.
+ *   - Argument errors are reported before anything is launched.  A failed
+ *     launch returns LUNA_ERR_CUDA.  Device-side bounded waits that gave up
+ *     are reported by luna_device_status().
+ *   - Computation: the feature map is evaluated in fp32 for both io types
+ *     (the listing casts the projections to float before the channel MLPs).
+ *     Accumulations are fp32.  With io = bf16 the tensor-core contractions take
+ *     bf16 operands; the normaliser phi(q)^T z is always an fp32 dot product.
+ */
+#ifndef LUNA_H
+#define LUNA_H
+
+#include <stddef.h>
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+typedef enum {
+    LUNA_OK = 0,
+    LUNA_ERR_INVALID_ARG = 1,    /* NULL pointer, negative size, bad enum            */
+    LUNA_ERR_UNSUPPORTED = 2,    /* valid but outside the supported shape range     */
+    LUNA_ERR_WORKSPACE = 3,      /* workspace / table / state buffer too small      */
+    LUNA_ERR_CUDA = 4,           /* a CUDA runtime call or launch failed            */
+    LUNA_ERR_DEVICE_TIMEOUT = 5  /* a bounded device-side wait gave up              */
+} luna_status;
+
+typedef enum { LUNA_F32 = 0, LUNA_BF16 = 1 } luna_dtype;
+
+/* Shape of the feature map (Eq. phi-def-scalarenv; listing defaults hidden = 64).
+ * Supported: 1 <= M, 1 <= L <= 16, M*L <= 128, 1 <= hidden <= 128, L*hidden <= 512. */
+typedef struct {
+    int M;      /* number of projections w_i (rows of W)       */
+    int L;      /* number of channel functions psi_l           */
+    int hidden; /* hidden width of each channel MLP            */
+} luna_phi_desc;
+
+/* Feature-map parameters, fp32 device arrays, row-major:
+ *   W [M][d], b [M], w1 [L][hidden], b1 [L][hidden], w2 [L][hidden], b2 [L].
+ * w1[l][k], b1[l][k] are fc1 of channel l (Linear(1, hidden)); w2[l][k], b2[l]
+ * are its fc2 (Linear(hidden, 1)). The same parameters serve queries and keys
+ * and are shared by all heads (listing: "shared ... over tokens/heads"). */
+typedef struct {
+    const float *W, *b, *w1, *b1, *w2, *b2;
+} luna_phi_params;
+
+/* Gradients of the feature-map parameters, fp32 device arrays with the shapes
+ * of luna_phi_params.  They are OVERWRITTEN (not accumulated) by luna_attn_bwd. */
+typedef struct {
+    float *dW, *db, *dw1, *db1, *dw2, *db2;
+} luna_phi_grads;
+
+/* Problem description (Sec. 3.1: Q, K in R^{n x d}; Sec. 4: values of width d_v).
+ * Supported: 1 <= d, dv <= 128; B, H, n >= 0 (an empty problem is a no-op).
+ * causal = 1 selects the streaming form (sums over j <= i).  chunk is the
+ * causal chunk length (0 selects 64; otherwise 16..128, multiple of 16).
+ * eps >= 0 guards the row normaliser: O_i = num_i / (den_i + eps); a row
+ * whose guarded normaliser is exactly 0 produces O_i = 0 and zero gradients. */
+typedef struct {
+    int B, H, n, d, dv;
+    int causal;
+    int chunk;
+    float eps;
+    luna_dtype io;
+} luna_attn_desc;
+
+/* Human-readable name of a status code (static string, never NULL). */
+const char *luna_status_string(luna_status s);
+
+/* Bytes of the prepared feature-map table for this descriptor and input width d
+ * (written to *bytes).  The table is an opaque device blob produced by
+ * luna_phi_prepare and consumed by every other call. */
+luna_status luna_phi_table_size(const luna_phi_desc *pd, int d, size_t *bytes);
+
+/* Builds the feature-map table from the parameters (Eq. phi-def-scalarenv,
+ * listing ScalarMLP): a copy of W and b, and for every channel the exact
+ * piecewise-linear form of psi_l.  A ReLU MLP of a scalar is linear between
+ * the kinks t = -b1/w1 of its hidden units, so on the merged, sorted kink list
+ * psi_l(u) = relu(alpha_{l,j} u + beta_{l,j}) on interval j.  Kinks are
+ * placed at the exact fp32 thresholds of fma(w1, u, b1) > 0, so the interval
+ * decides every hidden unit exactly as an fp32 evaluation of fc1 would.
+ * `table` is a device buffer of at least luna_phi_table_size bytes, 256-byte
+ * aligned; it must not be modified while a call that reads it is in flight.
+ * Parameters must be finite. */
+luna_status luna_phi_prepare(const luna_phi_desc *pd, int d, const luna_phi_params *params, void *table,
+                             size_t table_bytes, void *stream);
+
+/* phi(X) for `rows` rows of width d (Eq. phi-def-scalarenv).
+ * X: device, rows x d of type `xtype`; Phi: device fp32, rows x (M*L), feature
+ * index i*L + l.  Debug / interoperability entry point: the attention calls
+ * never materialise phi in memory. */
+luna_status luna_featmap(const luna_phi_desc *pd, int d, const void *table, const void *X, luna_dtype xtype,
+                         int64_t rows, float *Phi, void *stream);
+
+/* Bytes of scratch memory the calls need (written to *bytes).  `backward`
+ * selects the requirement of luna_attn_bwd (0 = luna_attn_fwd).  The caller
+ * owns the workspace; its contents on entry are irrelevant and on exit are
+ * unspecified.  Must be 256-byte aligned. */
+luna_status luna_workspace_size(const luna_attn_desc *ad, const luna_phi_desc *pd, int backward, size_t *bytes);
+
+/* Bytes of the optional forward state (the key statistics S, z of Sec. 4 per
+ * head; for the causal form, the prefix statistics at every state segment). */
+luna_status luna_state_size(const luna_attn_desc *ad, const luna_phi_desc *pd, size_t *bytes);
+
+/* Forward pass, Eq. (kernel-attn) (causal: streaming form).
+ * Q, K, V, lengths, O as in the conventions above.  `table` from
+ * luna_phi_prepare.  `state` is NULL or a device buffer of luna_state_size
+ * bytes that receives the key statistics for a later luna_attn_bwd.
+ * `workspace` holds ws_bytes >= luna_workspace_size(ad, pd, 0). */
+luna_status luna_attn_fwd(const luna_attn_desc *ad, const luna_phi_desc *pd, const void *table, const void *Q,
+                          const void *K, const void *V, const int32_t *lengths, void *O, void *state,
+                          void *workspace, size_t ws_bytes, void *stream);
+
+/* Backward pass of luna_attn_fwd: given dO = dLoss/dO, writes dQ, dK, dV and
+ * the parameter gradients `grads` (overwritten) of the same loss.
+ * `state` is NULL (the key statistics are recomputed from K and V) or the
+ * state written by luna_attn_fwd on the same Q, K, V, lengths and table.
+ * The derivative of each ReLU at 0 is taken as 0.  Parameter gradients are
+ * summed over all heads, rows and projections. */
+luna_status luna_attn_bwd(const luna_attn_desc *ad, const luna_phi_desc *pd, const void *table, const void *Q,
+                          const void *K, const void *V, const void *dO, const int32_t *lengths,
+                          const void *state, void *dQ, void *dK, void *dV, const luna_phi_grads *grads,
+                          void *workspace, size_t ws_bytes, void *stream);
+
+/* Synchronises `stream`, then reads and clears the device status word at the
+ * start of `workspace`.  Every luna_attn_fwd / luna_attn_bwd call clears the
+ * word when it starts; a device-side wait of that call that ran out of its
+ * iteration limit sets it (the kernel then abandons its work and returns, so
+ * the outputs of that call are undefined).  So this reports the LAST call that
+ * used this workspace: LUNA_OK, LUNA_ERR_DEVICE_TIMEOUT, or LUNA_ERR_CUDA if
+ * synchronising or the copy failed (including an earlier asynchronous fault). */
+luna_status luna_device_status(void *workspace, void *stream);
+
+/* Kernel timing (tracing aid, not needed for computation).  After
+ * luna_profile_start(name), every launch of the library kernel `name` (e.g.
+ * "bwd_query", "keystats"; the names are listed in the library's kernel
+ * launch sites) is bracketed by two CUDA events recorded on the stream it is
+ * launched on, up to 4096 launches.  luna_profile_stop waits for the recorded
+ * events and returns the summed launch durations in milliseconds and the
+ * number of launches, then stops recording.  Process-wide; one kernel name at
+ * a time. */
+luna_status luna_profile_start(const char *kernel);
+luna_status luna_profile_stop(double *total_ms, int *launches);
+
+/* Number of kernels this library has launched in this process since it was
+ * loaded (all entry points, all streams). */
+uint64_t luna_launch_count(void);
+
+/* Library version, e.g. 100 for 0.1.0. */
+int luna_version(void);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* LUNA_H */

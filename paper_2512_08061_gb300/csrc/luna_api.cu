@@ -1,0 +1,330 @@
+// C ABI of the LUNA library: argument checks, work planning, dispatch.
+#include <math.h>
+#include <string.h>
+
+#include <algorithm>
+
+#include "luna_simt.cuh"
+#include "luna_tc.cuh"
+
+using namespace luna;
+
+namespace {
+
+constexpr size_t kMaxSmem = 227 * 1024;
+
+int64_t cdiv(int64_t a, int64_t b) { return (a + b - 1) / b; }
+int64_t round_up(int64_t a, int64_t b) { return cdiv(a, b) * b; }
+
+luna_status check_phi(const luna_phi_desc *pd, int d) {
+    if (!pd) return LUNA_ERR_INVALID_ARG;
+    if (pd->M < 1 || pd->L < 1 || pd->hidden < 1 || d < 1) return LUNA_ERR_INVALID_ARG;
+    if (pd->L > kMaxL || pd->M * pd->L > kMaxFeat || pd->M > 32 || pd->hidden > kMaxHidden ||
+        pd->L * pd->hidden > kMaxUnits || d > kMaxD || pd->M * d > 4096)
+        return LUNA_ERR_UNSUPPORTED;
+    return LUNA_OK;
+}
+
+struct Plan {
+    TableLayout lay;
+    int BH = 0;
+    int nsplit = 0, rps = 0, nsplit_b = 0, rps_b = 0;
+    int seg_len = 0, nseg = 0;
+    int gsize = 0;
+    // workspace offsets (bytes)
+    size_t o_counters = 0, o_status = 0, o_Spart = 0, o_zpart = 0, o_Sfin = 0, o_zfin = 0;
+    size_t o_dSpart = 0, o_dzpart = 0, o_dSfin = 0, o_dzfin = 0, o_gpart = 0, o_hist = 0;
+    size_t o_segS = 0, o_segz = 0, o_segdS = 0, o_segdz = 0, o_rowstat = 0;
+    size_t ws_fwd = 0, ws_bwd = 0, state_bytes = 0;
+    TcPlan tc;
+};
+
+struct Bump {
+    size_t n = 0;
+    size_t take(size_t bytes) {
+        size_t o = n;
+        n += (bytes + 255) & ~size_t(255);
+        return o;
+    }
+};
+
+luna_status make_plan(const luna_attn_desc *ad, const luna_phi_desc *pd, Plan &p) {
+    if (!ad) return LUNA_ERR_INVALID_ARG;
+    if (ad->B < 0 || ad->H < 0 || ad->n < 0 || ad->d < 1 || ad->dv < 1) return LUNA_ERR_INVALID_ARG;
+    if (ad->io != LUNA_F32 && ad->io != LUNA_BF16) return LUNA_ERR_INVALID_ARG;
+    if (ad->causal != 0 && ad->causal != 1) return LUNA_ERR_INVALID_ARG;
+    if (!(ad->eps >= 0.0f) || isinf(ad->eps)) return LUNA_ERR_INVALID_ARG;
+    if (ad->chunk != 0 && (ad->chunk < 16 || ad->chunk > 128 || ad->chunk % 16 != 0)) return LUNA_ERR_INVALID_ARG;
+    luna_status st = check_phi(pd, ad->d);
+    if (st != LUNA_OK) return st;
+    if (ad->dv > kMaxD || ad->n > (1 << 24)) return LUNA_ERR_UNSUPPORTED;
+    if ((int64_t)ad->B * ad->H > (1 << 24)) return LUNA_ERR_UNSUPPORTED;
+
+    p.lay = table_layout(pd->M, pd->L, pd->hidden, ad->d);
+    const int BH = ad->B * ad->H, n = ad->n, D = p.lay.D, dv = ad->dv;
+    p.BH = BH;
+    p.gsize = pd->M * ad->d + pd->M + p.lay.nint * pd->L * 2;
+    if (BH == 0 || n == 0) return LUNA_OK;
+    // splits depend only on the descriptor, so workspace sizes are reproducible
+    {
+        int64_t target = std::max<int64_t>(1, cdiv(1216, BH));
+        int64_t ns = std::min<int64_t>(target, cdiv(n, 32));
+        p.rps = (int)round_up(cdiv(n, ns), 32);
+        p.nsplit = (int)cdiv(n, p.rps);
+        int64_t tb = std::max<int64_t>(1, cdiv(608, BH));
+        int64_t nb = std::min<int64_t>(tb, cdiv(n, 16));
+        p.rps_b = (int)round_up(cdiv(n, nb), 16);
+        p.nsplit_b = (int)cdiv(n, p.rps_b);
+        int64_t nc = std::min<int64_t>(std::min<int64_t>(target, 64), cdiv(n, 16));
+        p.seg_len = (int)round_up(cdiv(n, nc), 64);
+        p.nseg = (int)cdiv(n, p.seg_len);
+    }
+    const size_t f = sizeof(float);
+    const size_t SD = (size_t)D * dv;
+    Bump w;
+    p.o_status = w.take(sizeof(int));  // offset 0: device status word of the last call
+    p.o_counters = w.take(2 * (size_t)BH * sizeof(int));
+    if (!ad->causal) {
+        p.o_Spart = w.take((size_t)BH * p.nsplit * SD * f);
+        p.o_zpart = w.take((size_t)BH * p.nsplit * D * f);
+        p.o_Sfin = w.take((size_t)BH * SD * f);
+        p.o_zfin = w.take((size_t)BH * D * f);
+        p.ws_fwd = w.n;
+        p.o_dSpart = w.take((size_t)BH * p.nsplit_b * SD * f);
+        p.o_dzpart = w.take((size_t)BH * p.nsplit_b * D * f);
+        p.o_dSfin = w.take((size_t)BH * SD * f);
+        p.o_dzfin = w.take((size_t)BH * D * f);
+        p.o_gpart = w.take(2 * (size_t)BH * p.nsplit_b * p.gsize * f);
+        p.o_hist = w.take((size_t)p.gsize * f);
+        p.ws_bwd = w.n;
+        p.state_bytes = (size_t)BH * (SD + D) * f;
+    } else {
+        const int ns = p.nseg;
+        p.o_Spart = w.take((size_t)BH * ns * SD * f);
+        p.o_zpart = w.take((size_t)BH * ns * D * f);
+        p.o_segS = w.take((size_t)BH * (ns + 1) * SD * f);
+        p.o_segz = w.take((size_t)BH * (ns + 1) * D * f);
+        p.ws_fwd = w.n;
+        p.o_dSpart = w.take((size_t)BH * ns * SD * f);
+        p.o_dzpart = w.take((size_t)BH * ns * D * f);
+        p.o_segdS = w.take((size_t)BH * ns * SD * f);
+        p.o_segdz = w.take((size_t)BH * ns * D * f);
+        p.o_rowstat = w.take((size_t)BH * n * 2 * f);
+        p.o_gpart = w.take(2 * (size_t)BH * ns * p.gsize * f);
+        p.o_hist = w.take((size_t)p.gsize * f);
+        p.ws_bwd = w.n;
+        p.state_bytes = (size_t)BH * (ns + 1) * (SD + D) * f;
+    }
+    p.tc = tc_plan(*ad, p.lay);
+    if (p.tc.eligible) {
+        p.ws_fwd = std::max(p.ws_fwd, p.tc.ws_fwd);
+        p.ws_bwd = std::max(p.ws_bwd, p.tc.ws_bwd);
+    }
+    return LUNA_OK;
+}
+
+AttnArgs make_args(const luna_attn_desc *ad, const Plan &p, const void *table, const void *Q, const void *K,
+                   const void *V, const int32_t *lengths, void *ws) {
+    AttnArgs a;
+    memset(&a, 0, sizeof(a));
+    a.B = ad->B; a.H = ad->H; a.n = ad->n; a.d = ad->d; a.dv = ad->dv;
+    a.M = p.lay.M; a.L = p.lay.L; a.D = p.lay.D;
+    a.eps = ad->eps;
+    a.lay = p.lay;
+    a.table = static_cast<const char *>(table);
+    a.Q = Q; a.K = K; a.V = V;
+    a.lengths = lengths;
+    char *w = static_cast<char *>(ws);
+    a.counters = reinterpret_cast<int *>(w + p.o_counters);
+    a.nsplit = p.nsplit; a.rows_per_split = p.rps;
+    a.nsplit_b = p.nsplit_b; a.rows_per_split_b = p.rps_b;
+    a.gsize = p.gsize;
+    a.chunk = ad->chunk ? ad->chunk : 64;
+    a.seg_len = p.seg_len; a.nseg = p.nseg;
+    a.S_part = reinterpret_cast<float *>(w + p.o_Spart);
+    a.z_part = reinterpret_cast<float *>(w + p.o_zpart);
+    if (!ad->causal) {
+        a.S_fin = reinterpret_cast<float *>(w + p.o_Sfin);
+        a.z_fin = reinterpret_cast<float *>(w + p.o_zfin);
+    } else {
+        a.seg_S = reinterpret_cast<float *>(w + p.o_segS);
+        a.seg_z = reinterpret_cast<float *>(w + p.o_segz);
+    }
+    return a;
+}
+
+void point_state(const luna_attn_desc *ad, const Plan &p, AttnArgs &a, void *state) {
+    if (!state) return;
+    float *s = static_cast<float *>(state);
+    const size_t SD = (size_t)p.lay.D * ad->dv;
+    if (!ad->causal) {
+        a.S_fin = s;
+        a.z_fin = s + (size_t)p.BH * SD;
+    } else {
+        a.seg_S = s;
+        a.seg_z = s + (size_t)p.BH * (p.nseg + 1) * SD;
+    }
+}
+
+luna_status cuda_status(cudaError_t e) { return e == cudaSuccess ? LUNA_OK : LUNA_ERR_CUDA; }
+
+bool aligned(const void *p, size_t a) { return (reinterpret_cast<uintptr_t>(p) % a) == 0; }
+
+}  // namespace
+
+extern "C" {
+
+int luna_version(void) { return 100; }
+
+const char *luna_status_string(luna_status s) {
+    switch (s) {
+        case LUNA_OK: return "LUNA_OK";
+        case LUNA_ERR_INVALID_ARG: return "LUNA_ERR_INVALID_ARG";
+        case LUNA_ERR_UNSUPPORTED: return "LUNA_ERR_UNSUPPORTED";
+        case LUNA_ERR_WORKSPACE: return "LUNA_ERR_WORKSPACE";
+        case LUNA_ERR_CUDA: return "LUNA_ERR_CUDA";
+        case LUNA_ERR_DEVICE_TIMEOUT: return "LUNA_ERR_DEVICE_TIMEOUT";
+    }
+    return "LUNA_ERR_UNKNOWN";
+}
+
+luna_status luna_phi_table_size(const luna_phi_desc *pd, int d, size_t *bytes) {
+    if (!bytes) return LUNA_ERR_INVALID_ARG;
+    luna_status st = check_phi(pd, d);
+    if (st != LUNA_OK) return st;
+    *bytes = (size_t)table_layout(pd->M, pd->L, pd->hidden, d).bytes;
+    return LUNA_OK;
+}
+
+luna_status luna_phi_prepare(const luna_phi_desc *pd, int d, const luna_phi_params *params, void *table,
+                             size_t table_bytes, void *stream) {
+    luna_status st = check_phi(pd, d);
+    if (st != LUNA_OK) return st;
+    if (!params || !table || !params->W || !params->b || !params->w1 || !params->b1 || !params->w2 || !params->b2)
+        return LUNA_ERR_INVALID_ARG;
+    if (!aligned(table, 256)) return LUNA_ERR_INVALID_ARG;
+    TableLayout lay = table_layout(pd->M, pd->L, pd->hidden, d);
+    if (table_bytes < (size_t)lay.bytes) return LUNA_ERR_WORKSPACE;
+    return cuda_status(launch_phi_prepare(*params, lay, table, static_cast<cudaStream_t>(stream)));
+}
+
+luna_status luna_featmap(const luna_phi_desc *pd, int d, const void *table, const void *X, luna_dtype xtype,
+                         int64_t rows, float *Phi, void *stream) {
+    luna_status st = check_phi(pd, d);
+    if (st != LUNA_OK) return st;
+    if (rows < 0 || (xtype != LUNA_F32 && xtype != LUNA_BF16)) return LUNA_ERR_INVALID_ARG;
+    if (rows == 0) return LUNA_OK;
+    if (!table || !X || !Phi) return LUNA_ERR_INVALID_ARG;
+    TableLayout lay = table_layout(pd->M, pd->L, pd->hidden, d);
+    return cuda_status(launch_featmap(lay, static_cast<const char *>(table), X, xtype, rows, Phi,
+                                      static_cast<cudaStream_t>(stream)));
+}
+
+luna_status luna_workspace_size(const luna_attn_desc *ad, const luna_phi_desc *pd, int backward, size_t *bytes) {
+    if (!bytes) return LUNA_ERR_INVALID_ARG;
+    Plan p;
+    luna_status st = make_plan(ad, pd, p);
+    if (st != LUNA_OK) return st;
+    *bytes = backward ? p.ws_bwd : p.ws_fwd;
+    if (*bytes == 0) *bytes = 256;
+    return LUNA_OK;
+}
+
+luna_status luna_state_size(const luna_attn_desc *ad, const luna_phi_desc *pd, size_t *bytes) {
+    if (!bytes) return LUNA_ERR_INVALID_ARG;
+    Plan p;
+    luna_status st = make_plan(ad, pd, p);
+    if (st != LUNA_OK) return st;
+    *bytes = p.state_bytes ? p.state_bytes : 256;
+    return LUNA_OK;
+}
+
+luna_status luna_attn_fwd(const luna_attn_desc *ad, const luna_phi_desc *pd, const void *table, const void *Q,
+                          const void *K, const void *V, const int32_t *lengths, void *O, void *state,
+                          void *workspace, size_t ws_bytes, void *stream) {
+    Plan p;
+    luna_status st = make_plan(ad, pd, p);
+    if (st != LUNA_OK) return st;
+    if (p.BH == 0 || ad->n == 0) return LUNA_OK;
+    if (!table || !Q || !K || !V || !O || !workspace) return LUNA_ERR_INVALID_ARG;
+    if (!aligned(workspace, 256) || !aligned(table, 256) || (state && !aligned(state, 256)))
+        return LUNA_ERR_INVALID_ARG;
+    if (ws_bytes < p.ws_fwd) return LUNA_ERR_WORKSPACE;
+    cudaStream_t s = static_cast<cudaStream_t>(stream);
+    AttnArgs a = make_args(ad, p, table, Q, K, V, lengths, workspace);
+    a.O = O;
+    point_state(ad, p, a, state);
+    if ((!ad->causal ? simt_max_smem(a) : causal_max_smem(a)) > kMaxSmem && !p.tc.eligible)
+        return LUNA_ERR_UNSUPPORTED;
+    cudaError_t e = cudaMemsetAsync(workspace, 0, p.o_counters + 2 * sizeof(int) * (size_t)p.BH, s);
+    if (e != cudaSuccess) return LUNA_ERR_CUDA;
+    if (ad->causal) return cuda_status(launch_causal_fwd(a, ad->io, state != nullptr, s));
+    if (p.tc.eligible && tc_inputs_ok(p.tc, Q, K, V, O))
+        return cuda_status(launch_tc_fwd(p.tc, a, static_cast<char *>(workspace), s));
+    return cuda_status(launch_simt_fwd(a, ad->io, s));
+}
+
+luna_status luna_attn_bwd(const luna_attn_desc *ad, const luna_phi_desc *pd, const void *table, const void *Q,
+                          const void *K, const void *V, const void *dO, const int32_t *lengths, const void *state,
+                          void *dQ, void *dK, void *dV, const luna_phi_grads *grads, void *workspace,
+                          size_t ws_bytes, void *stream) {
+    Plan p;
+    luna_status st = make_plan(ad, pd, p);
+    if (st != LUNA_OK) return st;
+    if (!grads || !grads->dW || !grads->db || !grads->dw1 || !grads->db1 || !grads->dw2 || !grads->db2)
+        return LUNA_ERR_INVALID_ARG;
+    cudaStream_t s = static_cast<cudaStream_t>(stream);
+    if (p.BH == 0 || ad->n == 0) {  // empty problem: parameter gradients are zero
+        const size_t Md = (size_t)pd->M * ad->d, P = (size_t)pd->L * pd->hidden;
+        cudaError_t e = cudaMemsetAsync(grads->dW, 0, Md * 4, s);
+        if (e == cudaSuccess) e = cudaMemsetAsync(grads->db, 0, pd->M * 4, s);
+        if (e == cudaSuccess) e = cudaMemsetAsync(grads->dw1, 0, P * 4, s);
+        if (e == cudaSuccess) e = cudaMemsetAsync(grads->db1, 0, P * 4, s);
+        if (e == cudaSuccess) e = cudaMemsetAsync(grads->dw2, 0, P * 4, s);
+        if (e == cudaSuccess) e = cudaMemsetAsync(grads->db2, 0, pd->L * 4, s);
+        return cuda_status(e);
+    }
+    if (!table || !Q || !K || !V || !dO || !dQ || !dK || !dV || !workspace) return LUNA_ERR_INVALID_ARG;
+    if (!aligned(workspace, 256) || !aligned(table, 256) || (state && !aligned(state, 256)))
+        return LUNA_ERR_INVALID_ARG;
+    if (ws_bytes < p.ws_bwd) return LUNA_ERR_WORKSPACE;
+    AttnArgs a = make_args(ad, p, table, Q, K, V, lengths, workspace);
+    char *w = static_cast<char *>(workspace);
+    a.dO = dO; a.dQ = dQ; a.dK = dK; a.dV = dV;
+    a.grads = *grads;
+    a.dS_part = reinterpret_cast<float *>(w + p.o_dSpart);
+    a.dz_part = reinterpret_cast<float *>(w + p.o_dzpart);
+    a.gpart = reinterpret_cast<float *>(w + p.o_gpart);
+    a.hist = reinterpret_cast<float *>(w + p.o_hist);
+    if (!ad->causal) {
+        a.dS_fin = reinterpret_cast<float *>(w + p.o_dSfin);
+        a.dz_fin = reinterpret_cast<float *>(w + p.o_dzfin);
+    } else {
+        a.seg_dS = reinterpret_cast<float *>(w + p.o_segdS);
+        a.seg_dz = reinterpret_cast<float *>(w + p.o_segdz);
+        a.rowstat = reinterpret_cast<float *>(w + p.o_rowstat);
+    }
+    point_state(ad, p, a, const_cast<void *>(state));
+    if ((!ad->causal ? simt_max_smem(a) : causal_max_smem(a)) > kMaxSmem && !p.tc.eligible)
+        return LUNA_ERR_UNSUPPORTED;
+    cudaError_t e = cudaMemsetAsync(workspace, 0, p.o_counters + 2 * sizeof(int) * (size_t)p.BH, s);
+    if (e != cudaSuccess) return LUNA_ERR_CUDA;
+    if (ad->causal) return cuda_status(launch_causal_bwd(a, ad->io, state != nullptr, s));
+    if (p.tc.eligible && tc_inputs_ok(p.tc, Q, K, V, dO) && tc_inputs_ok(p.tc, dQ, dK, dV, nullptr))
+        return cuda_status(launch_tc_bwd(p.tc, a, w, state != nullptr, s));
+    return cuda_status(launch_simt_bwd(a, ad->io, state != nullptr, s));
+}
+
+luna_status luna_device_status(void *workspace, void *stream) {
+    if (!workspace) return LUNA_ERR_INVALID_ARG;
+    cudaStream_t s = static_cast<cudaStream_t>(stream);
+    int word = 0;
+    cudaError_t e = cudaMemcpyAsync(&word, workspace, sizeof(int), cudaMemcpyDeviceToHost, s);
+    if (e == cudaSuccess) e = cudaStreamSynchronize(s);
+    if (e == cudaSuccess && word != 0) e = cudaMemsetAsync(workspace, 0, sizeof(int), s);
+    if (e == cudaSuccess) e = cudaStreamSynchronize(s);
+    if (e != cudaSuccess) return LUNA_ERR_CUDA;
+    return word == 0 ? LUNA_OK : LUNA_ERR_DEVICE_TIMEOUT;
+}
+
+}  // extern "C"

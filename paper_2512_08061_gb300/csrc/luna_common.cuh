@@ -1,0 +1,98 @@
+// Internal definitions shared by the CUDA translation units of the LUNA library.
+#pragma once
+
+#include <cuda_bf16.h>
+#include <cuda_runtime.h>
+#include <stdint.h>
+
+#include "luna.h"
+
+namespace luna {
+
+constexpr int kTableMagic = 0x414E554C;  // "LUNA"
+constexpr int kTableVersion = 1;
+constexpr int kMaxD = 128;      // max d, dv
+constexpr int kMaxFeat = 128;   // max D = M * L
+constexpr int kMaxL = 16;
+constexpr int kMaxHidden = 128;
+constexpr int kMaxUnits = 512;  // max L * hidden
+
+__host__ __device__ inline int next_pow2(int x) {
+    int p = 1;
+    while (p < x) p <<= 1;
+    return p;
+}
+__host__ __device__ inline int64_t align16(int64_t x) { return (x + 15) & ~int64_t(15); }
+__host__ __device__ inline int64_t align256(int64_t x) { return (x + 255) & ~int64_t(255); }
+
+// Layout of the prepared feature-map table (byte offsets from its start).
+//   T      [Ppad]          sorted fp32 kink thresholds of all hidden units (+inf padding)
+//   AB     [nint][L][2]    per merged interval j and channel l: (alpha, beta) / sqrt(M)
+//   W      [M][d], b [M]   projection copy
+//   rank   [P]             position of unit (l,k) in the sorted kink list
+//   utype  [P]             +1: unit active iff u > T[rank] ; -1: active iff u <= T[rank]
+//   w1, b1, w2 [P], b2 [L] channel-MLP parameter copy (used by the gradient reduction)
+struct TableLayout {
+    int M, L, hid, d, D, P, Ppad, nint;
+    int64_t off_T, off_AB, off_W, off_b, off_rank, off_utype, off_w1, off_b1, off_w2, off_b2, bytes;
+};
+
+__host__ __device__ inline TableLayout table_layout(int M, int L, int hid, int d) {
+    TableLayout t;
+    t.M = M; t.L = L; t.hid = hid; t.d = d; t.D = M * L;
+    t.P = L * hid;
+    t.Ppad = next_pow2(t.P);
+    t.nint = t.P + 1;
+    int64_t o = 256;  // header
+    t.off_T = o;     o = align16(o + 4 * (int64_t)t.Ppad);
+    t.off_AB = o;    o = align16(o + 8 * (int64_t)t.nint * L);
+    t.off_W = o;     o = align16(o + 4 * (int64_t)M * d);
+    t.off_b = o;     o = align16(o + 4 * (int64_t)M);
+    t.off_rank = o;  o = align16(o + 4 * (int64_t)t.P);
+    t.off_utype = o; o = align16(o + 4 * (int64_t)t.P);
+    t.off_w1 = o;    o = align16(o + 4 * (int64_t)t.P);
+    t.off_b1 = o;    o = align16(o + 4 * (int64_t)t.P);
+    t.off_w2 = o;    o = align16(o + 4 * (int64_t)t.P);
+    t.off_b2 = o;    o = align16(o + 4 * (int64_t)L);
+    t.bytes = align256(o);
+    return t;
+}
+
+struct TableHeader {
+    int magic, version, M, L, hid, d, P, Ppad;
+};
+
+// ---------------------------------------------------------------------------
+// I/O element access
+
+template <typename T> struct IOType;
+template <> struct IOType<float> { static constexpr luna_dtype code = LUNA_F32; };
+template <> struct IOType<__nv_bfloat16> { static constexpr luna_dtype code = LUNA_BF16; };
+
+__device__ __forceinline__ float io_load(const float *p) { return *p; }
+__device__ __forceinline__ float io_load(const __nv_bfloat16 *p) { return __bfloat162float(*p); }
+__device__ __forceinline__ void io_store(float *p, float v) { *p = v; }
+__device__ __forceinline__ void io_store(__nv_bfloat16 *p, float v) { *p = __float2bfloat16_rn(v); }
+
+// ---------------------------------------------------------------------------
+// Feature map from the table
+
+// Number of sorted thresholds strictly below u (branch-free lower bound over a
+// power-of-two sized array whose tail is padded with +inf).
+__device__ __forceinline__ int interval_of(const float *T, int Ppad, float u) {
+    int pos = 0;
+    for (int s = Ppad >> 1; s > 0; s >>= 1) pos += (T[pos + s - 1] < u) ? s : 0;
+    pos += (T[pos] < u) ? 1 : 0;
+    return pos;
+}
+
+__device__ __forceinline__ int head_length(const int32_t *lengths, int b, int n) {
+    if (!lengths) return n;
+    int len = lengths[b];
+    return len < 0 ? 0 : (len > n ? n : len);
+}
+
+// Host-side launch helpers (defined in luna_api.cu)
+int device_sm_count();
+
+}  // namespace luna

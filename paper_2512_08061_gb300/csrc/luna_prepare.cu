@@ -1,0 +1,115 @@
+// Feature-map table: the exact piecewise-linear form of the channel MLPs.
+//
+// Each channel function of the listing's ScalarMLP is
+//     psi_l(u) = relu( b2[l] + sum_k w2[l,k] relu(w1[l,k] u + b1[l,k]) ),
+// a ReLU network of one scalar, hence linear in u between the kinks of its
+// hidden units.  Merging the kinks of all L*hidden units into one sorted list
+// T gives intervals j = #{p : T[p] < u} on which every hidden unit of every
+// channel is either on or off, so
+//     psi_l(u) = relu(alpha[j][l] * u + beta[j][l]).
+// The kink of unit k is placed at the exact fp32 threshold of fma(w1, u, b1),
+// so the interval reproduces the on/off decision of an fp32 evaluation of fc1
+// for every fp32 u.  The 1/sqrt(M) scale of Eq. (phi-def-scalarenv) is folded
+// into alpha and beta (it is positive, so relu commutes with it).
+#include <math.h>
+
+#include "luna_common.cuh"
+#include "luna_prof.cuh"
+
+namespace luna {
+
+namespace {
+
+__device__ float up_threshold(float w, float c) {
+    // largest fp32 u with fma(w,u,c) <= 0, for w > 0 (fma is monotone in u)
+    float t = -c / w;
+    for (int it = 0; it < 64 && fmaf(w, t, c) > 0.0f; ++it) t = nextafterf(t, -INFINITY);
+    for (int it = 0; it < 64 && fmaf(w, nextafterf(t, INFINITY), c) <= 0.0f; ++it) t = nextafterf(t, INFINITY);
+    return t;
+}
+
+__device__ float down_threshold(float w, float c) {
+    // largest fp32 u with fma(w,u,c) > 0, for w < 0
+    float t = -c / w;
+    for (int it = 0; it < 64 && !(fmaf(w, t, c) > 0.0f); ++it) t = nextafterf(t, -INFINITY);
+    for (int it = 0; it < 64 && fmaf(w, nextafterf(t, INFINITY), c) > 0.0f; ++it) t = nextafterf(t, INFINITY);
+    return t;
+}
+
+__global__ void __launch_bounds__(1024) k_phi_prepare(luna_phi_params prm, TableLayout lay, char *table) {
+    __shared__ float th[kMaxUnits];
+    __shared__ int ty[kMaxUnits];
+    __shared__ int rk[kMaxUnits];
+    __shared__ float w1s[kMaxUnits], b1s[kMaxUnits], w2s[kMaxUnits];
+    const int tid = threadIdx.x, nt = blockDim.x;
+    const int P = lay.P;
+
+    for (int k = tid; k < P; k += nt) {
+        float w = prm.w1[k], c = prm.b1[k];
+        w1s[k] = w; b1s[k] = c; w2s[k] = prm.w2[k];
+        if (w > 0.0f) { th[k] = up_threshold(w, c); ty[k] = 1; }
+        else if (w < 0.0f) { th[k] = down_threshold(w, c); ty[k] = -1; }
+        else { th[k] = INFINITY; ty[k] = (c > 0.0f) ? -1 : 1; }  // constant unit: always on / always off
+    }
+    __syncthreads();
+    // rank by (threshold, unit index): a stable total order
+    for (int k = tid; k < P; k += nt) {
+        float t = th[k];
+        int r = 0;
+        for (int q = 0; q < P; ++q) {
+            float s = th[q];
+            r += (s < t || (s == t && q < k)) ? 1 : 0;
+        }
+        rk[k] = r;
+    }
+    __syncthreads();
+
+    float *T = reinterpret_cast<float *>(table + lay.off_T);
+    float *AB = reinterpret_cast<float *>(table + lay.off_AB);
+    int *rank = reinterpret_cast<int *>(table + lay.off_rank);
+    int *utype = reinterpret_cast<int *>(table + lay.off_utype);
+    for (int k = tid; k < P; k += nt) {
+        T[rk[k]] = th[k];
+        rank[k] = rk[k];
+        utype[k] = ty[k];
+        reinterpret_cast<float *>(table + lay.off_w1)[k] = w1s[k];
+        reinterpret_cast<float *>(table + lay.off_b1)[k] = b1s[k];
+        reinterpret_cast<float *>(table + lay.off_w2)[k] = w2s[k];
+    }
+    for (int p = P + tid; p < lay.Ppad; p += nt) T[p] = INFINITY;
+
+    const float scale = 1.0f / sqrtf((float)lay.M);
+    const int hid = lay.hid, L = lay.L;
+    for (int e = tid; e < lay.nint * L; e += nt) {
+        int j = e / L, l = e % L;
+        float a = 0.0f, bsum = prm.b2[l];
+        for (int k = 0; k < hid; ++k) {
+            int u = l * hid + k;
+            bool on = (ty[u] > 0) ? (rk[u] < j) : (rk[u] >= j);
+            if (on) {
+                a = fmaf(w2s[u], w1s[u], a);
+                bsum = fmaf(w2s[u], b1s[u], bsum);
+            }
+        }
+        AB[2 * e] = a * scale;
+        AB[2 * e + 1] = bsum * scale;
+    }
+    float *W = reinterpret_cast<float *>(table + lay.off_W);
+    for (int e = tid; e < lay.M * lay.d; e += nt) W[e] = prm.W[e];
+    for (int e = tid; e < lay.M; e += nt) reinterpret_cast<float *>(table + lay.off_b)[e] = prm.b[e];
+    for (int e = tid; e < L; e += nt) reinterpret_cast<float *>(table + lay.off_b2)[e] = prm.b2[e];
+    if (tid == 0) {
+        TableHeader *h = reinterpret_cast<TableHeader *>(table);
+        h->magic = kTableMagic; h->version = kTableVersion;
+        h->M = lay.M; h->L = lay.L; h->hid = lay.hid; h->d = lay.d; h->P = P; h->Ppad = lay.Ppad;
+    }
+}
+
+}  // namespace
+
+cudaError_t launch_phi_prepare(const luna_phi_params &prm, const TableLayout &lay, void *table, cudaStream_t s) {
+    LUNA_LAUNCH("phi_prepare", k_phi_prepare, 1, 1024, 0, s, prm, lay, static_cast<char *>(table));
+    return cudaGetLastError();
+}
+
+}  // namespace luna

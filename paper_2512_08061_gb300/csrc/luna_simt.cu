@@ -1,0 +1,479 @@
+// Generic CUDA-core kernels of the LUNA attention path (fp32 arithmetic).
+//
+// They serve the fp32 I/O path (the parity bar there is 1e-4 relative, which
+// rules out bf16 tensor-core operands) and every shape the tensor-core path
+// does not specialise.  One thread block owns a (head, row range); all
+// statistics are fp32 and every cross-block reduction is performed in a fixed
+// order by the last block to arrive, so results are reproducible run to run
+// except for the order of shared-memory atomic adds in the gradient
+// histograms of the channel-MLP parameters.
+#include <math.h>
+
+#include "luna_prof.cuh"
+#include "luna_simt_dev.cuh"
+
+namespace luna {
+namespace {
+using namespace simt;
+
+// ---------------------------------------------------------------------------
+// feature map alone
+
+template <typename IO>
+__global__ void __launch_bounds__(kThreads) k_featmap(TableLayout lay, const char *table, const IO *X, int64_t rows,
+                                                      float *Phi) {
+    extern __shared__ __align__(16) float smem[];
+    Carve cv{smem};
+    SmemPhi s = carve_phi(cv, lay);
+    load_phi(s, lay, table);
+    __syncthreads();
+    const int M = lay.M, L = lay.L, d = lay.d, D = lay.D;
+    for (int64_t e = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; e < rows * M; e += (int64_t)gridDim.x * blockDim.x) {
+        const int64_t r = e / M;
+        const int i = (int)(e - r * M);
+        const IO *x = X + r * d;
+        const float *w = s.W + i * d;
+        float u = s.b[i];
+        for (int c = 0; c < d; ++c) u = fmaf(w[c], io_load(x + c), u);
+        const int j = interval_of(s.T, lay.Ppad, u);
+        const float *ab = s.AB + j * L * 2;
+        float *out = Phi + r * D + i * L;
+        for (int l = 0; l < L; ++l) out[l] = fmaxf(fmaf(ab[2 * l], u, ab[2 * l + 1]), 0.0f);
+    }
+}
+
+// ---------------------------------------------------------------------------
+// key statistics S = sum_j phi(k_j) v_j^T, z = sum_j phi(k_j)   (Sec. 4: S_KV, S_K1)
+
+template <typename IO>
+__global__ void __launch_bounds__(kThreads) k_keystats(AttnArgs a) {
+    extern __shared__ __align__(16) float smem[];
+    Carve cv{smem};
+    const TableLayout &lay = a.lay;
+    SmemPhi s = carve_phi(cv, lay);
+    float *sK = cv.take(kTileK * a.d);
+    float *sV = cv.take(kTileK * a.dv);
+    float *sPhi = cv.take(kTileK * a.D);
+    load_phi(s, lay, a.table);
+
+    const int bh = blockIdx.y, split = blockIdx.x;
+    const int len = head_length(a.lengths, bh / a.H, a.n);
+    const int r0 = split * a.rows_per_split;
+    const int r1 = min(len, r0 + a.rows_per_split);
+    const IO *K = static_cast<const IO *>(a.K) + (size_t)bh * a.n * a.d;
+    const IO *V = static_cast<const IO *>(a.V) + (size_t)bh * a.n * a.dv;
+
+    const int nc = (a.dv + 7) / 8, nf = (a.D + 7) / 8;
+    const bool active = threadIdx.x < nf * nc;
+    const int tf = active ? threadIdx.x / nc : 0, tc = active ? threadIdx.x % nc : 0;
+    const int f0 = tf * 8, c0 = tc * 8;
+    float acc[8][8] = {}, zacc[8] = {};
+    for (int t0 = r0; t0 < r1; t0 += kTileK) {
+        const int nr = min(kTileK, r1 - t0);
+        __syncthreads();
+        load_rows(sK, K + (size_t)t0 * a.d, nr * a.d);
+        load_rows(sV, V + (size_t)t0 * a.dv, nr * a.dv);
+        __syncthreads();
+        phi_tile(lay, s, sK, nr, sPhi, nullptr, nullptr);
+        __syncthreads();
+        if (active) outer_accumulate(acc, zacc, true, sPhi, a.D, sV, a.dv, nullptr, nr, f0, c0);
+    }
+    const size_t slot = (size_t)bh * a.nsplit + split;
+    store_tile(acc, zacc, active, tc, f0, c0, a.D, a.dv, a.S_part + slot * a.D * a.dv, a.z_part + slot * a.D);
+    if (last_arrival(a.counters + bh, a.nsplit)) {
+        if (a.seg_S) {  // causal: exclusive prefix at every segment start, total in slot nsplit
+            exclusive_scan(a.S_part + (size_t)bh * a.nsplit * a.D * a.dv, a.nsplit, a.D * a.dv,
+                           a.seg_S + (size_t)bh * (a.nsplit + 1) * a.D * a.dv, false);
+            exclusive_scan(a.z_part + (size_t)bh * a.nsplit * a.D, a.nsplit, a.D,
+                           a.seg_z + (size_t)bh * (a.nsplit + 1) * a.D, false);
+        } else {
+            ordered_sum(a.S_part + (size_t)bh * a.nsplit * a.D * a.dv, a.nsplit, a.D * a.dv,
+                        a.S_fin + (size_t)bh * a.D * a.dv);
+            ordered_sum(a.z_part + (size_t)bh * a.nsplit * a.D, a.nsplit, a.D, a.z_fin + (size_t)bh * a.D);
+        }
+        if (threadIdx.x == 0) a.counters[bh] = 0;
+    }
+}
+
+// ---------------------------------------------------------------------------
+// query side: O_i = phi(q_i)^T S / (phi(q_i)^T z + eps)   (Eq. kernel-attn)
+
+template <typename IO>
+__global__ void __launch_bounds__(kThreads) k_query(AttnArgs a) {
+    extern __shared__ __align__(16) float smem[];
+    const int bh = blockIdx.y;
+    const int q0 = blockIdx.x * kTileQ;
+    const int len = head_length(a.lengths, bh / a.H, a.n);
+    IO *O = static_cast<IO *>(a.O) + (size_t)bh * a.n * a.dv;
+    const int nrows = min(kTileQ, a.n - q0);
+    if (q0 >= len) {  // padded rows only
+        for (int e = threadIdx.x; e < nrows * a.dv; e += blockDim.x) io_store(O + (size_t)q0 * a.dv + e, 0.0f);
+        return;
+    }
+    Carve cv{smem};
+    const TableLayout &lay = a.lay;
+    SmemPhi s = carve_phi(cv, lay);
+    float *sS = cv.take(a.D * a.dv);
+    float *sz = cv.take(a.D);
+    float *sQ = cv.take(kTileQ * a.d);
+    float *sPhi = cv.take(kTileQ * a.D);
+    float *sden = cv.take(kTileQ);
+    load_phi(s, lay, a.table);
+    for (int e = threadIdx.x; e < a.D * a.dv; e += blockDim.x) sS[e] = a.S_fin[(size_t)bh * a.D * a.dv + e];
+    for (int e = threadIdx.x; e < a.D; e += blockDim.x) sz[e] = a.z_fin[(size_t)bh * a.D + e];
+    const int nr = min(nrows, len - q0);
+    load_rows(sQ, static_cast<const IO *>(a.Q) + ((size_t)bh * a.n + q0) * a.d, nr * a.d);
+    __syncthreads();
+    phi_tile(lay, s, sQ, nr, sPhi, nullptr, nullptr);
+    __syncthreads();
+    for (int r = threadIdx.x; r < nr; r += blockDim.x) {
+        float den = a.eps;
+        for (int f = 0; f < a.D; ++f) den = fmaf(sPhi[r * a.D + f], sz[f], den);
+        sden[r] = den;
+    }
+    __syncthreads();
+    for (int e = threadIdx.x; e < nrows * a.dv; e += blockDim.x) {
+        const int r = e / a.dv, c = e - r * a.dv;
+        float o = 0.0f;
+        if (r < nr && sden[r] != 0.0f) {
+            float num = 0.0f;
+            for (int f = 0; f < a.D; ++f) num = fmaf(sPhi[r * a.D + f], sS[f * a.dv + c], num);
+            o = num / sden[r];
+        }
+        io_store(O + (size_t)q0 * a.dv + e, o);
+    }
+}
+
+// query side of the backward pass (non-causal):
+//   dnum_i = do_i / den_i,  dden_i = -(do_i . o_i) / den_i
+//   dphi(q_i) = S dnum_i + z dden_i,  dS += phi(q_i) dnum_i^T,  dz += phi(q_i) dden_i
+template <typename IO>
+__global__ void __launch_bounds__(kThreads) k_bwd_query(AttnArgs a) {
+    extern __shared__ __align__(16) float smem[];
+    Carve cv{smem};
+    const TableLayout &lay = a.lay;
+    const int D = a.D, dv = a.dv, d = a.d, M = a.M;
+    SmemPhi s = carve_phi(cv, lay);
+    float *sS = cv.take(D * dv);
+    float *sz = cv.take(D);
+    float *sQ = cv.take(kTileB * d);
+    float *sdO = cv.take(kTileB * dv);
+    float *sPhi = cv.take(kTileB * D);
+    float *sdPhi = cv.take(kTileB * D);
+    float *sdnum = cv.take(kTileB * dv);
+    float *sden = cv.take(kTileB);
+    float *sdden = cv.take(kTileB);
+    float *sU = cv.take(kTileB * M);
+    int *sJ = reinterpret_cast<int *>(cv.take(kTileB * M));
+    float *sdU = cv.take(kTileB * M);
+    float *shist = cv.take(lay.nint * lay.L * 2);
+    load_phi(s, lay, a.table);
+    const int bh = blockIdx.y, split = blockIdx.x;
+    for (int e = threadIdx.x; e < D * dv; e += blockDim.x) sS[e] = a.S_fin[(size_t)bh * D * dv + e];
+    for (int e = threadIdx.x; e < D; e += blockDim.x) sz[e] = a.z_fin[(size_t)bh * D + e];
+    for (int e = threadIdx.x; e < lay.nint * lay.L * 2; e += blockDim.x) shist[e] = 0.0f;
+
+    const int len = head_length(a.lengths, bh / a.H, a.n);
+    const int r0 = split * a.rows_per_split_b;
+    const int rend = min(a.n, r0 + a.rows_per_split_b);
+    const int r1 = min(len, rend);
+    const IO *Q = static_cast<const IO *>(a.Q) + (size_t)bh * a.n * d;
+    const IO *dO = static_cast<const IO *>(a.dO) + (size_t)bh * a.n * dv;
+    IO *dQ = static_cast<IO *>(a.dQ) + (size_t)bh * a.n * d;
+    // padded rows of this range receive zero gradients
+    for (int e = threadIdx.x + max(r0, len) * d; e < rend * d; e += blockDim.x) io_store(dQ + e, 0.0f);
+
+    const int nc = (dv + 7) / 8, nf = (D + 7) / 8;
+    const bool active = threadIdx.x < nf * nc;
+    const int tf = active ? threadIdx.x / nc : 0, tc = active ? threadIdx.x % nc : 0;
+    const int f0 = tf * 8, c0 = tc * 8;
+    float acc[8][8] = {}, zacc[8] = {};
+    GradAcc g = {};
+    for (int t0 = r0; t0 < r1; t0 += kTileB) {
+        const int nr = min(kTileB, r1 - t0);
+        __syncthreads();
+        load_rows(sQ, Q + (size_t)t0 * d, nr * d);
+        load_rows(sdO, dO + (size_t)t0 * dv, nr * dv);
+        __syncthreads();
+        phi_tile(lay, s, sQ, nr, sPhi, sU, sJ);
+        __syncthreads();
+        for (int r = threadIdx.x; r < nr; r += blockDim.x) {
+            float den = a.eps;
+            for (int f = 0; f < D; ++f) den = fmaf(sPhi[r * D + f], sz[f], den);
+            sden[r] = den;
+        }
+        __syncthreads();
+        for (int e = threadIdx.x; e < nr * dv; e += blockDim.x) {  // o_i into sdnum for now
+            const int r = e / dv, c = e - r * dv;
+            float o = 0.0f;
+            if (sden[r] != 0.0f) {
+                float num = 0.0f;
+                for (int f = 0; f < D; ++f) num = fmaf(sPhi[r * D + f], sS[f * dv + c], num);
+                o = num / sden[r];
+            }
+            sdnum[e] = o;
+        }
+        __syncthreads();
+        for (int r = threadIdx.x; r < nr; r += blockDim.x) {
+            float dot = 0.0f;
+            for (int c = 0; c < dv; ++c) dot = fmaf(sdO[r * dv + c], sdnum[r * dv + c], dot);
+            sdden[r] = (sden[r] != 0.0f) ? -dot / sden[r] : 0.0f;
+        }
+        __syncthreads();
+        for (int e = threadIdx.x; e < nr * dv; e += blockDim.x) {
+            const int r = e / dv;
+            sdnum[e] = (sden[r] != 0.0f) ? sdO[e] / sden[r] : 0.0f;
+        }
+        __syncthreads();
+        for (int e = threadIdx.x; e < nr * D; e += blockDim.x) {
+            const int r = e / D, f = e - r * D;
+            float acc2 = sz[f] * sdden[r];
+            for (int c = 0; c < dv; ++c) acc2 = fmaf(sS[f * dv + c], sdnum[r * dv + c], acc2);
+            sdPhi[e] = acc2;
+        }
+        __syncthreads();
+        if (active) outer_accumulate(acc, zacc, true, sPhi, D, sdnum, dv, sdden, nr, f0, c0);
+        phi_backward_tile(lay, s, sQ, nr, sPhi, sdPhi, sU, sJ, sdU, shist, g);
+        store_dx(lay, s, sdU, nr, dQ + (size_t)t0 * d);
+    }
+    __syncthreads();
+    const size_t slot = (size_t)bh * a.nsplit_b + split;
+    store_tile(acc, zacc, active, tc, f0, c0, D, dv, a.dS_part + slot * D * dv, a.dz_part + slot * D);
+    store_grad_partial(lay, g, shist, a.gpart + slot * a.gsize);
+    if (last_arrival(a.counters + a.B * a.H + bh, a.nsplit_b)) {
+        ordered_sum(a.dS_part + (size_t)bh * a.nsplit_b * D * dv, a.nsplit_b, D * dv, a.dS_fin + (size_t)bh * D * dv);
+        ordered_sum(a.dz_part + (size_t)bh * a.nsplit_b * D, a.nsplit_b, D, a.dz_fin + (size_t)bh * D);
+        if (threadIdx.x == 0) a.counters[a.B * a.H + bh] = 0;
+    }
+}
+
+// key side of the backward pass (non-causal):
+//   dv_j = dS^T phi(k_j),  dphi(k_j) = dS v_j + dz
+template <typename IO>
+__global__ void __launch_bounds__(kThreads) k_bwd_key(AttnArgs a) {
+    extern __shared__ __align__(16) float smem[];
+    Carve cv{smem};
+    const TableLayout &lay = a.lay;
+    const int D = a.D, dv = a.dv, d = a.d, M = a.M;
+    SmemPhi s = carve_phi(cv, lay);
+    float *sdS = cv.take(D * dv);
+    float *sdz = cv.take(D);
+    float *sK = cv.take(kTileB * d);
+    float *sV = cv.take(kTileB * dv);
+    float *sPhi = cv.take(kTileB * D);
+    float *sdPhi = cv.take(kTileB * D);
+    float *sU = cv.take(kTileB * M);
+    int *sJ = reinterpret_cast<int *>(cv.take(kTileB * M));
+    float *sdU = cv.take(kTileB * M);
+    float *shist = cv.take(lay.nint * lay.L * 2);
+    load_phi(s, lay, a.table);
+    const int bh = blockIdx.y, split = blockIdx.x;
+    for (int e = threadIdx.x; e < D * dv; e += blockDim.x) sdS[e] = a.dS_fin[(size_t)bh * D * dv + e];
+    for (int e = threadIdx.x; e < D; e += blockDim.x) sdz[e] = a.dz_fin[(size_t)bh * D + e];
+    for (int e = threadIdx.x; e < lay.nint * lay.L * 2; e += blockDim.x) shist[e] = 0.0f;
+
+    const int len = head_length(a.lengths, bh / a.H, a.n);
+    const int r0 = split * a.rows_per_split_b;
+    const int rend = min(a.n, r0 + a.rows_per_split_b);
+    const int r1 = min(len, rend);
+    const IO *K = static_cast<const IO *>(a.K) + (size_t)bh * a.n * d;
+    const IO *V = static_cast<const IO *>(a.V) + (size_t)bh * a.n * dv;
+    IO *dK = static_cast<IO *>(a.dK) + (size_t)bh * a.n * d;
+    IO *dV = static_cast<IO *>(a.dV) + (size_t)bh * a.n * dv;
+    for (int e = threadIdx.x + max(r0, len) * d; e < rend * d; e += blockDim.x) io_store(dK + e, 0.0f);
+    for (int e = threadIdx.x + max(r0, len) * dv; e < rend * dv; e += blockDim.x) io_store(dV + e, 0.0f);
+
+    GradAcc g = {};
+    for (int t0 = r0; t0 < r1; t0 += kTileB) {
+        const int nr = min(kTileB, r1 - t0);
+        __syncthreads();
+        load_rows(sK, K + (size_t)t0 * d, nr * d);
+        load_rows(sV, V + (size_t)t0 * dv, nr * dv);
+        __syncthreads();
+        phi_tile(lay, s, sK, nr, sPhi, sU, sJ);
+        __syncthreads();
+        for (int e = threadIdx.x; e < nr * dv; e += blockDim.x) {
+            const int r = e / dv, c = e - r * dv;
+            float acc2 = 0.0f;
+            for (int f = 0; f < D; ++f) acc2 = fmaf(sPhi[r * D + f], sdS[f * dv + c], acc2);
+            io_store(dV + (size_t)t0 * dv + e, acc2);
+        }
+        for (int e = threadIdx.x; e < nr * D; e += blockDim.x) {
+            const int r = e / D, f = e - r * D;
+            float acc2 = sdz[f];
+            for (int c = 0; c < dv; ++c) acc2 = fmaf(sdS[f * dv + c], sV[r * dv + c], acc2);
+            sdPhi[e] = acc2;
+        }
+        __syncthreads();
+        phi_backward_tile(lay, s, sK, nr, sPhi, sdPhi, sU, sJ, sdU, shist, g);
+        store_dx(lay, s, sdU, nr, dK + (size_t)t0 * d);
+    }
+    __syncthreads();
+    const size_t slot = (size_t)a.B * a.H * a.nsplit_b + (size_t)bh * a.nsplit_b + split;
+    store_grad_partial(lay, g, shist, a.gpart + slot * a.gsize);
+}
+
+// ---------------------------------------------------------------------------
+// parameter gradients: ordered sum of the per-block partials, then the
+// channel-MLP gradients from the interval histogram.
+//   With g = dLoss/dPhi on active outputs, m0[j][l] = sum g, m1[j][l] = sum g*u
+//   over samples falling in interval j; for hidden unit (l,k) active on the
+//   intervals A_k:  G0 = sum_{j in A_k} m0, G1 = sum_{j in A_k} m1 and
+//     dw2 = (w1 G1 + b1 G0)/sqrt(M), dw1 = w2 G1/sqrt(M), db1 = w2 G0/sqrt(M),
+//     db2 = sum_j m0 / sqrt(M).
+
+__global__ void __launch_bounds__(kThreads) k_grad_sum(const float *gpart, int nparts, int gsize, float *out) {
+    for (int e = blockIdx.x * blockDim.x + threadIdx.x; e < gsize; e += gridDim.x * blockDim.x) {
+        float s = 0.0f;
+        for (int p = 0; p < nparts; ++p) s += gpart[(size_t)p * gsize + e];
+        out[e] = s;
+    }
+}
+
+__global__ void __launch_bounds__(kThreads) k_mlp_grads(TableLayout lay, const char *table, const float *gsum,
+                                                        luna_phi_grads grads) {
+    const int Md = lay.M * lay.d, L = lay.L, hid = lay.hid, nint = lay.nint;
+    const float *hist = gsum + Md + lay.M;
+    const int *rank = reinterpret_cast<const int *>(table + lay.off_rank);
+    const int *utype = reinterpret_cast<const int *>(table + lay.off_utype);
+    const float *w1 = reinterpret_cast<const float *>(table + lay.off_w1);
+    const float *b1 = reinterpret_cast<const float *>(table + lay.off_b1);
+    const float *w2 = reinterpret_cast<const float *>(table + lay.off_w2);
+    const float scale = 1.0f / sqrtf((float)lay.M);
+    for (int e = threadIdx.x; e < Md; e += blockDim.x) grads.dW[e] = gsum[e];
+    for (int e = threadIdx.x; e < lay.M; e += blockDim.x) grads.db[e] = gsum[Md + e];
+    for (int u = threadIdx.x; u < lay.P; u += blockDim.x) {
+        const int l = u / hid;
+        const int r = rank[u];
+        const bool up = utype[u] > 0;
+        float G0 = 0.0f, G1 = 0.0f;
+        for (int j = 0; j < nint; ++j) {
+            const bool on = up ? (r < j) : (r >= j);
+            if (on) {
+                G0 += hist[(j * L + l) * 2];
+                G1 += hist[(j * L + l) * 2 + 1];
+            }
+        }
+        grads.dw2[u] = (w1[u] * G1 + b1[u] * G0) * scale;
+        grads.dw1[u] = w2[u] * G1 * scale;
+        grads.db1[u] = w2[u] * G0 * scale;
+    }
+    for (int l = threadIdx.x; l < L; l += blockDim.x) {
+        float t = 0.0f;
+        for (int j = 0; j < nint; ++j) t += hist[(j * L + l) * 2];
+        grads.db2[l] = t * scale;
+    }
+}
+
+// ---------------------------------------------------------------------------
+// host side
+
+size_t smem_keystats(const AttnArgs &a) {
+    HostCarve cv; carve_phi_host(cv, a.lay);
+    cv.take(kTileK * a.d); cv.take(kTileK * a.dv); cv.take(kTileK * a.D);
+    return cv.bytes();
+}
+size_t smem_query(const AttnArgs &a) {
+    HostCarve cv; carve_phi_host(cv, a.lay);
+    cv.take(a.D * a.dv); cv.take(a.D); cv.take(kTileQ * a.d); cv.take(kTileQ * a.D); cv.take(kTileQ);
+    return cv.bytes();
+}
+size_t smem_bwd_query(const AttnArgs &a) {
+    HostCarve cv; carve_phi_host(cv, a.lay);
+    cv.take(a.D * a.dv); cv.take(a.D); cv.take(kTileB * a.d); cv.take(kTileB * a.dv); cv.take(kTileB * a.D);
+    cv.take(kTileB * a.D); cv.take(kTileB * a.dv); cv.take(kTileB); cv.take(kTileB); cv.take(kTileB * a.M);
+    cv.take(kTileB * a.M); cv.take(kTileB * a.M); cv.take(a.lay.nint * a.lay.L * 2);
+    return cv.bytes();
+}
+size_t smem_bwd_key(const AttnArgs &a) {
+    HostCarve cv; carve_phi_host(cv, a.lay);
+    cv.take(a.D * a.dv); cv.take(a.D); cv.take(kTileB * a.d); cv.take(kTileB * a.dv); cv.take(kTileB * a.D);
+    cv.take(kTileB * a.D); cv.take(kTileB * a.M); cv.take(kTileB * a.M); cv.take(kTileB * a.M);
+    cv.take(a.lay.nint * a.lay.L * 2);
+    return cv.bytes();
+}
+
+template <typename IO>
+cudaError_t stats_impl(const AttnArgs &a, cudaStream_t s) {
+    const size_t sm = smem_keystats(a);
+    cudaError_t e = set_smem(k_keystats<IO>, sm);
+    if (e != cudaSuccess) return e;
+    LUNA_LAUNCH("keystats", k_keystats<IO>, dim3(a.nsplit, a.B * a.H), kThreads, sm, s, a);
+    return cudaGetLastError();
+}
+
+template <typename IO>
+cudaError_t fwd_impl(const AttnArgs &a, cudaStream_t s) {
+    cudaError_t e = stats_impl<IO>(a, s);
+    if (e != cudaSuccess) return e;
+    const size_t sm = smem_query(a);
+    if ((e = set_smem(k_query<IO>, sm)) != cudaSuccess) return e;
+    LUNA_LAUNCH("query", k_query<IO>, dim3((a.n + kTileQ - 1) / kTileQ, a.B * a.H), kThreads, sm, s, a);
+    return cudaGetLastError();
+}
+
+template <typename IO>
+cudaError_t bwd_impl(const AttnArgs &a, bool have_stats, cudaStream_t s) {
+    cudaError_t e;
+    if (!have_stats && (e = stats_impl<IO>(a, s)) != cudaSuccess) return e;
+    size_t sm = smem_bwd_query(a);
+    if ((e = set_smem(k_bwd_query<IO>, sm)) != cudaSuccess) return e;
+    LUNA_LAUNCH("bwd_query", k_bwd_query<IO>, dim3(a.nsplit_b, a.B * a.H), kThreads, sm, s, a);
+    if ((e = cudaGetLastError()) != cudaSuccess) return e;
+    sm = smem_bwd_key(a);
+    if ((e = set_smem(k_bwd_key<IO>, sm)) != cudaSuccess) return e;
+    LUNA_LAUNCH("bwd_key", k_bwd_key<IO>, dim3(a.nsplit_b, a.B * a.H), kThreads, sm, s, a);
+    if ((e = cudaGetLastError()) != cudaSuccess) return e;
+    return launch_grad_reduce(a, 2 * a.B * a.H * a.nsplit_b, s);
+}
+
+}  // namespace
+
+size_t simt_max_smem(const AttnArgs &a) {
+    size_t m = smem_keystats(a);
+    m = m > smem_query(a) ? m : smem_query(a);
+    m = m > smem_bwd_query(a) ? m : smem_bwd_query(a);
+    m = m > smem_bwd_key(a) ? m : smem_bwd_key(a);
+    return m;
+}
+
+cudaError_t launch_grad_reduce(const AttnArgs &a, int nparts, cudaStream_t s) {
+    const int blocks = (a.gsize + kThreads - 1) / kThreads;
+    LUNA_LAUNCH("grad_sum", k_grad_sum, blocks, kThreads, 0, s, a.gpart, nparts, a.gsize, a.hist);
+    cudaError_t e = cudaGetLastError();
+    if (e != cudaSuccess) return e;
+    LUNA_LAUNCH("mlp_grads", k_mlp_grads, 1, kThreads, 0, s, a.lay, a.table, a.hist, a.grads);
+    return cudaGetLastError();
+}
+
+cudaError_t launch_featmap(const TableLayout &lay, const char *table, const void *X, luna_dtype xt, int64_t rows,
+                           float *Phi, cudaStream_t s) {
+    HostCarve cv; carve_phi_host(cv, lay);
+    const size_t sm = cv.bytes();
+    int64_t work = rows * lay.M;
+    int blocks = (int)((work + kThreads - 1) / kThreads);
+    if (blocks > 4096) blocks = 4096;
+    if (blocks < 1) blocks = 1;
+    cudaError_t e;
+    if (xt == LUNA_F32) {
+        if ((e = set_smem(k_featmap<float>, sm)) != cudaSuccess) return e;
+        k_featmap<float><<<blocks, kThreads, sm, s>>>(lay, table, static_cast<const float *>(X), rows, Phi);
+    } else {
+        if ((e = set_smem(k_featmap<__nv_bfloat16>, sm)) != cudaSuccess) return e;
+        k_featmap<__nv_bfloat16><<<blocks, kThreads, sm, s>>>(lay, table, static_cast<const __nv_bfloat16 *>(X),
+                                                              rows, Phi);
+    }
+    return cudaGetLastError();
+}
+
+cudaError_t launch_simt_stats(const AttnArgs &a, luna_dtype io, cudaStream_t s) {
+    return io == LUNA_F32 ? stats_impl<float>(a, s) : stats_impl<__nv_bfloat16>(a, s);
+}
+cudaError_t launch_simt_fwd(const AttnArgs &a, luna_dtype io, cudaStream_t s) {
+    return io == LUNA_F32 ? fwd_impl<float>(a, s) : fwd_impl<__nv_bfloat16>(a, s);
+}
+cudaError_t launch_simt_bwd(const AttnArgs &a, luna_dtype io, bool have_stats, cudaStream_t s) {
+    return io == LUNA_F32 ? bwd_impl<float>(a, have_stats, s) : bwd_impl<__nv_bfloat16>(a, have_stats, s);
+}
+
+}  // namespace luna

@@ -1,0 +1,47 @@
+// Launch arguments and entry points of the generic (CUDA-core, fp32) kernels.
+#pragma once
+
+#include "luna_common.cuh"
+
+namespace luna {
+
+struct AttnArgs {
+    int B, H, n, d, dv, M, L, D;
+    float eps;
+    TableLayout lay;
+    const char *table;
+    const void *Q, *K, *V, *dO;
+    void *O, *dQ, *dK, *dV;
+    const int32_t *lengths;
+    // non-causal statistics
+    int nsplit, rows_per_split;        // key-statistics splits per head
+    float *S_part, *z_part;            // [BH][nsplit][D][dv], [BH][nsplit][D]
+    float *S_fin, *z_fin;              // [BH][D][dv], [BH][D]
+    int *counters;                     // [2*BH], zero on entry
+    // backward
+    int nsplit_b, rows_per_split_b;
+    float *dS_part, *dz_part, *dS_fin, *dz_fin;
+    float *gpart;                      // [2 * BH * nsplit_b][gsize] parameter-gradient partials
+    int gsize;                         // M*d + M + nint*L*2
+    float *hist;                       // [nint][L][2] reduced histogram
+    luna_phi_grads grads;
+    // causal
+    int chunk, seg_len, nseg;          // state segments of seg_len rows (multiple of chunk)
+    float *seg_S, *seg_z;              // [BH][nseg+1][D][dv], [BH][nseg+1][D]: prefix at each segment start, total last
+    float *seg_dS, *seg_dz;            // [BH][nseg][D][dv], [BH][nseg][D]: suffix after segment end
+    float *rowstat;                    // [BH][n][2]: (den_i, dden_i) of the backward pass
+};
+
+cudaError_t launch_phi_prepare(const luna_phi_params &prm, const TableLayout &lay, void *table, cudaStream_t s);
+cudaError_t launch_featmap(const TableLayout &lay, const char *table, const void *X, luna_dtype xt, int64_t rows,
+                           float *Phi, cudaStream_t s);
+cudaError_t launch_simt_fwd(const AttnArgs &a, luna_dtype io, cudaStream_t s);
+cudaError_t launch_simt_stats(const AttnArgs &a, luna_dtype io, cudaStream_t s);
+cudaError_t launch_simt_bwd(const AttnArgs &a, luna_dtype io, bool have_stats, cudaStream_t s);
+cudaError_t launch_grad_reduce(const AttnArgs &a, int nparts, cudaStream_t s);
+cudaError_t launch_causal_fwd(const AttnArgs &a, luna_dtype io, bool write_state, cudaStream_t s);
+cudaError_t launch_causal_bwd(const AttnArgs &a, luna_dtype io, bool have_state, cudaStream_t s);
+size_t simt_max_smem(const AttnArgs &a);
+size_t causal_max_smem(const AttnArgs &a);
+
+}  // namespace luna

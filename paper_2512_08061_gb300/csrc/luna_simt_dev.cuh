@@ -1,0 +1,235 @@
+// Device helpers shared by the CUDA-core kernels (non-causal and causal).
+#pragma once
+
+#include "luna_simt.cuh"
+
+namespace luna {
+namespace simt {
+namespace {  // internal linkage in every translation unit that includes this
+
+constexpr int kThreads = 256;
+constexpr int kTileK = 32;  // rows per tile, key statistics
+constexpr int kTileQ = 32;  // rows per block, query pass
+constexpr int kTileB = 16;  // rows per tile, backward passes
+
+__host__ __device__ inline int r4(int x) { return (x + 3) & ~3; }
+
+struct Carve {
+    float *p;
+    __device__ float *take(int n) {
+        float *r = p;
+        p += r4(n);
+        return r;
+    }
+};
+
+struct HostCarve {
+    int n = 0;
+    void take(int k) { n += r4(k); }
+    size_t bytes() const { return (size_t)n * 4; }
+};
+
+struct SmemPhi {
+    float *T, *AB, *W, *b;
+};
+
+__device__ SmemPhi carve_phi(Carve &cv, const TableLayout &lay) {
+    SmemPhi s;
+    s.T = cv.take(lay.Ppad);
+    s.AB = cv.take(lay.nint * lay.L * 2);
+    s.W = cv.take(lay.M * lay.d);
+    s.b = cv.take(lay.M);
+    return s;
+}
+void carve_phi_host(HostCarve &cv, const TableLayout &lay) {
+    cv.take(lay.Ppad); cv.take(lay.nint * lay.L * 2); cv.take(lay.M * lay.d); cv.take(lay.M);
+}
+
+__device__ void load_phi(const SmemPhi &s, const TableLayout &lay, const char *table) {
+    const float *T = reinterpret_cast<const float *>(table + lay.off_T);
+    const float *AB = reinterpret_cast<const float *>(table + lay.off_AB);
+    const float *W = reinterpret_cast<const float *>(table + lay.off_W);
+    const float *b = reinterpret_cast<const float *>(table + lay.off_b);
+    for (int e = threadIdx.x; e < lay.Ppad; e += blockDim.x) s.T[e] = T[e];
+    for (int e = threadIdx.x; e < lay.nint * lay.L * 2; e += blockDim.x) s.AB[e] = AB[e];
+    for (int e = threadIdx.x; e < lay.M * lay.d; e += blockDim.x) s.W[e] = W[e];
+    for (int e = threadIdx.x; e < lay.M; e += blockDim.x) s.b[e] = b[e];
+}
+
+template <typename IO>
+__device__ void load_rows(float *dst, const IO *src, int count) {
+    for (int e = threadIdx.x; e < count; e += blockDim.x) dst[e] = io_load(src + e);
+}
+
+// phi for rows [0, nr) of a row tile sX (row stride d) into sPhi (row stride D).
+// Optionally keeps the projections u and their merged interval j.
+__device__ void phi_tile(const TableLayout &lay, const SmemPhi &s, const float *sX, int nr, float *sPhi, float *sU,
+                         int *sJ) {
+    const int M = lay.M, L = lay.L, d = lay.d, D = lay.D;
+    for (int e = threadIdx.x; e < nr * M; e += blockDim.x) {
+        const int r = e / M, i = e - r * M;
+        const float *x = sX + r * d;
+        const float *w = s.W + i * d;
+        float u = s.b[i];
+        for (int c = 0; c < d; ++c) u = fmaf(w[c], x[c], u);
+        const int j = interval_of(s.T, lay.Ppad, u);
+        const float *ab = s.AB + j * L * 2;
+        float *out = sPhi + r * D + i * L;
+        for (int l = 0; l < L; ++l) out[l] = fmaxf(fmaf(ab[2 * l], u, ab[2 * l + 1]), 0.0f);
+        if (sU) { sU[e] = u; sJ[e] = j; }
+    }
+}
+
+// acc[k][m] += sum_r A[r][f0+k] * Bm[r][c0+m];  z[k] += sum_r A[r][f0+k] * (w ? w[r] : 1)
+__device__ __forceinline__ void outer_accumulate(float (&acc)[8][8], float (&zacc)[8], bool do_z, const float *sA,
+                                                 int D, const float *sB, int dv, const float *sw, int nr, int f0,
+                                                 int c0) {
+    for (int r = 0; r < nr; ++r) {
+        float a8[8], b8[8];
+#pragma unroll
+        for (int k = 0; k < 8; ++k) {
+            a8[k] = (f0 + k < D) ? sA[r * D + f0 + k] : 0.0f;
+            b8[k] = (c0 + k < dv) ? sB[r * dv + c0 + k] : 0.0f;
+        }
+#pragma unroll
+        for (int k = 0; k < 8; ++k)
+#pragma unroll
+            for (int m = 0; m < 8; ++m) acc[k][m] = fmaf(a8[k], b8[m], acc[k][m]);
+        if (do_z) {
+            const float wr = sw ? sw[r] : 1.0f;
+#pragma unroll
+            for (int k = 0; k < 8; ++k) zacc[k] = fmaf(a8[k], wr, zacc[k]);
+        }
+    }
+}
+
+__device__ bool last_arrival(int *counter, int expected) {
+    __shared__ int s_flag;
+    __threadfence();
+    __syncthreads();
+    if (threadIdx.x == 0) s_flag = (atomicAdd(counter, 1) == expected - 1) ? 1 : 0;
+    __syncthreads();
+    if (s_flag) __threadfence();
+    return s_flag != 0;
+}
+
+// out[e] = sum_p part[p][e] in order p = 0..nparts-1
+__device__ void ordered_sum(const float *part, int nparts, int count, float *out) {
+    for (int e = threadIdx.x; e < count; e += blockDim.x) {
+        float s = 0.0f;
+        for (int p = 0; p < nparts; ++p) s += __ldcg(part + (size_t)p * count + e);
+        out[e] = s;
+    }
+}
+
+// Exclusive scan over partials in order: forward (out[p] = sum_{q<p} part[q],
+// out[nparts] = total) or reverse (out[p] = sum_{q>p} part[q]).
+__device__ void exclusive_scan(const float *part, int nparts, int count, float *out, bool reverse) {
+    for (int e = threadIdx.x; e < count; e += blockDim.x) {
+        float s = 0.0f;
+        if (!reverse) {
+            for (int p = 0; p < nparts; ++p) {
+                out[(size_t)p * count + e] = s;
+                s += __ldcg(part + (size_t)p * count + e);
+            }
+            out[(size_t)nparts * count + e] = s;
+        } else {
+            for (int p = nparts - 1; p >= 0; --p) {
+                out[(size_t)p * count + e] = s;
+                s += __ldcg(part + (size_t)p * count + e);
+            }
+        }
+    }
+}
+
+// Writes a (D x dv) register-tiled accumulator and its z-vector to a partial slot.
+__device__ void store_tile(const float (&acc)[8][8], const float (&zacc)[8], bool active, int tc, int f0, int c0,
+                           int D, int dv, float *Sp, float *zp) {
+    if (!active) return;
+#pragma unroll
+    for (int k = 0; k < 8; ++k)
+#pragma unroll
+        for (int m = 0; m < 8; ++m)
+            if (f0 + k < D && c0 + m < dv) Sp[(f0 + k) * dv + c0 + m] = acc[k][m];
+    if (tc == 0)
+#pragma unroll
+        for (int k = 0; k < 8; ++k)
+            if (f0 + k < D) zp[f0 + k] = zacc[k];
+}
+
+// ---------------------------------------------------------------------------
+// backward through phi for a tile: dU = sum_l dPhi * dphi/du, histogram of
+// the channel-MLP gradient statistics, then dX = dU W and dW += dU^T X.
+
+struct GradAcc {
+    float dW[16];  // entries threadIdx.x + k * blockDim.x of the M*d matrix
+    float db;      // entry threadIdx.x of b (if < M)
+};
+
+__device__ void phi_backward_tile(const TableLayout &lay, const SmemPhi &s, const float *sX, int nr,
+                                  const float *sPhi, const float *sdPhi, const float *sU, const int *sJ, float *sdU,
+                                  float *shist, GradAcc &g) {
+    const int M = lay.M, L = lay.L, d = lay.d, D = lay.D;
+    for (int e = threadIdx.x; e < nr * M; e += blockDim.x) {
+        const int r = e / M, i = e - r * M;
+        const float u = sU[e];
+        const int j = sJ[e];
+        const float *ab = s.AB + j * L * 2;
+        float du = 0.0f;
+        for (int l = 0; l < L; ++l) {
+            const int f = r * D + i * L + l;
+            if (sPhi[f] > 0.0f) {  // outer ReLU on
+                const float gl = sdPhi[f];
+                du = fmaf(gl, ab[2 * l], du);
+                if (gl != 0.0f) {
+                    atomicAdd(shist + (j * L + l) * 2, gl);
+                    atomicAdd(shist + (j * L + l) * 2 + 1, gl * u);
+                }
+            }
+        }
+        sdU[e] = du;
+    }
+    __syncthreads();
+    for (int k = 0; k < 16; ++k) {
+        const int e = threadIdx.x + k * blockDim.x;
+        if (e >= M * d) break;
+        const int i = e / d, c = e - i * d;
+        float acc = g.dW[k];
+        for (int r = 0; r < nr; ++r) acc = fmaf(sdU[r * M + i], sX[r * d + c], acc);
+        g.dW[k] = acc;
+    }
+    if (threadIdx.x < M)
+        for (int r = 0; r < nr; ++r) g.db += sdU[r * M + threadIdx.x];
+}
+
+template <typename IO>
+__device__ void store_dx(const TableLayout &lay, const SmemPhi &s, const float *sdU, int nr, IO *dX) {
+    const int M = lay.M, d = lay.d;
+    for (int e = threadIdx.x; e < nr * d; e += blockDim.x) {
+        const int r = e / d, c = e - r * d;
+        float acc = 0.0f;
+        for (int i = 0; i < M; ++i) acc = fmaf(sdU[r * M + i], s.W[i * d + c], acc);
+        io_store(dX + e, acc);
+    }
+}
+
+__device__ void store_grad_partial(const TableLayout &lay, const GradAcc &g, const float *shist, float *gp) {
+    const int Md = lay.M * lay.d;
+    for (int k = 0; k < 16; ++k) {
+        const int e = threadIdx.x + k * blockDim.x;
+        if (e >= Md) break;
+        gp[e] = g.dW[k];
+    }
+    if (threadIdx.x < lay.M) gp[Md + threadIdx.x] = g.db;
+    for (int e = threadIdx.x; e < lay.nint * lay.L * 2; e += blockDim.x) gp[Md + lay.M + e] = shist[e];
+}
+
+template <typename K>
+cudaError_t set_smem(K kernel, size_t bytes) {
+    return cudaFuncSetAttribute(kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)bytes);
+}
+
+
+}  // namespace
+}  // namespace simt
+}  // namespace luna

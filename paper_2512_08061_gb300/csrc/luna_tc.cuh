@@ -1,0 +1,18 @@
+// Tensor-core (tcgen05 / TMEM / TMA) path for bf16 I/O on sm_103a.
+#pragma once
+
+#include "luna_simt.cuh"
+
+namespace luna {
+
+struct TcPlan {
+    bool eligible = false;   // shape and dtype handled by the tensor-core kernels
+    size_t ws_fwd = 0, ws_bwd = 0;
+};
+
+TcPlan tc_plan(const luna_attn_desc &ad, const TableLayout &lay);
+bool tc_inputs_ok(const TcPlan &p, const void *a, const void *b, const void *c, const void *d);
+cudaError_t launch_tc_fwd(const TcPlan &p, const AttnArgs &a, char *ws, cudaStream_t s);
+cudaError_t launch_tc_bwd(const TcPlan &p, const AttnArgs &a, char *ws, bool have_stats, cudaStream_t s);
+
+}  // namespace luna

@@ -1,0 +1,234 @@
+"""Thin Python binding of the C ABI in include/luna.h (argument marshalling only).
+
+Every function here has the name of the C entry point it calls and does no
+arithmetic of its own: tensors are passed as device pointers, the stream as
+torch's current CUDA stream.  PyTorch provides device memory and streams.
+If the compiled library is missing this module raises at import time; there
+is no fallback implementation.
+"""
+from __future__ import annotations
+
+import ctypes
+import os
+
+import torch
+
+from . import build as _build
+
+LUNA_OK = 0
+STATUS_NAMES = {0: "LUNA_OK", 1: "LUNA_ERR_INVALID_ARG", 2: "LUNA_ERR_UNSUPPORTED", 3: "LUNA_ERR_WORKSPACE",
+                4: "LUNA_ERR_CUDA", 5: "LUNA_ERR_DEVICE_TIMEOUT"}
+LUNA_F32, LUNA_BF16 = 0, 1
+_DTYPES = {torch.float32: LUNA_F32, torch.bfloat16: LUNA_BF16}
+# names of the tensor-core kernels accepted by luna_profile_start
+TC_KERNELS: list[str] = []
+
+
+class LunaError(RuntimeError):
+    def __init__(self, status: int, where: str):
+        super().__init__(f"{where}: {STATUS_NAMES.get(status, status)}")
+        self.status = status
+
+
+class PhiDesc(ctypes.Structure):
+    _fields_ = [("M", ctypes.c_int), ("L", ctypes.c_int), ("hidden", ctypes.c_int)]
+
+
+class PhiParams(ctypes.Structure):
+    _fields_ = [(k, ctypes.c_void_p) for k in ("W", "b", "w1", "b1", "w2", "b2")]
+
+
+class PhiGrads(ctypes.Structure):
+    _fields_ = [(k, ctypes.c_void_p) for k in ("dW", "db", "dw1", "db1", "dw2", "db2")]
+
+
+class AttnDesc(ctypes.Structure):
+    _fields_ = [("B", ctypes.c_int), ("H", ctypes.c_int), ("n", ctypes.c_int), ("d", ctypes.c_int),
+                ("dv", ctypes.c_int), ("causal", ctypes.c_int), ("chunk", ctypes.c_int), ("eps", ctypes.c_float),
+                ("io", ctypes.c_int)]
+
+
+def library_path() -> str:
+    return _build.LIB
+
+
+def _load():
+    path = library_path()
+    if not os.path.exists(path):
+        raise ImportError(f"LUNA CUDA library not built ({path}); run paper_2512_08061_gb300.build.build()")
+    lib = ctypes.CDLL(path)
+    P, S, I, I64 = ctypes.c_void_p, ctypes.c_size_t, ctypes.c_int, ctypes.c_int64
+    pd, ad = ctypes.POINTER(PhiDesc), ctypes.POINTER(AttnDesc)
+    sig = {
+        "luna_status_string": ([I], ctypes.c_char_p),
+        "luna_version": ([], I),
+        "luna_phi_table_size": ([pd, I, ctypes.POINTER(S)], I),
+        "luna_phi_prepare": ([pd, I, ctypes.POINTER(PhiParams), P, S, P], I),
+        "luna_featmap": ([pd, I, P, P, I, I64, P, P], I),
+        "luna_workspace_size": ([ad, pd, I, ctypes.POINTER(S)], I),
+        "luna_state_size": ([ad, pd, ctypes.POINTER(S)], I),
+        "luna_attn_fwd": ([ad, pd, P, P, P, P, P, P, P, P, S, P], I),
+        "luna_attn_bwd": ([ad, pd, P, P, P, P, P, P, P, P, P, P, ctypes.POINTER(PhiGrads), P, S, P], I),
+        "luna_device_status": ([P, P], I),
+        "luna_profile_start": ([ctypes.c_char_p], I),
+        "luna_profile_stop": ([ctypes.POINTER(ctypes.c_double), ctypes.POINTER(I)], I),
+        "luna_launch_count": ([], ctypes.c_uint64),
+    }
+    for name, (args, res) in sig.items():
+        fn = getattr(lib, name)
+        fn.argtypes = args
+        fn.restype = res
+    return lib
+
+
+_lib = _load()
+EXPORTED = ("luna_status_string", "luna_version", "luna_phi_table_size", "luna_phi_prepare", "luna_featmap",
+            "luna_workspace_size", "luna_state_size", "luna_attn_fwd", "luna_attn_bwd", "luna_device_status",
+            "luna_profile_start", "luna_profile_stop", "luna_launch_count")
+
+
+def _ptr(t):
+    if t is None:
+        return None
+    return ctypes.c_void_p(t.data_ptr())
+
+
+def _stream(stream=None):
+    if stream is None:
+        stream = torch.cuda.current_stream()
+    return ctypes.c_void_p(stream.cuda_stream)
+
+
+def _check(st: int, where: str) -> None:
+    if st != LUNA_OK:
+        raise LunaError(st, where)
+
+
+def _io_code(t: torch.Tensor) -> int:
+    if t.dtype not in _DTYPES:
+        raise TypeError(f"unsupported dtype {t.dtype}")
+    return _DTYPES[t.dtype]
+
+
+def phi_desc(M: int, L: int, hidden: int) -> PhiDesc:
+    return PhiDesc(M, L, hidden)
+
+
+def attn_desc(B, H, n, d, dv, causal=False, chunk=0, eps=1e-6, io=LUNA_BF16) -> AttnDesc:
+    return AttnDesc(B, H, n, d, dv, int(bool(causal)), chunk, eps, io)
+
+
+def luna_status_string(status: int) -> str:
+    return _lib.luna_status_string(status).decode()
+
+
+def luna_version() -> int:
+    return _lib.luna_version()
+
+
+def luna_phi_table_size(pd: PhiDesc, d: int) -> int:
+    out = ctypes.c_size_t(0)
+    _check(_lib.luna_phi_table_size(ctypes.byref(pd), d, ctypes.byref(out)), "luna_phi_table_size")
+    return out.value
+
+
+def luna_phi_prepare(pd: PhiDesc, d: int, params: dict, table: torch.Tensor, stream=None) -> None:
+    pp = PhiParams(*[_ptr(params[k]) for k in ("W", "b", "w1", "b1", "w2", "b2")])
+    _check(_lib.luna_phi_prepare(ctypes.byref(pd), d, ctypes.byref(pp), _ptr(table), table.numel() * table.element_size(),
+                                 _stream(stream)), "luna_phi_prepare")
+
+
+def luna_featmap(pd: PhiDesc, d: int, table: torch.Tensor, X: torch.Tensor, Phi: torch.Tensor, stream=None) -> None:
+    rows = X.numel() // d if d else 0
+    _check(_lib.luna_featmap(ctypes.byref(pd), d, _ptr(table), _ptr(X), _io_code(X), rows, _ptr(Phi), _stream(stream)),
+           "luna_featmap")
+
+
+def luna_workspace_size(ad: AttnDesc, pd: PhiDesc, backward: bool) -> int:
+    out = ctypes.c_size_t(0)
+    _check(_lib.luna_workspace_size(ctypes.byref(ad), ctypes.byref(pd), int(bool(backward)), ctypes.byref(out)),
+           "luna_workspace_size")
+    return out.value
+
+
+def luna_state_size(ad: AttnDesc, pd: PhiDesc) -> int:
+    out = ctypes.c_size_t(0)
+    _check(_lib.luna_state_size(ctypes.byref(ad), ctypes.byref(pd), ctypes.byref(out)), "luna_state_size")
+    return out.value
+
+
+def luna_attn_fwd(ad, pd, table, Q, K, V, lengths, O, state, workspace, stream=None) -> None:
+    _check(_lib.luna_attn_fwd(ctypes.byref(ad), ctypes.byref(pd), _ptr(table), _ptr(Q), _ptr(K), _ptr(V),
+                              _ptr(lengths), _ptr(O), _ptr(state), _ptr(workspace),
+                              workspace.numel() * workspace.element_size(), _stream(stream)), "luna_attn_fwd")
+
+
+def luna_attn_bwd(ad, pd, table, Q, K, V, dO, lengths, state, dQ, dK, dV, grads: dict, workspace, stream=None) -> None:
+    pg = PhiGrads(*[_ptr(grads[k]) for k in ("dW", "db", "dw1", "db1", "dw2", "db2")])
+    _check(_lib.luna_attn_bwd(ctypes.byref(ad), ctypes.byref(pd), _ptr(table), _ptr(Q), _ptr(K), _ptr(V), _ptr(dO),
+                              _ptr(lengths), _ptr(state), _ptr(dQ), _ptr(dK), _ptr(dV), ctypes.byref(pg),
+                              _ptr(workspace), workspace.numel() * workspace.element_size(), _stream(stream)),
+           "luna_attn_bwd")
+
+
+def luna_device_status(workspace: torch.Tensor, stream=None) -> int:
+    return _lib.luna_device_status(_ptr(workspace), _stream(stream))
+
+
+def luna_profile_start(kernel: str) -> None:
+    _check(_lib.luna_profile_start(kernel.encode()), "luna_profile_start")
+
+
+def luna_profile_stop() -> tuple[float, int]:
+    ms, n = ctypes.c_double(0.0), ctypes.c_int(0)
+    _check(_lib.luna_profile_stop(ctypes.byref(ms), ctypes.byref(n)), "luna_profile_stop")
+    return ms.value, n.value
+
+
+def luna_launch_count() -> int:
+    return int(_lib.luna_launch_count())
+
+
+# ---------------------------------------------------------------------------
+# convenience: buffers sized by the library, allocated with torch
+
+def alloc_bytes(nbytes: int, device) -> torch.Tensor:
+    """A 256-byte aligned uint8 device buffer (torch's caching allocator aligns to 512)."""
+    return torch.empty(max(int(nbytes), 256), dtype=torch.uint8, device=device)
+
+
+class Luna:
+    """Owns the table, workspace and state buffers of one problem shape."""
+
+    def __init__(self, B, H, n, d, dv, M, L, hidden=64, causal=False, eps=1e-6, io=torch.bfloat16, chunk=0,
+                 device="cuda"):
+        self.pd = phi_desc(M, L, hidden)
+        self.ad = attn_desc(B, H, n, d, dv, causal, chunk, eps, _DTYPES[io])
+        self.d = d
+        self.device = torch.device(device)
+        self.table = alloc_bytes(luna_phi_table_size(self.pd, d), self.device)
+        self.ws = alloc_bytes(max(luna_workspace_size(self.ad, self.pd, False),
+                                  luna_workspace_size(self.ad, self.pd, True)), self.device)
+        self.state = alloc_bytes(luna_state_size(self.ad, self.pd), self.device)
+
+    def prepare(self, params: dict, stream=None):
+        luna_phi_prepare(self.pd, self.d, params, self.table, stream)
+
+    def forward(self, Q, K, V, lengths=None, O=None, save_state=True, stream=None):
+        if O is None:
+            O = torch.empty(Q.shape[:-1] + (self.ad.dv,), dtype=Q.dtype, device=Q.device)
+        luna_attn_fwd(self.ad, self.pd, self.table, Q, K, V, lengths, O, self.state if save_state else None,
+                      self.ws, stream)
+        return O
+
+    def backward(self, Q, K, V, dO, lengths=None, use_state=True, out=None, stream=None):
+        if out is None:
+            M, L, hid = self.pd.M, self.pd.L, self.pd.hidden
+            f32 = dict(dtype=torch.float32, device=Q.device)
+            out = {"dQ": torch.empty_like(Q), "dK": torch.empty_like(K), "dV": torch.empty_like(V),
+                   "dW": torch.empty(M, self.d, **f32), "db": torch.empty(M, **f32),
+                   "dw1": torch.empty(L, hid, **f32), "db1": torch.empty(L, hid, **f32),
+                   "dw2": torch.empty(L, hid, **f32), "db2": torch.empty(L, **f32)}
+        luna_attn_bwd(self.ad, self.pd, self.table, Q, K, V, dO, lengths, self.state if use_state else None,
+                      out["dQ"], out["dK"], out["dV"], out, self.ws, stream)
+        return out

@@ -1,0 +1,85 @@
+"""Helpers for the GPU parity tests: seeded cases, device transfer, error metric."""
+from __future__ import annotations
+
+import numpy as np
+
+import oracle
+import synth
+
+TOL = {"f32": 1e-4, "bf16": 2e-2}
+KINK_MARGIN = 1e-5
+
+
+def relerr(got, ref) -> float:
+    """max_i |g_i - r_i| / max(|r_i|, rms(r)): the element-wise relative error,
+    floored at the tensor's rms so that near-zero entries are judged on the
+    scale of the tensor."""
+    g = np.asarray(got, dtype=np.float64)
+    r = np.asarray(ref, dtype=np.float64)
+    if r.size == 0:
+        return 0.0
+    rms = float(np.sqrt(np.mean(r * r)))
+    if rms == 0.0:
+        return float(np.max(np.abs(g)))
+    return float(np.max(np.abs(g - r) / np.maximum(np.abs(r), rms)))
+
+
+def to_device(t: "synth.IOTensor"):
+    import torch
+    if t.io == "f32":
+        return torch.from_numpy(np.ascontiguousarray(t.raw)).cuda()
+    return torch.from_numpy(np.ascontiguousarray(t.raw).view(np.int16)).cuda().view(torch.bfloat16)
+
+
+def to_host(x) -> np.ndarray:
+    import torch
+    return x.detach().to(torch.float64).cpu().numpy()
+
+
+class Case:
+    def __init__(self, B, H, n, d, M, L, io, causal=False, seed=0, qkv_scale=1.0, len_range=None, hidden=64,
+                 eps=1e-6, dv=None, with_grad=False, lengths=None):
+        self.B, self.H, self.n, self.d, self.M, self.L = B, H, n, d, M, L
+        self.dv = dv or d
+        self.io, self.causal, self.eps, self.hidden = io, causal, eps, hidden
+        self.params = synth.phi_params(seed, d, M, L, hidden)
+        self.inp = synth.attn_inputs(seed, B, H, n, d, self.dv, io, qkv_scale, len_range, with_grad)
+        if lengths is not None:
+            self.inp["lengths"] = np.asarray(lengths, dtype=np.int32)
+        self.lengths = self.inp["lengths"]
+
+    # ---- device side
+    def luna(self, chunk=0):
+        import torch
+        import paper_2512_08061_gb300.luna as L
+        lu = L.Luna(self.B, self.H, self.n, self.d, self.dv, self.M, self.L, self.hidden, self.causal, self.eps,
+                    torch.float32 if self.io == "f32" else torch.bfloat16, chunk)
+        params = {k: torch.from_numpy(v).cuda() for k, v in self.params.items()}
+        lu.prepare(params)
+        self.dev = {k: to_device(self.inp[k]) for k in ("Q", "K", "V", "dO") if k in self.inp}
+        self.dev["lengths"] = None if self.lengths is None else torch.from_numpy(self.lengths).cuda()
+        return lu
+
+    def run_fwd(self, lu, save_state=True):
+        d = self.dev
+        return lu.forward(d["Q"], d["K"], d["V"], d["lengths"], save_state=save_state)
+
+    def run_bwd(self, lu, use_state=True):
+        d = self.dev
+        return lu.backward(d["Q"], d["K"], d["V"], d["dO"], d["lengths"], use_state=use_state)
+
+    # ---- oracle side
+    def oracle_fwd(self):
+        i = self.inp
+        return oracle.attn_fwd(self.params, i["Q"].value, i["K"].value, i["V"].value, self.lengths, self.causal,
+                               self.eps)
+
+    def oracle_bwd(self):
+        i = self.inp
+        return oracle.attn_bwd(self.params, i["Q"].value, i["K"].value, i["V"].value, i["dO"].value, self.lengths,
+                               self.causal, self.eps)
+
+    def smooth_rows(self, which: str) -> np.ndarray:
+        """Rows whose feature map has no ReLU argument within rounding distance of
+        its kink: there the gradient is unique at fp32 resolution."""
+        return oracle.kink_margin(self.params, self.inp[which].value) > KINK_MARGIN

@@ -1,0 +1,88 @@
+"""The C-ABI library loads and exports every entry point that include/luna.h
+declares; size queries and argument checks work without a GPU (no compute
+call is made here)."""
+import ctypes
+import os
+import re
+
+import pytest
+
+ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+
+
+@pytest.fixture(scope="module")
+def L():
+    from paper_2512_08061_gb300 import build
+    build.build()
+    import paper_2512_08061_gb300.luna as L
+    return L
+
+
+def declared_entry_points():
+    src = open(os.path.join(ROOT, "include", "luna.h")).read()
+    src = re.sub(r"/\*.*?\*/", "", src, flags=re.S)
+    return sorted(set(re.findall(r"\b(luna_[a-z_0-9]+)\s*\(", src)))
+
+
+def test_header_declares_the_boundary():
+    names = declared_entry_points()
+    for required in ("luna_phi_prepare", "luna_featmap", "luna_attn_fwd", "luna_attn_bwd", "luna_workspace_size",
+                     "luna_status_string"):
+        assert required in names
+
+
+def test_every_declared_symbol_is_exported(L):
+    lib = ctypes.CDLL(L.library_path())
+    for name in declared_entry_points():
+        assert hasattr(lib, name), f"{name} declared in include/luna.h but not exported"
+    assert set(L.EXPORTED) <= set(declared_entry_points())
+
+
+def test_status_strings(L):
+    assert L.luna_status_string(0) == "LUNA_OK"
+    assert L.luna_status_string(5) == "LUNA_ERR_DEVICE_TIMEOUT"
+    assert L.luna_version() >= 100
+
+
+def test_size_queries(L):
+    pd = L.phi_desc(8, 8, 64)
+    t = L.luna_phi_table_size(pd, 32)
+    assert t % 256 == 0 and t > 4 * (512 + 513 * 16)
+    ad = L.attn_desc(32, 4, 4096, 32, 32, False, 0, 1e-6, L.LUNA_BF16)
+    fwd, bwd = L.luna_workspace_size(ad, pd, False), L.luna_workspace_size(ad, pd, True)
+    assert 0 < fwd <= bwd
+    assert L.luna_state_size(ad, pd) >= 32 * 4 * (64 * 32 + 64) * 4
+    # empty problems need no real workspace
+    ad0 = L.attn_desc(0, 4, 4096, 32, 32)
+    assert L.luna_workspace_size(ad0, pd, True) == 256
+
+
+def test_argument_errors_return_before_launch(L):
+    pd = L.phi_desc(8, 8, 64)
+    with pytest.raises(L.LunaError) as e:
+        L.luna_phi_table_size(L.phi_desc(0, 8, 64), 32)
+    assert e.value.status == 1
+    with pytest.raises(L.LunaError) as e:
+        L.luna_phi_table_size(L.phi_desc(8, 8, 128), 32)  # L*hidden > 512
+    assert e.value.status == 2
+    with pytest.raises(L.LunaError) as e:
+        L.luna_workspace_size(L.attn_desc(1, 1, 16, 256, 32), pd, False)  # d > 128
+    assert e.value.status == 2
+    with pytest.raises(L.LunaError) as e:
+        L.luna_workspace_size(L.attn_desc(1, 1, 16, 32, 32, eps=-1.0), pd, False)
+    assert e.value.status == 1
+    with pytest.raises(L.LunaError) as e:
+        L.luna_workspace_size(L.attn_desc(1, 1, 16, 32, 32, chunk=17), pd, False)
+    assert e.value.status == 1
+    # NULL pointers are rejected before any CUDA call
+    lib = L._lib
+    ad = L.attn_desc(1, 1, 16, 32, 32)
+    st = lib.luna_attn_fwd(ctypes.byref(ad), ctypes.byref(pd), None, None, None, None, None, None, None, None, 0, None)
+    assert st == 1
+    st = lib.luna_phi_prepare(ctypes.byref(pd), 32, None, None, 0, None)
+    assert st == 1
+    # an empty problem is a successful no-op
+    ad0 = L.attn_desc(1, 1, 0, 32, 32)
+    st = lib.luna_attn_fwd(ctypes.byref(ad0), ctypes.byref(pd), None, None, None, None, None, None, None, None, 0,
+                           None)
+    assert st == 0

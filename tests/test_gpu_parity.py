@@ -1,0 +1,195 @@
+"""GPU parity: the CUDA path through the C ABI against the fp64 oracle on the
+same seeded inputs, at sizes that span several tiles and a ragged tail.
+
+Tolerances (max element-wise relative error, floored at the tensor's rms):
+1e-4 for fp32 I/O (fp32 arithmetic throughout) and 2e-2 for bf16 I/O (bf16
+tensor-core operands, fp32 accumulation).
+"""
+import math
+
+import numpy as np
+import pytest
+
+import oracle
+import synth
+from cases import TOL, Case, relerr, to_device, to_host
+
+pytestmark = pytest.mark.gpu
+
+
+@pytest.fixture(scope="module", autouse=True)
+def _lib():
+    torch = pytest.importorskip("torch")
+    if not torch.cuda.is_available():
+        pytest.skip("no CUDA device")
+    from paper_2512_08061_gb300 import build
+    build.build()
+
+
+# --------------------------------------------------------------------------
+# feature map
+
+@pytest.mark.parametrize("io,d,M", [("f32", 32, 8), ("bf16", 64, 8), ("f32", 128, 16), ("bf16", 128, 16)])
+def test_featmap(io, d, M):
+    import torch
+    import paper_2512_08061_gb300.luna as L
+    params = synth.phi_params(3, d, M, 8, 64)
+    X = synth.IOTensor(synth.normal(3, "fm.X", (1037, d)), io)
+    pd = L.phi_desc(M, 8, 64)
+    table = L.alloc_bytes(L.luna_phi_table_size(pd, d), "cuda")
+    L.luna_phi_prepare(pd, d, {k: torch.from_numpy(v).cuda() for k, v in params.items()}, table)
+    Phi = torch.empty(1037, M * 8, dtype=torch.float32, device="cuda")
+    L.luna_featmap(pd, d, table, to_device(X), Phi)
+    ref = oracle.featmap(params, X.value)
+    assert relerr(to_host(Phi), ref) < 1e-4
+    assert torch.all(Phi >= 0)
+
+
+def test_featmap_exact_at_kinks():
+    """Inputs placed exactly on (and one ulp around) the hidden-unit kinks: the
+    piecewise-linear table is continuous there and matches direct evaluation."""
+    import torch
+    import paper_2512_08061_gb300.luna as L
+    d = M = 4
+    Lc, hid = 8, 64
+    params = synth.phi_params(5, d, M, Lc, hid)
+    params["W"] = np.eye(d, dtype=np.float32)
+    params["b"] = np.zeros(d, dtype=np.float32)
+    t = (-params["b1"] / params["w1"]).astype(np.float32).ravel()
+    t = t[np.isfinite(t) & (np.abs(t) < 50)]
+    vals = np.concatenate([t, np.nextafter(t, np.float32(np.inf)), np.nextafter(t, np.float32(-np.inf))])
+    vals = np.resize(vals, (len(vals) + 3) // 4 * 4).astype(np.float32)
+    X = vals.reshape(-1, d)
+    pd = L.phi_desc(M, Lc, hid)
+    table = L.alloc_bytes(L.luna_phi_table_size(pd, d), "cuda")
+    L.luna_phi_prepare(pd, d, {k: torch.from_numpy(np.ascontiguousarray(v)).cuda() for k, v in params.items()}, table)
+    Phi = torch.empty(X.shape[0], M * Lc, dtype=torch.float32, device="cuda")
+    L.luna_featmap(pd, d, table, torch.from_numpy(X).cuda(), Phi)
+    ref = oracle.featmap(params, X.astype(np.float64))
+    assert relerr(to_host(Phi), ref) < 1e-5
+
+
+# --------------------------------------------------------------------------
+# forward
+
+FWD_CASES = [
+    # B, H, n, d, M, io, causal, len_range / lengths
+    dict(B=1, H=1, n=256, d=64, M=8, io="f32", causal=False),                  # the 256-token fp32 workload
+    dict(B=2, H=3, n=300, d=32, M=8, io="bf16", causal=False, lengths=[300, 177]),
+    dict(B=3, H=2, n=197, d=64, M=8, io="bf16", causal=False),                 # ViT-like ragged length
+    dict(B=1, H=2, n=333, d=128, M=16, io="bf16", causal=False, lengths=[260]),
+    dict(B=2, H=1, n=129, d=32, M=8, io="f32", causal=False, lengths=[1, 0]),
+    dict(B=1, H=2, n=300, d=32, M=8, io="f32", causal=True),
+    dict(B=2, H=2, n=270, d=64, M=8, io="bf16", causal=True, lengths=[270, 100]),
+    dict(B=1, H=1, n=400, d=128, M=16, io="bf16", causal=True),
+    dict(B=1, H=1, n=200, d=128, M=16, io="f32", causal=True),
+]
+
+
+def _case_id(c):
+    return f"{c['io']}-{'causal' if c['causal'] else 'full'}-B{c['B']}H{c['H']}n{c['n']}d{c['d']}M{c['M']}"
+
+
+@pytest.mark.parametrize("c", FWD_CASES, ids=_case_id)
+def test_forward(c):
+    case = Case(c["B"], c["H"], c["n"], c["d"], c["M"], 8, c["io"], c["causal"], seed=7,
+                qkv_scale=1.0 / math.sqrt(c["d"]), lengths=c.get("lengths"))
+    lu = case.luna()
+    O = to_host(case.run_fwd(lu))
+    ref = case.oracle_fwd()
+    assert relerr(O, ref) < TOL[c["io"]]
+    if case.lengths is not None:
+        for b, ln in enumerate(case.lengths):
+            assert np.all(O[b, :, ln:] == 0)
+
+
+# --------------------------------------------------------------------------
+# backward
+
+BWD_CASES = [
+    dict(B=1, H=1, n=256, d=64, M=8, io="f32", causal=False),
+    dict(B=2, H=3, n=300, d=32, M=8, io="bf16", causal=False, lengths=[300, 177]),
+    dict(B=1, H=2, n=197, d=64, M=8, io="bf16", causal=False),
+    dict(B=1, H=2, n=160, d=128, M=16, io="bf16", causal=False),
+    dict(B=1, H=2, n=300, d=32, M=8, io="f32", causal=True),
+    dict(B=2, H=1, n=270, d=64, M=8, io="bf16", causal=True, lengths=[270, 100]),
+    dict(B=1, H=1, n=200, d=128, M=16, io="bf16", causal=True),
+]
+
+
+@pytest.mark.parametrize("c", BWD_CASES, ids=_case_id)
+def test_backward(c):
+    case = Case(c["B"], c["H"], c["n"], c["d"], c["M"], 8, c["io"], c["causal"], seed=11,
+                qkv_scale=1.0 / math.sqrt(c["d"]), lengths=c.get("lengths"), with_grad=True)
+    lu = case.luna()
+    case.run_fwd(lu)
+    g = {k: to_host(v) for k, v in case.run_bwd(lu).items()}
+    ref = case.oracle_bwd()
+    tol = TOL[c["io"]]
+    okq, okk = case.smooth_rows("Q"), case.smooth_rows("K")
+    assert okq.mean() > 0.9 and okk.mean() > 0.9
+    assert relerr(g["dQ"][okq], ref["dQ"][okq]) < tol
+    assert relerr(g["dK"][okk], ref["dK"][okk]) < tol
+    assert relerr(g["dV"], ref["dV"]) < tol
+    for k in ("dQ", "dK", "dV"):
+        assert np.all(np.isfinite(g[k]))
+    for k in ("dW", "db", "dw1", "db1", "dw2", "db2"):
+        assert relerr(g[k], ref[k]) < tol, k
+    if case.lengths is not None:
+        for b, ln in enumerate(case.lengths):
+            for k in ("dQ", "dK", "dV"):
+                assert np.all(g[k][b, :, ln:] == 0)
+
+
+@pytest.mark.parametrize("causal", [False, True])
+def test_backward_with_and_without_saved_state(causal):
+    case = Case(2, 2, 200, 32, 8, 8, "f32", causal, seed=13, with_grad=True, lengths=[200, 150])
+    lu = case.luna()
+    case.run_fwd(lu)
+    a = {k: to_host(v) for k, v in case.run_bwd(lu, use_state=True).items()}
+    b = {k: to_host(v) for k, v in case.run_bwd(lu, use_state=False).items()}
+    for k in a:
+        assert relerr(a[k], b[k]) < 1e-5, k
+
+
+@pytest.mark.parametrize("causal", [False, True])
+def test_repeat_runs_are_bitwise_identical(causal):
+    case = Case(2, 2, 300, 64, 8, 8, "bf16", causal, seed=17, with_grad=True)
+    lu = case.luna()
+    O1 = to_host(case.run_fwd(lu))
+    g1 = {k: to_host(v) for k, v in case.run_bwd(lu).items()}
+    O2 = to_host(case.run_fwd(lu))
+    g2 = {k: to_host(v) for k, v in case.run_bwd(lu).items()}
+    assert np.array_equal(O1, O2)
+    for k in ("dQ", "dK", "dV"):
+        assert np.array_equal(g1[k], g2[k]), k
+
+
+def test_all_padded_and_empty():
+    import torch
+    case = Case(2, 1, 64, 32, 8, 8, "f32", False, seed=19, with_grad=True, lengths=[0, 0])
+    lu = case.luna()
+    O = to_host(case.run_fwd(lu))
+    assert np.all(O == 0)
+    g = case.run_bwd(lu)
+    for k, v in g.items():
+        assert torch.all(v == 0), k
+    # B = 0: a successful no-op that still defines the parameter gradients
+    empty = Case(0, 1, 64, 32, 8, 8, "f32", False, seed=19, with_grad=True)
+    lu = empty.luna()
+    g = empty.run_bwd(lu)
+    for k in ("dW", "db", "dw1", "db1", "dw2", "db2"):
+        assert torch.all(g[k] == 0)
+
+
+def test_unit_values_give_unit_outputs():
+    """V = 1 and eps = 0: every row with a positive normaliser outputs exactly 1
+    up to rounding (row-wise normalisation of Eq. kernel-attn)."""
+    import torch
+    case = Case(1, 2, 300, 32, 8, 8, "f32", False, seed=23, eps=0.0)
+    lu = case.luna()
+    case.dev["V"] = torch.ones_like(case.dev["V"])
+    O = to_host(case.run_fwd(lu))
+    nz = np.any(O != 0, axis=-1)
+    assert nz.mean() > 0.9
+    assert np.max(np.abs(O[nz] - 1.0)) < 1e-5
