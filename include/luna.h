@@ -166,6 +166,36 @@ luna_status luna_attn_bwd(const luna_attn_desc *ad, const luna_phi_desc *pd, con
  * synchronising or the copy failed (including an earlier asynchronous fault). */
 luna_status luna_device_status(void *workspace, void *stream);
 
+/* Size of the library-owned scratch array used by luna_attn_fwd_noalloc. */
+#define LUNA_NOALLOC_SCRATCH_BYTES (16u << 20)
+
+/* luna_attn_fwd without a caller-provided workspace.  The paper has no
+ * counterpart; this is a deployment convenience.
+ *
+ * Some callers hold only their input and output buffers and have no way to
+ * obtain device scratch memory: a custom operator inside an inference engine
+ * whose device-memory plan is fixed before it runs and that is handed nothing
+ * but its tensors, or host code that must not call into an allocator while it
+ * runs (fixed-latency loops).  For them this entry point allocates nothing:
+ * no cudaMalloc, cudaFree or allocating library routine is called.  Its
+ * scratch is one file-scope __device__ array of LUNA_NOALLOC_SCRATCH_BYTES
+ * (16 MiB) that every GPU which loads the library holds until the process
+ * exits; problems whose forward workspace (luna_workspace_size with
+ * backward = 0) exceeds it are rejected with LUNA_ERR_WORKSPACE before
+ * anything is launched.  Arguments and results are those of luna_attn_fwd
+ * with state = NULL (no key statistics are kept for a backward pass).
+ *
+ * The first call on a device, with that device current, looks up the array's
+ * device address (cudaGetSymbolAddress) and caches it; make that first call
+ * before any stream capture.  All calls in the process share the one array
+ * per device and leave their contents in it; each call clears what must start
+ * at zero.  Calls whose executions overlap on the GPU (different streams, or
+ * different host threads) race on the array and give undefined results: order
+ * them on one stream. */
+luna_status luna_attn_fwd_noalloc(const luna_attn_desc *ad, const luna_phi_desc *pd, const void *table,
+                                  const void *Q, const void *K, const void *V, const int32_t *lengths, void *O,
+                                  void *stream);
+
 /* Kernel timing (tracing aid, not needed for computation).  After
  * luna_profile_start(name), every launch of the library kernel `name` (e.g.
  * "bwd_query", "keystats"; the names are listed in the library's kernel

@@ -73,6 +73,7 @@ def _load():
         "luna_profile_start": ([ctypes.c_char_p], I),
         "luna_profile_stop": ([ctypes.POINTER(ctypes.c_double), ctypes.POINTER(I)], I),
         "luna_launch_count": ([], ctypes.c_uint64),
+        "luna_attn_fwd_noalloc": ([ad, pd, P, P, P, P, P, P, P], I),
     }
     for name, (args, res) in sig.items():
         fn = getattr(lib, name)
@@ -84,7 +85,7 @@ def _load():
 _lib = _load()
 EXPORTED = ("luna_status_string", "luna_version", "luna_phi_table_size", "luna_phi_prepare", "luna_featmap",
             "luna_workspace_size", "luna_state_size", "luna_attn_fwd", "luna_attn_bwd", "luna_device_status",
-            "luna_profile_start", "luna_profile_stop", "luna_launch_count")
+            "luna_profile_start", "luna_profile_stop", "luna_launch_count", "luna_attn_fwd_noalloc")
 
 
 def _ptr(t):
@@ -169,6 +170,14 @@ def luna_attn_bwd(ad, pd, table, Q, K, V, dO, lengths, state, dQ, dK, dV, grads:
                               _ptr(lengths), _ptr(state), _ptr(dQ), _ptr(dK), _ptr(dV), ctypes.byref(pg),
                               _ptr(workspace), workspace.numel() * workspace.element_size(), _stream(stream)),
            "luna_attn_bwd")
+
+
+def luna_attn_fwd_noalloc(ad, pd, table, Q, K, V, lengths, O, stream=None) -> None:
+    _check(_lib.luna_attn_fwd_noalloc(ctypes.byref(ad), ctypes.byref(pd), _ptr(table), _ptr(Q), _ptr(K), _ptr(V),
+                                      _ptr(lengths), _ptr(O), _stream(stream)), "luna_attn_fwd_noalloc")
+
+
+NOALLOC_SCRATCH_BYTES = 16 << 20
 
 
 def luna_device_status(workspace: torch.Tensor, stream=None) -> int:
