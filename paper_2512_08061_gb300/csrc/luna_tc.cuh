@@ -7,6 +7,7 @@ namespace luna {
 
 struct TcPlan {
     bool eligible = false;   // shape and dtype handled by the tensor-core kernels
+    int variant = -1;        // kernel instantiation (value width / projections)
     size_t ws_fwd = 0, ws_bwd = 0;
 };
 

@@ -103,6 +103,22 @@ def test_forward(c):
             assert np.all(O[b, :, ln:] == 0)
 
 
+@pytest.mark.parametrize("tiles", ["1", "5", "9"])
+@pytest.mark.parametrize("d,M", [(32, 8), (64, 8), (128, 16)])
+def test_forward_tensor_core_tile_loops(d, M, tiles, monkeypatch):
+    """bf16 forward through the tensor-core kernels with 1, 5 and 9 tiles of
+    128 rows per block: covers the staging ring wrapping around, ragged last
+    tiles, splits with no valid row, and several splits per head."""
+    monkeypatch.setenv("LUNA_TC_TILES_PER_SPLIT", tiles)
+    case = Case(2, 2, 1500, d, M, 8, "bf16", False, seed=41, qkv_scale=1.0 / math.sqrt(d),
+                lengths=[1500, 333])
+    lu = case.luna()
+    O = to_host(case.run_fwd(lu))
+    ref = case.oracle_fwd()
+    assert relerr(O, ref) < TOL["bf16"]
+    assert np.all(O[1, :, 333:] == 0)
+
+
 # --------------------------------------------------------------------------
 # backward
 
