@@ -90,8 +90,11 @@ luna_status make_plan(const luna_attn_desc *ad, const luna_phi_desc *pd, Plan &p
         p.o_Sfin = w.take((size_t)BH * SD * f);
         p.o_zfin = w.take((size_t)BH * D * f);
         p.ws_fwd = w.n;
-        p.o_dSpart = w.take((size_t)BH * p.nsplit_b * SD * f);
-        p.o_dzpart = w.take((size_t)BH * p.nsplit_b * D * f);
+        // per-head partial slots: generic splits, or (tensor-core path) runs of work items, never more
+        // than the forward split count
+        const size_t nslot = (size_t)std::max(p.nsplit, p.nsplit_b);
+        p.o_dSpart = w.take((size_t)BH * nslot * SD * f);
+        p.o_dzpart = w.take((size_t)BH * nslot * D * f);
         p.o_dSfin = w.take((size_t)BH * SD * f);
         p.o_dzfin = w.take((size_t)BH * D * f);
         p.o_gpart = w.take(2 * (size_t)BH * p.nsplit_b * p.gsize * f);

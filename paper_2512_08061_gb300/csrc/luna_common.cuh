@@ -16,6 +16,7 @@ constexpr int kMaxFeat = 128;   // max D = M * L
 constexpr int kMaxL = 16;
 constexpr int kMaxHidden = 128;
 constexpr int kMaxUnits = 512;  // max L * hidden
+constexpr int kEytzinger = 1024; // slots of the breadth-first kink tree (1023 nodes, P <= 512)
 
 __host__ __device__ inline int next_pow2(int x) {
     int p = 1;
@@ -27,6 +28,8 @@ __host__ __device__ inline int64_t align256(int64_t x) { return (x + 255) & ~int
 
 // Layout of the prepared feature-map table (byte offsets from its start).
 //   T      [Ppad]          sorted fp32 kink thresholds of all hidden units (+inf padding)
+//   Te     [1024]          the same thresholds in Eytzinger (breadth-first) order of a
+//                          complete 1023-node search tree, index 0 unused, +inf padding
 //   AB     [nint][L][2]    per merged interval j and channel l: (alpha, beta) / sqrt(M)
 //   W      [M][d], b [M]   projection copy
 //   rank   [P]             position of unit (l,k) in the sorted kink list
@@ -34,7 +37,7 @@ __host__ __device__ inline int64_t align256(int64_t x) { return (x + 255) & ~int
 //   w1, b1, w2 [P], b2 [L] channel-MLP parameter copy (used by the gradient reduction)
 struct TableLayout {
     int M, L, hid, d, D, P, Ppad, nint;
-    int64_t off_T, off_AB, off_W, off_b, off_rank, off_utype, off_w1, off_b1, off_w2, off_b2, bytes;
+    int64_t off_T, off_Te, off_AB, off_W, off_b, off_rank, off_utype, off_w1, off_b1, off_w2, off_b2, bytes;
 };
 
 __host__ __device__ inline TableLayout table_layout(int M, int L, int hid, int d) {
@@ -45,6 +48,7 @@ __host__ __device__ inline TableLayout table_layout(int M, int L, int hid, int d
     t.nint = t.P + 1;
     int64_t o = 256;  // header
     t.off_T = o;     o = align16(o + 4 * (int64_t)t.Ppad);
+    t.off_Te = o;    o = align16(o + 4 * (int64_t)kEytzinger);
     t.off_AB = o;    o = align16(o + 8 * (int64_t)t.nint * L);
     t.off_W = o;     o = align16(o + 4 * (int64_t)M * d);
     t.off_b = o;     o = align16(o + 4 * (int64_t)M);

@@ -117,7 +117,14 @@ __device__ bool last_arrival(int *counter, int expected) {
 __device__ void ordered_sum(const float *part, int nparts, int count, float *out) {
     for (int e = threadIdx.x; e < count; e += blockDim.x) {
         float s = 0.0f;
-        for (int p = 0; p < nparts; ++p) s += __ldcg(part + (size_t)p * count + e);
+        for (int p0 = 0; p0 < nparts; p0 += 8) {  // eight loads in flight, added in order
+            float v[8];
+#pragma unroll
+            for (int k = 0; k < 8; ++k) v[k] = (p0 + k < nparts) ? __ldcg(part + (size_t)(p0 + k) * count + e) : 0.0f;
+#pragma unroll
+            for (int k = 0; k < 8; ++k)
+                if (p0 + k < nparts) s += v[k];
+        }
         out[e] = s;
     }
 }

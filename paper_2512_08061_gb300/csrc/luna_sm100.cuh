@@ -54,14 +54,16 @@ __device__ __forceinline__ uint64_t globaltimer_ns() {
 
 // Waits for the phase with the given parity to complete; gives up after
 // `limit_ns` nanoseconds of wall time (default 1 s) and returns false.
+// mbarrier.try_wait itself suspends the thread in hardware for a bounded
+// time, so polling it back to back does not burn issue slots; the wall clock
+// is only consulted every 1024 polls.
 __device__ __forceinline__ bool mbar_wait(uint64_t *bar, uint32_t parity, uint64_t limit_ns = 1000000000ull) {
     if (mbar_try_wait(bar, parity)) return true;
     const uint64_t t0 = globaltimer_ns();
     while (true) {
-        for (int i = 0; i < 64; ++i)
+        for (int i = 0; i < 1024; ++i)
             if (mbar_try_wait(bar, parity)) return true;
         if (globaltimer_ns() - t0 > limit_ns) return false;
-        __nanosleep(32);
     }
 }
 

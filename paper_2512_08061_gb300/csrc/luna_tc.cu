@@ -1,40 +1,37 @@
 // Tensor-core (tcgen05 / TMEM / TMA) kernels for bf16 I/O on sm_103a.
 //
-// Every kernel works on tiles of 128 rows of one (batch, head) with 288
-// threads: warp 8 is the producer (one elected lane issues the TMA tile loads
-// and the tcgen05.mma instructions and commits them to mbarriers); warps 0..7
-// are workers, two per row (warps w and w+4 own TMEM lanes 32*(w%4)..+31 and
-// split the M projections of those rows between them).
+// Persistent kernels: one block per SM walks a contiguous range of work items
+// (head, chunk of 128-row tiles).  Warp roles in a block of 576 threads:
+//   warps 0..15  workers, four per row: warps w, w+4, w+8, w+12 own TMEM lanes
+//                32*(w%4)..+31 and each evaluates the feature map for a
+//                quarter of the M projections of those rows;
+//   warp 16      TMA: lane 0 streams the X (query / key) tiles, lane 1 the V
+//                tiles, each into its own ring of shared-memory stages;
+//   warp 17      MMA: lane 0 issues every tcgen05.mma and commits it to the
+//                mbarriers that release stages and wake the workers.
 //
-// Per tile, forward key pass (Sec. 4, S_KV and S_K1):
-//   TMA K, V -> smem (128B swizzle)
-//   MMA  U = K [W_hi; W_lo]^T                      (projections, TMEM)
-//   workers: u = U_hi + U_lo + b; interval j of u in the merged kink list;
-//            phi = relu(alpha_j u + beta_j) for the 8 channels -> bf16 tile
-//   MMA  S += phi^T V,  z += phi^T 1               (MN-major A and B, TMEM)
+// Forward key pass per tile (Sec. 4, S_KV and S_K1):
+//   MMA  U = K [W_hi; W_lo]^T                      (projections -> TMEM)
+//   workers: u = U_hi + U_lo + b; interval j of u in the breadth-first kink
+//            tree; phi = relu(alpha_j u + beta_j) for the 8 channels, written
+//            as bf16 hi and lo tiles; z += phi in fp32 registers
+//   MMA  S += [phi_hi | phi_lo]^T V                 (MN-major operands)
 // Forward query pass (Eq. kernel-attn):
-//   TMA Q -> MMA U -> phi tile + fp32 normaliser phi.z
+//   MMA U, workers phi(Q) (bf16) and the fp32 normaliser phi.z,
 //   MMA  num = phi [S_hi; S_lo]^T,  O = num / (phi.z + eps)
-// S is split into bf16 hi + lo parts so that the state enters the product with
-// ~16 significant bits; W likewise.  phi itself is rounded to bf16.
-#include <math.h>
-#include <stdlib.h>
-
-#include "luna_prof.cuh"
-#include "luna_sm100.cuh"
-#include "luna_simt_dev.cuh"
-#include "luna_tc.cuh"
+// S and W enter their products split into bf16 hi + lo parts.
+#include "luna_tc_dev.cuh"
 
 namespace luna {
 namespace {
 using namespace sm100;
 using namespace simt;
+using namespace tcdev;
 
-constexpr int kWorkers = 256;
-constexpr int kThreadsTC = kWorkers + 32;
-constexpr uint32_t kSmemLimit = 227 * 1024;
-constexpr int kPpad = 512;   // merged kink list (L * hidden <= 512, L = 8)
-constexpr int kNint = 513;   // intervals
+constexpr int kWorkerWarps = 16;
+constexpr int kWorkers = kWorkerWarps * 32;
+constexpr int kTmaWarp = 16, kMmaWarp = 17;
+constexpr int kThreadsTC = kWorkers + 64;
 
 template <int DX_, int DV_, int MP_>
 struct Cfg {
@@ -47,142 +44,94 @@ struct Cfg {
     static constexpr int NVB = VC / 64;
     static constexpr int NPB = D / 64;            // 64-feature blocks of a phi tile
     static constexpr int NU = 2 * MP;             // projection columns (hi, lo)
-    static constexpr int PP = MP / 2;             // projections per worker thread
-    static constexpr int NUS = 2;                 // projection stages in TMEM
+    static constexpr int PP = MP / 4;             // projections per worker thread
+    static constexpr bool MERGE = (D == 64);      // phi_hi and phi_lo stacked into one M = 128 operand
     static constexpr uint32_t XT = 128u * DX * 2;
     static constexpr uint32_t VT = 128u * VC * 2;
     static constexpr uint32_t PT = 128u * D * 2;  // one bf16 phi tile
     static constexpr uint32_t WOP = (uint32_t)NU * DX * 2;
-    static constexpr uint32_t ONES = 4096;
-    static constexpr uint32_t TABLE = (kPpad + kNint * 16 + 32) * 4;
+    static constexpr uint32_t TABLE = (kEytzinger + kNint * 16 + 32) * 4;
     static constexpr uint32_t MISC = 1024;
     static constexpr bool SMALL = XT <= 16384 && VT <= 16384;
-    // key pass: phi(K) as bf16 hi + lo tiles
+    // key pass
     static constexpr int NX_K = SMALL ? 3 : 2;
     static constexpr int NV_K = SMALL ? 3 : 1;
     static constexpr int NP_K = SMALL ? 2 : 1;
-    static constexpr uint32_t FIX_K = WOP + ONES + TABLE + MISC + 1024;
+    static constexpr uint32_t ZPART = 4u * D * 4;
+    static constexpr uint32_t SSTAGE = MERGE ? 64u * DV * 4 : 0u;
+    static constexpr uint32_t FIX_K = WOP + TABLE + ZPART + SSTAGE + MISC + 1024;
     static constexpr uint32_t SMEM_K = NX_K * XT + NV_K * VT + NP_K * 2 * PT + FIX_K;
-    static constexpr int TMEM_K_USED = NU * NUS + DV + 16;
-    static constexpr int TMEM_K = TMEM_K_USED <= 32 ? 32 : TMEM_K_USED <= 64 ? 64 : TMEM_K_USED <= 128 ? 128
-                                 : TMEM_K_USED <= 256 ? 256 : 512;
-    // query pass: phi(Q) as one bf16 tile
+    static constexpr int TMEM_K_USED = 2 * NU + 2 * DV;
+    static constexpr int TMEM_K = TMEM_K_USED <= 64 ? 64 : TMEM_K_USED <= 128 ? 128 : TMEM_K_USED <= 256 ? 256 : 512;
+    // query pass
     static constexpr uint32_t SOP = 2u * DV * D * 2;  // [S_hi; S_lo]^T operand
     static constexpr int NP_Q = SMALL ? 2 : 1;
     static constexpr int NX_Q = SMALL ? 4 : 2;
-    static constexpr uint32_t FIX_Q = WOP + SOP + TABLE + D * 4 + 2 * 2 * 128 * 4 + MISC + 1024;
+    static constexpr uint32_t FIX_Q = WOP + SOP + TABLE + D * 4 + 2 * 4 * 128 * 4 + MISC + 1024;
     static constexpr uint32_t SMEM_Q = NX_Q * XT + NP_Q * PT + FIX_Q;
-    static constexpr int NN_Q = (NU * NUS + 4 * DV <= 256) ? 2 : 1;
-    static constexpr int TMEM_Q_USED = NU * NUS + 2 * DV * NN_Q;
+    static constexpr int NN_Q = (2 * NU + 4 * DV <= 256) ? 2 : 1;
+    static constexpr int TMEM_Q_USED = 2 * NU + 2 * DV * NN_Q;
     static constexpr int TMEM_Q = TMEM_Q_USED <= 64 ? 64 : TMEM_Q_USED <= 128 ? 128 : TMEM_Q_USED <= 256 ? 256 : 512;
     static_assert(SMEM_K <= kSmemLimit && SMEM_Q <= kSmemLimit, "shared memory budget");
     static_assert(TMEM_K_USED <= 512 && TMEM_Q_USED <= 512, "tensor memory budget");
+    static_assert(PP == 2 || PP == 4, "projections per worker");
 };
 
-__device__ __forceinline__ uint8_t *align1024(uint8_t *p) {
-    return reinterpret_cast<uint8_t *>((reinterpret_cast<uintptr_t>(p) + 1023) & ~uintptr_t(1023));
-}
-
-__device__ __forceinline__ uint32_t pack_bf16x2(float a, float b) {
-    __nv_bfloat162 v = __floats2bfloat162_rn(a, b);
-    return *reinterpret_cast<uint32_t *>(&v);
-}
-
-__device__ __forceinline__ void split_bf16(float x, __nv_bfloat16 &hi, __nv_bfloat16 &lo) {
-    hi = __float2bfloat16_rn(x);
-    lo = __float2bfloat16_rn(x - __bfloat162float(hi));
-}
-
-__device__ __forceinline__ void report(int *status, int code) {
-    if (status) atomicOr(status, code);
-}
-
-// Bounded wait that turns into a no-op once this thread has seen a timeout, so
-// that every thread still runs the same sequence of block-level barriers and
-// the kernel terminates (its outputs are then undefined and the status word
-// reports LUNA_ERR_DEVICE_TIMEOUT).
-__device__ __forceinline__ void wait_or_fail(uint64_t *bar, uint32_t parity, bool &failed, int *status) {
-    if (failed) return;
-    if (!mbar_wait(bar, parity)) {
-        failed = true;
-        report(status, 1);
-    }
-}
-
-// Loads the kink list, the interval table and the projection bias into smem,
-// and writes the projection operand [W_hi; W_lo] (NU rows x DX, K-major SW128).
-template <class C>
-__device__ void stage_phi_table(const AttnArgs &a, float *sT, float *sAB, float *sbias, uint8_t *Wop, int tid,
-                                int nthreads) {
-    const TableLayout &lay = a.lay;
-    const float *T = reinterpret_cast<const float *>(a.table + lay.off_T);
-    for (int e = tid; e < kPpad; e += nthreads) sT[e] = e < lay.Ppad ? T[e] : INFINITY;
-    const float4 *AB4 = reinterpret_cast<const float4 *>(a.table + lay.off_AB);
-    for (int e = tid; e < lay.nint * 4; e += nthreads) reinterpret_cast<float4 *>(sAB)[e] = AB4[e];
-    const float *b = reinterpret_cast<const float *>(a.table + lay.off_b);
-    for (int e = tid; e < C::MP; e += nthreads) sbias[e] = b[e];
-    const float *W = reinterpret_cast<const float *>(a.table + lay.off_W);
-    for (int e = tid; e < C::NU * C::DX; e += nthreads) {
-        const int n = e / C::DX, c = e % C::DX;
-        const int i = n % C::MP;
-        const float w = (c < a.d) ? W[i * a.d + c] : 0.0f;
-        __nv_bfloat16 hi, lo;
-        split_bf16(w, hi, lo);
-        *reinterpret_cast<__nv_bfloat16 *>(Wop + (c / 64) * (C::NU * 128) + sw128_chunk(n, (c % 64) / 8) + (c % 8) * 2) =
-            (n < C::MP) ? hi : lo;
-    }
-}
-
-// Projection MMA: U[cols] = X tile (128 x DX) * [W_hi; W_lo]^T
-template <class C>
-__device__ __forceinline__ void issue_proj(uint32_t tmem_u, uint32_t xaddr, uint32_t waddr) {
-    constexpr uint32_t idesc = idesc_bf16(128, C::NU, false, false);
-#pragma unroll
-    for (int kb = 0; kb < C::KBX; ++kb)
-#pragma unroll
-        for (int k = 0; k < 4; ++k)
-            mma_bf16_ss(tmem_u, sdesc(xaddr + kb * 16384 + 32 * k, 16, 1024, kSwizzle128),
-                        sdesc(waddr + kb * (C::NU * 128) + 32 * k, 16, 1024, kSwizzle128), idesc, (kb | k) != 0);
-}
-
-// Worker: phi for projections [H*PP, H*PP+PP) of row r from the projection
-// columns in TMEM; writes the bf16 chunks of the phi tile (and, if plo is not
-// null, the bf16 residual phi - bf16(phi) into a second tile), zeros for rows
-// that are not valid; optionally accumulates the fp32 normaliser phi . z.
-template <class C, int H>
-__device__ __forceinline__ void phi_row_half(uint32_t tmem_u_row, const float *sT, const float *sAB,
-                                             const float *sbias, bool valid, int r, uint8_t *phi, uint8_t *plo,
-                                             const float *sz, float &den) {
-    uint32_t hv[C::PP], lv[C::PP];
-    if constexpr (C::PP == 4) {
+// Worker: phi for projections [Q*PP, Q*PP+PP) of row r from the projection
+// columns in TMEM.  The PP interval searches run interleaved over the
+// breadth-first kink tree (count of thresholds below u = final node - 1024).
+// Writes the bf16 chunks of the phi tile (and, if plo is not null, the bf16
+// residual phi - bf16(phi) into a second tile), zeros for rows that are not
+// valid.  Optionally adds phi into zacc (fp32 feature sums) and accumulates the
+// fp32 normaliser phi . z.
+template <class C, int Q>
+__device__ __forceinline__ void phi_row_quarter(uint32_t tmem_u_row, const float *sTe, const float *sAB,
+                                                const float *sbias, bool valid, int r, uint8_t *phi, uint8_t *plo,
+                                                float *zacc, const float *sz, float &den) {
+    constexpr int PP = C::PP;
+    float u[PP];
+    {
         uint32_t x[16];
         tmem_ld16(tmem_u_row, x);
-        tmem_wait_ld();
+        if constexpr (C::MP == 8) {
+            tmem_wait_ld();
 #pragma unroll
-        for (int q = 0; q < 4; ++q) { hv[q] = x[H * 4 + q]; lv[q] = x[8 + H * 4 + q]; }
-    } else {
-        uint32_t x[16], y[16];
-        tmem_ld16(tmem_u_row, x);
-        tmem_ld16(tmem_u_row + 16, y);
-        tmem_wait_ld();
+            for (int q = 0; q < PP; ++q) u[q] = __uint_as_float(x[Q * PP + q]) + __uint_as_float(x[8 + Q * PP + q]);
+        } else {
+            uint32_t y[16];
+            tmem_ld16(tmem_u_row + 16, y);
+            tmem_wait_ld();
 #pragma unroll
-        for (int q = 0; q < 8; ++q) { hv[q] = x[H * 8 + q]; lv[q] = y[H * 8 + q]; }
+            for (int q = 0; q < PP; ++q) u[q] = __uint_as_float(x[Q * PP + q]) + __uint_as_float(y[Q * PP + q]);
+        }
+    }
+    int node[PP];
+#pragma unroll
+    for (int q = 0; q < PP; ++q) {
+        u[q] += sbias[Q * PP + q];
+        node[q] = 1;
     }
 #pragma unroll
-    for (int q = 0; q < C::PP; ++q) {
-        constexpr int base = H * C::PP;
-        const int i = base + q;
+    for (int lvl = 0; lvl < 10; ++lvl)
+#pragma unroll
+        for (int q = 0; q < PP; ++q) node[q] = 2 * node[q] + (sTe[node[q]] < u[q] ? 1 : 0);
+#pragma unroll
+    for (int q = 0; q < PP; ++q) {
+        const int i = Q * PP + q;
         uint4 ph = make_uint4(0u, 0u, 0u, 0u), pl = make_uint4(0u, 0u, 0u, 0u);
         if (valid) {
-            const float u = __uint_as_float(hv[q]) + __uint_as_float(lv[q]) + sbias[i];
-            const int j = interval_of(sT, kPpad, u);
-            const float4 *ab = reinterpret_cast<const float4 *>(sAB) + j * 4;
+            const int j = node[q] - kEytzinger;
+            const float4 *ab = reinterpret_cast<const float4 *>(sAB) + (j << 2);
             float y[8];
 #pragma unroll
             for (int k = 0; k < 4; ++k) {
-                const float4 v = ab[k];
-                y[2 * k] = fmaxf(fmaf(v.x, u, v.y), 0.0f);
-                y[2 * k + 1] = fmaxf(fmaf(v.z, u, v.w), 0.0f);
+                const float4 v = ab[k ^ (j & 3)];
+                y[2 * k] = fmaxf(fmaf(v.x, u[q], v.y), 0.0f);
+                y[2 * k + 1] = fmaxf(fmaf(v.z, u[q], v.w), 0.0f);
+            }
+            if (zacc) {
+#pragma unroll
+                for (int l = 0; l < 8; ++l) zacc[q * 8 + l] += y[l];
             }
             if (sz) {
 #pragma unroll
@@ -204,17 +153,39 @@ __device__ __forceinline__ void phi_row_half(uint32_t tmem_u_row, const float *s
     }
 }
 
-template <int N>
-__device__ __forceinline__ void named_sync(int id) {
-    asm volatile("bar.sync %0, %1;" ::"r"(id), "r"(N) : "memory");
+template <class C>
+__device__ __forceinline__ void phi_row_any(int Q, uint32_t tmem_u_row, const float *sTe, const float *sAB,
+                                            const float *sbias, bool valid, int r, uint8_t *phi, uint8_t *plo,
+                                            float *zacc, const float *sz, float &den) {
+    switch (Q) {
+        case 0: phi_row_quarter<C, 0>(tmem_u_row, sTe, sAB, sbias, valid, r, phi, plo, zacc, sz, den); break;
+        case 1: phi_row_quarter<C, 1>(tmem_u_row, sTe, sAB, sbias, valid, r, phi, plo, zacc, sz, den); break;
+        case 2: phi_row_quarter<C, 2>(tmem_u_row, sTe, sAB, sbias, valid, r, phi, plo, zacc, sz, den); break;
+        default: phi_row_quarter<C, 3>(tmem_u_row, sTe, sAB, sbias, valid, r, phi, plo, zacc, sz, den); break;
+    }
+}
+
+// Projection MMA of tile g into TMEM stage g & 1.
+template <class C>
+__device__ __forceinline__ void issue_proj(uint32_t tmem_u, uint64_t dx, uint64_t dw) {
+    constexpr uint32_t idesc = idesc_bf16(128, C::NU, false, false);
+#pragma unroll
+    for (int kb = 0; kb < C::KBX; ++kb)
+#pragma unroll
+        for (int k = 0; k < 4; ++k)
+            mma_bf16_ss(tmem_u, dadd(dx, kb * 16384 + 32 * k), dadd(dw, kb * (C::NU * 128) + 32 * k), idesc,
+                        (kb | k) != 0);
 }
 
 // ---------------------------------------------------------------------------
-// forward key pass: S_KV = phi(K)^T V and S_K1 = phi(K)^T 1 per (head, split)
+// forward key pass: S_KV = phi(K)^T V and S_K1 = phi(K)^T 1 per (head, chunk)
 //
-// phi(K) enters the contraction as bf16 hi + lo tiles (two MMAs), so that the
-// key statistics carry ~16 significant bits of phi: the backward pass
-// subtracts nearly equal terms built from S and z.
+// phi(K) enters the contraction as bf16 hi + lo tiles so that the key
+// statistics carry ~16 significant bits of phi (the backward pass subtracts
+// nearly equal terms built from S and z); z is summed by the workers in fp32.
+// Each item's statistics go to its partial slot; the last chunk of a head to
+// finish sums the partials in chunk order (warps 0..3 only, so that the
+// pipeline keeps running).
 
 template <class C>
 __global__ void __launch_bounds__(kThreadsTC, 1)
@@ -222,189 +193,248 @@ __global__ void __launch_bounds__(kThreadsTC, 1)
               int *status) {
     extern __shared__ uint8_t smem_raw[];
     uint8_t *sm = align1024(smem_raw);
-    constexpr int NX = C::NX_K, NV = C::NV_K, NP = C::NP_K, NUS = C::NUS;
+    constexpr int NX = C::NX_K, NV = C::NV_K, NP = C::NP_K;
     uint8_t *Xb = sm;
     uint8_t *Vb = Xb + NX * C::XT;
     uint8_t *Pb = Vb + NV * C::VT;  // [NP][hi, lo]
     uint8_t *Wop = Pb + NP * 2 * C::PT;
-    uint8_t *Ones = Wop + C::WOP;
-    float *sT = reinterpret_cast<float *>(Ones + C::ONES);
-    float *sAB = sT + kPpad;
+    float *sTe = reinterpret_cast<float *>(Wop + C::WOP);
+    float *sAB = sTe + kEytzinger;
     float *sbias = sAB + kNint * 16;
-    uint64_t *bars = reinterpret_cast<uint64_t *>(sbias + 32);
+    float *zpart = sbias + 32;         // [4][D]
+    float *sstage = zpart + 4 * C::D;  // [64][DV] (stacked operand only)
+    uint64_t *bars = reinterpret_cast<uint64_t *>(sstage + C::SSTAGE / 4);
     uint64_t *fullx = bars;            // [NX] X tile landed
     uint64_t *xfree = fullx + NX;      // [NX] projection MMA consumed it
     uint64_t *fullv = xfree + NX;      // [NV] V tile landed
     uint64_t *vfree = fullv + NV;      // [NV] contraction consumed it
-    uint64_t *uready = vfree + NV;     // [NUS] projection in TMEM
-    uint64_t *phiready = uready + NUS; // [NP] workers wrote phi (count 256)
+    uint64_t *uready = vfree + NV;     // [2] projection in TMEM
+    uint64_t *phiready = uready + 2;   // [NP] workers wrote phi (count 512)
     uint64_t *pfree = phiready + NP;   // [NP] contraction consumed phi
-    uint64_t *accdone = pfree + NP;    // [1]
-    uint32_t *tslot = reinterpret_cast<uint32_t *>(accdone + 1);
+    uint64_t *accdone = pfree + NP;    // [2] item statistics complete
+    uint64_t *accfree = accdone + 2;   // [2] item statistics read (count 128)
+    uint32_t *tslot = reinterpret_cast<uint32_t *>(accfree + 2);
+    int *slast = reinterpret_cast<int *>(tslot + 1);
 
     const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
-    const int bh = blockIdx.y, split = blockIdx.x;
-    const int len = head_length(a.lengths, bh / a.H, a.n);
-    const int r0 = split * a.rows_per_split;
-    const int r1 = min(len, r0 + a.rows_per_split);
-    const int ntiles = r1 > r0 ? (r1 - r0 + 127) / 128 : 0;
+    const Items it(a);
 
     if (tid == 0) {
         for (int i = 0; i < NX; ++i) { mbar_init(fullx + i, 1); mbar_init(xfree + i, 1); }
         for (int i = 0; i < NV; ++i) { mbar_init(fullv + i, 1); mbar_init(vfree + i, 1); }
-        for (int i = 0; i < NUS; ++i) mbar_init(uready + i, 1);
+        for (int i = 0; i < 2; ++i) mbar_init(uready + i, 1);
         for (int i = 0; i < NP; ++i) { mbar_init(phiready + i, kWorkers); mbar_init(pfree + i, 1); }
-        mbar_init(accdone, 1);
+        for (int i = 0; i < 2; ++i) { mbar_init(accdone + i, 1); mbar_init(accfree + i, 128); }
         fence_mbar_init();
     }
     if (warp == 0) { tmem_alloc(tslot, C::TMEM_K); tmem_relinquish(); }
-    stage_phi_table<C>(a, sT, sAB, sbias, Wop, tid, kThreadsTC);
-    for (int e = tid; e < (int)C::ONES / 4; e += kThreadsTC)
-        reinterpret_cast<uint32_t *>(Ones)[e] = 0x3F803F80u;  // bf16 1.0 pairs
+    stage_phi_table<C>(a, sTe, sAB, sbias, Wop);
     fence_proxy_async_smem();
     tc_fence_before();
     __syncthreads();
     tc_fence_after();
     const uint32_t tbase = *tslot;
-    const uint32_t tmem_s = tbase + C::NU * NUS;  // S accumulator (DV cols)
-    const uint32_t tmem_z = tmem_s + C::DV;       // z accumulator (16 cols)
+    const uint32_t tmem_acc = tbase + 2 * C::NU;  // [2] x DV cols
 
-    if (warp == 8) {
-        if (lane == 0 && ntiles > 0) {
-            const uint32_t xa = smem_u32(Xb), va = smem_u32(Vb), pa = smem_u32(Pb), wa = smem_u32(Wop),
-                           oa = smem_u32(Ones);
-            auto load_x = [&](int t) {
-                const int x = t % NX;
-                mbar_arrive_expect_tx(fullx + x, C::XT);
-                for (int kb = 0; kb < C::KBX; ++kb)
-                    tma_load_3d(Xb + x * C::XT + kb * 16384, &mapK, kb * 64, r0 + t * 128, bh, fullx + x);
-            };
-            auto load_v = [&](int t) {
-                const int v = t % NV;
-                mbar_arrive_expect_tx(fullv + v, C::VT);
-                for (int vb = 0; vb < C::NVB; ++vb)
-                    tma_load_3d(Vb + v * C::VT + vb * 16384, &mapV, vb * 64, r0 + t * 128, bh, fullv + v);
-            };
-            auto proj = [&](int t) {
-                const int x = t % NX;
-                issue_proj<C>(tbase + (t % NUS) * C::NU, xa + x * C::XT, wa);
-                mma_commit(uready + (t % NUS));
+    if (warp == kTmaWarp) {
+        if (lane < 2) {
+            const int T = block_tiles(a, it);
+            TileCursor cur;
+            cur.start(a, it);
+            bool failed = false;
+            for (int g = 0; g < T && !failed; ++g, cur.next(a, it)) {
+                if (lane == 0) {
+                    const int x = g % NX;
+                    if (g >= NX) wait_or_fail(xfree + x, ((g - NX) / NX) & 1, failed, status);
+                    mbar_arrive_expect_tx(fullx + x, C::XT);
+                    for (int kb = 0; kb < C::KBX; ++kb)
+                        tma_load_3d(Xb + x * C::XT + kb * 16384, &mapK, kb * 64, cur.row0(), cur.g.bh, fullx + x);
+                } else {
+                    const int v = g % NV;
+                    if (g >= NV) wait_or_fail(vfree + v, ((g - NV) / NV) & 1, failed, status);
+                    mbar_arrive_expect_tx(fullv + v, C::VT);
+                    for (int vb = 0; vb < C::NVB; ++vb)
+                        tma_load_3d(Vb + v * C::VT + vb * 16384, &mapV, vb * 64, cur.row0(), cur.g.bh, fullv + v);
+                }
+            }
+        }
+    } else if (warp == kMmaWarp) {
+        if (lane == 0) {
+            const int T = block_tiles(a, it);
+            const uint64_t dx0 = sdesc(smem_u32(Xb), 16, 1024, kSwizzle128);
+            const uint64_t dw0 = sdesc(smem_u32(Wop), 16, 1024, kSwizzle128);
+            const uint64_t dp0 = sdesc(smem_u32(Pb), 16384, 1024, kSwizzle128);
+            const uint64_t dv0 = sdesc(smem_u32(Vb), 16384, 1024, kSwizzle128);
+            bool failed = false;
+            auto proj = [&](int g) {
+                const int x = g % NX;
+                wait_or_fail(fullx + x, (g / NX) & 1, failed, status);
+                tc_fence_after();
+                issue_proj<C>(tbase + (g & 1) * C::NU, dadd(dx0, x * C::XT), dw0);
+                mma_commit(uready + (g & 1));
                 mma_commit(xfree + x);
             };
-            bool failed = false;
-            for (int t = 0; t < NX && t < ntiles; ++t) load_x(t);
-            for (int t = 0; t < NV && t < ntiles; ++t) load_v(t);
-            wait_or_fail(fullx, 0, failed, status);
-            tc_fence_after();
-            proj(0);
-            for (int t = 0; t < ntiles && !failed; ++t) {
-                const int p = t % NP, v = t % NV;
-                if (t + 1 < ntiles) {
-                    wait_or_fail(fullx + (t + 1) % NX, ((t + 1) / NX) & 1, failed, status);
-                    tc_fence_after();
-                    proj(t + 1);
-                }
-                if (t + NX < ntiles) {
-                    wait_or_fail(xfree + t % NX, (t / NX) & 1, failed, status);
-                    load_x(t + NX);
-                }
-                wait_or_fail(phiready + p, (t / NP) & 1, failed, status);
-                wait_or_fail(fullv + v, (t / NV) & 1, failed, status);
-                tc_fence_after();
-                const uint32_t ph = pa + p * 2 * C::PT, pl = ph + C::PT, vt = va + v * C::VT;
-                constexpr uint32_t idS = idesc_bf16(C::D, C::DV, true, true);
-                constexpr uint32_t idZ = idesc_bf16(C::D, 16, true, false);
+            if (T > 0) proj(0);
+            if (T > 1) proj(1);
+            // runs: maximal stretches of this block's items that share a head; S accumulates over a run
+            int g = 0, ne = 0;
+            for (int i0 = it.begin; i0 < it.end && !failed;) {
+                const int bh = i0 / it.nchunk;
+                const int i1 = min(it.end, (bh + 1) * it.nchunk);
+                int run_tiles = 0;
+                for (int i = i0; i < i1; ++i) run_tiles += item_range(a, it, i).ntiles;
+                if (run_tiles > 0) {
+                    const int b = ne & 1;
+                    if (ne >= 2) wait_or_fail(accfree + b, ((ne - 2) >> 1) & 1, failed, status);
+                    const uint32_t tmem_s = tmem_acc + b * C::DV;
+                    for (int t = 0; t < run_tiles && !failed; ++t, ++g) {
+                        const int p = g % NP, v = g % NV;
+                        wait_or_fail(phiready + p, (g / NP) & 1, failed, status);
+                        wait_or_fail(fullv + v, (g / NV) & 1, failed, status);
+                        tc_fence_after();
+                        const uint64_t ph = dadd(dp0, p * 2 * C::PT), bv = dadd(dv0, v * C::VT);
+                        constexpr uint32_t idS = idesc_bf16(128, C::DV, true, true);
 #pragma unroll
-                for (int k = 0; k < 8; ++k) {
-                    const uint32_t acc = (t > 0 || k > 0) ? 1u : 0u;
-                    const uint64_t bv = sdesc(vt + 2048 * k, 16384, 1024, kSwizzle128);
-                    const uint64_t bo = sdesc(oa + (k / 4) * 2048 + 32 * (k % 4), 16, 1024, kSwizzle128);
-                    const uint64_t ah = sdesc(ph + 2048 * k, 16384, 1024, kSwizzle128);
-                    const uint64_t al = sdesc(pl + 2048 * k, 16384, 1024, kSwizzle128);
-                    mma_bf16_ss(tmem_s, ah, bv, idS, acc);
-                    mma_bf16_ss(tmem_s, al, bv, idS, 1u);
-                    mma_bf16_ss(tmem_z, ah, bo, idZ, acc);
-                    mma_bf16_ss(tmem_z, al, bo, idZ, 1u);
+                        for (int k = 0; k < 8; ++k) {
+                            const uint32_t acc = (t > 0 || k > 0) ? 1u : 0u;
+                            // stacked operand: rows 0..63 of A are phi_hi, rows 64..127 phi_lo (+16 KB)
+                            mma_bf16_ss(tmem_s, dadd(ph, 2048 * k), dadd(bv, 2048 * k), idS, acc);
+                            if constexpr (!C::MERGE)
+                                mma_bf16_ss(tmem_s, dadd(ph, C::PT + 2048 * k), dadd(bv, 2048 * k), idS, 1u);
+                        }
+                        mma_commit(pfree + p);
+                        mma_commit(vfree + v);
+                        if (t == run_tiles - 1) mma_commit(accdone + b);
+                        if (g + 2 < T) proj(g + 2);
+                    }
+                    ++ne;
                 }
-                mma_commit(pfree + p);
-                mma_commit(vfree + v);
-                if (t + NV < ntiles) {
-                    wait_or_fail(vfree + v, (t / NV) & 1, failed, status);
-                    load_v(t + NV);
-                }
+                i0 = i1;
             }
-            if (!failed) mma_commit(accdone);
-            else mbar_arrive(accdone);
         }
     } else {
-        const int h = warp >> 2, r = ((warp & 3) << 5) | lane;
+        const int Q = warp >> 2, r = ((warp & 3) << 5) | lane;
         const uint32_t lrow = (uint32_t)((warp & 3) << 5) << 16;
+        float zacc[C::PP * 8];
+#pragma unroll
+        for (int k = 0; k < C::PP * 8; ++k) zacc[k] = 0.0f;
         float dummy = 0.0f;
         bool failed = false;
-        for (int t = 0; t < ntiles; ++t) {
-            const int p = t % NP, v = t % NV;
-            const int nvalid = min(128, r1 - (r0 + t * 128));
-            wait_or_fail(uready + t % NUS, (t / NUS) & 1, failed, status);
-            if (t >= NP) wait_or_fail(pfree + p, ((t - NP) / NP) & 1, failed, status);
-            tc_fence_after();
-            uint8_t *ph = Pb + p * 2 * C::PT, *pl = ph + C::PT;
-            const bool valid = r < nvalid;
-            const uint32_t ucol = tbase + lrow + (t % NUS) * C::NU;
-            if (h == 0) phi_row_half<C, 0>(ucol, sT, sAB, sbias, valid, r, ph, pl, nullptr, dummy);
-            else phi_row_half<C, 1>(ucol, sT, sAB, sbias, valid, r, ph, pl, nullptr, dummy);
-            if (!valid && h == 0) {  // padded rows: clear V so that no garbage enters S
-                wait_or_fail(fullv + v, (t / NV) & 1, failed, status);
-                uint8_t *vrow = Vb + v * C::VT;
+        int g = 0, ne = 0;
+        for (int i0 = it.begin; i0 < it.end;) {
+            const int bh = i0 / it.nchunk;
+            const int i1 = min(it.end, (bh + 1) * it.nchunk);
+            int run_tiles = 0;
+            for (int item = i0; item < i1; ++item) {
+                const ItemRange ir = item_range(a, it, item);
+                run_tiles += ir.ntiles;
+                for (int t = 0; t < ir.ntiles; ++t, ++g) {
+                    const int p = g % NP, v = g % NV;
+                    const int nvalid = min(128, ir.r1 - (ir.r0 + t * 128));
+                    wait_or_fail(uready + (g & 1), (g >> 1) & 1, failed, status);
+                    if (g >= NP) wait_or_fail(pfree + p, ((g - NP) / NP) & 1, failed, status);
+                    tc_fence_after();
+                    uint8_t *ph = Pb + p * 2 * C::PT, *pl = ph + C::PT;
+                    const bool valid = r < nvalid;
+                    phi_row_any<C>(Q, tbase + lrow + (g & 1) * C::NU, sTe, sAB, sbias, valid, r, ph, pl, zacc,
+                                   nullptr, dummy);
+                    if (!valid && Q == 0) {  // padded rows: clear V so that no garbage enters S
+                        wait_or_fail(fullv + v, (g / NV) & 1, failed, status);
+                        uint8_t *vrow = Vb + v * C::VT;
 #pragma unroll
-                for (int vb = 0; vb < C::NVB; ++vb)
+                        for (int vb = 0; vb < C::NVB; ++vb)
 #pragma unroll
-                    for (int c = 0; c < 8; ++c)
-                        *reinterpret_cast<uint4 *>(vrow + vb * 16384 + sw128_chunk(r, c)) = make_uint4(0, 0, 0, 0);
+                            for (int c = 0; c < 8; ++c)
+                                *reinterpret_cast<uint4 *>(vrow + vb * 16384 + sw128_chunk(r, c)) =
+                                    make_uint4(0, 0, 0, 0);
+                    }
+                    fence_proxy_async_smem();
+                    tc_fence_before();
+                    mbar_arrive(phiready + p);
+                }
             }
-            fence_proxy_async_smem();
-            tc_fence_before();
-            mbar_arrive(phiready + p);
-        }
-    }
-    // epilogue: partial S, z of this split -> workspace; the last split reduces
-    const size_t slot = (size_t)bh * a.nsplit + split;
-    float *Sp = a.S_part + slot * C::D * C::DV;
-    float *zp = a.z_part + slot * C::D;
-    if (warp < 4) {
-        bool failed = false;
-        if (ntiles > 0) wait_or_fail(accdone, 0, failed, status);
-        const bool ok = !failed && ntiles > 0;
-        tc_fence_after();
-        // accumulator row f: M = 128 -> TMEM lane f; M = 64 -> lane 32*(f/16) + f%16
-        const int f = (C::D == 128) ? ((warp << 5) | lane) : ((warp << 4) | lane);
-        const bool holds = (C::D == 128) || lane < 16;
-        const uint32_t lrow = (uint32_t)(warp << 5) << 16;
+            // z of this run: sum the 128 rows of each warp group, then over the four row groups
 #pragma unroll
-        for (int c0 = 0; c0 < C::DV; c0 += 16) {
-            uint32_t x[16];
-            tmem_ld16(lrow + tmem_s + c0, x);
-            tmem_wait_ld();
-            if (holds) {
+            for (int k = 0; k < C::PP * 8; ++k) {
+                float v = zacc[k];
 #pragma unroll
-                for (int c = 0; c < 16; c += 4)
-                    *reinterpret_cast<float4 *>(Sp + f * C::DV + c0 + c) =
-                        ok ? make_float4(__uint_as_float(x[c]), __uint_as_float(x[c + 1]), __uint_as_float(x[c + 2]),
-                                         __uint_as_float(x[c + 3]))
-                           : make_float4(0.f, 0.f, 0.f, 0.f);
+                for (int o = 16; o > 0; o >>= 1) v += __shfl_xor_sync(0xffffffffu, v, o);
+                if (lane == 0) zpart[(warp & 3) * C::D + Q * C::PP * 8 + k] = v;
+                zacc[k] = 0.0f;
             }
+            named_sync<kWorkers>(1);
+            if (warp < 4) {
+                // run epilogue: statistics of this block's part of head bh -> its partial slot
+                const int c_first = owner_block((long long)bh * it.nchunk, it.total, gridDim.x);
+                const int c_last = owner_block((long long)(bh + 1) * it.nchunk - 1, it.total, gridDim.x);
+                const int nruns = c_last - c_first + 1;
+                const size_t slot = (size_t)bh * it.nchunk + (blockIdx.x - c_first);
+                float *Sp = a.S_part + slot * C::D * C::DV;
+                float *zp = a.z_part + slot * C::D;
+                const int row = (warp << 5) | lane;
+                const uint32_t lrow0 = (uint32_t)(warp << 5) << 16;
+                const bool have = run_tiles > 0;
+                const int b = ne & 1;
+                if (have) wait_or_fail(accdone + b, (ne >> 1) & 1, failed, status);
+                tc_fence_after();
+                const uint32_t tmem_s = tmem_acc + b * C::DV;
+                // accumulator rows: feature f, and (stacked operand) the lo part of feature f at row 64 + f
+                const int f = C::MERGE ? (row & 63) : row;
+                if (C::MERGE && row >= 64) {
+#pragma unroll
+                    for (int c0 = 0; c0 < C::DV; c0 += 16) {
+                        uint32_t x[16];
+                        if (have) { tmem_ld16(lrow0 + tmem_s + c0, x); tmem_wait_ld(); }
+#pragma unroll
+                        for (int c = 0; c < 16; ++c) sstage[f * C::DV + c0 + c] = have ? __uint_as_float(x[c]) : 0.0f;
+                    }
+                }
+                if constexpr (C::MERGE) named_sync<128>(2);
+                if (!C::MERGE || row < 64) {
+#pragma unroll
+                    for (int c0 = 0; c0 < C::DV; c0 += 16) {
+                        uint32_t x[16];
+                        if (have) { tmem_ld16(lrow0 + tmem_s + c0, x); tmem_wait_ld(); }
+#pragma unroll
+                        for (int c = 0; c < 16; c += 4) {
+                            float4 o;
+                            o.x = have ? __uint_as_float(x[c]) : 0.0f;
+                            o.y = have ? __uint_as_float(x[c + 1]) : 0.0f;
+                            o.z = have ? __uint_as_float(x[c + 2]) : 0.0f;
+                            o.w = have ? __uint_as_float(x[c + 3]) : 0.0f;
+                            if (C::MERGE) {
+                                o.x += sstage[f * C::DV + c0 + c];
+                                o.y += sstage[f * C::DV + c0 + c + 1];
+                                o.z += sstage[f * C::DV + c0 + c + 2];
+                                o.w += sstage[f * C::DV + c0 + c + 3];
+                            }
+                            *reinterpret_cast<float4 *>(Sp + f * C::DV + c0 + c) = o;
+                        }
+                    }
+                    zp[f] = zpart[f] + zpart[C::D + f] + zpart[2 * C::D + f] + zpart[3 * C::D + f];
+                }
+                tc_fence_before();
+                if (have) mbar_arrive(accfree + b);
+                // the last block of this head to finish sums the partials in block order
+                __threadfence();
+                named_sync<128>(2);
+                if (tid == 0) *slast = (atomicAdd(a.counters + bh, 1) == nruns - 1) ? 1 : 0;
+                named_sync<128>(2);
+                if (*slast) {
+                    __threadfence();
+                    ordered_sum4(a.S_part + (size_t)bh * it.nchunk * C::D * C::DV, nruns, C::D * C::DV,
+                                 a.S_fin + (size_t)bh * C::D * C::DV, tid, 128);
+                    ordered_sum4(a.z_part + (size_t)bh * it.nchunk * C::D, nruns, C::D, a.z_fin + (size_t)bh * C::D,
+                                 tid, 128);
+                    if (tid == 0) a.counters[bh] = 0;
+                }
+                named_sync<128>(2);
+            }
+            if (run_tiles > 0) ++ne;
+            i0 = i1;
         }
-        uint32_t x[16];
-        tmem_ld16(lrow + tmem_z, x);
-        tmem_wait_ld();
-        if (holds) zp[f] = ok ? __uint_as_float(x[0]) : 0.0f;
     }
     tc_fence_before();
-    if (last_arrival(a.counters + bh, a.nsplit)) {
-        ordered_sum(a.S_part + (size_t)bh * a.nsplit * C::D * C::DV, a.nsplit, C::D * C::DV,
-                    a.S_fin + (size_t)bh * C::D * C::DV);
-        ordered_sum(a.z_part + (size_t)bh * a.nsplit * C::D, a.nsplit, C::D, a.z_fin + (size_t)bh * C::D);
-        if (tid == 0) a.counters[bh] = 0;
-    }
     __syncthreads();
     if (warp == 0) tmem_dealloc(tbase, C::TMEM_K);
 }
@@ -417,161 +447,188 @@ __global__ void __launch_bounds__(kThreadsTC, 1)
     k_tc_query(const __grid_constant__ CUtensorMap mapQ, AttnArgs a, int *status) {
     extern __shared__ uint8_t smem_raw[];
     uint8_t *sm = align1024(smem_raw);
-    constexpr int NX = C::NX_Q, NP = C::NP_Q, NN = C::NN_Q, NUS = C::NUS;
+    constexpr int NX = C::NX_Q, NP = C::NP_Q, NN = C::NN_Q;
     uint8_t *Xb = sm;
     uint8_t *Pb = Xb + NX * C::XT;
     uint8_t *Wop = Pb + NP * C::PT;
     uint8_t *Sop = Wop + C::WOP;
-    float *sT = reinterpret_cast<float *>(Sop + C::SOP);
-    float *sAB = sT + kPpad;
+    float *sTe = reinterpret_cast<float *>(Sop + C::SOP);
+    float *sAB = sTe + kEytzinger;
     float *sbias = sAB + kNint * 16;
     float *sz = sbias + 32;
-    float *sden = sz + C::D;  // [2 tiles][2 halves][128 rows]
-    uint64_t *bars = reinterpret_cast<uint64_t *>(sden + 512);
+    float *sden = sz + C::D;  // [2 tiles][4 quarters][128 rows]
+    uint64_t *bars = reinterpret_cast<uint64_t *>(sden + 1024);
     uint64_t *fullx = bars;               // [NX]
     uint64_t *xfree = fullx + NX;         // [NX]
-    uint64_t *uready = xfree + NX;        // [NUS]
-    uint64_t *phiready = uready + NUS;    // [NP] count 256
+    uint64_t *uready = xfree + NX;        // [2]
+    uint64_t *phiready = uready + 2;      // [NP] count 512
     uint64_t *pfree = phiready + NP;      // [NP]
     uint64_t *numready = pfree + NP;      // [NN]
-    uint64_t *numfree = numready + NN;    // [NN] count 256
+    uint64_t *numfree = numready + NN;    // [NN] count 512
     uint32_t *tslot = reinterpret_cast<uint32_t *>(numfree + NN);
 
     const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
-    const int bh = blockIdx.y, split = blockIdx.x;
-    const int len = head_length(a.lengths, bh / a.H, a.n);
-    const int r0 = split * a.rows_per_split;
-    const int rend = min(a.n, r0 + a.rows_per_split);
-    const int r1 = min(len, rend);
-    const int ntiles = r1 > r0 ? (r1 - r0 + 127) / 128 : 0;
-    __nv_bfloat16 *O = static_cast<__nv_bfloat16 *>(a.O) + (size_t)bh * a.n * C::DV;
+    const Items it(a);
 
     if (tid == 0) {
         for (int i = 0; i < NX; ++i) { mbar_init(fullx + i, 1); mbar_init(xfree + i, 1); }
-        for (int i = 0; i < NUS; ++i) mbar_init(uready + i, 1);
+        for (int i = 0; i < 2; ++i) mbar_init(uready + i, 1);
         for (int i = 0; i < NP; ++i) { mbar_init(phiready + i, kWorkers); mbar_init(pfree + i, 1); }
         for (int i = 0; i < NN; ++i) { mbar_init(numready + i, 1); mbar_init(numfree + i, kWorkers); }
         fence_mbar_init();
     }
     if (warp == 0) { tmem_alloc(tslot, C::TMEM_Q); tmem_relinquish(); }
-    stage_phi_table<C>(a, sT, sAB, sbias, Wop, tid, kThreadsTC);
-    const float *Sg = a.S_fin + (size_t)bh * C::D * C::DV;
-    for (int e = tid; e < 2 * C::DV * C::D; e += kThreadsTC) {
-        const int n = e / C::D, f = e % C::D;  // operand row n: output column n % DV, hi (n < DV) or lo part
-        __nv_bfloat16 hi, lo;
-        split_bf16(Sg[f * C::DV + (n % C::DV)], hi, lo);
-        *reinterpret_cast<__nv_bfloat16 *>(Sop + (f / 64) * (2 * C::DV * 128) + sw128_chunk(n, (f % 64) / 8) +
-                                           (f % 8) * 2) = (n < C::DV) ? hi : lo;
+    stage_phi_table<C>(a, sTe, sAB, sbias, Wop);
+    // padded rows of every item of this block produce zeros
+    for (int item = it.begin; item < it.end; ++item) {
+        const ItemRange ir = item_range(a, it, item);
+        __nv_bfloat16 *O = static_cast<__nv_bfloat16 *>(a.O) + (size_t)ir.bh * a.n * C::DV;
+        const int z0 = max(ir.r0, ir.r1);
+        for (int e = tid; e < (ir.rend - z0) * C::DV / 8; e += kThreadsTC)
+            reinterpret_cast<uint4 *>(O + (size_t)z0 * C::DV)[e] = make_uint4(0, 0, 0, 0);
     }
-    for (int e = tid; e < C::D; e += kThreadsTC) sz[e] = a.z_fin[(size_t)bh * C::D + e];
-    // padded rows of this range produce zeros
-    for (int e = tid; e < (rend - max(r0, len)) * C::DV / 8; e += kThreadsTC)
-        reinterpret_cast<uint4 *>(O + (size_t)max(r0, len) * C::DV)[e] = make_uint4(0, 0, 0, 0);
     fence_proxy_async_smem();
     tc_fence_before();
     __syncthreads();
     tc_fence_after();
     const uint32_t tbase = *tslot;
-    const uint32_t tmem_num = tbase + C::NU * NUS;
+    const uint32_t tmem_num = tbase + 2 * C::NU;
 
-    if (warp == 8) {
-        if (lane == 0 && ntiles > 0) {
-            const uint32_t xa = smem_u32(Xb), pa = smem_u32(Pb), wa = smem_u32(Wop), sa = smem_u32(Sop);
-            auto load_x = [&](int t) {
-                const int x = t % NX;
+    if (warp == kTmaWarp) {
+        if (lane == 0) {
+            const int T = block_tiles(a, it);
+            TileCursor cur;
+            cur.start(a, it);
+            bool failed = false;
+            for (int g = 0; g < T && !failed; ++g, cur.next(a, it)) {
+                const int x = g % NX;
+                if (g >= NX) wait_or_fail(xfree + x, ((g - NX) / NX) & 1, failed, status);
                 mbar_arrive_expect_tx(fullx + x, C::XT);
                 for (int kb = 0; kb < C::KBX; ++kb)
-                    tma_load_3d(Xb + x * C::XT + kb * 16384, &mapQ, kb * 64, r0 + t * 128, bh, fullx + x);
-            };
-            auto proj = [&](int t) {
-                const int x = t % NX;
-                issue_proj<C>(tbase + (t % NUS) * C::NU, xa + x * C::XT, wa);
-                mma_commit(uready + (t % NUS));
+                    tma_load_3d(Xb + x * C::XT + kb * 16384, &mapQ, kb * 64, cur.row0(), cur.g.bh, fullx + x);
+            }
+        }
+    } else if (warp == kMmaWarp) {
+        if (lane == 0) {
+            const int T = block_tiles(a, it);
+            const uint64_t dx0 = sdesc(smem_u32(Xb), 16, 1024, kSwizzle128);
+            const uint64_t dw0 = sdesc(smem_u32(Wop), 16, 1024, kSwizzle128);
+            const uint64_t dp0 = sdesc(smem_u32(Pb), 16, 1024, kSwizzle128);
+            const uint64_t ds0 = sdesc(smem_u32(Sop), 16, 1024, kSwizzle128);
+            bool failed = false;
+            auto proj = [&](int g) {
+                const int x = g % NX;
+                wait_or_fail(fullx + x, (g / NX) & 1, failed, status);
+                tc_fence_after();
+                issue_proj<C>(tbase + (g & 1) * C::NU, dadd(dx0, x * C::XT), dw0);
+                mma_commit(uready + (g & 1));
                 mma_commit(xfree + x);
             };
-            bool failed = false;
-            for (int t = 0; t < NX && t < ntiles; ++t) load_x(t);
-            wait_or_fail(fullx, 0, failed, status);
-            tc_fence_after();
-            proj(0);
-            for (int t = 0; t < ntiles && !failed; ++t) {
-                const int p = t % NP, q = t % NN;
-                if (t + 1 < ntiles) {
-                    wait_or_fail(fullx + (t + 1) % NX, ((t + 1) / NX) & 1, failed, status);
-                    tc_fence_after();
-                    proj(t + 1);
-                }
-                if (t + NX < ntiles) {
-                    wait_or_fail(xfree + t % NX, (t / NX) & 1, failed, status);
-                    load_x(t + NX);
-                }
-                wait_or_fail(phiready + p, (t / NP) & 1, failed, status);
-                if (t >= NN) wait_or_fail(numfree + q, ((t - NN) / NN) & 1, failed, status);
+            if (T > 0) proj(0);
+            if (T > 1) proj(1);
+            for (int g = 0; g < T && !failed; ++g) {
+                const int p = g % NP, q = g % NN;
+                wait_or_fail(phiready + p, (g / NP) & 1, failed, status);
+                if (g >= NN) wait_or_fail(numfree + q, ((g - NN) / NN) & 1, failed, status);
                 tc_fence_after();
                 constexpr uint32_t idN = idesc_bf16(128, 2 * C::DV, false, false);
-                const uint32_t pt = pa + p * C::PT;
+                const uint64_t dp = dadd(dp0, p * C::PT);
 #pragma unroll
                 for (int kb = 0; kb < C::NPB; ++kb)
 #pragma unroll
                     for (int k = 0; k < 4; ++k)
-                        mma_bf16_ss(tmem_num + q * 2 * C::DV, sdesc(pt + kb * 16384 + 32 * k, 16, 1024, kSwizzle128),
-                                    sdesc(sa + kb * (2 * C::DV * 128) + 32 * k, 16, 1024, kSwizzle128), idN,
-                                    (kb | k) != 0);
+                        mma_bf16_ss(tmem_num + q * 2 * C::DV, dadd(dp, kb * 16384 + 32 * k),
+                                    dadd(ds0, kb * (2 * C::DV * 128) + 32 * k), idN, (kb | k) != 0);
                 mma_commit(numready + q);
                 mma_commit(pfree + p);
+                if (g + 2 < T) proj(g + 2);
             }
         }
     } else {
-        const int h = warp >> 2, r = ((warp & 3) << 5) | lane;
+        const int Q = warp >> 2, r = ((warp & 3) << 5) | lane;
         const uint32_t lrow = (uint32_t)((warp & 3) << 5) << 16;
         bool failed = false;
-        for (int t = 0; t < ntiles; ++t) {
-            const int p = t % NP, q = t % NN;
-            const int row0 = r0 + t * 128;
-            const int nvalid = min(128, r1 - row0);
-            wait_or_fail(uready + t % NUS, (t / NUS) & 1, failed, status);
-            if (t >= NP) wait_or_fail(pfree + p, ((t - NP) / NP) & 1, failed, status);
-            tc_fence_after();
-            uint8_t *pt = Pb + p * C::PT;
-            const bool valid = r < nvalid;
-            float den = 0.0f;
-            const uint32_t ucol = tbase + lrow + (t % NUS) * C::NU;
-            if (h == 0) phi_row_half<C, 0>(ucol, sT, sAB, sbias, valid, r, pt, nullptr, sz, den);
-            else phi_row_half<C, 1>(ucol, sT, sAB, sbias, valid, r, pt, nullptr, sz, den);
-            float *dslot = sden + (t & 1) * 256;
-            dslot[h * 128 + r] = den;
-            fence_proxy_async_smem();
-            tc_fence_before();
-            mbar_arrive(phiready + p);
-            named_sync<kWorkers>(1);  // both halves of every row have written their part of the normaliser
-            const float dsum = dslot[r] + dslot[128 + r] + a.eps;
-            wait_or_fail(numready + q, (t / NN) & 1, failed, status);
-            tc_fence_after();
-            // this thread writes output columns [h*DV/2, (h+1)*DV/2) of row r
-            constexpr int HC = C::DV / 2;
-            uint4 outv[HC / 8];
-#pragma unroll
-            for (int c0 = 0; c0 < HC; c0 += 16) {
-                uint32_t xh[16], xl[16];
-                const uint32_t col = tmem_num + q * 2 * C::DV + h * HC + c0;
-                tmem_ld16(lrow + col, xh);
-                tmem_ld16(lrow + col + C::DV, xl);
-                tmem_wait_ld();
-                float o[16];
-#pragma unroll
-                for (int c = 0; c < 16; ++c)
-                    o[c] = (dsum != 0.0f) ? (__uint_as_float(xh[c]) + __uint_as_float(xl[c])) / dsum : 0.0f;
-#pragma unroll
-                for (int c = 0; c < 16; c += 8)
-                    outv[(c0 + c) / 8] = make_uint4(pack_bf16x2(o[c], o[c + 1]), pack_bf16x2(o[c + 2], o[c + 3]),
-                                                    pack_bf16x2(o[c + 4], o[c + 5]), pack_bf16x2(o[c + 6], o[c + 7]));
+        int g = 0, cur_bh = -1;
+        for (int item = it.begin; item < it.end; ++item) {
+            const ItemRange ir = item_range(a, it, item);
+            if (ir.ntiles == 0) continue;
+            if (ir.bh != cur_bh) {
+                // operand [S_hi; S_lo]^T and z of this head.  Safe to overwrite: every worker has passed
+                // the previous tile's normaliser barrier and seen its contraction complete.
+                named_sync<kWorkers>(1);
+                const float *Sg = a.S_fin + (size_t)ir.bh * C::D * C::DV;
+                for (int e = tid; e < 2 * C::DV * C::D; e += kWorkers) {
+                    const int n = e / C::D, f = e % C::D;
+                    __nv_bfloat16 hi, lo;
+                    split_bf16(Sg[f * C::DV + (n % C::DV)], hi, lo);
+                    *reinterpret_cast<__nv_bfloat16 *>(Sop + (f / 64) * (2 * C::DV * 128) + sw128_chunk(n, (f % 64) / 8) +
+                                                       (f % 8) * 2) = (n < C::DV) ? hi : lo;
+                }
+                for (int e = tid; e < C::D; e += kWorkers) sz[e] = a.z_fin[(size_t)ir.bh * C::D + e];
+                named_sync<kWorkers>(1);
+                cur_bh = ir.bh;
             }
-            tc_fence_before();
-            mbar_arrive(numfree + q);
-            if (valid) {
-                uint4 *dst = reinterpret_cast<uint4 *>(O + (size_t)(row0 + r) * C::DV + h * HC);
+            __nv_bfloat16 *O = static_cast<__nv_bfloat16 *>(a.O) + (size_t)ir.bh * a.n * C::DV;
+            for (int t = 0; t < ir.ntiles; ++t, ++g) {
+                const int p = g % NP, q = g % NN;
+                const int row0 = ir.r0 + t * 128;
+                const int nvalid = min(128, ir.r1 - row0);
+                wait_or_fail(uready + (g & 1), (g >> 1) & 1, failed, status);
+                if (g >= NP) wait_or_fail(pfree + p, ((g - NP) / NP) & 1, failed, status);
+                tc_fence_after();
+                const bool valid = r < nvalid;
+                float den = 0.0f;
+                phi_row_any<C>(Q, tbase + lrow + (g & 1) * C::NU, sTe, sAB, sbias, valid, r, Pb + p * C::PT, nullptr,
+                               nullptr, sz, den);
+                float *dslot = sden + (g & 1) * 512;
+                dslot[Q * 128 + r] = den;
+                fence_proxy_async_smem();
+                tc_fence_before();
+                mbar_arrive(phiready + p);
+                named_sync<kWorkers>(1);  // all four parts of every row's normaliser are written
+                const float dsum = dslot[r] + dslot[128 + r] + dslot[256 + r] + dslot[384 + r] + a.eps;
+                wait_or_fail(numready + q, (g / NN) & 1, failed, status);
+                tc_fence_after();
+                // this thread writes output columns [Q*HC, (Q+1)*HC) of row r
+                constexpr int HC = C::DV / 4;
+                uint4 outv[HC / 8];
+                const uint32_t col = lrow + tmem_num + q * 2 * C::DV + Q * HC;
+                if constexpr (HC == 8) {
+                    uint32_t xh[8], xl[8];
+                    tmem_ld8(col, xh);
+                    tmem_ld8(col + C::DV, xl);
+                    tmem_wait_ld();
+                    float o[8];
 #pragma unroll
-                for (int k = 0; k < HC / 8; ++k) dst[k] = outv[k];
+                    for (int c = 0; c < 8; ++c)
+                        o[c] = (dsum != 0.0f) ? (__uint_as_float(xh[c]) + __uint_as_float(xl[c])) / dsum : 0.0f;
+                    outv[0] = make_uint4(pack_bf16x2(o[0], o[1]), pack_bf16x2(o[2], o[3]), pack_bf16x2(o[4], o[5]),
+                                         pack_bf16x2(o[6], o[7]));
+                } else {
+#pragma unroll
+                    for (int c0 = 0; c0 < HC; c0 += 16) {
+                        uint32_t xh[16], xl[16];
+                        tmem_ld16(col + c0, xh);
+                        tmem_ld16(col + c0 + C::DV, xl);
+                        tmem_wait_ld();
+                        float o[16];
+#pragma unroll
+                        for (int c = 0; c < 16; ++c)
+                            o[c] = (dsum != 0.0f) ? (__uint_as_float(xh[c]) + __uint_as_float(xl[c])) / dsum : 0.0f;
+#pragma unroll
+                        for (int c = 0; c < 16; c += 8)
+                            outv[(c0 + c) / 8] =
+                                make_uint4(pack_bf16x2(o[c], o[c + 1]), pack_bf16x2(o[c + 2], o[c + 3]),
+                                           pack_bf16x2(o[c + 4], o[c + 5]), pack_bf16x2(o[c + 6], o[c + 7]));
+                    }
+                }
+                tc_fence_before();
+                mbar_arrive(numfree + q);
+                if (valid) {
+                    uint4 *dst = reinterpret_cast<uint4 *>(O + (size_t)(row0 + r) * C::DV + Q * HC);
+#pragma unroll
+                    for (int k = 0; k < HC / 8; ++k) dst[k] = outv[k];
+                }
             }
         }
     }
@@ -580,7 +637,6 @@ __global__ void __launch_bounds__(kThreadsTC, 1)
     if (warp == 0) tmem_dealloc(tbase, C::TMEM_Q);
 }
 
-// ---------------------------------------------------------------------------
 // host side
 
 typedef CUresult (*EncodeTiledFn)(CUtensorMap *, CUtensorMapDataType, cuuint32_t, void *, const cuuint64_t *,
@@ -604,7 +660,7 @@ EncodeTiledFn encoder() {
 
 // (width, n, BH) bf16 tensor, boxes of 64 columns x 128 rows, 128B swizzle,
 // out-of-range elements read as zero.
-bool make_map(CUtensorMap *m, const void *base, int width, int n, int BH) {
+bool make_map_impl(CUtensorMap *m, const void *base, int width, int n, int BH) {
     EncodeTiledFn enc = encoder();
     if (!enc) return false;
     cuuint64_t dims[3] = {(cuuint64_t)width, (cuuint64_t)n, (cuuint64_t)BH};
@@ -618,40 +674,60 @@ bool make_map(CUtensorMap *m, const void *base, int width, int n, int BH) {
 
 int *status_word(const AttnArgs &a) { return reinterpret_cast<int *>(reinterpret_cast<char *>(a.counters) - 256); }
 
-// The tensor-core kernels split each head into ranges of whole 128-row tiles
-// (8 tiles by default; LUNA_TC_TILES_PER_SPLIT overrides it for tuning and for
-// tests of long per-block tile loops).  There are never more ranges than the
-// generic plan sized the workspace for.
-AttnArgs tc_splits(const AttnArgs &a) {
+// Work items of the persistent tensor-core kernels: chunks of whole 128-row
+// tiles of one head (4 tiles by default; LUNA_TC_TILES_PER_SPLIT overrides it
+// for tuning and for tests of long per-item tile loops).  There are never more
+// chunks per head than the generic plan sized the partial-sum workspace for.
+AttnArgs tc_items_impl(const AttnArgs &a) {
     AttnArgs b = a;
-    int tiles = 8;
+    const int ntile = (a.n + 127) / 128;
+    int tiles = 4;
     if (const char *env = getenv("LUNA_TC_TILES_PER_SPLIT")) {
         const int v = atoi(env);
         if (v > 0 && v < (1 << 20)) tiles = v;
     }
-    const int ntile = (a.n + 127) / 128;
     if (tiles > ntile) tiles = ntile > 0 ? ntile : 1;
     while ((ntile + tiles - 1) / tiles > a.nsplit) ++tiles;
     b.rows_per_split = tiles * 128;
-    b.nsplit = (a.n + b.rows_per_split - 1) / b.rows_per_split;
+    b.nsplit = (ntile + tiles - 1) / tiles;
     return b;
+}
+
+int sm_count_impl() {
+    static int n = 0;
+    if (n == 0) {
+        int dev = 0;
+        if (cudaGetDevice(&dev) != cudaSuccess || cudaDeviceGetAttribute(&n, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess || n <= 0)
+            n = 148;
+    }
+    return n;
+}
+
+template <class C>
+cudaError_t keys_tc(const AttnArgs &a, cudaStream_t s) {
+    CUtensorMap mK, mV;
+    if (!make_map_impl(&mK, a.K, a.d, a.n, a.B * a.H) || !make_map_impl(&mV, a.V, a.dv, a.n, a.B * a.H))
+        return cudaErrorInvalidValue;
+    cudaError_t e = cudaFuncSetAttribute(k_tc_keys<C>, cudaFuncAttributeMaxDynamicSharedMemorySize, C::SMEM_K);
+    if (e != cudaSuccess) return e;
+    const int items = a.B * a.H * a.nsplit;
+    const int grid = items < sm_count_impl() ? items : sm_count_impl();
+    LUNA_LAUNCH("tc_keys", k_tc_keys<C>, grid, kThreadsTC, C::SMEM_K, s, mK, mV, a, status_word(a));
+    return cudaGetLastError();
 }
 
 template <class C>
 cudaError_t fwd_tc(const AttnArgs &a0, cudaStream_t s) {
-    const AttnArgs a = tc_splits(a0);
-    CUtensorMap mK, mV, mQ;
-    if (!make_map(&mK, a.K, a.d, a.n, a.B * a.H) || !make_map(&mV, a.V, a.dv, a.n, a.B * a.H) ||
-        !make_map(&mQ, a.Q, a.d, a.n, a.B * a.H))
-        return cudaErrorInvalidValue;
-    cudaError_t e = cudaFuncSetAttribute(k_tc_keys<C>, cudaFuncAttributeMaxDynamicSharedMemorySize, C::SMEM_K);
+    const AttnArgs a = tc_items_impl(a0);
+    cudaError_t e = keys_tc<C>(a, s);
     if (e != cudaSuccess) return e;
+    CUtensorMap mQ;
+    if (!make_map_impl(&mQ, a.Q, a.d, a.n, a.B * a.H)) return cudaErrorInvalidValue;
     e = cudaFuncSetAttribute(k_tc_query<C>, cudaFuncAttributeMaxDynamicSharedMemorySize, C::SMEM_Q);
     if (e != cudaSuccess) return e;
-    int *st = status_word(a);
-    LUNA_LAUNCH("tc_keys", k_tc_keys<C>, dim3(a.nsplit, a.B * a.H), kThreadsTC, C::SMEM_K, s, mK, mV, a, st);
-    if ((e = cudaGetLastError()) != cudaSuccess) return e;
-    LUNA_LAUNCH("tc_query", k_tc_query<C>, dim3(a.nsplit, a.B * a.H), kThreadsTC, C::SMEM_Q, s, mQ, a, st);
+    const int items = a.B * a.H * a.nsplit;
+    const int grid = items < sm_count_impl() ? items : sm_count_impl();
+    LUNA_LAUNCH("tc_query", k_tc_query<C>, grid, kThreadsTC, C::SMEM_Q, s, mQ, a, status_word(a));
     return cudaGetLastError();
 }
 
@@ -669,10 +745,17 @@ int variant(const luna_attn_desc &ad, const TableLayout &lay) {
 
 }  // namespace
 
+bool tc_make_map(CUtensorMap *m, const void *base, int width, int n, int BH) {
+    return make_map_impl(m, base, width, n, BH);
+}
+int tc_sm_count() { return sm_count_impl(); }
+AttnArgs tc_work_items(const AttnArgs &a) { return tc_items_impl(a); }
+
 TcPlan tc_plan(const luna_attn_desc &ad, const TableLayout &lay) {
     TcPlan p;
     p.variant = variant(ad, lay);
     p.eligible = p.variant >= 0 && encoder() != nullptr;
+    p.bwd = p.eligible && tc_bwd_supported(ad, lay);
     return p;
 }
 
@@ -690,8 +773,24 @@ cudaError_t launch_tc_fwd(const TcPlan &p, const AttnArgs &a, char *, cudaStream
     return cudaErrorNotSupported;
 }
 
-cudaError_t launch_tc_bwd(const TcPlan &, const AttnArgs &a, char *, bool have_stats, cudaStream_t s) {
-    return launch_simt_bwd(a, LUNA_BF16, have_stats, s);
+cudaError_t launch_tc_stats(const AttnArgs &a0, cudaStream_t s) {
+    const TcPlan p = tc_plan(luna_attn_desc{a0.B, a0.H, a0.n, a0.d, a0.dv, 0, 0, a0.eps, LUNA_BF16}, a0.lay);
+    const AttnArgs a = tc_items_impl(a0);
+    switch (p.variant) {
+        case 0: return keys_tc<C32>(a, s);
+        case 1: return keys_tc<C64>(a, s);
+        case 2: return keys_tc<C128>(a, s);
+    }
+    return cudaErrorNotSupported;
+}
+
+cudaError_t launch_tc_bwd(const TcPlan &p, const AttnArgs &a, char *, bool have_stats, cudaStream_t s) {
+    if (p.bwd && tc_bwd_fits(a)) return launch_tc_bwd_kernels(a, have_stats, s);
+    if (!have_stats) {  // generic backward on the statistics of the tensor-core key pass
+        cudaError_t e = launch_tc_stats(a, s);
+        if (e != cudaSuccess) return e;
+    }
+    return launch_simt_bwd(a, LUNA_BF16, true, s);
 }
 
 }  // namespace luna

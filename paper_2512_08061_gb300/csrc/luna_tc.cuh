@@ -8,6 +8,7 @@ namespace luna {
 struct TcPlan {
     bool eligible = false;   // shape and dtype handled by the tensor-core kernels
     int variant = -1;        // kernel instantiation (value width / projections)
+    bool bwd = false;        // backward also on tensor cores
     size_t ws_fwd = 0, ws_bwd = 0;
 };
 
@@ -15,5 +16,9 @@ TcPlan tc_plan(const luna_attn_desc &ad, const TableLayout &lay);
 bool tc_inputs_ok(const TcPlan &p, const void *a, const void *b, const void *c, const void *d);
 cudaError_t launch_tc_fwd(const TcPlan &p, const AttnArgs &a, char *ws, cudaStream_t s);
 cudaError_t launch_tc_bwd(const TcPlan &p, const AttnArgs &a, char *ws, bool have_stats, cudaStream_t s);
+cudaError_t launch_tc_stats(const AttnArgs &a, cudaStream_t s);
+bool tc_bwd_supported(const luna_attn_desc &ad, const TableLayout &lay);
+bool tc_bwd_fits(const AttnArgs &a);
+cudaError_t launch_tc_bwd_kernels(const AttnArgs &a, bool have_stats, cudaStream_t s);
 
 }  // namespace luna

@@ -1,0 +1,1025 @@
+// Tensor-core backward pass (bf16 I/O, non-causal) on sm_103a.
+//
+// Given dO, the gradient of Eq. (kernel-attn) is (per row i, valid keys j):
+//   den_i = phi(q_i).z + eps,  P_i[f] = sum_c S[f][c] dO_i[c]
+//   dO_i . O_i = phi(q_i) . P_i / den_i,  dden_i = -(dO_i . O_i) / den_i
+//   dphi(q_i) = P_i / den_i + z dden_i,   dnum_i = dO_i / den_i
+//   dS = sum_i phi(q_i) dnum_i^T,  dz = sum_i phi(q_i) dden_i
+//   dphi(k_j) = dS v_j + dz,  dv_j = dS^T phi(k_j)
+// followed by the chain rule through the feature map (d/du of the piecewise
+// linear channel functions, histogram of the channel-MLP gradient statistics)
+// and the projections (dX = dU W, dW = sum dU^T X).
+//
+// Query-side kernel, per 128-row tile (warp roles as in the forward kernels,
+// but eight worker warps, two threads per row):
+//   MMA  U = Q [W_hi; W_mid; W_lo]^T         (u as accurate as fp32: it decides ReLU kinks)
+//   MMA  P = dO [S_hi; S_lo]^T             (dO exact in bf16, S as hi + lo)
+//   workers: phi(Q), den, dO.O, dphi, dU, histogram; tile G = [dO | dU | -(dO.O)]
+//   MMA  [phi/den as hi, lo]^T G  -> dS, dz   (per head run)
+//   MMA  Q^T [dU_hi | dU_lo]      -> dW^T     (whole block)
+// dO enters exactly and phi/den as a hi + lo pair: dS v_j + dz on the key side
+// cancels strongly, and a single bf16 rounding of phi/den there costs about
+// two percent of dK.
+//   MMA  dQ = dU W
+// Key-side kernel, per tile:
+//   MMA  U = K [W_hi; W_mid; W_lo]^T,  dphi = V [dS_hi; dS_lo]^T,  dV = phi [dS_hi; dS_lo]
+//   workers: phi(K), dphi + dz, dU, histogram; tile G = [dU]
+//   MMA  dK = dU W,  dW^T += K^T dU
+// Parameter-gradient partials (dW, db, histogram) are written once per block.
+#include "luna_tc_dev.cuh"
+
+namespace luna {
+namespace {
+using namespace sm100;
+using namespace simt;
+using namespace tcdev;
+
+constexpr int kBWorkers = 256;           // 8 warps, two threads per row
+constexpr int kBTma = 8, kBMma = 9;
+constexpr int kBThreads = kBWorkers + 64;
+constexpr uint32_t kBarBytes = 256;      // mbarriers, TMEM address, flag (each kernel below uses <= 26 slots)
+
+// d = dv = 32, D = 64 (M = 8 projections, L = 8 channels)
+struct B32 {
+    static constexpr int d = 32, DX = 64, DV = 32, MP = 8, D = 64, NU = 32, PP = 4;
+    static constexpr uint32_t TILE = 16384;  // 128 rows x 128 B
+    static constexpr int NKD = d / 16;       // k-steps over d
+    static constexpr int NKV = DV / 16;      // k-steps over dv
+    static constexpr uint32_t WOP = NU * 128;          // [W_hi; W_mid; W_lo; 0] (NU rows x 64)
+    static constexpr uint32_t WXP = d * 128;           // [W_hi; W_hi; W_lo; 0] per output column
+    static constexpr uint32_t SOP2 = 2 * D * 128;      // [S_hi; S_lo] rows per feature, K = dv
+    static constexpr uint32_t SOP = 2 * DV * 128;      // [S_hi; S_lo]^T rows per value column, K = D
+    static constexpr uint32_t HIST = kNint * 16 * 4;
+    // query side: stage = [phi/den (hi, lo interleaved by 16 features) x 2 tiles | Q tile]
+    static constexpr int NSQ = 2, NOQ = 2;
+    static constexpr uint32_t SMEM_Q = NSQ * 3 * TILE + NOQ * TILE + WOP + WXP + SOP2 + kTableBytes + D * 4 +
+                                       2 * 2 * 2 * 128 * 4 + HIST + MP * d * 4 + 64 + kBarBytes + 1024;
+    // key side
+    static constexpr int NSK = 2, NVK = 2;
+    static constexpr uint32_t SMEM_K = NSK * 2 * TILE + NVK * TILE + TILE + WOP + WXP + SOP + SOP2 + kTableBytes +
+                                       D * 4 + HIST + MP * d * 4 + 64 + kBarBytes + 1024;
+    static_assert(SMEM_Q <= kSmemLimit && SMEM_K <= kSmemLimit, "shared memory budget");
+};
+
+// Projection MMA (nk 16-wide k-steps of the X tile) into TMEM.
+template <class C>
+__device__ __forceinline__ void proj_mma(uint32_t tmem_u, uint64_t dx, uint64_t dw) {
+    constexpr uint32_t idesc = idesc_bf16(128, C::NU, false, false);
+#pragma unroll
+    for (int k = 0; k < C::NKD; ++k) mma_bf16_ss(tmem_u, dadd(dx, 32 * k), dadd(dw, 32 * k), idesc, k != 0);
+}
+
+// [W_hi; W_hi; W_lo; 0] as the K-major B operand of dX = [dU_hi | dU_lo | dU_hi | 0] W: row n = output column.
+template <class C>
+__device__ void stage_wx(const AttnArgs &a, uint8_t *Wx) {
+    const float *W = reinterpret_cast<const float *>(a.table + a.lay.off_W);
+    for (int e = threadIdx.x; e < C::d * 64; e += blockDim.x) {
+        const int n = e / 64, k = e % 64;
+        float v = 0.0f;
+        if (k < 3 * C::MP) {
+            __nv_bfloat16 hi, lo;
+            split_bf16(W[(k % C::MP) * a.d + n], hi, lo);
+            v = (k < 2 * C::MP) ? __bfloat162float(hi) : __bfloat162float(lo);
+        }
+        *reinterpret_cast<__nv_bfloat16 *>(Wx + sw128_chunk(n, k / 8) + (k % 8) * 2) = __float2bfloat16_rn(v);
+    }
+}
+
+// Operand rows per feature (hi rows 0..D-1, lo rows D..2D-1), K = value column:
+// the B operand of P = dO S^T and of dphi(k) = V dS^T.
+template <class C>
+__device__ void stage_rows_per_feature(const float *Sg, uint8_t *op, int tid, int nthr) {
+    for (int e = tid; e < 2 * C::D * 64; e += nthr) {
+        const int n = e / 64, c = e % 64, f = n % C::D;
+        float v = 0.0f;
+        if (c < C::DV) {
+            __nv_bfloat16 hi, lo;
+            split_bf16(Sg[f * C::DV + c], hi, lo);
+            v = (n < C::D) ? __bfloat162float(hi) : __bfloat162float(lo);
+        }
+        *reinterpret_cast<__nv_bfloat16 *>(op + sw128_chunk(n, c / 8) + (c % 8) * 2) = __float2bfloat16_rn(v);
+    }
+}
+
+// Operand rows per value column (hi rows 0..DV-1, lo rows DV..2DV-1), K = feature:
+// the B operand of dV = phi dS.
+template <class C>
+__device__ void stage_rows_per_column(const float *Sg, uint8_t *op, int tid, int nthr) {
+    for (int e = tid; e < 2 * C::DV * C::D; e += nthr) {
+        const int n = e / C::D, f = e % C::D, c = n % C::DV;
+        __nv_bfloat16 hi, lo;
+        split_bf16(Sg[f * C::DV + c], hi, lo);
+        *reinterpret_cast<__nv_bfloat16 *>(op + sw128_chunk(n, f / 8) + (f % 8) * 2) = (n < C::DV) ? hi : lo;
+    }
+}
+
+// Interval search for the PP projections of this thread (breadth-first kink tree).
+template <int PP>
+__device__ __forceinline__ void search(const float *sTe, const float (&u)[PP], int (&j)[PP]) {
+    int node[PP];
+#pragma unroll
+    for (int q = 0; q < PP; ++q) node[q] = 1;
+#pragma unroll
+    for (int lvl = 0; lvl < 10; ++lvl)
+#pragma unroll
+        for (int q = 0; q < PP; ++q) node[q] = 2 * node[q] + (sTe[node[q]] < u[q] ? 1 : 0);
+#pragma unroll
+    for (int q = 0; q < PP; ++q) j[q] = node[q] - kEytzinger;
+}
+
+// alpha, beta of the 8 channels on interval j (swizzled table) and phi = relu(alpha u + beta).
+__device__ __forceinline__ void channel_eval(const float *sAB, int j, float u, float (&al)[8], float (&y)[8]) {
+    const float4 *ab = reinterpret_cast<const float4 *>(sAB) + (j << 2);
+#pragma unroll
+    for (int k = 0; k < 4; ++k) {
+        const float4 v = ab[k ^ (j & 3)];
+        al[2 * k] = v.x;
+        al[2 * k + 1] = v.z;
+        y[2 * k] = fmaxf(fmaf(v.x, u, v.y), 0.0f);
+        y[2 * k + 1] = fmaxf(fmaf(v.z, u, v.w), 0.0f);
+    }
+}
+
+__device__ __forceinline__ uint4 pack8(const float (&y)[8]) {
+    return make_uint4(pack_bf16x2(y[0], y[1]), pack_bf16x2(y[2], y[3]), pack_bf16x2(y[4], y[5]),
+                      pack_bf16x2(y[6], y[7]));
+}
+
+// Backward through the channel functions for one projection value: g = dLoss/dphi on
+// the active outputs; adds g and g*u to the interval histogram, returns dLoss/du.
+__device__ __forceinline__ float channel_backward(float *hist, int j, float u, const float (&al)[8],
+                                                  const float (&y)[8], const float (&dphi)[8]) {
+    float du = 0.0f;
+#pragma unroll
+    for (int l = 0; l < 8; ++l) {
+        if (y[l] > 0.0f && dphi[l] != 0.0f) {
+            du = fmaf(dphi[l], al[l], du);
+            atomicAdd(hist + (j * 8 + l) * 2, dphi[l]);
+            atomicAdd(hist + (j * 8 + l) * 2 + 1, dphi[l] * u);
+        }
+    }
+    return du;
+}
+
+// Zeroes a row of a 128-row x 128 B tile (padded rows must not carry garbage
+// into contractions over rows).
+__device__ __forceinline__ void zero_row(uint8_t *tile, int r) {
+#pragma unroll
+    for (int c = 0; c < 8; ++c) *reinterpret_cast<uint4 *>(tile + sw128_chunk(r, c)) = make_uint4(0, 0, 0, 0);
+}
+
+// Writes the per-block parameter-gradient partial: dW (M x d) from smem, db
+// (block sum of per-thread values), the interval histogram.
+template <class C>
+__device__ void store_param_partial(const AttnArgs &a, const float *sdW, float *sdb, const float *hist, float *gp) {
+    const int Md = C::MP * a.d;
+    for (int e = threadIdx.x; e < Md; e += blockDim.x) gp[e] = sdW[e];
+    for (int e = threadIdx.x; e < C::MP; e += blockDim.x) gp[Md + e] = sdb[e];
+    for (int e = threadIdx.x; e < a.lay.nint * 16; e += blockDim.x) gp[Md + C::MP + e] = hist[e];
+}
+
+// ---------------------------------------------------------------------------
+// query side of the backward pass
+
+template <class C>
+__global__ void __launch_bounds__(kBThreads, 1)
+    k_tc_bwd_query(const __grid_constant__ CUtensorMap mapQ, const __grid_constant__ CUtensorMap mapdO, AttnArgs a,
+                   int *status) {
+    extern __shared__ uint8_t smem_raw[];
+    uint8_t *sm = align1024(smem_raw);
+    constexpr int NS = C::NSQ, NO = C::NOQ;
+    constexpr uint32_t T16 = C::TILE;
+    uint8_t *Sb = sm;                    // [NS] x (phi/den tiles x 2, Q tile)
+    uint8_t *Ob = Sb + NS * 3 * T16;     // [NO] dO tile, completed in place into G = [dO | dU | -(dO.O)]
+    uint8_t *Wop = Ob + NO * T16;
+    uint8_t *Wx = Wop + C::WOP;
+    uint8_t *Sop2 = Wx + C::WXP;
+    float *sTe = reinterpret_cast<float *>(Sop2 + C::SOP2);
+    float *sAB = sTe + kEytzinger;
+    float *sbias = sAB + kNint * 16;
+    float *sz = sbias + 32;
+    float *sred = sz + C::D;              // [2 tiles][den, dot][2 halves][128 rows]
+    float *hist = sred + 1024;            // [nint][8][2]
+    float *sdW = hist + kNint * 16;       // [M][d]
+    float *sdb = sdW + C::MP * C::d;      // [M] (padded to 16)
+    uint64_t *bars = reinterpret_cast<uint64_t *>(sdb + 16);
+    uint64_t *fullq = bars;               // [NS]
+    uint64_t *sfree = fullq + NS;         // [NS] phi and Q tile consumed
+    uint64_t *fullo = sfree + NS;         // [NO]
+    uint64_t *ofree = fullo + NO;         // [NO] G tile consumed
+    uint64_t *uready = ofree + NO;        // [2]
+    uint64_t *pready = uready + 2;        // [2]
+    uint64_t *gready = pready + 2;        // [2] count 256 (per tile parity)
+    uint64_t *dqready = gready + 2;       // [1]
+    uint64_t *dqfree = dqready + 1;       // [1] count 256
+    uint64_t *accdone = dqfree + 1;       // [2]
+    uint64_t *accfree = accdone + 2;      // [2] count 128
+    uint64_t *opready = accfree + 2;      // [1] count 256: per-head operands staged
+    uint64_t *wdone = opready + 1;        // [1] dW^T accumulator final
+    uint32_t *tslot = reinterpret_cast<uint32_t *>(wdone + 1);
+    int *slast = reinterpret_cast<int *>(tslot + 1);
+    static_assert((2 * NS + 2 * NO + 15) * 8 + 8 <= kBarBytes, "barrier area");
+
+    const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+    const Items it(a);
+    // TMEM: U [2 x 32] | P [2 x 128] | acc [2 x 64] | dQ [32] | dW^T (M = 64) [16]
+    constexpr uint32_t cU = 0, cP = 64, cA = 320, cQ = 448, cW = 480;
+
+    if (tid == 0) {
+        for (int i = 0; i < NS; ++i) { mbar_init(fullq + i, 1); mbar_init(sfree + i, 1); }
+        for (int i = 0; i < NO; ++i) { mbar_init(fullo + i, 1); mbar_init(ofree + i, 1); }
+        for (int i = 0; i < 2; ++i) {
+            mbar_init(uready + i, 1); mbar_init(pready + i, 1); mbar_init(gready + i, kBWorkers);
+            mbar_init(accdone + i, 1); mbar_init(accfree + i, 128);
+        }
+        mbar_init(dqready, 1);
+        mbar_init(dqfree, kBWorkers);
+        mbar_init(opready, kBWorkers);
+        mbar_init(wdone, 1);
+        fence_mbar_init();
+    }
+    if (warp == 0) { tmem_alloc(tslot, 512); tmem_relinquish(); }
+    stage_phi_table<C>(a, sTe, sAB, sbias, Wop);
+    stage_wx<C>(a, Wx);
+    for (int e = tid; e < kNint * 16; e += blockDim.x) hist[e] = 0.0f;
+    for (int e = tid; e < C::MP * C::d + 16; e += blockDim.x) sdW[e] = 0.0f;
+    // padded rows of every item produce zero gradients
+    for (int item = it.begin; item < it.end; ++item) {
+        const ItemRange ir = item_range(a, it, item);
+        __nv_bfloat16 *dQ = static_cast<__nv_bfloat16 *>(a.dQ) + (size_t)ir.bh * a.n * C::d;
+        const int z0 = max(ir.r0, ir.r1);
+        for (int e = tid; e < (ir.rend - z0) * C::d / 8; e += blockDim.x)
+            reinterpret_cast<uint4 *>(dQ + (size_t)z0 * C::d)[e] = make_uint4(0, 0, 0, 0);
+    }
+    fence_proxy_async_smem();
+    tc_fence_before();
+    __syncthreads();
+    tc_fence_after();
+    const uint32_t tbase = *tslot;
+
+    if (warp == kBTma) {
+        if (lane < 2) {
+            const int T = block_tiles(a, it);
+            TileCursor cur;
+            cur.start(a, it);
+            bool failed = false;
+            for (int g = 0; g < T && !failed; ++g, cur.next(a, it)) {
+                if (lane == 0) {
+                    const int s = g % NS;
+                    if (g >= NS) wait_or_fail(sfree + s, ((g - NS) / NS) & 1, failed, status);
+                    mbar_arrive_expect_tx(fullq + s, T16);
+                    tma_load_3d(Sb + s * 3 * T16 + 2 * T16, &mapQ, 0, cur.row0(), cur.g.bh, fullq + s);
+                } else {
+                    const int o = g % NO;
+                    if (g >= NO) wait_or_fail(ofree + o, ((g - NO) / NO) & 1, failed, status);
+                    mbar_arrive_expect_tx(fullo + o, T16);
+                    tma_load_3d(Ob + o * T16, &mapdO, 0, cur.row0(), cur.g.bh, fullo + o);
+                }
+            }
+        }
+    } else if (warp == kBMma) {
+        if (lane == 0) {
+            const int T = block_tiles(a, it);
+            const uint64_t dS0 = sdesc(smem_u32(Sb), 16384, 1024, kSwizzle128);
+            const uint64_t dO0 = sdesc(smem_u32(Ob), 16384, 1024, kSwizzle128);
+            const uint64_t dWo = sdesc(smem_u32(Wop), 16, 1024, kSwizzle128);
+            const uint64_t dWx = sdesc(smem_u32(Wx), 16, 1024, kSwizzle128);
+            const uint64_t dSp = sdesc(smem_u32(Sop2), 16, 1024, kSwizzle128);
+            bool failed = false;
+            auto proj = [&](int g) {
+                const int s = g % NS;
+                wait_or_fail(fullq + s, (g / NS) & 1, failed, status);
+                tc_fence_after();
+                proj_mma<C>(tbase + cU + (g & 1) * C::NU, dadd(dS0, s * 3 * T16 + 2 * T16), dWo);
+                mma_commit(uready + (g & 1));
+            };
+            auto pmma = [&](int g) {
+                const int o = g % NO;
+                wait_or_fail(fullo + o, (g / NO) & 1, failed, status);
+                tc_fence_after();
+                constexpr uint32_t idP = idesc_bf16(128, 2 * C::D, false, false);
+#pragma unroll
+                for (int k = 0; k < C::NKV; ++k)
+                    mma_bf16_ss(tbase + cP + (g & 1) * 128, dadd(dO0, o * T16 + 32 * k), dadd(dSp, 32 * k), idP, k != 0);
+                mma_commit(pready + (g & 1));
+            };
+            // runs: stretches of this block's tiles that share a head.  P of the first tile of a run
+            // waits for the workers to stage that head's operands (opready, one phase per run).
+            int op_phase = 0;
+            if (T > 0) { proj(0); wait_or_fail(opready, op_phase++ & 1, failed, status); pmma(0); }
+            if (T > 1) proj(1);
+            TileCursor cur;
+            cur.start(a, it);
+            int run_bh = -1, ne = 0, run_left = 0, tile_in_run = 0;
+            for (int g = 0; g < T && !failed; ++g) {
+                const int s = g % NS, o = g % NO;
+                if (cur.g.bh != run_bh) {  // a run starts at tile g
+                    run_bh = cur.g.bh;
+                    run_left = 0;
+                    for (int i = cur.item; i < it.end && i / it.nchunk == run_bh; ++i)
+                        run_left += item_range(a, it, i).ntiles;
+                    tile_in_run = 0;
+                    if (ne >= 2) wait_or_fail(accfree + (ne & 1), ((ne - 2) >> 1) & 1, failed, status);
+                }
+                const int b = ne & 1;
+                TileCursor nx = cur;
+                nx.next(a, it);
+                const bool next_new_run = (g + 1 < T) && nx.g.bh != cur.g.bh;
+                if (g + 1 < T && !next_new_run) pmma(g + 1);
+                wait_or_fail(gready + (g & 1), (g >> 1) & 1, failed, status);
+                if (g >= 1) wait_or_fail(dqfree, (g - 1) & 1, failed, status);
+                tc_fence_after();
+                // [phi/den hi, lo]^T G: dS (cols 0..31) and dz (cols 56, 57) of every feature, once as hi, once as lo
+                constexpr uint32_t idG = idesc_bf16(128, 64, true, true);
+#pragma unroll
+                for (int k = 0; k < 8; ++k)
+                    mma_bf16_ss(tbase + cA + b * 64, dadd(dS0, s * 3 * T16 + 2048 * k), dadd(dO0, o * T16 + 2048 * k),
+                                idG, (tile_in_run > 0 || k > 0) ? 1u : 0u);
+                // Q^T [dU_hi | dU_lo] (G cols 32..47): dW^T rows = input columns
+                constexpr uint32_t idW = idesc_bf16(64, 16, true, true);
+#pragma unroll
+                for (int k = 0; k < 8; ++k)
+                    mma_bf16_ss(tbase + cW, dadd(dS0, s * 3 * T16 + 2 * T16 + 2048 * k),
+                                dadd(dO0, o * T16 + 64 + 2048 * k), idW, (g > 0 || k > 0) ? 1u : 0u);
+                constexpr uint32_t idQ = idesc_bf16(128, C::d, false, false);
+#pragma unroll
+                for (int k = 0; k < 2; ++k)
+                    mma_bf16_ss(tbase + cQ, dadd(dO0, o * T16 + 64 + 32 * k), dadd(dWx, 32 * k), idQ, k != 0);
+                mma_commit(dqready);
+                mma_commit(ofree + o);
+                mma_commit(sfree + s);
+                ++tile_in_run;
+                if (--run_left == 0) { mma_commit(accdone + b); ++ne; }
+                if (next_new_run) { wait_or_fail(opready, op_phase++ & 1, failed, status); pmma(g + 1); }
+                if (g + 2 < T) proj(g + 2);
+                cur = nx;
+            }
+            if (T > 0 && !failed) mma_commit(wdone);
+            else mbar_arrive(wdone);
+        }
+    } else {
+        // workers
+        const int H = warp >> 2, r = ((warp & 3) << 5) | lane;
+        const uint32_t lrow = (uint32_t)((warp & 3) << 5) << 16;
+        bool failed = false;
+        float db_acc[C::PP];
+#pragma unroll
+        for (int q = 0; q < C::PP; ++q) db_acc[q] = 0.0f;
+        int g = 0, ne = 0;
+        for (int i0 = it.begin; i0 < it.end;) {
+            const int bh = i0 / it.nchunk;
+            const int i1 = min(it.end, (bh + 1) * it.nchunk);
+            int run_tiles = 0;
+            for (int i = i0; i < i1; ++i) run_tiles += item_range(a, it, i).ntiles;
+            if (run_tiles > 0) {
+                // operands of this head: [S_hi; S_lo] rows per feature, z (fp32)
+                named_sync<kBWorkers>(1);
+                stage_rows_per_feature<C>(a.S_fin + (size_t)bh * C::D * C::DV, Sop2, tid, kBWorkers);
+                for (int e = tid; e < C::D; e += kBWorkers) sz[e] = a.z_fin[(size_t)bh * C::D + e];
+                fence_proxy_async_smem();
+                named_sync<kBWorkers>(1);
+                mbar_arrive(opready);
+            }
+            __nv_bfloat16 *dQ = static_cast<__nv_bfloat16 *>(a.dQ) + (size_t)bh * a.n * C::d;
+            for (int item = i0; item < i1; ++item) {
+                const ItemRange ir = item_range(a, it, item);
+                for (int t = 0; t < ir.ntiles; ++t, ++g) {
+                    const int s = g % NS, o = g % NO;
+                    const int row0 = ir.r0 + t * 128;
+                    const int nvalid = min(128, ir.r1 - row0);
+                    const bool valid = r < nvalid;
+                    uint8_t *phit = Sb + s * 3 * T16, *qt = phit + 2 * T16, *gt = Ob + o * T16;
+                    wait_or_fail(uready + (g & 1), (g >> 1) & 1, failed, status);
+                    tc_fence_after();
+                    float u[C::PP];
+                    int j[C::PP];
+                    {
+                        uint32_t x[16], x2[8];
+                        tmem_ld16(tbase + lrow + cU + (g & 1) * C::NU, x);
+                        tmem_ld8(tbase + lrow + cU + (g & 1) * C::NU + 16, x2);
+                        tmem_wait_ld();
+#pragma unroll
+                        for (int q = 0; q < C::PP; ++q) {
+                            const int i = H * C::PP + q;
+                            u[q] = (__uint_as_float(x[i]) + __uint_as_float(x[8 + i])) + __uint_as_float(x2[i]) +
+                                   sbias[i];
+                        }
+                    }
+                    search<C::PP>(sTe, u, j);
+                    if (!valid && H == 0) zero_row(qt, r);  // padded rows: no contribution to dW
+                    // normaliser and dO.O from P = S dO
+                    wait_or_fail(pready + (g & 1), (g >> 1) & 1, failed, status);
+                    tc_fence_after();
+                    float denp = 0.0f, dotp = 0.0f;
+                    const uint32_t pcol = tbase + lrow + cP + (g & 1) * 128;
+#pragma unroll
+                    for (int q = 0; q < C::PP; ++q) {
+                        const int i = H * C::PP + q;
+                        float al[8], y[8];
+                        channel_eval(sAB, j[q], u[q], al, y);
+                        uint32_t ph[8], pl[8];
+                        tmem_ld8(pcol + 8 * i, ph);
+                        tmem_ld8(pcol + C::D + 8 * i, pl);
+                        tmem_wait_ld();
+#pragma unroll
+                        for (int l = 0; l < 8; ++l) {
+                            denp = fmaf(y[l], sz[8 * i + l], denp);
+                            dotp = fmaf(y[l], __uint_as_float(ph[l]) + __uint_as_float(pl[l]), dotp);
+                        }
+                    }
+                    float *rs = sred + (g & 1) * 512;
+                    rs[H * 128 + r] = denp;
+                    rs[256 + H * 128 + r] = dotp;
+                    named_sync<kBWorkers>(1);
+                    const float den = rs[r] + rs[128 + r] + a.eps;
+                    const float dotn = rs[256 + r] + rs[384 + r];  // = (dO.O) * den
+                    const bool live = valid && den != 0.0f;
+                    const float inv = live ? 1.0f / den : 0.0f;
+                    const float ndot = live ? -dotn * inv : 0.0f;  // -(dO.O)
+                    const float dden = ndot * inv;
+                    // gradients through the feature map; phi/den (bf16) for the stacked contraction
+                    float dU[C::PP];
+#pragma unroll
+                    for (int q = 0; q < C::PP; ++q) {
+                        const int i = H * C::PP + q;
+                        float al[8], y[8], dphi[8];
+                        channel_eval(sAB, j[q], u[q], al, y);
+                        {
+                            // phi/den as hi, lo; a row holds 16-feature groups [hi | lo | hi | lo] per 64-wide tile,
+                            // so that hi and lo of a feature meet in one TMEM lane quarter of the accumulator
+                            float yh[8], yl[8];
+#pragma unroll
+                            for (int l = 0; l < 8; ++l) {
+                                const float v = live ? y[l] * inv : 0.0f;  // select: padded rows may be non-finite
+                                yh[l] = __bfloat162float(__float2bfloat16_rn(v));
+                                yl[l] = v - yh[l];
+                            }
+                            const int ch = 4 * (i >> 1) + (i & 1), cl = ch + 2;
+                            *reinterpret_cast<uint4 *>(phit + (ch >> 3) * T16 + sw128_chunk(r, ch & 7)) = pack8(yh);
+                            *reinterpret_cast<uint4 *>(phit + (cl >> 3) * T16 + sw128_chunk(r, cl & 7)) = pack8(yl);
+                        }
+                        uint32_t ph[8], pl[8];
+                        tmem_ld8(pcol + 8 * i, ph);
+                        tmem_ld8(pcol + C::D + 8 * i, pl);
+                        tmem_wait_ld();
+#pragma unroll
+                        for (int l = 0; l < 8; ++l)
+                            dphi[l] = live ? (__uint_as_float(ph[l]) + __uint_as_float(pl[l])) * inv + sz[8 * i + l] * dden
+                                           : 0.0f;
+                        dU[q] = live ? channel_backward(hist, j[q], u[q], al, y, dphi) : 0.0f;
+                        db_acc[q] += dU[q];
+                    }
+                    // G = [dO (dv cols) | dU_hi | dU_lo | dU_hi | -(dO.O) hi, lo | 0] over the dO tile (in place)
+                    {
+                        if (!valid) {  // padded rows may hold anything (even non-finite values)
+                            const int c0 = H * (C::DV / 2);
+#pragma unroll
+                            for (int cc = 0; cc < C::DV / 2; cc += 8)
+                                *reinterpret_cast<uint4 *>(gt + sw128_chunk(r, (c0 + cc) / 8)) = make_uint4(0, 0, 0, 0);
+                        }
+                        __nv_bfloat16 hi[C::PP], lo[C::PP];
+#pragma unroll
+                        for (int q = 0; q < C::PP; ++q) split_bf16(dU[q], hi[q], lo[q]);
+                        // columns 32 + 4H .. : dU_hi;  40 + 4H: dU_lo;  48 + 4H: dU_hi (chunks 4, 5, 6)
+                        uint2 vh, vl;
+                        vh.x = (uint32_t)__bfloat16_as_ushort(hi[0]) | ((uint32_t)__bfloat16_as_ushort(hi[1]) << 16);
+                        vh.y = (uint32_t)__bfloat16_as_ushort(hi[2]) | ((uint32_t)__bfloat16_as_ushort(hi[3]) << 16);
+                        vl.x = (uint32_t)__bfloat16_as_ushort(lo[0]) | ((uint32_t)__bfloat16_as_ushort(lo[1]) << 16);
+                        vl.y = (uint32_t)__bfloat16_as_ushort(lo[2]) | ((uint32_t)__bfloat16_as_ushort(lo[3]) << 16);
+                        *reinterpret_cast<uint2 *>(gt + sw128_chunk(r, 4) + H * 8) = vh;
+                        *reinterpret_cast<uint2 *>(gt + sw128_chunk(r, 5) + H * 8) = vl;
+                        *reinterpret_cast<uint2 *>(gt + sw128_chunk(r, 6) + H * 8) = vh;
+                        if (H == 0) {  // chunk 7: -(dO.O) as hi, lo; zeros
+                            __nv_bfloat16 th, tl;
+                            split_bf16(ndot, th, tl);
+                            *reinterpret_cast<uint4 *>(gt + sw128_chunk(r, 7)) = make_uint4(
+                                (uint32_t)__bfloat16_as_ushort(th) | ((uint32_t)__bfloat16_as_ushort(tl) << 16), 0u, 0u, 0u);
+                        }
+                    }
+                    fence_proxy_async_smem();
+                    tc_fence_before();
+                    mbar_arrive(gready + (g & 1));
+                    // dQ
+                    wait_or_fail(dqready, g & 1, failed, status);
+                    tc_fence_after();
+                    {
+                        uint32_t x[16];
+                        tmem_ld16(tbase + lrow + cQ + H * 16, x);
+                        tmem_wait_ld();
+                        float f[16];
+#pragma unroll
+                        for (int c = 0; c < 16; ++c) f[c] = __uint_as_float(x[c]);
+                        tc_fence_before();
+                        mbar_arrive(dqfree);
+                        if (valid) {
+                            uint4 *dst = reinterpret_cast<uint4 *>(dQ + (size_t)(row0 + r) * C::d + H * 16);
+                            float f0[8], f1[8];
+#pragma unroll
+                            for (int c = 0; c < 8; ++c) { f0[c] = f[c]; f1[c] = f[8 + c]; }
+                            dst[0] = pack8(f0);
+                            dst[1] = pack8(f1);
+                        }
+                    }
+                }
+            }
+            // run epilogue (warps 0..3 own all 128 TMEM lanes): dS, dz partial of this head.  Warp w holds
+            // features 16w..16w+15, hi in lanes 0..15 and lo in lanes 16..31.
+            if (warp < 4) {
+                const int c_first = owner_block((long long)bh * it.nchunk, it.total, gridDim.x);
+                const int c_last = owner_block((long long)(bh + 1) * it.nchunk - 1, it.total, gridDim.x);
+                const int nruns = c_last - c_first + 1;
+                const size_t slot = (size_t)bh * it.nchunk + (blockIdx.x - c_first);
+                float *Sp = a.dS_part + slot * C::D * C::DV;
+                float *zp = a.dz_part + slot * C::D;
+                const uint32_t lr = (uint32_t)(warp << 5) << 16;
+                const bool have = run_tiles > 0;
+                const int b = ne & 1;
+                if (have) wait_or_fail(accdone + b, (ne >> 1) & 1, failed, status);
+                tc_fence_after();
+                const uint32_t acc = tbase + lr + cA + b * 64;
+                uint32_t x[16], y[16], w[16];
+                if (have) {
+                    tmem_ld16(acc, x);
+                    tmem_ld16(acc + 16, y);
+                    tmem_ld16(acc + 48, w);
+                    tmem_wait_ld();
+                }
+                float fx[16], fy[16];
+#pragma unroll
+                for (int c = 0; c < 16; ++c) {
+                    fx[c] = have ? __uint_as_float(x[c]) : 0.0f;
+                    fy[c] = have ? __uint_as_float(y[c]) : 0.0f;
+                    fx[c] += __shfl_down_sync(0xffffffffu, fx[c], 16);
+                    fy[c] += __shfl_down_sync(0xffffffffu, fy[c], 16);
+                }
+                float fz = have ? __uint_as_float(w[8]) + __uint_as_float(w[9]) : 0.0f;
+                fz += __shfl_down_sync(0xffffffffu, fz, 16);
+                if (lane < 16) {
+                    const int f = (warp << 4) | lane;
+#pragma unroll
+                    for (int c = 0; c < 16; c += 4) {
+                        *reinterpret_cast<float4 *>(Sp + f * C::DV + c) = make_float4(fx[c], fx[c + 1], fx[c + 2], fx[c + 3]);
+                        *reinterpret_cast<float4 *>(Sp + f * C::DV + 16 + c) =
+                            make_float4(fy[c], fy[c + 1], fy[c + 2], fy[c + 3]);
+                    }
+                    zp[f] = fz;
+                }
+                tc_fence_before();
+                if (have) mbar_arrive(accfree + b);
+                __threadfence();
+                named_sync<128>(2);
+                if (tid == 0) *slast = (atomicAdd(a.counters + a.B * a.H + bh, 1) == nruns - 1) ? 1 : 0;
+                named_sync<128>(2);
+                if (*slast) {
+                    __threadfence();
+                    ordered_sum4(a.dS_part + (size_t)bh * it.nchunk * C::D * C::DV, nruns, C::D * C::DV,
+                                 a.dS_fin + (size_t)bh * C::D * C::DV, tid, 128);
+                    ordered_sum4(a.dz_part + (size_t)bh * it.nchunk * C::D, nruns, C::D, a.dz_fin + (size_t)bh * C::D,
+                                 tid, 128);
+                    if (tid == 0) a.counters[a.B * a.H + bh] = 0;
+                }
+                named_sync<128>(2);
+            }
+            if (run_tiles > 0) ++ne;
+            i0 = i1;
+        }
+        // db: sum over the rows of each warp, then over warps
+#pragma unroll
+        for (int q = 0; q < C::PP; ++q) {
+            float v = db_acc[q];
+#pragma unroll
+            for (int o = 16; o > 0; o >>= 1) v += __shfl_xor_sync(0xffffffffu, v, o);
+            if (lane == 0) atomicAdd(sdb + H * C::PP + q, v);
+        }
+        // dW^T accumulator (M = 64: input column cd in lane 32*(cd/16) + cd%16)
+        if (warp < 4) {
+            const int T = block_tiles(a, it);
+            if (T > 0) wait_or_fail(wdone, 0, failed, status);
+            tc_fence_after();
+            uint32_t x[16];
+            tmem_ld16(tbase + ((uint32_t)(warp << 5) << 16) + cW, x);
+            tmem_wait_ld();
+            const int cd = (warp << 4) | lane;
+            if (T > 0 && lane < 16 && cd < C::d)
+#pragma unroll
+                for (int i = 0; i < C::MP; ++i) sdW[i * C::d + cd] = __uint_as_float(x[i]) + __uint_as_float(x[C::MP + i]);
+        }
+    }
+    tc_fence_before();
+    __syncthreads();
+    store_param_partial<C>(a, sdW, sdb, hist, a.gpart + (size_t)blockIdx.x * a.gsize);
+    __syncthreads();
+    if (warp == 0) tmem_dealloc(tbase, 512);
+}
+
+// ---------------------------------------------------------------------------
+// key side of the backward pass
+
+template <class C>
+__global__ void __launch_bounds__(kBThreads, 1)
+    k_tc_bwd_key(const __grid_constant__ CUtensorMap mapK, const __grid_constant__ CUtensorMap mapV, AttnArgs a,
+                 int *status) {
+    extern __shared__ uint8_t smem_raw[];
+    uint8_t *sm = align1024(smem_raw);
+    constexpr int NS = C::NSK, NV = C::NVK;
+    constexpr uint32_t T16 = C::TILE;
+    uint8_t *Sb = sm;                    // [NS] x (phi_hi tile, K tile)
+    uint8_t *Vb = Sb + NS * 2 * T16;     // [NV]
+    uint8_t *Gt = Vb + NV * T16;         // [dU_hi | dU_lo | dU_hi | 0]
+    uint8_t *Wop = Gt + T16;
+    uint8_t *Wx = Wop + C::WOP;
+    uint8_t *Sop = Wx + C::WXP;          // dV = phi [dS_hi; dS_lo]: rows per value column
+    uint8_t *Sop2 = Sop + C::SOP;        // dphi = V [dS_hi; dS_lo]^T: rows per feature
+    float *sTe = reinterpret_cast<float *>(Sop2 + C::SOP2);
+    float *sAB = sTe + kEytzinger;
+    float *sbias = sAB + kNint * 16;
+    float *sdz = sbias + 32;
+    float *hist = sdz + C::D;
+    float *sdW = hist + kNint * 16;
+    float *sdb = sdW + C::MP * C::d;
+    uint64_t *bars = reinterpret_cast<uint64_t *>(sdb + 16);
+    uint64_t *fullk = bars;              // [NS]
+    uint64_t *sfree = fullk + NS;        // [NS]
+    uint64_t *fullv = sfree + NS;        // [NV]
+    uint64_t *vfree = fullv + NV;        // [NV]
+    uint64_t *uready = vfree + NV;       // [2]
+    uint64_t *fready = uready + 2;       // [2] dphi in TMEM
+    uint64_t *phiready = fready + 2;     // [2] count 256
+    uint64_t *dvready = phiready + 2;    // [2]
+    uint64_t *dvfree = dvready + 2;      // [2] count 256
+    uint64_t *gready = dvfree + 2;       // [2] count 256
+    uint64_t *gfree = gready + 2;        // [1]
+    uint64_t *dkready = gfree + 1;       // [1]
+    uint64_t *dkfree = dkready + 1;      // [1] count 256
+    uint64_t *opready = dkfree + 1;      // [1] count 256
+    uint64_t *wdone = opready + 1;       // [1]
+    uint32_t *tslot = reinterpret_cast<uint32_t *>(wdone + 1);
+    static_assert((2 * NS + 2 * NV + 17) * 8 + 4 <= kBarBytes, "barrier area");
+
+    const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+    const Items it(a);
+    // TMEM: U [2 x 32] | dphi [2 x 128] | dV [2 x 64] | dK [32] | dW (M = 64) [16]
+    constexpr uint32_t cU = 0, cF = 64, cV = 320, cK = 448, cW = 480;
+
+    if (tid == 0) {
+        for (int i = 0; i < NS; ++i) { mbar_init(fullk + i, 1); mbar_init(sfree + i, 1); }
+        for (int i = 0; i < NV; ++i) { mbar_init(fullv + i, 1); mbar_init(vfree + i, 1); }
+        for (int i = 0; i < 2; ++i) {
+            mbar_init(uready + i, 1); mbar_init(fready + i, 1); mbar_init(phiready + i, kBWorkers);
+            mbar_init(dvready + i, 1); mbar_init(dvfree + i, kBWorkers); mbar_init(gready + i, kBWorkers);
+        }
+        mbar_init(dkready, 1);
+        mbar_init(dkfree, kBWorkers);
+        mbar_init(gfree, 1);
+        mbar_init(opready, kBWorkers);
+        mbar_init(wdone, 1);
+        fence_mbar_init();
+    }
+    if (warp == 0) { tmem_alloc(tslot, 512); tmem_relinquish(); }
+    stage_phi_table<C>(a, sTe, sAB, sbias, Wop);
+    stage_wx<C>(a, Wx);
+    for (int e = tid; e < kNint * 16; e += blockDim.x) hist[e] = 0.0f;
+    for (int e = tid; e < C::MP * C::d + 16; e += blockDim.x) sdW[e] = 0.0f;
+    for (int e = tid; e < (int)(T16 / 16); e += blockDim.x) reinterpret_cast<uint4 *>(Gt)[e] = make_uint4(0, 0, 0, 0);
+    for (int item = it.begin; item < it.end; ++item) {  // padded rows receive zero gradients
+        const ItemRange ir = item_range(a, it, item);
+        __nv_bfloat16 *dK = static_cast<__nv_bfloat16 *>(a.dK) + (size_t)ir.bh * a.n * C::d;
+        __nv_bfloat16 *dV = static_cast<__nv_bfloat16 *>(a.dV) + (size_t)ir.bh * a.n * C::DV;
+        const int z0 = max(ir.r0, ir.r1);
+        for (int e = tid; e < (ir.rend - z0) * C::d / 8; e += blockDim.x)
+            reinterpret_cast<uint4 *>(dK + (size_t)z0 * C::d)[e] = make_uint4(0, 0, 0, 0);
+        for (int e = tid; e < (ir.rend - z0) * C::DV / 8; e += blockDim.x)
+            reinterpret_cast<uint4 *>(dV + (size_t)z0 * C::DV)[e] = make_uint4(0, 0, 0, 0);
+    }
+    fence_proxy_async_smem();
+    tc_fence_before();
+    __syncthreads();
+    tc_fence_after();
+    const uint32_t tbase = *tslot;
+
+    if (warp == kBTma) {
+        if (lane < 2) {
+            const int T = block_tiles(a, it);
+            TileCursor cur;
+            cur.start(a, it);
+            bool failed = false;
+            for (int g = 0; g < T && !failed; ++g, cur.next(a, it)) {
+                if (lane == 0) {
+                    const int s = g % NS;
+                    if (g >= NS) wait_or_fail(sfree + s, ((g - NS) / NS) & 1, failed, status);
+                    mbar_arrive_expect_tx(fullk + s, T16);
+                    tma_load_3d(Sb + s * 2 * T16 + T16, &mapK, 0, cur.row0(), cur.g.bh, fullk + s);
+                } else {
+                    const int v = g % NV;
+                    if (g >= NV) wait_or_fail(vfree + v, ((g - NV) / NV) & 1, failed, status);
+                    mbar_arrive_expect_tx(fullv + v, T16);
+                    tma_load_3d(Vb + v * T16, &mapV, 0, cur.row0(), cur.g.bh, fullv + v);
+                }
+            }
+        }
+    } else if (warp == kBMma) {
+        if (lane == 0) {
+            const int T = block_tiles(a, it);
+            const uint64_t dS0 = sdesc(smem_u32(Sb), 16384, 1024, kSwizzle128);
+            const uint64_t dV0 = sdesc(smem_u32(Vb), 16384, 1024, kSwizzle128);
+            const uint64_t dG = sdesc(smem_u32(Gt), 16384, 1024, kSwizzle128);
+            const uint64_t dWo = sdesc(smem_u32(Wop), 16, 1024, kSwizzle128);
+            const uint64_t dWx = sdesc(smem_u32(Wx), 16, 1024, kSwizzle128);
+            const uint64_t dSa = sdesc(smem_u32(Sop), 16, 1024, kSwizzle128);
+            const uint64_t dSb = sdesc(smem_u32(Sop2), 16, 1024, kSwizzle128);
+            bool failed = false;
+            auto proj = [&](int g) {
+                const int s = g % NS;
+                wait_or_fail(fullk + s, (g / NS) & 1, failed, status);
+                tc_fence_after();
+                proj_mma<C>(tbase + cU + (g & 1) * C::NU, dadd(dS0, s * 2 * T16 + T16), dWo);
+                mma_commit(uready + (g & 1));
+            };
+            auto fmma = [&](int g) {  // dphi = V [dS_hi; dS_lo]^T
+                const int v = g % NV;
+                wait_or_fail(fullv + v, (g / NV) & 1, failed, status);
+                tc_fence_after();
+                constexpr uint32_t idF = idesc_bf16(128, 2 * C::D, false, false);
+#pragma unroll
+                for (int k = 0; k < C::NKV; ++k)
+                    mma_bf16_ss(tbase + cF + (g & 1) * 128, dadd(dV0, v * T16 + 32 * k), dadd(dSb, 32 * k), idF, k != 0);
+                mma_commit(fready + (g & 1));
+                mma_commit(vfree + v);
+            };
+            int op_phase = 0;
+            if (T > 0) { proj(0); wait_or_fail(opready, op_phase++ & 1, failed, status); fmma(0); }
+            if (T > 1) proj(1);
+            TileCursor cur;
+            cur.start(a, it);
+            for (int g = 0; g < T && !failed; ++g) {
+                const int s = g % NS;
+                TileCursor nx = cur;
+                nx.next(a, it);
+                const bool next_new_run = (g + 1 < T) && nx.g.bh != cur.g.bh;
+                if (g + 1 < T && !next_new_run) fmma(g + 1);
+                // dV = phi [dS_hi; dS_lo]  (phi K-major over the D features)
+                wait_or_fail(phiready + (g & 1), (g >> 1) & 1, failed, status);
+                if (g >= 2) wait_or_fail(dvfree + (g & 1), ((g - 2) >> 1) & 1, failed, status);
+                tc_fence_after();
+                constexpr uint32_t idV = idesc_bf16(128, 2 * C::DV, false, false);
+#pragma unroll
+                for (int k = 0; k < C::D / 16; ++k)
+                    mma_bf16_ss(tbase + cV + (g & 1) * 64, dadd(dS0, s * 2 * T16 + 32 * k), dadd(dSa, 32 * k), idV,
+                                k != 0);
+                mma_commit(dvready + (g & 1));
+                // dK = [dU_hi | dU_lo | dU_hi] W and dW^T += K^T dU
+                wait_or_fail(gready + (g & 1), (g >> 1) & 1, failed, status);
+                if (g >= 1) wait_or_fail(dkfree, (g - 1) & 1, failed, status);
+                tc_fence_after();
+                constexpr uint32_t idK = idesc_bf16(128, C::d, false, false);
+#pragma unroll
+                for (int k = 0; k < 2; ++k)
+                    mma_bf16_ss(tbase + cK, dadd(dG, 32 * k), dadd(dWx, 32 * k), idK, k != 0);
+                constexpr uint32_t idW = idesc_bf16(64, 16, true, true);
+#pragma unroll
+                for (int k = 0; k < 8; ++k)
+                    mma_bf16_ss(tbase + cW, dadd(dS0, s * 2 * T16 + T16 + 2048 * k), dadd(dG, 2048 * k), idW,
+                                (g > 0 || k > 0) ? 1u : 0u);
+                mma_commit(dkready);
+                mma_commit(gfree);
+                mma_commit(sfree + s);
+                if (next_new_run) { wait_or_fail(opready, op_phase++ & 1, failed, status); fmma(g + 1); }
+                if (g + 2 < T) proj(g + 2);
+                cur = nx;
+            }
+            if (T > 0 && !failed) mma_commit(wdone);
+            else mbar_arrive(wdone);
+        }
+    } else {
+        const int H = warp >> 2, r = ((warp & 3) << 5) | lane;
+        const uint32_t lrow = (uint32_t)((warp & 3) << 5) << 16;
+        bool failed = false;
+        float db_acc[C::PP];
+#pragma unroll
+        for (int q = 0; q < C::PP; ++q) db_acc[q] = 0.0f;
+        int g = 0;
+        for (int i0 = it.begin; i0 < it.end;) {
+            const int bh = i0 / it.nchunk;
+            const int i1 = min(it.end, (bh + 1) * it.nchunk);
+            int run_tiles = 0;
+            for (int i = i0; i < i1; ++i) run_tiles += item_range(a, it, i).ntiles;
+            if (run_tiles > 0) {
+                named_sync<kBWorkers>(1);
+                const float *dSg = a.dS_fin + (size_t)bh * C::D * C::DV;
+                stage_rows_per_column<C>(dSg, Sop, tid, kBWorkers);
+                stage_rows_per_feature<C>(dSg, Sop2, tid, kBWorkers);
+                for (int e = tid; e < C::D; e += kBWorkers) sdz[e] = a.dz_fin[(size_t)bh * C::D + e];
+                fence_proxy_async_smem();
+                named_sync<kBWorkers>(1);
+                mbar_arrive(opready);
+            }
+            __nv_bfloat16 *dK = static_cast<__nv_bfloat16 *>(a.dK) + (size_t)bh * a.n * C::d;
+            __nv_bfloat16 *dV = static_cast<__nv_bfloat16 *>(a.dV) + (size_t)bh * a.n * C::DV;
+            for (int item = i0; item < i1; ++item) {
+                const ItemRange ir = item_range(a, it, item);
+                for (int t = 0; t < ir.ntiles; ++t, ++g) {
+                    const int s = g % NS;
+                    const int row0 = ir.r0 + t * 128;
+                    const int nvalid = min(128, ir.r1 - row0);
+                    const bool valid = r < nvalid;
+                    uint8_t *phit = Sb + s * 2 * T16, *kt = phit + T16;
+                    wait_or_fail(uready + (g & 1), (g >> 1) & 1, failed, status);
+                    tc_fence_after();
+                    float u[C::PP];
+                    int j[C::PP];
+                    {
+                        uint32_t x[16], x2[8];
+                        tmem_ld16(tbase + lrow + cU + (g & 1) * C::NU, x);
+                        tmem_ld8(tbase + lrow + cU + (g & 1) * C::NU + 16, x2);
+                        tmem_wait_ld();
+#pragma unroll
+                        for (int q = 0; q < C::PP; ++q) {
+                            const int i = H * C::PP + q;
+                            u[q] = (__uint_as_float(x[i]) + __uint_as_float(x[8 + i])) + __uint_as_float(x2[i]) +
+                                   sbias[i];
+                        }
+                    }
+                    search<C::PP>(sTe, u, j);
+#pragma unroll
+                    for (int q = 0; q < C::PP; ++q) {
+                        float al[8], y[8];
+                        channel_eval(sAB, j[q], u[q], al, y);
+                        *reinterpret_cast<uint4 *>(phit + sw128_chunk(r, H * C::PP + q)) =
+                            valid ? pack8(y) : make_uint4(0, 0, 0, 0);
+                    }
+                    if (!valid && H == 0) zero_row(kt, r);
+                    fence_proxy_async_smem();
+                    tc_fence_before();
+                    mbar_arrive(phiready + (g & 1));
+                    // dphi(k) = dS v + dz  ->  dU, histogram
+                    wait_or_fail(fready + (g & 1), (g >> 1) & 1, failed, status);
+                    tc_fence_after();
+                    const uint32_t fcol = tbase + lrow + cF + (g & 1) * 128;
+                    float dU[C::PP];
+#pragma unroll
+                    for (int q = 0; q < C::PP; ++q) {
+                        const int i = H * C::PP + q;
+                        float al[8], y[8], dphi[8];
+                        channel_eval(sAB, j[q], u[q], al, y);
+                        uint32_t ph[8], pl[8];
+                        tmem_ld8(fcol + 8 * i, ph);
+                        tmem_ld8(fcol + C::D + 8 * i, pl);
+                        tmem_wait_ld();
+#pragma unroll
+                        for (int l = 0; l < 8; ++l) dphi[l] = __uint_as_float(ph[l]) + __uint_as_float(pl[l]) + sdz[8 * i + l];
+                        dU[q] = valid ? channel_backward(hist, j[q], u[q], al, y, dphi) : 0.0f;
+                        db_acc[q] += dU[q];
+                    }
+                    if (g >= 1) wait_or_fail(gfree, (g - 1) & 1, failed, status);
+                    {
+                        __nv_bfloat16 hi[C::PP], lo[C::PP];
+#pragma unroll
+                        for (int q = 0; q < C::PP; ++q) split_bf16(dU[q], hi[q], lo[q]);
+                        uint2 vh, vl;
+                        vh.x = (uint32_t)__bfloat16_as_ushort(hi[0]) | ((uint32_t)__bfloat16_as_ushort(hi[1]) << 16);
+                        vh.y = (uint32_t)__bfloat16_as_ushort(hi[2]) | ((uint32_t)__bfloat16_as_ushort(hi[3]) << 16);
+                        vl.x = (uint32_t)__bfloat16_as_ushort(lo[0]) | ((uint32_t)__bfloat16_as_ushort(lo[1]) << 16);
+                        vl.y = (uint32_t)__bfloat16_as_ushort(lo[2]) | ((uint32_t)__bfloat16_as_ushort(lo[3]) << 16);
+                        *reinterpret_cast<uint2 *>(Gt + sw128_chunk(r, 0) + H * 8) = vh;
+                        *reinterpret_cast<uint2 *>(Gt + sw128_chunk(r, 1) + H * 8) = vl;
+                        *reinterpret_cast<uint2 *>(Gt + sw128_chunk(r, 2) + H * 8) = vh;
+                    }
+                    fence_proxy_async_smem();
+                    tc_fence_before();
+                    mbar_arrive(gready + (g & 1));
+                    // dV = hi + lo
+                    wait_or_fail(dvready + (g & 1), (g >> 1) & 1, failed, status);
+                    tc_fence_after();
+                    {
+                        uint32_t xh[16], xl[16];
+                        const uint32_t vcol = tbase + lrow + cV + (g & 1) * 64 + H * 16;
+                        tmem_ld16(vcol, xh);
+                        tmem_ld16(vcol + C::DV, xl);
+                        tmem_wait_ld();
+                        tc_fence_before();
+                        mbar_arrive(dvfree + (g & 1));
+                        if (valid) {
+                            float f0[8], f1[8];
+#pragma unroll
+                            for (int c = 0; c < 8; ++c) {
+                                f0[c] = __uint_as_float(xh[c]) + __uint_as_float(xl[c]);
+                                f1[c] = __uint_as_float(xh[8 + c]) + __uint_as_float(xl[8 + c]);
+                            }
+                            uint4 *dst = reinterpret_cast<uint4 *>(dV + (size_t)(row0 + r) * C::DV + H * 16);
+                            dst[0] = pack8(f0);
+                            dst[1] = pack8(f1);
+                        }
+                    }
+                    // dK
+                    wait_or_fail(dkready, g & 1, failed, status);
+                    tc_fence_after();
+                    {
+                        uint32_t x[16];
+                        tmem_ld16(tbase + lrow + cK + H * 16, x);
+                        tmem_wait_ld();
+                        tc_fence_before();
+                        mbar_arrive(dkfree);
+                        if (valid) {
+                            float f0[8], f1[8];
+#pragma unroll
+                            for (int c = 0; c < 8; ++c) { f0[c] = __uint_as_float(x[c]); f1[c] = __uint_as_float(x[8 + c]); }
+                            uint4 *dst = reinterpret_cast<uint4 *>(dK + (size_t)(row0 + r) * C::d + H * 16);
+                            dst[0] = pack8(f0);
+                            dst[1] = pack8(f1);
+                        }
+                    }
+                }
+            }
+            i0 = i1;
+        }
+#pragma unroll
+        for (int q = 0; q < C::PP; ++q) {
+            float v = db_acc[q];
+#pragma unroll
+            for (int o = 16; o > 0; o >>= 1) v += __shfl_xor_sync(0xffffffffu, v, o);
+            if (lane == 0) atomicAdd(sdb + H * C::PP + q, v);
+        }
+        // dW^T accumulator (M = 64: input column cd in lane 32*(cd/16) + cd%16)
+        if (warp < 4) {
+            const int T = block_tiles(a, it);
+            if (T > 0) wait_or_fail(wdone, 0, failed, status);
+            tc_fence_after();
+            uint32_t x[16];
+            tmem_ld16(tbase + ((uint32_t)(warp << 5) << 16) + cW, x);
+            tmem_wait_ld();
+            const int cd = (warp << 4) | lane;
+            if (T > 0 && lane < 16 && cd < C::d)
+#pragma unroll
+                for (int i = 0; i < C::MP; ++i) sdW[i * C::d + cd] = __uint_as_float(x[i]) + __uint_as_float(x[C::MP + i]);
+        }
+    }
+    tc_fence_before();
+    __syncthreads();
+    store_param_partial<C>(a, sdW, sdb, hist, a.gpart + (size_t)(gridDim.x + blockIdx.x) * a.gsize);
+    __syncthreads();
+    if (warp == 0) tmem_dealloc(tbase, 512);
+}
+
+}  // namespace
+}  // namespace luna
+
+namespace luna {
+namespace {
+
+typedef CUresult (*EncodeTiledFnB)(CUtensorMap *, CUtensorMapDataType, cuuint32_t, void *, const cuuint64_t *,
+                                   const cuuint64_t *, const cuuint32_t *, const cuuint32_t *, CUtensorMapInterleave,
+                                   CUtensorMapSwizzle, CUtensorMapL2promotion, CUtensorMapFloatOOBfill);
+
+}  // namespace
+
+bool tc_make_map(CUtensorMap *m, const void *base, int width, int n, int BH);
+int tc_sm_count();
+AttnArgs tc_work_items(const AttnArgs &a);
+
+namespace {
+
+template <class C>
+cudaError_t bwd_tc(const AttnArgs &a0, bool have_stats, cudaStream_t s) {
+    const AttnArgs a = tc_work_items(a0);
+    const int items = a.B * a.H * a.nsplit;
+    const int grid = items < tc_sm_count() ? items : tc_sm_count();
+    cudaError_t e;
+    if (!have_stats && (e = launch_tc_stats(a0, s)) != cudaSuccess) return e;
+    CUtensorMap mQ, mdO, mK, mV;
+    if (!tc_make_map(&mQ, a.Q, a.d, a.n, a.B * a.H) || !tc_make_map(&mdO, a.dO, a.dv, a.n, a.B * a.H) ||
+        !tc_make_map(&mK, a.K, a.d, a.n, a.B * a.H) || !tc_make_map(&mV, a.V, a.dv, a.n, a.B * a.H))
+        return cudaErrorInvalidValue;
+    if ((e = cudaFuncSetAttribute(k_tc_bwd_query<C>, cudaFuncAttributeMaxDynamicSharedMemorySize, C::SMEM_Q)) !=
+        cudaSuccess)
+        return e;
+    if ((e = cudaFuncSetAttribute(k_tc_bwd_key<C>, cudaFuncAttributeMaxDynamicSharedMemorySize, C::SMEM_K)) !=
+        cudaSuccess)
+        return e;
+    int *st = reinterpret_cast<int *>(reinterpret_cast<char *>(a.counters) - 256);
+    LUNA_LAUNCH("tc_bwd_query", k_tc_bwd_query<C>, grid, kBThreads, C::SMEM_Q, s, mQ, mdO, a, st);
+    if ((e = cudaGetLastError()) != cudaSuccess) return e;
+    LUNA_LAUNCH("tc_bwd_key", k_tc_bwd_key<C>, grid, kBThreads, C::SMEM_K, s, mK, mV, a, st);
+    if ((e = cudaGetLastError()) != cudaSuccess) return e;
+    return launch_grad_reduce(a, 2 * grid, s);
+}
+
+}  // namespace
+
+bool tc_bwd_supported(const luna_attn_desc &ad, const TableLayout &lay) {
+    return ad.io == LUNA_BF16 && !ad.causal && lay.L == 8 && lay.P <= 512 && ad.d == 32 && ad.dv == 32 && lay.M == 8;
+}
+
+// One parameter-gradient partial per block and side: the persistent grid must fit the
+// partial slots the workspace holds (two per generic backward split).
+bool tc_bwd_fits(const AttnArgs &a0) {
+    const AttnArgs a = tc_work_items(a0);
+    const int items = a.B * a.H * a.nsplit;
+    const int grid = items < tc_sm_count() ? items : tc_sm_count();
+    return grid <= a0.B * a0.H * a0.nsplit_b;
+}
+
+cudaError_t launch_tc_bwd_kernels(const AttnArgs &a, bool have_stats, cudaStream_t s) {
+    return bwd_tc<B32>(a, have_stats, s);
+}
+
+}  // namespace luna

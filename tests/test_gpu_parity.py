@@ -157,6 +157,56 @@ def test_backward(c):
                 assert np.all(g[k][b, :, ln:] == 0)
 
 
+def _check_bwd(case, g, ref, tol):
+    okq, okk = case.smooth_rows("Q"), case.smooth_rows("K")
+    assert okq.mean() > 0.9 and okk.mean() > 0.9
+    assert relerr(g["dQ"][okq], ref["dQ"][okq]) < tol
+    assert relerr(g["dK"][okk], ref["dK"][okk]) < tol
+    assert relerr(g["dV"], ref["dV"]) < tol
+    for k in ("dW", "db", "dw1", "db1", "dw2", "db2"):
+        assert relerr(g[k], ref[k]) < tol, k
+
+
+@pytest.mark.parametrize("tiles", ["1", "3", "5"])
+def test_backward_tensor_core_tile_loops(tiles, monkeypatch):
+    """bf16 backward through the tensor-core kernels (d = 32, M = 8) with 1, 3
+    and 5 tiles of 128 rows per work item: per-head runs that span several
+    blocks and blocks that span several heads, the staging rings wrapping
+    around, ragged last tiles and items with no valid row."""
+    monkeypatch.setenv("LUNA_TC_TILES_PER_SPLIT", tiles)
+    case = Case(2, 3, 1100, 32, 8, 8, "bf16", False, seed=43, qkv_scale=1.0 / math.sqrt(32),
+                lengths=[1100, 290], with_grad=True)
+    lu = case.luna()
+    case.run_fwd(lu)
+    g = {k: to_host(v) for k, v in case.run_bwd(lu).items()}
+    _check_bwd(case, g, case.oracle_bwd(), TOL["bf16"])
+    for k in ("dQ", "dK", "dV"):
+        assert np.all(g[k][1, :, 290:] == 0)
+
+
+def test_backward_tensor_core_hidden_32():
+    """Tensor-core backward with a shorter kink list (hidden = 32: 256 kinks,
+    257 intervals), so the histogram is smaller than its maximum size."""
+    case = Case(1, 2, 400, 32, 8, 8, "bf16", False, seed=47, qkv_scale=1.0 / math.sqrt(32),
+                with_grad=True, hidden=32)
+    lu = case.luna()
+    case.run_fwd(lu)
+    g = {k: to_host(v) for k, v in case.run_bwd(lu).items()}
+    _check_bwd(case, g, case.oracle_bwd(), TOL["bf16"])
+
+
+def test_backward_tensor_core_repeat_bitwise():
+    """dQ, dK and dV of the tensor-core backward do not depend on the order of
+    floating-point atomics, so repeated runs agree bit for bit."""
+    case = Case(2, 2, 700, 32, 8, 8, "bf16", False, seed=53, with_grad=True)
+    lu = case.luna()
+    case.run_fwd(lu)
+    g1 = {k: to_host(v) for k, v in case.run_bwd(lu).items()}
+    g2 = {k: to_host(v) for k, v in case.run_bwd(lu).items()}
+    for k in ("dQ", "dK", "dV"):
+        assert np.array_equal(g1[k], g2[k]), k
+
+
 @pytest.mark.parametrize("causal", [False, True])
 def test_backward_with_and_without_saved_state(causal):
     case = Case(2, 2, 200, 32, 8, 8, "f32", causal, seed=13, with_grad=True, lengths=[200, 150])
