@@ -89,6 +89,10 @@ def kernel_bytes(w, lengths, kernel: str) -> float:
         "bwd_key": valid * (rd + rv) + total * (rd + rv) + stats,
         "causal_out": valid * (2 * rd + rv) + total * rv,
     }
+    # the tensor-core kernels move the same tensors as their generic counterparts
+    for tc, generic in (("tc_keys", "keystats"), ("tc_query", "query"), ("tc_bwd_query", "bwd_query"),
+                        ("tc_bwd_key", "bwd_key")):
+        table[tc] = table[generic]
     return float(table.get(kernel, 0.0))
 
 

@@ -322,47 +322,104 @@ __global__ void __launch_bounds__(kThreads) k_bwd_key(AttnArgs a) {
 //     dw2 = (w1 G1 + b1 G0)/sqrt(M), dw1 = w2 G1/sqrt(M), db1 = w2 G0/sqrt(M),
 //     db2 = sum_j m0 / sqrt(M).
 
-__global__ void __launch_bounds__(kThreads) k_grad_sum(const float *gpart, int nparts, int gsize, float *out) {
-    for (int e = blockIdx.x * blockDim.x + threadIdx.x; e < gsize; e += gridDim.x * blockDim.x) {
-        float s = 0.0f;
-        for (int p = 0; p < nparts; ++p) s += gpart[(size_t)p * gsize + e];
-        out[e] = s;
+// Sum of the per-block parameter-gradient partials, in the fixed order p = 0..nparts-1
+// per element: 64 elements per block, each summed by 4 threads over consecutive
+// quarters of the partials (8 loads in flight), then combined in quarter order.
+constexpr int kSumElems = 64, kSumSplit = 4;
+__global__ void __launch_bounds__(kSumElems * kSumSplit) k_grad_sum(const float *gpart, int nparts, int gsize,
+                                                                    float *out) {
+    __shared__ float part[kSumSplit][kSumElems];
+    const int el = threadIdx.x % kSumElems, q = threadIdx.x / kSumElems;
+    const int e = blockIdx.x * kSumElems + el;
+    const int p0 = (int)((long long)q * nparts / kSumSplit), p1 = (int)((long long)(q + 1) * nparts / kSumSplit);
+    float s = 0.0f;
+    if (e < gsize) {
+        int p = p0;
+        for (; p + 8 <= p1; p += 8) {
+            float v[8];
+#pragma unroll
+            for (int k = 0; k < 8; ++k) v[k] = __ldcg(gpart + (size_t)(p + k) * gsize + e);
+#pragma unroll
+            for (int k = 0; k < 8; ++k) s += v[k];
+        }
+        for (; p < p1; ++p) s += __ldcg(gpart + (size_t)p * gsize + e);
+    }
+    part[q][el] = s;
+    __syncthreads();
+    if (q == 0 && e < gsize) {
+        float t = part[0][el];
+#pragma unroll
+        for (int k = 1; k < kSumSplit; ++k) t += part[k][el];
+        out[e] = t;
     }
 }
 
-__global__ void __launch_bounds__(kThreads) k_mlp_grads(TableLayout lay, const char *table, const float *gsum,
-                                                        luna_phi_grads grads) {
+// Inclusive scan of x[0..n) into y (forward: prefix sums; backward: suffix sums)
+// by one warp, in a fixed order: lane c sums a contiguous chunk, the chunk totals
+// are scanned across lanes, then every lane writes its chunk.
+__device__ void warp_scan(const float *x, float *y, int n, bool backward) {
+    const int lane = threadIdx.x & 31;
+    const int chunk = (n + 31) / 32;
+    const int b = lane * chunk, e = min(n, b + chunk);
+    auto at = [&](int i) { return backward ? n - 1 - i : i; };
+    float t = 0.0f;
+    for (int i = b; i < e; ++i) t += x[at(i)];
+    float incl = t;
+#pragma unroll
+    for (int o = 1; o < 32; o <<= 1) {
+        const float v = __shfl_up_sync(0xffffffffu, incl, o);
+        if (lane >= o) incl += v;
+    }
+    float run = incl - t;  // exclusive prefix of this chunk
+    for (int i = b; i < e; ++i) {
+        run += x[at(i)];
+        y[at(i)] = run;
+    }
+}
+
+// Block l < L: hidden units of channel l from prefix and suffix sums of the
+// channel's interval histogram.  Block L: dW and db.
+__global__ void __launch_bounds__(128) k_mlp_grads(TableLayout lay, const char *table, const float *gsum,
+                                                   luna_phi_grads grads) {
+    __shared__ float h[2][kMaxUnits + 1], pre[2][kMaxUnits + 1], suf[2][kMaxUnits + 1];
     const int Md = lay.M * lay.d, L = lay.L, hid = lay.hid, nint = lay.nint;
+    const float scale = 1.0f / sqrtf((float)lay.M);
+    if ((int)blockIdx.x == L) {
+        for (int e = threadIdx.x; e < Md; e += blockDim.x) grads.dW[e] = gsum[e];
+        for (int e = threadIdx.x; e < lay.M; e += blockDim.x) grads.db[e] = gsum[Md + e];
+        return;
+    }
+    const int l = blockIdx.x;
     const float *hist = gsum + Md + lay.M;
+    for (int j = threadIdx.x; j < nint; j += blockDim.x) {
+        h[0][j] = hist[(j * L + l) * 2];
+        h[1][j] = hist[(j * L + l) * 2 + 1];
+    }
+    __syncthreads();
+    const int warp = threadIdx.x >> 5;  // warps 0, 1: prefix of m0, m1; warps 2, 3: suffix
+    warp_scan(h[warp & 1], (warp < 2 ? pre : suf)[warp & 1], nint, warp >= 2);
+    __syncthreads();
     const int *rank = reinterpret_cast<const int *>(table + lay.off_rank);
     const int *utype = reinterpret_cast<const int *>(table + lay.off_utype);
     const float *w1 = reinterpret_cast<const float *>(table + lay.off_w1);
     const float *b1 = reinterpret_cast<const float *>(table + lay.off_b1);
     const float *w2 = reinterpret_cast<const float *>(table + lay.off_w2);
-    const float scale = 1.0f / sqrtf((float)lay.M);
-    for (int e = threadIdx.x; e < Md; e += blockDim.x) grads.dW[e] = gsum[e];
-    for (int e = threadIdx.x; e < lay.M; e += blockDim.x) grads.db[e] = gsum[Md + e];
-    for (int u = threadIdx.x; u < lay.P; u += blockDim.x) {
-        const int l = u / hid;
+    for (int k = threadIdx.x; k < hid; k += blockDim.x) {
+        const int u = l * hid + k;
         const int r = rank[u];
-        const bool up = utype[u] > 0;
-        float G0 = 0.0f, G1 = 0.0f;
-        for (int j = 0; j < nint; ++j) {
-            const bool on = up ? (r < j) : (r >= j);
-            if (on) {
-                G0 += hist[(j * L + l) * 2];
-                G1 += hist[(j * L + l) * 2 + 1];
-            }
+        float G0, G1;
+        if (utype[u] > 0) {  // active on intervals j > r
+            G0 = r + 1 < nint ? suf[0][r + 1] : 0.0f;
+            G1 = r + 1 < nint ? suf[1][r + 1] : 0.0f;
+        } else {             // active on intervals j <= r
+            G0 = pre[0][r];
+            G1 = pre[1][r];
         }
         grads.dw2[u] = (w1[u] * G1 + b1[u] * G0) * scale;
         grads.dw1[u] = w2[u] * G1 * scale;
         grads.db1[u] = w2[u] * G0 * scale;
     }
-    for (int l = threadIdx.x; l < L; l += blockDim.x) {
-        float t = 0.0f;
-        for (int j = 0; j < nint; ++j) t += hist[(j * L + l) * 2];
-        grads.db2[l] = t * scale;
-    }
+    if (threadIdx.x == 0) grads.db2[l] = pre[0][nint - 1] * scale;
 }
 
 // ---------------------------------------------------------------------------
@@ -438,11 +495,11 @@ size_t simt_max_smem(const AttnArgs &a) {
 }
 
 cudaError_t launch_grad_reduce(const AttnArgs &a, int nparts, cudaStream_t s) {
-    const int blocks = (a.gsize + kThreads - 1) / kThreads;
-    LUNA_LAUNCH("grad_sum", k_grad_sum, blocks, kThreads, 0, s, a.gpart, nparts, a.gsize, a.hist);
+    LUNA_LAUNCH("grad_sum", k_grad_sum, (a.gsize + kSumElems - 1) / kSumElems, kSumElems * kSumSplit, 0, s, a.gpart,
+                nparts, a.gsize, a.hist);
     cudaError_t e = cudaGetLastError();
     if (e != cudaSuccess) return e;
-    LUNA_LAUNCH("mlp_grads", k_mlp_grads, 1, kThreads, 0, s, a.lay, a.table, a.hist, a.grads);
+    LUNA_LAUNCH("mlp_grads", k_mlp_grads, a.lay.L + 1, 128, 0, s, a.lay, a.table, a.hist, a.grads);
     return cudaGetLastError();
 }
 

@@ -145,6 +145,11 @@ __device__ __forceinline__ uint4 pack8(const float (&y)[8]) {
                       pack_bf16x2(y[6], y[7]));
 }
 
+// Interval histogram in shared memory: hist[c * 8 * kNint + l * kNint + j] holds,
+// for channel l and interval j, the sum of g (c = 0) and of g * u (c = 1); lanes
+// with different intervals fall into different banks.
+__device__ __forceinline__ int hist_at(int c, int l, int j) { return (c * 8 + l) * kNint + j; }
+
 // Backward through the channel functions for one projection value: g = dLoss/dphi on
 // the active outputs; adds g and g*u to the interval histogram, returns dLoss/du.
 __device__ __forceinline__ float channel_backward(float *hist, int j, float u, const float (&al)[8],
@@ -154,8 +159,8 @@ __device__ __forceinline__ float channel_backward(float *hist, int j, float u, c
     for (int l = 0; l < 8; ++l) {
         if (y[l] > 0.0f && dphi[l] != 0.0f) {
             du = fmaf(dphi[l], al[l], du);
-            atomicAdd(hist + (j * 8 + l) * 2, dphi[l]);
-            atomicAdd(hist + (j * 8 + l) * 2 + 1, dphi[l] * u);
+            atomicAdd(hist + hist_at(0, l, j), dphi[l]);
+            atomicAdd(hist + hist_at(1, l, j), dphi[l] * u);
         }
     }
     return du;
@@ -169,13 +174,14 @@ __device__ __forceinline__ void zero_row(uint8_t *tile, int r) {
 }
 
 // Writes the per-block parameter-gradient partial: dW (M x d) from smem, db
-// (block sum of per-thread values), the interval histogram.
+// (block sum of per-thread values), the interval histogram (as [interval][channel][g, g*u]).
 template <class C>
 __device__ void store_param_partial(const AttnArgs &a, const float *sdW, float *sdb, const float *hist, float *gp) {
     const int Md = C::MP * a.d;
     for (int e = threadIdx.x; e < Md; e += blockDim.x) gp[e] = sdW[e];
     for (int e = threadIdx.x; e < C::MP; e += blockDim.x) gp[Md + e] = sdb[e];
-    for (int e = threadIdx.x; e < a.lay.nint * 16; e += blockDim.x) gp[Md + C::MP + e] = hist[e];
+    for (int e = threadIdx.x; e < a.lay.nint * 16; e += blockDim.x)
+        gp[Md + C::MP + e] = hist[hist_at(e & 1, (e >> 1) & 7, e >> 4)];
 }
 
 // ---------------------------------------------------------------------------
@@ -199,7 +205,7 @@ __global__ void __launch_bounds__(kBThreads, 1)
     float *sbias = sAB + kNint * 16;
     float *sz = sbias + 32;
     float *sred = sz + C::D;              // [2 tiles][den, dot][2 halves][128 rows]
-    float *hist = sred + 1024;            // [nint][8][2]
+    float *hist = sred + 1024;            // [g, g*u][8][kNint]
     float *sdW = hist + kNint * 16;       // [M][d]
     float *sdb = sdW + C::MP * C::d;      // [M] (padded to 16)
     uint64_t *bars = reinterpret_cast<uint64_t *>(sdb + 16);
@@ -394,16 +400,17 @@ __global__ void __launch_bounds__(kBThreads, 1)
                     float u[C::PP];
                     int j[C::PP];
                     {
-                        uint32_t x[16], x2[8];
-                        tmem_ld16(tbase + lrow + cU + (g & 1) * C::NU, x);
-                        tmem_ld8(tbase + lrow + cU + (g & 1) * C::NU + 16, x2);
+                        // this thread's PP projections: columns H*PP.. of the hi, mid and lo parts
+                        uint32_t xh[4], xm[4], xl[4];
+                        const uint32_t ucol = tbase + lrow + cU + (g & 1) * C::NU + H * C::PP;
+                        tmem_ld4(ucol, xh);
+                        tmem_ld4(ucol + C::MP, xm);
+                        tmem_ld4(ucol + 2 * C::MP, xl);
                         tmem_wait_ld();
 #pragma unroll
-                        for (int q = 0; q < C::PP; ++q) {
-                            const int i = H * C::PP + q;
-                            u[q] = (__uint_as_float(x[i]) + __uint_as_float(x[8 + i])) + __uint_as_float(x2[i]) +
-                                   sbias[i];
-                        }
+                        for (int q = 0; q < C::PP; ++q)
+                            u[q] = (__uint_as_float(xh[q]) + __uint_as_float(xm[q])) + __uint_as_float(xl[q]) +
+                                   sbias[H * C::PP + q];
                     }
                     search<C::PP>(sTe, u, j);
                     if (!valid && H == 0) zero_row(qt, r);  // padded rows: no contribution to dW
@@ -828,16 +835,17 @@ __global__ void __launch_bounds__(kBThreads, 1)
                     float u[C::PP];
                     int j[C::PP];
                     {
-                        uint32_t x[16], x2[8];
-                        tmem_ld16(tbase + lrow + cU + (g & 1) * C::NU, x);
-                        tmem_ld8(tbase + lrow + cU + (g & 1) * C::NU + 16, x2);
+                        // this thread's PP projections: columns H*PP.. of the hi, mid and lo parts
+                        uint32_t xh[4], xm[4], xl[4];
+                        const uint32_t ucol = tbase + lrow + cU + (g & 1) * C::NU + H * C::PP;
+                        tmem_ld4(ucol, xh);
+                        tmem_ld4(ucol + C::MP, xm);
+                        tmem_ld4(ucol + 2 * C::MP, xl);
                         tmem_wait_ld();
 #pragma unroll
-                        for (int q = 0; q < C::PP; ++q) {
-                            const int i = H * C::PP + q;
-                            u[q] = (__uint_as_float(x[i]) + __uint_as_float(x[8 + i])) + __uint_as_float(x2[i]) +
-                                   sbias[i];
-                        }
+                        for (int q = 0; q < C::PP; ++q)
+                            u[q] = (__uint_as_float(xh[q]) + __uint_as_float(xm[q])) + __uint_as_float(xl[q]) +
+                                   sbias[H * C::PP + q];
                     }
                     search<C::PP>(sTe, u, j);
 #pragma unroll

@@ -20,8 +20,10 @@ constexpr int kPpad = 512;   // merged kink list (L * hidden <= 512, L = 8)
 constexpr int kNint = 513;   // intervals
 constexpr uint32_t kTableBytes = (kEytzinger + kNint * 16 + 32) * 4;
 
+// First 1024-byte boundary at or after p (a shared-memory array), formed by
+// pointer arithmetic on p so that the compiler still sees a shared address.
 __device__ __forceinline__ uint8_t *align1024(uint8_t *p) {
-    return reinterpret_cast<uint8_t *>((reinterpret_cast<uintptr_t>(p) + 1023) & ~uintptr_t(1023));
+    return p + ((1024u - (smem_u32(p) & 1023u)) & 1023u);
 }
 
 __device__ __forceinline__ uint32_t pack_bf16x2(float a, float b) {
