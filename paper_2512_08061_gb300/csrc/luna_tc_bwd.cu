@@ -34,29 +34,33 @@ using namespace sm100;
 using namespace simt;
 using namespace tcdev;
 
-constexpr int kBWorkers = 256;           // 8 warps, two threads per row
-constexpr int kBTma = 8, kBMma = 9;
+constexpr int kBWorkers = 512;           // 16 warps, four threads per row
+constexpr int kBRowThreads = kBWorkers / 128;
+constexpr int kBTma = 16, kBMma = 17;
 constexpr int kBThreads = kBWorkers + 64;
 constexpr uint32_t kBarBytes = 256;      // mbarriers, TMEM address, flag (each kernel below uses <= 26 slots)
 
 // d = dv = 32, D = 64 (M = 8 projections, L = 8 channels)
 struct B32 {
-    static constexpr int d = 32, DX = 64, DV = 32, MP = 8, D = 64, NU = 32, PP = 4;
+    static constexpr int d = 32, DX = 64, DV = 32, MP = 8, D = 64, NU = 32, PP = MP / kBRowThreads;
     static constexpr uint32_t TILE = 16384;  // 128 rows x 128 B
     static constexpr int NKD = d / 16;       // k-steps over d
     static constexpr int NKV = DV / 16;      // k-steps over dv
-    static constexpr uint32_t WOP = NU * 128;          // [W_hi; W_mid; W_lo; 0] (NU rows x 64)
-    static constexpr uint32_t WXP = d * 128;           // [W_hi; W_hi; W_lo; 0] per output column
+    // NU rows x 128 B: columns 0..31 hold [W_hi; W_mid; W_lo; 0] (the projection operand, K = d), columns
+    // 32..63 of row n the dX operand [W_hi; W_hi; W_lo; 0] of output column n (K = 32).
+    static constexpr uint32_t WOP = NU * 128;
+    static_assert(NU == d && d == 32, "dX operand shares the rows of the projection operand");
     static constexpr uint32_t SOP2 = 2 * D * 128;      // [S_hi; S_lo] rows per feature, K = dv
     static constexpr uint32_t SOP = 2 * DV * 128;      // [S_hi; S_lo]^T rows per value column, K = D
     static constexpr uint32_t HIST = kNint * 16 * 4;
     // query side: stage = [phi/den (hi, lo interleaved by 16 features) x 2 tiles | Q tile]
     static constexpr int NSQ = 2, NOQ = 2;
-    static constexpr uint32_t SMEM_Q = NSQ * 3 * TILE + NOQ * TILE + WOP + WXP + SOP2 + kTableBytes + D * 4 +
-                                       2 * 2 * 2 * 128 * 4 + HIST + MP * d * 4 + 64 + kBarBytes + 1024;
+    static constexpr uint32_t SRED = 2 * 2 * kBRowThreads * 128;  // floats: [tile parity][den, dot][part][row]
+    static constexpr uint32_t SMEM_Q = NSQ * 3 * TILE + NOQ * TILE + WOP + SOP2 + kTableBytes + D * 4 + SRED * 4 +
+                                       HIST + MP * d * 4 + 64 + kBarBytes + 1024;
     // key side
     static constexpr int NSK = 2, NVK = 2;
-    static constexpr uint32_t SMEM_K = NSK * 2 * TILE + NVK * TILE + TILE + WOP + WXP + SOP + SOP2 + kTableBytes +
+    static constexpr uint32_t SMEM_K = NSK * 2 * TILE + NVK * TILE + TILE + WOP + SOP + SOP2 + kTableBytes +
                                        D * 4 + HIST + MP * d * 4 + 64 + kBarBytes + 1024;
     static_assert(SMEM_Q <= kSmemLimit && SMEM_K <= kSmemLimit, "shared memory budget");
 };
@@ -69,19 +73,21 @@ __device__ __forceinline__ void proj_mma(uint32_t tmem_u, uint64_t dx, uint64_t 
     for (int k = 0; k < C::NKD; ++k) mma_bf16_ss(tmem_u, dadd(dx, 32 * k), dadd(dw, 32 * k), idesc, k != 0);
 }
 
-// [W_hi; W_hi; W_lo; 0] as the K-major B operand of dX = [dU_hi | dU_lo | dU_hi | 0] W: row n = output column.
+// [W_hi; W_hi; W_lo; 0] as the K-major B operand of dX = [dU_hi | dU_lo | dU_hi | 0] W: row n = output
+// column, K = 32, written into columns 32..63 of the rows of the projection operand (which reads only
+// columns 0..d-1).  Runs after stage_phi_table, separated by a block barrier.
 template <class C>
-__device__ void stage_wx(const AttnArgs &a, uint8_t *Wx) {
+__device__ void stage_wx(const AttnArgs &a, uint8_t *Wop) {
     const float *W = reinterpret_cast<const float *>(a.table + a.lay.off_W);
-    for (int e = threadIdx.x; e < C::d * 64; e += blockDim.x) {
-        const int n = e / 64, k = e % 64;
+    for (int e = threadIdx.x; e < C::d * 32; e += blockDim.x) {
+        const int n = e / 32, k = e % 32;
         float v = 0.0f;
         if (k < 3 * C::MP) {
             __nv_bfloat16 hi, lo;
             split_bf16(W[(k % C::MP) * a.d + n], hi, lo);
             v = (k < 2 * C::MP) ? __bfloat162float(hi) : __bfloat162float(lo);
         }
-        *reinterpret_cast<__nv_bfloat16 *>(Wx + sw128_chunk(n, k / 8) + (k % 8) * 2) = __float2bfloat16_rn(v);
+        *reinterpret_cast<__nv_bfloat16 *>(Wop + sw128_chunk(n, 4 + k / 8) + (k % 8) * 2) = __float2bfloat16_rn(v);
     }
 }
 
@@ -138,6 +144,15 @@ __device__ __forceinline__ void channel_eval(const float *sAB, int j, float u, f
         y[2 * k] = fmaxf(fmaf(v.x, u, v.y), 0.0f);
         y[2 * k + 1] = fmaxf(fmaf(v.z, u, v.w), 0.0f);
     }
+}
+
+// dU of two projections split into bf16 hi and lo, each pair packed into 32 bits.
+__device__ __forceinline__ void dU_pack(const float (&dU)[2], uint32_t &vh, uint32_t &vl) {
+    __nv_bfloat16 h0, l0, h1, l1;
+    split_bf16(dU[0], h0, l0);
+    split_bf16(dU[1], h1, l1);
+    vh = (uint32_t)__bfloat16_as_ushort(h0) | ((uint32_t)__bfloat16_as_ushort(h1) << 16);
+    vl = (uint32_t)__bfloat16_as_ushort(l0) | ((uint32_t)__bfloat16_as_ushort(l1) << 16);
 }
 
 __device__ __forceinline__ uint4 pack8(const float (&y)[8]) {
@@ -197,15 +212,14 @@ __global__ void __launch_bounds__(kBThreads, 1)
     constexpr uint32_t T16 = C::TILE;
     uint8_t *Sb = sm;                    // [NS] x (phi/den tiles x 2, Q tile)
     uint8_t *Ob = Sb + NS * 3 * T16;     // [NO] dO tile, completed in place into G = [dO | dU | -(dO.O)]
-    uint8_t *Wop = Ob + NO * T16;
-    uint8_t *Wx = Wop + C::WOP;
-    uint8_t *Sop2 = Wx + C::WXP;
+    uint8_t *Wop = Ob + NO * T16;         // projection and dX operands
+    uint8_t *Sop2 = Wop + C::WOP;
     float *sTe = reinterpret_cast<float *>(Sop2 + C::SOP2);
     float *sAB = sTe + kEytzinger;
     float *sbias = sAB + kNint * 16;
     float *sz = sbias + 32;
-    float *sred = sz + C::D;              // [2 tiles][den, dot][2 halves][128 rows]
-    float *hist = sred + 1024;            // [g, g*u][8][kNint]
+    float *sred = sz + C::D;              // [2 tiles][den, dot][kBRowThreads parts][128 rows]
+    float *hist = sred + C::SRED;         // [g, g*u][8][kNint]
     float *sdW = hist + kNint * 16;       // [M][d]
     float *sdb = sdW + C::MP * C::d;      // [M] (padded to 16)
     uint64_t *bars = reinterpret_cast<uint64_t *>(sdb + 16);
@@ -246,7 +260,8 @@ __global__ void __launch_bounds__(kBThreads, 1)
     }
     if (warp == 0) { tmem_alloc(tslot, 512); tmem_relinquish(); }
     stage_phi_table<C>(a, sTe, sAB, sbias, Wop);
-    stage_wx<C>(a, Wx);
+    __syncthreads();
+    stage_wx<C>(a, Wop);
     for (int e = tid; e < kNint * 16; e += blockDim.x) hist[e] = 0.0f;
     for (int e = tid; e < C::MP * C::d + 16; e += blockDim.x) sdW[e] = 0.0f;
     // padded rows of every item produce zero gradients
@@ -289,7 +304,7 @@ __global__ void __launch_bounds__(kBThreads, 1)
             const uint64_t dS0 = sdesc(smem_u32(Sb), 16384, 1024, kSwizzle128);
             const uint64_t dO0 = sdesc(smem_u32(Ob), 16384, 1024, kSwizzle128);
             const uint64_t dWo = sdesc(smem_u32(Wop), 16, 1024, kSwizzle128);
-            const uint64_t dWx = sdesc(smem_u32(Wx), 16, 1024, kSwizzle128);
+            const uint64_t dWx = dadd(dWo, 64);  // columns 32..63 of the same rows
             const uint64_t dSp = sdesc(smem_u32(Sop2), 16, 1024, kSwizzle128);
             bool failed = false;
             auto proj = [&](int g) {
@@ -364,7 +379,7 @@ __global__ void __launch_bounds__(kBThreads, 1)
             else mbar_arrive(wdone);
         }
     } else {
-        // workers
+        // workers: thread (H, r) handles projections H*PP .. H*PP+PP-1 of tile row r
         const int H = warp >> 2, r = ((warp & 3) << 5) | lane;
         const uint32_t lrow = (uint32_t)((warp & 3) << 5) << 16;
         bool failed = false;
@@ -401,11 +416,12 @@ __global__ void __launch_bounds__(kBThreads, 1)
                     int j[C::PP];
                     {
                         // this thread's PP projections: columns H*PP.. of the hi, mid and lo parts
-                        uint32_t xh[4], xm[4], xl[4];
+                        static_assert(C::PP == 2, "two projections per thread");
+                        uint32_t xh[2], xm[2], xl[2];
                         const uint32_t ucol = tbase + lrow + cU + (g & 1) * C::NU + H * C::PP;
-                        tmem_ld4(ucol, xh);
-                        tmem_ld4(ucol + C::MP, xm);
-                        tmem_ld4(ucol + 2 * C::MP, xl);
+                        tmem_ld2(ucol, xh);
+                        tmem_ld2(ucol + C::MP, xm);
+                        tmem_ld2(ucol + 2 * C::MP, xl);
                         tmem_wait_ld();
 #pragma unroll
                         for (int q = 0; q < C::PP; ++q)
@@ -434,12 +450,16 @@ __global__ void __launch_bounds__(kBThreads, 1)
                             dotp = fmaf(y[l], __uint_as_float(ph[l]) + __uint_as_float(pl[l]), dotp);
                         }
                     }
-                    float *rs = sred + (g & 1) * 512;
+                    float *rs = sred + (g & 1) * (C::SRED / 2);
                     rs[H * 128 + r] = denp;
-                    rs[256 + H * 128 + r] = dotp;
+                    rs[kBRowThreads * 128 + H * 128 + r] = dotp;
                     named_sync<kBWorkers>(1);
-                    const float den = rs[r] + rs[128 + r] + a.eps;
-                    const float dotn = rs[256 + r] + rs[384 + r];  // = (dO.O) * den
+                    float den = a.eps, dotn = 0.0f;  // dotn = (dO.O) * den; parts added in a fixed order
+#pragma unroll
+                    for (int h = 0; h < kBRowThreads; ++h) {
+                        den += rs[h * 128 + r];
+                        dotn += rs[kBRowThreads * 128 + h * 128 + r];
+                    }
                     const bool live = valid && den != 0.0f;
                     const float inv = live ? 1.0f / den : 0.0f;
                     const float ndot = live ? -dotn * inv : 0.0f;  // -(dO.O)
@@ -478,24 +498,14 @@ __global__ void __launch_bounds__(kBThreads, 1)
                     }
                     // G = [dO (dv cols) | dU_hi | dU_lo | dU_hi | -(dO.O) hi, lo | 0] over the dO tile (in place)
                     {
-                        if (!valid) {  // padded rows may hold anything (even non-finite values)
-                            const int c0 = H * (C::DV / 2);
-#pragma unroll
-                            for (int cc = 0; cc < C::DV / 2; cc += 8)
-                                *reinterpret_cast<uint4 *>(gt + sw128_chunk(r, (c0 + cc) / 8)) = make_uint4(0, 0, 0, 0);
-                        }
-                        __nv_bfloat16 hi[C::PP], lo[C::PP];
-#pragma unroll
-                        for (int q = 0; q < C::PP; ++q) split_bf16(dU[q], hi[q], lo[q]);
-                        // columns 32 + 4H .. : dU_hi;  40 + 4H: dU_lo;  48 + 4H: dU_hi (chunks 4, 5, 6)
-                        uint2 vh, vl;
-                        vh.x = (uint32_t)__bfloat16_as_ushort(hi[0]) | ((uint32_t)__bfloat16_as_ushort(hi[1]) << 16);
-                        vh.y = (uint32_t)__bfloat16_as_ushort(hi[2]) | ((uint32_t)__bfloat16_as_ushort(hi[3]) << 16);
-                        vl.x = (uint32_t)__bfloat16_as_ushort(lo[0]) | ((uint32_t)__bfloat16_as_ushort(lo[1]) << 16);
-                        vl.y = (uint32_t)__bfloat16_as_ushort(lo[2]) | ((uint32_t)__bfloat16_as_ushort(lo[3]) << 16);
-                        *reinterpret_cast<uint2 *>(gt + sw128_chunk(r, 4) + H * 8) = vh;
-                        *reinterpret_cast<uint2 *>(gt + sw128_chunk(r, 5) + H * 8) = vl;
-                        *reinterpret_cast<uint2 *>(gt + sw128_chunk(r, 6) + H * 8) = vh;
+                        if (!valid)  // padded rows may hold anything (even non-finite values): chunk H of dO
+                            *reinterpret_cast<uint4 *>(gt + sw128_chunk(r, H)) = make_uint4(0, 0, 0, 0);
+                        // columns 32 + PP*H .. : dU_hi;  40 + PP*H: dU_lo;  48 + PP*H: dU_hi (chunks 4, 5, 6)
+                        uint32_t vh, vl;
+                        dU_pack(dU, vh, vl);
+                        *reinterpret_cast<uint32_t *>(gt + sw128_chunk(r, 4) + H * 4) = vh;
+                        *reinterpret_cast<uint32_t *>(gt + sw128_chunk(r, 5) + H * 4) = vl;
+                        *reinterpret_cast<uint32_t *>(gt + sw128_chunk(r, 6) + H * 4) = vh;
                         if (H == 0) {  // chunk 7: -(dO.O) as hi, lo; zeros
                             __nv_bfloat16 th, tl;
                             split_bf16(ndot, th, tl);
@@ -510,22 +520,15 @@ __global__ void __launch_bounds__(kBThreads, 1)
                     wait_or_fail(dqready, g & 1, failed, status);
                     tc_fence_after();
                     {
-                        uint32_t x[16];
-                        tmem_ld16(tbase + lrow + cQ + H * 16, x);
+                        uint32_t x[8];
+                        tmem_ld8(tbase + lrow + cQ + H * 8, x);
                         tmem_wait_ld();
-                        float f[16];
+                        float f[8];
 #pragma unroll
-                        for (int c = 0; c < 16; ++c) f[c] = __uint_as_float(x[c]);
+                        for (int c = 0; c < 8; ++c) f[c] = __uint_as_float(x[c]);
                         tc_fence_before();
                         mbar_arrive(dqfree);
-                        if (valid) {
-                            uint4 *dst = reinterpret_cast<uint4 *>(dQ + (size_t)(row0 + r) * C::d + H * 16);
-                            float f0[8], f1[8];
-#pragma unroll
-                            for (int c = 0; c < 8; ++c) { f0[c] = f[c]; f1[c] = f[8 + c]; }
-                            dst[0] = pack8(f0);
-                            dst[1] = pack8(f1);
-                        }
+                        if (valid) *reinterpret_cast<uint4 *>(dQ + (size_t)(row0 + r) * C::d + H * 8) = pack8(f);
                     }
                 }
             }
@@ -633,9 +636,8 @@ __global__ void __launch_bounds__(kBThreads, 1)
     uint8_t *Sb = sm;                    // [NS] x (phi_hi tile, K tile)
     uint8_t *Vb = Sb + NS * 2 * T16;     // [NV]
     uint8_t *Gt = Vb + NV * T16;         // [dU_hi | dU_lo | dU_hi | 0]
-    uint8_t *Wop = Gt + T16;
-    uint8_t *Wx = Wop + C::WOP;
-    uint8_t *Sop = Wx + C::WXP;          // dV = phi [dS_hi; dS_lo]: rows per value column
+    uint8_t *Wop = Gt + T16;             // projection and dX operands
+    uint8_t *Sop = Wop + C::WOP;         // dV = phi [dS_hi; dS_lo]: rows per value column
     uint8_t *Sop2 = Sop + C::SOP;        // dphi = V [dS_hi; dS_lo]^T: rows per feature
     float *sTe = reinterpret_cast<float *>(Sop2 + C::SOP2);
     float *sAB = sTe + kEytzinger;
@@ -684,7 +686,8 @@ __global__ void __launch_bounds__(kBThreads, 1)
     }
     if (warp == 0) { tmem_alloc(tslot, 512); tmem_relinquish(); }
     stage_phi_table<C>(a, sTe, sAB, sbias, Wop);
-    stage_wx<C>(a, Wx);
+    __syncthreads();
+    stage_wx<C>(a, Wop);
     for (int e = tid; e < kNint * 16; e += blockDim.x) hist[e] = 0.0f;
     for (int e = tid; e < C::MP * C::d + 16; e += blockDim.x) sdW[e] = 0.0f;
     for (int e = tid; e < (int)(T16 / 16); e += blockDim.x) reinterpret_cast<uint4 *>(Gt)[e] = make_uint4(0, 0, 0, 0);
@@ -731,7 +734,7 @@ __global__ void __launch_bounds__(kBThreads, 1)
             const uint64_t dV0 = sdesc(smem_u32(Vb), 16384, 1024, kSwizzle128);
             const uint64_t dG = sdesc(smem_u32(Gt), 16384, 1024, kSwizzle128);
             const uint64_t dWo = sdesc(smem_u32(Wop), 16, 1024, kSwizzle128);
-            const uint64_t dWx = sdesc(smem_u32(Wx), 16, 1024, kSwizzle128);
+            const uint64_t dWx = dadd(dWo, 64);  // columns 32..63 of the same rows
             const uint64_t dSa = sdesc(smem_u32(Sop), 16, 1024, kSwizzle128);
             const uint64_t dSb = sdesc(smem_u32(Sop2), 16, 1024, kSwizzle128);
             bool failed = false;
@@ -836,11 +839,12 @@ __global__ void __launch_bounds__(kBThreads, 1)
                     int j[C::PP];
                     {
                         // this thread's PP projections: columns H*PP.. of the hi, mid and lo parts
-                        uint32_t xh[4], xm[4], xl[4];
+                        static_assert(C::PP == 2, "two projections per thread");
+                        uint32_t xh[2], xm[2], xl[2];
                         const uint32_t ucol = tbase + lrow + cU + (g & 1) * C::NU + H * C::PP;
-                        tmem_ld4(ucol, xh);
-                        tmem_ld4(ucol + C::MP, xm);
-                        tmem_ld4(ucol + 2 * C::MP, xl);
+                        tmem_ld2(ucol, xh);
+                        tmem_ld2(ucol + C::MP, xm);
+                        tmem_ld2(ucol + 2 * C::MP, xl);
                         tmem_wait_ld();
 #pragma unroll
                         for (int q = 0; q < C::PP; ++q)
@@ -880,17 +884,11 @@ __global__ void __launch_bounds__(kBThreads, 1)
                     }
                     if (g >= 1) wait_or_fail(gfree, (g - 1) & 1, failed, status);
                     {
-                        __nv_bfloat16 hi[C::PP], lo[C::PP];
-#pragma unroll
-                        for (int q = 0; q < C::PP; ++q) split_bf16(dU[q], hi[q], lo[q]);
-                        uint2 vh, vl;
-                        vh.x = (uint32_t)__bfloat16_as_ushort(hi[0]) | ((uint32_t)__bfloat16_as_ushort(hi[1]) << 16);
-                        vh.y = (uint32_t)__bfloat16_as_ushort(hi[2]) | ((uint32_t)__bfloat16_as_ushort(hi[3]) << 16);
-                        vl.x = (uint32_t)__bfloat16_as_ushort(lo[0]) | ((uint32_t)__bfloat16_as_ushort(lo[1]) << 16);
-                        vl.y = (uint32_t)__bfloat16_as_ushort(lo[2]) | ((uint32_t)__bfloat16_as_ushort(lo[3]) << 16);
-                        *reinterpret_cast<uint2 *>(Gt + sw128_chunk(r, 0) + H * 8) = vh;
-                        *reinterpret_cast<uint2 *>(Gt + sw128_chunk(r, 1) + H * 8) = vl;
-                        *reinterpret_cast<uint2 *>(Gt + sw128_chunk(r, 2) + H * 8) = vh;
+                        uint32_t vh, vl;
+                        dU_pack(dU, vh, vl);
+                        *reinterpret_cast<uint32_t *>(Gt + sw128_chunk(r, 0) + H * 4) = vh;
+                        *reinterpret_cast<uint32_t *>(Gt + sw128_chunk(r, 1) + H * 4) = vl;
+                        *reinterpret_cast<uint32_t *>(Gt + sw128_chunk(r, 2) + H * 4) = vh;
                     }
                     fence_proxy_async_smem();
                     tc_fence_before();
@@ -899,41 +897,34 @@ __global__ void __launch_bounds__(kBThreads, 1)
                     wait_or_fail(dvready + (g & 1), (g >> 1) & 1, failed, status);
                     tc_fence_after();
                     {
-                        uint32_t xh[16], xl[16];
-                        const uint32_t vcol = tbase + lrow + cV + (g & 1) * 64 + H * 16;
-                        tmem_ld16(vcol, xh);
-                        tmem_ld16(vcol + C::DV, xl);
+                        uint32_t xh[8], xl[8];
+                        const uint32_t vcol = tbase + lrow + cV + (g & 1) * 64 + H * 8;
+                        tmem_ld8(vcol, xh);
+                        tmem_ld8(vcol + C::DV, xl);
                         tmem_wait_ld();
                         tc_fence_before();
                         mbar_arrive(dvfree + (g & 1));
                         if (valid) {
-                            float f0[8], f1[8];
+                            float f[8];
 #pragma unroll
-                            for (int c = 0; c < 8; ++c) {
-                                f0[c] = __uint_as_float(xh[c]) + __uint_as_float(xl[c]);
-                                f1[c] = __uint_as_float(xh[8 + c]) + __uint_as_float(xl[8 + c]);
-                            }
-                            uint4 *dst = reinterpret_cast<uint4 *>(dV + (size_t)(row0 + r) * C::DV + H * 16);
-                            dst[0] = pack8(f0);
-                            dst[1] = pack8(f1);
+                            for (int c = 0; c < 8; ++c) f[c] = __uint_as_float(xh[c]) + __uint_as_float(xl[c]);
+                            *reinterpret_cast<uint4 *>(dV + (size_t)(row0 + r) * C::DV + H * 8) = pack8(f);
                         }
                     }
                     // dK
                     wait_or_fail(dkready, g & 1, failed, status);
                     tc_fence_after();
                     {
-                        uint32_t x[16];
-                        tmem_ld16(tbase + lrow + cK + H * 16, x);
+                        uint32_t x[8];
+                        tmem_ld8(tbase + lrow + cK + H * 8, x);
                         tmem_wait_ld();
                         tc_fence_before();
                         mbar_arrive(dkfree);
                         if (valid) {
-                            float f0[8], f1[8];
+                            float f[8];
 #pragma unroll
-                            for (int c = 0; c < 8; ++c) { f0[c] = __uint_as_float(x[c]); f1[c] = __uint_as_float(x[8 + c]); }
-                            uint4 *dst = reinterpret_cast<uint4 *>(dK + (size_t)(row0 + r) * C::d + H * 16);
-                            dst[0] = pack8(f0);
-                            dst[1] = pack8(f1);
+                            for (int c = 0; c < 8; ++c) f[c] = __uint_as_float(x[c]);
+                            *reinterpret_cast<uint4 *>(dK + (size_t)(row0 + r) * C::d + H * 8) = pack8(f);
                         }
                     }
                 }
