@@ -56,12 +56,13 @@ struct B32 {
     // query side: stage = [phi/den (hi, lo interleaved by 16 features) x 2 tiles | Q tile]
     static constexpr int NSQ = 2, NOQ = 2;
     static constexpr uint32_t SRED = 2 * 2 * kBRowThreads * 128;  // floats: [tile parity][den, dot][part][row]
+    static constexpr uint32_t SMAX = 2 * (kBWorkers / 32) * 4;
     static constexpr uint32_t SMEM_Q = NSQ * 3 * TILE + NOQ * TILE + WOP + SOP2 + kTableBytes + D * 4 + SRED * 4 +
-                                       HIST + MP * d * 4 + 64 + kBarBytes + 1024;
+                                       HIST + MP * d * 4 + 64 + SMAX + kBarBytes + 1024;
     // key side
     static constexpr int NSK = 2, NVK = 2;
     static constexpr uint32_t SMEM_K = NSK * 2 * TILE + NVK * TILE + TILE + WOP + SOP + SOP2 + kTableBytes +
-                                       D * 4 + HIST + MP * d * 4 + 64 + kBarBytes + 1024;
+                                       D * 4 + HIST + MP * d * 4 + 64 + SMAX + kBarBytes + 1024;
     static_assert(SMEM_Q <= kSmemLimit && SMEM_K <= kSmemLimit, "shared memory budget");
 };
 
@@ -160,25 +161,87 @@ __device__ __forceinline__ uint4 pack8(const float (&y)[8]) {
                       pack_bf16x2(y[6], y[7]));
 }
 
-// Interval histogram in shared memory: hist[c * 8 * kNint + l * kNint + j] holds,
-// for channel l and interval j, the sum of g (c = 0) and of g * u (c = 1); lanes
-// with different intervals fall into different banks.
+// Interval histogram of the channel-MLP gradient statistics: for channel l and
+// interval j, the sum of g (c = 0) and of g * u (c = 1) over the samples u that
+// fall into interval j, g = dLoss/dphi on an active output.
+//
+// Shared-memory fp32 atomics are compare-and-swap loops; int32 atomics are
+// native and about five times faster.  So every tile accumulates in fixed
+// point: g and g*u are quantised with power-of-two scales 2^s taken from the
+// tile's block-wide maxima (|q| < 2^20 per sample; a bin receives at most 1024
+// samples per tile, so it stays below 2^30), then the int32 bins are added,
+// rescaled, into the block's fp32 partial in global memory and cleared.  The
+// quantisation step is 2^-21 of the tile maximum.
+//
+// Layout in shared memory: bins[(c * 8 + l) * kNint + j] (lanes with different
+// intervals fall into different banks).
 __device__ __forceinline__ int hist_at(int c, int l, int j) { return (c * 8 + l) * kNint + j; }
 
-// Backward through the channel functions for one projection value: g = dLoss/dphi on
-// the active outputs; adds g and g*u to the interval histogram, returns dLoss/du.
-__device__ __forceinline__ float channel_backward(float *hist, int j, float u, const float (&al)[8],
-                                                  const float (&y)[8], const float (&dphi)[8]) {
-    float du = 0.0f;
+// 2^e as a float, e in [-126, 127] (IEEE-754 binary32: biased exponent, zero mantissa).
+__device__ __forceinline__ float pow2f(int e) { return __int_as_float((e + 127) << 23); }
+
+// Running maximum of |v| that turns into +inf once a non-finite value is seen.
+__device__ __forceinline__ float track_max(float m, float v) {
+    const float a = fabsf(v);
+    return a <= 3.402823466e38f ? fmaxf(m, a) : __int_as_float(0x7f800000);
+}
+
+struct HistScale {
+    float s0, s1, inv0, inv1;
+    bool bad;  // a non-finite g or g*u: the partial becomes NaN, as an fp32 sum would
+};
+
+// Scale 2^e with m * 2^e < 2^20: m < 2^ex for ex = (biased exponent of m) - 126.
+__device__ __forceinline__ void hist_scale_of(float m, float &sc, float &inv) {
+    const int ex = (int)((__float_as_uint(m) >> 23) & 255u) - 126;
+    const int e = max(-126, min(126, 20 - ex));
+    sc = pow2f(e);
+    inv = pow2f(-e);
+}
+
+// Block-wide maxima of |g| and |g*u| over the worker threads (one named barrier).
+// smax: 2 * (kBWorkers / 32) floats, reused by every tile (each tile has a later
+// worker barrier before the next write).
+__device__ __forceinline__ HistScale hist_block_scale(float m0, float m1, float *smax, int warp, int lane) {
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) {
+        m0 = fmaxf(m0, __shfl_xor_sync(0xffffffffu, m0, o));
+        m1 = fmaxf(m1, __shfl_xor_sync(0xffffffffu, m1, o));
+    }
+    constexpr int NW = kBWorkers / 32;
+    if (lane == 0) { smax[warp] = m0; smax[NW + warp] = m1; }
+    named_sync<kBWorkers>(1);
+    float M0 = 0.0f, M1 = 0.0f;
+#pragma unroll
+    for (int w = 0; w < NW; ++w) { M0 = fmaxf(M0, smax[w]); M1 = fmaxf(M1, smax[NW + w]); }
+    HistScale h;
+    h.bad = !(M0 <= 3.402823466e38f) || !(M1 <= 3.402823466e38f);
+    hist_scale_of(M0, h.s0, h.inv0);
+    hist_scale_of(M1, h.s1, h.inv1);
+    return h;
+}
+
+// Adds the 8 channel values g (zero where inactive) of one sample u in interval j.
+__device__ __forceinline__ void hist_add(int *bins, int j, float u, const float (&g)[8], const HistScale &h) {
 #pragma unroll
     for (int l = 0; l < 8; ++l) {
-        if (y[l] > 0.0f && dphi[l] != 0.0f) {
-            du = fmaf(dphi[l], al[l], du);
-            atomicAdd(hist + hist_at(0, l, j), dphi[l]);
-            atomicAdd(hist + hist_at(1, l, j), dphi[l] * u);
+        if (g[l] != 0.0f) {
+            atomicAdd(bins + hist_at(0, l, j), __float2int_rn(g[l] * h.s0));
+            atomicAdd(bins + hist_at(1, l, j), __float2int_rn(g[l] * u * h.s1));
         }
     }
-    return du;
+}
+
+// Adds the tile's bins into the block's fp32 partial ([interval][channel][g, g*u])
+// and clears them; thread t of nthr handles entries t, t + nthr, ...
+__device__ __forceinline__ void hist_flush(int *bins, float *part, int nint, const HistScale &h, int t, int nthr) {
+#pragma unroll 4
+    for (int e = t; e < nint * 16; e += nthr) {
+        const int at = hist_at(e & 1, (e >> 1) & 7, e >> 4);
+        const int v = bins[at];
+        bins[at] = 0;
+        part[e] += h.bad ? __int_as_float(0x7fc00000) : (float)v * ((e & 1) ? h.inv1 : h.inv0);
+    }
 }
 
 // Zeroes a row of a 128-row x 128 B tile (padded rows must not carry garbage
@@ -188,15 +251,13 @@ __device__ __forceinline__ void zero_row(uint8_t *tile, int r) {
     for (int c = 0; c < 8; ++c) *reinterpret_cast<uint4 *>(tile + sw128_chunk(r, c)) = make_uint4(0, 0, 0, 0);
 }
 
-// Writes the per-block parameter-gradient partial: dW (M x d) from smem, db
-// (block sum of per-thread values), the interval histogram (as [interval][channel][g, g*u]).
+// Writes dW (M x d, from smem) and db (block sum of per-thread values) into the
+// block's parameter-gradient partial; its histogram part is written tile by tile.
 template <class C>
-__device__ void store_param_partial(const AttnArgs &a, const float *sdW, float *sdb, const float *hist, float *gp) {
+__device__ void store_param_partial(const AttnArgs &a, const float *sdW, float *sdb, float *gp) {
     const int Md = C::MP * a.d;
     for (int e = threadIdx.x; e < Md; e += blockDim.x) gp[e] = sdW[e];
     for (int e = threadIdx.x; e < C::MP; e += blockDim.x) gp[Md + e] = sdb[e];
-    for (int e = threadIdx.x; e < a.lay.nint * 16; e += blockDim.x)
-        gp[Md + C::MP + e] = hist[hist_at(e & 1, (e >> 1) & 7, e >> 4)];
 }
 
 // ---------------------------------------------------------------------------
@@ -219,10 +280,11 @@ __global__ void __launch_bounds__(kBThreads, 1)
     float *sbias = sAB + kNint * 16;
     float *sz = sbias + 32;
     float *sred = sz + C::D;              // [2 tiles][den, dot][kBRowThreads parts][128 rows]
-    float *hist = sred + C::SRED;         // [g, g*u][8][kNint]
-    float *sdW = hist + kNint * 16;       // [M][d]
+    int *bins = reinterpret_cast<int *>(sred + C::SRED);  // fixed-point histogram of the current tile
+    float *sdW = reinterpret_cast<float *>(bins + kNint * 16);  // [M][d]
     float *sdb = sdW + C::MP * C::d;      // [M] (padded to 16)
-    uint64_t *bars = reinterpret_cast<uint64_t *>(sdb + 16);
+    float *smax = sdb + 16;               // [2][worker warps]
+    uint64_t *bars = reinterpret_cast<uint64_t *>(smax + 2 * (kBWorkers / 32));
     uint64_t *fullq = bars;               // [NS]
     uint64_t *sfree = fullq + NS;         // [NS] phi and Q tile consumed
     uint64_t *fullo = sfree + NS;         // [NO]
@@ -262,8 +324,10 @@ __global__ void __launch_bounds__(kBThreads, 1)
     stage_phi_table<C>(a, sTe, sAB, sbias, Wop);
     __syncthreads();
     stage_wx<C>(a, Wop);
-    for (int e = tid; e < kNint * 16; e += blockDim.x) hist[e] = 0.0f;
+    for (int e = tid; e < kNint * 16; e += blockDim.x) bins[e] = 0;
     for (int e = tid; e < C::MP * C::d + 16; e += blockDim.x) sdW[e] = 0.0f;
+    float *hpart = a.gpart + (size_t)blockIdx.x * a.gsize + C::MP * a.d + C::MP;  // histogram part of the partial
+    for (int e = tid; e < a.lay.nint * 16; e += blockDim.x) hpart[e] = 0.0f;
     // padded rows of every item produce zero gradients
     for (int item = it.begin; item < it.end; ++item) {
         const ItemRange ir = item_range(a, it, item);
@@ -465,11 +529,11 @@ __global__ void __launch_bounds__(kBThreads, 1)
                     const float ndot = live ? -dotn * inv : 0.0f;  // -(dO.O)
                     const float dden = ndot * inv;
                     // gradients through the feature map; phi/den (bf16) for the stacked contraction
-                    float dU[C::PP];
+                    float dU[C::PP], gv[C::PP][8], m0 = 0.0f, m1 = 0.0f;
 #pragma unroll
                     for (int q = 0; q < C::PP; ++q) {
                         const int i = H * C::PP + q;
-                        float al[8], y[8], dphi[8];
+                        float al[8], y[8];
                         channel_eval(sAB, j[q], u[q], al, y);
                         {
                             // phi/den as hi, lo; a row holds 16-feature groups [hi | lo | hi | lo] per 64-wide tile,
@@ -489,12 +553,19 @@ __global__ void __launch_bounds__(kBThreads, 1)
                         tmem_ld8(pcol + 8 * i, ph);
                         tmem_ld8(pcol + C::D + 8 * i, pl);
                         tmem_wait_ld();
+                        float du = 0.0f;
 #pragma unroll
-                        for (int l = 0; l < 8; ++l)
-                            dphi[l] = live ? (__uint_as_float(ph[l]) + __uint_as_float(pl[l])) * inv + sz[8 * i + l] * dden
-                                           : 0.0f;
-                        dU[q] = live ? channel_backward(hist, j[q], u[q], al, y, dphi) : 0.0f;
-                        db_acc[q] += dU[q];
+                        for (int l = 0; l < 8; ++l) {
+                            const float dphi =
+                                live ? (__uint_as_float(ph[l]) + __uint_as_float(pl[l])) * inv + sz[8 * i + l] * dden : 0.0f;
+                            const float gl = y[l] > 0.0f ? dphi : 0.0f;  // through the outer ReLU
+                            gv[q][l] = gl;
+                            du = fmaf(gl, al[l], du);
+                            m0 = track_max(m0, gl);
+                            m1 = track_max(m1, gl * u[q]);
+                        }
+                        dU[q] = du;
+                        db_acc[q] += du;
                     }
                     // G = [dO (dv cols) | dU_hi | dU_lo | dU_hi | -(dO.O) hi, lo | 0] over the dO tile (in place)
                     {
@@ -516,6 +587,15 @@ __global__ void __launch_bounds__(kBThreads, 1)
                     fence_proxy_async_smem();
                     tc_fence_before();
                     mbar_arrive(gready + (g & 1));
+                    // interval histogram of this tile (fixed point), then into the block partial
+                    {
+                        const HistScale hs = hist_block_scale(m0, m1, smax, warp, lane);
+                        if (!hs.bad)
+#pragma unroll
+                            for (int q = 0; q < C::PP; ++q) hist_add(bins, j[q], u[q], gv[q], hs);
+                        named_sync<kBWorkers>(1);
+                        hist_flush(bins, hpart, a.lay.nint, hs, tid, kBWorkers);
+                    }
                     // dQ
                     wait_or_fail(dqready, g & 1, failed, status);
                     tc_fence_after();
@@ -617,7 +697,7 @@ __global__ void __launch_bounds__(kBThreads, 1)
     }
     tc_fence_before();
     __syncthreads();
-    store_param_partial<C>(a, sdW, sdb, hist, a.gpart + (size_t)blockIdx.x * a.gsize);
+    store_param_partial<C>(a, sdW, sdb, a.gpart + (size_t)blockIdx.x * a.gsize);
     __syncthreads();
     if (warp == 0) tmem_dealloc(tbase, 512);
 }
@@ -643,10 +723,11 @@ __global__ void __launch_bounds__(kBThreads, 1)
     float *sAB = sTe + kEytzinger;
     float *sbias = sAB + kNint * 16;
     float *sdz = sbias + 32;
-    float *hist = sdz + C::D;
-    float *sdW = hist + kNint * 16;
+    int *bins = reinterpret_cast<int *>(sdz + C::D);  // fixed-point histogram of the current tile
+    float *sdW = reinterpret_cast<float *>(bins + kNint * 16);
     float *sdb = sdW + C::MP * C::d;
-    uint64_t *bars = reinterpret_cast<uint64_t *>(sdb + 16);
+    float *smax = sdb + 16;               // [2][worker warps]
+    uint64_t *bars = reinterpret_cast<uint64_t *>(smax + 2 * (kBWorkers / 32));
     uint64_t *fullk = bars;              // [NS]
     uint64_t *sfree = fullk + NS;        // [NS]
     uint64_t *fullv = sfree + NS;        // [NV]
@@ -688,8 +769,10 @@ __global__ void __launch_bounds__(kBThreads, 1)
     stage_phi_table<C>(a, sTe, sAB, sbias, Wop);
     __syncthreads();
     stage_wx<C>(a, Wop);
-    for (int e = tid; e < kNint * 16; e += blockDim.x) hist[e] = 0.0f;
+    for (int e = tid; e < kNint * 16; e += blockDim.x) bins[e] = 0;
     for (int e = tid; e < C::MP * C::d + 16; e += blockDim.x) sdW[e] = 0.0f;
+    float *hpart = a.gpart + (size_t)(gridDim.x + blockIdx.x) * a.gsize + C::MP * a.d + C::MP;
+    for (int e = tid; e < a.lay.nint * 16; e += blockDim.x) hpart[e] = 0.0f;
     for (int e = tid; e < (int)(T16 / 16); e += blockDim.x) reinterpret_cast<uint4 *>(Gt)[e] = make_uint4(0, 0, 0, 0);
     for (int item = it.begin; item < it.end; ++item) {  // padded rows receive zero gradients
         const ItemRange ir = item_range(a, it, item);
@@ -867,20 +950,28 @@ __global__ void __launch_bounds__(kBThreads, 1)
                     wait_or_fail(fready + (g & 1), (g >> 1) & 1, failed, status);
                     tc_fence_after();
                     const uint32_t fcol = tbase + lrow + cF + (g & 1) * 128;
-                    float dU[C::PP];
+                    float dU[C::PP], gv[C::PP][8], m0 = 0.0f, m1 = 0.0f;
 #pragma unroll
                     for (int q = 0; q < C::PP; ++q) {
                         const int i = H * C::PP + q;
-                        float al[8], y[8], dphi[8];
+                        float al[8], y[8];
                         channel_eval(sAB, j[q], u[q], al, y);
                         uint32_t ph[8], pl[8];
                         tmem_ld8(fcol + 8 * i, ph);
                         tmem_ld8(fcol + C::D + 8 * i, pl);
                         tmem_wait_ld();
+                        float du = 0.0f;
 #pragma unroll
-                        for (int l = 0; l < 8; ++l) dphi[l] = __uint_as_float(ph[l]) + __uint_as_float(pl[l]) + sdz[8 * i + l];
-                        dU[q] = valid ? channel_backward(hist, j[q], u[q], al, y, dphi) : 0.0f;
-                        db_acc[q] += dU[q];
+                        for (int l = 0; l < 8; ++l) {
+                            const float dphi = __uint_as_float(ph[l]) + __uint_as_float(pl[l]) + sdz[8 * i + l];
+                            const float gl = (valid && y[l] > 0.0f) ? dphi : 0.0f;
+                            gv[q][l] = gl;
+                            du = fmaf(gl, al[l], du);
+                            m0 = track_max(m0, gl);
+                            m1 = track_max(m1, gl * u[q]);
+                        }
+                        dU[q] = du;
+                        db_acc[q] += du;
                     }
                     if (g >= 1) wait_or_fail(gfree, (g - 1) & 1, failed, status);
                     {
@@ -893,6 +984,15 @@ __global__ void __launch_bounds__(kBThreads, 1)
                     fence_proxy_async_smem();
                     tc_fence_before();
                     mbar_arrive(gready + (g & 1));
+                    // interval histogram of this tile (fixed point), then into the block partial
+                    {
+                        const HistScale hs = hist_block_scale(m0, m1, smax, warp, lane);
+                        if (!hs.bad)
+#pragma unroll
+                            for (int q = 0; q < C::PP; ++q) hist_add(bins, j[q], u[q], gv[q], hs);
+                        named_sync<kBWorkers>(1);
+                        hist_flush(bins, hpart, a.lay.nint, hs, tid, kBWorkers);
+                    }
                     // dV = hi + lo
                     wait_or_fail(dvready + (g & 1), (g >> 1) & 1, failed, status);
                     tc_fence_after();
@@ -954,7 +1054,7 @@ __global__ void __launch_bounds__(kBThreads, 1)
     }
     tc_fence_before();
     __syncthreads();
-    store_param_partial<C>(a, sdW, sdb, hist, a.gpart + (size_t)(gridDim.x + blockIdx.x) * a.gsize);
+    store_param_partial<C>(a, sdW, sdb, a.gpart + (size_t)(gridDim.x + blockIdx.x) * a.gsize);
     __syncthreads();
     if (warp == 0) tmem_dealloc(tbase, 512);
 }
