@@ -121,11 +121,11 @@ __device__ __forceinline__ void phi_row_quarter(uint32_t tmem_u_row, const float
         uint4 ph = make_uint4(0u, 0u, 0u, 0u), pl = make_uint4(0u, 0u, 0u, 0u);
         if (valid) {
             const int j = node[q] - kEytzinger;
-            const float4 *ab = reinterpret_cast<const float4 *>(sAB) + (j << 2);
+            const float4 *ab = reinterpret_cast<const float4 *>(sAB);
             float y[8];
 #pragma unroll
             for (int k = 0; k < 4; ++k) {
-                const float4 v = ab[k ^ (j & 3)];
+                const float4 v = ab[ab_slot(j, k)];
                 y[2 * k] = fmaxf(fmaf(v.x, u[q], v.y), 0.0f);
                 y[2 * k + 1] = fmaxf(fmaf(v.z, u[q], v.w), 0.0f);
             }

@@ -62,7 +62,7 @@ struct B32 {
     // key side
     static constexpr int NSK = 2, NVK = 2;
     static constexpr uint32_t SMEM_K = NSK * 2 * TILE + NVK * TILE + TILE + WOP + SOP + SOP2 + kTableBytes +
-                                       D * 4 + HIST + MP * d * 4 + 64 + SMAX + kBarBytes + 1024;
+                                       D * 4 + HIST + MP * d * 4 + 64 + 2 * SMAX + kBarBytes + 1024;
     static_assert(SMEM_Q <= kSmemLimit && SMEM_K <= kSmemLimit, "shared memory budget");
 };
 
@@ -136,10 +136,10 @@ __device__ __forceinline__ void search(const float *sTe, const float (&u)[PP], i
 
 // alpha, beta of the 8 channels on interval j (swizzled table) and phi = relu(alpha u + beta).
 __device__ __forceinline__ void channel_eval(const float *sAB, int j, float u, float (&al)[8], float (&y)[8]) {
-    const float4 *ab = reinterpret_cast<const float4 *>(sAB) + (j << 2);
+    const float4 *ab = reinterpret_cast<const float4 *>(sAB);
 #pragma unroll
     for (int k = 0; k < 4; ++k) {
-        const float4 v = ab[k ^ (j & 3)];
+        const float4 v = ab[ab_slot(j, k)];
         al[2 * k] = v.x;
         al[2 * k + 1] = v.z;
         y[2 * k] = fmaxf(fmaf(v.x, u, v.y), 0.0f);
@@ -166,43 +166,41 @@ __device__ __forceinline__ uint4 pack8(const float (&y)[8]) {
 // fall into interval j, g = dLoss/dphi on an active output.
 //
 // Shared-memory fp32 atomics are compare-and-swap loops; int32 atomics are
-// native and about five times faster.  So every tile accumulates in fixed
-// point: g and g*u are quantised with power-of-two scales 2^s taken from the
-// tile's block-wide maxima (|q| < 2^20 per sample; a bin receives at most 1024
-// samples per tile, so it stays below 2^30), then the int32 bins are added,
-// rescaled, into the block's fp32 partial in global memory and cleared.  The
-// quantisation step is 2^-21 of the tile maximum.
+// native and about five times faster.  So the bins hold fixed-point int32
+// sums: every tile finds the block-wide maxima of |g| and |g*u| and quantises
+// with power-of-two scales 2^e such that |q| < 2^16 per sample.  A bin receives
+// at most 1024 samples per tile, so up to 16 tiles fit below 2^30.  The bins
+// are added, rescaled, into the block's fp32 partial in global memory and
+// cleared ("flushed") after 16 tiles, before a tile whose maximum needs a
+// coarser scale, and at the end; the quantisation step is 2^-16 of the largest
+// value since the last flush.
 //
 // Layout in shared memory: bins[(c * 8 + l) * kNint + j] (lanes with different
 // intervals fall into different banks).
 __device__ __forceinline__ int hist_at(int c, int l, int j) { return (c * 8 + l) * kNint + j; }
 
+constexpr int kHistQBits = 16;  // |q| < 2^16 per sample
+constexpr int kHistTiles = 16;  // tiles between flushes: 16 * 1024 * 2^16 = 2^30
+
 // 2^e as a float, e in [-126, 127] (IEEE-754 binary32: biased exponent, zero mantissa).
 __device__ __forceinline__ float pow2f(int e) { return __int_as_float((e + 127) << 23); }
 
-// Running maximum of |v| that turns into +inf once a non-finite value is seen.
-__device__ __forceinline__ float track_max(float m, float v) {
-    const float a = fabsf(v);
-    return a <= 3.402823466e38f ? fmaxf(m, a) : __int_as_float(0x7f800000);
+// Exponent e with m * 2^e < 2^kHistQBits: m < 2^ex for ex = (biased exponent of m) - 126.
+__device__ __forceinline__ int hist_exp_of(float m) {
+    const int ex = (int)((__float_as_uint(m) >> 23) & 255u) - 126;
+    return max(-126, min(126, kHistQBits - ex));
 }
 
-struct HistScale {
-    float s0, s1, inv0, inv1;
-    bool bad;  // a non-finite g or g*u: the partial becomes NaN, as an fp32 sum would
+// Block-uniform state of the fixed-point bins.
+struct HistAcc {
+    int e0 = 0, e1 = 0;  // exponents of the samples in the bins
+    int tiles = 0;       // tiles added since the last flush
 };
 
-// Scale 2^e with m * 2^e < 2^20: m < 2^ex for ex = (biased exponent of m) - 126.
-__device__ __forceinline__ void hist_scale_of(float m, float &sc, float &inv) {
-    const int ex = (int)((__float_as_uint(m) >> 23) & 255u) - 126;
-    const int e = max(-126, min(126, 20 - ex));
-    sc = pow2f(e);
-    inv = pow2f(-e);
-}
-
-// Block-wide maxima of |g| and |g*u| over the worker threads (one named barrier).
-// smax: 2 * (kBWorkers / 32) floats, reused by every tile (each tile has a later
-// worker barrier before the next write).
-__device__ __forceinline__ HistScale hist_block_scale(float m0, float m1, float *smax, int warp, int lane) {
+// Block-wide maxima of |g| and |g*u| over the worker threads (one named barrier);
+// +inf if any value was not finite.  smax: 2 * (kBWorkers / 32) floats that no
+// worker writes again before every worker has passed its next worker barrier.
+__device__ __forceinline__ void hist_block_max(float &m0, float &m1, float *smax, int warp, int lane) {
 #pragma unroll
     for (int o = 16; o > 0; o >>= 1) {
         m0 = fmaxf(m0, __shfl_xor_sync(0xffffffffu, m0, o));
@@ -211,37 +209,70 @@ __device__ __forceinline__ HistScale hist_block_scale(float m0, float m1, float 
     constexpr int NW = kBWorkers / 32;
     if (lane == 0) { smax[warp] = m0; smax[NW + warp] = m1; }
     named_sync<kBWorkers>(1);
-    float M0 = 0.0f, M1 = 0.0f;
+    m0 = 0.0f;
+    m1 = 0.0f;
 #pragma unroll
-    for (int w = 0; w < NW; ++w) { M0 = fmaxf(M0, smax[w]); M1 = fmaxf(M1, smax[NW + w]); }
-    HistScale h;
-    h.bad = !(M0 <= 3.402823466e38f) || !(M1 <= 3.402823466e38f);
-    hist_scale_of(M0, h.s0, h.inv0);
-    hist_scale_of(M1, h.s1, h.inv1);
-    return h;
+    for (int w = 0; w < NW; ++w) { m0 = fmaxf(m0, smax[w]); m1 = fmaxf(m1, smax[NW + w]); }
 }
 
-// Adds the 8 channel values g (zero where inactive) of one sample u in interval j.
-__device__ __forceinline__ void hist_add(int *bins, int j, float u, const float (&g)[8], const HistScale &h) {
-#pragma unroll
-    for (int l = 0; l < 8; ++l) {
-        if (g[l] != 0.0f) {
-            atomicAdd(bins + hist_at(0, l, j), __float2int_rn(g[l] * h.s0));
-            atomicAdd(bins + hist_at(1, l, j), __float2int_rn(g[l] * u * h.s1));
-        }
-    }
+// Running maximum of |v| that turns into +inf once a non-finite value is seen.
+__device__ __forceinline__ float track_max(float m, float v) {
+    const float a = fabsf(v);
+    return a <= 3.402823466e38f ? fmaxf(m, a) : __int_as_float(0x7f800000);
 }
 
-// Adds the tile's bins into the block's fp32 partial ([interval][channel][g, g*u])
-// and clears them; thread t of nthr handles entries t, t + nthr, ...
-__device__ __forceinline__ void hist_flush(int *bins, float *part, int nint, const HistScale &h, int t, int nthr) {
+// Adds the bins, rescaled, into the block's fp32 partial ([interval][channel][g, g*u])
+// and clears them (nan: adds NaN instead); thread t of nthr handles entries t, t + nthr, ...
+__device__ __forceinline__ void hist_flush(int *bins, float *part, int nint, const HistAcc &h, bool nan, int t,
+                                           int nthr) {
+    const float inv0 = pow2f(-h.e0), inv1 = pow2f(-h.e1);
 #pragma unroll 4
     for (int e = t; e < nint * 16; e += nthr) {
         const int at = hist_at(e & 1, (e >> 1) & 7, e >> 4);
         const int v = bins[at];
         bins[at] = 0;
-        part[e] += h.bad ? __int_as_float(0x7fc00000) : (float)v * ((e & 1) ? h.inv1 : h.inv0);
+        part[e] += nan ? __int_as_float(0x7fc00000) : (float)v * ((e & 1) ? inv1 : inv0);
     }
+}
+
+// The histogram step of one tile, for worker thread t: m0, m1 are this thread's
+// maxima of |g| and |g*u|; g[q][l] the channel values (zero where inactive) of
+// its samples u[q] in intervals j[q].
+template <int PP>
+__device__ __forceinline__ void hist_tile(int *bins, float *part, int nint, HistAcc &h, float m0, float m1,
+                                          float *smax, int warp, int lane, int t, const int (&j)[PP],
+                                          const float (&u)[PP], const float (&g)[PP][8]) {
+    hist_block_max(m0, m1, smax, warp, lane);  // also orders every earlier tile's atomics before a flush
+    const bool bad = !(m0 <= 3.402823466e38f) || !(m1 <= 3.402823466e38f);
+    const int e0 = hist_exp_of(m0), e1 = hist_exp_of(m1);
+    if (h.tiles > 0 && (bad || e0 < h.e0 || e1 < h.e1 || h.tiles == kHistTiles)) {
+        hist_flush(bins, part, nint, h, false, t, kBWorkers);
+        named_sync<kBWorkers>(1);  // bins cleared before this tile's atomics
+        h.tiles = 0;
+    }
+    if (bad) {  // no bins in use: mark the partial
+        hist_flush(bins, part, nint, h, true, t, kBWorkers);
+        return;
+    }
+    if (h.tiles == 0) { h.e0 = e0; h.e1 = e1; }
+    const float s0 = pow2f(h.e0), s1 = pow2f(h.e1);
+#pragma unroll
+    for (int q = 0; q < PP; ++q)
+#pragma unroll
+        for (int l = 0; l < 8; ++l) {
+            if (g[q][l] != 0.0f) {
+                atomicAdd(bins + hist_at(0, l, j[q]), __float2int_rn(g[q][l] * s0));
+                atomicAdd(bins + hist_at(1, l, j[q]), __float2int_rn(g[q][l] * u[q] * s1));
+            }
+        }
+    ++h.tiles;
+}
+
+// Final flush of the bins after the last tile of the block.
+__device__ __forceinline__ void hist_finish(int *bins, float *part, int nint, const HistAcc &h, int t) {
+    if (h.tiles == 0) return;
+    named_sync<kBWorkers>(1);  // every atomic done
+    hist_flush(bins, part, nint, h, false, t, kBWorkers);
 }
 
 // Zeroes a row of a 128-row x 128 B tile (padded rows must not carry garbage
@@ -450,6 +481,7 @@ __global__ void __launch_bounds__(kBThreads, 1)
         float db_acc[C::PP];
 #pragma unroll
         for (int q = 0; q < C::PP; ++q) db_acc[q] = 0.0f;
+        HistAcc hacc;
         int g = 0, ne = 0;
         for (int i0 = it.begin; i0 < it.end;) {
             const int bh = i0 / it.nchunk;
@@ -587,15 +619,9 @@ __global__ void __launch_bounds__(kBThreads, 1)
                     fence_proxy_async_smem();
                     tc_fence_before();
                     mbar_arrive(gready + (g & 1));
-                    // interval histogram of this tile (fixed point), then into the block partial
-                    {
-                        const HistScale hs = hist_block_scale(m0, m1, smax, warp, lane);
-                        if (!hs.bad)
-#pragma unroll
-                            for (int q = 0; q < C::PP; ++q) hist_add(bins, j[q], u[q], gv[q], hs);
-                        named_sync<kBWorkers>(1);
-                        hist_flush(bins, hpart, a.lay.nint, hs, tid, kBWorkers);
-                    }
+                    // interval histogram of this tile (smax: the den/dot barrier of the next tile
+                    // separates its reads from the next writes)
+                    hist_tile<C::PP>(bins, hpart, a.lay.nint, hacc, m0, m1, smax, warp, lane, tid, j, u, gv);
                     // dQ
                     wait_or_fail(dqready, g & 1, failed, status);
                     tc_fence_after();
@@ -673,6 +699,7 @@ __global__ void __launch_bounds__(kBThreads, 1)
             if (run_tiles > 0) ++ne;
             i0 = i1;
         }
+        hist_finish(bins, hpart, a.lay.nint, hacc, tid);
         // db: sum over the rows of each warp, then over warps
 #pragma unroll
         for (int q = 0; q < C::PP; ++q) {
@@ -726,8 +753,8 @@ __global__ void __launch_bounds__(kBThreads, 1)
     int *bins = reinterpret_cast<int *>(sdz + C::D);  // fixed-point histogram of the current tile
     float *sdW = reinterpret_cast<float *>(bins + kNint * 16);
     float *sdb = sdW + C::MP * C::d;
-    float *smax = sdb + 16;               // [2][worker warps]
-    uint64_t *bars = reinterpret_cast<uint64_t *>(smax + 2 * (kBWorkers / 32));
+    float *smax = sdb + 16;               // [tile parity][2][worker warps]
+    uint64_t *bars = reinterpret_cast<uint64_t *>(smax + 4 * (kBWorkers / 32));
     uint64_t *fullk = bars;              // [NS]
     uint64_t *sfree = fullk + NS;        // [NS]
     uint64_t *fullv = sfree + NS;        // [NV]
@@ -890,6 +917,7 @@ __global__ void __launch_bounds__(kBThreads, 1)
         float db_acc[C::PP];
 #pragma unroll
         for (int q = 0; q < C::PP; ++q) db_acc[q] = 0.0f;
+        HistAcc hacc;
         int g = 0;
         for (int i0 = it.begin; i0 < it.end;) {
             const int bh = i0 / it.nchunk;
@@ -984,15 +1012,10 @@ __global__ void __launch_bounds__(kBThreads, 1)
                     fence_proxy_async_smem();
                     tc_fence_before();
                     mbar_arrive(gready + (g & 1));
-                    // interval histogram of this tile (fixed point), then into the block partial
-                    {
-                        const HistScale hs = hist_block_scale(m0, m1, smax, warp, lane);
-                        if (!hs.bad)
-#pragma unroll
-                            for (int q = 0; q < C::PP; ++q) hist_add(bins, j[q], u[q], gv[q], hs);
-                        named_sync<kBWorkers>(1);
-                        hist_flush(bins, hpart, a.lay.nint, hs, tid, kBWorkers);
-                    }
+                    // interval histogram of this tile (smax alternates by tile: no other worker
+                    // barrier separates a tile's reads from the next tile's writes)
+                    hist_tile<C::PP>(bins, hpart, a.lay.nint, hacc, m0, m1, smax + (g & 1) * 2 * (kBWorkers / 32), warp,
+                                     lane, tid, j, u, gv);
                     // dV = hi + lo
                     wait_or_fail(dvready + (g & 1), (g >> 1) & 1, failed, status);
                     tc_fence_after();
@@ -1031,6 +1054,7 @@ __global__ void __launch_bounds__(kBThreads, 1)
             }
             i0 = i1;
         }
+        hist_finish(bins, hpart, a.lay.nint, hacc, tid);
 #pragma unroll
         for (int q = 0; q < C::PP; ++q) {
             float v = db_acc[q];

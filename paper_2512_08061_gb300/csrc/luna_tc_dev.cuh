@@ -60,9 +60,14 @@ __device__ __forceinline__ void named_sync(int id) {
 // Adds a byte offset to the start-address field of a shared-memory descriptor.
 __device__ __forceinline__ uint64_t dadd(uint64_t desc, uint32_t bytes) { return desc + (bytes >> 4); }
 
-// Loads the breadth-first kink list, the interval table (float4 k of entry j
-// stored at slot j*4 + (k ^ (j & 3)), so that the rows read by a quarter warp
-// spread over all banks) and the projection bias into smem, and writes the
+// Slot of float4 k (channels 2k, 2k+1: alpha, beta, alpha, beta) of interval j
+// in the shared interval table.  Lanes read rows j at random; the XOR with bits
+// 1-2 of j spreads the 16-byte reads of a warp over all eight 16-byte bank
+// groups (bit 0 of j already selects the upper or lower half of a 128-byte line).
+__device__ __forceinline__ int ab_slot(int j, int k) { return (j << 2) | (k ^ ((j >> 1) & 3)); }
+
+// Loads the breadth-first kink list, the interval table (slots ab_slot) and the
+// projection bias into smem, and writes the
 // projection operand (NU rows x DX, K-major SW128): W split into bf16 terms
 // W_hi + W_mid (NU = 2M, about 16 significant bits) or W_hi + W_mid + W_lo and
 // M zero rows (NU = 4M, about 24 bits, as fp32).
@@ -76,7 +81,7 @@ __device__ void stage_phi_table(const AttnArgs &a, float *sTe, float *sAB, float
 #pragma unroll 4
     for (int e = tid; e < lay.nint * 4; e += nthreads) {
         const int j = e >> 2, k = e & 3;
-        reinterpret_cast<float4 *>(sAB)[(j << 2) | (k ^ (j & 3))] = AB4[e];
+        reinterpret_cast<float4 *>(sAB)[ab_slot(j, k)] = AB4[e];
     }
     const float *b = reinterpret_cast<const float *>(a.table + lay.off_b);
     for (int e = tid; e < C::MP; e += nthreads) sbias[e] = b[e];
