@@ -62,7 +62,7 @@ struct B32 {
     // key side
     static constexpr int NSK = 2, NVK = 2;
     static constexpr uint32_t SMEM_K = NSK * 2 * TILE + NVK * TILE + TILE + WOP + SOP + SOP2 + kTableBytes +
-                                       D * 4 + HIST + MP * d * 4 + 64 + 2 * SMAX + kBarBytes + 1024;
+                                       D * 4 + HIST + MP * d * 4 + 64 + SMAX + kBarBytes + 1024;
     static_assert(SMEM_Q <= kSmemLimit && SMEM_K <= kSmemLimit, "shared memory budget");
 };
 
@@ -166,21 +166,22 @@ __device__ __forceinline__ uint4 pack8(const float (&y)[8]) {
 // fall into interval j, g = dLoss/dphi on an active output.
 //
 // Shared-memory fp32 atomics are compare-and-swap loops; int32 atomics are
-// native and about five times faster.  So the bins hold fixed-point int32
-// sums: every tile finds the block-wide maxima of |g| and |g*u| and quantises
-// with power-of-two scales 2^e such that |q| < 2^16 per sample.  A bin receives
-// at most 1024 samples per tile, so up to 16 tiles fit below 2^30.  The bins
-// are added, rescaled, into the block's fp32 partial in global memory and
-// cleared ("flushed") after 16 tiles, before a tile whose maximum needs a
-// coarser scale, and at the end; the quantisation step is 2^-16 of the largest
-// value since the last flush.
+// native and about five times faster.  So the bins hold fixed-point int32 sums
+// over groups of up to 16 tiles.  The first tile of a group finds the
+// block-wide maxima of the finite |g| and |g*u| and fixes power-of-two scales
+// 2^e with |q| < 2^16 for them; a bin receives at most 1024 samples per tile,
+// so 16 tiles stay below 2^30.  A later value that does not fit (it outgrew the
+// group's first tile, or is not finite) goes, unscaled, to an fp32 atomic on
+// the block's partial in global memory instead.  At the end of a group the bins
+// are added, rescaled, into that partial and cleared.  The quantisation step is
+// 2^-16 of the group's first-tile maximum.
 //
 // Layout in shared memory: bins[(c * 8 + l) * kNint + j] (lanes with different
-// intervals fall into different banks).
+// intervals fall into different banks); the partial is [interval][channel][g, g*u].
 __device__ __forceinline__ int hist_at(int c, int l, int j) { return (c * 8 + l) * kNint + j; }
 
 constexpr int kHistQBits = 16;  // |q| < 2^16 per sample
-constexpr int kHistTiles = 16;  // tiles between flushes: 16 * 1024 * 2^16 = 2^30
+constexpr int kHistTiles = 16;  // tiles per group: 16 * 1024 * 2^16 = 2^30
 
 // 2^e as a float, e in [-126, 127] (IEEE-754 binary32: biased exponent, zero mantissa).
 __device__ __forceinline__ float pow2f(int e) { return __int_as_float((e + 127) << 23); }
@@ -193,14 +194,21 @@ __device__ __forceinline__ int hist_exp_of(float m) {
 
 // Block-uniform state of the fixed-point bins.
 struct HistAcc {
-    int e0 = 0, e1 = 0;  // exponents of the samples in the bins
-    int tiles = 0;       // tiles added since the last flush
+    int e0 = 0, e1 = 0;  // exponents of the group
+    int tiles = 0;       // tiles of the current group added so far (0: no group open)
 };
 
-// Block-wide maxima of |g| and |g*u| over the worker threads (one named barrier);
-// +inf if any value was not finite.  smax: 2 * (kBWorkers / 32) floats that no
-// worker writes again before every worker has passed its next worker barrier.
-__device__ __forceinline__ void hist_block_max(float &m0, float &m1, float *smax, int warp, int lane) {
+// Running maximum of the finite |v|.
+__device__ __forceinline__ float finite_max(float m, float v) {
+    const float a = fabsf(v);
+    return a <= 3.402823466e38f ? fmaxf(m, a) : m;
+}
+
+// Opens a group from this thread's maxima of its first tile: block-wide maxima
+// (one worker barrier; smax holds 2 * (kBWorkers / 32) floats and is next
+// written after the group's closing barrier), then the scales.  Returns false
+// (no group) when every g of the tile is zero.
+__device__ __forceinline__ bool hist_open(HistAcc &h, float m0, float m1, float *smax, int warp, int lane) {
 #pragma unroll
     for (int o = 16; o > 0; o >>= 1) {
         m0 = fmaxf(m0, __shfl_xor_sync(0xffffffffu, m0, o));
@@ -213,66 +221,51 @@ __device__ __forceinline__ void hist_block_max(float &m0, float &m1, float *smax
     m1 = 0.0f;
 #pragma unroll
     for (int w = 0; w < NW; ++w) { m0 = fmaxf(m0, smax[w]); m1 = fmaxf(m1, smax[NW + w]); }
+    if (m0 == 0.0f && m1 == 0.0f) return false;
+    h.e0 = hist_exp_of(m0 > 0.0f ? m0 : m1);
+    h.e1 = hist_exp_of(m1 > 0.0f ? m1 : m0);
+    return true;
 }
 
-// Running maximum of |v| that turns into +inf once a non-finite value is seen.
-__device__ __forceinline__ float track_max(float m, float v) {
-    const float a = fabsf(v);
-    return a <= 3.402823466e38f ? fmaxf(m, a) : __int_as_float(0x7f800000);
-}
-
-// Adds the bins, rescaled, into the block's fp32 partial ([interval][channel][g, g*u])
-// and clears them (nan: adds NaN instead); thread t of nthr handles entries t, t + nthr, ...
-__device__ __forceinline__ void hist_flush(int *bins, float *part, int nint, const HistAcc &h, bool nan, int t,
-                                           int nthr) {
-    const float inv0 = pow2f(-h.e0), inv1 = pow2f(-h.e1);
-#pragma unroll 4
-    for (int e = t; e < nint * 16; e += nthr) {
-        const int at = hist_at(e & 1, (e >> 1) & 7, e >> 4);
-        const int v = bins[at];
-        bins[at] = 0;
-        part[e] += nan ? __int_as_float(0x7fc00000) : (float)v * ((e & 1) ? inv1 : inv0);
+// Adds value v of (c, l) for a sample in interval j: int32 bin if it fits the
+// group's scale s, else an fp32 atomic on the global partial.
+__device__ __forceinline__ void hist_put(int *bins, float *part, int c, int l, int j, float v, float s) {
+    if (v != 0.0f) {
+        const float q = v * s;
+        if (fabsf(q) < (float)(1 << kHistQBits))
+            atomicAdd(bins + hist_at(c, l, j), __float2int_rn(q));
+        else
+            atomicAdd(part + ((j * 8 + l) << 1) + c, v);
     }
 }
 
-// The histogram step of one tile, for worker thread t: m0, m1 are this thread's
-// maxima of |g| and |g*u|; g[q][l] the channel values (zero where inactive) of
-// its samples u[q] in intervals j[q].
+// Adds the tile's samples (8 channel values g each, zero where inactive) to the bins.
 template <int PP>
-__device__ __forceinline__ void hist_tile(int *bins, float *part, int nint, HistAcc &h, float m0, float m1,
-                                          float *smax, int warp, int lane, int t, const int (&j)[PP],
-                                          const float (&u)[PP], const float (&g)[PP][8]) {
-    hist_block_max(m0, m1, smax, warp, lane);  // also orders every earlier tile's atomics before a flush
-    const bool bad = !(m0 <= 3.402823466e38f) || !(m1 <= 3.402823466e38f);
-    const int e0 = hist_exp_of(m0), e1 = hist_exp_of(m1);
-    if (h.tiles > 0 && (bad || e0 < h.e0 || e1 < h.e1 || h.tiles == kHistTiles)) {
-        hist_flush(bins, part, nint, h, false, t, kBWorkers);
-        named_sync<kBWorkers>(1);  // bins cleared before this tile's atomics
-        h.tiles = 0;
-    }
-    if (bad) {  // no bins in use: mark the partial
-        hist_flush(bins, part, nint, h, true, t, kBWorkers);
-        return;
-    }
-    if (h.tiles == 0) { h.e0 = e0; h.e1 = e1; }
+__device__ __forceinline__ void hist_add(int *bins, float *part, const HistAcc &h, const int (&j)[PP],
+                                         const float (&u)[PP], const float (&g)[PP][8]) {
     const float s0 = pow2f(h.e0), s1 = pow2f(h.e1);
 #pragma unroll
     for (int q = 0; q < PP; ++q)
 #pragma unroll
         for (int l = 0; l < 8; ++l) {
-            if (g[q][l] != 0.0f) {
-                atomicAdd(bins + hist_at(0, l, j[q]), __float2int_rn(g[q][l] * s0));
-                atomicAdd(bins + hist_at(1, l, j[q]), __float2int_rn(g[q][l] * u[q] * s1));
-            }
+            hist_put(bins, part, 0, l, j[q], g[q][l], s0);
+            hist_put(bins, part, 1, l, j[q], g[q][l] * u[q], s1);
         }
-    ++h.tiles;
 }
 
-// Final flush of the bins after the last tile of the block.
-__device__ __forceinline__ void hist_finish(int *bins, float *part, int nint, const HistAcc &h, int t) {
-    if (h.tiles == 0) return;
-    named_sync<kBWorkers>(1);  // every atomic done
-    hist_flush(bins, part, nint, h, false, t, kBWorkers);
+// Closes the group: after a worker barrier (every atomic done), adds the bins,
+// rescaled, into the partial and clears them; thread t handles entries t, t + kBWorkers, ...
+__device__ __forceinline__ void hist_close(int *bins, float *part, int nint, HistAcc &h, int t) {
+    named_sync<kBWorkers>(1);
+    const float inv0 = pow2f(-h.e0), inv1 = pow2f(-h.e1);
+#pragma unroll 4
+    for (int e = t; e < nint * 16; e += kBWorkers) {
+        const int at = hist_at(e & 1, (e >> 1) & 7, e >> 4);
+        const int v = bins[at];
+        bins[at] = 0;
+        part[e] = __ldcg(part + e) + (float)v * ((e & 1) ? inv1 : inv0);  // L2 copy: fp32 atomics went there
+    }
+    h.tiles = 0;
 }
 
 // Zeroes a row of a 128-row x 128 B tile (padded rows must not carry garbage
@@ -560,8 +553,33 @@ __global__ void __launch_bounds__(kBThreads, 1)
                     const float inv = live ? 1.0f / den : 0.0f;
                     const float ndot = live ? -dotn * inv : 0.0f;  // -(dO.O)
                     const float dden = ndot * inv;
+                    // first tile of a histogram group: the maxima of |g| and |g*u| fix its scales
+                    bool hon = hacc.tiles > 0;
+                    if (!hon) {
+                        float m0 = 0.0f, m1 = 0.0f;
+#pragma unroll
+                        for (int q = 0; q < C::PP; ++q) {
+                            const int i = H * C::PP + q;
+                            float al[8], y[8];
+                            channel_eval(sAB, j[q], u[q], al, y);
+                            uint32_t ph[8], pl[8];
+                            tmem_ld8(pcol + 8 * i, ph);
+                            tmem_ld8(pcol + C::D + 8 * i, pl);
+                            tmem_wait_ld();
+#pragma unroll
+                            for (int l = 0; l < 8; ++l) {
+                                const float dphi = live ? (__uint_as_float(ph[l]) + __uint_as_float(pl[l])) * inv +
+                                                              sz[8 * i + l] * dden
+                                                        : 0.0f;
+                                const float gl = y[l] > 0.0f ? dphi : 0.0f;
+                                m0 = finite_max(m0, gl);
+                                m1 = finite_max(m1, gl * u[q]);
+                            }
+                        }
+                        hon = hist_open(hacc, m0, m1, smax, warp, lane);
+                    }
                     // gradients through the feature map; phi/den (bf16) for the stacked contraction
-                    float dU[C::PP], gv[C::PP][8], m0 = 0.0f, m1 = 0.0f;
+                    float dU[C::PP], gv[C::PP][8];
 #pragma unroll
                     for (int q = 0; q < C::PP; ++q) {
                         const int i = H * C::PP + q;
@@ -593,8 +611,6 @@ __global__ void __launch_bounds__(kBThreads, 1)
                             const float gl = y[l] > 0.0f ? dphi : 0.0f;  // through the outer ReLU
                             gv[q][l] = gl;
                             du = fmaf(gl, al[l], du);
-                            m0 = track_max(m0, gl);
-                            m1 = track_max(m1, gl * u[q]);
                         }
                         dU[q] = du;
                         db_acc[q] += du;
@@ -619,9 +635,10 @@ __global__ void __launch_bounds__(kBThreads, 1)
                     fence_proxy_async_smem();
                     tc_fence_before();
                     mbar_arrive(gready + (g & 1));
-                    // interval histogram of this tile (smax: the den/dot barrier of the next tile
-                    // separates its reads from the next writes)
-                    hist_tile<C::PP>(bins, hpart, a.lay.nint, hacc, m0, m1, smax, warp, lane, tid, j, u, gv);
+                    if (hon) {  // interval histogram (after the MMA warp has its operands)
+                        hist_add<C::PP>(bins, hpart, hacc, j, u, gv);
+                        if (++hacc.tiles == kHistTiles) hist_close(bins, hpart, a.lay.nint, hacc, tid);
+                    }
                     // dQ
                     wait_or_fail(dqready, g & 1, failed, status);
                     tc_fence_after();
@@ -699,7 +716,7 @@ __global__ void __launch_bounds__(kBThreads, 1)
             if (run_tiles > 0) ++ne;
             i0 = i1;
         }
-        hist_finish(bins, hpart, a.lay.nint, hacc, tid);
+        if (hacc.tiles > 0) hist_close(bins, hpart, a.lay.nint, hacc, tid);
         // db: sum over the rows of each warp, then over warps
 #pragma unroll
         for (int q = 0; q < C::PP; ++q) {
@@ -753,8 +770,8 @@ __global__ void __launch_bounds__(kBThreads, 1)
     int *bins = reinterpret_cast<int *>(sdz + C::D);  // fixed-point histogram of the current tile
     float *sdW = reinterpret_cast<float *>(bins + kNint * 16);
     float *sdb = sdW + C::MP * C::d;
-    float *smax = sdb + 16;               // [tile parity][2][worker warps]
-    uint64_t *bars = reinterpret_cast<uint64_t *>(smax + 4 * (kBWorkers / 32));
+    float *smax = sdb + 16;               // [2][worker warps]
+    uint64_t *bars = reinterpret_cast<uint64_t *>(smax + 2 * (kBWorkers / 32));
     uint64_t *fullk = bars;              // [NS]
     uint64_t *sfree = fullk + NS;        // [NS]
     uint64_t *fullv = sfree + NS;        // [NV]
@@ -978,7 +995,30 @@ __global__ void __launch_bounds__(kBThreads, 1)
                     wait_or_fail(fready + (g & 1), (g >> 1) & 1, failed, status);
                     tc_fence_after();
                     const uint32_t fcol = tbase + lrow + cF + (g & 1) * 128;
-                    float dU[C::PP], gv[C::PP][8], m0 = 0.0f, m1 = 0.0f;
+                    // first tile of a histogram group: the maxima of |g| and |g*u| fix its scales
+                    bool hon = hacc.tiles > 0;
+                    if (!hon) {
+                        float m0 = 0.0f, m1 = 0.0f;
+#pragma unroll
+                        for (int q = 0; q < C::PP; ++q) {
+                            const int i = H * C::PP + q;
+                            float al[8], y[8];
+                            channel_eval(sAB, j[q], u[q], al, y);
+                            uint32_t ph[8], pl[8];
+                            tmem_ld8(fcol + 8 * i, ph);
+                            tmem_ld8(fcol + C::D + 8 * i, pl);
+                            tmem_wait_ld();
+#pragma unroll
+                            for (int l = 0; l < 8; ++l) {
+                                const float dphi = __uint_as_float(ph[l]) + __uint_as_float(pl[l]) + sdz[8 * i + l];
+                                const float gl = (valid && y[l] > 0.0f) ? dphi : 0.0f;
+                                m0 = finite_max(m0, gl);
+                                m1 = finite_max(m1, gl * u[q]);
+                            }
+                        }
+                        hon = hist_open(hacc, m0, m1, smax, warp, lane);
+                    }
+                    float dU[C::PP], gv[C::PP][8];
 #pragma unroll
                     for (int q = 0; q < C::PP; ++q) {
                         const int i = H * C::PP + q;
@@ -995,8 +1035,6 @@ __global__ void __launch_bounds__(kBThreads, 1)
                             const float gl = (valid && y[l] > 0.0f) ? dphi : 0.0f;
                             gv[q][l] = gl;
                             du = fmaf(gl, al[l], du);
-                            m0 = track_max(m0, gl);
-                            m1 = track_max(m1, gl * u[q]);
                         }
                         dU[q] = du;
                         db_acc[q] += du;
@@ -1012,10 +1050,10 @@ __global__ void __launch_bounds__(kBThreads, 1)
                     fence_proxy_async_smem();
                     tc_fence_before();
                     mbar_arrive(gready + (g & 1));
-                    // interval histogram of this tile (smax alternates by tile: no other worker
-                    // barrier separates a tile's reads from the next tile's writes)
-                    hist_tile<C::PP>(bins, hpart, a.lay.nint, hacc, m0, m1, smax + (g & 1) * 2 * (kBWorkers / 32), warp,
-                                     lane, tid, j, u, gv);
+                    if (hon) {  // interval histogram (after the MMA warp has its operands)
+                        hist_add<C::PP>(bins, hpart, hacc, j, u, gv);
+                        if (++hacc.tiles == kHistTiles) hist_close(bins, hpart, a.lay.nint, hacc, tid);
+                    }
                     // dV = hi + lo
                     wait_or_fail(dvready + (g & 1), (g >> 1) & 1, failed, status);
                     tc_fence_after();
@@ -1054,7 +1092,7 @@ __global__ void __launch_bounds__(kBThreads, 1)
             }
             i0 = i1;
         }
-        hist_finish(bins, hpart, a.lay.nint, hacc, tid);
+        if (hacc.tiles > 0) hist_close(bins, hpart, a.lay.nint, hacc, tid);
 #pragma unroll
         for (int q = 0; q < C::PP; ++q) {
             float v = db_acc[q];
