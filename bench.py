@@ -19,6 +19,7 @@ bounded sample of the same workload.
 from __future__ import annotations
 
 import argparse
+import hashlib
 import json
 import math
 import os
@@ -94,6 +95,40 @@ def kernel_bytes(w, lengths, kernel: str) -> float:
                         ("tc_bwd_key", "bwd_key")):
         table[tc] = table[generic]
     return float(table.get(kernel, 0.0))
+
+
+def csrc_digest() -> str:
+    """sha256 over the CUDA sources of the library (file names and contents)."""
+    h = hashlib.sha256()
+    base = os.path.join(ROOT, "paper_2512_08061_gb300", "csrc")
+    for f in sorted(os.listdir(base)):
+        if f.endswith((".cu", ".cuh")):
+            h.update(f.encode())
+            with open(os.path.join(base, f), "rb") as fh:
+                h.update(fh.read())
+    return h.hexdigest()
+
+
+def measured_traffic(kernel: str, workload: str):
+    """DRAM bytes (read + write) per launch of `kernel` from the committed ncu
+    summaries (lines `traffic <workload> k_<kernel> <bytes> <sources sha256>`),
+    or None when no summary was taken on the current sources."""
+    pdir = os.path.join(ROOT, "profiles")
+    digest = csrc_digest()
+    try:
+        names = sorted(os.listdir(pdir))
+    except OSError:
+        return None, None
+    for f in names:
+        if not f.endswith(".md"):
+            continue
+        with open(os.path.join(pdir, f)) as fh:
+            for line in fh:
+                parts = line.strip().strip("`").split()
+                if len(parts) == 5 and parts[0] == "traffic" and parts[1] == workload and parts[2] == "k_" + kernel:
+                    if parts[4] == digest:
+                        return float(parts[3]), "profiles/" + f
+    return None, None
 
 
 def step_bytes(w, lengths) -> float:
@@ -310,9 +345,10 @@ def run_gpu(args, w):
         byts = kernel_bytes(w, lengths, dominant)
         dur = dom_ms / dom_n * 1e-3
         achieved = byts / dur / 1e9 if byts else None
+        traffic, traffic_src = measured_traffic(dominant, w.name)
         roof = {"bound": "hbm", "kernel": dominant, "achieved": achieved, "peak": hbm, "unit": "GB/s",
-                "frac": (achieved / hbm) if achieved else None, "traffic": None, "peak_source": peak_src,
-                "algorithmic_bytes": byts, "launch_ms": dom_ms / dom_n, "launches": dom_n}
+                "frac": (achieved / hbm) if achieved else None, "traffic": traffic, "traffic_source": traffic_src,
+                "peak_source": peak_src, "algorithmic_bytes": byts, "launch_ms": dom_ms / dom_n, "launches": dom_n}
     sb, sf = step_bytes(w, lengths), step_flops(w, lengths)
     t_roof = max(sb / (hbm * 1e9), sf / (tflops * 1e12))
     result = {
