@@ -36,68 +36,88 @@ __device__ float down_threshold(float w, float c) {
     return t;
 }
 
-// Every block recomputes the thresholds and their ranks (512 x 512 compares)
-// and then fills its slice of the (interval, channel) table; block 0 also
-// writes the kink lists, the ranks and the parameter copies.  Per-unit values
-// are kept in shared memory in [k][l] order, so that the eight channels read by
-// a warp fall into eight consecutive banks.
-constexpr int kPrepThreads = 256;
+// One launch: every block computes the kink threshold of every hidden unit and
+// sorts the (threshold, unit index) pairs (a bitonic network over one element
+// per thread: warp shuffles for partners within a warp, shared memory across
+// warps; a stable total order), then computes its slice of alpha and beta,
+// eight threads per (interval, channel) entry; block 0 also writes the sorted
+// and breadth-first kink lists, each unit's rank and active side, and the
+// parameter copies.
+constexpr int kPrepThreads = kMaxUnits;                       // one thread per (padded) unit
+constexpr int kPrepSplit = 8;                                 // threads per (interval, channel) entry
+constexpr int kPrepEntries = kPrepThreads / kPrepSplit;       // entries per block
+
+__device__ __forceinline__ bool pair_less(float ta, int ka, float tb, int kb) {
+    return ta < tb || (ta == tb && ka < kb);
+}
 
 __global__ void __launch_bounds__(kPrepThreads) k_phi_prepare(luna_phi_params prm, TableLayout lay, char *table) {
-    __shared__ float th[kMaxUnits];
-    __shared__ int ty[kMaxUnits];
-    __shared__ int rk[kMaxUnits];
-    __shared__ float w1t[kMaxUnits], b1t[kMaxUnits], w2t[kMaxUnits];  // [k][l]
-    __shared__ int tyt[kMaxUnits], rkt[kMaxUnits];                     // [k][l]
-    __shared__ float srt[kMaxUnits];                                   // thresholds in sorted order
+    __shared__ float sk[kMaxUnits];
+    __shared__ int si[kMaxUnits];
+    __shared__ float w1t[kMaxUnits], b1t[kMaxUnits], w2t[kMaxUnits];  // per-unit values in [k][l] order
+    __shared__ int tyt[kMaxUnits], rkt[kMaxUnits];
     const int tid = threadIdx.x, nt = blockDim.x;
-    const int P = lay.P, L = lay.L, hid = lay.hid;
-
-    for (int k = tid; k < P; k += nt) {
-        const float w = prm.w1[k], c = prm.b1[k];
-        if (w > 0.0f) { th[k] = up_threshold(w, c); ty[k] = 1; }
-        else if (w < 0.0f) { th[k] = down_threshold(w, c); ty[k] = -1; }
-        else { th[k] = INFINITY; ty[k] = (c > 0.0f) ? -1 : 1; }  // constant unit: always on / always off
+    const int P = lay.P, N = lay.Ppad, L = lay.L, hid = lay.hid;  // N: power of two >= P, <= kMaxUnits
+    float key = INFINITY;  // this thread's element: unit tid, padding (+inf, index >= P) sorts last
+    int idx = tid;
+    if (tid < P) {
+        const float w = prm.w1[tid], c = prm.b1[tid];
+        int ty;
+        if (w > 0.0f) { key = up_threshold(w, c); ty = 1; }
+        else if (w < 0.0f) { key = down_threshold(w, c); ty = -1; }
+        else { key = INFINITY; ty = (c > 0.0f) ? -1 : 1; }  // constant unit: always on / always off
+        const int tpos = (tid % hid) * L + tid / hid;
+        w1t[tpos] = w; b1t[tpos] = c; w2t[tpos] = prm.w2[tid]; tyt[tpos] = ty;
     }
-    __syncthreads();
-    // rank by (threshold, unit index): a stable total order
-    for (int k = tid; k < P; k += nt) {
-        const float t = th[k];
-        int r = 0;
-        for (int q = 0; q < P; ++q) {
-            const float sq = th[q];
-            r += (sq < t || (sq == t && q < k)) ? 1 : 0;
+    // bitonic sort of the first N elements (positions >= N sort among themselves)
+    for (int size = 2; size <= N; size <<= 1) {
+        for (int stride = size >> 1; stride > 0; stride >>= 1) {
+            float pk;
+            int pi;
+            if (stride >= 32) {
+                sk[tid] = key; si[tid] = idx;
+                __syncthreads();
+                pk = sk[tid ^ stride]; pi = si[tid ^ stride];
+                __syncthreads();
+            } else {
+                pk = __shfl_xor_sync(0xffffffffu, key, stride);
+                pi = __shfl_xor_sync(0xffffffffu, idx, stride);
+            }
+            // the lower position of a pair keeps the smaller element in an ascending
+            // run (the larger in a descending one); elements are distinct
+            const bool keep_min = ((tid & stride) == 0) == ((tid & size) == 0);
+            if (pair_less(pk, pi, key, idx) == keep_min) { key = pk; idx = pi; }
         }
-        rk[k] = r;
-        srt[r] = t;
-        const int l = k / hid, kk = k % hid, tpos = kk * L + l;
-        w1t[tpos] = prm.w1[k]; b1t[tpos] = prm.b1[k]; w2t[tpos] = prm.w2[k];
-        tyt[tpos] = ty[k]; rkt[tpos] = r;
     }
+    sk[tid] = key;
+    si[tid] = idx;
+    if (idx < P) rkt[(idx % hid) * L + idx / hid] = tid;
     __syncthreads();
 
-    float *T = reinterpret_cast<float *>(table + lay.off_T);
     if (blockIdx.x == 0) {
+        float *T = reinterpret_cast<float *>(table + lay.off_T);
         int *rank = reinterpret_cast<int *>(table + lay.off_rank);
         int *utype = reinterpret_cast<int *>(table + lay.off_utype);
-        for (int k = tid; k < P; k += nt) {
-            T[rk[k]] = th[k];
-            rank[k] = rk[k];
-            utype[k] = ty[k];
-            reinterpret_cast<float *>(table + lay.off_w1)[k] = prm.w1[k];
-            reinterpret_cast<float *>(table + lay.off_b1)[k] = prm.b1[k];
-            reinterpret_cast<float *>(table + lay.off_w2)[k] = prm.w2[k];
+        for (int r = tid; r < N; r += nt) {
+            T[r] = sk[r];  // sorted kinks, +inf padding
+            if (si[r] < P) rank[si[r]] = r;
         }
-        for (int p = P + tid; p < lay.Ppad; p += nt) T[p] = INFINITY;
-        // breadth-first (Eytzinger) copy: node e at depth d, position p in its
-        // level holds the in-order element (2p+1) * 2^(9-d) - 1
+        for (int k = tid; k < P; k += nt) {
+            const int tpos = (k % hid) * L + k / hid;
+            utype[k] = tyt[tpos];
+            reinterpret_cast<float *>(table + lay.off_w1)[k] = w1t[tpos];
+            reinterpret_cast<float *>(table + lay.off_b1)[k] = b1t[tpos];
+            reinterpret_cast<float *>(table + lay.off_w2)[k] = w2t[tpos];
+        }
+        // breadth-first (Eytzinger) copy: node e at depth d, position p in its level
+        // holds the in-order element (2p+1) * 2^(9-d) - 1
         float *Te = reinterpret_cast<float *>(table + lay.off_Te);
         for (int e = tid; e < kEytzinger; e += nt) {
             float v = INFINITY;
             if (e > 0) {
                 const int d = 31 - __clz(e);
                 const int idx = ((2 * (e - (1 << d)) + 1) << (9 - d)) - 1;
-                if (idx < P) v = srt[idx];
+                if (idx < P) v = sk[idx];
             }
             Te[e] = v;
         }
@@ -111,13 +131,18 @@ __global__ void __launch_bounds__(kPrepThreads) k_phi_prepare(luna_phi_params pr
             h->M = lay.M; h->L = lay.L; h->hid = lay.hid; h->d = lay.d; h->P = P; h->Ppad = lay.Ppad;
         }
     }
-    // alpha, beta of every (interval j, channel l), scaled by 1/sqrt(M)
+    // alpha, beta of (interval j, channel l), scaled by 1/sqrt(M): thread p of the
+    // entry's eight sums units k = p, p + 8, ... in order, then the eight partial
+    // sums are added in a fixed tree order.
     float *AB = reinterpret_cast<float *>(table + lay.off_AB);
     const float scale = 1.0f / sqrtf((float)lay.M);
-    for (int e = blockIdx.x * nt + tid; e < lay.nint * L; e += gridDim.x * nt) {
-        const int j = e / L, l = e % L;
-        float a = 0.0f, bsum = prm.b2[l];
-        for (int k = 0; k < hid; ++k) {
+    const int p = tid % kPrepSplit;
+    for (int e0 = blockIdx.x * kPrepEntries; e0 < lay.nint * L; e0 += gridDim.x * kPrepEntries) {
+        const int e = e0 + tid / kPrepSplit;
+        const bool live = e < lay.nint * L;
+        const int j = live ? e / L : 0, l = live ? e % L : 0;
+        float a = 0.0f, bsum = 0.0f;
+        for (int k = p; k < hid; k += kPrepSplit) {
             const int u = k * L + l;
             const bool on = (tyt[u] > 0) ? (rkt[u] < j) : (rkt[u] >= j);
             if (on) {
@@ -125,15 +150,22 @@ __global__ void __launch_bounds__(kPrepThreads) k_phi_prepare(luna_phi_params pr
                 bsum = fmaf(w2t[u], b1t[u], bsum);
             }
         }
-        AB[2 * e] = a * scale;
-        AB[2 * e + 1] = bsum * scale;
+#pragma unroll
+        for (int o = 1; o < kPrepSplit; o <<= 1) {
+            a += __shfl_xor_sync(0xffffffffu, a, o);
+            bsum += __shfl_xor_sync(0xffffffffu, bsum, o);
+        }
+        if (live && p == 0) {
+            AB[2 * e] = a * scale;
+            AB[2 * e + 1] = (bsum + prm.b2[l]) * scale;
+        }
     }
 }
 
 }  // namespace
 
 cudaError_t launch_phi_prepare(const luna_phi_params &prm, const TableLayout &lay, void *table, cudaStream_t s) {
-    const int blocks = (lay.nint * lay.L + kPrepThreads - 1) / kPrepThreads;
+    const int blocks = (lay.nint * lay.L + kPrepEntries - 1) / kPrepEntries;
     LUNA_LAUNCH("phi_prepare", k_phi_prepare, blocks, kPrepThreads, 0, s, prm, lay, static_cast<char *>(table));
     return cudaGetLastError();
 }
