@@ -3,6 +3,7 @@
 #include <string.h>
 
 #include <algorithm>
+#include <stdlib.h>
 
 #include "luna_simt.cuh"
 #include "luna_tc.cuh"
@@ -76,7 +77,11 @@ luna_status make_plan(const luna_attn_desc *ad, const luna_phi_desc *pd, Plan &p
         p.rps_b = (int)round_up(cdiv(n, nb), 16);
         p.nsplit_b = (int)cdiv(n, p.rps_b);
         int64_t nc = std::min<int64_t>(std::min<int64_t>(target, 64), cdiv(n, 16));
-        p.seg_len = (int)round_up(cdiv(n, nc), 64);
+        p.seg_len = (int)round_up(cdiv(n, nc), 128);  // whole 128-row tiles (tensor-core streaming form)
+        if (const char *env = getenv("LUNA_CAUSAL_SEG_ROWS")) {  // tuning and tests: fixed segment length
+            const long v = atol(env);
+            if (v >= 128 && v % 128 == 0 && v < (1L << 24)) p.seg_len = (int)v;
+        }
         p.nseg = (int)cdiv(n, p.seg_len);
     }
     const size_t f = sizeof(float);
@@ -261,7 +266,10 @@ luna_status luna_attn_fwd(const luna_attn_desc *ad, const luna_phi_desc *pd, con
         return LUNA_ERR_UNSUPPORTED;
     cudaError_t e = cudaMemsetAsync(workspace, 0, p.o_counters + 2 * sizeof(int) * (size_t)p.BH, s);
     if (e != cudaSuccess) return LUNA_ERR_CUDA;
-    if (ad->causal) return cuda_status(launch_causal_fwd(a, ad->io, state != nullptr, s));
+    if (ad->causal) {
+        if (p.tc.causal_fwd && tc_inputs_ok(TcPlan{true}, Q, K, V, O)) return cuda_status(launch_tc_causal_fwd(a, s));
+        return cuda_status(launch_causal_fwd(a, ad->io, state != nullptr, s));
+    }
     if (p.tc.eligible && tc_inputs_ok(p.tc, Q, K, V, O))
         return cuda_status(launch_tc_fwd(p.tc, a, static_cast<char *>(workspace), s));
     return cuda_status(launch_simt_fwd(a, ad->io, s));

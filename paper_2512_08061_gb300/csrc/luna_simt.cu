@@ -328,11 +328,11 @@ __global__ void __launch_bounds__(kThreads) k_bwd_key(AttnArgs a) {
 constexpr int kSumElems = 64, kSumSplit = 4;
 __global__ void __launch_bounds__(kSumElems * kSumSplit) k_grad_sum(const float *gpart, int nparts, int gsize,
                                                                     float *out) {
-    __shared__ float part[kSumSplit][kSumElems];
+    __shared__ double part[kSumSplit][kSumElems];
     const int el = threadIdx.x % kSumElems, q = threadIdx.x / kSumElems;
     const int e = blockIdx.x * kSumElems + el;
     const int p0 = (int)((long long)q * nparts / kSumSplit), p1 = (int)((long long)(q + 1) * nparts / kSumSplit);
-    float s = 0.0f;
+    double s = 0.0;
     if (e < gsize) {
         int p = p0;
         for (; p + 8 <= p1; p += 8) {
@@ -347,30 +347,30 @@ __global__ void __launch_bounds__(kSumElems * kSumSplit) k_grad_sum(const float 
     part[q][el] = s;
     __syncthreads();
     if (q == 0 && e < gsize) {
-        float t = part[0][el];
+        double t = part[0][el];
 #pragma unroll
         for (int k = 1; k < kSumSplit; ++k) t += part[k][el];
-        out[e] = t;
+        out[e] = (float)t;
     }
 }
 
-// Inclusive scan of x[0..n) into y (forward: prefix sums; backward: suffix sums)
+// Inclusive scan of x[0..n) into y (forward: prefix sums; backward: suffix sums), accumulated in fp64,
 // by one warp, in a fixed order: lane c sums a contiguous chunk, the chunk totals
 // are scanned across lanes, then every lane writes its chunk.
-__device__ void warp_scan(const float *x, float *y, int n, bool backward) {
+__device__ void warp_scan(const float *x, double *y, int n, bool backward) {
     const int lane = threadIdx.x & 31;
     const int chunk = (n + 31) / 32;
     const int b = lane * chunk, e = min(n, b + chunk);
     auto at = [&](int i) { return backward ? n - 1 - i : i; };
-    float t = 0.0f;
+    double t = 0.0;  // fp64: the sums over intervals cancel
     for (int i = b; i < e; ++i) t += x[at(i)];
-    float incl = t;
+    double incl = t;
 #pragma unroll
     for (int o = 1; o < 32; o <<= 1) {
-        const float v = __shfl_up_sync(0xffffffffu, incl, o);
+        const double v = __shfl_up_sync(0xffffffffu, incl, o);
         if (lane >= o) incl += v;
     }
-    float run = incl - t;  // exclusive prefix of this chunk
+    double run = incl - t;  // exclusive prefix of this chunk
     for (int i = b; i < e; ++i) {
         run += x[at(i)];
         y[at(i)] = run;
@@ -381,7 +381,8 @@ __device__ void warp_scan(const float *x, float *y, int n, bool backward) {
 // channel's interval histogram.  Block L: dW and db.
 __global__ void __launch_bounds__(128) k_mlp_grads(TableLayout lay, const char *table, const float *gsum,
                                                    luna_phi_grads grads) {
-    __shared__ float h[2][kMaxUnits + 1], pre[2][kMaxUnits + 1], suf[2][kMaxUnits + 1];
+    __shared__ float h[2][kMaxUnits + 1];
+    __shared__ double pre[2][kMaxUnits + 1], suf[2][kMaxUnits + 1];  // fp64: dw2 = w1 G1 + b1 G0 cancels
     const int Md = lay.M * lay.d, L = lay.L, hid = lay.hid, nint = lay.nint;
     const float scale = 1.0f / sqrtf((float)lay.M);
     if ((int)blockIdx.x == L) {
@@ -407,19 +408,19 @@ __global__ void __launch_bounds__(128) k_mlp_grads(TableLayout lay, const char *
     for (int k = threadIdx.x; k < hid; k += blockDim.x) {
         const int u = l * hid + k;
         const int r = rank[u];
-        float G0, G1;
+        double G0, G1;
         if (utype[u] > 0) {  // active on intervals j > r
-            G0 = r + 1 < nint ? suf[0][r + 1] : 0.0f;
-            G1 = r + 1 < nint ? suf[1][r + 1] : 0.0f;
+            G0 = r + 1 < nint ? suf[0][r + 1] : 0.0;
+            G1 = r + 1 < nint ? suf[1][r + 1] : 0.0;
         } else {             // active on intervals j <= r
             G0 = pre[0][r];
             G1 = pre[1][r];
         }
-        grads.dw2[u] = (w1[u] * G1 + b1[u] * G0) * scale;
-        grads.dw1[u] = w2[u] * G1 * scale;
-        grads.db1[u] = w2[u] * G0 * scale;
+        grads.dw2[u] = (float)(((double)w1[u] * G1 + (double)b1[u] * G0) * (double)scale);
+        grads.dw1[u] = (float)((double)w2[u] * G1 * (double)scale);
+        grads.db1[u] = (float)((double)w2[u] * G0 * (double)scale);
     }
-    if (threadIdx.x == 0) grads.db2[l] = pre[0][nint - 1] * scale;
+    if (threadIdx.x == 0) grads.db2[l] = (float)(pre[0][nint - 1] * (double)scale);
 }
 
 // ---------------------------------------------------------------------------

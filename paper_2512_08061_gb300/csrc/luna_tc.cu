@@ -183,9 +183,11 @@ __device__ __forceinline__ void issue_proj(uint32_t tmem_u, uint64_t dx, uint64_
 // phi(K) enters the contraction as bf16 hi + lo tiles so that the key
 // statistics carry ~16 significant bits of phi (the backward pass subtracts
 // nearly equal terms built from S and z); z is summed by the workers in fp32.
-// Each item's statistics go to its partial slot; the last chunk of a head to
-// finish sums the partials in chunk order (warps 0..3 only, so that the
-// pipeline keeps running).
+// Each run's statistics go to its partial slot; the last run of a head to
+// finish sums the partials in order (warps 0..3 only, so that the pipeline
+// keeps running).  Per-item mode (the state segments of the streaming form,
+// a.seg_S set): every item is its own run, its statistics go to slot
+// (head, item), and nothing is summed here.
 
 template <class C>
 __global__ void __launch_bounds__(kThreadsTC, 1)
@@ -218,6 +220,7 @@ __global__ void __launch_bounds__(kThreadsTC, 1)
 
     const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
     const Items it(a);
+    const bool per_item = a.seg_S != nullptr;
 
     if (tid == 0) {
         for (int i = 0; i < NX; ++i) { mbar_init(fullx + i, 1); mbar_init(xfree + i, 1); }
@@ -280,7 +283,7 @@ __global__ void __launch_bounds__(kThreadsTC, 1)
             int g = 0, ne = 0;
             for (int i0 = it.begin; i0 < it.end && !failed;) {
                 const int bh = i0 / it.nchunk;
-                const int i1 = min(it.end, (bh + 1) * it.nchunk);
+                const int i1 = per_item ? i0 + 1 : min(it.end, (bh + 1) * it.nchunk);
                 int run_tiles = 0;
                 for (int i = i0; i < i1; ++i) run_tiles += item_range(a, it, i).ntiles;
                 if (run_tiles > 0) {
@@ -323,7 +326,7 @@ __global__ void __launch_bounds__(kThreadsTC, 1)
         int g = 0, ne = 0;
         for (int i0 = it.begin; i0 < it.end;) {
             const int bh = i0 / it.nchunk;
-            const int i1 = min(it.end, (bh + 1) * it.nchunk);
+            const int i1 = per_item ? i0 + 1 : min(it.end, (bh + 1) * it.nchunk);
             int run_tiles = 0;
             for (int item = i0; item < i1; ++item) {
                 const ItemRange ir = item_range(a, it, item);
@@ -368,7 +371,7 @@ __global__ void __launch_bounds__(kThreadsTC, 1)
                 const int c_first = owner_block((long long)bh * it.nchunk, it.total, gridDim.x);
                 const int c_last = owner_block((long long)(bh + 1) * it.nchunk - 1, it.total, gridDim.x);
                 const int nruns = c_last - c_first + 1;
-                const size_t slot = (size_t)bh * it.nchunk + (blockIdx.x - c_first);
+                const size_t slot = per_item ? (size_t)i0 : (size_t)bh * it.nchunk + (blockIdx.x - c_first);
                 float *Sp = a.S_part + slot * C::D * C::DV;
                 float *zp = a.z_part + slot * C::D;
                 const int row = (warp << 5) | lane;
@@ -418,7 +421,7 @@ __global__ void __launch_bounds__(kThreadsTC, 1)
                 // the last block of this head to finish sums the partials in block order
                 __threadfence();
                 named_sync<128>(2);
-                if (tid == 0) *slast = (atomicAdd(a.counters + bh, 1) == nruns - 1) ? 1 : 0;
+                if (tid == 0) *slast = (!per_item && atomicAdd(a.counters + bh, 1) == nruns - 1) ? 1 : 0;
                 named_sync<128>(2);
                 if (*slast) {
                     __threadfence();
@@ -756,6 +759,11 @@ TcPlan tc_plan(const luna_attn_desc &ad, const TableLayout &lay) {
     p.variant = variant(ad, lay);
     p.eligible = p.variant >= 0 && encoder() != nullptr;
     p.bwd = p.eligible && tc_bwd_supported(ad, lay);
+    if (ad.causal) {
+        luna_attn_desc nc = ad;
+        nc.causal = 0;
+        p.causal_fwd = encoder() != nullptr && variant(nc, lay) >= 0 && tc_causal_supported(ad, lay);
+    }
     return p;
 }
 
@@ -769,6 +777,16 @@ cudaError_t launch_tc_fwd(const TcPlan &p, const AttnArgs &a, char *, cudaStream
         case 0: return fwd_tc<C32>(a, s);
         case 1: return fwd_tc<C64>(a, s);
         case 2: return fwd_tc<C128>(a, s);
+    }
+    return cudaErrorNotSupported;
+}
+
+cudaError_t launch_tc_keys_items(const AttnArgs &a, cudaStream_t s) {
+    const TcPlan p = tc_plan(luna_attn_desc{a.B, a.H, a.n, a.d, a.dv, 0, 0, a.eps, LUNA_BF16}, a.lay);
+    switch (p.variant) {
+        case 0: return keys_tc<C32>(a, s);
+        case 1: return keys_tc<C64>(a, s);
+        case 2: return keys_tc<C128>(a, s);
     }
     return cudaErrorNotSupported;
 }

@@ -9,6 +9,7 @@ struct TcPlan {
     bool eligible = false;   // shape and dtype handled by the tensor-core kernels
     int variant = -1;        // kernel instantiation (value width / projections)
     bool bwd = false;        // backward also on tensor cores
+    bool causal_fwd = false; // streaming-form forward on tensor cores
     size_t ws_fwd = 0, ws_bwd = 0;
 };
 
@@ -20,5 +21,9 @@ cudaError_t launch_tc_stats(const AttnArgs &a, cudaStream_t s);
 bool tc_bwd_supported(const luna_attn_desc &ad, const TableLayout &lay);
 bool tc_bwd_fits(const AttnArgs &a);
 cudaError_t launch_tc_bwd_kernels(const AttnArgs &a, bool have_stats, cudaStream_t s);
+// key statistics of every work item (a.rows_per_split rows, a.nsplit per head) into S_part, z_part
+cudaError_t launch_tc_keys_items(const AttnArgs &a, cudaStream_t s);
+bool tc_causal_supported(const luna_attn_desc &ad, const TableLayout &lay);
+cudaError_t launch_tc_causal_fwd(const AttnArgs &a, cudaStream_t s);
 
 }  // namespace luna

@@ -24,6 +24,23 @@ def relerr(got, ref) -> float:
     return float(np.max(np.abs(g - r) / np.maximum(np.abs(r), rms)))
 
 
+def relerr_rows(got, ref) -> float:
+    """max_i |g_i - r_i| / max(|r_i|, rms of r_i's row): the element-wise
+    relative error floored at the rms of its row (last axis).  Used for outputs
+    of the streaming form, where every row is its own normalised average of the
+    values and the first rows of a sequence are an order of magnitude larger
+    than the last."""
+    g = np.asarray(got, dtype=np.float64)
+    r = np.asarray(ref, dtype=np.float64)
+    if r.size == 0:
+        return 0.0
+    rms = np.sqrt(np.mean(r * r, axis=-1, keepdims=True))
+    floor = np.maximum(np.abs(r), rms)
+    err = np.abs(g - r)
+    zero = floor == 0.0
+    return float(max(np.max(np.where(zero, 0.0, err / np.where(zero, 1.0, floor))), np.max(np.where(zero, err, 0.0))))
+
+
 def to_device(t: "synth.IOTensor"):
     import torch
     if t.io == "f32":
