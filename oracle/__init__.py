@@ -71,6 +71,7 @@ def lib():
             L.oracle_attn_bwd.argtypes = [phi, _I, _I, _I, _I, _I, _D, _P, _P, _P, _P, _P, _P, _P, _P] + [_P] * 6
             L.oracle_max_threads.restype = _I
             L.oracle_set_threads.argtypes = [_I]
+            L.oracle_set_abs_terms.argtypes = [_I]
             _lib = L
     return _lib
 
@@ -169,6 +170,19 @@ def attn_quadratic(params, Q, K, V, lengths=None, causal=False, eps=1e-6) -> np.
     lib().oracle_attn_quadratic(p.ref(), B, H, n, dv, int(bool(causal)), float(eps),
                                 Q.ctypes.data, K.ctypes.data, V.ctypes.data, lp, O.ctypes.data)
     return O
+
+
+def attn_bwd_abs_terms(params, Q, K, V, dO, lengths=None, causal=False, eps=1e-6) -> dict:
+    """For every feature-map parameter gradient, the sum of the absolute values
+    of its per-sample contributions (same chain rule as attn_bwd, with |term|
+    accumulated): the scale of the rounding error of a finite-precision
+    evaluation of that gradient sum."""
+    lib().oracle_set_abs_terms(1)
+    try:
+        g = attn_bwd(params, Q, K, V, dO, lengths, causal, eps)
+    finally:
+        lib().oracle_set_abs_terms(0)
+    return {k: g[k] for k in ("dW", "db", "dw1", "db1", "dw2", "db2")}
 
 
 def attn_bwd(params, Q, K, V, dO, lengths=None, causal=False, eps=1e-6) -> dict:

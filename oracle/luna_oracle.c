@@ -143,6 +143,13 @@ void oracle_kink_margin(const oracle_phi *p, const double *X, int64_t rows, doub
 
 /* Backward of phi for `rows` rows: given dPhi, writes dX and accumulates the
  * parameter gradients into g, by the chain rule through every hidden unit. */
+/* When set, the parameter gradients accumulate the absolute value of every
+ * per-sample contribution instead (sum |term| of each gradient sum: the scale
+ * of the rounding error of any finite-precision evaluation of that sum). */
+static int abs_terms = 0;
+void oracle_set_abs_terms(int on) { abs_terms = on ? 1 : 0; }
+static double term(double v) { return abs_terms ? fabs(v) : v; }
+
 static void phi_rows_backward(const oracle_phi *p, const double *X, int64_t rows, const double *dPhi,
                               double *dX, oracle_grads *g) {
     const int D = p->M * p->L, d = p->d;
@@ -162,20 +169,20 @@ static void phi_rows_backward(const oracle_phi *p, const double *X, int64_t rows
                 const double *w1 = p->w1 + (size_t)l * p->hid;
                 const double *b1 = p->b1 + (size_t)l * p->hid;
                 const double *w2 = p->w2 + (size_t)l * p->hid;
-                g->db2[l] += dy;
+                g->db2[l] += term(dy);
                 for (int k = 0; k < p->hid; ++k) {
                     double a = w1[k] * u + b1[k];
                     if (!(a > 0.0)) continue;
-                    g->dw2[(size_t)l * p->hid + k] += dy * a;
+                    g->dw2[(size_t)l * p->hid + k] += term(dy * a);
                     double dh = dy * w2[k];
-                    g->dw1[(size_t)l * p->hid + k] += dh * u;
-                    g->db1[(size_t)l * p->hid + k] += dh;
+                    g->dw1[(size_t)l * p->hid + k] += term(dh * u);
+                    g->db1[(size_t)l * p->hid + k] += term(dh);
                     du += dh * w1[k];
                 }
             }
-            g->db[i] += du;
+            g->db[i] += term(du);
             for (int c = 0; c < d; ++c) {
-                g->dW[(size_t)i * d + c] += du * x[c];
+                g->dW[(size_t)i * d + c] += term(du * x[c]);
                 dx[c] += du * p->W[(size_t)i * d + c];
             }
         }

@@ -12,7 +12,7 @@ import pytest
 
 import oracle
 import synth
-from cases import TOL, Case, relerr, relerr_rows, to_device, to_host
+from cases import TOL, Case, relerr, relerr_rows, sum_err, to_device, to_host
 
 pytestmark = pytest.mark.gpu
 
@@ -166,8 +166,13 @@ def test_backward(c):
     assert relerr(g["dV"], ref["dV"]) < tol
     for k in ("dQ", "dK", "dV"):
         assert np.all(np.isfinite(g[k]))
-    for k in ("dW", "db", "dw1", "db1", "dw2", "db2"):
-        assert relerr(g[k], ref[k]) < tol, k
+    if c["io"] == "f32":  # fp32 sums over every sample: rounding bound in ulps of sum |terms|
+        A = case.oracle_bwd_abs_terms()
+        for k in ("dW", "db", "dw1", "db1", "dw2", "db2"):
+            assert sum_err(g[k], ref[k], A[k], tol) <= 1.0, k
+    else:
+        for k in ("dW", "db", "dw1", "db1", "dw2", "db2"):
+            assert relerr(g[k], ref[k]) < tol, k
     if case.lengths is not None:
         for b, ln in enumerate(case.lengths):
             for k in ("dQ", "dK", "dV"):

@@ -18,7 +18,7 @@ MUTANTS = {
     "wrong sign of d(den)": ("dden[i] = -dot / den;", "dden[i] = dot / den;"),
     "exclusive causal mask": ("int jmax = causal ? i + 1 : len;", "int jmax = causal ? i : len;"),
     "fc2 weight gradient without activation": (
-        "g->dw2[(size_t)l * p->hid + k] += dy * a;", "g->dw2[(size_t)l * p->hid + k] += dy;"),
+        "g->dw2[(size_t)l * p->hid + k] += term(dy * a);", "g->dw2[(size_t)l * p->hid + k] += term(dy);"),
     "eps dropped from the linear form": (
         "double den = eps;\n        for (int f = 0; f < D; ++f) den += phq[f] * z[f];",
         "double den = 0;\n        for (int f = 0; f < D; ++f) den += phq[f] * z[f];"),

@@ -285,3 +285,33 @@ def test_gradients_zero_on_padding():
         g = oracle.attn_bwd(p, Q, K, V, dO, lengths, causal=causal)
         for k in ("dQ", "dK", "dV"):
             assert np.all(g[k][0, :, 12:] == 0)
+
+
+def test_abs_terms_bound_the_gradients():
+    """The absolute-contribution mode sums |term| over the same per-sample terms
+    as the gradients: it bounds every gradient element (triangle inequality) and
+    equals it when every term of a sum has the same sign (one row, one unit:
+    the query and key paths of that row give same-signed terms here)."""
+    d, M, L, hid = 3, 2, 2, 3
+    p = _rand_params(31, d, M, L, hid)
+    Q, K, V = _rand_inputs(31, 1, 2, 5, d, 2, scale=1.5)
+    dO = synth.normal(31, "abs.dO", V.shape)
+    for causal in (False, True):
+        g = oracle.attn_bwd(p, Q, K, V, dO, None, causal=causal, eps=1e-3)
+        a = oracle.attn_bwd_abs_terms(p, Q, K, V, dO, None, causal=causal, eps=1e-3)
+        for k in ("dW", "db", "dw1", "db1", "dw2", "db2"):
+            assert np.all(a[k] >= np.abs(g[k]) * (1 - 1e-12) - 1e-300), k
+        # the mode is switched off again afterwards
+        g2 = oracle.attn_bwd(p, Q, K, V, dO, None, causal=causal, eps=1e-3)
+        for k in g:
+            np.testing.assert_array_equal(g[k], g2[k])
+    # one row, one projection, one channel, one hidden unit: two same-signed terms per sum
+    p1 = {"W": np.array([[1.0]]), "b": np.array([0.0]), "w1": np.array([[1.0]]), "b1": np.array([[0.5]]),
+          "w2": np.array([[2.0]]), "b2": np.array([0.1])}
+    X = np.array([[[[0.7]]]])
+    V1 = np.array([[[[1.3]]]])
+    dO1 = np.array([[[[-0.4]]]])
+    g = oracle.attn_bwd(p1, X, X, V1, dO1, None, causal=False, eps=0.25)
+    a = oracle.attn_bwd_abs_terms(p1, X, X, V1, dO1, None, causal=False, eps=0.25)
+    for k in ("dW", "db", "dw1", "db1", "dw2", "db2"):
+        np.testing.assert_allclose(a[k], np.abs(g[k]), rtol=1e-14, atol=0)
