@@ -21,6 +21,7 @@ cudaError_t launch_tc_stats(const AttnArgs &a, cudaStream_t s);
 bool tc_bwd_supported(const luna_attn_desc &ad, const TableLayout &lay);
 bool tc_bwd_fits(const AttnArgs &a);
 cudaError_t launch_tc_bwd_kernels(const AttnArgs &a, bool have_stats, cudaStream_t s);
+cudaError_t launch_tc_bwd_wide(const AttnArgs &a, bool have_stats, cudaStream_t s);  // d = dv = 64
 // key statistics of every work item (a.rows_per_split rows, a.nsplit per head) into S_part, z_part
 cudaError_t launch_tc_keys_items(const AttnArgs &a, cudaStream_t s);
 bool tc_causal_supported(const luna_attn_desc &ad, const TableLayout &lay);

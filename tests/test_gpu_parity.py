@@ -190,13 +190,14 @@ def _check_bwd(case, g, ref, tol):
 
 
 @pytest.mark.parametrize("tiles", ["1", "3", "5"])
-def test_backward_tensor_core_tile_loops(tiles, monkeypatch):
-    """bf16 backward through the tensor-core kernels (d = 32, M = 8) with 1, 3
-    and 5 tiles of 128 rows per work item: per-head runs that span several
-    blocks and blocks that span several heads, the staging rings wrapping
-    around, ragged last tiles and items with no valid row."""
+@pytest.mark.parametrize("d", [32, 64])
+def test_backward_tensor_core_tile_loops(d, tiles, monkeypatch):
+    """bf16 backward through the tensor-core kernels (d = 32 and d = 64, M = 8)
+    with 1, 3 and 5 tiles of 128 rows per work item: per-head runs that span
+    several blocks and blocks that span several heads, the staging rings
+    wrapping around, ragged last tiles and items with no valid row."""
     monkeypatch.setenv("LUNA_TC_TILES_PER_SPLIT", tiles)
-    case = Case(2, 3, 1100, 32, 8, 8, "bf16", False, seed=43, qkv_scale=1.0 / math.sqrt(32),
+    case = Case(2, 3, 1100, d, 8, 8, "bf16", False, seed=43, qkv_scale=1.0 / math.sqrt(d),
                 lengths=[1100, 290], with_grad=True)
     lu = case.luna()
     case.run_fwd(lu)
