@@ -356,22 +356,28 @@ __global__ void __launch_bounds__(kThreadsTC, 1)
                     mbar_arrive(phiready + p);
                 }
             }
-            // z of this run: sum the 128 rows of each warp group, then over the four row groups
+            // z of this run: sum the 128 rows of each warp group, then over the four row groups.  The
+            // first barrier keeps these writes behind the previous run's epilogue (warps 0..3 read zpart
+            // there while the other workers may already have finished a run without tiles).
 #pragma unroll
             for (int k = 0; k < C::PP * 8; ++k) {
                 float v = zacc[k];
 #pragma unroll
                 for (int o = 16; o > 0; o >>= 1) v += __shfl_xor_sync(0xffffffffu, v, o);
-                if (lane == 0) zpart[(warp & 3) * C::D + Q * C::PP * 8 + k] = v;
+                zacc[k] = v;
+            }
+            named_sync<kWorkers>(1);
+#pragma unroll
+            for (int k = 0; k < C::PP * 8; ++k) {
+                if (lane == 0) zpart[(warp & 3) * C::D + Q * C::PP * 8 + k] = zacc[k];
                 zacc[k] = 0.0f;
             }
             named_sync<kWorkers>(1);
             if (warp < 4) {
                 // run epilogue: statistics of this block's part of head bh -> its partial slot
-                const int c_first = owner_block((long long)bh * it.nchunk, it.total, gridDim.x);
-                const int c_last = owner_block((long long)(bh + 1) * it.nchunk - 1, it.total, gridDim.x);
-                const int nruns = c_last - c_first + 1;
-                const size_t slot = per_item ? (size_t)i0 : (size_t)bh * it.nchunk + (blockIdx.x - c_first);
+                const RunSlot rs = run_slot(it, bh);
+                const int nruns = rs.nruns;
+                const size_t slot = per_item ? (size_t)i0 : (size_t)bh * it.nchunk + rs.rank;
                 float *Sp = a.S_part + slot * C::D * C::DV;
                 float *zp = a.z_part + slot * C::D;
                 const int row = (warp << 5) | lane;

@@ -121,21 +121,23 @@ __device__ __forceinline__ uint4 pack8(const float (&y)[8]) {
 //
 // Shared-memory fp32 atomics are compare-and-swap loops; int32 atomics are
 // native and about five times faster.  So the bins hold fixed-point int32 sums
-// over groups of up to 16 tiles.  The first tile of a group finds the
-// block-wide maxima of the finite |g| and |g*u| and fixes power-of-two scales
-// 2^e with |q| < 2^16 for them; a bin receives at most 1024 samples per tile,
-// so 16 tiles stay below 2^30.  A later value that does not fit (it outgrew the
-// group's first tile, or is not finite) goes, unscaled, to an fp32 atomic on
-// the block's partial in global memory instead.  At the end of a group the bins
-// are added, rescaled, into that partial and cleared.  The quantisation step is
-// 2^-16 of the group's first-tile maximum.
+// over groups of kHistTiles tiles, quantised with power-of-two scales 2^e such
+// that |q| < 2^kHistQBits for the scale's reference maxima of |g| and |g*u|; a
+// bin receives at most 1024 samples per tile, so a group stays below 2^30.  The
+// block's first group takes its reference maxima from a pre-pass over its
+// first tile with a nonzero g, every later group from the block-wide maxima of
+// the group before it.  A value that does not fit (it outgrew the reference,
+// or is not finite) goes, unscaled, to an fp32 atomic on the block's partial in
+// global memory instead.  At the end of a group the bins are added, rescaled,
+// into that partial and cleared.  The quantisation step is 2^-18 of the
+// reference maximum.
 //
 // Layout in shared memory: bins[(c * 8 + l) * kNint + j] (lanes with different
 // intervals fall into different banks); the partial is [interval][channel][g, g*u].
 __device__ __forceinline__ int hist_at(int c, int l, int j) { return (c * 8 + l) * kNint + j; }
 
-constexpr int kHistQBits = 16;  // |q| < 2^16 per sample
-constexpr int kHistTiles = 16;  // tiles per group: 16 * 1024 * 2^16 = 2^30
+constexpr int kHistQBits = 18;  // |q| < 2^18 per sample
+constexpr int kHistTiles = 4;   // tiles per group: 4 * 1024 * 2^18 = 2^30
 
 // 2^e as a float, e in [-126, 127] (IEEE-754 binary32: biased exponent, zero mantissa).
 __device__ __forceinline__ float pow2f(int e) { return __int_as_float((e + 127) << 23); }
@@ -148,8 +150,10 @@ __device__ __forceinline__ int hist_exp_of(float m) {
 
 // Block-uniform state of the fixed-point bins.
 struct HistAcc {
-    int e0 = 0, e1 = 0;  // exponents of the group
-    int tiles = 0;       // tiles of the current group added so far (0: no group open)
+    int e0 = 0, e1 = 0;        // exponents of the current group
+    int tiles = 0;             // tiles of the current group added so far
+    bool open = false;         // scales known (from the first nonzero tile, then from the previous group)
+    float m0 = 0.f, m1 = 0.f;  // this thread's maxima of the finite |g|, |g*u| added to the current group
 };
 
 // Running maximum of the finite |v|.
@@ -158,11 +162,10 @@ __device__ __forceinline__ float finite_max(float m, float v) {
     return a <= 3.402823466e38f ? fmaxf(m, a) : m;
 }
 
-// Opens a group from this thread's maxima of its first tile: block-wide maxima
-// (one worker barrier; smax holds 2 * (kBWorkers / 32) floats and is next
-// written after the group's closing barrier), then the scales.  Returns false
-// (no group) when every g of the tile is zero.
-__device__ __forceinline__ bool hist_open(HistAcc &h, float m0, float m1, float *smax, int warp, int lane) {
+// Block-wide maxima of the workers' m0, m1 (one worker barrier; smax holds
+// 2 * (kBWorkers / 32) floats and is written again only after a later worker
+// barrier), then the scales: false (scales unchanged) when both are zero.
+__device__ __forceinline__ bool hist_scales(HistAcc &h, float m0, float m1, float *smax, int warp, int lane) {
 #pragma unroll
     for (int o = 16; o > 0; o >>= 1) {
         m0 = fmaxf(m0, __shfl_xor_sync(0xffffffffu, m0, o));
@@ -181,6 +184,14 @@ __device__ __forceinline__ bool hist_open(HistAcc &h, float m0, float m1, float 
     return true;
 }
 
+// Opens the first group of the block from this thread's maxima over its first
+// tile (a pre-pass); later groups take their scales from the previous group.
+// Returns false while every g seen so far is zero.
+__device__ __forceinline__ bool hist_open(HistAcc &h, float m0, float m1, float *smax, int warp, int lane) {
+    h.open = hist_scales(h, m0, m1, smax, warp, lane);
+    return h.open;
+}
+
 // Adds value v of (c, l) for a sample in interval j: int32 bin if it fits the
 // group's scale s, else an fp32 atomic on the global partial.
 __device__ __forceinline__ void hist_put(int *bins, float *part, int c, int l, int j, float v, float s) {
@@ -193,23 +204,30 @@ __device__ __forceinline__ void hist_put(int *bins, float *part, int c, int l, i
     }
 }
 
-// Adds the tile's samples (8 channel values g each, zero where inactive) to the bins.
+// Adds the tile's samples (8 channel values g each, zero where inactive) to the
+// bins and tracks this thread's maxima for the next group's scales.
 template <int PP>
-__device__ __forceinline__ void hist_add(int *bins, float *part, const HistAcc &h, const int (&j)[PP],
+__device__ __forceinline__ void hist_add(int *bins, float *part, HistAcc &h, const int (&j)[PP],
                                          const float (&u)[PP], const float (&g)[PP][8]) {
     const float s0 = pow2f(h.e0), s1 = pow2f(h.e1);
 #pragma unroll
     for (int q = 0; q < PP; ++q)
 #pragma unroll
         for (int l = 0; l < 8; ++l) {
+            const float gu = g[q][l] * u[q];
             hist_put(bins, part, 0, l, j[q], g[q][l], s0);
-            hist_put(bins, part, 1, l, j[q], g[q][l] * u[q], s1);
+            hist_put(bins, part, 1, l, j[q], gu, s1);
+            h.m0 = finite_max(h.m0, g[q][l]);
+            h.m1 = finite_max(h.m1, gu);
         }
 }
 
 // Closes the group: after a worker barrier (every atomic done), adds the bins,
-// rescaled, into the partial and clears them; thread t handles entries t, t + kBWorkers, ...
-__device__ __forceinline__ void hist_close(int *bins, float *part, int nint, HistAcc &h, int t) {
+// rescaled, into the partial and clears them (thread t handles entries t,
+// t + kBWorkers, ...); with `next`, the group's block-wide maxima then give the
+// scales of the next group (unchanged if it was all zero).
+__device__ __forceinline__ void hist_close(int *bins, float *part, int nint, HistAcc &h, int t, bool next,
+                                           float *smax, int warp, int lane) {
     named_sync<kBWorkers>(1);
     const float inv0 = pow2f(-h.e0), inv1 = pow2f(-h.e1);
 #pragma unroll 4
@@ -219,7 +237,9 @@ __device__ __forceinline__ void hist_close(int *bins, float *part, int nint, His
         bins[at] = 0;
         part[e] = __ldcg(part + e) + (float)v * ((e & 1) ? inv1 : inv0);  // L2 copy: fp32 atomics went there
     }
+    if (next) hist_scales(h, h.m0, h.m1, smax, warp, lane);
     h.tiles = 0;
+    h.m0 = h.m1 = 0.0f;
 }
 
 // Zeroes a row of a 128-row x 128 B tile (padded rows must not carry garbage

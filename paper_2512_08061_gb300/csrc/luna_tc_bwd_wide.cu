@@ -321,8 +321,8 @@ __global__ void __launch_bounds__(kBThreads, 1)
                     const float inv = live ? 1.0f / den : 0.0f;
                     const float ndot = live ? -dotn * inv : 0.0f;  // -(dO.O)
                     const float dden = ndot * inv;
-                    bool hon = hacc.tiles > 0;
-                    if (!hon) {  // first tile of a histogram group: the maxima fix its scales
+                    bool hon = hacc.open;
+                    if (!hon) {  // first tile with a nonzero g in the block: a pre-pass fixes the histogram scales
                         float m0 = 0.0f, m1 = 0.0f;
 #pragma unroll
                         for (int q = 0; q < C::PP; ++q) {
@@ -404,7 +404,7 @@ __global__ void __launch_bounds__(kBThreads, 1)
                     mbar_arrive(gready);
                     if (hon) {
                         hist_add<C::PP>(bins, hpart, hacc, j, u, gv);
-                        if (++hacc.tiles == kHistTiles) hist_close(bins, hpart, a.lay.nint, hacc, tid);
+                        if (++hacc.tiles == kHistTiles) hist_close(bins, hpart, a.lay.nint, hacc, tid, true, smax, warp, lane);
                     }
                     // dQ
                     wait_or_fail(dqready, g & 1, failed, status);
@@ -429,10 +429,9 @@ __global__ void __launch_bounds__(kBThreads, 1)
             // run epilogue (warps 0..3): dS, dz partial of this head; warp w holds features 16w..16w+15,
             // hi in lanes 0..15 and lo in lanes 16..31
             if (warp < 4) {
-                const int c_first = owner_block((long long)bh * it.nchunk, it.total, gridDim.x);
-                const int c_last = owner_block((long long)(bh + 1) * it.nchunk - 1, it.total, gridDim.x);
-                const int nruns = c_last - c_first + 1;
-                const size_t slot = (size_t)bh * it.nchunk + (blockIdx.x - c_first);
+                const RunSlot rs = run_slot(it, bh);
+                const int nruns = rs.nruns;
+                const size_t slot = (size_t)bh * it.nchunk + rs.rank;
                 float *Sp = a.dS_part + slot * C::D * C::DV;
                 float *zp = a.dz_part + slot * C::D;
                 const uint32_t lr = (uint32_t)(warp << 5) << 16;
@@ -484,7 +483,7 @@ __global__ void __launch_bounds__(kBThreads, 1)
             if (run_tiles > 0) ++ne;
             i0 = i1;
         }
-        if (hacc.tiles > 0) hist_close(bins, hpart, a.lay.nint, hacc, tid);
+        if (hacc.tiles > 0) hist_close(bins, hpart, a.lay.nint, hacc, tid, false, smax, warp, lane);
 #pragma unroll
         for (int q = 0; q < C::PP; ++q) {
             float v = db_acc[q];
@@ -756,7 +755,7 @@ __global__ void __launch_bounds__(kBThreads, 1)
                     // dphi(k) = dS v + dz  ->  dU, histogram
                     wait_or_fail(fready, g & 1, failed, status);
                     tc_fence_after();
-                    bool hon = hacc.tiles > 0;
+                    bool hon = hacc.open;
                     if (!hon) {
                         float m0 = 0.0f, m1 = 0.0f;
 #pragma unroll
@@ -812,7 +811,7 @@ __global__ void __launch_bounds__(kBThreads, 1)
                     mbar_arrive(gready);
                     if (hon) {
                         hist_add<C::PP>(bins, hpart, hacc, j, u, gv);
-                        if (++hacc.tiles == kHistTiles) hist_close(bins, hpart, a.lay.nint, hacc, tid);
+                        if (++hacc.tiles == kHistTiles) hist_close(bins, hpart, a.lay.nint, hacc, tid, true, smax, warp, lane);
                     }
                     // dV = hi + lo
                     wait_or_fail(dvready, g & 1, failed, status);
@@ -859,7 +858,7 @@ __global__ void __launch_bounds__(kBThreads, 1)
             }
             i0 = i1;
         }
-        if (hacc.tiles > 0) hist_close(bins, hpart, a.lay.nint, hacc, tid);
+        if (hacc.tiles > 0) hist_close(bins, hpart, a.lay.nint, hacc, tid, false, smax, warp, lane);
 #pragma unroll
         for (int q = 0; q < C::PP; ++q) {
             float v = db_acc[q];

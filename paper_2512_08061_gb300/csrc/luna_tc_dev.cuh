@@ -129,9 +129,18 @@ __device__ __forceinline__ ItemRange item_range(const AttnArgs &a, const Items &
     return g;
 }
 
-// Block of the persistent grid whose contiguous item range contains `item`.
-__device__ __forceinline__ int owner_block(long long item, long long total, int G) {
-    return (int)(((item + 1) * G - 1) / total);
+// The blocks that own items of head bh (a contiguous block range): how many
+// there are, and how many of them come before this block.
+struct RunSlot {
+    int rank, nruns;
+};
+
+__device__ __forceinline__ RunSlot run_slot(const Items &it, int bh) {
+    const long long total = it.total;
+    const int G = gridDim.x;
+    const int c_first = (int)((((long long)bh * it.nchunk + 1) * G - 1) / total);
+    const int c_last = (int)((((long long)(bh + 1) * it.nchunk) * G - 1) / total);
+    return RunSlot{(int)blockIdx.x - c_first, c_last - c_first + 1};
 }
 
 // out[e] = sum_{p < np} part[p][e] in order p = 0..np-1, for e < count
