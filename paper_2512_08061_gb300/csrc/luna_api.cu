@@ -36,6 +36,7 @@ struct Plan {
     size_t o_counters = 0, o_status = 0, o_Spart = 0, o_zpart = 0, o_Sfin = 0, o_zfin = 0;
     size_t o_dSpart = 0, o_dzpart = 0, o_dSfin = 0, o_dzfin = 0, o_gpart = 0, o_hist = 0;
     size_t o_segS = 0, o_segz = 0, o_segdS = 0, o_segdz = 0, o_rowstat = 0;
+    size_t o_dphi = 0, o_phik = 0, o_pq2 = 0;  // streaming-form backward on tensor cores
     size_t ws_fwd = 0, ws_bwd = 0, state_bytes = 0;
     TcPlan tc;
 };
@@ -127,6 +128,15 @@ luna_status make_plan(const luna_attn_desc *ad, const luna_phi_desc *pd, Plan &p
     if (p.tc.eligible) {
         p.ws_fwd = std::max(p.ws_fwd, p.tc.ws_fwd);
         p.ws_bwd = std::max(p.ws_bwd, p.tc.ws_bwd);
+    }
+    if (ad->causal && p.tc.causal_bwd) {  // dphi (fp32), phi(k) and phi(q)/den as hi|lo (bf16) of every row
+        Bump wb;
+        wb.n = p.ws_bwd;
+        const size_t R = (size_t)BH * n;
+        p.o_dphi = wb.take(R * D * f);
+        p.o_phik = wb.take(R * 2 * D * 2);
+        p.o_pq2 = wb.take(R * 2 * D * 2);
+        p.ws_bwd = wb.n;
     }
     return LUNA_OK;
 }
@@ -320,7 +330,15 @@ luna_status luna_attn_bwd(const luna_attn_desc *ad, const luna_phi_desc *pd, con
         return LUNA_ERR_UNSUPPORTED;
     cudaError_t e = cudaMemsetAsync(workspace, 0, p.o_counters + 2 * sizeof(int) * (size_t)p.BH, s);
     if (e != cudaSuccess) return LUNA_ERR_CUDA;
-    if (ad->causal) return cuda_status(launch_causal_bwd(a, ad->io, state != nullptr, s));
+    if (ad->causal) {
+        if (p.tc.causal_bwd && tc_inputs_ok(TcPlan{true}, Q, K, V, dO) && tc_inputs_ok(TcPlan{true}, dQ, dK, dV, nullptr)) {
+            a.dphi = reinterpret_cast<float *>(w + p.o_dphi);
+            a.phik = w + p.o_phik;
+            a.pq2 = w + p.o_pq2;
+            return cuda_status(launch_tc_causal_bwd(a, state != nullptr, s));
+        }
+        return cuda_status(launch_causal_bwd(a, ad->io, state != nullptr, s));
+    }
     if (p.tc.eligible && tc_inputs_ok(p.tc, Q, K, V, dO) && tc_inputs_ok(p.tc, dQ, dK, dV, nullptr))
         return cuda_status(launch_tc_bwd(p.tc, a, w, state != nullptr, s));
     return cuda_status(launch_simt_bwd(a, ad->io, state != nullptr, s));

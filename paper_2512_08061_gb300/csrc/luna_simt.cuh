@@ -30,6 +30,9 @@ struct AttnArgs {
     float *seg_S, *seg_z;              // [BH][nseg+1][D][dv], [BH][nseg+1][D]: prefix at each segment start, total last
     float *seg_dS, *seg_dz;            // [BH][nseg][D][dv], [BH][nseg][D]: suffix after segment end
     float *rowstat;                    // [BH][n][2]: (den_i, dden_i) of the backward pass
+    // streaming-form backward on tensor cores
+    float *dphi;                       // [BH][n][D] fp32: dLoss/dphi of Q, then of K
+    void *phik, *pq2;                  // [BH][n][2D] bf16 phi(k), phi(q)/den, each as (hi | lo)
 };
 
 cudaError_t launch_phi_prepare(const luna_phi_params &prm, const TableLayout &lay, void *table, cudaStream_t s);

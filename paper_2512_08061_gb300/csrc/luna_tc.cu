@@ -667,14 +667,14 @@ EncodeTiledFn encoder() {
     return fn;
 }
 
-// (width, n, BH) bf16 tensor, boxes of 64 columns x 128 rows, 128B swizzle,
+// (width, n, BH) bf16 tensor, boxes of 64 columns x `rows` rows, 128B swizzle,
 // out-of-range elements read as zero.
-bool make_map_impl(CUtensorMap *m, const void *base, int width, int n, int BH) {
+bool make_map_impl(CUtensorMap *m, const void *base, int width, int n, int BH, int rows = 128) {
     EncodeTiledFn enc = encoder();
     if (!enc) return false;
     cuuint64_t dims[3] = {(cuuint64_t)width, (cuuint64_t)n, (cuuint64_t)BH};
     cuuint64_t strides[2] = {(cuuint64_t)width * 2, (cuuint64_t)n * width * 2};
-    cuuint32_t box[3] = {64, 128, 1};
+    cuuint32_t box[3] = {64, (cuuint32_t)rows, 1};
     cuuint32_t es[3] = {1, 1, 1};
     return enc(m, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 3, const_cast<void *>(base), dims, strides, box, es,
                CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
@@ -757,6 +757,9 @@ int variant(const luna_attn_desc &ad, const TableLayout &lay) {
 bool tc_make_map(CUtensorMap *m, const void *base, int width, int n, int BH) {
     return make_map_impl(m, base, width, n, BH);
 }
+bool tc_make_map_rows(CUtensorMap *m, const void *base, int width, int n, int BH, int rows) {
+    return make_map_impl(m, base, width, n, BH, rows);
+}
 int tc_sm_count() { return sm_count_impl(); }
 AttnArgs tc_work_items(const AttnArgs &a) { return tc_items_impl(a); }
 
@@ -769,6 +772,7 @@ TcPlan tc_plan(const luna_attn_desc &ad, const TableLayout &lay) {
         luna_attn_desc nc = ad;
         nc.causal = 0;
         p.causal_fwd = encoder() != nullptr && variant(nc, lay) >= 0 && tc_causal_supported(ad, lay);
+        p.causal_bwd = p.causal_fwd;
     }
     return p;
 }

@@ -10,6 +10,7 @@ struct TcPlan {
     int variant = -1;        // kernel instantiation (value width / projections)
     bool bwd = false;        // backward also on tensor cores
     bool causal_fwd = false; // streaming-form forward on tensor cores
+    bool causal_bwd = false; // streaming-form backward on tensor cores
     size_t ws_fwd = 0, ws_bwd = 0;
 };
 
@@ -26,5 +27,8 @@ cudaError_t launch_tc_bwd_wide(const AttnArgs &a, bool have_stats, cudaStream_t 
 cudaError_t launch_tc_keys_items(const AttnArgs &a, cudaStream_t s);
 bool tc_causal_supported(const luna_attn_desc &ad, const TableLayout &lay);
 cudaError_t launch_tc_causal_fwd(const AttnArgs &a, cudaStream_t s);
+// segment prefixes of S, z (work items = state segments)
+cudaError_t launch_tc_causal_stats(const AttnArgs &a, cudaStream_t s);
+cudaError_t launch_tc_causal_bwd(const AttnArgs &a, bool have_state, cudaStream_t s);
 
 }  // namespace luna

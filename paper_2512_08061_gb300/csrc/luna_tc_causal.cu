@@ -454,17 +454,25 @@ bool tc_causal_supported(const luna_attn_desc &ad, const TableLayout &lay) {
     return ad.io == LUNA_BF16 && ad.causal && lay.L == 8 && lay.P <= 512 && ad.d == 128 && ad.dv == 128 && lay.M == 16;
 }
 
-cudaError_t launch_tc_causal_fwd(const AttnArgs &a0, cudaStream_t s) {
-    using C = K128;
+cudaError_t launch_tc_causal_stats(const AttnArgs &a0, cudaStream_t s) {
     AttnArgs a = a0;
     a.rows_per_split = a0.seg_len;  // work item = state segment (whole 128-row tiles)
     a.nsplit = a0.nseg;
     cudaError_t e = launch_tc_keys_items(a, s);
     if (e != cudaSuccess) return e;
-    const int BH = a.B * a.H;
     const size_t SD4 = (size_t)a.D * a.dv / 4;
-    LUNA_LAUNCH("seg_scan", k_seg_scan, dim3((unsigned)((SD4 + 255) / 256), BH), 256, 0, s, a);
-    if ((e = cudaGetLastError()) != cudaSuccess) return e;
+    LUNA_LAUNCH("seg_scan", k_seg_scan, dim3((unsigned)((SD4 + 255) / 256), a.B * a.H), 256, 0, s, a);
+    return cudaGetLastError();
+}
+
+cudaError_t launch_tc_causal_fwd(const AttnArgs &a0, cudaStream_t s) {
+    using C = K128;
+    AttnArgs a = a0;
+    a.rows_per_split = a0.seg_len;  // work item = state segment (whole 128-row tiles)
+    a.nsplit = a0.nseg;
+    cudaError_t e = launch_tc_causal_stats(a, s);
+    if (e != cudaSuccess) return e;
+    const int BH = a.B * a.H;
     CUtensorMap mQ, mK, mV;
     if (!tc_make_map(&mQ, a.Q, a.d, a.n, BH) || !tc_make_map(&mK, a.K, a.d, a.n, BH) ||
         !tc_make_map(&mV, a.V, a.dv, a.n, BH))

@@ -230,6 +230,39 @@ def test_backward_tensor_core_repeat_bitwise():
         assert np.array_equal(g1[k], g2[k]), k
 
 
+@pytest.mark.parametrize("seg_rows", ["128", "384", "1280"])
+def test_backward_tensor_core_causal(seg_rows, monkeypatch):
+    """Streaming-form backward through the tensor-core kernels (d = 128, M = 16):
+    state segments of 2, 6 and 20 tiles of 64 rows (the running S and dS carried
+    across tiles in TMEM, the reverse scan of the segment sums), ragged last
+    tiles, a sequence with padding and segments that hold no valid row."""
+    monkeypatch.setenv("LUNA_CAUSAL_SEG_ROWS", seg_rows)
+    case = Case(2, 2, 1100, 128, 16, 8, "bf16", True, seed=61, qkv_scale=1.0 / math.sqrt(128),
+                lengths=[1100, 333], with_grad=True)
+    lu = case.luna()
+    case.run_fwd(lu)
+    g = {k: to_host(v) for k, v in case.run_bwd(lu).items()}
+    _check_bwd(case, g, case.oracle_bwd(), TOL["bf16"])
+    for k in ("dQ", "dK", "dV"):
+        assert np.all(np.isfinite(g[k]))
+        assert np.all(g[k][1, :, 333:] == 0)
+
+
+def test_backward_tensor_core_causal_state_and_repeat():
+    """The tensor-core streaming-form backward gives the same bits with the
+    forward's saved segment prefixes as without them, and on a repeated run."""
+    case = Case(1, 2, 700, 128, 16, 8, "bf16", True, seed=67, qkv_scale=1.0 / math.sqrt(128),
+                with_grad=True)
+    lu = case.luna()
+    case.run_fwd(lu)
+    a = {k: to_host(v) for k, v in case.run_bwd(lu, use_state=True).items()}
+    b = {k: to_host(v) for k, v in case.run_bwd(lu, use_state=False).items()}
+    c = {k: to_host(v) for k, v in case.run_bwd(lu, use_state=False).items()}
+    for k in ("dQ", "dK", "dV"):
+        assert np.array_equal(a[k], b[k]), k
+        assert np.array_equal(b[k], c[k]), k
+
+
 @pytest.mark.parametrize("causal", [False, True])
 def test_backward_with_and_without_saved_state(causal):
     case = Case(2, 2, 200, 32, 8, 8, "f32", causal, seed=13, with_grad=True, lengths=[200, 150])
