@@ -19,6 +19,7 @@ bounded sample of the same workload.
 from __future__ import annotations
 
 import argparse
+import dataclasses
 import hashlib
 import json
 import math
@@ -51,6 +52,8 @@ def parse():
     ap.add_argument("--no-e2e", action="store_true")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--cpu-seconds", type=float, default=12.0, help="target CPU work of the oracle sample")
+    ap.add_argument("--seq-len", type=int, default=0,
+                    help="shorter sequence length n for profiler captures of a small case (the JSON line reports it)")
     return ap.parse_args()
 
 
@@ -92,8 +95,15 @@ def kernel_bytes(w, lengths, kernel: str) -> float:
     }
     # the tensor-core kernels move the same tensors as their generic counterparts
     for tc, generic in (("tc_keys", "keystats"), ("tc_query", "query"), ("tc_bwd_query", "bwd_query"),
-                        ("tc_bwd_key", "bwd_key")):
+                        ("tc_bwd_key", "bwd_key"), ("tc_causal", "causal_out")):
         table[tc] = table[generic]
+    # streaming-form backward stages: their inputs and outputs, including the rows they
+    # hand to the next stage (fp32 dphi; bf16 hi|lo phi(k) and phi(q)/den; den, -dO.O)
+    D = w.D
+    table["tcc_query"] = valid * (2 * rd + 2 * rv) + valid * (D * 4 + 8) + total * 2 * (2 * D * 2)
+    table["tcc_dstats"] = valid * (2 * D * 2 + rv + 4)
+    table["tcc_key"] = valid * (2 * (2 * D * 2) + 2 * rv + 4) + total * rv + valid * D * 4
+    table["tc_phi_bwd"] = valid * (rd + D * 4) + total * rd
     return float(table.get(kernel, 0.0))
 
 
@@ -345,7 +355,7 @@ def run_gpu(args, w):
         byts = kernel_bytes(w, lengths, dominant)
         dur = dom_ms / dom_n * 1e-3
         achieved = byts / dur / 1e9 if byts else None
-        traffic, traffic_src = measured_traffic(dominant, w.name)
+        traffic, traffic_src = measured_traffic(dominant, w.name) if args.seq_len <= 0 else (None, None)
         roof = {"bound": "hbm", "kernel": dominant, "achieved": achieved, "peak": hbm, "unit": "GB/s",
                 "frac": (achieved / hbm) if achieved else None, "traffic": traffic, "traffic_source": traffic_src,
                 "peak_source": peak_src, "algorithmic_bytes": byts, "launch_ms": dom_ms / dom_n, "launches": dom_n}
@@ -455,6 +465,10 @@ def run_reference(args, w):
 def main():
     args = parse()
     w = WORKLOADS[args.workload]
+    if args.seq_len > 0:
+        n = args.seq_len
+        w = dataclasses.replace(w, n=n, len_range=None if w.len_range is None else
+                                (min(w.len_range[0], n), min(w.len_range[1], n)))
     res = run_reference(args, w) if args.impl == "reference" else run_gpu(args, w)
     if res is not None:
         print(json.dumps(res), flush=True)

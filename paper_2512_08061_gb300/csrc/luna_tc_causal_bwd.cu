@@ -311,6 +311,7 @@ __global__ void __launch_bounds__(kCBThreads, 1)
 #pragma unroll
                         for (int k = 0; k < 4; ++k)
                             mma_bf16_ss(tbase + cZc, dadd(dL1, 32 * k), dadd(hl ? dPm : dKm, 2048 * k), idZc, (hl | k) != 0);
+                    mma_commit(aready);  // the workers mask F while P = dO S^T runs
 #pragma unroll
                     for (int h = 0; h < 2; ++h)
 #pragma unroll
@@ -319,7 +320,6 @@ __global__ void __launch_bounds__(kCBThreads, 1)
                             for (int k = 0; k < 4; ++k)
                                 mma_bf16_ss(tbase + cP, dadd(dOk, kb * T8 + 32 * k),
                                             dadd(h ? dSl : dSh, kb * C::T16 + 32 * k), idP, (h | kb | k) != 0);
-                    mma_commit(aready);
                 }
                 wait_or_fail(fready, g & 1, failed, status);
                 tc_fence_after();
@@ -467,9 +467,15 @@ __global__ void __launch_bounds__(kCBThreads, 1)
                 wait_or_fail(aready, g & 1, failed, status);
                 tc_fence_after();
                 float zi[16];
+                uint32_t xf[16];
                 {
-                    uint32_t x[32];
-                    ld32(tbase + lq + cZc + 32 * cg, x);
+                    uint32_t x[32], x1[16];
+                    tmem_ld16(tbase + lq + cZc + 32 * cg, x1);
+                    tmem_ld16(tbase + lq + cZc + 32 * cg + 16, *reinterpret_cast<uint32_t (*)[16]>(x + 16));
+                    tmem_ld16(tbase + lq + cU + 16 * cg, xf);
+                    tmem_wait_ld();
+#pragma unroll
+                    for (int k = 0; k < 16; ++k) x[k] = x1[k];
                     float zc[16];
                     half_cols<16>(x, zc, lane);
                     float dpart = 0.0f;
@@ -481,11 +487,8 @@ __global__ void __launch_bounds__(kCBThreads, 1)
                     sred[part * 64 + r] = dpart;
                 }
                 {
-                    uint32_t x[16];
-                    tmem_ld16(tbase + lq + cU + 16 * cg, x);
-                    tmem_wait_ld();
                     float fv[8];
-                    half_cols<8>(x, fv, lane);
+                    half_cols<8>(xf, fv, lane);
                     const int j0 = 8 * part;
 #pragma unroll
                     for (int k = 0; k < 8; ++k) fv[k] = (valid && j0 + k <= r) ? fv[k] : 0.0f;
@@ -786,7 +789,8 @@ __global__ void __launch_bounds__(kCBThreads, 1)
     uint64_t *bars = reinterpret_cast<uint64_t *>(sdz + C::D);
     uint64_t *full = bars, *infree = bars + 1, *c1ready = bars + 2, *mready = bars + 3;
     uint64_t *c3ready = bars + 4, *accfree = bars + 5, *sopready = bars + 6;
-    uint32_t *tslot = reinterpret_cast<uint32_t *>(bars + 7);
+    uint64_t *dvready = bars + 7, *dfready = bars + 8;
+    uint32_t *tslot = reinterpret_cast<uint32_t *>(bars + 9);
 
     const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
     const Items it(a);
@@ -796,6 +800,7 @@ __global__ void __launch_bounds__(kCBThreads, 1)
     if (tid == 0) {
         mbar_init(full, 1); mbar_init(infree, 1); mbar_init(c1ready, 1); mbar_init(mready, kCBWorkers);
         mbar_init(c3ready, 1); mbar_init(accfree, kCBWorkers); mbar_init(sopready, kCBWorkers);
+        mbar_init(dvready, 1); mbar_init(dfready, 1);
         fence_mbar_init();
     }
     if (warp == 0) { tmem_alloc(tslot, 512); tmem_relinquish(); }
@@ -891,6 +896,7 @@ __global__ void __launch_bounds__(kCBThreads, 1)
                         mma_bf16_ss(tbase + cV, dadd(dCh, 32 * k), dadd(dOm, 2048 * k), idV, 1u);
                         mma_bf16_ss(tbase + cV, dadd(dCl, 32 * k), dadd(dOm, 2048 * k), idV, 1u);
                     }
+                    mma_commit(dvready);
                     // dphi = V [dS_hi; dS_lo]^T + E phi~(Q)   (E hi x phi~ hi, lo; E lo x phi~ hi)
                     constexpr uint32_t idF = idesc_bf16(64, C::D, false, false);
                     constexpr uint32_t idFm = idesc_bf16(64, C::D, false, true);
@@ -908,6 +914,7 @@ __global__ void __launch_bounds__(kCBThreads, 1)
                         mma_bf16_ss(tbase + cF, dadd(dEh, 32 * k), dadd(dPqM, 2 * T8 + 2048 * k), idFm, 1u);
                         mma_bf16_ss(tbase + cF, dadd(dEl, 32 * k), dadd(dPqM, 2048 * k), idFm, 1u);
                     }
+                    mma_commit(dfready);
                     // dS += phi~(Q)^T dO, dz += phi~(Q)^T [ndot_hi, ndot_lo]
                     constexpr uint32_t idS = idesc_bf16(128, C::DV, true, true);
                     constexpr uint32_t idZ = idesc_bf16(128, 16, true, false);
@@ -973,14 +980,15 @@ __global__ void __launch_bounds__(kCBThreads, 1)
                 const int nvalid = min(64, ir.r1 - row0);
                 const bool valid = r < nvalid;
                 // masked C and E + ndot; padded query rows of dO cleared; ndot operand
+                const int i0 = 8 * part;
+                float nd[8], ndr = 0.0f;  // -dO.O of this thread's 8 query columns and of its own row
+#pragma unroll
+                for (int k = 0; k < 8; ++k)
+                    nd[k] = (i0 + k < nvalid) ? __ldcg(a.rowstat + 2 * (hrow + row0 + i0 + k) + 1) : 0.0f;
+                if (part == 0 && valid) ndr = __ldcg(a.rowstat + 2 * (hrow + row0 + r) + 1);
                 wait_or_fail(c1ready, g & 1, failed, status);
                 tc_fence_after();
                 {
-                    const int i0 = 8 * part;
-                    float nd[8];
-#pragma unroll
-                    for (int k = 0; k < 8; ++k)
-                        nd[k] = (i0 + k < nvalid) ? __ldcg(a.rowstat + 2 * (hrow + row0 + i0 + k) + 1) : 0.0f;
                     uint32_t x[16];
                     tmem_ld16(tbase + lq + cV + 16 * cg, x);
                     tmem_wait_ld();
@@ -1006,9 +1014,7 @@ __global__ void __launch_bounds__(kCBThreads, 1)
                     *reinterpret_cast<uint4 *>(El + sw128_chunk(r, part)) = el;
                 }
                 if (part == 0) {
-                    float nd = 0.0f;
-                    if (valid) nd = __ldcg(a.rowstat + 2 * (hrow + row0 + r) + 1);
-                    else {
+                    if (!valid) {
 #pragma unroll
                         for (int kb = 0; kb < 2; ++kb)
 #pragma unroll
@@ -1016,7 +1022,7 @@ __global__ void __launch_bounds__(kCBThreads, 1)
                                 *reinterpret_cast<uint4 *>(Ob + kb * T8 + sw128_chunk(r, c)) = make_uint4(0, 0, 0, 0);
                     }
                     __nv_bfloat16 hi, lo;
-                    split_bf16(nd, hi, lo);
+                    split_bf16(ndr, hi, lo);
                     *reinterpret_cast<__nv_bfloat16 *>(Nd + sw128_chunk(0, r / 8) + (r % 8) * 2) = hi;
                     *reinterpret_cast<__nv_bfloat16 *>(Nd + sw128_chunk(1, r / 8) + (r % 8) * 2) = lo;
                 }
@@ -1024,23 +1030,27 @@ __global__ void __launch_bounds__(kCBThreads, 1)
                 tc_fence_before();
                 mbar_arrive(mready);
                 // dV, dphi(k) = dphi + dz (the state after this tile's rows)
-                wait_or_fail(c3ready, g & 1, failed, status);
+                wait_or_fail(dvready, g & 1, failed, status);
                 tc_fence_after();
                 {
                     uint32_t x[32];
                     ld32(tbase + lq + cV + 32 * cg, x);
                     float dv[16];
                     half_cols<16>(x, dv, lane);
+                    if (valid) {
+                        uint4 *dst = reinterpret_cast<uint4 *>(static_cast<__nv_bfloat16 *>(a.dV) +
+                                                               (hrow + row0 + r) * C::DV + 16 * part);
+                        dst[0] = pack8f(dv);
+                        dst[1] = pack8f(dv + 8);
+                    }
+                    wait_or_fail(dfready, g & 1, failed, status);
+                    tc_fence_after();
                     ld32(tbase + lq + cF + 32 * cg, x);
                     float df[16];
                     half_cols<16>(x, df, lane);
                     tc_fence_before();
                     mbar_arrive(accfree);
                     if (valid) {
-                        uint4 *dst = reinterpret_cast<uint4 *>(static_cast<__nv_bfloat16 *>(a.dV) +
-                                                               (hrow + row0 + r) * C::DV + 16 * part);
-                        dst[0] = pack8f(dv);
-                        dst[1] = pack8f(dv + 8);
                         float4 *fp = reinterpret_cast<float4 *>(a.dphi + (hrow + row0 + r) * C::D + 16 * part);
 #pragma unroll
                         for (int k = 0; k < 4; ++k)
@@ -1050,6 +1060,8 @@ __global__ void __launch_bounds__(kCBThreads, 1)
                     }
                 }
                 named_sync<kCBWorkers>(1);  // every sdz read before it changes
+                wait_or_fail(c3ready, g & 1, failed, status);
+                tc_fence_after();
                 if (tr + 1 < nt) {  // dS, dz after this tile -> operand and sdz of the next (earlier) tile
                     const int f = 32 * q + lane, c0 = 32 * cg;
                     uint32_t x[32];
