@@ -157,6 +157,34 @@ luna_status luna_attn_bwd(const luna_attn_desc *ad, const luna_phi_desc *pd, con
                           const void *state, void *dQ, void *dK, void *dV, const luna_phi_grads *grads,
                           void *workspace, size_t ws_bytes, void *stream);
 
+/* Location of the final state of a streaming-form forward pass (ad->causal = 1)
+ * inside a `state` buffer written by luna_attn_fwd: the key statistics over all
+ * valid tokens of each sequence, S = sum_j phi(k_j) v_j^T and z = sum_j phi(k_j)
+ * (Eq. kernel-attn, streaming form of Sec. 3.2).  Head (b, h) holds S at
+ * *S + (b*H + h) * *S_stride (D x dv fp32, row-major) and z at
+ * *z + (b*H + h) * *z_stride (D fp32).  No device memory is touched; the
+ * pointers are for luna_attn_decode, which continues each sequence after its
+ * last valid token.  LUNA_ERR_INVALID_ARG for a non-causal descriptor or NULL
+ * arguments. */
+luna_status luna_state_final(const luna_attn_desc *ad, const luna_phi_desc *pd, void *state, float **S,
+                             int64_t *S_stride, float **z, int64_t *z_stride);
+
+/* One step of the streaming form (recurrent decode; the abstract and Sec. 3.2
+ * name the associative streaming form of Eq. kernel-attn): for every (b, h)
+ * and the new token's q, k, v,
+ *     S <- S + phi(k) v^T,   z <- z + phi(k),   o = phi(q)^T S / (phi(q)^T z + eps)
+ * i.e. the causal output of the token that follows the state's tokens.
+ * q, k: (B, H, d); v, o: (B, H, dv), element type ad->io, one token per
+ * (b, h); ad->n, ad->causal and ad->chunk are ignored.  S, z: fp32 device
+ * arrays updated in place, head (b, h) at S + (b*H + h) * S_stride ([D][dv]
+ * row-major) and z + (b*H + h) * z_stride ([D]); a stride of 0 selects the
+ * dense layout (D*dv, D), a smaller nonzero stride is LUNA_ERR_INVALID_ARG.
+ * A head whose guarded normaliser is exactly 0 produces o = 0.  No workspace;
+ * B*H = 0 is a no-op. */
+luna_status luna_attn_decode(const luna_attn_desc *ad, const luna_phi_desc *pd, const void *table, const void *q,
+                             const void *k, const void *v, void *o, float *S, int64_t S_stride, float *z,
+                             int64_t z_stride, void *stream);
+
 /* Synchronises `stream`, then reads and clears the device status word at the
  * start of `workspace`.  Every luna_attn_fwd / luna_attn_bwd call clears the
  * word when it starts; a device-side wait of that call that ran out of its

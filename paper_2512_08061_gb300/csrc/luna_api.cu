@@ -344,6 +344,54 @@ luna_status luna_attn_bwd(const luna_attn_desc *ad, const luna_phi_desc *pd, con
     return cuda_status(launch_simt_bwd(a, ad->io, state != nullptr, s));
 }
 
+luna_status luna_state_final(const luna_attn_desc *ad, const luna_phi_desc *pd, void *state, float **S,
+                             int64_t *S_stride, float **z, int64_t *z_stride) {
+    if (!S || !S_stride || !z || !z_stride) return LUNA_ERR_INVALID_ARG;
+    Plan p;
+    luna_status st = make_plan(ad, pd, p);
+    if (st != LUNA_OK) return st;
+    if (!ad->causal) return LUNA_ERR_INVALID_ARG;
+    if (!state) return LUNA_ERR_INVALID_ARG;
+    const int64_t SD = (int64_t)p.lay.D * ad->dv, ns = p.nseg;
+    float *base = static_cast<float *>(state);
+    *S = base + ns * SD;  // segment prefixes [BH][nseg + 1][D][dv]: entry nseg is the total
+    *S_stride = (ns + 1) * SD;
+    *z = base + (int64_t)p.BH * (ns + 1) * SD + ns * p.lay.D;
+    *z_stride = (ns + 1) * p.lay.D;
+    return LUNA_OK;
+}
+
+luna_status luna_attn_decode(const luna_attn_desc *ad, const luna_phi_desc *pd, const void *table, const void *q,
+                             const void *k, const void *v, void *o, float *S, int64_t S_stride, float *z,
+                             int64_t z_stride, void *stream) {
+    if (!ad) return LUNA_ERR_INVALID_ARG;
+    if (ad->B < 0 || ad->H < 0 || ad->d < 1 || ad->dv < 1) return LUNA_ERR_INVALID_ARG;
+    if (ad->io != LUNA_F32 && ad->io != LUNA_BF16) return LUNA_ERR_INVALID_ARG;
+    if (!(ad->eps >= 0.0f) || isinf(ad->eps)) return LUNA_ERR_INVALID_ARG;
+    luna_status st = check_phi(pd, ad->d);
+    if (st != LUNA_OK) return st;
+    if (ad->dv > kMaxD) return LUNA_ERR_UNSUPPORTED;
+    const int64_t BH = (int64_t)ad->B * ad->H;
+    if (BH > (1 << 24)) return LUNA_ERR_UNSUPPORTED;
+    const TableLayout lay = table_layout(pd->M, pd->L, pd->hidden, ad->d);
+    const int64_t SD = (int64_t)lay.D * ad->dv;
+    if (S_stride == 0) S_stride = SD;
+    if (z_stride == 0) z_stride = lay.D;
+    if (S_stride < SD || z_stride < lay.D) return LUNA_ERR_INVALID_ARG;
+    if (BH == 0) return LUNA_OK;
+    if (!table || !q || !k || !v || !o || !S || !z) return LUNA_ERR_INVALID_ARG;
+    if (!aligned(table, 256)) return LUNA_ERR_INVALID_ARG;
+    DecodeArgs a;
+    a.BH = (int)BH; a.d = ad->d; a.dv = ad->dv; a.M = lay.M; a.L = lay.L; a.D = lay.D;
+    a.eps = ad->eps;
+    a.lay = lay;
+    a.table = static_cast<const char *>(table);
+    a.q = q; a.k = k; a.v = v; a.o = o;
+    a.S = S; a.z = z;
+    a.S_stride = S_stride; a.z_stride = z_stride;
+    return cuda_status(launch_decode(a, ad->io, static_cast<cudaStream_t>(stream)));
+}
+
 luna_status luna_device_status(void *workspace, void *stream) {
     if (!workspace) return LUNA_ERR_INVALID_ARG;
     cudaStream_t s = static_cast<cudaStream_t>(stream);

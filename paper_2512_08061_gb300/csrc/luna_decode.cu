@@ -1,0 +1,126 @@
+// One step of the streaming form (recurrent decode): for every (batch, head),
+// with the state (S, z) after t tokens and the new token (q, k, v),
+//     S <- S + phi(k) v^T,   z <- z + phi(k),   o = phi(q)^T S / (phi(q)^T z + eps)
+// (the associative streaming form of Eq. kernel-attn named in the abstract and
+// Sec. 3.2; the state after the token is the inclusive prefix of the causal form).
+//
+// One block per head.  The work per head is two projections of width d, 2*M
+// interval searches and channel evaluations, and one pass over the D x dv
+// fp32 state (read, update, write back) with the output accumulated on the
+// way: the state traffic bounds the step, so it is CUDA-core code that reads
+// and writes every state element once, coalesced along the value columns.
+#include <math.h>
+
+#include "luna_common.cuh"
+#include "luna_prof.cuh"
+#include "luna_simt.cuh"
+
+namespace luna {
+
+namespace {
+
+constexpr int kDecThreads = 256;
+
+template <typename IO> __device__ __forceinline__ float ld_io(const IO *p, int64_t i);
+template <> __device__ __forceinline__ float ld_io<float>(const float *p, int64_t i) { return p[i]; }
+template <> __device__ __forceinline__ float ld_io<__nv_bfloat16>(const __nv_bfloat16 *p, int64_t i) {
+    return __bfloat162float(p[i]);
+}
+template <typename IO> __device__ __forceinline__ void st_io(IO *p, int64_t i, float v);
+template <> __device__ __forceinline__ void st_io<float>(float *p, int64_t i, float v) { p[i] = v; }
+template <> __device__ __forceinline__ void st_io<__nv_bfloat16>(__nv_bfloat16 *p, int64_t i, float v) {
+    p[i] = __float2bfloat16_rn(v);
+}
+
+template <typename IO>
+__global__ void __launch_bounds__(kDecThreads) k_decode(DecodeArgs a) {
+    __shared__ float sx[2][kMaxD];        // q, k
+    __shared__ float sv[kMaxD];
+    __shared__ float sphi[2][kMaxFeat];   // phi(q), phi(k)
+    __shared__ float su[2][32];           // projections of q and k
+    __shared__ float so[kDecThreads];     // output partials [feature group][column]
+    __shared__ float sden[kDecThreads / 32];
+    const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+    const int64_t bh = blockIdx.x;
+    const int d = a.d, dv = a.dv, M = a.M, L = a.L, D = a.D;
+    for (int e = tid; e < d; e += blockDim.x) {
+        sx[0][e] = ld_io(static_cast<const IO *>(a.q), bh * d + e);
+        sx[1][e] = ld_io(static_cast<const IO *>(a.k), bh * d + e);
+    }
+    for (int e = tid; e < dv; e += blockDim.x) sv[e] = ld_io(static_cast<const IO *>(a.v), bh * dv + e);
+    __syncthreads();
+    // u = W x + b for x = q, k: one warp per dot product
+    const float *W = reinterpret_cast<const float *>(a.table + a.lay.off_W);
+    const float *bias = reinterpret_cast<const float *>(a.table + a.lay.off_b);
+    for (int p = warp; p < 2 * M; p += blockDim.x / 32) {
+        const int side = p / M, m = p % M;
+        float acc = 0.0f;
+        for (int c = lane; c < d; c += 32) acc = fmaf(W[m * d + c], sx[side][c], acc);
+#pragma unroll
+        for (int o = 16; o > 0; o >>= 1) acc += __shfl_xor_sync(0xffffffffu, acc, o);
+        if (lane == 0) su[side][m] = acc + bias[m];
+    }
+    __syncthreads();
+    // phi: interval of u in the breadth-first kink tree, then relu(alpha u + beta) per channel
+    const float *Te = reinterpret_cast<const float *>(a.table + a.lay.off_Te);
+    const float2 *AB = reinterpret_cast<const float2 *>(a.table + a.lay.off_AB);
+    for (int p = tid; p < 2 * M; p += blockDim.x) {
+        const int side = p / M, m = p % M;
+        const float u = su[side][m];
+        int node = 1;
+        for (int lvl = 0; lvl < 10; ++lvl) node = 2 * node + (__ldg(Te + node) < u ? 1 : 0);
+        const int j = node - kEytzinger;
+        for (int l = 0; l < L; ++l) {
+            const float2 ab = __ldg(AB + (size_t)j * L + l);
+            sphi[side][m * L + l] = fmaxf(fmaf(ab.x, u, ab.y), 0.0f);
+        }
+    }
+    __syncthreads();
+    // z <- z + phi(k); den = phi(q).z + eps
+    float *z = a.z + bh * a.z_stride;
+    float dp = 0.0f;
+    for (int f = tid; f < D; f += blockDim.x) {
+        const float zf = z[f] + sphi[1][f];
+        z[f] = zf;
+        dp = fmaf(sphi[0][f], zf, dp);
+    }
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) dp += __shfl_xor_sync(0xffffffffu, dp, o);
+    if (lane == 0) sden[warp] = dp;
+    // S <- S + phi(k) v^T and the numerator phi(q)^T S: thread (g, c) owns column c and features f = g (mod G)
+    const int G = kDecThreads / dv;  // feature groups (dv <= 128, so G >= 2)
+    const int g = tid / dv, c = tid % dv;
+    float num = 0.0f;
+    if (g < G) {
+        float *S = a.S + bh * a.S_stride;
+        const float vc = sv[c];
+#pragma unroll 8
+        for (int f = g; f < D; f += G) {
+            const float s = fmaf(sphi[1][f], vc, S[(int64_t)f * dv + c]);
+            S[(int64_t)f * dv + c] = s;
+            num = fmaf(sphi[0][f], s, num);
+        }
+    }
+    so[tid] = num;
+    __syncthreads();
+    if (tid < dv) {
+        float den = a.eps;
+        for (int w = 0; w < kDecThreads / 32; ++w) den += sden[w];
+        float acc = 0.0f;
+        for (int gg = 0; gg < G; ++gg) acc += so[gg * dv + tid];
+        st_io(static_cast<IO *>(a.o), bh * dv + tid, den != 0.0f ? acc / den : 0.0f);
+    }
+}
+
+}  // namespace
+
+cudaError_t launch_decode(const DecodeArgs &a, luna_dtype io, cudaStream_t s) {
+    if (a.BH == 0) return cudaSuccess;
+    if (io == LUNA_F32)
+        LUNA_LAUNCH("decode", k_decode<float>, a.BH, kDecThreads, 0, s, a);
+    else
+        LUNA_LAUNCH("decode", k_decode<__nv_bfloat16>, a.BH, kDecThreads, 0, s, a);
+    return cudaGetLastError();
+}
+
+}  // namespace luna

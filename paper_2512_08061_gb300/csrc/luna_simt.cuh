@@ -35,6 +35,19 @@ struct AttnArgs {
     void *phik, *pq2;                  // [BH][n][2D] bf16 phi(k), phi(q)/den, each as (hi | lo)
 };
 
+// one step of the streaming form for every (batch, head): state S [D][dv], z [D] (fp32, in place)
+struct DecodeArgs {
+    int BH, d, dv, M, L, D;
+    float eps;
+    TableLayout lay;
+    const char *table;
+    const void *q, *k, *v;
+    void *o;
+    float *S, *z;
+    int64_t S_stride, z_stride;  // elements between consecutive heads
+};
+cudaError_t launch_decode(const DecodeArgs &a, luna_dtype io, cudaStream_t s);
+
 cudaError_t launch_phi_prepare(const luna_phi_params &prm, const TableLayout &lay, void *table, cudaStream_t s);
 cudaError_t launch_featmap(const TableLayout &lay, const char *table, const void *X, luna_dtype xt, int64_t rows,
                            float *Phi, cudaStream_t s);

@@ -75,6 +75,9 @@ def _load():
         "luna_profile_stop": ([ctypes.POINTER(ctypes.c_double), ctypes.POINTER(I)], I),
         "luna_launch_count": ([], ctypes.c_uint64),
         "luna_attn_fwd_noalloc": ([ad, pd, P, P, P, P, P, P, P], I),
+        "luna_state_final": ([ad, pd, P, ctypes.POINTER(P), ctypes.POINTER(I64), ctypes.POINTER(P),
+                              ctypes.POINTER(I64)], I),
+        "luna_attn_decode": ([ad, pd, P, P, P, P, P, P, I64, P, I64, P], I),
     }
     for name, (args, res) in sig.items():
         fn = getattr(lib, name)
@@ -86,7 +89,8 @@ def _load():
 _lib = _load()
 EXPORTED = ("luna_status_string", "luna_version", "luna_phi_table_size", "luna_phi_prepare", "luna_featmap",
             "luna_workspace_size", "luna_state_size", "luna_attn_fwd", "luna_attn_bwd", "luna_device_status",
-            "luna_profile_start", "luna_profile_stop", "luna_launch_count", "luna_attn_fwd_noalloc")
+            "luna_profile_start", "luna_profile_stop", "luna_launch_count", "luna_attn_fwd_noalloc",
+            "luna_state_final", "luna_attn_decode")
 
 
 def _ptr(t):
@@ -181,6 +185,22 @@ def luna_attn_fwd_noalloc(ad, pd, table, Q, K, V, lengths, O, stream=None) -> No
 NOALLOC_SCRATCH_BYTES = 16 << 20
 
 
+def luna_state_final(ad, pd, state) -> tuple[int, int, int, int]:
+    """(S address, S stride, z address, z stride) of the final causal state inside `state` (floats)."""
+    S, Ss, z, zs = ctypes.c_void_p(), ctypes.c_int64(), ctypes.c_void_p(), ctypes.c_int64()
+    _check(_lib.luna_state_final(ctypes.byref(ad), ctypes.byref(pd), _ptr(state), ctypes.byref(S), ctypes.byref(Ss),
+                                 ctypes.byref(z), ctypes.byref(zs)), "luna_state_final")
+    return S.value, Ss.value, z.value, zs.value
+
+
+def luna_attn_decode(ad, pd, table, q, k, v, o, S, S_stride, z, z_stride, stream=None) -> None:
+    """S, z: tensors (their data pointers are used) or raw device addresses."""
+    sp = _ptr(S) if isinstance(S, torch.Tensor) else ctypes.c_void_p(S)
+    zp = _ptr(z) if isinstance(z, torch.Tensor) else ctypes.c_void_p(z)
+    _check(_lib.luna_attn_decode(ctypes.byref(ad), ctypes.byref(pd), _ptr(table), _ptr(q), _ptr(k), _ptr(v), _ptr(o),
+                                 sp, S_stride, zp, z_stride, _stream(stream)), "luna_attn_decode")
+
+
 def luna_device_status(workspace: torch.Tensor, stream=None) -> int:
     return _lib.luna_device_status(_ptr(workspace), _stream(stream))
 
@@ -242,3 +262,12 @@ class Luna:
         luna_attn_bwd(self.ad, self.pd, self.table, Q, K, V, dO, lengths, self.state if use_state else None,
                       out["dQ"], out["dK"], out["dV"], out, self.ws, stream)
         return out
+
+    def decode(self, q, k, v, o=None, stream=None):
+        """One streaming-form step per (b, h) from the final state of the last causal forward
+        (saved with save_state=True), which it advances in place.  q, k: (B, H, d); v: (B, H, dv)."""
+        if o is None:
+            o = torch.empty(q.shape[:-1] + (self.ad.dv,), dtype=q.dtype, device=q.device)
+        S, Ss, z, zs = luna_state_final(self.ad, self.pd, self.state)
+        luna_attn_decode(self.ad, self.pd, self.table, q, k, v, o, S, Ss, z, zs, stream)
+        return o

@@ -86,3 +86,42 @@ def test_argument_errors_return_before_launch(L):
     st = lib.luna_attn_fwd(ctypes.byref(ad0), ctypes.byref(pd), None, None, None, None, None, None, None, None, 0,
                            None)
     assert st == 0
+
+
+def test_decode_arguments_and_state_layout(L):
+    """luna_attn_decode and luna_state_final check their arguments before any
+    launch; the final causal state sits at segment nseg of each head's block of
+    nseg + 1 segment prefixes (S first for all heads, then z)."""
+    lib = L._lib
+    pd = L.phi_desc(16, 8, 64)
+    ad = L.attn_desc(2, 3, 1000, 128, 128, causal=True)
+    P, I64 = ctypes.c_void_p, ctypes.c_int64
+    # NULL tensors, a too-small stride and a bad eps are rejected
+    st = lib.luna_attn_decode(ctypes.byref(ad), ctypes.byref(pd), None, None, None, None, None, None, 0, None, 0, None)
+    assert st == 1
+    st = lib.luna_attn_decode(ctypes.byref(ad), ctypes.byref(pd), P(256), P(256), P(256), P(256), P(256), P(256),
+                              128 * 128 - 1, P(256), 0, None)
+    assert st == 1
+    bad = L.attn_desc(2, 3, 1000, 128, 128, causal=True, eps=-1.0)
+    st = lib.luna_attn_decode(ctypes.byref(bad), ctypes.byref(pd), P(256), P(256), P(256), P(256), P(256), P(256),
+                              0, P(256), 0, None)
+    assert st == 1
+    # B*H = 0 is a no-op
+    ad0 = L.attn_desc(0, 3, 1, 128, 128)
+    assert lib.luna_attn_decode(ctypes.byref(ad0), ctypes.byref(pd), None, None, None, None, None, None, 0, None, 0,
+                                None) == 0
+    # state layout: nseg from the state size, S and z offsets of the last segment
+    SD, D, BH = 128 * 128, 128, 6
+    size = L.luna_state_size(ad, pd)
+    nseg1 = size // (4 * BH * (SD + D))
+    assert size == 4 * BH * nseg1 * (SD + D)
+    base = 1 << 20
+    S, Ss, z, zs = (ctypes.c_void_p(), I64(), ctypes.c_void_p(), I64())
+    assert lib.luna_state_final(ctypes.byref(ad), ctypes.byref(pd), P(base), ctypes.byref(S), ctypes.byref(Ss),
+                                ctypes.byref(z), ctypes.byref(zs)) == 0
+    assert Ss.value == nseg1 * SD and zs.value == nseg1 * D
+    assert S.value == base + 4 * (nseg1 - 1) * SD
+    assert z.value == base + 4 * (BH * nseg1 * SD + (nseg1 - 1) * D)
+    nc = L.attn_desc(2, 3, 1000, 128, 128, causal=False)
+    assert lib.luna_state_final(ctypes.byref(nc), ctypes.byref(pd), P(base), ctypes.byref(S), ctypes.byref(Ss),
+                                ctypes.byref(z), ctypes.byref(zs)) == 1

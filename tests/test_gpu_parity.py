@@ -315,3 +315,33 @@ def test_unit_values_give_unit_outputs():
     nz = np.any(O != 0, axis=-1)
     assert nz.mean() > 0.9
     assert np.max(np.abs(O[nz] - 1.0)) < 1e-5
+
+
+@pytest.mark.parametrize("io,d,dv,M", [("bf16", 128, 128, 16), ("f32", 64, 64, 8), ("f32", 64, 32, 8)])
+def test_decode_continues_the_streaming_form(io, d, dv, M):
+    """Recurrent decode (luna_attn_decode): a causal forward over the first
+    tokens of each (padded) sequence saves its state; three decode steps then
+    feed the tokens that follow each sequence's last valid one.  Each step's
+    output equals the oracle's causal output at that position of the extended
+    sequence (streaming form, Sec. 3.2)."""
+    import torch
+    import paper_2512_08061_gb300.luna as L
+    B, H, n0, T = 2, 2, 300, 3
+    lens = [300, 177]
+    case = Case(B, H, n0 + T, d, M, 8, io, True, seed=71, qkv_scale=1.0 / math.sqrt(d), dv=dv,
+                lengths=[ln + T for ln in lens])
+    dt = torch.float32 if io == "f32" else torch.bfloat16
+    lu = L.Luna(B, H, n0, d, dv, M, 8, 64, True, case.eps, dt)
+    lu.prepare({k: torch.from_numpy(v).cuda() for k, v in case.params.items()})
+    full = {k: to_device(case.inp[k]) for k in ("Q", "K", "V")}
+    pre = {k: v[:, :, :n0].contiguous() for k, v in full.items()}
+    lu.forward(pre["Q"], pre["K"], pre["V"], torch.tensor(lens, dtype=torch.int32, device="cuda"), save_state=True)
+    outs = []
+    for t in range(T):
+        tok = {k: torch.stack([v[b, :, lens[b] + t] for b in range(B)]).contiguous() for k, v in full.items()}
+        outs.append(to_host(lu.decode(tok["Q"], tok["K"], tok["V"])))
+    ref = case.oracle_fwd()
+    tol = TOL[io]
+    for t in range(T):
+        want = np.stack([ref[b, :, lens[b] + t] for b in range(B)])
+        assert relerr_rows(outs[t], want) < tol, t
