@@ -462,6 +462,131 @@ def run_reference(args, w):
             "e2e": {"value": value, "unit": "tokens/s", "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}}
 
 
+DECODE_METRIC = "LUNA decode tokens/sec (one token per sequence per step) on 1 GB300; % of HBM roofline"
+
+
+def decode_bytes(w) -> float:
+    """Bytes of one decode step: every fp32 state element read and written once, and the
+    token's q, k, v read and o written."""
+    eb = 4 if w.io == "f32" else 2
+    return float(w.B * w.H * (2 * (w.D * w.dv + w.D) * 4 + (2 * w.d + 2 * w.dv) * eb))
+
+
+def run_decode(args, w):
+    """Streaming inference: a causal prefill of w.n tokens saves the state, then every step
+    advances all B x H heads by one token through luna_attn_decode (state updated in place)."""
+    import torch
+    import torch.distributed as tdist
+
+    rank, local_rank, world = dist_env()
+    torch.cuda.set_device(local_rank)
+    if world > 1:
+        tdist.init_process_group("nccl", device_id=torch.device("cuda", local_rank))
+    from paper_2512_08061_gb300 import build
+    if rank == 0 or world == 1:
+        build.build()
+    if world > 1:
+        tdist.barrier()
+    import paper_2512_08061_gb300.luna as L
+
+    dev = torch.device("cuda", local_rank)
+    io_dtype = torch.float32 if w.io == "f32" else torch.bfloat16
+    inp, params = host_inputs(w)
+
+    def pinned(t):
+        if t.io == "f32":
+            return torch.from_numpy(np.ascontiguousarray(t.raw)).pin_memory()
+        return torch.from_numpy(np.ascontiguousarray(t.raw).view(np.int16)).view(torch.bfloat16).pin_memory()
+
+    pre = {k: pinned(inp[k]).to(dev) for k in ("Q", "K", "V")}
+    lu = L.Luna(w.B, w.H, w.n, w.d, w.dv, w.M, w.L, w.hidden, True, w.eps, io_dtype, w.chunk, dev)
+    lu.prepare({k: torch.from_numpy(v).to(dev) for k, v in params.items()})
+    lu.forward(pre["Q"], pre["K"], pre["V"], None, save_state=True)
+    host = {k: pinned(synth.IOTensor(synth.normal(w.seed, f"decode.{k}", (w.B, w.H, n)) * w.qkv_scale, w.io))
+            for k, n in (("q", w.d), ("k", w.d), ("v", w.dv))}
+    tok = {k: v.to(dev) for k, v in host.items()}
+    o = torch.empty(w.B, w.H, w.dv, dtype=io_dtype, device=dev)
+    S, Ss, z, zs = L.luna_state_final(lu.ad, lu.pd, lu.state)
+    flush = torch.empty(2 * L2_BYTES, dtype=torch.uint8, device=dev)
+    stream = torch.cuda.current_stream()
+
+    def step(t):
+        L.luna_attn_decode(lu.ad, lu.pd, lu.table, t["q"], t["k"], t["v"], o, S, Ss, z, zs)
+
+    def timed(n_steps, fn):
+        evs = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)) for _ in range(n_steps)]
+        for s0, s1 in evs:
+            flush.zero_()
+            s0.record(stream)
+            fn()
+            s1.record(stream)
+        torch.cuda.synchronize()
+        return sum(s0.elapsed_time(s1) for s0, s1 in evs)
+
+    for _ in range(max(args.warmup, 3)):
+        step(tok)
+    torch.cuda.synchronize()
+    if world > 1:
+        tdist.barrier()
+    uuid = str(getattr(torch.cuda.get_device_properties(local_rank), "uuid", "") or "")
+    clocks = ClockSampler(("GPU-" + uuid if uuid and not uuid.startswith("GPU-") else uuid) or str(local_rank))
+    L.luna_profile_start("decode")
+    n0 = L.luna_launch_count()
+    ms_step = timed(args.steps, lambda: step(tok)) / args.steps
+    launches = L.luna_launch_count() - n0
+    dom_ms, dom_n = L.luna_profile_stop()
+    clk = clocks.stop()
+    if world > 1:
+        t = torch.tensor([ms_step], device=dev)
+        tdist.all_reduce(t, op=tdist.ReduceOp.MAX)
+        ms_step = float(t.item())
+    e2e = None
+    if not args.no_e2e:
+        o_host = torch.empty(o.shape, dtype=o.dtype).pin_memory()
+
+        def e2e_step():
+            step({k: v.to(dev, non_blocking=True) for k, v in host.items()})
+            o_host.copy_(o, non_blocking=True)
+
+        for _ in range(2):
+            e2e_step()
+        torch.cuda.synchronize()
+        e2e_ms = timed(max(3, args.steps // 4), e2e_step) / max(3, args.steps // 4)
+        if world > 1:
+            t = torch.tensor([e2e_ms], device=dev)
+            tdist.all_reduce(t, op=tdist.ReduceOp.MAX)
+            e2e_ms = float(t.item())
+        e2e = {"value": w.B * world / (e2e_ms * 1e-3), "unit": "tokens/s",
+               "h2d_bytes_per_step": int(sum(v.numel() * v.element_size() for v in host.values())),
+               "d2h_bytes_per_step": int(o_host.numel() * o_host.element_size()), "ms_per_step": e2e_ms}
+    hbm, _, peak_src = peaks()
+    byts = decode_bytes(w)
+    roof = None
+    if dom_n:
+        achieved = byts / (dom_ms / dom_n * 1e-3) / 1e9
+        roof = {"bound": "hbm", "kernel": "decode", "achieved": achieved, "peak": hbm, "unit": "GB/s",
+                "frac": achieved / hbm, "traffic": None, "traffic_source": None, "peak_source": peak_src,
+                "algorithmic_bytes": byts, "launch_ms": dom_ms / dom_n, "launches": dom_n}
+    result = {
+        "metric": DECODE_METRIC, "value": w.B * world / (ms_step * 1e-3), "unit": "tokens/s", "n_gpus": world,
+        "steps": args.steps, "warmup": args.warmup, "ms_per_step": ms_step, "higher_is_better": True,
+        "scaling": "weak", "vs_baseline": None, "dtype": w.io, "data": "synthetic",
+        "config": {"workload": f"{w.name}: B={w.B} H={w.H}, one token per sequence per step after a causal "
+                               f"prefill of n={w.n}, d={w.d} D={w.D} (M={w.M}, L={w.L}), {w.io}, fp32 state",
+                   "global_batch": w.B * world, "seq_len": w.n, "parallelism": f"replicas{world}",
+                   "l2": "flushed before every timed step (2x L2 buffer written outside the events)"},
+        "step_roofline": {"bytes": byts, "time_ms": byts / (hbm * 1e9) * 1e3,
+                          "frac": byts / (hbm * 1e9) * 1e3 / ms_step},
+        "roofline": roof, "per_kernel_ms": {"decode": dom_ms / dom_n if dom_n else None},
+        "e2e": e2e, "gpu_launches": int(launches), "clocks": clk,
+        "cpu_baseline": None,
+        "cpu_baseline_note": "the oracle keeps no state between calls; decode parity is tested against its causal form",
+    }
+    if world > 1:
+        tdist.destroy_process_group()
+    return result if rank == 0 else None
+
+
 def main():
     args = parse()
     w = WORKLOADS[args.workload]
@@ -469,6 +594,16 @@ def main():
         n = args.seq_len
         w = dataclasses.replace(w, n=n, len_range=None if w.len_range is None else
                                 (min(w.len_range[0], n), min(w.len_range[1], n)))
+    if w.decode:
+        if args.impl == "reference":
+            res = None if dist_env()[0] != 0 else {
+                "impl": "reference",
+                "unavailable": "the oracle keeps no state between calls (decode parity is tested against its causal form)"}
+        else:
+            res = run_decode(args, w)
+        if res is not None:
+            print(json.dumps(res), flush=True)
+        return
     res = run_reference(args, w) if args.impl == "reference" else run_gpu(args, w)
     if res is not None:
         print(json.dumps(res), flush=True)

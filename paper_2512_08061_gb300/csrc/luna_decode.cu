@@ -8,7 +8,9 @@
 // interval searches and channel evaluations, and one pass over the D x dv
 // fp32 state (read, update, write back) with the output accumulated on the
 // way: the state traffic bounds the step, so it is CUDA-core code that reads
-// and writes every state element once, coalesced along the value columns.
+// and writes every state element once, in 16-byte accesses along the value
+// columns.  The kink tree is staged in shared memory so that the searches do
+// not wait on ten dependent global loads.
 #include <math.h>
 
 #include "luna_common.cuh"
@@ -38,8 +40,9 @@ __global__ void __launch_bounds__(kDecThreads) k_decode(DecodeArgs a) {
     __shared__ float sv[kMaxD];
     __shared__ float sphi[2][kMaxFeat];   // phi(q), phi(k)
     __shared__ float su[2][32];           // projections of q and k
-    __shared__ float so[kDecThreads];     // output partials [feature group][column]
+    __shared__ float so[4 * kDecThreads]; // output partials [feature group][column]
     __shared__ float sden[kDecThreads / 32];
+    __shared__ __align__(16) float sTe[kEytzinger];
     const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
     const int64_t bh = blockIdx.x;
     const int d = a.d, dv = a.dv, M = a.M, L = a.L, D = a.D;
@@ -48,6 +51,8 @@ __global__ void __launch_bounds__(kDecThreads) k_decode(DecodeArgs a) {
         sx[1][e] = ld_io(static_cast<const IO *>(a.k), bh * d + e);
     }
     for (int e = tid; e < dv; e += blockDim.x) sv[e] = ld_io(static_cast<const IO *>(a.v), bh * dv + e);
+    const float4 *Te4 = reinterpret_cast<const float4 *>(a.table + a.lay.off_Te);
+    for (int e = tid; e < kEytzinger / 4; e += blockDim.x) reinterpret_cast<float4 *>(sTe)[e] = __ldg(Te4 + e);
     __syncthreads();
     // u = W x + b for x = q, k: one warp per dot product
     const float *W = reinterpret_cast<const float *>(a.table + a.lay.off_W);
@@ -62,13 +67,12 @@ __global__ void __launch_bounds__(kDecThreads) k_decode(DecodeArgs a) {
     }
     __syncthreads();
     // phi: interval of u in the breadth-first kink tree, then relu(alpha u + beta) per channel
-    const float *Te = reinterpret_cast<const float *>(a.table + a.lay.off_Te);
     const float2 *AB = reinterpret_cast<const float2 *>(a.table + a.lay.off_AB);
     for (int p = tid; p < 2 * M; p += blockDim.x) {
         const int side = p / M, m = p % M;
         const float u = su[side][m];
         int node = 1;
-        for (int lvl = 0; lvl < 10; ++lvl) node = 2 * node + (__ldg(Te + node) < u ? 1 : 0);
+        for (int lvl = 0; lvl < 10; ++lvl) node = 2 * node + (sTe[node] < u ? 1 : 0);
         const int j = node - kEytzinger;
         for (int l = 0; l < L; ++l) {
             const float2 ab = __ldg(AB + (size_t)j * L + l);
@@ -87,21 +91,46 @@ __global__ void __launch_bounds__(kDecThreads) k_decode(DecodeArgs a) {
 #pragma unroll
     for (int o = 16; o > 0; o >>= 1) dp += __shfl_xor_sync(0xffffffffu, dp, o);
     if (lane == 0) sden[warp] = dp;
-    // S <- S + phi(k) v^T and the numerator phi(q)^T S: thread (g, c) owns column c and features f = g (mod G)
-    const int G = kDecThreads / dv;  // feature groups (dv <= 128, so G >= 2)
-    const int g = tid / dv, c = tid % dv;
-    float num = 0.0f;
+    // S <- S + phi(k) v^T and the numerator phi(q)^T S.  With dv % 4 == 0 and a 16-byte aligned state,
+    // thread (g, c4) owns columns 4*c4 .. 4*c4+3 and features f = g (mod G); else one column per thread.
+    float *S = a.S + bh * a.S_stride;
+    const bool vec = (dv % 4 == 0) && ((reinterpret_cast<uintptr_t>(S) & 15) == 0) && (a.S_stride % 4 == 0);
+    const int cw = vec ? dv / 4 : dv;  // column units per feature row
+    const int G = kDecThreads / cw;    // feature groups (dv <= 128: G >= 2)
+    const int g = tid / cw, cu = tid % cw;
+    float num[4] = {0.0f, 0.0f, 0.0f, 0.0f};
     if (g < G) {
-        float *S = a.S + bh * a.S_stride;
-        const float vc = sv[c];
+        if (vec) {
+            const float4 vc = make_float4(sv[4 * cu], sv[4 * cu + 1], sv[4 * cu + 2], sv[4 * cu + 3]);
+            float4 *S4 = reinterpret_cast<float4 *>(S);
 #pragma unroll 8
-        for (int f = g; f < D; f += G) {
-            const float s = fmaf(sphi[1][f], vc, S[(int64_t)f * dv + c]);
-            S[(int64_t)f * dv + c] = s;
-            num = fmaf(sphi[0][f], s, num);
+            for (int f = g; f < D; f += G) {
+                const float pk = sphi[1][f], pq = sphi[0][f];
+                float4 s = S4[(int64_t)f * cw + cu];
+                s.x = fmaf(pk, vc.x, s.x); s.y = fmaf(pk, vc.y, s.y);
+                s.z = fmaf(pk, vc.z, s.z); s.w = fmaf(pk, vc.w, s.w);
+                S4[(int64_t)f * cw + cu] = s;
+                num[0] = fmaf(pq, s.x, num[0]); num[1] = fmaf(pq, s.y, num[1]);
+                num[2] = fmaf(pq, s.z, num[2]); num[3] = fmaf(pq, s.w, num[3]);
+            }
+        } else {
+            const float vc = sv[cu];
+#pragma unroll 8
+            for (int f = g; f < D; f += G) {
+                const float s = fmaf(sphi[1][f], vc, S[(int64_t)f * dv + cu]);
+                S[(int64_t)f * dv + cu] = s;
+                num[0] = fmaf(sphi[0][f], s, num[0]);
+            }
         }
     }
-    so[tid] = num;
+    if (g < G) {
+        if (vec) {
+#pragma unroll
+            for (int e = 0; e < 4; ++e) so[g * dv + 4 * cu + e] = num[e];
+        } else {
+            so[g * dv + cu] = num[0];
+        }
+    }
     __syncthreads();
     if (tid < dv) {
         float den = a.eps;

@@ -1,4 +1,4 @@
-"""The five synthetic workloads (shapes, dtypes, seeds and value recipes).
+"""The synthetic workloads (shapes, dtypes, seeds and value recipes).
 
 They stand in for the paper's evaluation settings (Long Range Arena encoders,
 BERT-base, ViT-B/16 and a long-context causal stream) by shape only: the
@@ -30,6 +30,7 @@ class Workload:
     hidden: int = 64
     chunk: int = 64
     eps: float = 1e-6
+    decode: bool = False  # one streaming-form step per (batch, head) after a causal prefill of n tokens
 
     @property
     def dv(self) -> int:
@@ -56,4 +57,8 @@ WORKLOADS = {
                     causal=False, backward=False, seed=3, qkv_scale=1.0),
     "causal_long": Workload("causal_long", B=2, H=32, n=65536, d=128, M=16, L=8, io="bf16",
                             causal=True, backward=True, seed=4, qkv_scale=1.0 / math.sqrt(128)),
+    # streaming inference: 64 sequences x 32 heads advance by one token per step from the state of a
+    # 1024-token causal prefill (the long-context head shape)
+    "decode": Workload("decode", B=64, H=32, n=1024, d=128, M=16, L=8, io="bf16",
+                       causal=True, backward=False, seed=5, qkv_scale=1.0 / math.sqrt(128), decode=True),
 }
