@@ -61,6 +61,23 @@ def dist_env():
     return int(os.environ.get("RANK", 0)), int(os.environ.get("LOCAL_RANK", 0)), int(os.environ.get("WORLD_SIZE", 1))
 
 
+def max_over_ranks(value: float, device, world: int) -> float:
+    """The largest of the ranks' values (a replicated step takes as long as its slowest rank);
+    the value itself on one rank."""
+    if world <= 1:
+        return float(value)
+    import torch
+    import torch.distributed as tdist
+    t = torch.tensor([float(value)], dtype=torch.float64, device=device)
+    tdist.all_reduce(t, op=tdist.ReduceOp.MAX)
+    return float(t.item())
+
+
+def job_throughput(units_per_rank: float, world: int, ms: float) -> float:
+    """Whole-job rate: the units every rank processed, over the slowest rank's time (ms)."""
+    return units_per_rank * world / (ms * 1e-3)
+
+
 def peaks():
     try:
         with open(os.path.join(ROOT, "MEASURED_PEAKS.json")) as f:
@@ -304,17 +321,11 @@ def run_gpu(args, w):
     clk = clocks.stop()
     torch.cuda.synchronize()
     ms_step = ms_total / args.steps
-    if world > 1:
-        t = torch.tensor([ms_step], device=dev)
-        tdist.all_reduce(t, op=tdist.ReduceOp.MAX)
-        ms_step = float(t.item())
+    ms_step = max_over_ranks(ms_step, dev, world)
 
     # forward-only throughput (same flush discipline)
     fwd_ms = timed(args.steps, lambda: step(devt, backward=False)) / args.steps
-    if world > 1:
-        t = torch.tensor([fwd_ms], device=dev)
-        tdist.all_reduce(t, op=tdist.ReduceOp.MAX)
-        fwd_ms = float(t.item())
+    fwd_ms = max_over_ranks(fwd_ms, dev, world)
 
     # end to end through the public API with host buffers
     e2e = None
@@ -341,11 +352,8 @@ def run_gpu(args, w):
             e2e_step()
         torch.cuda.synchronize()
         e2e_ms = timed(max(3, args.steps // 4), e2e_step) / max(3, args.steps // 4)
-        if world > 1:
-            t = torch.tensor([e2e_ms], device=dev)
-            tdist.all_reduce(t, op=tdist.ReduceOp.MAX)
-            e2e_ms = float(t.item())
-        e2e = {"value": w.tokens * world / (e2e_ms * 1e-3), "unit": "tokens/s", "h2d_bytes_per_step": int(bi),
+        e2e_ms = max_over_ranks(e2e_ms, dev, world)
+        e2e = {"value": job_throughput(w.tokens, world, e2e_ms), "unit": "tokens/s", "h2d_bytes_per_step": int(bi),
                "d2h_bytes_per_step": int(bo), "ms_per_step": e2e_ms}
 
     hbm, tflops, peak_src = peaks()
@@ -363,7 +371,7 @@ def run_gpu(args, w):
     t_roof = max(sb / (hbm * 1e9), sf / (tflops * 1e12))
     result = {
         "metric": METRIC,
-        "value": w.tokens * world / (ms_step * 1e-3),
+        "value": job_throughput(w.tokens, world, ms_step),
         "unit": "tokens/s",
         "n_gpus": world,
         "steps": args.steps,
@@ -380,7 +388,7 @@ def run_gpu(args, w):
                                + (f", lengths U[{w.len_range[0]},{w.len_range[1]}]" if w.len_range else ""),
                    "global_batch": w.B * world, "seq_len": w.n, "parallelism": f"replicas{world}",
                    "l2": "flushed before every timed step (2x L2 buffer written outside the events)"},
-        "fwd": {"value": w.tokens * world / (fwd_ms * 1e-3), "unit": "tokens/s", "ms_per_step": fwd_ms},
+        "fwd": {"value": job_throughput(w.tokens, world, fwd_ms), "unit": "tokens/s", "ms_per_step": fwd_ms},
         "step_roofline": {"bytes": sb, "tensor_flops": sf, "time_ms": t_roof * 1e3,
                           "frac": t_roof * 1e3 / ms_step},
         "roofline": roof,
@@ -536,10 +544,7 @@ def run_decode(args, w):
     launches = L.luna_launch_count() - n0
     dom_ms, dom_n = L.luna_profile_stop()
     clk = clocks.stop()
-    if world > 1:
-        t = torch.tensor([ms_step], device=dev)
-        tdist.all_reduce(t, op=tdist.ReduceOp.MAX)
-        ms_step = float(t.item())
+    ms_step = max_over_ranks(ms_step, dev, world)
     e2e = None
     if not args.no_e2e:
         o_host = torch.empty(o.shape, dtype=o.dtype).pin_memory()
@@ -552,11 +557,8 @@ def run_decode(args, w):
             e2e_step()
         torch.cuda.synchronize()
         e2e_ms = timed(max(3, args.steps // 4), e2e_step) / max(3, args.steps // 4)
-        if world > 1:
-            t = torch.tensor([e2e_ms], device=dev)
-            tdist.all_reduce(t, op=tdist.ReduceOp.MAX)
-            e2e_ms = float(t.item())
-        e2e = {"value": w.B * world / (e2e_ms * 1e-3), "unit": "tokens/s",
+        e2e_ms = max_over_ranks(e2e_ms, dev, world)
+        e2e = {"value": job_throughput(w.B, world, e2e_ms), "unit": "tokens/s",
                "h2d_bytes_per_step": int(sum(v.numel() * v.element_size() for v in host.values())),
                "d2h_bytes_per_step": int(o_host.numel() * o_host.element_size()), "ms_per_step": e2e_ms}
     hbm, _, peak_src = peaks()
@@ -568,7 +570,7 @@ def run_decode(args, w):
                 "frac": achieved / hbm, "traffic": None, "traffic_source": None, "peak_source": peak_src,
                 "algorithmic_bytes": byts, "launch_ms": dom_ms / dom_n, "launches": dom_n}
     result = {
-        "metric": DECODE_METRIC, "value": w.B * world / (ms_step * 1e-3), "unit": "tokens/s", "n_gpus": world,
+        "metric": DECODE_METRIC, "value": job_throughput(w.B, world, ms_step), "unit": "tokens/s", "n_gpus": world,
         "steps": args.steps, "warmup": args.warmup, "ms_per_step": ms_step, "higher_is_better": True,
         "scaling": "weak", "vs_baseline": None, "dtype": w.io, "data": "synthetic",
         "config": {"workload": f"{w.name}: B={w.B} H={w.H}, one token per sequence per step after a causal "
