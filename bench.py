@@ -609,8 +609,9 @@ def run_decode(args, w):
     roof = None
     if dom_n:
         achieved = byts / (dom_ms / dom_n * 1e-3) / 1e9
+        traffic, traffic_src = measured_traffic("decode", w.name) if args.seq_len <= 0 else (None, None)
         roof = {"bound": "hbm", "kernel": "decode", "achieved": achieved, "peak": hbm, "unit": "GB/s",
-                "frac": achieved / hbm, "traffic": None, "traffic_source": None, "peak_source": peak_src,
+                "frac": achieved / hbm, "traffic": traffic, "traffic_source": traffic_src, "peak_source": peak_src,
                 "algorithmic_bytes": byts, "launch_ms": dom_ms / dom_n, "launches": dom_n}
     result = {
         "metric": DECODE_METRIC, "value": job_throughput(w.B, world, ms_step), "unit": "tokens/s", "n_gpus": world,
