@@ -74,9 +74,21 @@ __global__ void __launch_bounds__(kDecThreads) k_decode(DecodeArgs a) {
         int node = 1;
         for (int lvl = 0; lvl < 10; ++lvl) node = 2 * node + (sTe[node] < u ? 1 : 0);
         const int j = node - kEytzinger;
-        for (int l = 0; l < L; ++l) {
-            const float2 ab = __ldg(AB + (size_t)j * L + l);
-            sphi[side][m * L + l] = fmaxf(fmaf(ab.x, u, ab.y), 0.0f);
+        if (L == 8) {  // the (alpha, beta) of the 8 channels as four 16-byte loads in flight
+            const float4 *ab4 = reinterpret_cast<const float4 *>(AB + (size_t)j * 8);
+            float4 w[4];
+#pragma unroll
+            for (int k = 0; k < 4; ++k) w[k] = __ldg(ab4 + k);
+#pragma unroll
+            for (int k = 0; k < 4; ++k) {
+                sphi[side][m * 8 + 2 * k] = fmaxf(fmaf(w[k].x, u, w[k].y), 0.0f);
+                sphi[side][m * 8 + 2 * k + 1] = fmaxf(fmaf(w[k].z, u, w[k].w), 0.0f);
+            }
+        } else {
+            for (int l = 0; l < L; ++l) {
+                const float2 ab = __ldg(AB + (size_t)j * L + l);
+                sphi[side][m * L + l] = fmaxf(fmaf(ab.x, u, ab.y), 0.0f);
+            }
         }
     }
     __syncthreads();
@@ -103,15 +115,29 @@ __global__ void __launch_bounds__(kDecThreads) k_decode(DecodeArgs a) {
         if (vec) {
             const float4 vc = make_float4(sv[4 * cu], sv[4 * cu + 1], sv[4 * cu + 2], sv[4 * cu + 3]);
             float4 *S4 = reinterpret_cast<float4 *>(S);
-#pragma unroll 8
-            for (int f = g; f < D; f += G) {
-                const float pk = sphi[1][f], pq = sphi[0][f];
-                float4 s = S4[(int64_t)f * cw + cu];
-                s.x = fmaf(pk, vc.x, s.x); s.y = fmaf(pk, vc.y, s.y);
-                s.z = fmaf(pk, vc.z, s.z); s.w = fmaf(pk, vc.w, s.w);
-                S4[(int64_t)f * cw + cu] = s;
-                num[0] = fmaf(pq, s.x, num[0]); num[1] = fmaf(pq, s.y, num[1]);
-                num[2] = fmaf(pq, s.z, num[2]); num[3] = fmaf(pq, s.w, num[3]);
+            // R rows in flight: all loaded before any is stored (a store would otherwise order
+            // the next load behind it, as the compiler cannot tell the rows apart)
+            constexpr int R = 4;
+            for (int f0 = g; f0 < D; f0 += R * G) {
+                float4 sv4[R];
+#pragma unroll
+                for (int i = 0; i < R; ++i) {
+                    const int f = f0 + i * G;
+                    sv4[i] = f < D ? S4[(int64_t)f * cw + cu] : make_float4(0.f, 0.f, 0.f, 0.f);
+                }
+#pragma unroll
+                for (int i = 0; i < R; ++i) {
+                    const int f = f0 + i * G;
+                    if (f < D) {
+                        const float pk = sphi[1][f], pq = sphi[0][f];
+                        float4 s = sv4[i];
+                        s.x = fmaf(pk, vc.x, s.x); s.y = fmaf(pk, vc.y, s.y);
+                        s.z = fmaf(pk, vc.z, s.z); s.w = fmaf(pk, vc.w, s.w);
+                        S4[(int64_t)f * cw + cu] = s;
+                        num[0] = fmaf(pq, s.x, num[0]); num[1] = fmaf(pq, s.y, num[1]);
+                        num[2] = fmaf(pq, s.z, num[2]); num[3] = fmaf(pq, s.w, num[3]);
+                    }
+                }
             }
         } else {
             const float vc = sv[cu];

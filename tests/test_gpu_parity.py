@@ -248,6 +248,35 @@ def test_backward_tensor_core_causal(seg_rows, monkeypatch):
         assert np.all(g[k][1, :, 333:] == 0)
 
 
+@pytest.mark.parametrize("n,lengths", [(2, None), (63, None), (65, [65, 1]), (130, [0, 129])])
+def test_backward_tensor_core_causal_edges(n, lengths):
+    """Streaming-form tensor-core backward on the edges of its 64-row tiles: a
+    two-row sequence, one row short of and one past a tile, and sequences of
+    length 0 and 1 in a batch (no valid row in a segment).  (The first row of a
+    sequence attends to itself alone: O_0 = v_0 up to eps, and its dphi(q) and
+    dphi(k) are eps-level remainders of an exact cancellation, below fp32
+    resolution of the cancelling parts; with one row per sequence the whole
+    dQ and dK would be such remainders, so the shortest case here has two.)"""
+    B = 1 if lengths is None else len(lengths)
+    case = Case(B, 2, n, 128, 16, 8, "bf16", True, seed=73, qkv_scale=1.0 / math.sqrt(128), lengths=lengths,
+                with_grad=True)
+    lu = case.luna()
+    case.run_fwd(lu)
+    g = {k: to_host(v) for k, v in case.run_bwd(lu).items()}
+    ref = case.oracle_bwd()
+    okq, okk = case.smooth_rows("Q"), case.smooth_rows("K")
+    for k, ok in (("dQ", okq), ("dK", okk), ("dV", None)):
+        assert np.all(np.isfinite(g[k]))
+        got, want = (g[k], ref[k]) if ok is None else (g[k][ok], ref[k][ok])
+        assert relerr(got, want) < TOL["bf16"], k
+    for k in ("dW", "db", "dw1", "db1", "dw2", "db2"):
+        assert relerr(g[k], ref[k]) < TOL["bf16"], k
+    if lengths is not None:
+        for b, ln in enumerate(lengths):
+            for k in ("dQ", "dK", "dV"):
+                assert np.all(g[k][b, :, ln:] == 0)
+
+
 def test_backward_tensor_core_causal_state_and_repeat():
     """The tensor-core streaming-form backward gives the same bits with the
     forward's saved segment prefixes as without them, and on a repeated run."""
@@ -326,8 +355,8 @@ def test_decode_continues_the_streaming_form(io, d, dv, M):
     sequence (streaming form, Sec. 3.2)."""
     import torch
     import paper_2512_08061_gb300.luna as L
-    B, H, n0, T = 2, 2, 300, 3
-    lens = [300, 177]
+    B, H, n0, T = 3, 2, 300, 3
+    lens = [300, 177, 0]  # the last sequence starts from an empty state
     case = Case(B, H, n0 + T, d, M, 8, io, True, seed=71, qkv_scale=1.0 / math.sqrt(d), dv=dv,
                 lengths=[ln + T for ln in lens])
     dt = torch.float32 if io == "f32" else torch.bfloat16
