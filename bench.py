@@ -24,6 +24,7 @@ import hashlib
 import json
 import math
 import os
+import re
 import statistics
 import subprocess
 import sys
@@ -124,24 +125,62 @@ def kernel_bytes(w, lengths, kernel: str) -> float:
     return float(table.get(kernel, 0.0))
 
 
-def csrc_digest() -> str:
-    """sha256 over the CUDA sources of the library (file names and contents)."""
+CSRC = os.path.join(ROOT, "paper_2512_08061_gb300", "csrc")
+
+
+def _includes(name: str, seen: set) -> None:
+    """`name` and the library headers it includes, transitively."""
+    if name in seen or not os.path.exists(os.path.join(CSRC, name)):
+        return
+    seen.add(name)
+    with open(os.path.join(CSRC, name)) as fh:
+        for line in fh:
+            m = re.match(r'\s*#\s*include\s+"([^"]+)"', line)
+            if m:
+                _includes(m.group(1), seen)
+
+
+def kernel_source(kernel: str):
+    """The CUDA source file that defines `k_<kernel>`, or None."""
+    pat = re.compile(r"\bk_" + re.escape(kernel) + r"\s*\(")
+    for f in sorted(os.listdir(CSRC)):
+        if f.endswith(".cu"):
+            with open(os.path.join(CSRC, f)) as fh:
+                if any(pat.search(line) and "__global__" in line for line in fh):
+                    return f
+    for f in sorted(os.listdir(CSRC)):  # definitions whose __global__ sits on the line before the name
+        if f.endswith(".cu"):
+            with open(os.path.join(CSRC, f)) as fh:
+                if pat.search(fh.read()):
+                    return f
+    return None
+
+
+def csrc_digest(kernel: str | None = None) -> str:
+    """sha256 over CUDA sources (file names and contents): the file that defines k_<kernel> and the
+    library headers it includes; with no kernel, every source of the library."""
+    files = set()
+    if kernel is not None:
+        src = kernel_source(kernel)
+        if src is not None:
+            _includes(src, files)
+    if not files:
+        files = {f for f in os.listdir(CSRC) if f.endswith((".cu", ".cuh"))}
     h = hashlib.sha256()
-    base = os.path.join(ROOT, "paper_2512_08061_gb300", "csrc")
-    for f in sorted(os.listdir(base)):
-        if f.endswith((".cu", ".cuh")):
-            h.update(f.encode())
-            with open(os.path.join(base, f), "rb") as fh:
-                h.update(fh.read())
+    for f in sorted(files):
+        h.update(f.encode())
+        with open(os.path.join(CSRC, f), "rb") as fh:
+            h.update(fh.read())
     return h.hexdigest()
 
 
 def measured_traffic(kernel: str, workload: str):
     """DRAM bytes (read + write) per launch of `kernel` from the committed ncu
-    summaries (lines `traffic <workload> k_<kernel> <bytes> <sources sha256>`),
-    or None when no summary was taken on the current sources."""
+    summaries (lines `traffic <workload> k_<kernel> <bytes> <sources sha256>`, the digest over the
+    kernel's own source file and the headers it includes), or None when no summary was taken on the
+    current sources."""
     pdir = os.path.join(ROOT, "profiles")
-    digest = csrc_digest()
+    digest = csrc_digest(kernel)
     try:
         names = sorted(os.listdir(pdir))
     except OSError:
