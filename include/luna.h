@@ -194,6 +194,17 @@ luna_status luna_attn_decode(const luna_attn_desc *ad, const luna_phi_desc *pd, 
  * synchronising or the copy failed (including an earlier asynchronous fault). */
 luna_status luna_device_status(void *workspace, void *stream);
 
+/* Diagnostic of the failure path (not needed for computation): launches one
+ * block that waits on a device-side barrier phase nothing ever completes,
+ * gives up after limit_ns nanoseconds of wall time (1 <= limit_ns <= 1e9) and
+ * sets the status word at the start of `workspace` exactly as a kernel of
+ * luna_attn_fwd / luna_attn_bwd whose bounded wait ran out does.  A following
+ * luna_device_status(workspace) then reports LUNA_ERR_DEVICE_TIMEOUT and clears
+ * the word; the CUDA context stays usable and later calls run normally.
+ * `workspace` as for luna_attn_fwd (256-byte aligned); LUNA_ERR_INVALID_ARG for
+ * NULL or a limit out of range. */
+luna_status luna_selftest_wait(void *workspace, int64_t limit_ns, void *stream);
+
 /* Size of the library-owned scratch array used by luna_attn_fwd_noalloc. */
 #define LUNA_NOALLOC_SCRATCH_BYTES (16u << 20)
 

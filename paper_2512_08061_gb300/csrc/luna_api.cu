@@ -392,6 +392,13 @@ luna_status luna_attn_decode(const luna_attn_desc *ad, const luna_phi_desc *pd, 
     return cuda_status(launch_decode(a, ad->io, static_cast<cudaStream_t>(stream)));
 }
 
+luna_status luna_selftest_wait(void *workspace, int64_t limit_ns, void *stream) {
+    if (!workspace || !aligned(workspace, 256) || limit_ns <= 0 || limit_ns > 1000000000LL)
+        return LUNA_ERR_INVALID_ARG;
+    return cuda_status(launch_selftest_wait(static_cast<int *>(workspace), (long long)limit_ns,
+                                            static_cast<cudaStream_t>(stream)));
+}
+
 luna_status luna_device_status(void *workspace, void *stream) {
     if (!workspace) return LUNA_ERR_INVALID_ARG;
     cudaStream_t s = static_cast<cudaStream_t>(stream);

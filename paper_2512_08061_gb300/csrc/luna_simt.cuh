@@ -47,6 +47,7 @@ struct DecodeArgs {
     int64_t S_stride, z_stride;  // elements between consecutive heads
 };
 cudaError_t launch_decode(const DecodeArgs &a, luna_dtype io, cudaStream_t s);
+cudaError_t launch_selftest_wait(int *status, long long limit_ns, cudaStream_t s);
 
 cudaError_t launch_phi_prepare(const luna_phi_params &prm, const TableLayout &lay, void *table, cudaStream_t s);
 cudaError_t launch_featmap(const TableLayout &lay, const char *table, const void *X, luna_dtype xt, int64_t rows,

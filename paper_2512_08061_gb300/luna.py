@@ -78,6 +78,7 @@ def _load():
         "luna_state_final": ([ad, pd, P, ctypes.POINTER(P), ctypes.POINTER(I64), ctypes.POINTER(P),
                               ctypes.POINTER(I64)], I),
         "luna_attn_decode": ([ad, pd, P, P, P, P, P, P, I64, P, I64, P], I),
+        "luna_selftest_wait": ([P, I64, P], I),
     }
     for name, (args, res) in sig.items():
         fn = getattr(lib, name)
@@ -90,7 +91,7 @@ _lib = _load()
 EXPORTED = ("luna_status_string", "luna_version", "luna_phi_table_size", "luna_phi_prepare", "luna_featmap",
             "luna_workspace_size", "luna_state_size", "luna_attn_fwd", "luna_attn_bwd", "luna_device_status",
             "luna_profile_start", "luna_profile_stop", "luna_launch_count", "luna_attn_fwd_noalloc",
-            "luna_state_final", "luna_attn_decode")
+            "luna_state_final", "luna_attn_decode", "luna_selftest_wait")
 
 
 def _ptr(t):
@@ -203,6 +204,10 @@ def luna_attn_decode(ad, pd, table, q, k, v, o, S, S_stride, z, z_stride, stream
 
 def luna_device_status(workspace: torch.Tensor, stream=None) -> int:
     return _lib.luna_device_status(_ptr(workspace), _stream(stream))
+
+
+def luna_selftest_wait(workspace: torch.Tensor, limit_ns: int, stream=None) -> None:
+    _check(_lib.luna_selftest_wait(_ptr(workspace), int(limit_ns), _stream(stream)), "luna_selftest_wait")
 
 
 def luna_profile_start(kernel: str) -> None:

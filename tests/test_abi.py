@@ -125,3 +125,10 @@ def test_decode_arguments_and_state_layout(L):
     nc = L.attn_desc(2, 3, 1000, 128, 128, causal=False)
     assert lib.luna_state_final(ctypes.byref(nc), ctypes.byref(pd), P(base), ctypes.byref(S), ctypes.byref(Ss),
                                 ctypes.byref(z), ctypes.byref(zs)) == 1
+
+
+def test_selftest_wait_arguments(L):
+    lib = L._lib
+    assert lib.luna_selftest_wait(None, 10_000_000, None) == 1
+    assert lib.luna_selftest_wait(ctypes.c_void_p(256), 0, None) == 1
+    assert lib.luna_selftest_wait(ctypes.c_void_p(256), 2_000_000_000, None) == 1

@@ -374,3 +374,21 @@ def test_decode_continues_the_streaming_form(io, d, dv, M):
     for t in range(T):
         want = np.stack([ref[b, :, lens[b] + t] for b in range(B)])
         assert relerr_rows(outs[t], want) < tol, t
+
+
+def test_bounded_wait_reports_timeout_and_context_stays_usable():
+    """Failure path of the bounded device waits: a wait on a barrier phase that
+    nothing completes gives up after 10 ms and sets the workspace's status word;
+    luna_device_status reports LUNA_ERR_DEVICE_TIMEOUT once and clears it, and
+    the same context then computes the same results as before."""
+    import paper_2512_08061_gb300.luna as L
+    case = Case(1, 2, 256, 64, 8, 8, "f32", False, seed=3)
+    lu = case.luna()
+    O1 = to_host(case.run_fwd(lu))
+    assert L.luna_device_status(lu.ws) == 0
+    L.luna_selftest_wait(lu.ws, 10_000_000)
+    assert L.luna_device_status(lu.ws) == 5  # LUNA_ERR_DEVICE_TIMEOUT
+    assert L.luna_device_status(lu.ws) == 0  # read once, then cleared
+    O2 = to_host(case.run_fwd(lu))
+    assert np.array_equal(O1, O2)
+    assert L.luna_device_status(lu.ws) == 0
