@@ -46,7 +46,7 @@ def build(force: bool = False) -> str:
 class _Phi(ctypes.Structure):
     _fields_ = [("d", ctypes.c_int), ("M", ctypes.c_int), ("L", ctypes.c_int), ("hid", ctypes.c_int)] + [
         (k, ctypes.c_void_p) for k in ("W", "b", "w1", "b1", "w2", "b2")
-    ]
+    ] + [("shared", ctypes.c_int)]
 
 
 _P = ctypes.c_void_p
@@ -89,18 +89,22 @@ def _f64(a) -> np.ndarray:
 
 
 class PhiParams:
-    """fp64 copies of the feature-map parameters (W, b, w1, b1, w2, b2)."""
+    """fp64 copies of the feature-map parameters (W, b, w1, b1, w2, b2).  One MLP per
+    channel: w1, b1, w2 of shape (L, hidden); the shared-channel MLP: w1, b1 of shape
+    (hidden,) and w2 of shape (L, hidden)."""
 
     def __init__(self, params: dict):
         self.arrays = {k: _f64(params[k]) for k in ("W", "b", "w1", "b1", "w2", "b2")}
         W = self.arrays["W"]
         self.M, self.d = W.shape
-        self.L, self.hid = self.arrays["w1"].shape
+        self.shared = self.arrays["w1"].ndim == 1
+        self.L, self.hid = self.arrays["w2"].shape
         assert self.arrays["b"].shape == (self.M,)
-        assert self.arrays["b1"].shape == self.arrays["w2"].shape == (self.L, self.hid)
+        assert self.arrays["w1"].shape == self.arrays["b1"].shape == ((self.hid,) if self.shared else (self.L, self.hid))
         assert self.arrays["b2"].shape == (self.L,)
         self.struct = _Phi(self.d, self.M, self.L, self.hid,
-                           *[self.arrays[k].ctypes.data for k in ("W", "b", "w1", "b1", "w2", "b2")])
+                           *[self.arrays[k].ctypes.data for k in ("W", "b", "w1", "b1", "w2", "b2")],
+                           int(self.shared))
 
     @property
     def D(self) -> int:
@@ -195,7 +199,7 @@ def attn_bwd(params, Q, K, V, dO, lengths=None, causal=False, eps=1e-6) -> dict:
     out = {
         "dQ": np.empty(Q.shape), "dK": np.empty(K.shape), "dV": np.empty(V.shape),
         "dW": np.empty((p.M, p.d)), "db": np.empty((p.M,)),
-        "dw1": np.empty((p.L, p.hid)), "db1": np.empty((p.L, p.hid)),
+        "dw1": np.empty(p.arrays["w1"].shape), "db1": np.empty(p.arrays["b1"].shape),
         "dw2": np.empty((p.L, p.hid)), "db2": np.empty((p.L,)),
     }
     lib().oracle_attn_bwd(p.ref(), B, H, n, dv, int(bool(causal)), float(eps),

@@ -23,6 +23,9 @@
  *     with k(x,y) = phi(x)^T phi(y) (Eq. kernel-attn read right to left).
  *   - the backward pass by the direct chain rule, sample by sample through
  *     every hidden unit of every channel MLP (ReLU'(0) taken as 0).
+ *   - the listing's shared_channels variant: one scalar MLP with L outputs
+ *     (fc1: 1 -> hid shared by the channels, fc2: hid -> L), so channel l
+ *     reads the same hidden units with its own fc2 row.
  *
  * Parity pinned by the CPU tests: hand-computed feature maps, the brute-force
  * quadratic form, closed-form special cases (constant channels give a plain
@@ -44,11 +47,15 @@ typedef struct {
     int hid;          /* hidden width of each channel MLP                */
     const double *W;  /* M x d                                           */
     const double *b;  /* M                                               */
-    const double *w1; /* L x hid, fc1 weight of channel l (fan-in 1)     */
-    const double *b1; /* L x hid                                         */
+    const double *w1; /* L x hid, fc1 weight of channel l (fan-in 1); hid if shared */
+    const double *b1; /* L x hid; hid if shared                          */
     const double *w2; /* L x hid, fc2 weight of channel l (fan-out 1)    */
     const double *b2; /* L                                               */
+    int shared;       /* 1: one MLP for all channels (fc1 shared)        */
 } oracle_phi;
+
+/* offset of channel l's fc1 row (the one shared row when shared) */
+static size_t fc1_row(const oracle_phi *p, int l) { return (size_t)(p->shared ? 0 : l) * p->hid; }
 
 typedef struct {
     double *dW, *db, *dw1, *db1, *dw2, *db2;
@@ -81,8 +88,8 @@ static double project(const oracle_phi *p, int i, const double *x) {
 
 /* y_l(u) = fc2(relu(fc1(u))) before the non-negativity ReLU (listing: ScalarMLP) */
 static double channel_pre(const oracle_phi *p, int l, double u) {
-    const double *w1 = p->w1 + (size_t)l * p->hid;
-    const double *b1 = p->b1 + (size_t)l * p->hid;
+    const double *w1 = p->w1 + fc1_row(p, l);
+    const double *b1 = p->b1 + fc1_row(p, l);
     const double *w2 = p->w2 + (size_t)l * p->hid;
     double y = p->b2[l];
     for (int k = 0; k < p->hid; ++k) y += w2[k] * relu(w1[k] * u + b1[k]);
@@ -117,8 +124,8 @@ void oracle_kink_margin(const oracle_phi *p, const double *X, int64_t rows, doub
         for (int i = 0; i < p->M; ++i) {
             double u = project(p, i, x);
             for (int l = 0; l < p->L; ++l) {
-                const double *w1 = p->w1 + (size_t)l * p->hid;
-                const double *b1 = p->b1 + (size_t)l * p->hid;
+                const double *w1 = p->w1 + fc1_row(p, l);
+                const double *b1 = p->b1 + fc1_row(p, l);
                 const double *w2 = p->w2 + (size_t)l * p->hid;
                 double y = p->b2[l], ysc = fabs(p->b2[l]);
                 for (int k = 0; k < p->hid; ++k) {
@@ -166,8 +173,8 @@ static void phi_rows_backward(const oracle_phi *p, const double *X, int64_t rows
                 if (!(y > 0.0)) continue; /* outer ReLU inactive */
                 double dy = dPhi[r * D + i * p->L + l] * s;
                 if (dy == 0.0) continue;
-                const double *w1 = p->w1 + (size_t)l * p->hid;
-                const double *b1 = p->b1 + (size_t)l * p->hid;
+                const double *w1 = p->w1 + fc1_row(p, l);
+                const double *b1 = p->b1 + fc1_row(p, l);
                 const double *w2 = p->w2 + (size_t)l * p->hid;
                 g->db2[l] += term(dy);
                 for (int k = 0; k < p->hid; ++k) {
@@ -175,8 +182,8 @@ static void phi_rows_backward(const oracle_phi *p, const double *X, int64_t rows
                     if (!(a > 0.0)) continue;
                     g->dw2[(size_t)l * p->hid + k] += term(dy * a);
                     double dh = dy * w2[k];
-                    g->dw1[(size_t)l * p->hid + k] += term(dh * u);
-                    g->db1[(size_t)l * p->hid + k] += term(dh);
+                    g->dw1[fc1_row(p, l) + k] += term(dh * u);  /* shared: summed over the channels */
+                    g->db1[fc1_row(p, l) + k] += term(dh);
                     du += dh * w1[k];
                 }
             }
@@ -399,17 +406,17 @@ void oracle_attn_bwd(const oracle_phi *p, int B, int H, int n, int dv, int causa
         attn_bwd_head(p, n, dv, causal, eps, Q + qo, K + qo, V + vo, dO + vo, head_len(lengths, bh / H, n),
                       dQ + qo, dK + qo, dV + vo, &g);
     }
-    /* ordered reduction over heads */
+    /* ordered reduction over heads (fc1 gradients: hid entries when the MLP is shared) */
     double *outs[6] = {dW, db, dw1, db1, dw2, db2};
-    size_t sizes[6] = {nW, nb, nh, nh, nh, nb2};
-    size_t off = 0;
+    const size_t n1 = p->shared ? (size_t)hid : nh;
+    size_t sizes[6] = {nW, nb, n1, n1, nh, nb2};
+    size_t offs[6] = {0, nW, nW + nb, nW + nb + nh, nW + nb + 2 * nh, nW + nb + 3 * nh};
     for (int t = 0; t < 6; ++t) {
         for (size_t e = 0; e < sizes[t]; ++e) {
             double acc = 0.0;
-            for (int bh = 0; bh < BH; ++bh) acc += part[(size_t)bh * per + off + e];
+            for (int bh = 0; bh < BH; ++bh) acc += part[(size_t)bh * per + offs[t] + e];
             outs[t][e] = acc;
         }
-        off += sizes[t];
     }
     free(part);
 }

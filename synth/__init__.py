@@ -128,20 +128,23 @@ class IOTensor:
 # ---------------------------------------------------------------------------
 # parameter and input recipes
 
-def phi_params(seed: int, d: int, M: int, L: int, hidden: int = 64) -> dict:
+def phi_params(seed: int, d: int, M: int, L: int, hidden: int = 64, shared: bool = False) -> dict:
     """Feature-map parameters, initialised as the paper's listing does.
 
     W ~ N(0,1)/sqrt(d) and b = 0 for the projections; each channel MLP uses the
     documented default of a linear layer (uniform in +-1/sqrt(fan_in)):
     fc1 (fan_in 1) in U(-1, 1), fc2 (fan_in = hidden) in U(-1/sqrt(hidden), ...).
+    With `shared`, one MLP serves all channels (the listing's shared_channels):
+    fc1 has `hidden` units (w1, b1 of shape (hidden,)) and fc2 has L outputs.
     All values are rounded to fp32.
     """
     bound2 = 1.0 / math.sqrt(hidden)
+    fc1 = (hidden,) if shared else (L, hidden)
     p = {
         "W": normal(seed, "phi.W", (M, d)) / math.sqrt(d),
         "b": np.zeros((M,)),
-        "w1": uniform(seed, "phi.w1", (L, hidden), -1.0, 1.0),
-        "b1": uniform(seed, "phi.b1", (L, hidden), -1.0, 1.0),
+        "w1": uniform(seed, "phi.w1", fc1, -1.0, 1.0),
+        "b1": uniform(seed, "phi.b1", fc1, -1.0, 1.0),
         "w2": uniform(seed, "phi.w2", (L, hidden), -bound2, bound2),
         "b2": uniform(seed, "phi.b2", (L,), -bound2, bound2),
     }

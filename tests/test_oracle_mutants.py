@@ -26,6 +26,9 @@ MUTANTS = {
         "for (int f = 0; f < D; ++f) num += phq[f] * S[(size_t)f * dv + c];",
         "for (int f = 0; f < D; ++f) num += phq[f] * S[(size_t)c * D + f];"),
     "inner ReLU mask dropped in backward": ("if (!(a > 0.0)) continue;\n                    g->dw2", "g->dw2"),
+    "shared fc1 read per channel": ("return (size_t)(p->shared ? 0 : l) * p->hid;", "return (size_t)l * p->hid;"),
+    "shared fc1 gradient not summed over channels": (
+        "g->dw1[fc1_row(p, l) + k] += term(dh * u);", "g->dw1[(size_t)l * p->hid + k] += term(dh * u);"),
 }
 
 

@@ -24,8 +24,8 @@ def _hand_params():
     return g, p
 
 
-def _rand_params(seed, d, M, L, hid):
-    return {k: v.astype(np.float64) for k, v in synth.phi_params(seed, d, M, L, hid).items()}
+def _rand_params(seed, d, M, L, hid, shared=False):
+    return {k: v.astype(np.float64) for k, v in synth.phi_params(seed, d, M, L, hid, shared).items()}
 
 
 def _rand_inputs(seed, B, H, n, d, dv, scale=1.0):
@@ -58,6 +58,58 @@ def test_phi_relu_special_case():
          "w2": np.ones((1, 1)), "b2": np.zeros(1)}
     X = synth.normal(7, "relu.X", (11, d))
     np.testing.assert_allclose(oracle.featmap(p, X), np.maximum(X, 0) / math.sqrt(d), rtol=0, atol=1e-15)
+
+
+def test_shared_mlp_with_one_channel_is_the_per_channel_mlp():
+    """Listing: ScalarMLP(L=1) is the same module whether it serves as the one
+    shared MLP or as the per-channel MLP of a single channel."""
+    d, M, hid = 4, 3, 5
+    ps = _rand_params(41, d, M, 1, hid, shared=True)
+    pc = dict(ps, w1=ps["w1"].reshape(1, hid), b1=ps["b1"].reshape(1, hid))
+    Q, K, V = _rand_inputs(41, 1, 2, 7, d, 3, scale=1.5)
+    dO = synth.normal(41, "shared1.dO", V.shape)
+    np.testing.assert_array_equal(oracle.featmap(ps, Q), oracle.featmap(pc, Q))
+    gs = oracle.attn_bwd(ps, Q, K, V, dO, causal=True)
+    gc = oracle.attn_bwd(pc, Q, K, V, dO, causal=True)
+    for k in gs:
+        np.testing.assert_allclose(gs[k].reshape(-1), gc[k].reshape(-1), rtol=1e-14, atol=0)
+
+
+def test_shared_mlp_by_hand():
+    """Shared-channel MLP (listing: one ScalarMLP with L outputs): fc1 units
+    relu(u), relu(-u) and fc2 rows selecting one unit each give
+    phi(x) = [relu(u), relu(-u)] / sqrt(M) for u = w^T x + b."""
+    p = {"W": np.array([[1.0, -2.0]]), "b": np.array([0.5]), "w1": np.array([1.0, -1.0]),
+         "b1": np.array([0.0, 0.0]), "w2": np.array([[1.0, 0.0], [0.0, 1.0]]), "b2": np.array([0.0, 0.0])}
+    X = np.array([[1.0, 0.0], [0.0, 1.0], [3.0, 1.0], [-1.0, 0.25]])
+    u = X @ p["W"][0] + p["b"][0]  # 1.5, -1.5, 1.5, -1.0
+    np.testing.assert_allclose(oracle.featmap(p, X), np.stack([np.maximum(u, 0), np.maximum(-u, 0)], axis=1),
+                               rtol=0, atol=1e-15)
+
+
+def test_shared_fc1_gradient_sums_over_channels():
+    """In the shared-channel MLP every channel reads every hidden unit, so the
+    fc1 gradients collect the chain rule through all channels: central finite
+    differences of sum(O * dO) in fp64 (both channels active on both units)."""
+    p = {"W": np.array([[0.8, -0.6]]), "b": np.array([0.1]), "w1": np.array([1.0, -1.0]),
+         "b1": np.array([0.1, 0.2]), "w2": np.array([[1.0, 0.5], [0.5, 1.0]]), "b2": np.array([0.05, 0.05])}
+    Q, K, V = _rand_inputs(43, 1, 1, 6, 2, 2, scale=1.5)
+    dO = synth.normal(43, "sharedfd.dO", V.shape)
+    for causal in (False, True):
+        g = oracle.attn_bwd(p, Q, K, V, dO, causal=causal, eps=1e-3)
+        h = 1e-6
+        for name, key in (("dw1", "w1"), ("db1", "b1"), ("dw2", "w2")):
+            arr = p[key].reshape(-1)
+            num = np.empty_like(arr)
+            for e in range(arr.size):
+                x0 = arr[e]
+                arr[e] = x0 + h
+                lp = _loss(p, Q, K, V, dO, None, causal, 1e-3)
+                arr[e] = x0 - h
+                lm = _loss(p, Q, K, V, dO, None, causal, 1e-3)
+                arr[e] = x0
+                num[e] = (lp - lm) / (2 * h)
+            np.testing.assert_allclose(g[name].reshape(-1), num, rtol=2e-5, atol=2e-7 * max(1.0, np.abs(num).max()))
 
 
 def test_phi_nonnegative_and_scale():
@@ -228,11 +280,12 @@ def _loss(p, Q, K, V, dO, lengths, causal, eps):
     return float(np.sum(oracle.attn_fwd(p, Q, K, V, lengths, causal=causal, eps=eps) * dO))
 
 
+@pytest.mark.parametrize("shared", [False, True])
 @pytest.mark.parametrize("causal", [False, True])
-def test_gradients_match_finite_differences(causal):
+def test_gradients_match_finite_differences(causal, shared):
     d, M, L, hid, n = 3, 2, 2, 3, 6
-    rng_seed = 21 if causal else 20
-    p = _rand_params(rng_seed, d, M, L, hid)
+    rng_seed = (21 if causal else 20) + (10 if shared else 0)
+    p = _rand_params(rng_seed, d, M, L, hid, shared)
     # push projections away from zero so that the hidden-unit pattern is rich
     Q, K, V = _rand_inputs(rng_seed, 2, 1, n, d, 2, scale=1.5)
     dO = synth.normal(rng_seed, "fd.dO", V.shape)
