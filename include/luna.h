@@ -63,24 +63,31 @@ typedef enum {
 typedef enum { LUNA_F32 = 0, LUNA_BF16 = 1 } luna_dtype;
 
 /* Shape of the feature map (Eq. phi-def-scalarenv; listing defaults hidden = 64).
+ * shared_channels = 0: one scalar MLP per channel (the listing's default);
+ * 1: one scalar MLP with L outputs serves all channels (the listing's
+ * shared_channels = True: fc1 Linear(1, hidden) shared, fc2 Linear(hidden, L)).
  * Supported: 1 <= M, 1 <= L <= 16, M*L <= 128, 1 <= hidden <= 128, L*hidden <= 512. */
 typedef struct {
-    int M;      /* number of projections w_i (rows of W)       */
-    int L;      /* number of channel functions psi_l           */
-    int hidden; /* hidden width of each channel MLP            */
+    int M;               /* number of projections w_i (rows of W)       */
+    int L;               /* number of channel functions psi_l           */
+    int hidden;          /* hidden width of each (or the shared) MLP     */
+    int shared_channels; /* 0 or 1, see above                           */
 } luna_phi_desc;
 
 /* Feature-map parameters, fp32 device arrays, row-major:
- *   W [M][d], b [M], w1 [L][hidden], b1 [L][hidden], w2 [L][hidden], b2 [L].
+ *   W [M][d], b [M], w1 [L][hidden], b1 [L][hidden], w2 [L][hidden], b2 [L];
+ *   with shared_channels, w1 and b1 are [hidden] (the one fc1).
  * w1[l][k], b1[l][k] are fc1 of channel l (Linear(1, hidden)); w2[l][k], b2[l]
- * are its fc2 (Linear(hidden, 1)). The same parameters serve queries and keys
- * and are shared by all heads (listing: "shared ... over tokens/heads"). */
+ * are its fc2 (Linear(hidden, 1)), or row l of the shared fc2. The same
+ * parameters serve queries and keys and are shared by all heads (listing:
+ * "shared ... over tokens/heads"). */
 typedef struct {
     const float *W, *b, *w1, *b1, *w2, *b2;
 } luna_phi_params;
 
 /* Gradients of the feature-map parameters, fp32 device arrays with the shapes
- * of luna_phi_params.  They are OVERWRITTEN (not accumulated) by luna_attn_bwd. */
+ * of luna_phi_params (dw1, db1 of [hidden] with shared_channels).  They are
+ * OVERWRITTEN (not accumulated) by luna_attn_bwd. */
 typedef struct {
     float *dW, *db, *dw1, *db1, *dw2, *db2;
 } luna_phi_grads;

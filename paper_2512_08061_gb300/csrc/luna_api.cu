@@ -20,6 +20,7 @@ int64_t round_up(int64_t a, int64_t b) { return cdiv(a, b) * b; }
 luna_status check_phi(const luna_phi_desc *pd, int d) {
     if (!pd) return LUNA_ERR_INVALID_ARG;
     if (pd->M < 1 || pd->L < 1 || pd->hidden < 1 || d < 1) return LUNA_ERR_INVALID_ARG;
+    if (pd->shared_channels != 0 && pd->shared_channels != 1) return LUNA_ERR_INVALID_ARG;
     if (pd->L > kMaxL || pd->M * pd->L > kMaxFeat || pd->M > 32 || pd->hidden > kMaxHidden ||
         pd->L * pd->hidden > kMaxUnits || d > kMaxD || pd->M * d > 4096)
         return LUNA_ERR_UNSUPPORTED;
@@ -62,7 +63,7 @@ luna_status make_plan(const luna_attn_desc *ad, const luna_phi_desc *pd, Plan &p
     if (ad->dv > kMaxD || ad->n > (1 << 24)) return LUNA_ERR_UNSUPPORTED;
     if ((int64_t)ad->B * ad->H > (1 << 24)) return LUNA_ERR_UNSUPPORTED;
 
-    p.lay = table_layout(pd->M, pd->L, pd->hidden, ad->d);
+    p.lay = table_layout(pd->M, pd->L, pd->hidden, ad->d, pd->shared_channels);
     const int BH = ad->B * ad->H, n = ad->n, D = p.lay.D, dv = ad->dv;
     p.BH = BH;
     p.gsize = pd->M * ad->d + pd->M + p.lay.nint * pd->L * 2;
@@ -210,7 +211,7 @@ luna_status luna_phi_table_size(const luna_phi_desc *pd, int d, size_t *bytes) {
     if (!bytes) return LUNA_ERR_INVALID_ARG;
     luna_status st = check_phi(pd, d);
     if (st != LUNA_OK) return st;
-    *bytes = (size_t)table_layout(pd->M, pd->L, pd->hidden, d).bytes;
+    *bytes = (size_t)table_layout(pd->M, pd->L, pd->hidden, d, pd->shared_channels).bytes;
     return LUNA_OK;
 }
 
@@ -221,7 +222,7 @@ luna_status luna_phi_prepare(const luna_phi_desc *pd, int d, const luna_phi_para
     if (!params || !table || !params->W || !params->b || !params->w1 || !params->b1 || !params->w2 || !params->b2)
         return LUNA_ERR_INVALID_ARG;
     if (!aligned(table, 256)) return LUNA_ERR_INVALID_ARG;
-    TableLayout lay = table_layout(pd->M, pd->L, pd->hidden, d);
+    TableLayout lay = table_layout(pd->M, pd->L, pd->hidden, d, pd->shared_channels);
     if (table_bytes < (size_t)lay.bytes) return LUNA_ERR_WORKSPACE;
     return cuda_status(launch_phi_prepare(*params, lay, table, static_cast<cudaStream_t>(stream)));
 }
@@ -233,7 +234,7 @@ luna_status luna_featmap(const luna_phi_desc *pd, int d, const void *table, cons
     if (rows < 0 || (xtype != LUNA_F32 && xtype != LUNA_BF16)) return LUNA_ERR_INVALID_ARG;
     if (rows == 0) return LUNA_OK;
     if (!table || !X || !Phi) return LUNA_ERR_INVALID_ARG;
-    TableLayout lay = table_layout(pd->M, pd->L, pd->hidden, d);
+    TableLayout lay = table_layout(pd->M, pd->L, pd->hidden, d, pd->shared_channels);
     return cuda_status(launch_featmap(lay, static_cast<const char *>(table), X, xtype, rows, Phi,
                                       static_cast<cudaStream_t>(stream)));
 }
@@ -297,10 +298,11 @@ luna_status luna_attn_bwd(const luna_attn_desc *ad, const luna_phi_desc *pd, con
     cudaStream_t s = static_cast<cudaStream_t>(stream);
     if (p.BH == 0 || ad->n == 0) {  // empty problem: parameter gradients are zero
         const size_t Md = (size_t)pd->M * ad->d, P = (size_t)pd->L * pd->hidden;
+        const size_t P1 = pd->shared_channels ? (size_t)pd->hidden : P;  // fc1 entries
         cudaError_t e = cudaMemsetAsync(grads->dW, 0, Md * 4, s);
         if (e == cudaSuccess) e = cudaMemsetAsync(grads->db, 0, pd->M * 4, s);
-        if (e == cudaSuccess) e = cudaMemsetAsync(grads->dw1, 0, P * 4, s);
-        if (e == cudaSuccess) e = cudaMemsetAsync(grads->db1, 0, P * 4, s);
+        if (e == cudaSuccess) e = cudaMemsetAsync(grads->dw1, 0, P1 * 4, s);
+        if (e == cudaSuccess) e = cudaMemsetAsync(grads->db1, 0, P1 * 4, s);
         if (e == cudaSuccess) e = cudaMemsetAsync(grads->dw2, 0, P * 4, s);
         if (e == cudaSuccess) e = cudaMemsetAsync(grads->db2, 0, pd->L * 4, s);
         return cuda_status(e);
@@ -373,7 +375,7 @@ luna_status luna_attn_decode(const luna_attn_desc *ad, const luna_phi_desc *pd, 
     if (ad->dv > kMaxD) return LUNA_ERR_UNSUPPORTED;
     const int64_t BH = (int64_t)ad->B * ad->H;
     if (BH > (1 << 24)) return LUNA_ERR_UNSUPPORTED;
-    const TableLayout lay = table_layout(pd->M, pd->L, pd->hidden, ad->d);
+    const TableLayout lay = table_layout(pd->M, pd->L, pd->hidden, ad->d, pd->shared_channels);
     const int64_t SD = (int64_t)lay.D * ad->dv;
     if (S_stride == 0) S_stride = SD;
     if (z_stride == 0) z_stride = lay.D;

@@ -32,18 +32,20 @@ __host__ __device__ inline int64_t align256(int64_t x) { return (x + 255) & ~int
 //                          complete 1023-node search tree, index 0 unused, +inf padding
 //   AB     [nint][L][2]    per merged interval j and channel l: (alpha, beta) / sqrt(M)
 //   W      [M][d], b [M]   projection copy
-//   rank   [P]             position of unit (l,k) in the sorted kink list
+//   rank   [P]             position of unit (l,k) (shared MLP: unit k) in the sorted kink list
 //   utype  [P]             +1: unit active iff u > T[rank] ; -1: active iff u <= T[rank]
-//   w1, b1, w2 [P], b2 [L] channel-MLP parameter copy (used by the gradient reduction)
+//   w1, b1 [P], w2 [L*hid], b2 [L]  channel-MLP parameter copy (used by the gradient reduction)
 struct TableLayout {
     int M, L, hid, d, D, P, Ppad, nint;
+    int shared;  // one MLP for all channels: P = hid kinks (else P = L * hid)
     int64_t off_T, off_Te, off_AB, off_W, off_b, off_rank, off_utype, off_w1, off_b1, off_w2, off_b2, bytes;
 };
 
-__host__ __device__ inline TableLayout table_layout(int M, int L, int hid, int d) {
+__host__ __device__ inline TableLayout table_layout(int M, int L, int hid, int d, int shared = 0) {
     TableLayout t;
     t.M = M; t.L = L; t.hid = hid; t.d = d; t.D = M * L;
-    t.P = L * hid;
+    t.shared = shared ? 1 : 0;
+    t.P = shared ? hid : L * hid;
     t.Ppad = next_pow2(t.P);
     t.nint = t.P + 1;
     int64_t o = 256;  // header
@@ -56,7 +58,7 @@ __host__ __device__ inline TableLayout table_layout(int M, int L, int hid, int d
     t.off_utype = o; o = align16(o + 4 * (int64_t)t.P);
     t.off_w1 = o;    o = align16(o + 4 * (int64_t)t.P);
     t.off_b1 = o;    o = align16(o + 4 * (int64_t)t.P);
-    t.off_w2 = o;    o = align16(o + 4 * (int64_t)t.P);
+    t.off_w2 = o;    o = align16(o + 4 * (int64_t)L * hid);
     t.off_b2 = o;    o = align16(o + 4 * (int64_t)L);
     t.bytes = align256(o);
     return t;

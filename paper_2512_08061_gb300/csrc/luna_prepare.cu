@@ -1,9 +1,11 @@
 // Feature-map table: the exact piecewise-linear form of the channel MLPs.
 //
 // Each channel function of the listing's ScalarMLP is
-//     psi_l(u) = relu( b2[l] + sum_k w2[l,k] relu(w1[l,k] u + b1[l,k]) ),
-// a ReLU network of one scalar, hence linear in u between the kinks of its
-// hidden units.  Merging the kinks of all L*hidden units into one sorted list
+//     psi_l(u) = relu( b2[l] + sum_k w2[l,k] relu(w1[l,k] u + b1[l,k]) )
+// (with the shared-channel MLP, w1[k], b1[k] for every l), a ReLU network of
+// one scalar, hence linear in u between the kinks of its hidden units.
+// Merging the kinks of all P hidden units (L*hidden, or hidden when shared)
+// into one sorted list
 // T gives intervals j = #{p : T[p] < u} on which every hidden unit of every
 // channel is either on or off, so
 //     psi_l(u) = relu(alpha[j][l] * u + beta[j][l]).
@@ -51,10 +53,17 @@ __device__ __forceinline__ bool pair_less(float ta, int ka, float tb, int kb) {
     return ta < tb || (ta == tb && ka < kb);
 }
 
+// Position of input unit `unit` (fc1 index: l*hid + k, or k when shared) in the
+// per-unit arrays, which are kept in [k][l] order (k only when shared).
+__device__ __forceinline__ int unit_pos(const TableLayout &lay, int unit) {
+    return lay.shared ? unit : (unit % lay.hid) * lay.L + unit / lay.hid;
+}
+
 __global__ void __launch_bounds__(kPrepThreads) k_phi_prepare(luna_phi_params prm, TableLayout lay, char *table) {
     __shared__ float sk[kMaxUnits];
     __shared__ int si[kMaxUnits];
-    __shared__ float w1t[kMaxUnits], b1t[kMaxUnits], w2t[kMaxUnits];  // per-unit values in [k][l] order
+    __shared__ float w1t[kMaxUnits], b1t[kMaxUnits];  // per-unit fc1 values
+    __shared__ float w2t[kMaxUnits];                  // fc2 weight of (unit k, channel l) at k*L + l
     __shared__ int tyt[kMaxUnits], rkt[kMaxUnits];
     const int tid = threadIdx.x, nt = blockDim.x;
     const int P = lay.P, N = lay.Ppad, L = lay.L, hid = lay.hid;  // N: power of two >= P, <= kMaxUnits
@@ -66,9 +75,10 @@ __global__ void __launch_bounds__(kPrepThreads) k_phi_prepare(luna_phi_params pr
         if (w > 0.0f) { key = up_threshold(w, c); ty = 1; }
         else if (w < 0.0f) { key = down_threshold(w, c); ty = -1; }
         else { key = INFINITY; ty = (c > 0.0f) ? -1 : 1; }  // constant unit: always on / always off
-        const int tpos = (tid % hid) * L + tid / hid;
-        w1t[tpos] = w; b1t[tpos] = c; w2t[tpos] = prm.w2[tid]; tyt[tpos] = ty;
+        const int tpos = unit_pos(lay, tid);
+        w1t[tpos] = w; b1t[tpos] = c; tyt[tpos] = ty;
     }
+    for (int e = tid; e < L * hid; e += nt) w2t[(e % hid) * L + e / hid] = prm.w2[e];  // w2[l][k]
     // bitonic sort of the first N elements (positions >= N sort among themselves)
     for (int size = 2; size <= N; size <<= 1) {
         for (int stride = size >> 1; stride > 0; stride >>= 1) {
@@ -91,7 +101,7 @@ __global__ void __launch_bounds__(kPrepThreads) k_phi_prepare(luna_phi_params pr
     }
     sk[tid] = key;
     si[tid] = idx;
-    if (idx < P) rkt[(idx % hid) * L + idx / hid] = tid;
+    if (idx < P) rkt[unit_pos(lay, idx)] = tid;
     __syncthreads();
 
     if (blockIdx.x == 0) {
@@ -103,12 +113,12 @@ __global__ void __launch_bounds__(kPrepThreads) k_phi_prepare(luna_phi_params pr
             if (si[r] < P) rank[si[r]] = r;
         }
         for (int k = tid; k < P; k += nt) {
-            const int tpos = (k % hid) * L + k / hid;
+            const int tpos = unit_pos(lay, k);
             utype[k] = tyt[tpos];
             reinterpret_cast<float *>(table + lay.off_w1)[k] = w1t[tpos];
             reinterpret_cast<float *>(table + lay.off_b1)[k] = b1t[tpos];
-            reinterpret_cast<float *>(table + lay.off_w2)[k] = w2t[tpos];
         }
+        for (int e = tid; e < L * hid; e += nt) reinterpret_cast<float *>(table + lay.off_w2)[e] = prm.w2[e];
         // breadth-first (Eytzinger) copy: node e at depth d, position p in its level
         // holds the in-order element (2p+1) * 2^(9-d) - 1
         float *Te = reinterpret_cast<float *>(table + lay.off_Te);
@@ -143,11 +153,12 @@ __global__ void __launch_bounds__(kPrepThreads) k_phi_prepare(luna_phi_params pr
         const int j = live ? e / L : 0, l = live ? e % L : 0;
         float a = 0.0f, bsum = 0.0f;
         for (int k = p; k < hid; k += kPrepSplit) {
-            const int u = k * L + l;
+            const int u = lay.shared ? k : k * L + l;  // the unit's kink and fc1
             const bool on = (tyt[u] > 0) ? (rkt[u] < j) : (rkt[u] >= j);
             if (on) {
-                a = fmaf(w2t[u], w1t[u], a);
-                bsum = fmaf(w2t[u], b1t[u], bsum);
+                const float w2 = w2t[k * L + l];
+                a = fmaf(w2, w1t[u], a);
+                bsum = fmaf(w2, b1t[u], bsum);
             }
         }
 #pragma unroll

@@ -378,9 +378,11 @@ __device__ void warp_scan(const float *x, double *y, int n, bool backward) {
 }
 
 // Block l < L: hidden units of channel l from prefix and suffix sums of the
-// channel's interval histogram.  Block L: dW and db.
+// channel's interval histogram.  Block L: dW and db.  With the shared-channel
+// MLP every channel reads every hidden unit: block l writes its channel's fc1
+// contributions to fc1_part ([dw1 | db1][l][k], fp64), summed by k_mlp_fc1_sum.
 __global__ void __launch_bounds__(128) k_mlp_grads(TableLayout lay, const char *table, const float *gsum,
-                                                   luna_phi_grads grads) {
+                                                   luna_phi_grads grads, double *fc1_part) {
     __shared__ float h[2][kMaxUnits + 1];
     __shared__ double pre[2][kMaxUnits + 1], suf[2][kMaxUnits + 1];  // fp64: dw2 = w1 G1 + b1 G0 cancels
     const int Md = lay.M * lay.d, L = lay.L, hid = lay.hid, nint = lay.nint;
@@ -406,7 +408,8 @@ __global__ void __launch_bounds__(128) k_mlp_grads(TableLayout lay, const char *
     const float *b1 = reinterpret_cast<const float *>(table + lay.off_b1);
     const float *w2 = reinterpret_cast<const float *>(table + lay.off_w2);
     for (int k = threadIdx.x; k < hid; k += blockDim.x) {
-        const int u = l * hid + k;
+        const int u = lay.shared ? k : l * hid + k;  // the unit: its kink and fc1
+        const int uw = l * hid + k;                  // fc2 weight (l, k)
         const int r = rank[u];
         double G0, G1;
         if (utype[u] > 0) {  // active on intervals j > r
@@ -416,11 +419,31 @@ __global__ void __launch_bounds__(128) k_mlp_grads(TableLayout lay, const char *
             G0 = pre[0][r];
             G1 = pre[1][r];
         }
-        grads.dw2[u] = (float)(((double)w1[u] * G1 + (double)b1[u] * G0) * (double)scale);
-        grads.dw1[u] = (float)((double)w2[u] * G1 * (double)scale);
-        grads.db1[u] = (float)((double)w2[u] * G0 * (double)scale);
+        grads.dw2[uw] = (float)(((double)w1[u] * G1 + (double)b1[u] * G0) * (double)scale);
+        const double c1 = (double)w2[uw] * G1 * (double)scale, c0 = (double)w2[uw] * G0 * (double)scale;
+        if (lay.shared) {
+            fc1_part[(size_t)l * hid + k] = c1;
+            fc1_part[(size_t)(L + l) * hid + k] = c0;
+        } else {
+            grads.dw1[u] = (float)c1;
+            grads.db1[u] = (float)c0;
+        }
     }
     if (threadIdx.x == 0) grads.db2[l] = (float)(pre[0][nint - 1] * (double)scale);
+}
+
+// Shared-channel MLP: dw1[k], db1[k] = sums over the channels (in order) of their contributions.
+__global__ void __launch_bounds__(128) k_mlp_fc1_sum(TableLayout lay, const double *fc1_part, luna_phi_grads grads) {
+    const int L = lay.L, hid = lay.hid;
+    for (int k = threadIdx.x; k < hid; k += blockDim.x) {
+        double a = 0.0, b = 0.0;
+        for (int l = 0; l < L; ++l) {
+            a += fc1_part[(size_t)l * hid + k];
+            b += fc1_part[(size_t)(L + l) * hid + k];
+        }
+        grads.dw1[k] = (float)a;
+        grads.db1[k] = (float)b;
+    }
 }
 
 // ---------------------------------------------------------------------------
@@ -500,7 +523,11 @@ cudaError_t launch_grad_reduce(const AttnArgs &a, int nparts, cudaStream_t s) {
                 nparts, a.gsize, a.hist);
     cudaError_t e = cudaGetLastError();
     if (e != cudaSuccess) return e;
-    LUNA_LAUNCH("mlp_grads", k_mlp_grads, a.lay.L + 1, 128, 0, s, a.lay, a.table, a.hist, a.grads);
+    // the partials have been summed: their buffer holds the shared MLP's per-channel fc1 terms
+    double *fc1_part = reinterpret_cast<double *>(a.gpart);
+    LUNA_LAUNCH("mlp_grads", k_mlp_grads, a.lay.L + 1, 128, 0, s, a.lay, a.table, a.hist, a.grads, fc1_part);
+    if ((e = cudaGetLastError()) != cudaSuccess || !a.lay.shared) return e;
+    LUNA_LAUNCH("mlp_fc1_sum", k_mlp_fc1_sum, 1, 128, 0, s, a.lay, fc1_part, a.grads);
     return cudaGetLastError();
 }
 

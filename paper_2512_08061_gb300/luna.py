@@ -32,7 +32,7 @@ class LunaError(RuntimeError):
 
 
 class PhiDesc(ctypes.Structure):
-    _fields_ = [("M", ctypes.c_int), ("L", ctypes.c_int), ("hidden", ctypes.c_int)]
+    _fields_ = [("M", ctypes.c_int), ("L", ctypes.c_int), ("hidden", ctypes.c_int), ("shared_channels", ctypes.c_int)]
 
 
 class PhiParams(ctypes.Structure):
@@ -117,8 +117,8 @@ def _io_code(t: torch.Tensor) -> int:
     return _DTYPES[t.dtype]
 
 
-def phi_desc(M: int, L: int, hidden: int) -> PhiDesc:
-    return PhiDesc(M, L, hidden)
+def phi_desc(M: int, L: int, hidden: int, shared: bool = False) -> PhiDesc:
+    return PhiDesc(M, L, hidden, int(bool(shared)))
 
 
 def attn_desc(B, H, n, d, dv, causal=False, chunk=0, eps=1e-6, io=LUNA_BF16) -> AttnDesc:
@@ -236,8 +236,8 @@ class Luna:
     """Owns the table, workspace and state buffers of one problem shape."""
 
     def __init__(self, B, H, n, d, dv, M, L, hidden=64, causal=False, eps=1e-6, io=torch.bfloat16, chunk=0,
-                 device="cuda"):
-        self.pd = phi_desc(M, L, hidden)
+                 device="cuda", shared=False):
+        self.pd = phi_desc(M, L, hidden, shared)
         self.ad = attn_desc(B, H, n, d, dv, causal, chunk, eps, _DTYPES[io])
         self.d = d
         self.device = torch.device(device)
@@ -260,9 +260,10 @@ class Luna:
         if out is None:
             M, L, hid = self.pd.M, self.pd.L, self.pd.hidden
             f32 = dict(dtype=torch.float32, device=Q.device)
+            fc1 = (hid,) if self.pd.shared_channels else (L, hid)
             out = {"dQ": torch.empty_like(Q), "dK": torch.empty_like(K), "dV": torch.empty_like(V),
                    "dW": torch.empty(M, self.d, **f32), "db": torch.empty(M, **f32),
-                   "dw1": torch.empty(L, hid, **f32), "db1": torch.empty(L, hid, **f32),
+                   "dw1": torch.empty(fc1, **f32), "db1": torch.empty(fc1, **f32),
                    "dw2": torch.empty(L, hid, **f32), "db2": torch.empty(L, **f32)}
         luna_attn_bwd(self.ad, self.pd, self.table, Q, K, V, dO, lengths, self.state if use_state else None,
                       out["dQ"], out["dK"], out["dV"], out, self.ws, stream)

@@ -73,11 +73,11 @@ def to_host(x) -> np.ndarray:
 
 class Case:
     def __init__(self, B, H, n, d, M, L, io, causal=False, seed=0, qkv_scale=1.0, len_range=None, hidden=64,
-                 eps=1e-6, dv=None, with_grad=False, lengths=None):
+                 eps=1e-6, dv=None, with_grad=False, lengths=None, shared=False):
         self.B, self.H, self.n, self.d, self.M, self.L = B, H, n, d, M, L
         self.dv = dv or d
-        self.io, self.causal, self.eps, self.hidden = io, causal, eps, hidden
-        self.params = synth.phi_params(seed, d, M, L, hidden)
+        self.io, self.causal, self.eps, self.hidden, self.shared = io, causal, eps, hidden, shared
+        self.params = synth.phi_params(seed, d, M, L, hidden, shared)
         self.inp = synth.attn_inputs(seed, B, H, n, d, self.dv, io, qkv_scale, len_range, with_grad)
         if lengths is not None:
             self.inp["lengths"] = np.asarray(lengths, dtype=np.int32)
@@ -88,7 +88,7 @@ class Case:
         import torch
         import paper_2512_08061_gb300.luna as L
         lu = L.Luna(self.B, self.H, self.n, self.d, self.dv, self.M, self.L, self.hidden, self.causal, self.eps,
-                    torch.float32 if self.io == "f32" else torch.bfloat16, chunk)
+                    torch.float32 if self.io == "f32" else torch.bfloat16, chunk, shared=self.shared)
         params = {k: torch.from_numpy(v).cuda() for k, v in self.params.items()}
         lu.prepare(params)
         self.dev = {k: to_device(self.inp[k]) for k in ("Q", "K", "V", "dO") if k in self.inp}

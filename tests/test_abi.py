@@ -132,3 +132,15 @@ def test_selftest_wait_arguments(L):
     assert lib.luna_selftest_wait(None, 10_000_000, None) == 1
     assert lib.luna_selftest_wait(ctypes.c_void_p(256), 0, None) == 1
     assert lib.luna_selftest_wait(ctypes.c_void_p(256), 2_000_000_000, None) == 1
+
+
+def test_shared_channel_descriptor(L):
+    """shared_channels must be 0 or 1; the shared-channel table holds the kinks of
+    the one fc1 (hidden of them), so it is smaller than the per-channel table."""
+    with pytest.raises(L.LunaError) as e:
+        pd = L.PhiDesc(8, 8, 64, 2)
+        L.luna_phi_table_size(pd, 32)
+    assert e.value.status == 1
+    per = L.luna_phi_table_size(L.phi_desc(8, 8, 64), 32)
+    shared = L.luna_phi_table_size(L.phi_desc(8, 8, 64, shared=True), 32)
+    assert 0 < shared < per

@@ -392,3 +392,48 @@ def test_bounded_wait_reports_timeout_and_context_stays_usable():
     O2 = to_host(case.run_fwd(lu))
     assert np.array_equal(O1, O2)
     assert L.luna_device_status(lu.ws) == 0
+
+
+@pytest.mark.parametrize("io,d,M,causal", [("bf16", 32, 8, False), ("f32", 64, 8, True), ("bf16", 128, 16, True),
+                                           ("bf16", 64, 8, False)])
+def test_shared_channel_mlp(io, d, M, causal):
+    """The listing's shared_channels option (one MLP with L outputs): forward and
+    backward through the tensor-core path (bf16 non-causal d = 32 and 64, the
+    streaming form at d = 128) and the generic path (fp32), every gradient
+    including dw1, db1 of the one shared fc1 (summed over the channels)."""
+    case = Case(2, 2, 300, d, M, 8, io, causal, seed=79, qkv_scale=1.0 / math.sqrt(d), lengths=[300, 177],
+                with_grad=True, shared=True)
+    lu = case.luna()
+    O = to_host(case.run_fwd(lu))
+    ref = case.oracle_fwd()
+    assert (relerr_rows(O, ref) if causal else relerr(O, ref)) < TOL[io]
+    g = {k: to_host(v) for k, v in case.run_bwd(lu).items()}
+    rb = case.oracle_bwd()
+    okq, okk = case.smooth_rows("Q"), case.smooth_rows("K")
+    assert relerr(g["dQ"][okq], rb["dQ"][okq]) < TOL[io]
+    assert relerr(g["dK"][okk], rb["dK"][okk]) < TOL[io]
+    assert relerr(g["dV"], rb["dV"]) < TOL[io]
+    assert g["dw1"].shape == (64,) and g["db1"].shape == (64,)
+    if io == "f32":
+        A = case.oracle_bwd_abs_terms()
+        for k in ("dW", "db", "dw1", "db1", "dw2", "db2"):
+            assert sum_err(g[k], rb[k], A[k], TOL[io]) <= 1.0, k
+    else:
+        for k in ("dW", "db", "dw1", "db1", "dw2", "db2"):
+            assert relerr(g[k], rb[k]) < TOL[io], k
+
+
+def test_shared_channel_featmap():
+    """luna_featmap of the shared-channel MLP against the oracle, with the
+    kinks of the one fc1 (64 kinks, 65 intervals)."""
+    import torch
+    import paper_2512_08061_gb300.luna as L
+    d, M = 64, 8
+    params = synth.phi_params(83, d, M, 8, 64, shared=True)
+    X = synth.IOTensor(synth.normal(83, "fms.X", (777, d)), "f32")
+    pd = L.phi_desc(M, 8, 64, shared=True)
+    table = L.alloc_bytes(L.luna_phi_table_size(pd, d), "cuda")
+    L.luna_phi_prepare(pd, d, {k: torch.from_numpy(v).cuda() for k, v in params.items()}, table)
+    Phi = torch.empty(777, M * 8, dtype=torch.float32, device="cuda")
+    L.luna_featmap(pd, d, table, to_device(X), Phi)
+    assert relerr(to_host(Phi), oracle.featmap(params, X.value)) < 1e-4
