@@ -121,9 +121,10 @@ __device__ __forceinline__ uint4 pack8(const float (&y)[8]) {
 //
 // Shared-memory fp32 atomics are compare-and-swap loops; int32 atomics are
 // native and about five times faster.  So the bins hold fixed-point int32 sums
-// over groups of kHistTiles tiles, quantised with power-of-two scales 2^e such
+// over groups of hist_tiles() tiles, quantised with power-of-two scales 2^e such
 // that |q| < 2^kHistQBits for the scale's reference maxima of |g| and |g*u|; a
-// bin receives at most 1024 samples per tile, so a group stays below 2^30.  The
+// group holds at most 4096 samples (four tiles of 128 rows x 8 projections,
+// two of 128 x 16), so a bin stays below 2^30.  The
 // block's first group takes its reference maxima from a pre-pass over its
 // first tile with a nonzero g, every later group from the block-wide maxima of
 // the group before it.  A value that does not fit (it outgrew the reference,
@@ -137,7 +138,13 @@ __device__ __forceinline__ uint4 pack8(const float (&y)[8]) {
 __device__ __forceinline__ int hist_at(int c, int l, int j) { return (c * 8 + l) * kNint + j; }
 
 constexpr int kHistQBits = 18;  // |q| < 2^18 per sample
-constexpr int kHistTiles = 4;   // tiles per group: 4 * 1024 * 2^18 = 2^30
+constexpr int kHistSamples = 4096;  // samples per group: 4096 * 2^18 = 2^30
+// Tiles per group for 128-row tiles of MP projections each.
+template <int MP>
+__host__ __device__ constexpr int hist_tiles() {
+    static_assert(kHistSamples % (128 * MP) == 0, "whole tiles per group");
+    return kHistSamples / (128 * MP);
+}
 
 // 2^e as a float, e in [-126, 127] (IEEE-754 binary32: biased exponent, zero mantissa).
 __device__ __forceinline__ float pow2f(int e) { return __int_as_float((e + 127) << 23); }
@@ -204,22 +211,50 @@ __device__ __forceinline__ void hist_put(int *bins, float *part, int c, int l, i
     }
 }
 
-// Adds the tile's samples (8 channel values g each, zero where inactive) to the
-// bins and tracks this thread's maxima for the next group's scales.
+// x * s rounded to the nearest integer (ties to even), for |x s| < 2^22: one
+// fused multiply-add onto 1.5 * 2^23, where the float spacing is 1, rounds the
+// exact product once; the integer is then the low bits of the sum.  Same
+// result as __float2int_rn(x * s) for a power-of-two s, without the
+// conversion unit.
+__device__ __forceinline__ int round_scaled(float x, float s) {
+    return __float_as_int(fmaf(x, s, 12582912.0f)) - 0x4B400000;
+}
+
+// Adds the tile's samples (8 channel values g each, zero where inactive, and
+// du = sum_l g_l alpha_l) to the bins and tracks this thread's maxima for the
+// next group's scales.  A sample whose largest |g| and |g u| fit the group's
+// scales and whose du is finite (so no g is NaN or infinite) takes the fast
+// path: every value fits, so the per-value range test is skipped.  The scales
+// are powers of two, so g * (u s1) equals (g u) s1 exactly.
 template <int PP>
 __device__ __forceinline__ void hist_add(int *bins, float *part, HistAcc &h, const int (&j)[PP],
-                                         const float (&u)[PP], const float (&g)[PP][8]) {
+                                         const float (&u)[PP], const float (&g)[PP][8], const float (&du)[PP]) {
     const float s0 = pow2f(h.e0), s1 = pow2f(h.e1);
+    constexpr float kQ = (float)(1 << kHistQBits);
 #pragma unroll
-    for (int q = 0; q < PP; ++q)
+    for (int q = 0; q < PP; ++q) {
+        float mg = 0.0f;
 #pragma unroll
-        for (int l = 0; l < 8; ++l) {
-            const float gu = g[q][l] * u[q];
-            hist_put(bins, part, 0, l, j[q], g[q][l], s0);
-            hist_put(bins, part, 1, l, j[q], gu, s1);
-            h.m0 = finite_max(h.m0, g[q][l]);
-            h.m1 = finite_max(h.m1, gu);
+        for (int l = 0; l < 8; ++l) mg = fmaxf(mg, fabsf(g[q][l]));
+        const float mgu = mg * fabsf(u[q]);
+        h.m0 = finite_max(h.m0, mg);
+        h.m1 = finite_max(h.m1, mgu);
+        if (mg * s0 < kQ && mgu * s1 < kQ && du[q] - du[q] == 0.0f) {
+            const float us1 = u[q] * s1;
+#pragma unroll
+            for (int l = 0; l < 8; ++l)
+                if (g[q][l] != 0.0f) {
+                    atomicAdd(bins + hist_at(0, l, j[q]), round_scaled(g[q][l], s0));
+                    atomicAdd(bins + hist_at(1, l, j[q]), round_scaled(g[q][l], us1));
+                }
+        } else {
+#pragma unroll
+            for (int l = 0; l < 8; ++l) {
+                hist_put(bins, part, 0, l, j[q], g[q][l], s0);
+                hist_put(bins, part, 1, l, j[q], g[q][l] * u[q], s1);
+            }
         }
+    }
 }
 
 // Closes the group: after a worker barrier (every atomic done), adds the bins,

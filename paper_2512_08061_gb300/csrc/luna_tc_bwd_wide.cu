@@ -403,8 +403,8 @@ __global__ void __launch_bounds__(kBThreads, 1)
                     tc_fence_before();
                     mbar_arrive(gready);
                     if (hon) {
-                        hist_add<C::PP>(bins, hpart, hacc, j, u, gv);
-                        if (++hacc.tiles == kHistTiles) hist_close(bins, hpart, a.lay.nint, hacc, tid, true, smax, warp, lane);
+                        hist_add<C::PP>(bins, hpart, hacc, j, u, gv, dU);
+                        if (++hacc.tiles == hist_tiles<C::MP>()) hist_close(bins, hpart, a.lay.nint, hacc, tid, true, smax, warp, lane);
                     }
                     // dQ
                     wait_or_fail(dqready, g & 1, failed, status);
@@ -810,8 +810,8 @@ __global__ void __launch_bounds__(kBThreads, 1)
                     tc_fence_before();
                     mbar_arrive(gready);
                     if (hon) {
-                        hist_add<C::PP>(bins, hpart, hacc, j, u, gv);
-                        if (++hacc.tiles == kHistTiles) hist_close(bins, hpart, a.lay.nint, hacc, tid, true, smax, warp, lane);
+                        hist_add<C::PP>(bins, hpart, hacc, j, u, gv, dU);
+                        if (++hacc.tiles == hist_tiles<C::MP>()) hist_close(bins, hpart, a.lay.nint, hacc, tid, true, smax, warp, lane);
                     }
                     // dV = hi + lo
                     wait_or_fail(dvready, g & 1, failed, status);

@@ -30,6 +30,7 @@ struct P128 {
                                      2 * (kBWorkers / 32) * 4 + kBarBytes + 1024;
     static_assert(SMEM <= kSmemLimit, "shared memory budget");
     static_assert(PP == 4, "four projections per thread");
+    static_assert(hist_tiles<MP>() == 2, "two 2048-sample tiles per histogram group");
 };
 
 // [W_hi; W_hi; W_lo; 0] (16 rows each) as the K-major B operand of dX = G W: row n = output column.
@@ -191,6 +192,16 @@ __global__ void __launch_bounds__(kBThreads, 1)
                 const int row0 = ir.r0 + t * 128;
                 const bool valid = r < min(128, ir.r1 - row0);
                 const float *dp = dphi + ((size_t)ir.bh * a.n + row0 + r) * C::D + H * C::PP * 8;
+                // this thread's 32 dphi values, requested before the waits and the search
+                float4 pv[C::PP][2];
+#pragma unroll
+                for (int q = 0; q < C::PP; ++q) {
+                    pv[q][0] = pv[q][1] = make_float4(0.f, 0.f, 0.f, 0.f);
+                    if (valid) {
+                        pv[q][0] = __ldcg(reinterpret_cast<const float4 *>(dp + 8 * q));
+                        pv[q][1] = __ldcg(reinterpret_cast<const float4 *>(dp + 8 * q + 4));
+                    }
+                }
                 wait_or_fail(uready + (g & 1), (g >> 1) & 1, failed, status);
                 tc_fence_after();
                 float u[C::PP];
@@ -215,8 +226,7 @@ __global__ void __launch_bounds__(kBThreads, 1)
                     for (int q = 0; q < C::PP; ++q) {
                         float al[8], y[8];
                         channel_eval(sAB, j[q], u[q], al, y);
-                        float4 p0 = make_float4(0.f, 0.f, 0.f, 0.f), p1 = p0;
-                        if (valid) { p0 = __ldcg(reinterpret_cast<const float4 *>(dp + 8 * q)); p1 = __ldcg(reinterpret_cast<const float4 *>(dp + 8 * q + 4)); }
+                        const float4 p0 = pv[q][0], p1 = pv[q][1];
                         const float dv[8] = {p0.x, p0.y, p0.z, p0.w, p1.x, p1.y, p1.z, p1.w};
 #pragma unroll
                         for (int l = 0; l < 8; ++l) {
@@ -232,8 +242,7 @@ __global__ void __launch_bounds__(kBThreads, 1)
                 for (int q = 0; q < C::PP; ++q) {
                     float al[8], y[8];
                     channel_eval(sAB, j[q], u[q], al, y);
-                    float4 p0 = make_float4(0.f, 0.f, 0.f, 0.f), p1 = p0;
-                    if (valid) { p0 = __ldcg(reinterpret_cast<const float4 *>(dp + 8 * q)); p1 = __ldcg(reinterpret_cast<const float4 *>(dp + 8 * q + 4)); }
+                    const float4 p0 = pv[q][0], p1 = pv[q][1];
                     const float dv[8] = {p0.x, p0.y, p0.z, p0.w, p1.x, p1.y, p1.z, p1.w};
                     float du = 0.0f;
 #pragma unroll
@@ -260,8 +269,8 @@ __global__ void __launch_bounds__(kBThreads, 1)
                 tc_fence_before();
                 mbar_arrive(gready);
                 if (hon) {
-                    hist_add<C::PP>(bins, hpart, hacc, j, u, gv);
-                    if (++hacc.tiles == kHistTiles) hist_close(bins, hpart, a.lay.nint, hacc, tid, true, smax, warp, lane);
+                    hist_add<C::PP>(bins, hpart, hacc, j, u, gv, dU);
+                    if (++hacc.tiles == hist_tiles<C::MP>()) hist_close(bins, hpart, a.lay.nint, hacc, tid, true, smax, warp, lane);
                 }
                 // dX
                 wait_or_fail(dxready, g & 1, failed, status);

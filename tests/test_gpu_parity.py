@@ -230,6 +230,28 @@ def test_backward_tensor_core_repeat_bitwise():
         assert np.array_equal(g1[k], g2[k]), k
 
 
+@pytest.mark.parametrize("d,M,causal", [(32, 8, False), (64, 8, False), (128, 16, True)])
+def test_backward_tensor_core_histogram_ranges(d, M, causal, monkeypatch):
+    """The fixed-point interval histogram of the channel-MLP gradient
+    statistics when the output gradient is zero on the first 300 rows of every
+    sequence (no scale until a later tile) and then grows by four orders of
+    magnitude along the sequence, so that every group of tiles outgrows the
+    scales taken from the group before it and its large values go to the
+    unscaled fallback.  One work item per head, so that a block walks many
+    groups."""
+    n = 1100
+    monkeypatch.setenv("LUNA_TC_TILES_PER_SPLIT", "9")
+    monkeypatch.setenv("LUNA_CAUSAL_SEG_ROWS", "1152")
+    case = Case(2, 2, n, d, M, 8, "bf16", causal, seed=83, qkv_scale=1.0 / math.sqrt(d), with_grad=True)
+    ramp = 10.0 ** (4.0 * np.arange(n) / n)
+    ramp[:300] = 0.0
+    case.inp["dO"] = synth.IOTensor(case.inp["dO"].value * ramp[None, None, :, None], "bf16")
+    lu = case.luna()
+    case.run_fwd(lu)
+    g = {k: to_host(v) for k, v in case.run_bwd(lu).items()}
+    _check_bwd(case, g, case.oracle_bwd(), TOL["bf16"])
+
+
 @pytest.mark.parametrize("seg_rows", ["128", "384", "1280"])
 def test_backward_tensor_core_causal(seg_rows, monkeypatch):
     """Streaming-form backward through the tensor-core kernels (d = 128, M = 16):
