@@ -123,22 +123,26 @@ __device__ __forceinline__ uint4 pack8(const float (&y)[8]) {
 // native and about five times faster.  So the bins hold fixed-point int32 sums
 // over groups of hist_tiles() tiles, quantised with power-of-two scales 2^e such
 // that |q| < 2^kHistQBits for the scale's reference maxima of |g| and |g*u|; a
-// group holds at most 4096 samples (four tiles of 128 rows x 8 projections,
-// two of 128 x 16), so a bin stays below 2^30.  The
+// group holds at most 16384 samples (16 tiles of 128 rows x 8 projections,
+// 8 of 128 x 16), so a bin stays below 2^30.  The
 // block's first group takes its reference maxima from a pre-pass over its
 // first tile with a nonzero g, every later group from the block-wide maxima of
 // the group before it.  A value that does not fit (it outgrew the reference,
 // or is not finite) goes, unscaled, to an fp32 atomic on the block's partial in
 // global memory instead.  At the end of a group the bins are added, rescaled,
-// into that partial and cleared.  The quantisation step is 2^-18 of the
-// reference maximum.
+// into that partial and cleared.  The quantisation step is 2^-16 of the
+// reference maximum; a sample's rounding error is at most half of it, and
+// the errors of a bin's samples are independent, so a sum of N samples is off
+// by about 2^-17 sqrt(N / 3) reference maxima (far below the bf16 rounding of
+// the kernels' operands).  Large groups keep the block-wide flushes (a worker
+// barrier and a pass over every bin) rare.
 //
 // Layout in shared memory: bins[(c * 8 + l) * kNint + j] (lanes with different
 // intervals fall into different banks); the partial is [interval][channel][g, g*u].
 __device__ __forceinline__ int hist_at(int c, int l, int j) { return (c * 8 + l) * kNint + j; }
 
-constexpr int kHistQBits = 18;  // |q| < 2^18 per sample
-constexpr int kHistSamples = 4096;  // samples per group: 4096 * 2^18 = 2^30
+constexpr int kHistQBits = 16;      // |q| < 2^16 per sample
+constexpr int kHistSamples = 16384;  // samples per group: 16384 * 2^16 = 2^30
 // Tiles per group for 128-row tiles of MP projections each.
 template <int MP>
 __host__ __device__ constexpr int hist_tiles() {

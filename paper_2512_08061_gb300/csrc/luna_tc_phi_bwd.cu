@@ -30,7 +30,7 @@ struct P128 {
                                      2 * (kBWorkers / 32) * 4 + kBarBytes + 1024;
     static_assert(SMEM <= kSmemLimit, "shared memory budget");
     static_assert(PP == 4, "four projections per thread");
-    static_assert(hist_tiles<MP>() == 2, "two 2048-sample tiles per histogram group");
+    static_assert(hist_tiles<MP>() == 8, "eight 2048-sample tiles per histogram group");
 };
 
 // [W_hi; W_hi; W_lo; 0] (16 rows each) as the K-major B operand of dX = G W: row n = output column.
@@ -47,6 +47,13 @@ __device__ void stage_wx64(const AttnArgs &a, uint8_t *dst) {
         }
         *reinterpret_cast<__nv_bfloat16 *>(dst + sw128_chunk(n, k / 8) + (k % 8) * 2) = __float2bfloat16_rn(v);
     }
+}
+
+// 32 bytes from global memory (32-byte aligned), cached in L2 only.
+__device__ __forceinline__ void ld_cg_v8(const float *p, float4 &a, float4 &b) {
+    asm volatile("ld.global.cg.v8.f32 {%0, %1, %2, %3, %4, %5, %6, %7}, [%8];"
+                 : "=f"(a.x), "=f"(a.y), "=f"(a.z), "=f"(a.w), "=f"(b.x), "=f"(b.y), "=f"(b.z), "=f"(b.w)
+                 : "l"(p));
 }
 
 template <class C>
@@ -192,15 +199,13 @@ __global__ void __launch_bounds__(kBThreads, 1)
                 const int row0 = ir.r0 + t * 128;
                 const bool valid = r < min(128, ir.r1 - row0);
                 const float *dp = dphi + ((size_t)ir.bh * a.n + row0 + r) * C::D + H * C::PP * 8;
-                // this thread's 32 dphi values, requested before the waits and the search
+                // this thread's 32 dphi values, requested before the waits and the search: one 32-byte
+                // load per projection (a whole sector; dphi rows are 512 bytes, 32-byte aligned)
                 float4 pv[C::PP][2];
 #pragma unroll
                 for (int q = 0; q < C::PP; ++q) {
                     pv[q][0] = pv[q][1] = make_float4(0.f, 0.f, 0.f, 0.f);
-                    if (valid) {
-                        pv[q][0] = __ldcg(reinterpret_cast<const float4 *>(dp + 8 * q));
-                        pv[q][1] = __ldcg(reinterpret_cast<const float4 *>(dp + 8 * q + 4));
-                    }
+                    if (valid) ld_cg_v8(dp + 8 * q, pv[q][0], pv[q][1]);
                 }
                 wait_or_fail(uready + (g & 1), (g >> 1) & 1, failed, status);
                 tc_fence_after();

@@ -237,11 +237,12 @@ def test_backward_tensor_core_histogram_ranges(d, M, causal, monkeypatch):
     sequence (no scale until a later tile) and then grows by four orders of
     magnitude along the sequence, so that every group of tiles outgrows the
     scales taken from the group before it and its large values go to the
-    unscaled fallback.  One work item per head, so that a block walks many
-    groups."""
-    n = 1100
-    monkeypatch.setenv("LUNA_TC_TILES_PER_SPLIT", "9")
-    monkeypatch.setenv("LUNA_CAUSAL_SEG_ROWS", "1152")
+    unscaled fallback.  One work item per head (18 tiles of 128 rows), so that
+    a block walks more than one group (16 tiles of 128 rows x 8 projections,
+    8 tiles of 128 x 16)."""
+    n = 2200
+    monkeypatch.setenv("LUNA_TC_TILES_PER_SPLIT", "18")
+    monkeypatch.setenv("LUNA_CAUSAL_SEG_ROWS", "2304")
     case = Case(2, 2, n, d, M, 8, "bf16", causal, seed=83, qkv_scale=1.0 / math.sqrt(d), with_grad=True)
     ramp = 10.0 ** (4.0 * np.arange(n) / n)
     ramp[:300] = 0.0
