@@ -443,13 +443,11 @@ __global__ void __launch_bounds__(kCBThreads, 1)
                     *reinterpret_cast<uint4 *>(Kb + boff + sw128_chunk(r, m0 % 8 + 1)) = kh1;
                     *reinterpret_cast<uint4 *>(Pk + boff + sw128_chunk(r, m0 % 8)) = kl0;
                     *reinterpret_cast<uint4 *>(Pk + boff + sw128_chunk(r, m0 % 8 + 1)) = kl1;
-                    if (valid) {
+                    if (valid) {  // workspace rows (32-byte aligned): [hi | lo] of the D features
                         uint4 *dst = reinterpret_cast<uint4 *>(static_cast<__nv_bfloat16 *>(a.phik) +
                                                                (hrow + row0 + r) * 2 * C::D + 16 * part);
-                        dst[0] = kh0;
-                        dst[1] = kh1;
-                        dst[C::D / 8] = kl0;
-                        dst[C::D / 8 + 1] = kl1;
+                        st_v8(dst, kh0, kh1);
+                        st_v8(dst + C::D / 8, kl0, kl1);
                     }
                 }
                 if (!valid && part == 0) {  // padded keys: clear V so that no garbage enters S
@@ -528,10 +526,12 @@ __global__ void __launch_bounds__(kCBThreads, 1)
                         dq[k] = live ? (pv[k] + zi[k] * ndot) * inv : 0.0f;
                         pt[k] = phq[k] * inv;
                     }
-                    if (valid) {
+                    if (valid) {  // workspace rows, 32-byte aligned
                         float4 *dst = reinterpret_cast<float4 *>(a.dphi + (hrow + row0 + r) * C::D + 16 * part);
 #pragma unroll
-                        for (int k = 0; k < 4; ++k) dst[k] = make_float4(dq[4 * k], dq[4 * k + 1], dq[4 * k + 2], dq[4 * k + 3]);
+                        for (int k = 0; k < 2; ++k)
+                            st_v8(dst + 2 * k, f4_bits(make_float4(dq[8 * k], dq[8 * k + 1], dq[8 * k + 2], dq[8 * k + 3])),
+                                  f4_bits(make_float4(dq[8 * k + 4], dq[8 * k + 5], dq[8 * k + 6], dq[8 * k + 7])));
                         uint4 h0, l0, h1, l1;
                         const float p0[8] = {pt[0], pt[1], pt[2], pt[3], pt[4], pt[5], pt[6], pt[7]};
                         const float p1[8] = {pt[8], pt[9], pt[10], pt[11], pt[12], pt[13], pt[14], pt[15]};
@@ -539,8 +539,8 @@ __global__ void __launch_bounds__(kCBThreads, 1)
                         split8(p1, h1, l1);
                         uint4 *pq = reinterpret_cast<uint4 *>(static_cast<__nv_bfloat16 *>(a.pq2) +
                                                               (hrow + row0 + r) * 2 * C::D + 16 * part);
-                        pq[0] = h0; pq[1] = h1;
-                        pq[C::D / 8] = l0; pq[C::D / 8 + 1] = l1;
+                        st_v8(pq, h0, h1);
+                        st_v8(pq + C::D / 8, l0, l1);
                         if (part == 0)
                             *reinterpret_cast<float2 *>(a.rowstat + 2 * (hrow + row0 + r)) =
                                 make_float2(live ? den : 1.0f, live ? ndot : 0.0f);
@@ -1050,13 +1050,15 @@ __global__ void __launch_bounds__(kCBThreads, 1)
                     half_cols<16>(x, df, lane);
                     tc_fence_before();
                     mbar_arrive(accfree);
-                    if (valid) {
+                    if (valid) {  // workspace rows, 32-byte aligned
                         float4 *fp = reinterpret_cast<float4 *>(a.dphi + (hrow + row0 + r) * C::D + 16 * part);
+                        float o[16];
 #pragma unroll
-                        for (int k = 0; k < 4; ++k)
-                            fp[k] = make_float4(df[4 * k] + sdz[16 * part + 4 * k], df[4 * k + 1] + sdz[16 * part + 4 * k + 1],
-                                                df[4 * k + 2] + sdz[16 * part + 4 * k + 2],
-                                                df[4 * k + 3] + sdz[16 * part + 4 * k + 3]);
+                        for (int k = 0; k < 16; ++k) o[k] = df[k] + sdz[16 * part + k];
+#pragma unroll
+                        for (int k = 0; k < 2; ++k)
+                            st_v8(fp + 2 * k, f4_bits(make_float4(o[8 * k], o[8 * k + 1], o[8 * k + 2], o[8 * k + 3])),
+                                  f4_bits(make_float4(o[8 * k + 4], o[8 * k + 5], o[8 * k + 6], o[8 * k + 7])));
                     }
                 }
                 named_sync<kCBWorkers>(1);  // every sdz read before it changes

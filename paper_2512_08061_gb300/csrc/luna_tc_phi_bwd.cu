@@ -49,13 +49,6 @@ __device__ void stage_wx64(const AttnArgs &a, uint8_t *dst) {
     }
 }
 
-// 32 bytes from global memory (32-byte aligned), cached in L2 only.
-__device__ __forceinline__ void ld_cg_v8(const float *p, float4 &a, float4 &b) {
-    asm volatile("ld.global.cg.v8.f32 {%0, %1, %2, %3, %4, %5, %6, %7}, [%8];"
-                 : "=f"(a.x), "=f"(a.y), "=f"(a.z), "=f"(a.w), "=f"(b.x), "=f"(b.y), "=f"(b.z), "=f"(b.w)
-                 : "l"(p));
-}
-
 template <class C>
 __global__ void __launch_bounds__(kBThreads, 1)
     k_tc_phi_bwd(const __grid_constant__ CUtensorMap mapX, AttnArgs a, const float *dphi, __nv_bfloat16 *dXg,
