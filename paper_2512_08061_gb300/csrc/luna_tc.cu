@@ -600,6 +600,7 @@ __global__ void __launch_bounds__(kThreadsTC, 1)
                 tc_fence_after();
                 // this thread writes output columns [Q*HC, (Q+1)*HC) of row r
                 constexpr int HC = C::DV / 4;
+                const float inv = dsum != 0.0f ? 1.0f / dsum : 0.0f;  // one division per row
                 uint4 outv[HC / 8];
                 const uint32_t col = lrow + tmem_num + q * 2 * C::DV + Q * HC;
                 if constexpr (HC == 8) {
@@ -609,8 +610,7 @@ __global__ void __launch_bounds__(kThreadsTC, 1)
                     tmem_wait_ld();
                     float o[8];
 #pragma unroll
-                    for (int c = 0; c < 8; ++c)
-                        o[c] = (dsum != 0.0f) ? (__uint_as_float(xh[c]) + __uint_as_float(xl[c])) / dsum : 0.0f;
+                    for (int c = 0; c < 8; ++c) o[c] = (__uint_as_float(xh[c]) + __uint_as_float(xl[c])) * inv;
                     outv[0] = make_uint4(pack_bf16x2(o[0], o[1]), pack_bf16x2(o[2], o[3]), pack_bf16x2(o[4], o[5]),
                                          pack_bf16x2(o[6], o[7]));
                 } else {
@@ -622,8 +622,7 @@ __global__ void __launch_bounds__(kThreadsTC, 1)
                         tmem_wait_ld();
                         float o[16];
 #pragma unroll
-                        for (int c = 0; c < 16; ++c)
-                            o[c] = (dsum != 0.0f) ? (__uint_as_float(xh[c]) + __uint_as_float(xl[c])) / dsum : 0.0f;
+                        for (int c = 0; c < 16; ++c) o[c] = (__uint_as_float(xh[c]) + __uint_as_float(xl[c])) * inv;
 #pragma unroll
                         for (int c = 0; c < 16; c += 8)
                             outv[(c0 + c) / 8] =

@@ -14,6 +14,10 @@
 //        work  A masked to keys j <= i, its row sums, A as bf16
 //        MMA   num += A V,  S += phi(K)^T V,  z += phi(K)^T 1
 //        work  O = num / (phi(q).z + rowsum(A) + eps);  S -> bf16 operand of the next tile
+//      The MMA warp issues the next tile's U_q (into a second TMEM slot) right
+//      after num and A, so that the X buffer takes the next K tile while the
+//      workers mask the scores, and the next U_k after the O products, while
+//      the workers write O.
 //      S, phi and the scores enter the products as one bf16 rounding (the
 //      forward output is bf16; the backward pass recomputes its own state from
 //      the exact segment prefixes of step 2).  The normaliser uses the same
@@ -48,38 +52,48 @@ struct K128 {
     static_assert(PT == 2 * TILE && XT == 2 * TILE && VT == 2 * TILE && ST == 2 * TILE, "two 64-column blocks");
 };
 
-// TMEM columns: U (q: 0..31, k: 32..63) | num | A | S | z
-constexpr uint32_t cU = 0, cN = 64, cA = 192, cS = 320, cZ = 448;
+// TMEM columns: U (q of even tiles: 0..31, k: 32..63) | num | A | S | z | q of odd tiles
+constexpr uint32_t cU = 0, cN = 64, cA = 192, cS = 320, cZ = 448, cUq1 = 464;
+__host__ __device__ constexpr uint32_t col_uq(int g) { return (g & 1) ? cUq1 : cU; }
 
-// phi of projections Qd*PP .. Qd*PP+PP-1 of one row from the projection columns
-// (hi at u0, mid at u0 + MP): bf16 chunks into the phi tile (zeros if !valid);
-// returns the fp32 dot product of those features with sz (if sz is not null).
+// phi of projections Qd*PP .. Qd*PP+PP-1 of one row of the Q tile and of the
+// K tile, from their projection columns (hi at u, mid at u + MP): bf16 chunks
+// into the phi tiles (zeros if !valid).  The 2 * PP interval searches run
+// interleaved.  Returns the fp32 dot product of the bf16 phi(q) features with
+// sz, the normaliser part that the numerator's rounding matches.
 template <class C>
-__device__ __forceinline__ float phi_quarter(uint32_t u0, int Qd, const float *sTe, const float *sAB,
-                                             const float *sbias, bool valid, int r, uint8_t *tile, const float *sz) {
+__device__ __forceinline__ float phi_quarter_qk(uint32_t uq, uint32_t uk, int Qd, const float *sTe, const float *sAB,
+                                                const float *sbias, bool valid, int r, uint8_t *tq, uint8_t *tk,
+                                                const float *sz) {
     constexpr int PP = C::PP;
-    float u[PP];
+    static_assert(PP == 4, "four projections per thread");
+    float u[2 * PP];
     {
-        uint32_t xh[4], xm[4];
-        static_assert(PP == 4, "four projections per thread");
-        tmem_ld4(u0 + Qd * PP, xh);
-        tmem_ld4(u0 + C::MP + Qd * PP, xm);
+        uint32_t qh[4], qm[4], kh[4], km[4];
+        tmem_ld4(uq + Qd * PP, qh);
+        tmem_ld4(uq + C::MP + Qd * PP, qm);
+        tmem_ld4(uk + Qd * PP, kh);
+        tmem_ld4(uk + C::MP + Qd * PP, km);
         tmem_wait_ld();
 #pragma unroll
-        for (int q = 0; q < PP; ++q) u[q] = __uint_as_float(xh[q]) + __uint_as_float(xm[q]) + sbias[Qd * PP + q];
+        for (int q = 0; q < PP; ++q) {
+            const float b = sbias[Qd * PP + q];
+            u[q] = __uint_as_float(qh[q]) + __uint_as_float(qm[q]) + b;
+            u[PP + q] = __uint_as_float(kh[q]) + __uint_as_float(km[q]) + b;
+        }
     }
-    int node[PP];
+    int node[2 * PP];
 #pragma unroll
-    for (int q = 0; q < PP; ++q) node[q] = 1;
+    for (int q = 0; q < 2 * PP; ++q) node[q] = 1;
 #pragma unroll
     for (int lvl = 0; lvl < 10; ++lvl)
 #pragma unroll
-        for (int q = 0; q < PP; ++q) node[q] = 2 * node[q] + (sTe[node[q]] < u[q] ? 1 : 0);
+        for (int q = 0; q < 2 * PP; ++q) node[q] = 2 * node[q] + (sTe[node[q]] < u[q] ? 1 : 0);
     float dot = 0.0f;
     const float4 *ab = reinterpret_cast<const float4 *>(sAB);
 #pragma unroll
-    for (int q = 0; q < PP; ++q) {
-        const int i = Qd * PP + q, j = node[q] - kEytzinger;
+    for (int q = 0; q < 2 * PP; ++q) {
+        const int i = Qd * PP + (q % PP), j = node[q] - kEytzinger;
         uint4 w = make_uint4(0u, 0u, 0u, 0u);
         if (valid) {
             float y[8];
@@ -91,7 +105,7 @@ __device__ __forceinline__ float phi_quarter(uint32_t u0, int Qd, const float *s
             }
             w = make_uint4(pack_bf16x2(y[0], y[1]), pack_bf16x2(y[2], y[3]), pack_bf16x2(y[4], y[5]),
                            pack_bf16x2(y[6], y[7]));
-            if (sz) {  // with the bf16 phi that the numerator uses
+            if (q < PP) {  // with the bf16 phi that the numerator uses
                 const __nv_bfloat162 *yb = reinterpret_cast<const __nv_bfloat162 *>(&w);
 #pragma unroll
                 for (int k = 0; k < 4; ++k) {
@@ -100,7 +114,7 @@ __device__ __forceinline__ float phi_quarter(uint32_t u0, int Qd, const float *s
                 }
             }
         }
-        *reinterpret_cast<uint4 *>(tile + (i / 8) * C::TILE + sw128_chunk(r, i % 8)) = w;
+        *reinterpret_cast<uint4 *>((q < PP ? tq : tk) + (i / 8) * C::TILE + sw128_chunk(r, i % 8)) = w;
     }
     return dot;
 }
@@ -205,24 +219,23 @@ __global__ void __launch_bounds__(kCThreads, 1)
             const uint64_t dS = sdesc(smem_u32(Sop), C::TILE, 1024, kSwizzle128);   // MN-major (N = values)
             const uint64_t dO1 = sdesc(smem_u32(Ones), 16, 1024, kSwizzle128);      // K-major, 16 rows
             bool failed = false;
-            // projections of tile g: U_q from load 2g, U_k from load 2g+1
-            auto proj = [&](int g) {
+            // projections of tile g: U_q from load 2g (into the q slot of g's parity), U_k from load 2g+1
+            auto proj = [&](int g, int h) {
                 constexpr uint32_t idU = idesc_bf16(128, C::NU, false, false);
-                for (int h = 0; h < 2; ++h) {
-                    const int L = 2 * g + h;
-                    wait_or_fail(fullx, L & 1, failed, status);
-                    tc_fence_after();
+                const int L = 2 * g + h;
+                wait_or_fail(fullx, L & 1, failed, status);
+                tc_fence_after();
+                const uint32_t col = h == 0 ? col_uq(g) : cU + C::NU;
 #pragma unroll
-                    for (int kb = 0; kb < C::KBX; ++kb)
+                for (int kb = 0; kb < C::KBX; ++kb)
 #pragma unroll
-                        for (int k = 0; k < 4; ++k)
-                            mma_bf16_ss(tbase + cU + h * C::NU, dadd(dX, kb * C::TILE + 32 * k),
-                                        dadd(dW, kb * (C::NU * 128) + 32 * k), idU, (kb | k) != 0);
-                    mma_commit(xfree);
-                }
-                mma_commit(uready);
+                    for (int k = 0; k < 4; ++k)
+                        mma_bf16_ss(tbase + col, dadd(dX, kb * C::TILE + 32 * k), dadd(dW, kb * (C::NU * 128) + 32 * k),
+                                    idU, (kb | k) != 0);
+                mma_commit(xfree);
+                if (h == 1) mma_commit(uready);
             };
-            if (T > 0) proj(0);
+            if (T > 0) { proj(0, 0); proj(0, 1); }
             TileCursor cur;
             cur.start(a, it);
             int tile_in_item = 0, last_item = -1;
@@ -245,11 +258,9 @@ __global__ void __launch_bounds__(kCThreads, 1)
                     mma_bf16_ss(tbase + cA, dadd(dPqK, ka), dadd(dPkK, ka), idA, kk != 0);
                 }
                 mma_commit(aready);
-                // projections of the next tile (the workers have read U(g): they arrived on pready after ufree)
-                if (g + 1 < T) {
-                    wait_or_fail(ufree, g & 1, failed, status);
-                    proj(g + 1);
-                }
+                // U_q of the next tile into the other q slot (its Q tile was loaded once U_k(g) freed the X
+                // buffer), so that the load of its K tile starts now
+                if (g + 1 < T) proj(g + 1, 0);
                 wait_or_fail(a2ready, g & 1, failed, status);
                 wait_or_fail(fullv, g & 1, failed, status);
                 tc_fence_after();
@@ -270,6 +281,12 @@ __global__ void __launch_bounds__(kCThreads, 1)
                                 (tile_in_item > 0 || kk > 0) ? 1u : 0u);
                 mma_commit(oready);
                 mma_commit(vfree);
+                // U_k of the next tile (the workers have read U_k(g): they arrived on ufree in phase 1), while
+                // they write O and the state operand
+                if (g + 1 < T) {
+                    wait_or_fail(ufree, g & 1, failed, status);
+                    proj(g + 1, 1);
+                }
                 ++tile_in_item;
             }
         }
@@ -318,8 +335,8 @@ __global__ void __launch_bounds__(kCThreads, 1)
                 // phase 1: phi(Q), phi(K), phi(q).z
                 wait_or_fail(uready, g & 1, failed, status);
                 tc_fence_after();
-                const float dq = phi_quarter<C>(tbase + lrow + cU, Qd, sTe, sAB, sbias, valid, r, Pq, sz);
-                phi_quarter<C>(tbase + lrow + cU + C::NU, Qd, sTe, sAB, sbias, valid, r, Pk, nullptr);
+                const float dq = phi_quarter_qk<C>(tbase + lrow + col_uq(g), tbase + lrow + cU + C::NU, Qd, sTe, sAB,
+                                                   sbias, valid, r, Pq, Pk, sz);
                 tc_fence_before();
                 mbar_arrive(ufree);
                 if (!valid && Qd == 0) {  // padded key rows: clear V so that no garbage enters num or S
@@ -369,11 +386,12 @@ __global__ void __launch_bounds__(kCThreads, 1)
                     tmem_ld16(tbase + lrow + cN + 32 * Qd + 16, x1);
                     tmem_wait_ld();
                     if (valid) {
+                        const float inv = dsum != 0.0f ? 1.0f / dsum : 0.0f;  // one division per row
                         float o[32];
 #pragma unroll
                         for (int c = 0; c < 16; ++c) {
-                            o[c] = dsum != 0.0f ? __uint_as_float(x0[c]) / dsum : 0.0f;
-                            o[16 + c] = dsum != 0.0f ? __uint_as_float(x1[c]) / dsum : 0.0f;
+                            o[c] = __uint_as_float(x0[c]) * inv;
+                            o[16 + c] = __uint_as_float(x1[c]) * inv;
                         }
                         uint4 *dst = reinterpret_cast<uint4 *>(O + (size_t)(row0 + r) * C::DV + 32 * Qd);
 #pragma unroll
