@@ -252,6 +252,24 @@ __global__ void __launch_bounds__(kBThreads, 1)
 #pragma unroll
         for (int q = 0; q < C::PP; ++q) db_acc[q] = 0.0f;
         HistAcc hacc;
+        // dQ of tile g is read out during tile g + 1 (after its feature-map work, before its G tile), so
+        // that the dQ product runs while the workers start the next tile
+        int pend_g = -1, pend_row = -1;  // tile, and this thread's row of [B*H*n] in it (-1: padded; the
+                                         // rows of tensors that fit in device memory stay below 2^31)
+        auto dq_out = [&](int gp, int row) {
+            wait_or_fail(dqready, gp & 1, failed, status);
+            tc_fence_after();
+            uint32_t x[8];
+            tmem_ld8(tbase + lrow + cQ + H * 8, x);
+            tmem_wait_ld();
+            float f[8];
+#pragma unroll
+            for (int c = 0; c < 8; ++c) f[c] = __uint_as_float(x[c]);
+            tc_fence_before();
+            mbar_arrive(dqfree);
+            if (row >= 0)
+                *reinterpret_cast<uint4 *>(static_cast<__nv_bfloat16 *>(a.dQ) + (size_t)row * C::d + H * 8) = pack8(f);
+        };
         int g = 0, ne = 0;
         for (int i0 = it.begin; i0 < it.end;) {
             const int bh = i0 / it.nchunk;
@@ -267,7 +285,6 @@ __global__ void __launch_bounds__(kBThreads, 1)
                 named_sync<kBWorkers>(1);
                 mbar_arrive(opready);
             }
-            __nv_bfloat16 *dQ = static_cast<__nv_bfloat16 *>(a.dQ) + (size_t)bh * a.n * C::d;
             for (int item = i0; item < i1; ++item) {
                 const ItemRange ir = item_range(a, it, item);
                 for (int t = 0; t < ir.ntiles; ++t, ++g) {
@@ -392,6 +409,7 @@ __global__ void __launch_bounds__(kBThreads, 1)
                         dU[q] = du;
                         db_acc[q] += du;
                     }
+                    if (pend_g >= 0) dq_out(pend_g, pend_row);
                     // G = [dO (dv cols) | dU_hi | dU_lo | dU_hi | -(dO.O) hi, lo | 0] over the dO tile (in place)
                     {
                         if (!valid)  // padded rows may hold anything (even non-finite values): chunk H of dO
@@ -416,20 +434,8 @@ __global__ void __launch_bounds__(kBThreads, 1)
                         hist_add<C::PP>(bins, hpart, hacc, j, u, gv, dU);
                         if (++hacc.tiles == hist_tiles<C::MP>()) hist_close(bins, hpart, a.lay.nint, hacc, tid, true, smax, warp, lane);
                     }
-                    // dQ
-                    wait_or_fail(dqready, g & 1, failed, status);
-                    tc_fence_after();
-                    {
-                        uint32_t x[8];
-                        tmem_ld8(tbase + lrow + cQ + H * 8, x);
-                        tmem_wait_ld();
-                        float f[8];
-#pragma unroll
-                        for (int c = 0; c < 8; ++c) f[c] = __uint_as_float(x[c]);
-                        tc_fence_before();
-                        mbar_arrive(dqfree);
-                        if (valid) *reinterpret_cast<uint4 *>(dQ + (size_t)(row0 + r) * C::d + H * 8) = pack8(f);
-                    }
+                    pend_g = g;
+                    pend_row = valid ? bh * a.n + row0 + r : -1;
                 }
             }
             // run epilogue (warps 0..3 own all 128 TMEM lanes): dS, dz partial of this head.  Warp w holds
@@ -492,6 +498,7 @@ __global__ void __launch_bounds__(kBThreads, 1)
             if (run_tiles > 0) ++ne;
             i0 = i1;
         }
+        if (pend_g >= 0) dq_out(pend_g, pend_row);
         if (hacc.tiles > 0) hist_close(bins, hpart, a.lay.nint, hacc, tid, false, smax, warp, lane);
         // db: sum over the rows of each warp, then over warps
 #pragma unroll
