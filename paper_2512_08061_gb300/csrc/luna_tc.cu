@@ -557,13 +557,64 @@ __global__ void __launch_bounds__(kThreadsTC, 1)
         const int Q = warp >> 2, r = ((warp & 3) << 5) | lane;
         const uint32_t lrow = (uint32_t)((warp & 3) << 5) << 16;
         bool failed = false;
+        // O of tile g is written during tile g + 1 (after its feature map and normaliser barrier), so that
+        // the numerator product runs while the workers start the next tile
+        int pend_g = -1, pend_row = -1;  // tile, and this thread's row of [B*H*n] in it (-1: padded; the
+                                         // rows of tensors that fit in device memory stay below 2^31)
+        float pend_dsum = 0.0f;
+        auto o_out = [&](int gp, int row, float dsum) {
+            const int q = gp % NN;
+            wait_or_fail(numready + q, (gp / NN) & 1, failed, status);
+            tc_fence_after();
+            // this thread writes output columns [Q*HC, (Q+1)*HC) of the row
+            constexpr int HC = C::DV / 4;
+            const float inv = dsum != 0.0f ? 1.0f / dsum : 0.0f;  // one division per row
+            uint4 outv[HC / 8];
+            const uint32_t col = lrow + tmem_num + q * 2 * C::DV + Q * HC;
+            if constexpr (HC == 8) {
+                uint32_t xh[8], xl[8];
+                tmem_ld8(col, xh);
+                tmem_ld8(col + C::DV, xl);
+                tmem_wait_ld();
+                float o[8];
+#pragma unroll
+                for (int c = 0; c < 8; ++c) o[c] = (__uint_as_float(xh[c]) + __uint_as_float(xl[c])) * inv;
+                outv[0] = make_uint4(pack_bf16x2(o[0], o[1]), pack_bf16x2(o[2], o[3]), pack_bf16x2(o[4], o[5]),
+                                     pack_bf16x2(o[6], o[7]));
+            } else {
+#pragma unroll
+                for (int c0 = 0; c0 < HC; c0 += 16) {
+                    uint32_t xh[16], xl[16];
+                    tmem_ld16(col + c0, xh);
+                    tmem_ld16(col + c0 + C::DV, xl);
+                    tmem_wait_ld();
+                    float o[16];
+#pragma unroll
+                    for (int c = 0; c < 16; ++c) o[c] = (__uint_as_float(xh[c]) + __uint_as_float(xl[c])) * inv;
+#pragma unroll
+                    for (int c = 0; c < 16; c += 8)
+                        outv[(c0 + c) / 8] =
+                            make_uint4(pack_bf16x2(o[c], o[c + 1]), pack_bf16x2(o[c + 2], o[c + 3]),
+                                       pack_bf16x2(o[c + 4], o[c + 5]), pack_bf16x2(o[c + 6], o[c + 7]));
+                }
+            }
+            tc_fence_before();
+            mbar_arrive(numfree + q);
+            if (row >= 0) {
+                uint4 *dst = reinterpret_cast<uint4 *>(static_cast<__nv_bfloat16 *>(a.O) + (size_t)row * C::DV + Q * HC);
+#pragma unroll
+                for (int k = 0; k < HC / 8; ++k) dst[k] = outv[k];
+            }
+        };
         int g = 0, cur_bh = -1;
         for (int item = it.begin; item < it.end; ++item) {
             const ItemRange ir = item_range(a, it, item);
             if (ir.ntiles == 0) continue;
             if (ir.bh != cur_bh) {
-                // operand [S_hi; S_lo]^T and z of this head.  Safe to overwrite: every worker has passed
-                // the previous tile's normaliser barrier and seen its contraction complete.
+                // operand [S_hi; S_lo]^T and z of this head.  Safe to overwrite once the pending output is
+                // written (its contraction, the last to read the operand, is then complete) and every worker
+                // has passed the barrier below.
+                if (pend_g >= 0) { o_out(pend_g, pend_row, pend_dsum); pend_g = -1; }
                 named_sync<kWorkers>(1);
                 const float *Sg = a.S_fin + (size_t)ir.bh * C::D * C::DV;
                 for (int e = tid; e < 2 * C::DV * C::D; e += kWorkers) {
@@ -577,9 +628,8 @@ __global__ void __launch_bounds__(kThreadsTC, 1)
                 named_sync<kWorkers>(1);
                 cur_bh = ir.bh;
             }
-            __nv_bfloat16 *O = static_cast<__nv_bfloat16 *>(a.O) + (size_t)ir.bh * a.n * C::DV;
             for (int t = 0; t < ir.ntiles; ++t, ++g) {
-                const int p = g % NP, q = g % NN;
+                const int p = g % NP;
                 const int row0 = ir.r0 + t * 128;
                 const int nvalid = min(128, ir.r1 - row0);
                 wait_or_fail(uready + (g & 1), (g >> 1) & 1, failed, status);
@@ -595,50 +645,15 @@ __global__ void __launch_bounds__(kThreadsTC, 1)
                 tc_fence_before();
                 mbar_arrive(phiready + p);
                 named_sync<kWorkers>(1);  // all four parts of every row's normaliser are written
+                // read now: the slot is written again two tiles on, after the next tile's barrier
                 const float dsum = dslot[r] + dslot[128 + r] + dslot[256 + r] + dslot[384 + r] + a.eps;
-                wait_or_fail(numready + q, (g / NN) & 1, failed, status);
-                tc_fence_after();
-                // this thread writes output columns [Q*HC, (Q+1)*HC) of row r
-                constexpr int HC = C::DV / 4;
-                const float inv = dsum != 0.0f ? 1.0f / dsum : 0.0f;  // one division per row
-                uint4 outv[HC / 8];
-                const uint32_t col = lrow + tmem_num + q * 2 * C::DV + Q * HC;
-                if constexpr (HC == 8) {
-                    uint32_t xh[8], xl[8];
-                    tmem_ld8(col, xh);
-                    tmem_ld8(col + C::DV, xl);
-                    tmem_wait_ld();
-                    float o[8];
-#pragma unroll
-                    for (int c = 0; c < 8; ++c) o[c] = (__uint_as_float(xh[c]) + __uint_as_float(xl[c])) * inv;
-                    outv[0] = make_uint4(pack_bf16x2(o[0], o[1]), pack_bf16x2(o[2], o[3]), pack_bf16x2(o[4], o[5]),
-                                         pack_bf16x2(o[6], o[7]));
-                } else {
-#pragma unroll
-                    for (int c0 = 0; c0 < HC; c0 += 16) {
-                        uint32_t xh[16], xl[16];
-                        tmem_ld16(col + c0, xh);
-                        tmem_ld16(col + c0 + C::DV, xl);
-                        tmem_wait_ld();
-                        float o[16];
-#pragma unroll
-                        for (int c = 0; c < 16; ++c) o[c] = (__uint_as_float(xh[c]) + __uint_as_float(xl[c])) * inv;
-#pragma unroll
-                        for (int c = 0; c < 16; c += 8)
-                            outv[(c0 + c) / 8] =
-                                make_uint4(pack_bf16x2(o[c], o[c + 1]), pack_bf16x2(o[c + 2], o[c + 3]),
-                                           pack_bf16x2(o[c + 4], o[c + 5]), pack_bf16x2(o[c + 6], o[c + 7]));
-                    }
-                }
-                tc_fence_before();
-                mbar_arrive(numfree + q);
-                if (valid) {
-                    uint4 *dst = reinterpret_cast<uint4 *>(O + (size_t)(row0 + r) * C::DV + Q * HC);
-#pragma unroll
-                    for (int k = 0; k < HC / 8; ++k) dst[k] = outv[k];
-                }
+                if (pend_g >= 0) o_out(pend_g, pend_row, pend_dsum);
+                pend_g = g;
+                pend_row = valid ? ir.bh * a.n + row0 + r : -1;
+                pend_dsum = dsum;
             }
         }
+        if (pend_g >= 0) o_out(pend_g, pend_row, pend_dsum);
     }
     tc_fence_before();
     __syncthreads();
