@@ -84,26 +84,25 @@ struct Cfg {
 // residual phi - bf16(phi) into a second tile), zeros for rows that are not
 // valid.  Optionally adds phi into zacc (fp32 feature sums) and accumulates the
 // fp32 normaliser phi . z.
-template <class C, int Q>
-__device__ __forceinline__ void phi_row_quarter(uint32_t tmem_u_row, const float *sTe, const float *sAB,
+template <class C>
+__device__ __forceinline__ void phi_row_quarter(int Q, uint32_t tmem_u_row, const float *sTe, const float *sAB,
                                                 const float *sbias, bool valid, int r, uint8_t *phi, uint8_t *plo,
                                                 float *zacc, const float *sz, float &den) {
     constexpr int PP = C::PP;
     float u[PP];
     {
-        uint32_t x[16];
-        tmem_ld16(tmem_u_row, x);
-        if constexpr (C::MP == 8) {
-            tmem_wait_ld();
-#pragma unroll
-            for (int q = 0; q < PP; ++q) u[q] = __uint_as_float(x[Q * PP + q]) + __uint_as_float(x[8 + Q * PP + q]);
+        // this thread's PP projections: hi parts at columns Q*PP.., lo parts MP columns further
+        uint32_t xh[PP], xl[PP];
+        if constexpr (PP == 2) {
+            tmem_ld2(tmem_u_row + Q * PP, xh);
+            tmem_ld2(tmem_u_row + C::MP + Q * PP, xl);
         } else {
-            uint32_t y[16];
-            tmem_ld16(tmem_u_row + 16, y);
-            tmem_wait_ld();
-#pragma unroll
-            for (int q = 0; q < PP; ++q) u[q] = __uint_as_float(x[Q * PP + q]) + __uint_as_float(y[Q * PP + q]);
+            tmem_ld4(tmem_u_row + Q * PP, xh);
+            tmem_ld4(tmem_u_row + C::MP + Q * PP, xl);
         }
+        tmem_wait_ld();
+#pragma unroll
+        for (int q = 0; q < PP; ++q) u[q] = __uint_as_float(xh[q]) + __uint_as_float(xl[q]);
     }
     int node[PP];
 #pragma unroll
@@ -150,18 +149,6 @@ __device__ __forceinline__ void phi_row_quarter(uint32_t tmem_u_row, const float
         const uint32_t off = (i / 8) * 16384 + sw128_chunk(r, i % 8);
         *reinterpret_cast<uint4 *>(phi + off) = ph;
         if (plo) *reinterpret_cast<uint4 *>(plo + off) = pl;
-    }
-}
-
-template <class C>
-__device__ __forceinline__ void phi_row_any(int Q, uint32_t tmem_u_row, const float *sTe, const float *sAB,
-                                            const float *sbias, bool valid, int r, uint8_t *phi, uint8_t *plo,
-                                            float *zacc, const float *sz, float &den) {
-    switch (Q) {
-        case 0: phi_row_quarter<C, 0>(tmem_u_row, sTe, sAB, sbias, valid, r, phi, plo, zacc, sz, den); break;
-        case 1: phi_row_quarter<C, 1>(tmem_u_row, sTe, sAB, sbias, valid, r, phi, plo, zacc, sz, den); break;
-        case 2: phi_row_quarter<C, 2>(tmem_u_row, sTe, sAB, sbias, valid, r, phi, plo, zacc, sz, den); break;
-        default: phi_row_quarter<C, 3>(tmem_u_row, sTe, sAB, sbias, valid, r, phi, plo, zacc, sz, den); break;
     }
 }
 
@@ -339,7 +326,7 @@ __global__ void __launch_bounds__(kThreadsTC, 1)
                     tc_fence_after();
                     uint8_t *ph = Pb + p * 2 * C::PT, *pl = ph + C::PT;
                     const bool valid = r < nvalid;
-                    phi_row_any<C>(Q, tbase + lrow + (g & 1) * C::NU, sTe, sAB, sbias, valid, r, ph, pl, zacc,
+                    phi_row_quarter<C>(Q, tbase + lrow + (g & 1) * C::NU, sTe, sAB, sbias, valid, r, ph, pl, zacc,
                                    nullptr, dummy);
                     if (!valid && Q == 0) {  // padded rows: clear V so that no garbage enters S
                         wait_or_fail(fullv + v, (g / NV) & 1, failed, status);
@@ -637,7 +624,7 @@ __global__ void __launch_bounds__(kThreadsTC, 1)
                 tc_fence_after();
                 const bool valid = r < nvalid;
                 float den = 0.0f;
-                phi_row_any<C>(Q, tbase + lrow + (g & 1) * C::NU, sTe, sAB, sbias, valid, r, Pb + p * C::PT, nullptr,
+                phi_row_quarter<C>(Q, tbase + lrow + (g & 1) * C::NU, sTe, sAB, sbias, valid, r, Pb + p * C::PT, nullptr,
                                nullptr, sz, den);
                 float *dslot = sden + (g & 1) * 512;
                 dslot[Q * 128 + r] = den;
