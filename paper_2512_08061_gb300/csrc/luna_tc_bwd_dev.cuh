@@ -215,6 +215,21 @@ __device__ __forceinline__ void hist_put(int *bins, float *part, int c, int l, i
     }
 }
 
+// The per-value path of hist_add for a sample some of whose values outgrew the
+// group's scales (or are not finite): rare, so it stays out of line and the
+// common path keeps the kernels' loops small in the instruction cache.  The
+// values come by value (an array argument would move the caller's array to
+// local memory).
+__device__ __noinline__ void hist_add_slow(int *bins, float *part, int j, float u, float s0, float s1, float g0,
+                                           float g1, float g2, float g3, float g4, float g5, float g6, float g7) {
+    const float g[8] = {g0, g1, g2, g3, g4, g5, g6, g7};
+#pragma unroll
+    for (int l = 0; l < 8; ++l) {
+        hist_put(bins, part, 0, l, j, g[l], s0);
+        hist_put(bins, part, 1, l, j, g[l] * u, s1);
+    }
+}
+
 // x * s rounded to the nearest integer (ties to even), for |x s| < 2^22: one
 // fused multiply-add onto 1.5 * 2^23, where the float spacing is 1, rounds the
 // exact product once; the integer is then the low bits of the sum.  Same
@@ -252,11 +267,8 @@ __device__ __forceinline__ void hist_add(int *bins, float *part, HistAcc &h, con
                     atomicAdd(bins + hist_at(1, l, j[q]), round_scaled(g[q][l], us1));
                 }
         } else {
-#pragma unroll
-            for (int l = 0; l < 8; ++l) {
-                hist_put(bins, part, 0, l, j[q], g[q][l], s0);
-                hist_put(bins, part, 1, l, j[q], g[q][l] * u[q], s1);
-            }
+            hist_add_slow(bins, part, j[q], u[q], s0, s1, g[q][0], g[q][1], g[q][2], g[q][3], g[q][4], g[q][5],
+                          g[q][6], g[q][7]);
         }
     }
 }

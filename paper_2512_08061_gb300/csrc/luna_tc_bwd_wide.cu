@@ -342,29 +342,6 @@ __global__ void __launch_bounds__(kBThreads, 1)
                     const float ndot = live ? -dotn * inv : 0.0f;  // -(dO.O)
                     const float dden = ndot * inv;
                     bool hon = hacc.open;
-                    if (!hon) {  // first tile with a nonzero g in the block: a pre-pass fixes the histogram scales
-                        float m0 = 0.0f, m1 = 0.0f;
-#pragma unroll
-                        for (int q = 0; q < C::PP; ++q) {
-                            const int i = H * C::PP + q;
-                            float al[8], y[8];
-                            channel_eval(sAB, j[q], u[q], al, y);
-                            uint32_t ph[8], pl[8];
-                            tmem_ld8(tbase + lrow + cP + 8 * i, ph);
-                            tmem_ld8(tbase + lrow + cP + C::D + 8 * i, pl);
-                            tmem_wait_ld();
-#pragma unroll
-                            for (int l = 0; l < 8; ++l) {
-                                const float dphi = live ? (__uint_as_float(ph[l]) + __uint_as_float(pl[l])) * inv +
-                                                              sz[8 * i + l] * dden
-                                                        : 0.0f;
-                                const float gl = y[l] > 0.0f ? dphi : 0.0f;
-                                m0 = finite_max(m0, gl);
-                                m1 = finite_max(m1, gl * u[q]);
-                            }
-                        }
-                        hon = hist_open(hacc, m0, m1, smax, warp, lane);
-                    }
                     // gradients through the feature map; phi/den (bf16 hi, lo) for the dS / dz contractions
                     float dU[C::PP], gv[C::PP][8];
 #pragma unroll
@@ -423,6 +400,17 @@ __global__ void __launch_bounds__(kBThreads, 1)
                     fence_proxy_async_smem();
                     tc_fence_before();
                     mbar_arrive(gready);
+                    if (!hon) {  // first tile with a nonzero g in the block: its maxima give the first scales
+                        float m0 = 0.0f, m1 = 0.0f;
+#pragma unroll
+                        for (int q = 0; q < C::PP; ++q)
+#pragma unroll
+                            for (int l = 0; l < 8; ++l) {
+                                m0 = finite_max(m0, gv[q][l]);
+                                m1 = finite_max(m1, gv[q][l] * u[q]);
+                            }
+                        hon = hist_open(hacc, m0, m1, smax, warp, lane);
+                    }
                     if (hon) {
                         hist_add<C::PP>(bins, hpart, hacc, j, u, gv, dU);
                         if (++hacc.tiles == hist_tiles<C::MP>()) hist_close(bins, hpart, a.lay.nint, hacc, tid, true, smax, warp, lane);
@@ -762,27 +750,6 @@ __global__ void __launch_bounds__(kBThreads, 1)
                     wait_or_fail(fready, g & 1, failed, status);
                     tc_fence_after();
                     bool hon = hacc.open;
-                    if (!hon) {
-                        float m0 = 0.0f, m1 = 0.0f;
-#pragma unroll
-                        for (int q = 0; q < C::PP; ++q) {
-                            const int i = H * C::PP + q;
-                            float al[8], y[8];
-                            channel_eval(sAB, j[q], u[q], al, y);
-                            uint32_t ph[8], pl[8];
-                            tmem_ld8(tbase + lrow + cF + 8 * i, ph);
-                            tmem_ld8(tbase + lrow + cF + C::D + 8 * i, pl);
-                            tmem_wait_ld();
-#pragma unroll
-                            for (int l = 0; l < 8; ++l) {
-                                const float dphi = __uint_as_float(ph[l]) + __uint_as_float(pl[l]) + sdz[8 * i + l];
-                                const float gl = (valid && y[l] > 0.0f) ? dphi : 0.0f;
-                                m0 = finite_max(m0, gl);
-                                m1 = finite_max(m1, gl * u[q]);
-                            }
-                        }
-                        hon = hist_open(hacc, m0, m1, smax, warp, lane);
-                    }
                     float dU[C::PP], gv[C::PP][8];
 #pragma unroll
                     for (int q = 0; q < C::PP; ++q) {
@@ -815,6 +782,17 @@ __global__ void __launch_bounds__(kBThreads, 1)
                     fence_proxy_async_smem();
                     tc_fence_before();
                     mbar_arrive(gready);
+                    if (!hon) {  // first tile with a nonzero g in the block: its maxima give the first scales
+                        float m0 = 0.0f, m1 = 0.0f;
+#pragma unroll
+                        for (int q = 0; q < C::PP; ++q)
+#pragma unroll
+                            for (int l = 0; l < 8; ++l) {
+                                m0 = finite_max(m0, gv[q][l]);
+                                m1 = finite_max(m1, gv[q][l] * u[q]);
+                            }
+                        hon = hist_open(hacc, m0, m1, smax, warp, lane);
+                    }
                     if (hon) {
                         hist_add<C::PP>(bins, hpart, hacc, j, u, gv, dU);
                         if (++hacc.tiles == hist_tiles<C::MP>()) hist_close(bins, hpart, a.lay.nint, hacc, tid, true, smax, warp, lane);

@@ -218,23 +218,6 @@ __global__ void __launch_bounds__(kBThreads, 1)
                 }
                 search<C::PP>(sTe, u, j);
                 bool hon = hacc.open;
-                if (!hon) {
-                    float m0 = 0.0f, m1 = 0.0f;
-#pragma unroll
-                    for (int q = 0; q < C::PP; ++q) {
-                        float al[8], y[8];
-                        channel_eval(sAB, j[q], u[q], al, y);
-                        const float4 p0 = pv[q][0], p1 = pv[q][1];
-                        const float dv[8] = {p0.x, p0.y, p0.z, p0.w, p1.x, p1.y, p1.z, p1.w};
-#pragma unroll
-                        for (int l = 0; l < 8; ++l) {
-                            const float gl = (valid && y[l] > 0.0f) ? dv[l] : 0.0f;
-                            m0 = finite_max(m0, gl);
-                            m1 = finite_max(m1, gl * u[q]);
-                        }
-                    }
-                    hon = hist_open(hacc, m0, m1, smax, warp, lane);
-                }
                 float dU[C::PP], gv[C::PP][8];
 #pragma unroll
                 for (int q = 0; q < C::PP; ++q) {
@@ -266,6 +249,17 @@ __global__ void __launch_bounds__(kBThreads, 1)
                 fence_proxy_async_smem();
                 tc_fence_before();
                 mbar_arrive(gready);
+                if (!hon) {  // first tile with a nonzero g in the block: its maxima give the first scales
+                    float m0 = 0.0f, m1 = 0.0f;
+#pragma unroll
+                    for (int q = 0; q < C::PP; ++q)
+#pragma unroll
+                        for (int l = 0; l < 8; ++l) {
+                            m0 = finite_max(m0, gv[q][l]);
+                            m1 = finite_max(m1, gv[q][l] * u[q]);
+                        }
+                    hon = hist_open(hacc, m0, m1, smax, warp, lane);
+                }
                 if (hon) {
                     hist_add<C::PP>(bins, hpart, hacc, j, u, gv, dU);
                     if (++hacc.tiles == hist_tiles<C::MP>()) hist_close(bins, hpart, a.lay.nint, hacc, tid, true, smax, warp, lane);
