@@ -38,6 +38,7 @@ struct Plan {
     size_t o_dSpart = 0, o_dzpart = 0, o_dSfin = 0, o_dzfin = 0, o_gpart = 0, o_hist = 0;
     size_t o_segS = 0, o_segz = 0, o_segdS = 0, o_segdz = 0, o_rowstat = 0;
     size_t o_dphi = 0, o_phik = 0, o_pq2 = 0;  // streaming-form backward on tensor cores
+    size_t o_items = 0;                        // split of the tensor-core work items (non-causal)
     size_t ws_fwd = 0, ws_bwd = 0, state_bytes = 0;
     TcPlan tc;
 };
@@ -96,6 +97,7 @@ luna_status make_plan(const luna_attn_desc *ad, const luna_phi_desc *pd, Plan &p
         p.o_zpart = w.take((size_t)BH * p.nsplit * D * f);
         p.o_Sfin = w.take((size_t)BH * SD * f);
         p.o_zfin = w.take((size_t)BH * D * f);
+        p.o_items = w.take((kMaxGrid + 1 + 2 * (size_t)BH) * sizeof(int));
         p.ws_fwd = w.n;
         // per-head partial slots: generic splits, or (tensor-core path) runs of work items, never more
         // than the forward split count
@@ -165,6 +167,7 @@ AttnArgs make_args(const luna_attn_desc *ad, const Plan &p, const void *table, c
     if (!ad->causal) {
         a.S_fin = reinterpret_cast<float *>(w + p.o_Sfin);
         a.z_fin = reinterpret_cast<float *>(w + p.o_zfin);
+        a.items_ws = reinterpret_cast<int *>(w + p.o_items);
     } else {
         a.seg_S = reinterpret_cast<float *>(w + p.o_segS);
         a.seg_z = reinterpret_cast<float *>(w + p.o_segz);

@@ -33,6 +33,11 @@ struct AttnArgs {
     // streaming-form backward on tensor cores
     float *dphi;                       // [BH][n][D] fp32: dLoss/dphi of Q, then of K
     void *phik, *pq2;                  // [BH][n][2D] bf16 phi(k), phi(q)/den, each as (hi | lo)
+    // tensor-core work items balanced by valid tiles (non-causal, with lengths): workspace for the split
+    // ([kMaxGrid + 1] block starts, [2*BH] runs), and the split in use (null: by count)
+    int *items_ws;
+    const int *split;                  // block b takes items split[b] .. split[b+1]-1
+    const int *runs;                   // [2*BH]: first and last block holding an item of head bh
 };
 
 // one step of the streaming form for every (batch, head): state S [D][dv], z [D] (fp32, in place)

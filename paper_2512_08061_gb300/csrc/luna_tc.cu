@@ -362,7 +362,7 @@ __global__ void __launch_bounds__(kThreadsTC, 1)
             named_sync<kWorkers>(1);
             if (warp < 4) {
                 // run epilogue: statistics of this block's part of head bh -> its partial slot
-                const RunSlot rs = run_slot(it, bh);
+                const RunSlot rs = run_slot(a, it, bh);
                 const int nruns = rs.nruns;
                 const size_t slot = per_item ? (size_t)i0 : (size_t)bh * it.nchunk + rs.rank;
                 float *Sp = a.S_part + slot * C::D * C::DV;
@@ -703,6 +703,104 @@ AttnArgs tc_items_impl(const AttnArgs &a) {
     return b;
 }
 
+// Valid 128-row tiles of work item i (chunk i % nsplit of head i / nsplit).
+__device__ __forceinline__ int item_tiles(const AttnArgs &a, int i) {
+    const int bh = i / a.nsplit, c = i - bh * a.nsplit;
+    const int len = head_length(a.lengths, bh / a.H, a.n);
+    const int r0 = c * a.rows_per_split, r1 = min(len, min(a.n, r0 + a.rows_per_split));
+    return r1 > r0 ? (r1 - r0 + 127) / 128 : 0;
+}
+
+// Split of the work items over a grid of G persistent blocks (one block of 1024 threads): each block gets a
+// contiguous, non-empty item range holding about 1/G of the valid tiles (block b starts at the first item
+// before which at least b/G of them lie), and each head the first and last block holding one of its items.
+// The tile prefix lives in shared memory (kSplitItems items at most; more items keep the split by count).
+constexpr int kSplitThreads = 1024;
+constexpr int kSplitItems = 12 * 1024;
+__global__ void __launch_bounds__(kSplitThreads) k_tile_split(AttnArgs a, int G) {
+    __shared__ int wsum[kSplitThreads / 32];
+    __shared__ int ssplit[kMaxGrid + 1];
+    extern __shared__ int prefix[];  // [total + 1] tiles before item i
+    const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+    const int total = a.B * a.H * a.nsplit;
+    int *split = a.items_ws;               // [G + 1]
+    int *runs = split + kMaxGrid + 1;      // [2 * BH]
+    const int per = (total + kSplitThreads - 1) / kSplitThreads;
+    const int i0 = min(total, tid * per), i1 = min(total, i0 + per);
+    int mine = 0;
+    for (int i = i0; i < i1; ++i) {
+        const int t = item_tiles(a, i);
+        prefix[i] = t;
+        mine += t;
+    }
+    // block-wide scans (warp shuffles, then over the warps); op 0: sum, op 1: max
+    auto scan = [&](int v, bool mx) {
+        int incl = v;
+#pragma unroll
+        for (int o = 1; o < 32; o <<= 1) {
+            const int w = __shfl_up_sync(0xffffffffu, incl, o);
+            if (lane >= o) incl = mx ? max(incl, w) : incl + w;
+        }
+        if (lane == 31) wsum[warp] = incl;
+        __syncthreads();
+        if (warp == 0) {
+            int w = wsum[lane];
+#pragma unroll
+            for (int o = 1; o < 32; o <<= 1) {
+                const int u = __shfl_up_sync(0xffffffffu, w, o);
+                if (lane >= o) w = mx ? max(w, u) : w + u;
+            }
+            wsum[lane] = w;
+        }
+        __syncthreads();
+        const int before = warp > 0 ? wsum[warp - 1] : (mx ? INT_MIN : 0);
+        const int r = mx ? max(before, incl) : before + incl;  // inclusive over the block
+        const int last = wsum[kSplitThreads / 32 - 1];
+        __syncthreads();  // wsum is reused by the next scan
+        return make_int2(r, last);
+    };
+    const int2 sc = scan(mine, false);
+    int run = sc.x - mine;
+    for (int i = i0; i < i1; ++i) {
+        const int t = prefix[i];
+        prefix[i] = run;
+        run += t;
+    }
+    const int T = sc.y;
+    if (tid == 0) prefix[total] = T;
+    __syncthreads();
+    // lb[b]: first item with at least b*T/G tiles before it.  Every block must get an item (total >= G), so
+    // start[b] = b + min(max over b' <= b of (lb[b'] - b'), total - G): strictly increasing, start[0] = 0.
+    int lbm = INT_MIN;
+    if (tid < G) {
+        const long long target = (long long)tid * T / G;
+        int lo = 0, hi = total;
+        while (lo < hi) {
+            const int mid = (lo + hi) >> 1;
+            if (prefix[mid] < target) lo = mid + 1; else hi = mid;
+        }
+        lbm = lo - tid;
+    }
+    const int2 mx = scan(lbm, true);
+    if (tid < G) ssplit[tid] = tid + min(mx.x, total - G);
+    if (tid == 0) ssplit[G] = total;
+    __syncthreads();
+    for (int b = tid; b <= G; b += kSplitThreads) split[b] = ssplit[b];
+    // owner of item i: the block b with ssplit[b] <= i < ssplit[b + 1]
+    auto owner = [&](int i) {
+        int lo = 0, hi = G - 1;
+        while (lo < hi) {
+            const int mid = (lo + hi + 1) >> 1;
+            if (ssplit[mid] <= i) lo = mid; else hi = mid - 1;
+        }
+        return lo;
+    };
+    for (int bh = tid; bh < a.B * a.H; bh += kSplitThreads) {
+        runs[2 * bh] = owner(bh * a.nsplit);
+        runs[2 * bh + 1] = owner((bh + 1) * a.nsplit - 1);
+    }
+}
+
 int sm_count_impl() {
     static int n = 0;
     if (n == 0) {
@@ -713,6 +811,29 @@ int sm_count_impl() {
     return n;
 }
 
+int grid_impl(const AttnArgs &a) {
+    const int items = a.B * a.H * a.nsplit;
+    return items < sm_count_impl() ? items : sm_count_impl();
+}
+
+AttnArgs balanced_impl(const AttnArgs &a0, cudaStream_t s, cudaError_t *err) {
+    AttnArgs a = tc_items_impl(a0);
+    *err = cudaSuccess;
+    if (a.split != nullptr || a.lengths == nullptr || a.items_ws == nullptr) return a;
+    const int G = grid_impl(a);
+    const int total = a.B * a.H * a.nsplit;
+    if (G < 1 || G > kMaxGrid || total > kSplitItems) return a;
+    const size_t smem = ((size_t)total + 1) * sizeof(int);
+    if (smem > 48 * 1024 &&
+        (*err = cudaFuncSetAttribute(k_tile_split, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem)) != cudaSuccess)
+        return a;
+    LUNA_LAUNCH("tile_split", k_tile_split, 1, kSplitThreads, smem, s, a, G);
+    if ((*err = cudaGetLastError()) != cudaSuccess) return a;
+    a.split = a.items_ws;
+    a.runs = a.split + kMaxGrid + 1;
+    return a;
+}
+
 template <class C>
 cudaError_t keys_tc(const AttnArgs &a, cudaStream_t s) {
     CUtensorMap mK, mV;
@@ -720,24 +841,21 @@ cudaError_t keys_tc(const AttnArgs &a, cudaStream_t s) {
         return cudaErrorInvalidValue;
     cudaError_t e = cudaFuncSetAttribute(k_tc_keys<C>, cudaFuncAttributeMaxDynamicSharedMemorySize, C::SMEM_K);
     if (e != cudaSuccess) return e;
-    const int items = a.B * a.H * a.nsplit;
-    const int grid = items < sm_count_impl() ? items : sm_count_impl();
-    LUNA_LAUNCH("tc_keys", k_tc_keys<C>, grid, kThreadsTC, C::SMEM_K, s, mK, mV, a, status_word(a));
+    LUNA_LAUNCH("tc_keys", k_tc_keys<C>, grid_impl(a), kThreadsTC, C::SMEM_K, s, mK, mV, a, status_word(a));
     return cudaGetLastError();
 }
 
 template <class C>
 cudaError_t fwd_tc(const AttnArgs &a0, cudaStream_t s) {
-    const AttnArgs a = tc_items_impl(a0);
-    cudaError_t e = keys_tc<C>(a, s);
+    cudaError_t e;
+    const AttnArgs a = balanced_impl(a0, s, &e);
     if (e != cudaSuccess) return e;
+    if ((e = keys_tc<C>(a, s)) != cudaSuccess) return e;
     CUtensorMap mQ;
     if (!make_map_impl(&mQ, a.Q, a.d, a.n, a.B * a.H)) return cudaErrorInvalidValue;
     e = cudaFuncSetAttribute(k_tc_query<C>, cudaFuncAttributeMaxDynamicSharedMemorySize, C::SMEM_Q);
     if (e != cudaSuccess) return e;
-    const int items = a.B * a.H * a.nsplit;
-    const int grid = items < sm_count_impl() ? items : sm_count_impl();
-    LUNA_LAUNCH("tc_query", k_tc_query<C>, grid, kThreadsTC, C::SMEM_Q, s, mQ, a, status_word(a));
+    LUNA_LAUNCH("tc_query", k_tc_query<C>, grid_impl(a), kThreadsTC, C::SMEM_Q, s, mQ, a, status_word(a));
     return cudaGetLastError();
 }
 
@@ -763,6 +881,8 @@ bool tc_make_map_rows(CUtensorMap *m, const void *base, int width, int n, int BH
 }
 int tc_sm_count() { return sm_count_impl(); }
 AttnArgs tc_work_items(const AttnArgs &a) { return tc_items_impl(a); }
+AttnArgs tc_balanced_items(const AttnArgs &a, cudaStream_t s, cudaError_t *err) { return balanced_impl(a, s, err); }
+int tc_grid(const AttnArgs &items) { return grid_impl(items); }
 
 TcPlan tc_plan(const luna_attn_desc &ad, const TableLayout &lay) {
     TcPlan p;
@@ -804,7 +924,9 @@ cudaError_t launch_tc_keys_items(const AttnArgs &a, cudaStream_t s) {
 
 cudaError_t launch_tc_stats(const AttnArgs &a0, cudaStream_t s) {
     const TcPlan p = tc_plan(luna_attn_desc{a0.B, a0.H, a0.n, a0.d, a0.dv, 0, 0, a0.eps, LUNA_BF16}, a0.lay);
-    const AttnArgs a = tc_items_impl(a0);
+    cudaError_t e;
+    const AttnArgs a = balanced_impl(a0, s, &e);  // the split of the forward pass: the same sums in the same order
+    if (e != cudaSuccess) return e;
     switch (p.variant) {
         case 0: return keys_tc<C32>(a, s);
         case 1: return keys_tc<C64>(a, s);

@@ -19,6 +19,11 @@ bool tc_inputs_ok(const TcPlan &p, const void *a, const void *b, const void *c, 
 cudaError_t launch_tc_fwd(const TcPlan &p, const AttnArgs &a, char *ws, cudaStream_t s);
 cudaError_t launch_tc_bwd(const TcPlan &p, const AttnArgs &a, char *ws, bool have_stats, cudaStream_t s);
 cudaError_t launch_tc_stats(const AttnArgs &a, cudaStream_t s);
+// Work items of the persistent non-causal kernels (chunks of whole 128-row tiles of one head) and, for
+// padded sequences, their split over the grid balanced by valid tiles (a small split kernel on s).
+AttnArgs tc_balanced_items(const AttnArgs &a, cudaStream_t s, cudaError_t *err);
+int tc_grid(const AttnArgs &items);  // persistent grid of the non-causal kernels
+constexpr int kMaxGrid = 1024;       // split entries the workspace holds
 bool tc_bwd_supported(const luna_attn_desc &ad, const TableLayout &lay);
 bool tc_bwd_fits(const AttnArgs &a);
 cudaError_t launch_tc_bwd_kernels(const AttnArgs &a, bool have_stats, cudaStream_t s);

@@ -422,7 +422,7 @@ __global__ void __launch_bounds__(kBThreads, 1)
             // run epilogue (warps 0..3): dS, dz partial of this head; warp w holds features 16w..16w+15,
             // hi in lanes 0..15 and lo in lanes 16..31
             if (warp < 4) {
-                const RunSlot rs = run_slot(it, bh);
+                const RunSlot rs = run_slot(a, it, bh);
                 const int nruns = rs.nruns;
                 const size_t slot = (size_t)bh * it.nchunk + rs.rank;
                 float *Sp = a.dS_part + slot * C::D * C::DV;
@@ -873,16 +873,14 @@ __global__ void __launch_bounds__(kBThreads, 1)
 }  // namespace
 
 bool tc_make_map(CUtensorMap *m, const void *base, int width, int n, int BH);
-int tc_sm_count();
-AttnArgs tc_work_items(const AttnArgs &a);
 
 cudaError_t launch_tc_bwd_wide(const AttnArgs &a0, bool have_stats, cudaStream_t s) {
     using C = B64;
-    const AttnArgs a = tc_work_items(a0);
-    const int items = a.B * a.H * a.nsplit;
-    const int grid = items < tc_sm_count() ? items : tc_sm_count();
     cudaError_t e;
-    if (!have_stats && (e = launch_tc_stats(a0, s)) != cudaSuccess) return e;
+    const AttnArgs a = tc_balanced_items(a0, s, &e);
+    if (e != cudaSuccess) return e;
+    const int grid = tc_grid(a);
+    if (!have_stats && (e = launch_tc_stats(a, s)) != cudaSuccess) return e;
     CUtensorMap mQ, mdO, mK, mV;
     if (!tc_make_map(&mQ, a.Q, a.d, a.n, a.B * a.H) || !tc_make_map(&mdO, a.dO, a.dv, a.n, a.B * a.H) ||
         !tc_make_map(&mK, a.K, a.d, a.n, a.B * a.H) || !tc_make_map(&mV, a.V, a.dv, a.n, a.B * a.H))

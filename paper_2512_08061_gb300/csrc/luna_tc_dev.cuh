@@ -108,8 +108,13 @@ struct Items {
         rows = a.rows_per_split;
         nchunk = a.nsplit;
         total = a.B * a.H * nchunk;
-        begin = (int)((long long)blockIdx.x * total / gridDim.x);
-        end = (int)((long long)(blockIdx.x + 1) * total / gridDim.x);
+        if (a.split) {  // balanced by valid tiles (padded sequences)
+            begin = a.split[blockIdx.x];
+            end = a.split[blockIdx.x + 1];
+        } else {
+            begin = (int)((long long)blockIdx.x * total / gridDim.x);
+            end = (int)((long long)(blockIdx.x + 1) * total / gridDim.x);
+        }
     }
 };
 
@@ -135,7 +140,8 @@ struct RunSlot {
     int rank, nruns;
 };
 
-__device__ __forceinline__ RunSlot run_slot(const Items &it, int bh) {
+__device__ __forceinline__ RunSlot run_slot(const AttnArgs &a, const Items &it, int bh) {
+    if (a.runs) return RunSlot{(int)blockIdx.x - a.runs[2 * bh], a.runs[2 * bh + 1] - a.runs[2 * bh] + 1};
     const long long total = it.total;
     const int G = gridDim.x;
     const int c_first = (int)((((long long)bh * it.nchunk + 1) * G - 1) / total);

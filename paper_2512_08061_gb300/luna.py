@@ -21,7 +21,7 @@ STATUS_NAMES = {0: "LUNA_OK", 1: "LUNA_ERR_INVALID_ARG", 2: "LUNA_ERR_UNSUPPORTE
 LUNA_F32, LUNA_BF16 = 0, 1
 _DTYPES = {torch.float32: LUNA_F32, torch.bfloat16: LUNA_BF16}
 # names of the tensor-core kernels accepted by luna_profile_start
-TC_KERNELS: list[str] = ["tc_keys", "tc_query", "tc_bwd_query", "tc_bwd_key", "tc_causal", "seg_scan",
+TC_KERNELS: list[str] = ["tile_split", "tc_keys", "tc_query", "tc_bwd_query", "tc_bwd_key", "tc_causal", "seg_scan",
                          "tcc_query", "tcc_dstats", "seg_rscan", "tcc_key", "tc_phi_bwd"]
 
 
