@@ -322,17 +322,29 @@ __global__ void __launch_bounds__(kThreads) k_bwd_key(AttnArgs a) {
 //     dw2 = (w1 G1 + b1 G0)/sqrt(M), dw1 = w2 G1/sqrt(M), db1 = w2 G0/sqrt(M),
 //     db2 = sum_j m0 / sqrt(M).
 
+// Compensated (Neumaier) fp32 summation: s + c carries the running sum with about twice fp32's
+// precision (fp64 arithmetic runs at a small fraction of the fp32 rate on this part).
+struct CompSum {
+    float s = 0.0f, c = 0.0f;
+    __device__ __forceinline__ void add(float x) {
+        const float t = s + x;
+        c += fabsf(s) >= fabsf(x) ? (s - t) + x : (x - t) + s;
+        s = t;
+    }
+};
+
 // Sum of the per-block parameter-gradient partials, in the fixed order p = 0..nparts-1
-// per element: 64 elements per block, each summed by 4 threads over consecutive
-// quarters of the partials (8 loads in flight), then combined in quarter order.
-constexpr int kSumElems = 64, kSumSplit = 4;
+// per element: 64 elements per block, each summed by 8 threads over consecutive
+// eighths of the partials (8 loads in flight, compensated fp32), then the eight parts
+// combined in order in fp64.
+constexpr int kSumElems = 64, kSumSplit = 8;
 __global__ void __launch_bounds__(kSumElems * kSumSplit) k_grad_sum(const float *gpart, int nparts, int gsize,
                                                                     float *out) {
     __shared__ double part[kSumSplit][kSumElems];
     const int el = threadIdx.x % kSumElems, q = threadIdx.x / kSumElems;
     const int e = blockIdx.x * kSumElems + el;
     const int p0 = (int)((long long)q * nparts / kSumSplit), p1 = (int)((long long)(q + 1) * nparts / kSumSplit);
-    double s = 0.0;
+    CompSum cs;
     if (e < gsize) {
         int p = p0;
         for (; p + 8 <= p1; p += 8) {
@@ -340,11 +352,11 @@ __global__ void __launch_bounds__(kSumElems * kSumSplit) k_grad_sum(const float 
 #pragma unroll
             for (int k = 0; k < 8; ++k) v[k] = __ldcg(gpart + (size_t)(p + k) * gsize + e);
 #pragma unroll
-            for (int k = 0; k < 8; ++k) s += v[k];
+            for (int k = 0; k < 8; ++k) cs.add(v[k]);
         }
-        for (; p < p1; ++p) s += __ldcg(gpart + (size_t)p * gsize + e);
+        for (; p < p1; ++p) cs.add(__ldcg(gpart + (size_t)p * gsize + e));
     }
-    part[q][el] = s;
+    part[q][el] = (double)cs.s + (double)cs.c;
     __syncthreads();
     if (q == 0 && e < gsize) {
         double t = part[0][el];
