@@ -38,6 +38,7 @@ struct AttnArgs {
     int *items_ws;
     const int *split;                  // block b takes items split[b] .. split[b+1]-1
     const int *runs;                   // [2*BH]: first and last block holding an item of head bh
+    int padded_zeroed;                 // the outputs' rows past each sequence's length are already zero
 };
 
 // one step of the streaming form for every (batch, head): state S [D][dv], z [D] (fp32, in place)

@@ -475,8 +475,8 @@ __global__ void __launch_bounds__(kThreadsTC, 1)
     }
     if (warp == 0) { tmem_alloc(tslot, C::TMEM_Q); tmem_relinquish(); }
     stage_phi_table<C>(a, sTe, sAB, sbias, Wop);
-    // padded rows of every item of this block produce zeros
-    for (int item = it.begin; item < it.end; ++item) {
+    // padded rows of every item of this block produce zeros (unless the split kernel zeroed them)
+    for (int item = it.begin; item < it.end && !a.padded_zeroed; ++item) {
         const ItemRange ir = item_range(a, it, item);
         __nv_bfloat16 *O = static_cast<__nv_bfloat16 *>(a.O) + (size_t)ir.bh * a.n * C::DV;
         const int z0 = max(ir.r0, ir.r1);
@@ -717,7 +717,26 @@ __device__ __forceinline__ int item_tiles(const AttnArgs &a, int i) {
 // The tile prefix lives in shared memory (kSplitItems items at most; more items keep the split by count).
 constexpr int kSplitThreads = 1024;
 constexpr int kSplitItems = 12 * 1024;
-__global__ void __launch_bounds__(kSplitThreads) k_tile_split(AttnArgs a, int G) {
+// Blocks 1.. of the launch zero the rows past each sequence's length of the outputs in zmask (1: O, 2: dQ,
+// 4: dK, 8: dV), head by head with the whole GPU's store bandwidth, so that the persistent kernels skip it.
+__global__ void __launch_bounds__(kSplitThreads) k_tile_split(AttnArgs a, int G, int zmask) {
+    if (blockIdx.x > 0) {
+        const int Z = gridDim.x - 1;
+        for (int bh = blockIdx.x - 1; bh < a.B * a.H; bh += Z) {
+            const int len = head_length(a.lengths, bh / a.H, a.n);
+            if (len >= a.n) continue;
+            auto zero = [&](void *X, int w) {  // w: bf16 elements per row (a multiple of 8)
+                uint4 *p = reinterpret_cast<uint4 *>(static_cast<__nv_bfloat16 *>(X) + ((size_t)bh * a.n + len) * w);
+                const int cnt = (a.n - len) * (w / 8);
+                for (int e = threadIdx.x; e < cnt; e += blockDim.x) p[e] = make_uint4(0, 0, 0, 0);
+            };
+            if (zmask & 1) zero(a.O, a.dv);
+            if (zmask & 2) zero(a.dQ, a.d);
+            if (zmask & 4) zero(a.dK, a.d);
+            if (zmask & 8) zero(a.dV, a.dv);
+        }
+        return;
+    }
     __shared__ int wsum[kSplitThreads / 32];
     __shared__ int ssplit[kMaxGrid + 1];
     extern __shared__ int prefix[];  // [total + 1] tiles before item i
@@ -816,7 +835,7 @@ int grid_impl(const AttnArgs &a) {
     return items < sm_count_impl() ? items : sm_count_impl();
 }
 
-AttnArgs balanced_impl(const AttnArgs &a0, cudaStream_t s, cudaError_t *err) {
+AttnArgs balanced_impl(const AttnArgs &a0, cudaStream_t s, cudaError_t *err, int zmask) {
     AttnArgs a = tc_items_impl(a0);
     *err = cudaSuccess;
     if (a.split != nullptr || a.lengths == nullptr || a.items_ws == nullptr) return a;
@@ -827,10 +846,12 @@ AttnArgs balanced_impl(const AttnArgs &a0, cudaStream_t s, cudaError_t *err) {
     if (smem > 48 * 1024 &&
         (*err = cudaFuncSetAttribute(k_tile_split, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem)) != cudaSuccess)
         return a;
-    LUNA_LAUNCH("tile_split", k_tile_split, 1, kSplitThreads, smem, s, a, G);
+    const int zblocks = zmask ? std::min(a.B * a.H, sm_count_impl()) : 0;
+    LUNA_LAUNCH("tile_split", k_tile_split, 1 + zblocks, kSplitThreads, smem, s, a, G, zmask);
     if ((*err = cudaGetLastError()) != cudaSuccess) return a;
     a.split = a.items_ws;
     a.runs = a.split + kMaxGrid + 1;
+    a.padded_zeroed = zmask != 0;
     return a;
 }
 
@@ -848,7 +869,7 @@ cudaError_t keys_tc(const AttnArgs &a, cudaStream_t s) {
 template <class C>
 cudaError_t fwd_tc(const AttnArgs &a0, cudaStream_t s) {
     cudaError_t e;
-    const AttnArgs a = balanced_impl(a0, s, &e);
+    const AttnArgs a = balanced_impl(a0, s, &e, 1);  // the query pass writes O
     if (e != cudaSuccess) return e;
     if ((e = keys_tc<C>(a, s)) != cudaSuccess) return e;
     CUtensorMap mQ;
@@ -881,7 +902,9 @@ bool tc_make_map_rows(CUtensorMap *m, const void *base, int width, int n, int BH
 }
 int tc_sm_count() { return sm_count_impl(); }
 AttnArgs tc_work_items(const AttnArgs &a) { return tc_items_impl(a); }
-AttnArgs tc_balanced_items(const AttnArgs &a, cudaStream_t s, cudaError_t *err) { return balanced_impl(a, s, err); }
+AttnArgs tc_balanced_items(const AttnArgs &a, cudaStream_t s, cudaError_t *err, int zmask) {
+    return balanced_impl(a, s, err, zmask);
+}
 int tc_grid(const AttnArgs &items) { return grid_impl(items); }
 
 TcPlan tc_plan(const luna_attn_desc &ad, const TableLayout &lay) {
@@ -925,7 +948,7 @@ cudaError_t launch_tc_keys_items(const AttnArgs &a, cudaStream_t s) {
 cudaError_t launch_tc_stats(const AttnArgs &a0, cudaStream_t s) {
     const TcPlan p = tc_plan(luna_attn_desc{a0.B, a0.H, a0.n, a0.d, a0.dv, 0, 0, a0.eps, LUNA_BF16}, a0.lay);
     cudaError_t e;
-    const AttnArgs a = balanced_impl(a0, s, &e);  // the split of the forward pass: the same sums in the same order
+    const AttnArgs a = balanced_impl(a0, s, &e, 0);  // the split of the forward pass: the same sums in the same order
     if (e != cudaSuccess) return e;
     switch (p.variant) {
         case 0: return keys_tc<C32>(a, s);

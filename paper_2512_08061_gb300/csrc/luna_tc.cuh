@@ -21,7 +21,8 @@ cudaError_t launch_tc_bwd(const TcPlan &p, const AttnArgs &a, char *ws, bool hav
 cudaError_t launch_tc_stats(const AttnArgs &a, cudaStream_t s);
 // Work items of the persistent non-causal kernels (chunks of whole 128-row tiles of one head) and, for
 // padded sequences, their split over the grid balanced by valid tiles (a small split kernel on s).
-AttnArgs tc_balanced_items(const AttnArgs &a, cudaStream_t s, cudaError_t *err);
+// zmask: outputs whose padded rows the split launch zeroes (1: O, 2: dQ, 4: dK, 8: dV).
+AttnArgs tc_balanced_items(const AttnArgs &a, cudaStream_t s, cudaError_t *err, int zmask);
 int tc_grid(const AttnArgs &items);  // persistent grid of the non-causal kernels
 constexpr int kMaxGrid = 1024;       // split entries the workspace holds
 bool tc_bwd_supported(const luna_attn_desc &ad, const TableLayout &lay);

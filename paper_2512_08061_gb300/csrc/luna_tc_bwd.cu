@@ -129,8 +129,8 @@ __global__ void __launch_bounds__(kBThreads, 1)
     for (int e = tid; e < C::MP * C::d + 16; e += blockDim.x) sdW[e] = 0.0f;
     float *hpart = a.gpart + (size_t)blockIdx.x * a.gsize + C::MP * a.d + C::MP;  // histogram part of the partial
     for (int e = tid; e < a.lay.nint * 16; e += blockDim.x) hpart[e] = 0.0f;
-    // padded rows of every item produce zero gradients
-    for (int item = it.begin; item < it.end; ++item) {
+    // padded rows of every item produce zero gradients (unless the split kernel zeroed them)
+    for (int item = it.begin; item < it.end && !a.padded_zeroed; ++item) {
         const ItemRange ir = item_range(a, it, item);
         __nv_bfloat16 *dQ = static_cast<__nv_bfloat16 *>(a.dQ) + (size_t)ir.bh * a.n * C::d;
         const int z0 = max(ir.r0, ir.r1);
@@ -588,7 +588,7 @@ __global__ void __launch_bounds__(kBThreads, 1)
     float *hpart = a.gpart + (size_t)(gridDim.x + blockIdx.x) * a.gsize + C::MP * a.d + C::MP;
     for (int e = tid; e < a.lay.nint * 16; e += blockDim.x) hpart[e] = 0.0f;
     for (int e = tid; e < (int)(T16 / 16); e += blockDim.x) reinterpret_cast<uint4 *>(Gt)[e] = make_uint4(0, 0, 0, 0);
-    for (int item = it.begin; item < it.end; ++item) {  // padded rows receive zero gradients
+    for (int item = it.begin; item < it.end && !a.padded_zeroed; ++item) {  // padded rows: zero gradients
         const ItemRange ir = item_range(a, it, item);
         __nv_bfloat16 *dK = static_cast<__nv_bfloat16 *>(a.dK) + (size_t)ir.bh * a.n * C::d;
         __nv_bfloat16 *dV = static_cast<__nv_bfloat16 *>(a.dV) + (size_t)ir.bh * a.n * C::DV;
@@ -901,7 +901,7 @@ namespace {
 template <class C>
 cudaError_t bwd_tc(const AttnArgs &a0, bool have_stats, cudaStream_t s) {
     cudaError_t e;
-    const AttnArgs a = tc_balanced_items(a0, s, &e);
+    const AttnArgs a = tc_balanced_items(a0, s, &e, 2 | 4 | 8);  // dQ, dK, dV
     if (e != cudaSuccess) return e;
     const int grid = tc_grid(a);
     if (!have_stats && (e = launch_tc_stats(a, s)) != cudaSuccess) return e;

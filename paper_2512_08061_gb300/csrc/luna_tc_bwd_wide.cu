@@ -117,7 +117,7 @@ __global__ void __launch_bounds__(kBThreads, 1)
     for (int e = tid; e < (int)(T16 / 16); e += blockDim.x) reinterpret_cast<uint4 *>(Gt)[e] = make_uint4(0, 0, 0, 0);
     float *hpart = a.gpart + (size_t)blockIdx.x * a.gsize + C::MP * a.d + C::MP;
     for (int e = tid; e < a.lay.nint * 16; e += blockDim.x) hpart[e] = 0.0f;
-    for (int item = it.begin; item < it.end; ++item) {  // padded rows receive zero gradients
+    for (int item = it.begin; item < it.end && !a.padded_zeroed; ++item) {  // padded rows: zero gradients
         const ItemRange ir = item_range(a, it, item);
         __nv_bfloat16 *dQ = static_cast<__nv_bfloat16 *>(a.dQ) + (size_t)ir.bh * a.n * C::d;
         const int z0 = max(ir.r0, ir.r1);
@@ -575,7 +575,7 @@ __global__ void __launch_bounds__(kBThreads, 1)
     for (int e = tid; e < (int)(T16 / 16); e += blockDim.x) reinterpret_cast<uint4 *>(Gt)[e] = make_uint4(0, 0, 0, 0);
     float *hpart = a.gpart + (size_t)(gridDim.x + blockIdx.x) * a.gsize + C::MP * a.d + C::MP;
     for (int e = tid; e < a.lay.nint * 16; e += blockDim.x) hpart[e] = 0.0f;
-    for (int item = it.begin; item < it.end; ++item) {  // padded rows receive zero gradients
+    for (int item = it.begin; item < it.end && !a.padded_zeroed; ++item) {  // padded rows: zero gradients
         const ItemRange ir = item_range(a, it, item);
         __nv_bfloat16 *dK = static_cast<__nv_bfloat16 *>(a.dK) + (size_t)ir.bh * a.n * C::d;
         __nv_bfloat16 *dV = static_cast<__nv_bfloat16 *>(a.dV) + (size_t)ir.bh * a.n * C::DV;
@@ -877,7 +877,7 @@ bool tc_make_map(CUtensorMap *m, const void *base, int width, int n, int BH);
 cudaError_t launch_tc_bwd_wide(const AttnArgs &a0, bool have_stats, cudaStream_t s) {
     using C = B64;
     cudaError_t e;
-    const AttnArgs a = tc_balanced_items(a0, s, &e);
+    const AttnArgs a = tc_balanced_items(a0, s, &e, 2 | 4 | 8);  // dQ, dK, dV
     if (e != cudaSuccess) return e;
     const int grid = tc_grid(a);
     if (!have_stats && (e = launch_tc_stats(a, s)) != cudaSuccess) return e;
