@@ -230,6 +230,36 @@ def test_backward_tensor_core_repeat_bitwise():
         assert np.array_equal(g1[k], g2[k]), k
 
 
+@pytest.mark.parametrize("d,tiles", [(32, "1"), (32, "4"), (64, "2")])
+def test_backward_tensor_core_balanced_split(d, tiles, monkeypatch):
+    """Work items split over the persistent grid by valid tiles: sequences of
+    length 0, 1, a tile minus one, one, plus one, half and full in one batch,
+    so that whole runs of items hold no tile, every block must still get an
+    item, and one head's items spread over several blocks (partial slots and
+    the last-block reduction of each head).  The output rows past each length
+    are zeroed by the split launch."""
+    monkeypatch.setenv("LUNA_TC_TILES_PER_SPLIT", tiles)
+    lengths = [1500, 0, 1, 127, 128, 129, 750, 1499]
+    case = Case(len(lengths), 2, 1500, d, 8, 8, "bf16", False, seed=89, qkv_scale=1.0 / math.sqrt(d),
+                lengths=lengths, with_grad=True)
+    lu = case.luna()
+    O = to_host(case.run_fwd(lu))
+    ref_O = case.oracle_fwd()
+    assert relerr(O, ref_O) < TOL["bf16"]
+    g = {k: to_host(v) for k, v in case.run_bwd(lu).items()}
+    ref = case.oracle_bwd()
+    okq, okk = case.smooth_rows("Q"), case.smooth_rows("K")
+    for k, ok in (("dQ", okq), ("dK", okk), ("dV", None)):
+        got, want = (g[k], ref[k]) if ok is None else (g[k][ok], ref[k][ok])
+        assert relerr(got, want) < TOL["bf16"], k
+    for k in ("dW", "db", "dw1", "db1", "dw2", "db2"):
+        assert relerr(g[k], ref[k]) < TOL["bf16"], k
+    for b, ln in enumerate(lengths):
+        assert np.all(O[b, :, ln:] == 0)
+        for k in ("dQ", "dK", "dV"):
+            assert np.all(g[k][b, :, ln:] == 0), (k, b)
+
+
 @pytest.mark.parametrize("d,M,causal", [(32, 8, False), (64, 8, False), (128, 16, True)])
 def test_backward_tensor_core_histogram_ranges(d, M, causal, monkeypatch):
     """The fixed-point interval histogram of the channel-MLP gradient
