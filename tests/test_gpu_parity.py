@@ -218,10 +218,12 @@ def test_backward_tensor_core_hidden_32():
     _check_bwd(case, g, case.oracle_bwd(), TOL["bf16"])
 
 
-def test_backward_tensor_core_repeat_bitwise():
+@pytest.mark.parametrize("d,lengths", [(32, None), (64, None), (32, [700, 333])])
+def test_backward_tensor_core_repeat_bitwise(d, lengths):
     """dQ, dK and dV of the tensor-core backward do not depend on the order of
-    floating-point atomics, so repeated runs agree bit for bit."""
-    case = Case(2, 2, 700, 32, 8, 8, "bf16", False, seed=53, with_grad=True)
+    floating-point atomics, so repeated runs agree bit for bit (d = 32 and 64,
+    and with padded sequences, whose work items are split by valid tiles)."""
+    case = Case(2, 2, 700, d, 8, 8, "bf16", False, seed=53, with_grad=True, lengths=lengths)
     lu = case.luna()
     case.run_fwd(lu)
     g1 = {k: to_host(v) for k, v in case.run_bwd(lu).items()}
