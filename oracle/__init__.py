@@ -46,7 +46,7 @@ def build(force: bool = False) -> str:
 class _Phi(ctypes.Structure):
     _fields_ = [("d", ctypes.c_int), ("M", ctypes.c_int), ("L", ctypes.c_int), ("hid", ctypes.c_int)] + [
         (k, ctypes.c_void_p) for k in ("W", "b", "w1", "b1", "w2", "b2")
-    ] + [("shared", ctypes.c_int)]
+    ] + [("shared", ctypes.c_int), ("ch_rms_target", ctypes.c_double), ("chs", ctypes.c_void_p)]
 
 
 _P = ctypes.c_void_p
@@ -69,6 +69,7 @@ def lib():
             L.oracle_attn_fwd.argtypes = [phi, _I, _I, _I, _I, _I, _D, _P, _P, _P, _P, _P]
             L.oracle_attn_quadratic.argtypes = [phi, _I, _I, _I, _I, _I, _D, _P, _P, _P, _P, _P]
             L.oracle_attn_bwd.argtypes = [phi, _I, _I, _I, _I, _I, _D, _P, _P, _P, _P, _P, _P, _P, _P] + [_P] * 6
+            L.oracle_ch_rms.argtypes = [phi, _P, _I, _I, _I, _P, _P, _P]
             L.oracle_max_threads.restype = _I
             L.oracle_set_threads.argtypes = [_I]
             L.oracle_set_abs_terms.argtypes = [_I]
@@ -91,9 +92,12 @@ def _f64(a) -> np.ndarray:
 class PhiParams:
     """fp64 copies of the feature-map parameters (W, b, w1, b1, w2, b2).  One MLP per
     channel: w1, b1, w2 of shape (L, hidden); the shared-channel MLP: w1, b1 of shape
-    (hidden,) and w2 of shape (L, hidden)."""
+    (hidden,) and w2 of shape (L, hidden).  ch_rms_target > 0 turns on the channel RMS
+    normalisation: every channel's MLP outputs are scaled by
+    s_l = min(target / (rms_l + 1e-6), 1) with rms_l over the valid rows of the input
+    the feature map is applied to (the queries and the keys separately)."""
 
-    def __init__(self, params: dict):
+    def __init__(self, params: dict, ch_rms_target: float = 0.0):
         self.arrays = {k: _f64(params[k]) for k in ("W", "b", "w1", "b1", "w2", "b2")}
         W = self.arrays["W"]
         self.M, self.d = W.shape
@@ -104,7 +108,8 @@ class PhiParams:
         assert self.arrays["b2"].shape == (self.L,)
         self.struct = _Phi(self.d, self.M, self.L, self.hid,
                            *[self.arrays[k].ctypes.data for k in ("W", "b", "w1", "b1", "w2", "b2")],
-                           int(self.shared))
+                           int(self.shared), float(ch_rms_target), None)
+        self.ch_rms_target = float(ch_rms_target)
 
     @property
     def D(self) -> int:
@@ -118,8 +123,22 @@ def _as_params(params) -> PhiParams:
     return params if isinstance(params, PhiParams) else PhiParams(params)
 
 
+def ch_rms(params, X, lengths=None):
+    """Channel RMS statistics of the MLP outputs over the valid rows of X (B,H,n,d):
+    (s, rms), each of shape (L,), s = min(target / (rms + 1e-6), 1)."""
+    p = _as_params(params)
+    X = _f64(X)
+    B, H, n, d = X.shape
+    la, lp = _lens(lengths, B)
+    s = np.empty(p.L)
+    rms = np.empty(p.L)
+    lib().oracle_ch_rms(p.ref(), X.ctypes.data, B, H, n, lp, s.ctypes.data, rms.ctypes.data)
+    return s, rms
+
+
 def featmap(params, X) -> np.ndarray:
-    """phi(X) for rows of X (..., d) -> (..., M*L), feature index i*L + l."""
+    """phi(X) for rows of X (..., d) -> (..., M*L), feature index i*L + l.  With channel
+    RMS normalisation the statistics are those of all rows of X."""
     p = _as_params(params)
     X = _f64(X)
     rows = X.size // p.d

@@ -26,6 +26,11 @@
  *   - the listing's shared_channels variant: one scalar MLP with L outputs
  *     (fc1: 1 -> hid shared by the channels, fc2: hid -> L), so channel l
  *     reads the same hidden units with its own fc2 row.
+ *   - the listing's ch_rms channel normalisation: per call of the feature map
+ *     (once over Q, once over K), every channel's MLP outputs are scaled by
+ *     s_l = min(target / (rms_l + 1e-6), 1), rms_l = sqrt(mean y_l^2 + 1e-6)
+ *     over every valid row and projection of that call's input; the backward
+ *     pass carries the dependence of s_l on every output of the channel.
  *
  * Parity pinned by the CPU tests: hand-computed feature maps, the brute-force
  * quadratic form, closed-form special cases (constant channels give a plain
@@ -52,6 +57,8 @@ typedef struct {
     const double *w2; /* L x hid, fc2 weight of channel l (fan-out 1)    */
     const double *b2; /* L                                               */
     int shared;       /* 1: one MLP for all channels (fc1 shared)        */
+    double ch_rms_target; /* > 0: channel RMS normalisation to this target */
+    const double *chs;    /* per-channel scales s_l in effect (NULL: 1); set per input by the callers */
 } oracle_phi;
 
 /* offset of channel l's fc1 row (the one shared row when shared) */
@@ -98,19 +105,70 @@ static double channel_pre(const oracle_phi *p, int l, double u) {
 
 double oracle_psi(const oracle_phi *p, int l, double u) { return relu(channel_pre(p, l, u)); }
 
-/* phi(x) = (1/sqrt(M)) [psi_l(w_i^T x + b_i)]_{i,l},  index i*L + l */
+/* phi(x) = (1/sqrt(M)) [s_l psi_l(w_i^T x + b_i)]_{i,l},  index i*L + l (s_l = 1 without ch_rms) */
 static void phi_row(const oracle_phi *p, const double *x, double *out) {
     const double s = 1.0 / sqrt((double)p->M);
     for (int i = 0; i < p->M; ++i) {
         double u = project(p, i, x);
-        for (int l = 0; l < p->L; ++l) out[i * p->L + l] = s * relu(channel_pre(p, l, u));
+        for (int l = 0; l < p->L; ++l)
+            out[i * p->L + l] = s * (p->chs ? p->chs[l] : 1.0) * relu(channel_pre(p, l, u));
     }
 }
 
-void oracle_featmap(const oracle_phi *p, const double *X, int64_t rows, double *Phi) {
-    const int D = p->M * p->L;
+static int head_len(const int32_t *lengths, int b, int n);
+
+/* Channel RMS statistics of one input X (B x H x n rows of width d; rows at or
+ * past a sequence's length excluded): rms_l = sqrt(mean y_l^2 + 1e-6) over
+ * every valid row and projection of the MLP outputs y_l = psi_l(u), the scale
+ * s_l = min(target / (rms_l + 1e-6), 1), and the sample count N = rows x M.
+ * The sums are taken head by head and added in head order. */
+#define CH_RMS_EPS 1e-6
+static void ch_rms_scales(const oracle_phi *p, const double *X, int B, int H, int n, const int32_t *lengths,
+                          double *s, double *rms, double *count) {
+    const int L = p->L, d = p->d, BH = B * H;
+    double *part = (double *)calloc((size_t)(BH > 0 ? BH : 1) * L, sizeof(double));
+    double rows = 0.0;
+#pragma omp parallel for schedule(dynamic, 1)
+    for (int bh = 0; bh < BH; ++bh) {
+        const int len = head_len(lengths, bh / H, n);
+        for (int r = 0; r < len; ++r) {
+            const double *x = X + ((size_t)bh * n + r) * d;
+            for (int i = 0; i < p->M; ++i) {
+                const double u = project(p, i, x);
+                for (int l = 0; l < L; ++l) {
+                    const double y = relu(channel_pre(p, l, u));
+                    part[(size_t)bh * L + l] += y * y;
+                }
+            }
+        }
+    }
+    for (int bh = 0; bh < BH; ++bh) rows += head_len(lengths, bh / H, n);
+    *count = rows * p->M;
+    for (int l = 0; l < L; ++l) {
+        double sum = 0.0;
+        for (int bh = 0; bh < BH; ++bh) sum += part[(size_t)bh * L + l];
+        const double mean = *count > 0.0 ? sum / *count : 0.0;
+        rms[l] = sqrt(mean + CH_RMS_EPS);
+        const double r = p->ch_rms_target / (rms[l] + CH_RMS_EPS);
+        s[l] = r < 1.0 ? r : 1.0;
+    }
+    free(part);
+}
+
+void oracle_featmap(const oracle_phi *p0, const double *X, int64_t rows, double *Phi) {
+    const int D = p0->M * p0->L;
+    oracle_phi pc = *p0;
+    const oracle_phi *p = &pc;
+    double *sc = (double *)malloc(sizeof(double) * 3 * (size_t)p0->L);
+    pc.chs = NULL;
+    if (p0->ch_rms_target > 0.0) {  /* the statistics of this call's rows (all valid) */
+        double cnt;
+        ch_rms_scales(p0, X, 1, 1, (int)rows, NULL, sc, sc + p0->L, &cnt);
+        pc.chs = sc;
+    }
 #pragma omp parallel for schedule(static)
     for (int64_t r = 0; r < rows; ++r) phi_row(p, X + r * p->d, Phi + r * D);
+    free(sc);
 }
 
 /* Smallest relative distance of any ReLU argument of the feature map of a row
@@ -157,8 +215,12 @@ static int abs_terms = 0;
 void oracle_set_abs_terms(int on) { abs_terms = on ? 1 : 0; }
 static double term(double v) { return abs_terms ? fabs(v) : v; }
 
+/* With channel RMS normalisation (p->chs set), the gradient reaching the MLP
+ * output y_l = psi_l(u) of one sample is (1/sqrt(M)) s_l dPhi + kappa_l y_l:
+ * the first term through the scaled output, the second through s_l, which
+ * depends on every sample of the channel (kappa from ch_rms_kappa). */
 static void phi_rows_backward(const oracle_phi *p, const double *X, int64_t rows, const double *dPhi,
-                              double *dX, oracle_grads *g) {
+                              const double *kappa, double *dX, oracle_grads *g) {
     const int D = p->M * p->L, d = p->d;
     const double s = 1.0 / sqrt((double)p->M);
     for (int64_t r = 0; r < rows; ++r) {
@@ -172,6 +234,7 @@ static void phi_rows_backward(const oracle_phi *p, const double *X, int64_t rows
                 double y = channel_pre(p, l, u);
                 if (!(y > 0.0)) continue; /* outer ReLU inactive */
                 double dy = dPhi[r * D + i * p->L + l] * s;
+                if (p->chs) dy = dy * p->chs[l] + (kappa ? kappa[l] * y : 0.0);
                 if (dy == 0.0) continue;
                 const double *w1 = p->w1 + fc1_row(p, l);
                 const double *b1 = p->b1 + fc1_row(p, l);
@@ -207,9 +270,9 @@ static int head_len(const int32_t *lengths, int b, int n) {
 /* ------------------------------------------------------------------------ */
 /* forward, linear (sufficient-statistics) form                              */
 
-static void attn_fwd_head(const oracle_phi *p, int n, int dv, int causal, double eps, const double *Q,
-                          const double *K, const double *V, int len, double *O) {
-    const int D = p->M * p->L, d = p->d;
+static void attn_fwd_head(const oracle_phi *pq_, const oracle_phi *pk_, int n, int dv, int causal, double eps,
+                          const double *Q, const double *K, const double *V, int len, double *O) {
+    const int D = pq_->M * pq_->L, d = pq_->d;
     double *phq = (double *)malloc(sizeof(double) * D);
     double *phk = (double *)malloc(sizeof(double) * D);
     double *S = (double *)calloc((size_t)D * dv, sizeof(double));
@@ -217,7 +280,7 @@ static void attn_fwd_head(const oracle_phi *p, int n, int dv, int causal, double
     memset(O, 0, sizeof(double) * (size_t)n * dv);
     if (!causal) {
         for (int j = 0; j < len; ++j) {
-            phi_row(p, K + (size_t)j * d, phk);
+            phi_row(pk_, K + (size_t)j * d, phk);
             for (int f = 0; f < D; ++f) {
                 z[f] += phk[f];
                 for (int c = 0; c < dv; ++c) S[(size_t)f * dv + c] += phk[f] * V[(size_t)j * dv + c];
@@ -226,13 +289,13 @@ static void attn_fwd_head(const oracle_phi *p, int n, int dv, int causal, double
     }
     for (int i = 0; i < len; ++i) {
         if (causal) { /* S_i = S_{i-1} + phi(k_i) v_i^T, z_i likewise */
-            phi_row(p, K + (size_t)i * d, phk);
+            phi_row(pk_, K + (size_t)i * d, phk);
             for (int f = 0; f < D; ++f) {
                 z[f] += phk[f];
                 for (int c = 0; c < dv; ++c) S[(size_t)f * dv + c] += phk[f] * V[(size_t)i * dv + c];
             }
         }
-        phi_row(p, Q + (size_t)i * d, phq);
+        phi_row(pq_, Q + (size_t)i * d, phq);
         double den = eps;
         for (int f = 0; f < D; ++f) den += phq[f] * z[f];
         if (den == 0.0) continue;
@@ -245,15 +308,50 @@ static void attn_fwd_head(const oracle_phi *p, int n, int dv, int causal, double
     free(phq); free(phk); free(S); free(z);
 }
 
+/* The feature maps applied to the queries and to the keys: both p itself, or,
+ * with channel RMS normalisation, p with the scales of the statistics of all
+ * valid query rows (pq) and of all valid key rows (pk).  st holds, per side,
+ * s (L), rms (L) and the sample count N. */
+typedef struct {
+    oracle_phi pq, pk;
+    double *st;
+} side_maps;
+
+static void side_maps_init(side_maps *sm, const oracle_phi *p, const double *Q, const double *K, int B, int H,
+                           int n, const int32_t *lengths) {
+    const int L = p->L;
+    sm->pq = *p;
+    sm->pk = *p;
+    sm->pq.chs = sm->pk.chs = NULL;
+    sm->st = (double *)calloc(2 * (2 * (size_t)L + 1), sizeof(double));
+    if (p->ch_rms_target > 0.0) {
+        double *sq = sm->st, *sk = sm->st + 2 * L + 1;
+        ch_rms_scales(p, Q, B, H, n, lengths, sq, sq + L, sq + 2 * L);
+        ch_rms_scales(p, K, B, H, n, lengths, sk, sk + L, sk + 2 * L);
+        sm->pq.chs = sq;
+        sm->pk.chs = sk;
+    }
+}
+
 void oracle_attn_fwd(const oracle_phi *p, int B, int H, int n, int dv, int causal, double eps, const double *Q,
                      const double *K, const double *V, const int32_t *lengths, double *O) {
     const int d = p->d;
+    side_maps sm;
+    side_maps_init(&sm, p, Q, K, B, H, n, lengths);
 #pragma omp parallel for schedule(dynamic, 1)
     for (int bh = 0; bh < B * H; ++bh) {
         int b = bh / H;
         size_t qo = (size_t)bh * n * d, vo = (size_t)bh * n * dv;
-        attn_fwd_head(p, n, dv, causal, eps, Q + qo, K + qo, V + vo, head_len(lengths, b, n), O + vo);
+        attn_fwd_head(&sm.pq, &sm.pk, n, dv, causal, eps, Q + qo, K + qo, V + vo, head_len(lengths, b, n), O + vo);
     }
+    free(sm.st);
+}
+
+/* Channel RMS scales of the rows of X (B x H x n x d, valid rows only): s and rms (L each). */
+void oracle_ch_rms(const oracle_phi *p, const double *X, int B, int H, int n, const int32_t *lengths, double *s,
+                   double *rms) {
+    double cnt;
+    ch_rms_scales(p, X, B, H, n, lengths, s, rms, &cnt);
 }
 
 /* ------------------------------------------------------------------------ */
@@ -263,6 +361,8 @@ void oracle_attn_quadratic(const oracle_phi *p, int B, int H, int n, int dv, int
                            const double *Q, const double *K, const double *V, const int32_t *lengths,
                            double *O) {
     const int D = p->M * p->L, d = p->d;
+    side_maps sm;
+    side_maps_init(&sm, p, Q, K, B, H, n, lengths);
 #pragma omp parallel for schedule(dynamic, 1)
     for (int bh = 0; bh < B * H; ++bh) {
         int len = head_len(lengths, bh / H, n);
@@ -271,8 +371,8 @@ void oracle_attn_quadratic(const oracle_phi *p, int B, int H, int n, int dv, int
         double *PQ = (double *)malloc(sizeof(double) * (size_t)(len > 0 ? len : 1) * D);
         double *PK = (double *)malloc(sizeof(double) * (size_t)(len > 0 ? len : 1) * D);
         for (int i = 0; i < len; ++i) {
-            phi_row(p, q + (size_t)i * d, PQ + (size_t)i * D);
-            phi_row(p, k + (size_t)i * d, PK + (size_t)i * D);
+            phi_row(&sm.pq, q + (size_t)i * d, PQ + (size_t)i * D);
+            phi_row(&sm.pk, k + (size_t)i * d, PK + (size_t)i * D);
         }
         memset(o, 0, sizeof(double) * (size_t)n * dv);
         for (int i = 0; i < len; ++i) {
@@ -293,15 +393,16 @@ void oracle_attn_quadratic(const oracle_phi *p, int B, int H, int n, int dv, int
         }
         free(PQ); free(PK);
     }
+    free(sm.st);
 }
 
 /* ------------------------------------------------------------------------ */
 /* backward                                                                  */
 
-static void attn_bwd_head(const oracle_phi *p, int n, int dv, int causal, double eps, const double *Q,
-                          const double *K, const double *V, const double *dO, int len, double *dQ, double *dK,
-                          double *dV, oracle_grads *g) {
-    const int D = p->M * p->L, d = p->d;
+static void attn_bwd_head(const oracle_phi *pq_, const oracle_phi *pk_, int n, int dv, int causal, double eps,
+                          const double *Q, const double *K, const double *V, const double *dO, int len, double *dQ,
+                          double *dK, double *dV, oracle_grads *g, double *dPQ_out, double *dPK_out) {
+    const int D = pq_->M * pq_->L, d = pq_->d;
     size_t nl = (size_t)(len > 0 ? len : 1);
     double *PQ = (double *)malloc(sizeof(double) * nl * D);
     double *PK = (double *)malloc(sizeof(double) * nl * D);
@@ -316,8 +417,8 @@ static void attn_bwd_head(const oracle_phi *p, int n, int dv, int causal, double
     memset(dK, 0, sizeof(double) * (size_t)n * d);
     memset(dV, 0, sizeof(double) * (size_t)n * dv);
     for (int i = 0; i < len; ++i) {
-        phi_row(p, Q + (size_t)i * d, PQ + (size_t)i * D);
-        phi_row(p, K + (size_t)i * d, PK + (size_t)i * D);
+        phi_row(pq_, Q + (size_t)i * d, PQ + (size_t)i * D);
+        phi_row(pk_, K + (size_t)i * d, PK + (size_t)i * D);
     }
     if (!causal) {
         for (int j = 0; j < len; ++j)
@@ -383,8 +484,13 @@ static void attn_bwd_head(const oracle_phi *p, int n, int dv, int causal, double
             dPK[(size_t)j * D + f] = acc;
         }
     }
-    phi_rows_backward(p, Q, len, dPQ, dQ, g);
-    phi_rows_backward(p, K, len, dPK, dK, g);
+    if (dPQ_out) {  /* channel RMS normalisation: the caller finishes the chain rule */
+        memcpy(dPQ_out, dPQ, sizeof(double) * (size_t)len * D);
+        memcpy(dPK_out, dPK, sizeof(double) * (size_t)len * D);
+    } else {
+        phi_rows_backward(pq_, Q, len, dPQ, NULL, dQ, g);
+        phi_rows_backward(pk_, K, len, dPK, NULL, dK, g);
+    }
     free(PQ); free(PK); free(dPQ); free(dPK); free(dnum); free(dden); free(S); free(z); free(o);
 }
 
@@ -395,17 +501,76 @@ void oracle_attn_bwd(const oracle_phi *p, int B, int H, int n, int dv, int causa
     const int d = p->d, M = p->M, L = p->L, hid = p->hid;
     const size_t nW = (size_t)M * d, nb = M, nh = (size_t)L * hid, nb2 = L;
     const size_t per = nW + nb + 3 * nh + nb2;
-    const int BH = B * H;
-    double *part = (double *)calloc((size_t)BH * per, sizeof(double));
+    const int BH = B * H, D = M * L;
+    double *part = (double *)calloc((size_t)(BH > 0 ? BH : 1) * per, sizeof(double));
+    side_maps sm;
+    side_maps_init(&sm, p, Q, K, B, H, n, lengths);
+    const int norm = p->ch_rms_target > 0.0;
+    /* with channel RMS normalisation: dPhi of every valid row of both sides, kept for the second phase */
+    double *dPQ = NULL, *dPK = NULL;
+    if (norm) {
+        dPQ = (double *)calloc((size_t)(BH > 0 ? BH : 1) * n * D, sizeof(double));
+        dPK = (double *)calloc((size_t)(BH > 0 ? BH : 1) * n * D, sizeof(double));
+    }
 #pragma omp parallel for schedule(dynamic, 1)
     for (int bh = 0; bh < BH; ++bh) {
         double *base = part + (size_t)bh * per;
         oracle_grads g = {base, base + nW, base + nW + nb, base + nW + nb + nh, base + nW + nb + 2 * nh,
                           base + nW + nb + 3 * nh};
-        size_t qo = (size_t)bh * n * d, vo = (size_t)bh * n * dv;
-        attn_bwd_head(p, n, dv, causal, eps, Q + qo, K + qo, V + vo, dO + vo, head_len(lengths, bh / H, n),
-                      dQ + qo, dK + qo, dV + vo, &g);
+        size_t qo = (size_t)bh * n * d, vo = (size_t)bh * n * dv, po = (size_t)bh * n * D;
+        attn_bwd_head(&sm.pq, &sm.pk, n, dv, causal, eps, Q + qo, K + qo, V + vo, dO + vo,
+                      head_len(lengths, bh / H, n), dQ + qo, dK + qo, dV + vo, &g, norm ? dPQ + po : NULL,
+                      norm ? dPK + po : NULL);
     }
+    if (norm) {
+        /* kappa_l = ds_l/drms_l * drms_l/dy (without the factor y) * A_l per side, where
+         * A_l = sum over valid rows t and projections i of (1/sqrt(M)) dPhi_{t,i,l} y_{t,i,l};
+         * s_l = target/(rms_l + eps) has ds/drms = -target/(rms_l + eps)^2 where not clamped,
+         * and drms_l/dy = y/(N rms_l). */
+        const double c = 1.0 / sqrt((double)M);
+        double *A = (double *)calloc((size_t)(BH > 0 ? BH : 1) * 2 * L, sizeof(double));
+        double *kappa = (double *)calloc(2 * (size_t)L, sizeof(double));
+#pragma omp parallel for schedule(dynamic, 1)
+        for (int bh = 0; bh < BH; ++bh) {
+            const int len = head_len(lengths, bh / H, n);
+            for (int side = 0; side < 2; ++side) {
+                const double *X = (side ? K : Q) + (size_t)bh * n * d;
+                const double *dP = (side ? dPK : dPQ) + (size_t)bh * n * D;
+                double *a = A + ((size_t)bh * 2 + side) * L;
+                for (int r = 0; r < len; ++r)
+                    for (int i = 0; i < M; ++i) {
+                        const double u = project(p, i, X + (size_t)r * d);
+                        for (int l = 0; l < L; ++l)
+                            a[l] += c * dP[(size_t)r * D + i * L + l] * relu(channel_pre(p, l, u));
+                    }
+            }
+        }
+        for (int side = 0; side < 2; ++side) {
+            const double *st = sm.st + side * (2 * (size_t)L + 1);
+            const double N = st[2 * L];
+            for (int l = 0; l < L; ++l) {
+                double a = 0.0;
+                for (int bh = 0; bh < BH; ++bh) a += A[((size_t)bh * 2 + side) * L + l];
+                const double rms = st[L + l];
+                const double r = p->ch_rms_target / (rms + CH_RMS_EPS);
+                kappa[side * L + l] = (N > 0.0 && r <= 1.0)
+                                     ? -p->ch_rms_target / ((rms + CH_RMS_EPS) * (rms + CH_RMS_EPS)) / (N * rms) * a
+                                     : 0.0;
+            }
+        }
+#pragma omp parallel for schedule(dynamic, 1)
+        for (int bh = 0; bh < BH; ++bh) {
+            double *base = part + (size_t)bh * per;
+            oracle_grads g = {base, base + nW, base + nW + nb, base + nW + nb + nh, base + nW + nb + 2 * nh,
+                              base + nW + nb + 3 * nh};
+            const int len = head_len(lengths, bh / H, n);
+            size_t qo = (size_t)bh * n * d, po = (size_t)bh * n * D;
+            phi_rows_backward(&sm.pq, Q + qo, len, dPQ + po, kappa, dQ + qo, &g);
+            phi_rows_backward(&sm.pk, K + qo, len, dPK + po, kappa + L, dK + qo, &g);
+        }
+        free(A); free(kappa); free(dPQ); free(dPK);
+    }
+    free(sm.st);
     /* ordered reduction over heads (fc1 gradients: hid entries when the MLP is shared) */
     double *outs[6] = {dW, db, dw1, db1, dw2, db2};
     const size_t n1 = p->shared ? (size_t)hid : nh;

@@ -1,5 +1,6 @@
 """The oracle pins are sensitive: plausible mistakes planted in a temporary
-copy of the oracle source (on the CPU) make at least one pin fail."""
+copy of the oracle source (on the CPU) make at least one pin fail.  Mistakes
+in the channel RMS normalisation are checked against its own pin file."""
 import os
 import shutil
 import subprocess
@@ -31,11 +32,29 @@ MUTANTS = {
         "g->dw1[fc1_row(p, l) + k] += term(dh * u);", "g->dw1[(size_t)l * p->hid + k] += term(dh * u);"),
 }
 
+CH_RMS_PINS = "tests/test_oracle_ch_rms.py"
+CH_RMS_MUTANTS = {
+    "channel RMS: scale term dropped from the backward": (
+        "if (p->chs) dy = dy * p->chs[l] + (kappa ? kappa[l] * y : 0.0);", "if (p->chs) dy = dy * p->chs[l];"),
+    "channel RMS: mean over rows only": ("*count = rows * p->M;", "*count = rows;"),
+    "channel RMS: scale not clamped at 1": ("s[l] = r < 1.0 ? r : 1.0;", "s[l] = r;"),
+    "channel RMS: padded rows in the statistics": (
+        "for (int bh = 0; bh < BH; ++bh) rows += head_len(lengths, bh / H, n);\n    *count",
+        "for (int bh = 0; bh < BH; ++bh) rows += n;\n    *count"),
+    "channel RMS: key statistics taken from the queries": (
+        "ch_rms_scales(p, K, B, H, n, lengths, sk, sk + L, sk + 2 * L);",
+        "ch_rms_scales(p, Q, B, H, n, lengths, sk, sk + L, sk + 2 * L);"),
+    "channel RMS: sign of the scale derivative": (
+        "? -p->ch_rms_target / ((rms + CH_RMS_EPS) * (rms + CH_RMS_EPS)) / (N * rms) * a",
+        "? p->ch_rms_target / ((rms + CH_RMS_EPS) * (rms + CH_RMS_EPS)) / (N * rms) * a"),
+}
 
-@pytest.mark.parametrize("name", sorted(MUTANTS))
+
+@pytest.mark.parametrize("name", sorted(MUTANTS) + sorted(CH_RMS_MUTANTS))
 def test_planted_mistake_is_caught(name, tmp_path):
     src = open(os.path.join(ROOT, "oracle", "luna_oracle.c")).read()
-    a, b = MUTANTS[name]
+    a, b = MUTANTS[name] if name in MUTANTS else CH_RMS_MUTANTS[name]
+    pins = CH_RMS_PINS if name in CH_RMS_MUTANTS else "tests/test_oracle_pins.py"
     assert a in src, f"mutation site for {name!r} not found"
     work = tmp_path / "w"
     shutil.copytree(os.path.join(ROOT, "oracle"), work / "oracle", ignore=shutil.ignore_patterns("_build", "__pycache__"))
@@ -43,5 +62,5 @@ def test_planted_mistake_is_caught(name, tmp_path):
     shutil.copytree(os.path.join(ROOT, "tests"), work / "tests", ignore=shutil.ignore_patterns("__pycache__"))
     (work / "oracle" / "luna_oracle.c").write_text(src.replace(a, b, 1))
     r = subprocess.run([sys.executable, "-m", "pytest", "-q", "-x", "-p", "no:cacheprovider",
-                        "tests/test_oracle_pins.py"], cwd=str(work), capture_output=True, text=True, timeout=600)
+                        pins], cwd=str(work), capture_output=True, text=True, timeout=600)
     assert r.returncode != 0, f"mutant {name!r} survived the pins:\n{r.stdout[-2000:]}"
