@@ -66,12 +66,23 @@ typedef enum { LUNA_F32 = 0, LUNA_BF16 = 1 } luna_dtype;
  * shared_channels = 0: one scalar MLP per channel (the listing's default);
  * 1: one scalar MLP with L outputs serves all channels (the listing's
  * shared_channels = True: fc1 Linear(1, hidden) shared, fc2 Linear(hidden, L)).
+ * ch_rms_target > 0 turns on the listing's channel RMS normalisation
+ * (ch_rms): each application of the feature map, once to all queries and once
+ * to all keys of the batch, scales channel l of the MLP outputs y_l by
+ * s_l = min(target / (rms_l + 1e-6), 1), rms_l = sqrt(mean y_l^2 + 1e-6) over
+ * every valid row (rows at or past a sequence's length excluded) and every
+ * projection; the backward pass includes the dependence of s_l on every
+ * sample.  0 = off (the listing's default); negative, NaN or infinite is
+ * LUNA_ERR_INVALID_ARG.  With it on, only the non-causal luna_attn_fwd /
+ * luna_attn_bwd are supported (the causal form, luna_featmap and
+ * luna_attn_decode give LUNA_ERR_UNSUPPORTED).
  * Supported: 1 <= M, 1 <= L <= 16, M*L <= 128, 1 <= hidden <= 128, L*hidden <= 512. */
 typedef struct {
     int M;               /* number of projections w_i (rows of W)       */
     int L;               /* number of channel functions psi_l           */
     int hidden;          /* hidden width of each (or the shared) MLP     */
     int shared_channels; /* 0 or 1, see above                           */
+    float ch_rms_target; /* channel RMS normalisation target, 0 = off   */
 } luna_phi_desc;
 
 /* Feature-map parameters, fp32 device arrays, row-major:

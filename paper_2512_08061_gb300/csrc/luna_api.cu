@@ -21,6 +21,7 @@ luna_status check_phi(const luna_phi_desc *pd, int d) {
     if (!pd) return LUNA_ERR_INVALID_ARG;
     if (pd->M < 1 || pd->L < 1 || pd->hidden < 1 || d < 1) return LUNA_ERR_INVALID_ARG;
     if (pd->shared_channels != 0 && pd->shared_channels != 1) return LUNA_ERR_INVALID_ARG;
+    if (!(pd->ch_rms_target >= 0.0f) || isinf(pd->ch_rms_target)) return LUNA_ERR_INVALID_ARG;
     if (pd->L > kMaxL || pd->M * pd->L > kMaxFeat || pd->M > 32 || pd->hidden > kMaxHidden ||
         pd->L * pd->hidden > kMaxUnits || d > kMaxD || pd->M * d > 4096)
         return LUNA_ERR_UNSUPPORTED;
@@ -39,6 +40,8 @@ struct Plan {
     size_t o_segS = 0, o_segz = 0, o_segdS = 0, o_segdz = 0, o_rowstat = 0;
     size_t o_dphi = 0, o_phik = 0, o_pq2 = 0;  // streaming-form backward on tensor cores
     size_t o_items = 0;                        // split of the tensor-core work items (non-causal)
+    float ch_target = 0.0f;                    // channel RMS normalisation (non-causal; 0: off)
+    size_t o_chpart = 0, o_chstat = 0, o_chsigma = 0, o_chkappa = 0, o_chT = 0;
     size_t ws_fwd = 0, ws_bwd = 0, state_bytes = 0;
     TcPlan tc;
 };
@@ -62,6 +65,8 @@ luna_status make_plan(const luna_attn_desc *ad, const luna_phi_desc *pd, Plan &p
     luna_status st = check_phi(pd, ad->d);
     if (st != LUNA_OK) return st;
     if (ad->dv > kMaxD || ad->n > (1 << 24)) return LUNA_ERR_UNSUPPORTED;
+    if (pd->ch_rms_target > 0.0f && ad->causal) return LUNA_ERR_UNSUPPORTED;  // non-causal form only
+    p.ch_target = pd->ch_rms_target;
     if ((int64_t)ad->B * ad->H > (1 << 24)) return LUNA_ERR_UNSUPPORTED;
 
     p.lay = table_layout(pd->M, pd->L, pd->hidden, ad->d, pd->shared_channels);
@@ -98,6 +103,13 @@ luna_status make_plan(const luna_attn_desc *ad, const luna_phi_desc *pd, Plan &p
         p.o_Sfin = w.take((size_t)BH * SD * f);
         p.o_zfin = w.take((size_t)BH * D * f);
         p.o_items = w.take((kMaxGrid + 1 + 2 * (size_t)BH) * sizeof(int));
+        if (p.ch_target > 0.0f) {
+            p.o_chpart = w.take(2 * (size_t)BH * p.nsplit_b * p.lay.L * f);
+            p.o_chstat = w.take(8 * (size_t)kMaxL * sizeof(double));
+            p.o_chsigma = w.take((size_t)kMaxL * f);
+            p.o_chkappa = w.take(2 * (size_t)kMaxL * f);
+            p.o_chT = w.take((size_t)BH * p.lay.L * sizeof(double));
+        }
         p.ws_fwd = w.n;
         // per-head partial slots: generic splits, or (tensor-core path) runs of work items, never more
         // than the forward split count
@@ -106,7 +118,8 @@ luna_status make_plan(const luna_attn_desc *ad, const luna_phi_desc *pd, Plan &p
         p.o_dzpart = w.take((size_t)BH * nslot * D * f);
         p.o_dSfin = w.take((size_t)BH * SD * f);
         p.o_dzfin = w.take((size_t)BH * D * f);
-        p.o_gpart = w.take(2 * (size_t)BH * p.nsplit_b * p.gsize * f);
+        // with channel normalisation, as many partials again for the scale term of the backward
+        p.o_gpart = w.take((p.ch_target > 0.0f ? 4 : 2) * (size_t)BH * p.nsplit_b * p.gsize * f);
         p.o_hist = w.take((size_t)p.gsize * f);
         p.ws_bwd = w.n;
         p.state_bytes = (size_t)BH * (SD + D) * f;
@@ -168,6 +181,15 @@ AttnArgs make_args(const luna_attn_desc *ad, const Plan &p, const void *table, c
         a.S_fin = reinterpret_cast<float *>(w + p.o_Sfin);
         a.z_fin = reinterpret_cast<float *>(w + p.o_zfin);
         a.items_ws = reinterpret_cast<int *>(w + p.o_items);
+        if (p.ch_target > 0.0f) {
+            a.ch_target = p.ch_target;
+            a.ch_io = ad->io;
+            a.ch_part = reinterpret_cast<float *>(w + p.o_chpart);
+            a.ch_stat = reinterpret_cast<double *>(w + p.o_chstat);
+            a.ch_sigma = reinterpret_cast<float *>(w + p.o_chsigma);
+            a.ch_kappa = reinterpret_cast<float *>(w + p.o_chkappa);
+            a.ch_T = reinterpret_cast<double *>(w + p.o_chT);
+        }
     } else {
         a.seg_S = reinterpret_cast<float *>(w + p.o_segS);
         a.seg_z = reinterpret_cast<float *>(w + p.o_segz);
@@ -235,6 +257,7 @@ luna_status luna_featmap(const luna_phi_desc *pd, int d, const void *table, cons
     luna_status st = check_phi(pd, d);
     if (st != LUNA_OK) return st;
     if (rows < 0 || (xtype != LUNA_F32 && xtype != LUNA_BF16)) return LUNA_ERR_INVALID_ARG;
+    if (pd->ch_rms_target > 0.0f) return LUNA_ERR_UNSUPPORTED;
     if (rows == 0) return LUNA_OK;
     if (!table || !X || !Phi) return LUNA_ERR_INVALID_ARG;
     TableLayout lay = table_layout(pd->M, pd->L, pd->hidden, d, pd->shared_channels);
@@ -278,8 +301,10 @@ luna_status luna_attn_fwd(const luna_attn_desc *ad, const luna_phi_desc *pd, con
     point_state(ad, p, a, state);
     if ((!ad->causal ? simt_max_smem(a) : causal_max_smem(a)) > kMaxSmem && !p.tc.eligible)
         return LUNA_ERR_UNSUPPORTED;
+    if (a.ch_sigma && chrms_max_smem(a) > kMaxSmem) return LUNA_ERR_UNSUPPORTED;
     cudaError_t e = cudaMemsetAsync(workspace, 0, p.o_counters + 2 * sizeof(int) * (size_t)p.BH, s);
     if (e != cudaSuccess) return LUNA_ERR_CUDA;
+    if (a.ch_sigma && (e = launch_chrms_stats(a, ad->io, s)) != cudaSuccess) return LUNA_ERR_CUDA;
     if (ad->causal) {
         if (p.tc.causal_fwd && tc_inputs_ok(TcPlan{true}, Q, K, V, O)) return cuda_status(launch_tc_causal_fwd(a, s));
         return cuda_status(launch_causal_fwd(a, ad->io, state != nullptr, s));
@@ -333,8 +358,10 @@ luna_status luna_attn_bwd(const luna_attn_desc *ad, const luna_phi_desc *pd, con
     point_state(ad, p, a, const_cast<void *>(state));
     if ((!ad->causal ? simt_max_smem(a) : causal_max_smem(a)) > kMaxSmem && !p.tc.eligible)
         return LUNA_ERR_UNSUPPORTED;
+    if (a.ch_sigma && chrms_max_smem(a) > kMaxSmem) return LUNA_ERR_UNSUPPORTED;
     cudaError_t e = cudaMemsetAsync(workspace, 0, p.o_counters + 2 * sizeof(int) * (size_t)p.BH, s);
     if (e != cudaSuccess) return LUNA_ERR_CUDA;
+    if (a.ch_sigma && (e = launch_chrms_stats(a, ad->io, s)) != cudaSuccess) return LUNA_ERR_CUDA;
     if (ad->causal) {
         if (p.tc.causal_bwd && tc_inputs_ok(TcPlan{true}, Q, K, V, dO) && tc_inputs_ok(TcPlan{true}, dQ, dK, dV, nullptr)) {
             a.dphi = reinterpret_cast<float *>(w + p.o_dphi);
@@ -376,6 +403,7 @@ luna_status luna_attn_decode(const luna_attn_desc *ad, const luna_phi_desc *pd, 
     luna_status st = check_phi(pd, ad->d);
     if (st != LUNA_OK) return st;
     if (ad->dv > kMaxD) return LUNA_ERR_UNSUPPORTED;
+    if (pd->ch_rms_target > 0.0f) return LUNA_ERR_UNSUPPORTED;  // a batch statistic: no single-token step
     const int64_t BH = (int64_t)ad->B * ad->H;
     if (BH > (1 << 24)) return LUNA_ERR_UNSUPPORTED;
     const TableLayout lay = table_layout(pd->M, pd->L, pd->hidden, ad->d, pd->shared_channels);

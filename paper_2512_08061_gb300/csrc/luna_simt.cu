@@ -492,7 +492,8 @@ cudaError_t stats_impl(const AttnArgs &a, cudaStream_t s) {
     cudaError_t e = set_smem(k_keystats<IO>, sm);
     if (e != cudaSuccess) return e;
     LUNA_LAUNCH("keystats", k_keystats<IO>, dim3(a.nsplit, a.B * a.H), kThreads, sm, s, a);
-    return cudaGetLastError();
+    if ((e = cudaGetLastError()) != cudaSuccess) return e;
+    return launch_chrms_scale_state(a, s);
 }
 
 template <typename IO>
@@ -513,11 +514,14 @@ cudaError_t bwd_impl(const AttnArgs &a, bool have_stats, cudaStream_t s) {
     if ((e = set_smem(k_bwd_query<IO>, sm)) != cudaSuccess) return e;
     LUNA_LAUNCH("bwd_query", k_bwd_query<IO>, dim3(a.nsplit_b, a.B * a.H), kThreads, sm, s, a);
     if ((e = cudaGetLastError()) != cudaSuccess) return e;
+    if ((e = launch_chrms_dstate(a, s)) != cudaSuccess) return e;
     sm = smem_bwd_key(a);
     if ((e = set_smem(k_bwd_key<IO>, sm)) != cudaSuccess) return e;
     LUNA_LAUNCH("bwd_key", k_bwd_key<IO>, dim3(a.nsplit_b, a.B * a.H), kThreads, sm, s, a);
     if ((e = cudaGetLastError()) != cudaSuccess) return e;
-    return launch_grad_reduce(a, 2 * a.B * a.H * a.nsplit_b, s);
+    int nparts = 0;
+    if ((e = launch_chrms_backward(a, 2 * a.B * a.H * a.nsplit_b, &nparts, s)) != cudaSuccess) return e;
+    return launch_grad_reduce(a, nparts, s);
 }
 
 }  // namespace

@@ -39,6 +39,14 @@ struct AttnArgs {
     const int *split;                  // block b takes items split[b] .. split[b+1]-1
     const int *runs;                   // [2*BH]: first and last block holding an item of head bh
     int padded_zeroed;                 // the outputs' rows past each sequence's length are already zero
+    // channel RMS normalisation of the feature map (non-causal; ch_sigma null: off)
+    float ch_target;                   // the listing's ch_rms_target
+    luna_dtype ch_io;                  // element type of Q, K, dQ, dK
+    float *ch_part;                    // [2][BH * nsplit_b][L]: per-block sums of phi^2, queries then keys
+    double *ch_stat;                   // [8][kMaxL]: per side s, rms, target/(rms+eps), unused; [3][0] = N
+    float *ch_sigma;                   // [kMaxL]: s^q_l s^k_l
+    double *ch_T;                      // [BH][L]: per-head sums of S' . dS + z' dz over each channel's rows
+    float *ch_kappa;                   // [2][kMaxL]: factor of y_l in dLoss/dy_l from the scale, per side
 };
 
 // one step of the streaming form for every (batch, head): state S [D][dv], z [D] (fp32, in place)
@@ -65,6 +73,15 @@ cudaError_t launch_grad_reduce(const AttnArgs &a, int nparts, cudaStream_t s);
 cudaError_t launch_causal_fwd(const AttnArgs &a, luna_dtype io, bool write_state, cudaStream_t s);
 cudaError_t launch_causal_bwd(const AttnArgs &a, luna_dtype io, bool have_state, cudaStream_t s);
 size_t simt_max_smem(const AttnArgs &a);
+// channel RMS normalisation: statistics and scales of both sides; S, z rows times sigma (after any key
+// statistics); dS, dz rows times sigma and the per-head sums T (between the query- and key-side backward
+// kernels); the scale term of the backward (before the parameter-gradient reduction: its partials follow
+// the main_parts ones, *nparts is the new count).  Each is a no-op when ch_sigma is null.
+cudaError_t launch_chrms_stats(const AttnArgs &a, luna_dtype io, cudaStream_t s);
+cudaError_t launch_chrms_scale_state(const AttnArgs &a, cudaStream_t s);
+cudaError_t launch_chrms_dstate(const AttnArgs &a, cudaStream_t s);
+cudaError_t launch_chrms_backward(const AttnArgs &a, int main_parts, int *nparts, cudaStream_t s);
+size_t chrms_max_smem(const AttnArgs &a);
 size_t causal_max_smem(const AttnArgs &a);
 
 }  // namespace luna

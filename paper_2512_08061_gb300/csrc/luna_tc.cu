@@ -872,6 +872,7 @@ cudaError_t fwd_tc(const AttnArgs &a0, cudaStream_t s) {
     const AttnArgs a = balanced_impl(a0, s, &e, 1);  // the query pass writes O
     if (e != cudaSuccess) return e;
     if ((e = keys_tc<C>(a, s)) != cudaSuccess) return e;
+    if ((e = launch_chrms_scale_state(a, s)) != cudaSuccess) return e;
     CUtensorMap mQ;
     if (!make_map_impl(&mQ, a.Q, a.d, a.n, a.B * a.H)) return cudaErrorInvalidValue;
     e = cudaFuncSetAttribute(k_tc_query<C>, cudaFuncAttributeMaxDynamicSharedMemorySize, C::SMEM_Q);
@@ -951,11 +952,13 @@ cudaError_t launch_tc_stats(const AttnArgs &a0, cudaStream_t s) {
     const AttnArgs a = balanced_impl(a0, s, &e, 0);  // the split of the forward pass: the same sums in the same order
     if (e != cudaSuccess) return e;
     switch (p.variant) {
-        case 0: return keys_tc<C32>(a, s);
-        case 1: return keys_tc<C64>(a, s);
-        case 2: return keys_tc<C128>(a, s);
+        case 0: e = keys_tc<C32>(a, s); break;
+        case 1: e = keys_tc<C64>(a, s); break;
+        case 2: e = keys_tc<C128>(a, s); break;
+        default: return cudaErrorNotSupported;
     }
-    return cudaErrorNotSupported;
+    if (e != cudaSuccess) return e;
+    return launch_chrms_scale_state(a, s);
 }
 
 cudaError_t launch_tc_bwd(const TcPlan &p, const AttnArgs &a, char *, bool have_stats, cudaStream_t s) {

@@ -918,9 +918,12 @@ cudaError_t bwd_tc(const AttnArgs &a0, bool have_stats, cudaStream_t s) {
     int *st = reinterpret_cast<int *>(reinterpret_cast<char *>(a.counters) - 256);
     LUNA_LAUNCH("tc_bwd_query", k_tc_bwd_query<C>, grid, kBThreads, C::SMEM_Q, s, mQ, mdO, a, st);
     if ((e = cudaGetLastError()) != cudaSuccess) return e;
+    if ((e = launch_chrms_dstate(a, s)) != cudaSuccess) return e;
     LUNA_LAUNCH("tc_bwd_key", k_tc_bwd_key<C>, grid, kBThreads, C::SMEM_K, s, mK, mV, a, st);
     if ((e = cudaGetLastError()) != cudaSuccess) return e;
-    return launch_grad_reduce(a, 2 * grid, s);
+    int nparts = 0;
+    if ((e = launch_chrms_backward(a, 2 * grid, &nparts, s)) != cudaSuccess) return e;
+    return launch_grad_reduce(a, nparts, s);
 }
 
 }  // namespace

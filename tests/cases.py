@@ -73,8 +73,9 @@ def to_host(x) -> np.ndarray:
 
 class Case:
     def __init__(self, B, H, n, d, M, L, io, causal=False, seed=0, qkv_scale=1.0, len_range=None, hidden=64,
-                 eps=1e-6, dv=None, with_grad=False, lengths=None, shared=False):
+                 eps=1e-6, dv=None, with_grad=False, lengths=None, shared=False, ch_rms_target=0.0):
         self.B, self.H, self.n, self.d, self.M, self.L = B, H, n, d, M, L
+        self.ch_rms_target = ch_rms_target
         self.dv = dv or d
         self.io, self.causal, self.eps, self.hidden, self.shared = io, causal, eps, hidden, shared
         self.params = synth.phi_params(seed, d, M, L, hidden, shared)
@@ -88,7 +89,8 @@ class Case:
         import torch
         import paper_2512_08061_gb300.luna as L
         lu = L.Luna(self.B, self.H, self.n, self.d, self.dv, self.M, self.L, self.hidden, self.causal, self.eps,
-                    torch.float32 if self.io == "f32" else torch.bfloat16, chunk, shared=self.shared)
+                    torch.float32 if self.io == "f32" else torch.bfloat16, chunk, shared=self.shared,
+                    ch_rms_target=self.ch_rms_target)
         params = {k: torch.from_numpy(v).cuda() for k, v in self.params.items()}
         lu.prepare(params)
         self.dev = {k: to_device(self.inp[k]) for k in ("Q", "K", "V", "dO") if k in self.inp}
@@ -104,19 +106,24 @@ class Case:
         return lu.backward(d["Q"], d["K"], d["V"], d["dO"], d["lengths"], use_state=use_state)
 
     # ---- oracle side
+    @property
+    def phi(self):
+        """The oracle's feature map: the parameters, with the channel normalisation when it is on."""
+        return oracle.PhiParams(self.params, self.ch_rms_target) if self.ch_rms_target else self.params
+
     def oracle_fwd(self):
         i = self.inp
-        return oracle.attn_fwd(self.params, i["Q"].value, i["K"].value, i["V"].value, self.lengths, self.causal,
+        return oracle.attn_fwd(self.phi, i["Q"].value, i["K"].value, i["V"].value, self.lengths, self.causal,
                                self.eps)
 
     def oracle_bwd(self):
         i = self.inp
-        return oracle.attn_bwd(self.params, i["Q"].value, i["K"].value, i["V"].value, i["dO"].value, self.lengths,
+        return oracle.attn_bwd(self.phi, i["Q"].value, i["K"].value, i["V"].value, i["dO"].value, self.lengths,
                                self.causal, self.eps)
 
     def oracle_bwd_abs_terms(self):
         i = self.inp
-        return oracle.attn_bwd_abs_terms(self.params, i["Q"].value, i["K"].value, i["V"].value, i["dO"].value,
+        return oracle.attn_bwd_abs_terms(self.phi, i["Q"].value, i["K"].value, i["V"].value, i["dO"].value,
                                          self.lengths, self.causal, self.eps)
 
     def smooth_rows(self, which: str) -> np.ndarray:

@@ -492,3 +492,47 @@ def test_shared_channel_featmap():
     Phi = torch.empty(777, M * 8, dtype=torch.float32, device="cuda")
     L.luna_featmap(pd, d, table, to_device(X), Phi)
     assert relerr(to_host(Phi), oracle.featmap(params, X.value)) < 1e-4
+
+
+def _median_channel_rms(case):
+    """A target between the channels' RMS values: some channels clamped, some not."""
+    p = oracle.PhiParams(case.params, 1.0)
+    rq = oracle.ch_rms(p, case.inp["Q"].value, case.lengths)[1]
+    rk = oracle.ch_rms(p, case.inp["K"].value, case.lengths)[1]
+    return float(np.median(np.concatenate([rq, rk])))
+
+
+@pytest.mark.parametrize("io,d,M,lengths", [("bf16", 32, 8, [300, 177]), ("bf16", 64, 8, None),
+                                            ("bf16", 128, 16, [300, 1]), ("f32", 16, 4, [300, 41])])
+def test_channel_rms_normalisation(io, d, M, lengths):
+    """The listing's ch_rms option, non-causal: statistics over all valid query
+    rows and all valid key rows, forward and backward (with the dependence of
+    the scales on every sample), through the tensor-core path (bf16 d = 32 and
+    64), the generic backward on tensor-core statistics (bf16 d = 128) and the
+    generic path (fp32); the backward with the forward's saved state and with
+    the statistics recomputed."""
+    case = Case(2, 2, 300, d, M, 8, io, False, seed=91, qkv_scale=1.0 / math.sqrt(d), lengths=lengths,
+                with_grad=True)
+    case.ch_rms_target = _median_channel_rms(case)
+    lu = case.luna()
+    O = to_host(case.run_fwd(lu))
+    ref = case.oracle_fwd()
+    assert relerr(O, ref) < TOL[io]
+    okq, okk = case.smooth_rows("Q"), case.smooth_rows("K")
+    assert okq.mean() > 0.9 and okk.mean() > 0.9
+    rb = case.oracle_bwd()
+    A = case.oracle_bwd_abs_terms() if io == "f32" else None
+    for use_state in (True, False):
+        g = {k: to_host(v) for k, v in case.run_bwd(lu, use_state=use_state).items()}
+        assert relerr(g["dQ"][okq], rb["dQ"][okq]) < TOL[io], use_state
+        assert relerr(g["dK"][okk], rb["dK"][okk]) < TOL[io], use_state
+        assert relerr(g["dV"], rb["dV"]) < TOL[io], use_state
+        for k in ("dW", "db", "dw1", "db1", "dw2", "db2"):
+            if io == "f32":
+                assert sum_err(g[k], rb[k], A[k], TOL[io]) <= 1.0, (k, use_state)
+            else:
+                assert relerr(g[k], rb[k]) < TOL[io], (k, use_state)
+        if case.lengths is not None:
+            for b, ln in enumerate(case.lengths):
+                for k in ("dQ", "dK", "dV"):
+                    assert np.all(g[k][b, :, ln:] == 0)
