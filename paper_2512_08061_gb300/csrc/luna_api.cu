@@ -104,7 +104,7 @@ luna_status make_plan(const luna_attn_desc *ad, const luna_phi_desc *pd, Plan &p
         p.o_zfin = w.take((size_t)BH * D * f);
         p.o_items = w.take((kMaxGrid + 1 + 2 * (size_t)BH) * sizeof(int));
         if (p.ch_target > 0.0f) {
-            p.o_chpart = w.take(2 * (size_t)BH * p.nsplit_b * p.lay.L * f);
+            p.o_chpart = w.take(2 * (size_t)kChStatBlocks * p.lay.L * f);
             p.o_chstat = w.take(8 * (size_t)kMaxL * sizeof(double));
             p.o_chsigma = w.take((size_t)kMaxL * f);
             p.o_chkappa = w.take(2 * (size_t)kMaxL * f);
@@ -118,8 +118,8 @@ luna_status make_plan(const luna_attn_desc *ad, const luna_phi_desc *pd, Plan &p
         p.o_dzpart = w.take((size_t)BH * nslot * D * f);
         p.o_dSfin = w.take((size_t)BH * SD * f);
         p.o_dzfin = w.take((size_t)BH * D * f);
-        // with channel normalisation, as many partials again for the scale term of the backward
-        p.o_gpart = w.take((p.ch_target > 0.0f ? 4 : 2) * (size_t)BH * p.nsplit_b * p.gsize * f);
+        // with channel normalisation, the partials of the scale term of the backward follow
+        p.o_gpart = w.take((2 * (size_t)BH * p.nsplit_b + (p.ch_target > 0.0f ? 2 * kChKBlocks : 0)) * p.gsize * f);
         p.o_hist = w.take((size_t)p.gsize * f);
         p.ws_bwd = w.n;
         p.state_bytes = (size_t)BH * (SD + D) * f;

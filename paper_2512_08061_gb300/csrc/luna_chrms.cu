@@ -35,6 +35,7 @@ using namespace simt;
 namespace {
 
 constexpr int kRed = 256;          // threads of the one-block reductions (a power of two)
+constexpr int kKWarps = 4;         // warps per block of the kappa-term pass
 constexpr double kChEps = 1e-6;    // the listing's eps, inside and outside the square root
 
 // Sum of one value per thread in a fixed order (tree over the threads), fp64.
@@ -50,40 +51,62 @@ __device__ double block_sum(double v, double *sh) {
     return r;
 }
 
-// Sum of phi^2 per channel over the valid rows of one (split, head) block of X (Q or K) and
-// every projection: part[(bh * nsplit_b + split) * L + l].
-template <typename IO>
-__global__ void __launch_bounds__(kThreads) k_chrms_stats(AttnArgs a, const void *Xv, float *part) {
+// Sum of phi^2 per channel over the valid rows and every projection of one side (blockIdx.y: 0 = Q,
+// 1 = K): one thread per (row, projection) item in a grid-stride loop, no block barriers in the loop;
+// block partials at part[(side * gridDim.x + blockIdx.x) * L + l].  W sits transposed in shared
+// memory (WT[c][i]), so the lanes of a row, which differ in i, read consecutive words.
+template <typename IO, bool VEC>
+__global__ void __launch_bounds__(kThreads) k_chrms_stats(AttnArgs a, float *part) {
     extern __shared__ __align__(16) float smem[];
-    Carve cv{smem};
     const TableLayout &lay = a.lay;
-    const int D = a.D, d = a.d, M = a.M, L = a.L;
-    SmemPhi s = carve_phi(cv, lay);
-    float *sX = cv.take(kTileK * d);
-    float *sPhi = cv.take(kTileK * D);
-    float *sred = cv.take(kThreads);
-    load_phi(s, lay, a.table);
-    const int bh = blockIdx.y, split = blockIdx.x;
-    const int len = head_length(a.lengths, bh / a.H, a.n);
-    const int r0 = split * a.rows_per_split_b;
-    const int r1 = min(len, min(a.n, r0 + a.rows_per_split_b));
-    const IO *X = static_cast<const IO *>(Xv) + (size_t)bh * a.n * d;
+    const int d = a.d, M = a.M, L = a.L, P = lay.Ppad;
+    float *sT = smem;
+    float *sAB = sT + r4(P);
+    float *sWT = sAB + r4(lay.nint * L * 2);
+    float *sb = sWT + r4(M * d);
+    float *sred = sb + r4(M);
+    {
+        const float *T = reinterpret_cast<const float *>(a.table + lay.off_T);
+        const float *AB = reinterpret_cast<const float *>(a.table + lay.off_AB);
+        const float *W = reinterpret_cast<const float *>(a.table + lay.off_W);
+        const float *b = reinterpret_cast<const float *>(a.table + lay.off_b);
+        for (int e = threadIdx.x; e < P; e += blockDim.x) sT[e] = T[e];
+        for (int e = threadIdx.x; e < lay.nint * L * 2; e += blockDim.x) sAB[e] = AB[e];
+        for (int e = threadIdx.x; e < M * d; e += blockDim.x) sWT[(e % d) * M + e / d] = W[e];
+        for (int e = threadIdx.x; e < M; e += blockDim.x) sb[e] = b[e];
+    }
+    __syncthreads();
+    const int side = blockIdx.y;
+    const IO *X = static_cast<const IO *>(side ? a.K : a.Q);
+    const int64_t items = (int64_t)a.B * a.H * a.n * M;
     float acc[kMaxL];
 #pragma unroll
     for (int l = 0; l < kMaxL; ++l) acc[l] = 0.0f;
-    for (int t0 = r0; t0 < r1; t0 += kTileK) {
-        const int nr = min(kTileK, r1 - t0);
-        __syncthreads();
-        load_rows(sX, X + (size_t)t0 * d, nr * d);
-        __syncthreads();
-        phi_tile(lay, s, sX, nr, sPhi, nullptr, nullptr);
-        __syncthreads();
-        for (int e = threadIdx.x; e < nr * M; e += blockDim.x) {  // (row, projection) e: features e*L + l
-            const float *ph = sPhi + (size_t)e * L;
+    for (int64_t e = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; e < items; e += (int64_t)gridDim.x * blockDim.x) {
+        const int64_t row = e / M;
+        const int i = (int)(e - row * M);
+        const int64_t bh = row / a.n;
+        if ((int)(row - bh * a.n) >= head_length(a.lengths, (int)(bh / a.H), a.n)) continue;
+        const IO *x = X + row * d;
+        float u = sb[i];
+        if (VEC) {  // 16-byte loads: 8 bf16 or 4 fp32 values
+            constexpr int V = 16 / sizeof(IO);
+            for (int c0 = 0; c0 < d; c0 += V) {
+                const uint4 raw = __ldg(reinterpret_cast<const uint4 *>(x + c0));
+                const IO *v = reinterpret_cast<const IO *>(&raw);
 #pragma unroll
-            for (int l = 0; l < kMaxL; ++l)
-                if (l < L) acc[l] = fmaf(ph[l], ph[l], acc[l]);
+                for (int k = 0; k < V; ++k) u = fmaf(sWT[(c0 + k) * M + i], io_load(v + k), u);
+            }
+        } else {
+            for (int c = 0; c < d; ++c) u = fmaf(sWT[c * M + i], io_load(x + c), u);
         }
+        const float *ab = sAB + interval_of(sT, P, u) * L * 2;
+#pragma unroll
+        for (int l = 0; l < kMaxL; ++l)
+            if (l < L) {
+                const float y = fmaxf(fmaf(ab[2 * l], u, ab[2 * l + 1]), 0.0f);
+                acc[l] = fmaf(y, y, acc[l]);
+            }
     }
 #pragma unroll
     for (int l = 0; l < kMaxL; ++l) {
@@ -95,37 +118,48 @@ __global__ void __launch_bounds__(kThreads) k_chrms_stats(AttnArgs a, const void
             if ((int)threadIdx.x < o) sred[threadIdx.x] += sred[threadIdx.x + o];
             __syncthreads();
         }
-        if (threadIdx.x == 0) part[((size_t)bh * a.nsplit_b + split) * L + l] = sred[0];
+        if (threadIdx.x == 0) part[((size_t)side * gridDim.x + blockIdx.x) * L + l] = sred[0];
     }
 }
 
-// Statistics of both sides from the block partials (ordered sums, fp64):
-// stat[(side*4 + 0..2)*kMaxL + l] = s_l, rms_l, target/(rms_l + eps); stat[3*kMaxL] = N
-// (samples per side: valid rows x M); sigma[l] = s^q_l s^k_l.
+// Sum over p < n of x[p * stride] by one warp, lanes over p, then a fixed shuffle tree (fp64).
+__device__ double warp_sum_strided(const float *x, int n, int stride) {
+    const int lane = threadIdx.x & 31;
+    double v = 0.0;
+    for (int p = lane; p < n; p += 32) v += x[(size_t)p * stride];
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) v += __shfl_xor_sync(0xffffffffu, v, o);
+    return v;
+}
+
+// Statistics of both sides from the block partials (fixed-order sums, fp64), one warp per
+// (side, channel): stat[(side*4 + 0..2)*kMaxL + l] = s_l, rms_l, target/(rms_l + eps);
+// stat[3*kMaxL] = N (samples per side: valid rows x M); sigma[l] = s^q_l s^k_l.
 __global__ void __launch_bounds__(kRed) k_chrms_scales(AttnArgs a, const float *part, int nparts, float target,
                                                        double *stat, float *sigma) {
     __shared__ double sh[kRed];
-    const int BH = a.B * a.H, L = a.L;
+    __shared__ double ssc[2 * kMaxL];
+    const int BH = a.B * a.H, L = a.L, warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     double rows = 0.0;
     for (int bh = threadIdx.x; bh < BH; bh += blockDim.x) rows += head_length(a.lengths, bh / a.H, a.n);
     const double N = block_sum(rows, sh) * a.M;
-    for (int side = 0; side < 2; ++side)
-        for (int l = 0; l < L; ++l) {
-            double v = 0.0;
-            for (int p = threadIdx.x; p < nparts; p += blockDim.x) v += part[((size_t)side * nparts + p) * L + l];
-            v = block_sum(v, sh);
-            if (threadIdx.x == 0) {
-                const double mean = N > 0.0 ? v * a.M / N : 0.0;  // y = sqrt(M) phi
-                const double rms = sqrt(mean + kChEps);
-                const double r = (double)target / (rms + kChEps);
-                stat[(side * 4 + 0) * kMaxL + l] = r < 1.0 ? r : 1.0;
-                stat[(side * 4 + 1) * kMaxL + l] = rms;
-                stat[(side * 4 + 2) * kMaxL + l] = r;
-            }
+    for (int q = warp; q < 2 * L; q += blockDim.x >> 5) {
+        const int side = q / L, l = q - side * L;
+        const double v = warp_sum_strided(part + (size_t)side * nparts * L + l, nparts, L);
+        if (lane == 0) {
+            const double mean = N > 0.0 ? v * a.M / N : 0.0;  // y = sqrt(M) phi
+            const double rms = sqrt(mean + kChEps);
+            const double r = (double)target / (rms + kChEps);
+            const double sl = r < 1.0 ? r : 1.0;
+            stat[(side * 4 + 0) * kMaxL + l] = sl;
+            stat[(side * 4 + 1) * kMaxL + l] = rms;
+            stat[(side * 4 + 2) * kMaxL + l] = r;
+            ssc[side * kMaxL + l] = sl;
         }
+    }
     if (threadIdx.x == 0) stat[3 * kMaxL] = N;
     __syncthreads();
-    if ((int)threadIdx.x < L) sigma[threadIdx.x] = (float)(stat[threadIdx.x] * stat[4 * kMaxL + threadIdx.x]);
+    if ((int)threadIdx.x < L) sigma[threadIdx.x] = (float)(ssc[threadIdx.x] * ssc[kMaxL + threadIdx.x]);
 }
 
 // rows f of S [BH][D][dv] and z [BH][D] times sigma_{f mod L}
@@ -165,14 +199,14 @@ __global__ void __launch_bounds__(128) k_chrms_dstate(AttnArgs a, const float *s
 // at 1 (target/(rms + eps) > 1) or the side has no samples.
 __global__ void __launch_bounds__(kRed) k_chrms_kappa(AttnArgs a, const double *T, float target, const double *stat,
                                                       float *kappa) {
-    __shared__ double sh[kRed];
-    const int BH = a.B * a.H, L = a.L;
+    const int BH = a.B * a.H, L = a.L, warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     const double N = stat[3 * kMaxL];
-    for (int l = 0; l < L; ++l) {
+    for (int l = warp; l < L; l += blockDim.x >> 5) {
         double v = 0.0;
-        for (int bh = threadIdx.x; bh < BH; bh += blockDim.x) v += T[(size_t)bh * L + l];
-        v = block_sum(v, sh);
-        if (threadIdx.x == 0)
+        for (int bh = lane; bh < BH; bh += 32) v += T[(size_t)bh * L + l];
+#pragma unroll
+        for (int o = 16; o > 0; o >>= 1) v += __shfl_xor_sync(0xffffffffu, v, o);
+        if (lane == 0)
             for (int side = 0; side < 2; ++side) {
                 const double s = stat[(side * 4 + 0) * kMaxL + l], rms = stat[(side * 4 + 1) * kMaxL + l];
                 const double r = stat[(side * 4 + 2) * kMaxL + l];
@@ -182,102 +216,145 @@ __global__ void __launch_bounds__(kRed) k_chrms_kappa(AttnArgs a, const double *
     }
 }
 
+// The kappa term of both sides (blockIdx.y: 0 = Q, 1 = K): dLoss/dphi = M kappa_l phi on every valid
+// sample, through the chain rule of the unnormalised feature map.  Each warp takes 32 consecutive rows
+// (lane = row) in a grid-stride loop: it stages them in shared memory (row stride d + 1, so the lanes'
+// rows fall in distinct banks), computes every projection's u, interval, channels and dU, then, with
+// the lanes over input columns, adds dU W to the rows of dQ / dK and dU^T X, column sums of dU to the
+// block's dW, db.  One parameter-gradient partial per block at gpart[(side * gridDim.x + blockIdx.x) *
+// gsize]; its interval histogram is accumulated in place by fp32 reductions in L2 (atomic adds without
+// a return value), which do not serialise like fp32 atomics in shared memory.
 template <typename IO>
-__device__ void add_dx(const TableLayout &lay, const SmemPhi &s, const float *sdU, int nr, IO *dX) {
-    const int M = lay.M, d = lay.d;
-    for (int e = threadIdx.x; e < nr * d; e += blockDim.x) {
-        const int r = e / d, c = e - r * d;
-        float acc = io_load(dX + e);
-        for (int i = 0; i < M; ++i) acc = fmaf(sdU[r * M + i], s.W[i * d + c], acc);
-        io_store(dX + e, acc);
-    }
-}
-
-// The kappa term of one side: dLoss/dphi = M kappa_l phi on every valid sample, through the
-// chain rule of the (unnormalised) feature map; adds to dQ or dK and writes one parameter-gradient
-// partial per (split, head) block at gpart[(side * BH * nsplit_b + bh * nsplit_b + split) * gsize].
-template <typename IO>
-__global__ void __launch_bounds__(kThreads) k_chrms_phi_bwd(AttnArgs a, int side, const float *kappa, float *gpart) {
+__global__ void __launch_bounds__(kKWarps * 32) k_chrms_kterm(AttnArgs a, const float *kappa, float *gpart) {
     extern __shared__ __align__(16) float smem[];
-    Carve cv{smem};
     const TableLayout &lay = a.lay;
-    const int D = a.D, d = a.d, M = a.M, L = a.L;
-    SmemPhi s = carve_phi(cv, lay);
-    float *sX = cv.take(kTileB * d);
-    float *sPhi = cv.take(kTileB * D);
-    float *sdPhi = cv.take(kTileB * D);
-    float *sU = cv.take(kTileB * M);
-    int *sJ = reinterpret_cast<int *>(cv.take(kTileB * M));
-    float *sdU = cv.take(kTileB * M);
-    float *shist = cv.take(lay.nint * L * 2);
-    float *sk = cv.take(kMaxL);
-    load_phi(s, lay, a.table);
-    for (int e = threadIdx.x; e < lay.nint * L * 2; e += blockDim.x) shist[e] = 0.0f;
-    if ((int)threadIdx.x < L) sk[threadIdx.x] = kappa[side * kMaxL + threadIdx.x] * (float)M;
-    const int bh = blockIdx.y, split = blockIdx.x;
-    const int len = head_length(a.lengths, bh / a.H, a.n);
-    const int r0 = split * a.rows_per_split_b;
-    const int r1 = min(len, min(a.n, r0 + a.rows_per_split_b));
-    const IO *X = static_cast<const IO *>(side ? a.K : a.Q) + (size_t)bh * a.n * d;
-    IO *dX = static_cast<IO *>(side ? a.dK : a.dQ) + (size_t)bh * a.n * d;
-    GradAcc g = {};
-    for (int t0 = r0; t0 < r1; t0 += kTileB) {
-        const int nr = min(kTileB, r1 - t0);
-        __syncthreads();
-        load_rows(sX, X + (size_t)t0 * d, nr * d);
-        __syncthreads();
-        phi_tile(lay, s, sX, nr, sPhi, sU, sJ);
-        __syncthreads();
-        for (int e = threadIdx.x; e < nr * D; e += blockDim.x) sdPhi[e] = sk[e % L] * sPhi[e];  // D = M*L
-        __syncthreads();
-        phi_backward_tile(lay, s, sX, nr, sPhi, sdPhi, sU, sJ, sdU, shist, g);
-        add_dx(lay, s, sdU, nr, dX + (size_t)t0 * d);
+    const int d = a.d, M = a.M, L = a.L, P = lay.Ppad, NH = lay.nint * L * 2;
+    const int dp = d + 1, mp = M + 1;
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    const int side = blockIdx.y;
+    float *sT = smem;
+    float *sAB = sT + r4(P);
+    float *sW = sAB + r4(NH);
+    float *sb = sW + r4(M * d);
+    float *sdW = sb + r4(M);
+    float *sdb = sdW + r4(M * d);
+    float *sk = sdb + r4(M);
+    float *sx = sk + r4(kMaxL) + warp * (r4(32 * dp) + r4(32 * mp));
+    float *sdu = sx + r4(32 * dp);
+    const int Md = M * d;
+    float *gp = gpart + ((size_t)side * gridDim.x + blockIdx.x) * a.gsize;
+    float *ghist = gp + Md + M;
+    {
+        const float *T = reinterpret_cast<const float *>(a.table + lay.off_T);
+        const float *AB = reinterpret_cast<const float *>(a.table + lay.off_AB);
+        const float *W = reinterpret_cast<const float *>(a.table + lay.off_W);
+        const float *b = reinterpret_cast<const float *>(a.table + lay.off_b);
+        for (int e = threadIdx.x; e < P; e += blockDim.x) sT[e] = T[e];
+        for (int e = threadIdx.x; e < NH; e += blockDim.x) { sAB[e] = AB[e]; ghist[e] = 0.0f; }
+        for (int e = threadIdx.x; e < M * d; e += blockDim.x) { sW[e] = W[e]; sdW[e] = 0.0f; }
+        for (int e = threadIdx.x; e < M; e += blockDim.x) { sb[e] = b[e]; sdb[e] = 0.0f; }
+        if ((int)threadIdx.x < L) sk[threadIdx.x] = kappa[side * kMaxL + threadIdx.x] * (float)M;
     }
     __syncthreads();
-    const size_t slot = (size_t)side * a.B * a.H * a.nsplit_b + (size_t)bh * a.nsplit_b + split;
-    store_grad_partial(lay, g, shist, gpart + slot * a.gsize);
+    const IO *X = static_cast<const IO *>(side ? a.K : a.Q);
+    IO *dX = static_cast<IO *>(side ? a.dK : a.dQ);
+    const int64_t rows = (int64_t)a.B * a.H * a.n;
+    const int64_t ngroups = (rows + 31) / 32;
+    for (int64_t grp = (int64_t)blockIdx.x * kKWarps + warp; grp < ngroups; grp += (int64_t)gridDim.x * kKWarps) {
+        const int64_t row0 = grp * 32, myrow = row0 + lane;
+        bool valid = false;
+        if (myrow < rows) {
+            const int64_t bh = myrow / a.n;
+            valid = (int)(myrow - bh * a.n) < head_length(a.lengths, (int)(bh / a.H), a.n);
+        }
+        const unsigned vmask = __ballot_sync(0xffffffffu, valid);
+        if (vmask == 0u) continue;
+        for (int r = 0; r < 32; ++r) {
+            const bool vr = (vmask >> r) & 1u;
+            for (int c = lane; c < d; c += 32) sx[r * dp + c] = vr ? io_load(X + (row0 + r) * d + c) : 0.0f;
+        }
+        __syncwarp();
+        for (int i = 0; i < M; ++i) {
+            float du = 0.0f;
+            if (valid) {
+                const float *w = sW + i * d, *x = sx + lane * dp;
+                float u = sb[i];
+                for (int c = 0; c < d; ++c) u = fmaf(w[c], x[c], u);
+                const int j = interval_of(sT, P, u);
+                const float *ab = sAB + j * L * 2;
+                float *h = ghist + j * L * 2;
+                for (int l = 0; l < L; ++l) {
+                    const float ph = fmaxf(fmaf(ab[2 * l], u, ab[2 * l + 1]), 0.0f);
+                    if (ph > 0.0f) {  // outer ReLU on
+                        const float g = sk[l] * ph;
+                        du = fmaf(g, ab[2 * l], du);
+                        if (g != 0.0f) {
+                            atomicAdd(h + 2 * l, g);
+                            atomicAdd(h + 2 * l + 1, g * u);
+                        }
+                    }
+                }
+            }
+            sdu[lane * mp + i] = du;
+        }
+        __syncwarp();
+        for (int c = lane; c < d; c += 32) {
+            float cur[32];  // the 32 rows' current values, all loaded before any store
+#pragma unroll
+            for (int r = 0; r < 32; ++r) cur[r] = ((vmask >> r) & 1u) ? io_load(dX + (row0 + r) * d + c) : 0.0f;
+#pragma unroll
+            for (int r = 0; r < 32; ++r) {
+                if (!((vmask >> r) & 1u)) continue;
+                float acc = 0.0f;
+                for (int i = 0; i < M; ++i) acc = fmaf(sdu[r * mp + i], sW[i * d + c], acc);
+                io_store(dX + (row0 + r) * d + c, cur[r] + acc);
+            }
+            for (int i = 0; i < M; ++i) {
+                float acc = 0.0f;
+                for (int r = 0; r < 32; ++r) acc = fmaf(sdu[r * mp + i], sx[r * dp + c], acc);
+                atomicAdd(sdW + i * d + c, acc);
+            }
+        }
+        if (lane < M) {
+            float acc = 0.0f;
+            for (int r = 0; r < 32; ++r) acc += sdu[r * mp + lane];
+            atomicAdd(sdb + lane, acc);
+        }
+        __syncwarp();
+    }
+    __syncthreads();
+    for (int e = threadIdx.x; e < Md; e += blockDim.x) gp[e] = sdW[e];
+    for (int e = threadIdx.x; e < M; e += blockDim.x) gp[Md + e] = sdb[e];
 }
 
 size_t smem_stats(const AttnArgs &a) {
-    HostCarve cv; carve_phi_host(cv, a.lay);
-    cv.take(kTileK * a.d); cv.take(kTileK * a.D); cv.take(kThreads);
-    return cv.bytes();
+    return (size_t)(r4(a.lay.Ppad) + r4(a.lay.nint * a.lay.L * 2) + r4(a.M * a.d) + r4(a.M) + kThreads) * 4;
 }
-size_t smem_phi_bwd(const AttnArgs &a) {
-    HostCarve cv; carve_phi_host(cv, a.lay);
-    cv.take(kTileB * a.d); cv.take(kTileB * a.D); cv.take(kTileB * a.D);
-    cv.take(kTileB * a.M); cv.take(kTileB * a.M); cv.take(kTileB * a.M);
-    cv.take(a.lay.nint * a.lay.L * 2); cv.take(kMaxL);
-    return cv.bytes();
+size_t smem_kterm(const AttnArgs &a) {
+    const int NH = a.lay.nint * a.L * 2;
+    return (size_t)(r4(a.lay.Ppad) + r4(NH) + 2 * r4(a.M * a.d) + 2 * r4(a.M) + r4(kMaxL) +
+                    kKWarps * (r4(32 * (a.d + 1)) + r4(32 * (a.M + 1)))) * 4;
 }
 
-template <typename IO>
+template <typename IO, bool VEC>
 cudaError_t stats_impl(const AttnArgs &a, cudaStream_t s) {
-    const int nparts = a.B * a.H * a.nsplit_b;
     const size_t sm = smem_stats(a);
-    cudaError_t e = set_smem(k_chrms_stats<IO>, sm);
+    cudaError_t e = set_smem(k_chrms_stats<IO, VEC>, sm);
     if (e != cudaSuccess) return e;
-    for (int side = 0; side < 2; ++side) {
-        LUNA_LAUNCH("chrms_stats", k_chrms_stats<IO>, dim3(a.nsplit_b, a.B * a.H), kThreads, sm, s, a,
-                    side ? a.K : a.Q, a.ch_part + (size_t)side * nparts * a.L);
-        if ((e = cudaGetLastError()) != cudaSuccess) return e;
-    }
-    LUNA_LAUNCH("chrms_scales", k_chrms_scales, 1, kRed, 0, s, a, a.ch_part, nparts, a.ch_target, a.ch_stat,
+    LUNA_LAUNCH("chrms_stats", (k_chrms_stats<IO, VEC>), dim3(kChStatBlocks, 2), kThreads, sm, s, a, a.ch_part);
+    if ((e = cudaGetLastError()) != cudaSuccess) return e;
+    LUNA_LAUNCH("chrms_scales", k_chrms_scales, 1, kRed, 0, s, a, a.ch_part, kChStatBlocks, a.ch_target, a.ch_stat,
                 a.ch_sigma);
     return cudaGetLastError();
 }
 
 template <typename IO>
-cudaError_t phi_bwd_impl(const AttnArgs &a, float *gpart, cudaStream_t s) {
-    const size_t sm = smem_phi_bwd(a);
-    cudaError_t e = set_smem(k_chrms_phi_bwd<IO>, sm);
+cudaError_t kterm_impl(const AttnArgs &a, float *gpart, cudaStream_t s) {
+    const size_t sm = smem_kterm(a);
+    cudaError_t e = set_smem(k_chrms_kterm<IO>, sm);
     if (e != cudaSuccess) return e;
-    for (int side = 0; side < 2; ++side) {
-        LUNA_LAUNCH("chrms_phi_bwd", k_chrms_phi_bwd<IO>, dim3(a.nsplit_b, a.B * a.H), kThreads, sm, s, a, side,
-                    a.ch_kappa, gpart);
-        if ((e = cudaGetLastError()) != cudaSuccess) return e;
-    }
-    return cudaSuccess;
+    LUNA_LAUNCH("chrms_kterm", k_chrms_kterm<IO>, dim3(kChKBlocks, 2), kKWarps * 32, sm, s, a, a.ch_kappa, gpart);
+    return cudaGetLastError();
 }
 
 int blocks_for(int64_t n) {
@@ -288,12 +365,17 @@ int blocks_for(int64_t n) {
 }  // namespace
 
 size_t chrms_max_smem(const AttnArgs &a) {
-    const size_t x = smem_stats(a), y = smem_phi_bwd(a);
+    const size_t x = smem_stats(a), y = smem_kterm(a);
     return x > y ? x : y;
 }
 
 cudaError_t launch_chrms_stats(const AttnArgs &a, luna_dtype io, cudaStream_t s) {
-    return io == LUNA_F32 ? stats_impl<float>(a, s) : stats_impl<__nv_bfloat16>(a, s);
+    // 16-byte row loads when every row starts on a 16-byte boundary
+    const size_t rb = (size_t)a.d * (io == LUNA_F32 ? 4 : 2);
+    const bool vec = rb % 16 == 0 && (reinterpret_cast<uintptr_t>(a.Q) & 15) == 0 &&
+                     (reinterpret_cast<uintptr_t>(a.K) & 15) == 0;
+    if (io == LUNA_F32) return vec ? stats_impl<float, true>(a, s) : stats_impl<float, false>(a, s);
+    return vec ? stats_impl<__nv_bfloat16, true>(a, s) : stats_impl<__nv_bfloat16, false>(a, s);
 }
 
 cudaError_t launch_chrms_scale_state(const AttnArgs &a, cudaStream_t s) {
@@ -317,9 +399,9 @@ cudaError_t launch_chrms_backward(const AttnArgs &a, int main_parts, int *nparts
     cudaError_t e = cudaGetLastError();
     if (e != cudaSuccess) return e;
     float *gpart = a.gpart + (size_t)main_parts * a.gsize;
-    e = a.ch_io == LUNA_F32 ? phi_bwd_impl<float>(a, gpart, s) : phi_bwd_impl<__nv_bfloat16>(a, gpart, s);
+    e = a.ch_io == LUNA_F32 ? kterm_impl<float>(a, gpart, s) : kterm_impl<__nv_bfloat16>(a, gpart, s);
     if (e != cudaSuccess) return e;
-    *nparts = main_parts + 2 * a.B * a.H * a.nsplit_b;
+    *nparts = main_parts + 2 * kChKBlocks;
     return cudaSuccess;
 }
 

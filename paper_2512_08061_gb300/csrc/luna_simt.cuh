@@ -42,12 +42,17 @@ struct AttnArgs {
     // channel RMS normalisation of the feature map (non-causal; ch_sigma null: off)
     float ch_target;                   // the listing's ch_rms_target
     luna_dtype ch_io;                  // element type of Q, K, dQ, dK
-    float *ch_part;                    // [2][BH * nsplit_b][L]: per-block sums of phi^2, queries then keys
+    float *ch_part;                    // [2][kChStatBlocks][L]: per-block sums of phi^2, queries then keys
     double *ch_stat;                   // [8][kMaxL]: per side s, rms, target/(rms+eps), unused; [3][0] = N
     float *ch_sigma;                   // [kMaxL]: s^q_l s^k_l
     double *ch_T;                      // [BH][L]: per-head sums of S' . dS + z' dz over each channel's rows
     float *ch_kappa;                   // [2][kMaxL]: factor of y_l in dLoss/dy_l from the scale, per side
 };
+
+// blocks per side of the channel-statistics kernel and of the scale-term backward pass (fixed counts:
+// the sums do not depend on the device)
+constexpr int kChStatBlocks = 304;
+constexpr int kChKBlocks = 304;
 
 // one step of the streaming form for every (batch, head): state S [D][dv], z [D] (fp32, in place)
 struct DecodeArgs {
