@@ -55,7 +55,14 @@ def parse():
     ap.add_argument("--cpu-seconds", type=float, default=12.0, help="target CPU work of the oracle sample")
     ap.add_argument("--seq-len", type=int, default=0,
                     help="shorter sequence length n for profiler captures of a small case (the JSON line reports it)")
-    return ap.parse_args()
+    ap.add_argument("--ch-rms-target", type=float, default=0.0,
+                    help="channel RMS normalisation of the feature map with this target (non-causal workloads)")
+    args = ap.parse_args()
+    if args.ch_rms_target < 0:
+        ap.error("--ch-rms-target must be >= 0")
+    if args.ch_rms_target > 0 and (WORKLOADS[args.workload].causal or WORKLOADS[args.workload].decode):
+        ap.error("--ch-rms-target: the channel normalisation is built for the non-causal form only")
+    return args
 
 
 def dist_env():
@@ -122,6 +129,10 @@ def kernel_bytes(w, lengths, kernel: str) -> float:
     table["tcc_dstats"] = valid * (2 * D * 2 + rv + 4)
     table["tcc_key"] = valid * (2 * (2 * D * 2) + 2 * rv + 4) + total * rv + valid * D * 4
     table["tc_phi_bwd"] = valid * (rd + D * 4) + total * rd
+    # channel normalisation, both sides per launch: the statistics read every valid row of Q and K;
+    # the scale-term pass reads them and reads and writes the same rows of dQ and dK
+    table["chrms_stats"] = 2 * valid * rd
+    table["chrms_kterm"] = 2 * valid * 3 * rd
     return float(table.get(kernel, 0.0))
 
 
@@ -300,7 +311,8 @@ def run_gpu(args, w):
     devt = {k: v.to(dev, non_blocking=True) for k, v in host.items()}
     lengths_d = None if lengths_h is None else lengths_h.to(dev)
     params_d = {k: torch.from_numpy(v).to(dev) for k, v in params.items()}
-    lu = L.Luna(w.B, w.H, w.n, w.d, w.dv, w.M, w.L, w.hidden, w.causal, w.eps, io_dtype, w.chunk, dev)
+    lu = L.Luna(w.B, w.H, w.n, w.d, w.dv, w.M, w.L, w.hidden, w.causal, w.eps, io_dtype, w.chunk, dev,
+                ch_rms_target=args.ch_rms_target)
     O = torch.empty_like(devt["V"])
     grads = None
     if w.backward:
@@ -336,6 +348,8 @@ def run_gpu(args, w):
     # dominant kernel: the library kernel with the largest device time in one step
     kernels = ["phi_prepare", "keystats", "query", "bwd_query", "bwd_key", "grad_sum", "mlp_grads",
                "causal_out", "causal_bwd_seg", "causal_dq", "causal_dkv"] + L.TC_KERNELS
+    if args.ch_rms_target > 0:
+        kernels += ["chrms_stats", "chrms_scales", "chrms_scale", "chrms_dstate", "chrms_kappa", "chrms_kterm"]
     per_kernel = {}
     for k in kernels:
         L.luna_profile_start(k)
@@ -467,7 +481,8 @@ def run_gpu(args, w):
         "config": {"workload": f"{w.name}: B={w.B} H={w.H} n={w.n} d={w.d} D={w.D} (M={w.M}, L={w.L}), "
                                f"{w.io}, {'causal' if w.causal else 'non-causal'}, "
                                f"{'fwd+bwd' if w.backward else 'fwd'}"
-                               + (f", lengths U[{w.len_range[0]},{w.len_range[1]}]" if w.len_range else ""),
+                               + (f", lengths U[{w.len_range[0]},{w.len_range[1]}]" if w.len_range else "")
+                               + ch_rms_label(args),
                    "global_batch": w.B * world, "seq_len": w.n, "parallelism": f"replicas{world}",
                    "l2": "flushed before every timed step (2x L2 buffer written outside the events)"},
         "fwd": {"value": job_throughput(w.tokens, world, fwd_ms), "unit": "tokens/s", "ms_per_step": fwd_ms},
@@ -480,7 +495,7 @@ def run_gpu(args, w):
         "clocks": clk,
     }
     if rank == 0 and world == 1 and not args.no_cpu_baseline:
-        result["cpu_baseline"] = cpu_baseline(w, args.cpu_seconds)
+        result["cpu_baseline"] = cpu_baseline(w, args.cpu_seconds, args.ch_rms_target)
     if world > 1:
         tdist.destroy_process_group()
     return result if rank == 0 else None
@@ -489,7 +504,11 @@ def run_gpu(args, w):
 # --------------------------------------------------------------------------
 # the CPU oracle (reported baseline, and the --impl reference arm)
 
-def oracle_run(w, units: int) -> float:
+def ch_rms_label(args) -> str:
+    return f", channel RMS normalisation target {args.ch_rms_target:g}" if args.ch_rms_target > 0 else ""
+
+
+def oracle_run(w, units: int, ch_rms_target: float = 0.0) -> float:
     """Runs the fp64 oracle (fwd, and bwd for training workloads) on the first
     `units` (batch, head) units of the workload's own input streams; returns
     the wall time in seconds."""
@@ -504,7 +523,7 @@ def oracle_run(w, units: int) -> float:
     V = synth.IOTensor(synth.normal(w.seed, "attn.V", (units, 1, w.n, w.dv)) * w.qkv_scale, w.io).value
     dO = synth.IOTensor(synth.normal(w.seed, "attn.dO", (units, 1, w.n, w.dv)), w.io).value if w.backward else None
     lengths = None if ln is None else np.array([ln[(u // w.H) % w.B] for u in range(units)], dtype=np.int32)
-    p = oracle.PhiParams(synth.phi_params(w.seed, w.d, w.M, w.L, w.hidden))
+    p = oracle.PhiParams(synth.phi_params(w.seed, w.d, w.M, w.L, w.hidden), ch_rms_target)
     t0 = time.perf_counter()
     oracle.attn_fwd(p, Q, K, V, lengths, w.causal, w.eps)
     if w.backward:
@@ -517,12 +536,12 @@ def tokens_per_s(w, units, seconds) -> float:
     return w.n / (w.H * seconds / units)
 
 
-def cpu_baseline(w, target_s):
+def cpu_baseline(w, target_s, ch_rms_target=0.0):
     import oracle
     threads = oracle.max_threads()
-    t1 = oracle_run(w, threads)
+    t1 = oracle_run(w, threads, ch_rms_target)
     units = int(min(max(threads, threads * round(target_s / max(t1, 1e-3))), 4 * w.B * w.H))
-    t = oracle_run(w, units) if units != threads else t1
+    t = oracle_run(w, units, ch_rms_target) if units != threads else t1
     return {"value": tokens_per_s(w, units, t), "unit": "tokens/s", "cores": threads, "kind": "oracle",
             "sample": f"{units} (batch, head) units of {w.n} tokens, fwd{'+bwd' if w.backward else ''}, "
                       f"{t:.1f} s on {threads} threads, scaled to B*H={w.B * w.H} units per step"}
@@ -535,17 +554,18 @@ def run_reference(args, w):
     import oracle
     threads = oracle.max_threads()
     if args.warmup > 0:
-        oracle_run(w, 1)
+        oracle_run(w, 1, args.ch_rms_target)
     per = []
     for _ in range(args.steps):
-        t = oracle_run(w, threads)
+        t = oracle_run(w, threads, args.ch_rms_target)
         per.append(tokens_per_s(w, threads, t))
     value = statistics.median(per)
     sample = f"{threads} (batch, head) units of {w.n} tokens per step on {threads} threads"
     return {"metric": METRIC, "value": value, "unit": "tokens/s", "n_gpus": world, "steps": args.steps,
             "warmup": args.warmup, "ms_per_step": w.tokens / value * 1e3, "higher_is_better": True,
             "scaling": "weak", "vs_baseline": None, "dtype": "f64", "data": "synthetic", "impl": "reference",
-            "config": {"workload": f"{w.name}: B={w.B} H={w.H} n={w.n} d={w.d} D={w.D}, fp64 CPU oracle",
+            "config": {"workload": f"{w.name}: B={w.B} H={w.H} n={w.n} d={w.d} D={w.D}, fp64 CPU oracle"
+                                   + ch_rms_label(args),
                        "global_batch": w.B, "seq_len": w.n, "parallelism": "cpu"},
             "cpu_baseline": {"value": value, "unit": "tokens/s", "cores": threads, "kind": "oracle",
                              "sample": sample},

@@ -5,24 +5,24 @@
 // the mean over every valid row and projection of that input (a reduction over
 // the whole batch).
 //
-// The attention kernels stay as they are: with phi the unnormalised map, the
+// The attention kernels stay as they are.  With phi the unnormalised map, the
 // kernel value of Eq. (kernel-attn) is sum_f sigma_l(f) phi_f(q) phi_f(k) with
 // sigma_l = s^q_l s^k_l (s >= 0 commutes with the outer ReLU).  So
 //   forward:  S, z from the unnormalised keys, rows f scaled by sigma_l(f), then
 //             the query pass as before;
-//   backward: the query-side kernel (reading the scaled S, z) gives dLoss/dphi(q)
+//   backward: the query-side kernel, reading the scaled S, z, gives dLoss/dphi(q)
 //             of the unnormalised map directly; dS, dz scaled by sigma before the
-//             key-side kernel give dLoss/dphi(k) and dV.  Those are the gradients
-//             with s held fixed.  The dependence of s_l on every sample adds
-//             kappa_l y_l to dLoss/dy_l of every sample of the side, with
-//                 kappa_l = ds_l/drms_l * A_l / (N rms_l),
-//                 A_l = sum over the side's samples of dLoss/dy_l * y_l / s_l ... (*)
-//             and for the non-causal form (*) times s_l equals, on both sides,
-//                 T_l = sum_heads sum_{f in channel l} (S'_f . dS_f + z'_f dz_f)
-//             (S', z' the scaled statistics, dS, dz before scaling): the sample
-//             sums of phi(q) dphi(q) and phi(k) dphi(k) collapse onto the head's
-//             statistics.  The kappa term then runs through the ordinary chain
-//             rule of the feature map as dLoss/dphi = M kappa_l phi (phi = y/sqrt(M)).
+//             key-side kernel give dLoss/dphi(k) and dV.  These are the gradients
+//             with s held fixed.
+// The dependence of s_l on every sample of a side adds kappa_l y_l to dLoss/dy_l
+// of each of that side's samples, where
+//     kappa_l = ds_l/drms_l * A_l / (N rms_l),   ds_l/drms_l = -target / (rms_l + 1e-6)^2
+// (zero where s_l is clamped at 1), N the side's sample count and A_l the sum over
+// the side's samples of y_l times dLoss/d(s_l y_l).  For the non-causal form
+//     s_l A_l = T_l = sum over heads and the channel's feature rows f of (S'_f . dS_f + z'_f dz_f)
+// on both sides (S', z' the scaled statistics, dS, dz before scaling): the sample
+// sums collapse onto each head's statistics.  The kappa term then runs through the
+// ordinary chain rule of the feature map as dLoss/dphi = M kappa_l phi (phi = y/sqrt(M)).
 #include <math.h>
 
 #include "luna_prof.cuh"
