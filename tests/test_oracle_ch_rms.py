@@ -188,19 +188,22 @@ def _loss(p, target, Q, K, V, dO, lengths, causal, eps):
     return float(np.sum(oracle.attn_fwd(oracle.PhiParams(p, target), Q, K, V, lengths, causal, eps) * dO))
 
 
-@pytest.mark.parametrize("mix", ["clamped", "mixed"])
+@pytest.mark.parametrize("mix", ["clamped", "mixed", "shared"])
 @pytest.mark.parametrize("causal", [False, True])
 def test_gradients_match_finite_differences(causal, mix):
+    """Every gradient with the normalisation on (every live channel clamped, a mix
+    of clamped and unclamped channels, and the shared-channel MLP with every live
+    channel clamped) against central differences of the forward pass."""
     d, M, L, hid, n = 3, 2, 3, 3, 6
-    seed = 46 + (1 if causal else 0) + (2 if mix == "mixed" else 0)
-    p = _rand_params(seed, d, M, L, hid)
+    seed = 46 + (1 if causal else 0) + {"clamped": 0, "mixed": 2, "shared": 4}[mix]
+    p = _rand_params(seed, d, M, L, hid, shared=(mix == "shared"))
     Q, K, V = _rand_inputs(seed, 2, 1, n, d, 2, scale=1.5)
     dO = synth.normal(seed, "r.dO", V.shape)
     lengths = np.array([n, 4], dtype=np.int32)
     eps = 1e-3
     rms = np.concatenate([_rms_all(p, Q, lengths), _rms_all(p, K, lengths)])
-    if mix == "clamped":
-        target = 0.5 * float(rms.min())
+    if mix in ("clamped", "shared"):
+        target = 0.5 * float(rms[rms > 0.01].min())
     else:  # between the channels' RMS values, away from every one of them
         srt = np.sort(rms)
         gaps = srt[1:] / srt[:-1]
