@@ -169,7 +169,10 @@ luna_status luna_attn_fwd(const luna_attn_desc *ad, const luna_phi_desc *pd, con
  * `state` is NULL (the key statistics are recomputed from K and V) or the
  * state written by luna_attn_fwd on the same Q, K, V, lengths and table.
  * The derivative of each ReLU at 0 is taken as 0.  Parameter gradients are
- * summed over all heads, rows and projections. */
+ * summed over all heads, rows and projections.  With pd->ch_rms_target > 0 the
+ * channel statistics of Q and K are recomputed by every call, and a `state`
+ * must come from luna_attn_fwd with the same descriptors (it holds the
+ * normalised key statistics). */
 luna_status luna_attn_bwd(const luna_attn_desc *ad, const luna_phi_desc *pd, const void *table, const void *Q,
                           const void *K, const void *V, const void *dO, const int32_t *lengths,
                           const void *state, void *dQ, void *dK, void *dV, const luna_phi_grads *grads,
