@@ -49,3 +49,24 @@ def test_channel_rms_option():
         r = subprocess.run([sys.executable, os.path.join(ROOT, "bench.py"), "--workload", wl, "--ch-rms-target", "0.1"],
                            cwd=ROOT, capture_output=True, text=True, timeout=120)
         assert r.returncode == 2 and "non-causal form only" in r.stderr
+
+
+def test_algorithmic_bytes_by_hand():
+    """Per-launch algorithmic bytes on a small non-causal case worked out by hand:
+    B = 2, H = 1, n = 256, d = dv = 32, D = 64, bf16, lengths (256, 100):
+    valid rows 356, all rows 512, statistics 2 x (64*32 + 64) x 4 B = 16896 B."""
+    sys.path.insert(0, ROOT)
+    import dataclasses
+    import numpy as np
+    import bench
+    from synth.workloads import WORKLOADS
+    w = dataclasses.replace(WORKLOADS["lra"], B=2, H=1, n=256)
+    ln = np.array([256, 100], dtype=np.int32)
+    row = 32 * 2  # one row of Q, K, V or their gradients in bf16
+    assert bench.kernel_bytes(w, ln, "tc_keys") == 356 * 2 * row + 16896
+    assert bench.kernel_bytes(w, ln, "tc_query") == 356 * row + 512 * row + 16896
+    assert bench.kernel_bytes(w, ln, "tc_bwd_query") == 356 * 2 * row + 512 * row + 2 * 16896
+    assert bench.kernel_bytes(w, ln, "tc_bwd_key") == 356 * 2 * row + 512 * 2 * row + 16896
+    assert bench.kernel_bytes(w, ln, "chrms_stats") == 2 * 356 * row
+    assert bench.kernel_bytes(w, ln, "chrms_kterm") == 2 * 356 * 3 * row
+    assert bench.kernel_bytes(w, ln, "no_such_kernel") == 0.0
