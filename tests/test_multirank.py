@@ -34,7 +34,7 @@ def _rank(rank: int, world: int, port: int, q) -> None:
         mine = 1.5 + 2.0 * rank  # this rank's step time (ms)
         step_ms = bench.max_over_ranks(mine, "cpu", world)
         rate = bench.job_throughput(1000, world, step_ms)
-        args = argparse.Namespace(steps=1, warmup=0, cpu_seconds=1.0)
+        args = argparse.Namespace(steps=1, warmup=0, cpu_seconds=1.0, ch_rms_target=0.0)
         ref = bench.run_reference(args, WORKLOADS["tiny_f32"])
         tdist.barrier()
         tdist.destroy_process_group()
