@@ -46,7 +46,7 @@ def build(force: bool = False) -> str:
 class _Phi(ctypes.Structure):
     _fields_ = [("d", ctypes.c_int), ("M", ctypes.c_int), ("L", ctypes.c_int), ("hid", ctypes.c_int)] + [
         (k, ctypes.c_void_p) for k in ("W", "b", "w1", "b1", "w2", "b2")
-    ] + [("shared", ctypes.c_int), ("ch_rms_target", ctypes.c_double), ("chs", ctypes.c_void_p)]
+    ] + [("shared", ctypes.c_int), ("ch_rms_target", ctypes.c_double), ("chs", ctypes.c_void_p), ("heads", ctypes.c_int)]
 
 
 _P = ctypes.c_void_p
@@ -73,6 +73,13 @@ def lib():
             L.oracle_max_threads.restype = _I
             L.oracle_set_threads.argtypes = [_I]
             L.oracle_set_abs_terms.argtypes = [_I]
+            L.oracle_phi_size.restype = ctypes.c_size_t
+            L.oracle_phi_offset.restype = ctypes.c_size_t
+            L.oracle_phi_offset.argtypes = [_I]
+            # the mirror of the C struct must have its layout
+            assert L.oracle_phi_size() == ctypes.sizeof(_Phi)
+            for i, f in enumerate(("W", "shared", "ch_rms_target", "chs", "heads")):
+                assert L.oracle_phi_offset(i) == getattr(_Phi, f).offset, f
             _lib = L
     return _lib
 
@@ -92,7 +99,9 @@ def _f64(a) -> np.ndarray:
 class PhiParams:
     """fp64 copies of the feature-map parameters (W, b, w1, b1, w2, b2).  One MLP per
     channel: w1, b1, w2 of shape (L, hidden); the shared-channel MLP: w1, b1 of shape
-    (hidden,) and w2 of shape (L, hidden).  ch_rms_target > 0 turns on the channel RMS
+    (hidden,) and w2 of shape (L, hidden).  Per-head parameters carry a leading head axis
+    on every array (W of shape (H, M, d), ...): head h of every sequence then uses slice h,
+    and the gradients keep that axis.  ch_rms_target > 0 turns on the channel RMS
     normalisation: every channel's MLP outputs are scaled by
     s_l = min(target / (rms_l + 1e-6), 1) with rms_l over the valid rows of the input
     the feature map is applied to (the queries and the keys separately)."""
@@ -100,20 +109,31 @@ class PhiParams:
     def __init__(self, params: dict, ch_rms_target: float = 0.0):
         self.arrays = {k: _f64(params[k]) for k in ("W", "b", "w1", "b1", "w2", "b2")}
         W = self.arrays["W"]
-        self.M, self.d = W.shape
-        self.shared = self.arrays["w1"].ndim == 1
-        self.L, self.hid = self.arrays["w2"].shape
-        assert self.arrays["b"].shape == (self.M,)
-        assert self.arrays["w1"].shape == self.arrays["b1"].shape == ((self.hid,) if self.shared else (self.L, self.hid))
-        assert self.arrays["b2"].shape == (self.L,)
+        self.heads = W.shape[0] if W.ndim == 3 else 0
+        lead = (self.heads,) if self.heads else ()
+        self.M, self.d = W.shape[-2:]
+        core = {k: v.shape[len(lead):] for k, v in self.arrays.items()}
+        self.shared = len(core["w1"]) == 1
+        self.L, self.hid = core["w2"]
+        assert all(v.shape[:len(lead)] == lead for v in self.arrays.values())
+        assert core["b"] == (self.M,)
+        assert core["w1"] == core["b1"] == ((self.hid,) if self.shared else (self.L, self.hid))
+        assert core["b2"] == (self.L,)
+        if self.heads and ch_rms_target > 0:
+            raise ValueError("channel normalisation with per-head parameters is not defined here")
         self.struct = _Phi(self.d, self.M, self.L, self.hid,
                            *[self.arrays[k].ctypes.data for k in ("W", "b", "w1", "b1", "w2", "b2")],
-                           int(self.shared), float(ch_rms_target), None)
+                           int(self.shared), float(ch_rms_target), None, int(self.heads))
         self.ch_rms_target = float(ch_rms_target)
 
     @property
     def D(self) -> int:
         return self.M * self.L
+
+    def head(self, h: int) -> "PhiParams":
+        """The parameters of head h (per-head parameters only)."""
+        assert self.heads
+        return PhiParams({k: v[h] for k, v in self.arrays.items()})
 
     def ref(self):
         return ctypes.byref(self.struct)
@@ -127,6 +147,7 @@ def ch_rms(params, X, lengths=None):
     """Channel RMS statistics of the MLP outputs over the valid rows of X (B,H,n,d):
     (s, rms), each of shape (L,), s = min(target / (rms + 1e-6), 1)."""
     p = _as_params(params)
+    assert not p.heads
     X = _f64(X)
     B, H, n, d = X.shape
     la, lp = _lens(lengths, B)
@@ -138,9 +159,13 @@ def ch_rms(params, X, lengths=None):
 
 def featmap(params, X) -> np.ndarray:
     """phi(X) for rows of X (..., d) -> (..., M*L), feature index i*L + l.  With channel
-    RMS normalisation the statistics are those of all rows of X."""
+    RMS normalisation the statistics are those of all rows of X.  With per-head parameters
+    X is (..., H, n, d) and head h's rows use head h's parameters."""
     p = _as_params(params)
     X = _f64(X)
+    if p.heads:
+        assert X.ndim >= 3 and X.shape[-3] == p.heads
+        return np.stack([featmap(p.head(h), X[..., h, :, :]) for h in range(p.heads)], axis=-3)
     rows = X.size // p.d
     out = np.empty(X.shape[:-1] + (p.D,), dtype=np.float64)
     lib().oracle_featmap(p.ref(), X.ctypes.data, rows, out.ctypes.data)
@@ -150,6 +175,9 @@ def featmap(params, X) -> np.ndarray:
 def kink_margin(params, X) -> np.ndarray:
     p = _as_params(params)
     X = _f64(X)
+    if p.heads:
+        assert X.ndim >= 3 and X.shape[-3] == p.heads
+        return np.stack([kink_margin(p.head(h), X[..., h, :, :]) for h in range(p.heads)], axis=-2)
     out = np.empty(X.shape[:-1], dtype=np.float64)
     lib().oracle_kink_margin(p.ref(), X.ctypes.data, X.size // p.d, out.ctypes.data)
     return out
@@ -157,6 +185,7 @@ def kink_margin(params, X) -> np.ndarray:
 
 def psi(params, l: int, u: float) -> float:
     p = _as_params(params)
+    assert not p.heads
     return lib().oracle_psi(p.ref(), int(l), float(u))
 
 
@@ -175,6 +204,7 @@ def attn_fwd(params, Q, K, V, lengths=None, causal=False, eps=1e-6) -> np.ndarra
     B, H, n, d = Q.shape
     dv = V.shape[-1]
     assert d == p.d and K.shape == Q.shape and V.shape[:3] == Q.shape[:3]
+    assert p.heads in (0, H)
     la, lp = _lens(lengths, B)
     O = np.empty(V.shape, dtype=np.float64)
     lib().oracle_attn_fwd(p.ref(), B, H, n, dv, int(bool(causal)), float(eps),
@@ -188,6 +218,7 @@ def attn_quadratic(params, Q, K, V, lengths=None, causal=False, eps=1e-6) -> np.
     Q, K, V = _f64(Q), _f64(K), _f64(V)
     B, H, n, d = Q.shape
     dv = V.shape[-1]
+    assert p.heads in (0, H)
     la, lp = _lens(lengths, B)
     O = np.empty(V.shape, dtype=np.float64)
     lib().oracle_attn_quadratic(p.ref(), B, H, n, dv, int(bool(causal)), float(eps),
@@ -214,13 +245,10 @@ def attn_bwd(params, Q, K, V, dO, lengths=None, causal=False, eps=1e-6) -> dict:
     Q, K, V, dO = _f64(Q), _f64(K), _f64(V), _f64(dO)
     B, H, n, d = Q.shape
     dv = V.shape[-1]
+    assert p.heads in (0, H)
     la, lp = _lens(lengths, B)
-    out = {
-        "dQ": np.empty(Q.shape), "dK": np.empty(K.shape), "dV": np.empty(V.shape),
-        "dW": np.empty((p.M, p.d)), "db": np.empty((p.M,)),
-        "dw1": np.empty(p.arrays["w1"].shape), "db1": np.empty(p.arrays["b1"].shape),
-        "dw2": np.empty((p.L, p.hid)), "db2": np.empty((p.L,)),
-    }
+    out = {"dQ": np.empty(Q.shape), "dK": np.empty(K.shape), "dV": np.empty(V.shape)}
+    out.update({"d" + k: np.empty(p.arrays[k].shape) for k in ("W", "b", "w1", "b1", "w2", "b2")})
     lib().oracle_attn_bwd(p.ref(), B, H, n, dv, int(bool(causal)), float(eps),
                           Q.ctypes.data, K.ctypes.data, V.ctypes.data, dO.ctypes.data, lp,
                           out["dQ"].ctypes.data, out["dK"].ctypes.data, out["dV"].ctypes.data,

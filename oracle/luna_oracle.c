@@ -26,6 +26,10 @@
  *   - the listing's shared_channels variant: one scalar MLP with L outputs
  *     (fc1: 1 -> hid shared by the channels, fc2: hid -> L), so channel l
  *     reads the same hidden units with its own fc2 row.
+ *   - per-head parameters (the conversion experiments instantiate the feature
+ *     map's parameters per layer and head, Sec. 5 / appendix): head h of every
+ *     sequence uses its own W, b and channel MLPs; their gradients are summed
+ *     over the batch only.
  *   - the listing's ch_rms channel normalisation: per call of the feature map
  *     (once over Q, once over K), every channel's MLP outputs are scaled by
  *     s_l = min(target / (rms_l + 1e-6), 1), rms_l = sqrt(mean y_l^2 + 1e-6)
@@ -38,6 +42,7 @@
  * central finite differences of the backward pass.
  */
 #include <math.h>
+#include <stddef.h>
 #include <stdint.h>
 #include <stdlib.h>
 #include <string.h>
@@ -59,7 +64,37 @@ typedef struct {
     int shared;       /* 1: one MLP for all channels (fc1 shared)        */
     double ch_rms_target; /* > 0: channel RMS normalisation to this target */
     const double *chs;    /* per-channel scales s_l in effect (NULL: 1); set per input by the callers */
+    int heads;            /* > 0: parameters per head (arrays carry a leading head axis of this size) */
 } oracle_phi;
+
+/* Layout of oracle_phi, checked by the Python binding against its mirror of the struct. */
+size_t oracle_phi_size(void) { return sizeof(oracle_phi); }
+size_t oracle_phi_offset(int field) {
+    switch (field) {
+        case 0: return offsetof(oracle_phi, W);
+        case 1: return offsetof(oracle_phi, shared);
+        case 2: return offsetof(oracle_phi, ch_rms_target);
+        case 3: return offsetof(oracle_phi, chs);
+        case 4: return offsetof(oracle_phi, heads);
+    }
+    return (size_t)-1;
+}
+
+/* The parameters of head h: p itself, or with per-head parameters the h-th slice of every array. */
+static oracle_phi head_view(const oracle_phi *p, int h) {
+    oracle_phi q = *p;
+    if (p->heads > 0) {
+        const size_t n1 = (size_t)(p->shared ? 1 : p->L) * p->hid, n2 = (size_t)p->L * p->hid;
+        q.W = p->W + (size_t)h * p->M * p->d;
+        q.b = p->b + (size_t)h * p->M;
+        q.w1 = p->w1 + (size_t)h * n1;
+        q.b1 = p->b1 + (size_t)h * n1;
+        q.w2 = p->w2 + (size_t)h * n2;
+        q.b2 = p->b2 + (size_t)h * p->L;
+        q.heads = 0;
+    }
+    return q;
+}
 
 /* offset of channel l's fc1 row (the one shared row when shared) */
 static size_t fc1_row(const oracle_phi *p, int l) { return (size_t)(p->shared ? 0 : l) * p->hid; }
@@ -342,7 +377,8 @@ void oracle_attn_fwd(const oracle_phi *p, int B, int H, int n, int dv, int causa
     for (int bh = 0; bh < B * H; ++bh) {
         int b = bh / H;
         size_t qo = (size_t)bh * n * d, vo = (size_t)bh * n * dv;
-        attn_fwd_head(&sm.pq, &sm.pk, n, dv, causal, eps, Q + qo, K + qo, V + vo, head_len(lengths, b, n), O + vo);
+        const oracle_phi vq = head_view(&sm.pq, bh % H), vk = head_view(&sm.pk, bh % H);
+        attn_fwd_head(&vq, &vk, n, dv, causal, eps, Q + qo, K + qo, V + vo, head_len(lengths, b, n), O + vo);
     }
     free(sm.st);
 }
@@ -370,9 +406,10 @@ void oracle_attn_quadratic(const oracle_phi *p, int B, int H, int n, int dv, int
         double *o = O + (size_t)bh * n * dv;
         double *PQ = (double *)malloc(sizeof(double) * (size_t)(len > 0 ? len : 1) * D);
         double *PK = (double *)malloc(sizeof(double) * (size_t)(len > 0 ? len : 1) * D);
+        const oracle_phi vq = head_view(&sm.pq, bh % H), vk = head_view(&sm.pk, bh % H);
         for (int i = 0; i < len; ++i) {
-            phi_row(&sm.pq, q + (size_t)i * d, PQ + (size_t)i * D);
-            phi_row(&sm.pk, k + (size_t)i * d, PK + (size_t)i * D);
+            phi_row(&vq, q + (size_t)i * d, PQ + (size_t)i * D);
+            phi_row(&vk, k + (size_t)i * d, PK + (size_t)i * D);
         }
         memset(o, 0, sizeof(double) * (size_t)n * dv);
         for (int i = 0; i < len; ++i) {
@@ -518,7 +555,8 @@ void oracle_attn_bwd(const oracle_phi *p, int B, int H, int n, int dv, int causa
         oracle_grads g = {base, base + nW, base + nW + nb, base + nW + nb + nh, base + nW + nb + 2 * nh,
                           base + nW + nb + 3 * nh};
         size_t qo = (size_t)bh * n * d, vo = (size_t)bh * n * dv, po = (size_t)bh * n * D;
-        attn_bwd_head(&sm.pq, &sm.pk, n, dv, causal, eps, Q + qo, K + qo, V + vo, dO + vo,
+        const oracle_phi vq = head_view(&sm.pq, bh % H), vk = head_view(&sm.pk, bh % H);
+        attn_bwd_head(&vq, &vk, n, dv, causal, eps, Q + qo, K + qo, V + vo, dO + vo,
                       head_len(lengths, bh / H, n), dQ + qo, dK + qo, dV + vo, &g, norm ? dPQ + po : NULL,
                       norm ? dPK + po : NULL);
     }
@@ -537,11 +575,12 @@ void oracle_attn_bwd(const oracle_phi *p, int B, int H, int n, int dv, int causa
                 const double *X = (side ? K : Q) + (size_t)bh * n * d;
                 const double *dP = (side ? dPK : dPQ) + (size_t)bh * n * D;
                 double *a = A + ((size_t)bh * 2 + side) * L;
+                const oracle_phi v = head_view(p, bh % H);
                 for (int r = 0; r < len; ++r)
                     for (int i = 0; i < M; ++i) {
-                        const double u = project(p, i, X + (size_t)r * d);
+                        const double u = project(&v, i, X + (size_t)r * d);
                         for (int l = 0; l < L; ++l)
-                            a[l] += c * dP[(size_t)r * D + i * L + l] * relu(channel_pre(p, l, u));
+                            a[l] += c * dP[(size_t)r * D + i * L + l] * relu(channel_pre(&v, l, u));
                     }
             }
         }
@@ -565,23 +604,27 @@ void oracle_attn_bwd(const oracle_phi *p, int B, int H, int n, int dv, int causa
                               base + nW + nb + 3 * nh};
             const int len = head_len(lengths, bh / H, n);
             size_t qo = (size_t)bh * n * d, po = (size_t)bh * n * D;
-            phi_rows_backward(&sm.pq, Q + qo, len, dPQ + po, kappa, dQ + qo, &g);
-            phi_rows_backward(&sm.pk, K + qo, len, dPK + po, kappa + L, dK + qo, &g);
+            const oracle_phi vq = head_view(&sm.pq, bh % H), vk = head_view(&sm.pk, bh % H);
+            phi_rows_backward(&vq, Q + qo, len, dPQ + po, kappa, dQ + qo, &g);
+            phi_rows_backward(&vk, K + qo, len, dPK + po, kappa + L, dK + qo, &g);
         }
         free(A); free(kappa); free(dPQ); free(dPK);
     }
     free(sm.st);
-    /* ordered reduction over heads (fc1 gradients: hid entries when the MLP is shared) */
+    /* ordered reduction over the heads (fc1 gradients: hid entries when the MLP is shared); with
+     * per-head parameters, head h's gradients are the sum over the batch of its units b*H + h */
     double *outs[6] = {dW, db, dw1, db1, dw2, db2};
     const size_t n1 = p->shared ? (size_t)hid : nh;
     size_t sizes[6] = {nW, nb, n1, n1, nh, nb2};
     size_t offs[6] = {0, nW, nW + nb, nW + nb + nh, nW + nb + 2 * nh, nW + nb + 3 * nh};
-    for (int t = 0; t < 6; ++t) {
-        for (size_t e = 0; e < sizes[t]; ++e) {
-            double acc = 0.0;
-            for (int bh = 0; bh < BH; ++bh) acc += part[(size_t)bh * per + offs[t] + e];
-            outs[t][e] = acc;
-        }
-    }
+    const int G = p->heads > 0 ? H : 1;
+    for (int t = 0; t < 6; ++t)
+        for (int h = 0; h < G; ++h)
+            for (size_t e = 0; e < sizes[t]; ++e) {
+                double acc = 0.0;
+                for (int bh = 0; bh < BH; ++bh)
+                    if (G == 1 || bh % H == h) acc += part[(size_t)bh * per + offs[t] + e];
+                outs[t][(size_t)h * sizes[t] + e] = acc;
+            }
     free(part);
 }

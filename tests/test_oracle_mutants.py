@@ -1,6 +1,7 @@
 """The oracle pins are sensitive: plausible mistakes planted in a temporary
 copy of the oracle source (on the CPU) make at least one pin fail.  Mistakes
-in the channel RMS normalisation are checked against its own pin file."""
+in the channel RMS normalisation and in the per-head parameters are checked
+against their own pin files."""
 import os
 import shutil
 import subprocess
@@ -50,11 +51,25 @@ CH_RMS_MUTANTS = {
 }
 
 
-@pytest.mark.parametrize("name", sorted(MUTANTS) + sorted(CH_RMS_MUTANTS))
+PER_HEAD_PINS = "tests/test_oracle_per_head.py"
+PER_HEAD_MUTANTS = {
+    "per-head parameters of the wrong head": (
+        "const oracle_phi vq = head_view(&sm.pq, bh % H), vk = head_view(&sm.pk, bh % H);\n        attn_fwd_head(",
+        "const oracle_phi vq = head_view(&sm.pq, (bh + 1) % H), vk = head_view(&sm.pk, (bh + 1) % H);\n"
+        "        attn_fwd_head("),
+    "per-head gradients summed over every head": (
+        "if (G == 1 || bh % H == h) acc +=", "if (1) acc +="),
+}
+
+ALL = {**{k: (v, "tests/test_oracle_pins.py") for k, v in MUTANTS.items()},
+       **{k: (v, CH_RMS_PINS) for k, v in CH_RMS_MUTANTS.items()},
+       **{k: (v, PER_HEAD_PINS) for k, v in PER_HEAD_MUTANTS.items()}}
+
+
+@pytest.mark.parametrize("name", sorted(ALL))
 def test_planted_mistake_is_caught(name, tmp_path):
     src = open(os.path.join(ROOT, "oracle", "luna_oracle.c")).read()
-    a, b = MUTANTS[name] if name in MUTANTS else CH_RMS_MUTANTS[name]
-    pins = CH_RMS_PINS if name in CH_RMS_MUTANTS else "tests/test_oracle_pins.py"
+    (a, b), pins = ALL[name]
     assert a in src, f"mutation site for {name!r} not found"
     work = tmp_path / "w"
     shutil.copytree(os.path.join(ROOT, "oracle"), work / "oracle", ignore=shutil.ignore_patterns("_build", "__pycache__"))
