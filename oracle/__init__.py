@@ -46,7 +46,8 @@ def build(force: bool = False) -> str:
 class _Phi(ctypes.Structure):
     _fields_ = [("d", ctypes.c_int), ("M", ctypes.c_int), ("L", ctypes.c_int), ("hid", ctypes.c_int)] + [
         (k, ctypes.c_void_p) for k in ("W", "b", "w1", "b1", "w2", "b2")
-    ] + [("shared", ctypes.c_int), ("ch_rms_target", ctypes.c_double), ("chs", ctypes.c_void_p), ("heads", ctypes.c_int)]
+    ] + [("shared", ctypes.c_int), ("ch_rms_target", ctypes.c_double), ("chs", ctypes.c_void_p), ("heads", ctypes.c_int),
+         ("signed_out", ctypes.c_int)]
 
 
 _P = ctypes.c_void_p
@@ -78,7 +79,7 @@ def lib():
             L.oracle_phi_offset.argtypes = [_I]
             # the mirror of the C struct must have its layout
             assert L.oracle_phi_size() == ctypes.sizeof(_Phi)
-            for i, f in enumerate(("W", "shared", "ch_rms_target", "chs", "heads")):
+            for i, f in enumerate(("W", "shared", "ch_rms_target", "chs", "heads", "signed_out")):
                 assert L.oracle_phi_offset(i) == getattr(_Phi, f).offset, f
             _lib = L
     return _lib
@@ -101,12 +102,13 @@ class PhiParams:
     channel: w1, b1, w2 of shape (L, hidden); the shared-channel MLP: w1, b1 of shape
     (hidden,) and w2 of shape (L, hidden).  Per-head parameters carry a leading head axis
     on every array (W of shape (H, M, d), ...): head h of every sequence then uses slice h,
-    and the gradients keep that axis.  ch_rms_target > 0 turns on the channel RMS
+    and the gradients keep that axis.  nonneg=False is the listing's option of that name:
+    the channel outputs without the outer ReLU.  ch_rms_target > 0 turns on the channel RMS
     normalisation: every channel's MLP outputs are scaled by
     s_l = min(target / (rms_l + 1e-6), 1) with rms_l over the valid rows of the input
     the feature map is applied to (the queries and the keys separately)."""
 
-    def __init__(self, params: dict, ch_rms_target: float = 0.0):
+    def __init__(self, params: dict, ch_rms_target: float = 0.0, nonneg: bool = True):
         self.arrays = {k: _f64(params[k]) for k in ("W", "b", "w1", "b1", "w2", "b2")}
         W = self.arrays["W"]
         self.heads = W.shape[0] if W.ndim == 3 else 0
@@ -123,8 +125,9 @@ class PhiParams:
             raise ValueError("channel normalisation with per-head parameters is not defined here")
         self.struct = _Phi(self.d, self.M, self.L, self.hid,
                            *[self.arrays[k].ctypes.data for k in ("W", "b", "w1", "b1", "w2", "b2")],
-                           int(self.shared), float(ch_rms_target), None, int(self.heads))
+                           int(self.shared), float(ch_rms_target), None, int(self.heads), int(not nonneg))
         self.ch_rms_target = float(ch_rms_target)
+        self.nonneg = bool(nonneg)
 
     @property
     def D(self) -> int:
@@ -133,7 +136,7 @@ class PhiParams:
     def head(self, h: int) -> "PhiParams":
         """The parameters of head h (per-head parameters only)."""
         assert self.heads
-        return PhiParams({k: v[h] for k, v in self.arrays.items()})
+        return PhiParams({k: v[h] for k, v in self.arrays.items()}, nonneg=self.nonneg)
 
     def ref(self):
         return ctypes.byref(self.struct)

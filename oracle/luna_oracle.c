@@ -26,6 +26,8 @@
  *   - the listing's shared_channels variant: one scalar MLP with L outputs
  *     (fc1: 1 -> hid shared by the channels, fc2: hid -> L), so channel l
  *     reads the same hidden units with its own fc2 row.
+ *   - the listing's nonneg = False: the channel outputs without the outer
+ *     ReLU (features of either sign).
  *   - per-head parameters (the conversion experiments instantiate the feature
  *     map's parameters per layer and head, Sec. 5 / appendix): head h of every
  *     sequence uses its own W, b and channel MLPs; their gradients are summed
@@ -65,6 +67,7 @@ typedef struct {
     double ch_rms_target; /* > 0: channel RMS normalisation to this target */
     const double *chs;    /* per-channel scales s_l in effect (NULL: 1); set per input by the callers */
     int heads;            /* > 0: parameters per head (arrays carry a leading head axis of this size) */
+    int signed_out;       /* 1: the listing's nonneg = False (no outer ReLU); 0: its default */
 } oracle_phi;
 
 /* Layout of oracle_phi, checked by the Python binding against its mirror of the struct. */
@@ -76,6 +79,7 @@ size_t oracle_phi_offset(int field) {
         case 2: return offsetof(oracle_phi, ch_rms_target);
         case 3: return offsetof(oracle_phi, chs);
         case 4: return offsetof(oracle_phi, heads);
+        case 5: return offsetof(oracle_phi, signed_out);
     }
     return (size_t)-1;
 }
@@ -138,7 +142,13 @@ static double channel_pre(const oracle_phi *p, int l, double u) {
     return y;
 }
 
-double oracle_psi(const oracle_phi *p, int l, double u) { return relu(channel_pre(p, l, u)); }
+/* psi_l(u): the channel output, through the outer ReLU unless the outputs are signed */
+static double channel_out(const oracle_phi *p, int l, double u) {
+    const double y = channel_pre(p, l, u);
+    return p->signed_out ? y : relu(y);
+}
+
+double oracle_psi(const oracle_phi *p, int l, double u) { return channel_out(p, l, u); }
 
 /* phi(x) = (1/sqrt(M)) [s_l psi_l(w_i^T x + b_i)]_{i,l},  index i*L + l (s_l = 1 without ch_rms) */
 static void phi_row(const oracle_phi *p, const double *x, double *out) {
@@ -146,7 +156,7 @@ static void phi_row(const oracle_phi *p, const double *x, double *out) {
     for (int i = 0; i < p->M; ++i) {
         double u = project(p, i, x);
         for (int l = 0; l < p->L; ++l)
-            out[i * p->L + l] = s * (p->chs ? p->chs[l] : 1.0) * relu(channel_pre(p, l, u));
+            out[i * p->L + l] = s * (p->chs ? p->chs[l] : 1.0) * channel_out(p, l, u);
     }
 }
 
@@ -171,7 +181,7 @@ static void ch_rms_scales(const oracle_phi *p, const double *X, int B, int H, in
             for (int i = 0; i < p->M; ++i) {
                 const double u = project(p, i, x);
                 for (int l = 0; l < L; ++l) {
-                    const double y = relu(channel_pre(p, l, u));
+                    const double y = channel_out(p, l, u);
                     part[(size_t)bh * L + l] += y * y;
                 }
             }
@@ -231,7 +241,7 @@ void oracle_kink_margin(const oracle_phi *p, const double *X, int64_t rows, doub
                     y += w2[k] * relu(a);
                     ysc += fabs(w2[k] * relu(a));
                 }
-                if (ysc > 0.0) {
+                if (ysc > 0.0 && !p->signed_out) {  /* the outer ReLU's kink */
                     double rel = fabs(y) / ysc;
                     if (rel < m) m = rel;
                 }
@@ -267,7 +277,7 @@ static void phi_rows_backward(const oracle_phi *p, const double *X, int64_t rows
             double du = 0.0;
             for (int l = 0; l < p->L; ++l) {
                 double y = channel_pre(p, l, u);
-                if (!(y > 0.0)) continue; /* outer ReLU inactive */
+                if (!p->signed_out && !(y > 0.0)) continue; /* outer ReLU inactive */
                 double dy = dPhi[r * D + i * p->L + l] * s;
                 if (p->chs) dy = dy * p->chs[l] + (kappa ? kappa[l] * y : 0.0);
                 if (dy == 0.0) continue;
@@ -580,7 +590,7 @@ void oracle_attn_bwd(const oracle_phi *p, int B, int H, int n, int dv, int causa
                     for (int i = 0; i < M; ++i) {
                         const double u = project(&v, i, X + (size_t)r * d);
                         for (int l = 0; l < L; ++l)
-                            a[l] += c * dP[(size_t)r * D + i * L + l] * relu(channel_pre(&v, l, u));
+                            a[l] += c * dP[(size_t)r * D + i * L + l] * channel_out(&v, l, u);
                     }
             }
         }

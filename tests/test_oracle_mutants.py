@@ -1,7 +1,7 @@
 """The oracle pins are sensitive: plausible mistakes planted in a temporary
 copy of the oracle source (on the CPU) make at least one pin fail.  Mistakes
-in the channel RMS normalisation and in the per-head parameters are checked
-against their own pin files."""
+in the channel RMS normalisation, the per-head parameters and the signed
+channel outputs are checked against their own pin files."""
 import os
 import shutil
 import subprocess
@@ -61,7 +61,15 @@ PER_HEAD_MUTANTS = {
         "if (G == 1 || bh % H == h) acc +=", "if (1) acc +="),
 }
 
+SIGNED_PINS = "tests/test_oracle_signed.py"
+SIGNED_MUTANTS = {
+    "signed outputs still through the outer ReLU": ("return p->signed_out ? y : relu(y);", "return relu(y);"),
+    "signed outputs: backward still masks by the outer ReLU": (
+        "if (!p->signed_out && !(y > 0.0)) continue;", "if (!(y > 0.0)) continue;"),
+}
+
 ALL = {**{k: (v, "tests/test_oracle_pins.py") for k, v in MUTANTS.items()},
+       **{k: (v, SIGNED_PINS) for k, v in SIGNED_MUTANTS.items()},
        **{k: (v, CH_RMS_PINS) for k, v in CH_RMS_MUTANTS.items()},
        **{k: (v, PER_HEAD_PINS) for k, v in PER_HEAD_MUTANTS.items()}}
 
