@@ -575,6 +575,61 @@ def run_reference(args, w):
 DECODE_METRIC = "LUNA decode tokens/sec (one token per sequence per step) on 1 GB300; % of HBM roofline"
 
 
+def decode_oracle_run(w, units: int) -> float:
+    """One decode step of the first `units` (batch, head) units by the fp64 oracle as it stands: it keeps
+    no state between calls, so each unit's output for the new token is its causal output at position
+    n + 1, recomputed over the prefill and the token.  Returns the wall time in seconds."""
+    import oracle
+    tensors = {}
+    for name, tok, width in (("Q", "q", w.d), ("K", "k", w.d), ("V", "v", w.dv)):
+        pre = synth.normal(w.seed, f"attn.{name}", (units, 1, w.n, width)) * w.qkv_scale
+        new = synth.normal(w.seed, f"decode.{tok}", (units, 1, 1, width)) * w.qkv_scale
+        tensors[name] = synth.IOTensor(np.concatenate([pre, new], axis=2), w.io).value
+    p = oracle.PhiParams(synth.phi_params(w.seed, w.d, w.M, w.L, w.hidden))
+    t0 = time.perf_counter()
+    oracle.attn_fwd(p, tensors["Q"], tensors["K"], tensors["V"], None, True, w.eps)
+    return time.perf_counter() - t0
+
+
+def decode_tokens_per_s(w, units, seconds) -> float:
+    # one step = one token for each of the B sequences = B*H units
+    return units / (w.H * seconds)
+
+
+def decode_cpu_baseline(w, target_s):
+    import oracle
+    threads = oracle.max_threads()
+    t1 = decode_oracle_run(w, threads)
+    units = int(min(max(threads, threads * round(target_s / max(t1, 1e-3))), w.B * w.H))
+    t = decode_oracle_run(w, units) if units != threads else t1
+    return {"value": decode_tokens_per_s(w, units, t), "unit": "tokens/s", "cores": threads, "kind": "oracle",
+            "sample": f"{units} (batch, head) units, each recomputing its causal output over the {w.n}-token "
+                      f"prefill and the new token (the oracle keeps no state), {t:.1f} s on {threads} threads, "
+                      f"scaled to B*H={w.B * w.H} units per step"}
+
+
+def run_reference_decode(args, w):
+    rank, _, world = dist_env()
+    if rank != 0:
+        return None
+    import oracle
+    threads = oracle.max_threads()
+    if args.warmup > 0:
+        decode_oracle_run(w, 1)
+    per = [decode_tokens_per_s(w, threads, decode_oracle_run(w, threads)) for _ in range(args.steps)]
+    value = statistics.median(per)
+    sample = (f"{threads} (batch, head) units per step on {threads} threads, each recomputing its causal output "
+              f"over the {w.n}-token prefill and the new token")
+    return {"metric": DECODE_METRIC, "value": value, "unit": "tokens/s", "n_gpus": world, "steps": args.steps,
+            "warmup": args.warmup, "ms_per_step": w.B / value * 1e3, "higher_is_better": True, "scaling": "weak",
+            "vs_baseline": None, "dtype": "f64", "data": "synthetic", "impl": "reference",
+            "config": {"workload": f"{w.name}: B={w.B} H={w.H}, one token per sequence per step after a causal "
+                                   f"prefill of n={w.n}, d={w.d} D={w.D}, fp64 CPU oracle",
+                       "global_batch": w.B, "seq_len": w.n, "parallelism": "cpu"},
+            "cpu_baseline": {"value": value, "unit": "tokens/s", "cores": threads, "kind": "oracle", "sample": sample},
+            "e2e": {"value": value, "unit": "tokens/s", "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}}
+
+
 def decode_bytes(w) -> float:
     """Bytes of one decode step: every fp32 state element read and written once, and the
     token's q, k, v read and o written."""
@@ -684,9 +739,9 @@ def run_decode(args, w):
                           "frac": byts / (hbm * 1e9) * 1e3 / ms_step},
         "roofline": roof, "per_kernel_ms": {"decode": dom_ms / dom_n if dom_n else None},
         "e2e": e2e, "gpu_launches": int(launches), "clocks": clk,
-        "cpu_baseline": None,
-        "cpu_baseline_note": "the oracle keeps no state between calls; decode parity is tested against its causal form",
     }
+    if rank == 0 and world == 1 and not args.no_cpu_baseline:
+        result["cpu_baseline"] = decode_cpu_baseline(w, args.cpu_seconds)
     if world > 1:
         tdist.destroy_process_group()
     return result if rank == 0 else None
@@ -700,12 +755,7 @@ def main():
         w = dataclasses.replace(w, n=n, len_range=None if w.len_range is None else
                                 (min(w.len_range[0], n), min(w.len_range[1], n)))
     if w.decode:
-        if args.impl == "reference":
-            res = None if dist_env()[0] != 0 else {
-                "impl": "reference",
-                "unavailable": "the oracle keeps no state between calls (decode parity is tested against its causal form)"}
-        else:
-            res = run_decode(args, w)
+        res = run_reference_decode(args, w) if args.impl == "reference" else run_decode(args, w)
         if res is not None:
             print(json.dumps(res), flush=True)
         return

@@ -34,9 +34,13 @@ def test_reference_arm_line():
     assert e2e["h2d_bytes_per_step"] == 0 and e2e["d2h_bytes_per_step"] == 0
 
 
-def test_reference_arm_decode_is_unavailable():
+def test_reference_arm_decode():
+    """The decode workload's reference arm: the oracle recomputes each sampled head's causal
+    output over the prefill and the new token (it keeps no state)."""
     d = _run("--impl", "reference", "--workload", "decode", "--steps", "1", "--warmup", "0")
-    assert d["impl"] == "reference" and "unavailable" in d
+    assert d["impl"] == "reference" and d["value"] > 0 and d["unit"] == "tokens/s" and "decode" in d["metric"]
+    assert d["cpu_baseline"]["kind"] == "oracle" and d["cpu_baseline"]["value"] == d["value"]
+    assert d["e2e"]["h2d_bytes_per_step"] == 0 and "prefill of n=1024" in d["config"]["workload"]
 
 
 def test_channel_rms_option():
