@@ -4,17 +4,24 @@
 A step is one pass of the whole path over one batch of synthetic input: the
 feature-map table is prepared from the parameters, the forward pass runs
 (saving the key statistics) and the backward pass produces dQ, dK, dV and the
-parameter gradients.  The default workload is the Long-Range-Arena-shaped
-encoder attention (B=32, H=4, n=4096, d=32, D=64, bf16 I/O, valid lengths
-uniform in [2048, 4096]).  Tokens per step = B * n.
+parameter gradients.  The default workload is the long-context streaming form
+(causal_long: B=2, H=32, n=65536, d=128, D=128, bf16 I/O, fwd+bwd); the
+Long-Range-Arena-shaped encoder attention (lra: B=32, H=4, n=4096, d=32, D=64,
+valid lengths uniform in [2048, 4096], non-causal) is measured in the same run
+and reported under its own key.  Tokens per step = B * n.
 
-  python bench.py [--gpus N] [--steps K] [--warmup W] [--workload NAME] [--impl reference]
+  python bench.py [--gpus N] [--steps K] [--warmup W] [--workload NAME] [--also NAMES] [--impl reference]
+
+Every kernel's roofline fraction counts only the method's own tensors that it
+reads or writes (Q, K, V, dO, O, dQ, dK, dV and the per-head key statistics);
+rows that one stage hands to the next are traffic, not algorithmic bytes.
 
 Multi-GPU (torchrun): every rank runs an independent replica of the workload
 (the (batch, head) units are independent; there is no data-path collective),
 so scaling is weak and value = all ranks' tokens / max-over-ranks time.
 `--impl reference` times the fp64 CPU oracle instead (rank 0 only), on a
-bounded sample of the same workload.
+bounded sample of the same workload (the first 4096 tokens of each sequence
+for the streaming form), and reports the rate of that sample.
 """
 from __future__ import annotations
 
@@ -48,7 +55,10 @@ def parse():
     ap.add_argument("--gpus", type=int, default=1)
     ap.add_argument("--steps", type=int, default=100)
     ap.add_argument("--warmup", type=int, default=5)
-    ap.add_argument("--workload", default="lra", choices=sorted(WORKLOADS))
+    ap.add_argument("--workload", default="causal_long", choices=sorted(WORKLOADS))
+    ap.add_argument("--also", default="lra",
+                    help="comma-separated workloads also measured in the same run, each under its own key "
+                         "(empty: none)")
     ap.add_argument("--impl", default="gb300", choices=["gb300", "reference"])
     ap.add_argument("--no-e2e", action="store_true")
     ap.add_argument("--no-cpu-baseline", action="store_true")
@@ -62,6 +72,12 @@ def parse():
         ap.error("--ch-rms-target must be >= 0")
     if args.ch_rms_target > 0 and (WORKLOADS[args.workload].causal or WORKLOADS[args.workload].decode):
         ap.error("--ch-rms-target: the channel normalisation is built for the non-causal form only")
+    args.also = [a for a in args.also.split(",") if a]
+    for a in args.also:
+        if a not in WORKLOADS or WORKLOADS[a].decode:
+            ap.error(f"--also: unknown or decode workload {a}")
+    if args.seq_len > 0 or args.ch_rms_target > 0:
+        args.also = []
     return args
 
 
@@ -96,7 +112,7 @@ def peaks():
 
 
 # --------------------------------------------------------------------------
-# algorithmic bytes and flops ("Roofline accounting")
+# algorithmic bytes and flops of the method's own inputs and outputs
 
 def row_counts(w, lengths):
     valid = int(np.sum(lengths)) * w.H if lengths is not None else w.B * w.H * w.n
@@ -104,9 +120,14 @@ def row_counts(w, lengths):
 
 
 def kernel_bytes(w, lengths, kernel: str) -> float:
-    """Algorithmic HBM bytes of one launch of a kernel: every valid input row
-    read once, every output row written once (padded output rows are written
-    as zeros), the (D x dv + D) fp32 statistics per head read or written once."""
+    """Algorithmic HBM bytes of one launch of a kernel: the method's own tensors
+    that the kernel reads or writes (Q, K, V, dO read on their valid rows; O,
+    dQ, dK, dV written on every row, padded rows as zeros) and, for the
+    non-causal passes, the (D x dv + D) fp32 key statistics per head that the
+    method hands from the key pass to the query pass.  Rows that one stage of
+    the streaming-form backward writes for the next one (dphi, phi(k),
+    phi(q)/den) are this implementation's staging, not the method's: they count
+    as traffic (ncu), never as algorithmic bytes."""
     eb = 4 if w.io == "f32" else 2
     valid, total = row_counts(w, lengths)
     stats = w.B * w.H * (w.D * w.dv + w.D) * 4
@@ -117,22 +138,22 @@ def kernel_bytes(w, lengths, kernel: str) -> float:
         "bwd_query": valid * (rd + rv) + total * rd + 2 * stats,
         "bwd_key": valid * (rd + rv) + total * (rd + rv) + stats,
         "causal_out": valid * (2 * rd + rv) + total * rv,
+        # streaming-form backward on tensor cores: the method's tensors each stage touches
+        "tcc_query": valid * (2 * rd + 2 * rv),   # Q, K, V, dO
+        "tcc_dstats": 0,                          # staging rows only
+        "tcc_key": valid * 2 * rv + total * rv,   # V, dO; dV
+        "tc_phi_bwd": valid * rd + total * rd,    # Q (or K); dQ (or dK)
+        # channel normalisation, both sides per launch: the statistics read every valid row of Q and K;
+        # the scale-term pass reads them and reads and writes the same rows of dQ and dK
+        "chrms_stats": 2 * valid * rd,
+        "chrms_kterm": 2 * valid * 3 * rd,
     }
     # the tensor-core kernels move the same tensors as their generic counterparts
     for tc, generic in (("tc_keys", "keystats"), ("tc_query", "query"), ("tc_bwd_query", "bwd_query"),
                         ("tc_bwd_key", "bwd_key"), ("tc_causal", "causal_out")):
         table[tc] = table[generic]
-    # streaming-form backward stages: their inputs and outputs, including the rows they
-    # hand to the next stage (fp32 dphi; bf16 hi|lo phi(k) and phi(q)/den; den, -dO.O)
-    D = w.D
-    table["tcc_query"] = valid * (2 * rd + 2 * rv) + valid * (D * 4 + 8) + total * 2 * (2 * D * 2)
-    table["tcc_dstats"] = valid * (2 * D * 2 + rv + 4)
-    table["tcc_key"] = valid * (2 * (2 * D * 2) + 2 * rv + 4) + total * rv + valid * D * 4
-    table["tc_phi_bwd"] = valid * (rd + D * 4) + total * rd
-    # channel normalisation, both sides per launch: the statistics read every valid row of Q and K;
-    # the scale-term pass reads them and reads and writes the same rows of dQ and dK
-    table["chrms_stats"] = 2 * valid * rd
-    table["chrms_kterm"] = 2 * valid * 3 * rd
+    if w.causal:  # the streaming form's key pass per state segment reads K and V; its statistics are staging
+        table["tc_keys"] = valid * (rd + rv)
     return float(table.get(kernel, 0.0))
 
 
@@ -280,22 +301,20 @@ def host_inputs(w):
     return inp, params
 
 
-def run_gpu(args, w):
-    import torch
-    import torch.distributed as tdist
+def workload_label(w, ch_rms_target=0.0) -> str:
+    return (f"{w.name}: B={w.B} H={w.H} n={w.n} d={w.d} D={w.D} (M={w.M}, L={w.L}), {w.io}, "
+            f"{'causal' if w.causal else 'non-causal'}, {'fwd+bwd' if w.backward else 'fwd'}"
+            + (f", lengths U[{w.len_range[0]},{w.len_range[1]}]" if w.len_range else "")
+            + (f", channel RMS normalisation target {ch_rms_target:g}" if ch_rms_target > 0 else ""))
 
-    rank, local_rank, world = dist_env()
-    torch.cuda.set_device(local_rank)
-    if world > 1:
-        tdist.init_process_group("nccl", device_id=torch.device("cuda", local_rank))
-    from paper_2512_08061_gb300 import build
-    if rank == 0 or world == 1:
-        build.build()
-    if world > 1:
-        tdist.barrier()
+
+def measure_workload(args, w, dev, world, steps, ch_rms_target=0.0, with_e2e=True):
+    """Times `steps` steps of workload w on this rank's GPU (after the warm-up), the forward alone, every
+    library kernel of a step (live CUDA events on the launching stream) and, with_e2e, the step end to end
+    from pinned host buffers.  Returns the measurements of this rank (times are max over ranks)."""
+    import torch
     import paper_2512_08061_gb300.luna as L
 
-    dev = torch.device("cuda", local_rank)
     inp, params = host_inputs(w)
     io_dtype = torch.float32 if w.io == "f32" else torch.bfloat16
 
@@ -312,15 +331,20 @@ def run_gpu(args, w):
     lengths_d = None if lengths_h is None else lengths_h.to(dev)
     params_d = {k: torch.from_numpy(v).to(dev) for k, v in params.items()}
     lu = L.Luna(w.B, w.H, w.n, w.d, w.dv, w.M, w.L, w.hidden, w.causal, w.eps, io_dtype, w.chunk, dev,
-                ch_rms_target=args.ch_rms_target)
+                ch_rms_target=ch_rms_target)
     O = torch.empty_like(devt["V"])
     grads = None
+    f32 = dict(dtype=torch.float32, device=dev)
+
+    def grad_buffers():
+        return {"dQ": torch.empty_like(devt["Q"]), "dK": torch.empty_like(devt["K"]),
+                "dV": torch.empty_like(devt["V"]), "dW": torch.empty(w.M, w.d, **f32),
+                "db": torch.empty(w.M, **f32), "dw1": torch.empty(w.L, w.hidden, **f32),
+                "db1": torch.empty(w.L, w.hidden, **f32), "dw2": torch.empty(w.L, w.hidden, **f32),
+                "db2": torch.empty(w.L, **f32)}
+
     if w.backward:
-        f32 = dict(dtype=torch.float32, device=dev)
-        grads = {"dQ": torch.empty_like(devt["Q"]), "dK": torch.empty_like(devt["K"]), "dV": torch.empty_like(devt["V"]),
-                 "dW": torch.empty(w.M, w.d, **f32), "db": torch.empty(w.M, **f32),
-                 "dw1": torch.empty(w.L, w.hidden, **f32), "db1": torch.empty(w.L, w.hidden, **f32),
-                 "dw2": torch.empty(w.L, w.hidden, **f32), "db2": torch.empty(w.L, **f32)}
+        grads = grad_buffers()
     flush = torch.empty(2 * L2_BYTES, dtype=torch.uint8, device=dev)
     stream = torch.cuda.current_stream()
 
@@ -345,10 +369,10 @@ def run_gpu(args, w):
         step(devt)
     torch.cuda.synchronize()
 
-    # dominant kernel: the library kernel with the largest device time in one step
+    # every library kernel of one step, timed live with CUDA events on its launching stream
     kernels = ["phi_prepare", "keystats", "query", "bwd_query", "bwd_key", "grad_sum", "mlp_grads",
                "causal_out", "causal_bwd_seg", "causal_dq", "causal_dkv"] + L.TC_KERNELS
-    if args.ch_rms_target > 0:
+    if ch_rms_target > 0:
         kernels += ["chrms_stats", "chrms_scales", "chrms_scale", "chrms_dstate", "chrms_kappa", "chrms_kterm"]
     per_kernel = {}
     for k in kernels:
@@ -356,46 +380,43 @@ def run_gpu(args, w):
         step(devt)
         ms, n = L.luna_profile_stop()
         if n:
-            per_kernel[k] = ms / n
-    dominant = max(per_kernel, key=per_kernel.get) if per_kernel else None
+            per_kernel[k] = (ms, n)
+    dominant = max(per_kernel, key=lambda k: per_kernel[k][0]) if per_kernel else None
 
     # timed region
     if world > 1:
+        import torch.distributed as tdist
         tdist.barrier()
     torch.cuda.synchronize()
-    uuid = str(getattr(torch.cuda.get_device_properties(local_rank), "uuid", "") or "")
-    clocks = ClockSampler(("GPU-" + uuid if uuid and not uuid.startswith("GPU-") else uuid) or str(local_rank))
+    uuid = str(getattr(torch.cuda.get_device_properties(dev), "uuid", "") or "")
+    clocks = ClockSampler(("GPU-" + uuid if uuid and not uuid.startswith("GPU-") else uuid) or str(dev.index))
     if dominant:
         L.luna_profile_start(dominant)
     n0 = L.luna_launch_count()
-    ms_total = timed(args.steps, lambda: step(devt))
+    ms_total = timed(steps, lambda: step(devt))
     launches = L.luna_launch_count() - n0
     dom_ms, dom_n = L.luna_profile_stop() if dominant else (0.0, 0)
     clk = clocks.stop()
     torch.cuda.synchronize()
-    ms_step = ms_total / args.steps
-    ms_step = max_over_ranks(ms_step, dev, world)
+    ms_step = max_over_ranks(ms_total / steps, dev, world)
 
     # forward-only throughput (same flush discipline)
-    fwd_ms = timed(args.steps, lambda: step(devt, backward=False)) / args.steps
-    fwd_ms = max_over_ranks(fwd_ms, dev, world)
+    fwd_ms = max_over_ranks(timed(steps, lambda: step(devt, backward=False)) / steps, dev, world)
 
-    # end to end through the public API with host buffers: every step copies its inputs in from pinned
-    # host memory and its results out; steps are pipelined two deep on three streams (copy-in, compute,
-    # copy-out), with double-buffered device inputs and outputs, so that step i+1's inputs arrive and step
-    # i-1's results leave while step i computes.  Events keep every dependency: a step computes after its
-    # own inputs have landed, its results leave after it has computed, and a buffer is refilled only after
-    # the step that last used it is done with it.
+    # End to end through the public API with host buffers: every step copies its inputs in from pinned host
+    # memory and reads all of its results back (O; with the backward also dQ, dK, dV and the parameter
+    # gradients).  Steps are pipelined two deep on three streams (copy-in, compute, copy-out) with
+    # double-buffered device inputs and outputs, so that step i+1's inputs arrive and step i-1's results
+    # leave while step i computes.  Events keep every dependency: a step computes after its own inputs have
+    # landed, its results leave after it has computed, and a buffer is refilled only after the step that
+    # last used it is done with it.
     e2e = None
-    if not args.no_e2e:
+    if with_e2e:
         nb = 2
         dev_in = [{k: torch.empty_like(devt[k]) for k in host} for _ in range(nb)]
         len_in = [None if lengths_h is None else torch.empty_like(lengths_d) for _ in range(nb)]
-        dev_out = [dict({"O": torch.empty_like(O)}, **({k: torch.empty_like(v) for k, v in grads.items()} if grads else {}))
-                   for _ in range(nb)]
-        # the step's result read back: a training step's parameter gradients (O, dQ, dK, dV are activations
-        # and activation gradients that stay on the device for the neighbouring layers); a forward step's O
-        result_keys = [k for k in ("dW", "db", "dw1", "db1", "dw2", "db2")] if grads else ["O"]
+        dev_out = [dict({"O": torch.empty_like(O)}, **(grad_buffers() if grads else {})) for _ in range(nb)]
+        result_keys = list(dev_out[0].keys())
         host_out = [{k: torch.empty(dev_out[0][k].shape, dtype=dev_out[0][k].dtype).pin_memory() for k in result_keys}
                     for _ in range(nb)]
         bi = sum(v.numel() * v.element_size() for v in host.values()) + (
@@ -442,7 +463,7 @@ def run_gpu(args, w):
 
         e2e_run(2 * nb)
         torch.cuda.synchronize()
-        n_e2e = max(8, args.steps // 2)
+        n_e2e = max(8, steps // 2)
         t0, t1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
         e2e_run(n_e2e, t0, t1)
         torch.cuda.synchronize()
@@ -450,10 +471,18 @@ def run_gpu(args, w):
         e2e = {"value": job_throughput(w.tokens, world, e2e_ms), "unit": "tokens/s", "h2d_bytes_per_step": int(bi),
                "d2h_bytes_per_step": int(bo), "ms_per_step": e2e_ms,
                "pipelining": "copy-in of step i+1 and copy-out of step i-1 overlap the compute of step i",
-               "result": "parameter gradients dW, db, dw1, db1, dw2, db2" if grads else "O"}
+               "result": ", ".join(result_keys) + " read back every step"}
+        del dev_in, dev_out, host_out
 
     hbm, tflops, peak_src = peaks()
     lengths = inp["lengths"]
+    kern = {}
+    for k, (ms, n) in per_kernel.items():
+        byts = kernel_bytes(w, lengths, k)
+        launch_ms = ms / n
+        kern[k] = {"launch_ms": launch_ms, "launches_per_step": n, "share": ms / max(1e-12, sum(
+            v[0] for v in per_kernel.values())), "algorithmic_bytes": byts,
+            "frac": (byts / (launch_ms * 1e-3) / 1e9 / hbm) if byts else 0.0}
     roof = None
     if dominant and dom_n:
         byts = kernel_bytes(w, lengths, dominant)
@@ -462,38 +491,74 @@ def run_gpu(args, w):
         traffic, traffic_src = measured_traffic(dominant, w.name) if args.seq_len <= 0 else (None, None)
         roof = {"bound": "hbm", "kernel": dominant, "achieved": achieved, "peak": hbm, "unit": "GB/s",
                 "frac": (achieved / hbm) if achieved else None, "traffic": traffic, "traffic_source": traffic_src,
-                "peak_source": peak_src, "algorithmic_bytes": byts, "launch_ms": dom_ms / dom_n, "launches": dom_n}
+                "peak_source": peak_src, "algorithmic_bytes": byts, "launch_ms": dom_ms / dom_n, "launches": dom_n,
+                "of": f"{peak_src} HBM copy bandwidth"}
     sb, sf = step_bytes(w, lengths), step_flops(w, lengths)
     t_roof = max(sb / (hbm * 1e9), sf / (tflops * 1e12))
+    out = {"workload": workload_label(w, ch_rms_target), "value": job_throughput(w.tokens, world, ms_step),
+           "ms_per_step": ms_step, "fwd": {"value": job_throughput(w.tokens, world, fwd_ms), "unit": "tokens/s",
+                                           "ms_per_step": fwd_ms},
+           "step_roofline": {"bytes": sb, "tensor_flops": sf, "time_ms": t_roof * 1e3, "frac": t_roof * 1e3 / ms_step,
+                             "bound": "hbm" if sb / (hbm * 1e9) >= sf / (tflops * 1e12) else "tensor"},
+           "roofline": roof, "kernels": kern, "e2e": e2e, "gpu_launches": int(launches), "clocks": clk,
+           "steps": steps}
+    del lu, devt, O, grads, flush
+    torch.cuda.empty_cache()
+    return out
+
+
+def run_gpu(args, w):
+    import torch
+    import torch.distributed as tdist
+
+    rank, local_rank, world = dist_env()
+    torch.cuda.set_device(local_rank)
+    if world > 1:
+        tdist.init_process_group("nccl", device_id=torch.device("cuda", local_rank))
+    from paper_2512_08061_gb300 import build
+    if rank == 0 or world == 1:
+        build.build()
+    if world > 1:
+        tdist.barrier()
+
+    dev = torch.device("cuda", local_rank)
+    head = measure_workload(args, w, dev, world, args.steps, args.ch_rms_target, not args.no_e2e)
+    # the other long-sequence workload (LRA-shaped, non-causal), measured in the same run and reported under
+    # its own key
+    also = {}
+    for name in args.also:
+        if name and name != w.name:
+            w2 = WORKLOADS[name]
+            also[name] = measure_workload(args, w2, dev, world, max(3, min(args.steps, 50)), 0.0, not args.no_e2e)
     result = {
         "metric": METRIC,
-        "value": job_throughput(w.tokens, world, ms_step),
+        "value": head["value"],
         "unit": "tokens/s",
         "n_gpus": world,
         "steps": args.steps,
         "warmup": args.warmup,
-        "ms_per_step": ms_step,
+        "ms_per_step": head["ms_per_step"],
         "higher_is_better": True,
         "scaling": "weak",
         "vs_baseline": None,
         "dtype": w.io,
         "data": "synthetic",
-        "config": {"workload": f"{w.name}: B={w.B} H={w.H} n={w.n} d={w.d} D={w.D} (M={w.M}, L={w.L}), "
-                               f"{w.io}, {'causal' if w.causal else 'non-causal'}, "
-                               f"{'fwd+bwd' if w.backward else 'fwd'}"
-                               + (f", lengths U[{w.len_range[0]},{w.len_range[1]}]" if w.len_range else "")
-                               + ch_rms_label(args),
-                   "global_batch": w.B * world, "seq_len": w.n, "parallelism": f"replicas{world}",
+        "config": {"workload": head["workload"], "global_batch": w.B * world, "seq_len": w.n,
+                   "parallelism": f"replicas{world}",
                    "l2": "flushed before every timed step (2x L2 buffer written outside the events)"},
-        "fwd": {"value": job_throughput(w.tokens, world, fwd_ms), "unit": "tokens/s", "ms_per_step": fwd_ms},
-        "step_roofline": {"bytes": sb, "tensor_flops": sf, "time_ms": t_roof * 1e3,
-                          "frac": t_roof * 1e3 / ms_step},
-        "roofline": roof,
-        "per_kernel_ms": per_kernel,
-        "e2e": e2e,
-        "gpu_launches": int(launches),
-        "clocks": clk,
+        "fwd": head["fwd"],
+        "step_roofline": head["step_roofline"],
+        "roofline": head["roofline"],
+        "kernels": head["kernels"],
+        "per_kernel_ms": {k: v["launch_ms"] for k, v in head["kernels"].items()},
+        "e2e": head["e2e"],
+        "gpu_launches": head["gpu_launches"],
+        "clocks": head["clocks"],
     }
+    for name, m in also.items():
+        result[name] = {k: m[k] for k in ("workload", "value", "ms_per_step", "fwd", "step_roofline", "roofline",
+                                          "kernels", "e2e", "gpu_launches", "clocks", "steps")}
+        result[name]["unit"] = "tokens/s"
     if rank == 0 and world == 1 and not args.no_cpu_baseline:
         result["cpu_baseline"] = cpu_baseline(w, args.cpu_seconds, args.ch_rms_target)
     if world > 1:
@@ -504,25 +569,33 @@ def run_gpu(args, w):
 # --------------------------------------------------------------------------
 # the CPU oracle (reported baseline, and the --impl reference arm)
 
-def ch_rms_label(args) -> str:
-    return f", channel RMS normalisation target {args.ch_rms_target:g}" if args.ch_rms_target > 0 else ""
+def sample_rows(w) -> int:
+    """Rows per (batch, head) unit that one oracle sample takes: the whole sequence for the non-causal
+    workloads (every query reads every key), the first 4096 tokens of each sequence for the streaming form,
+    whose cost per token is the same at every position (a prefix of a causal sequence is its own causal
+    problem)."""
+    return min(w.n, 4096) if w.causal else w.n
 
 
-def oracle_run(w, units: int, ch_rms_target: float = 0.0) -> float:
-    """Runs the fp64 oracle (fwd, and bwd for training workloads) on the first
-    `units` (batch, head) units of the workload's own input streams; returns
-    the wall time in seconds."""
+def oracle_run(w, units: int, ch_rms_target: float = 0.0, rows: int | None = None) -> float:
+    """Runs the fp64 oracle (fwd, and bwd for training workloads) on the first `units` (batch, head) units of
+    the workload's own input streams, on their first `rows` tokens (default: all); returns the wall time in
+    seconds."""
     import oracle
+    n = w.n if rows is None else rows
     ln = None
     if w.len_range is not None:
         ln = synth.randint(w.seed, "attn.lengths", (w.B,), w.len_range[0], w.len_range[1]).astype(np.int32)
-    # (units, 1, n, d) has the same flat order as the first `units` heads of (B, H, n, d)
+    # (units, 1, w.n, d) has the same flat order as the first `units` heads of (B, H, n, d)
     shape = (units, 1, w.n, w.d)
-    Q = synth.IOTensor(synth.normal(w.seed, "attn.Q", shape) * w.qkv_scale, w.io).value
-    K = synth.IOTensor(synth.normal(w.seed, "attn.K", shape) * w.qkv_scale, w.io).value
-    V = synth.IOTensor(synth.normal(w.seed, "attn.V", (units, 1, w.n, w.dv)) * w.qkv_scale, w.io).value
-    dO = synth.IOTensor(synth.normal(w.seed, "attn.dO", (units, 1, w.n, w.dv)), w.io).value if w.backward else None
-    lengths = None if ln is None else np.array([ln[(u // w.H) % w.B] for u in range(units)], dtype=np.int32)
+    Q = synth.IOTensor(synth.normal(w.seed, "attn.Q", shape) * w.qkv_scale, w.io).value[:, :, :n]
+    K = synth.IOTensor(synth.normal(w.seed, "attn.K", shape) * w.qkv_scale, w.io).value[:, :, :n]
+    V = synth.IOTensor(synth.normal(w.seed, "attn.V", (units, 1, w.n, w.dv)) * w.qkv_scale, w.io).value[:, :, :n]
+    dO = (synth.IOTensor(synth.normal(w.seed, "attn.dO", (units, 1, w.n, w.dv)), w.io).value[:, :, :n]
+          if w.backward else None)
+    Q, K, V = (np.ascontiguousarray(t) for t in (Q, K, V))
+    dO = None if dO is None else np.ascontiguousarray(dO)
+    lengths = None if ln is None else np.array([min(n, ln[(u // w.H) % w.B]) for u in range(units)], dtype=np.int32)
     p = oracle.PhiParams(synth.phi_params(w.seed, w.d, w.M, w.L, w.hidden), ch_rms_target)
     t0 = time.perf_counter()
     oracle.attn_fwd(p, Q, K, V, lengths, w.causal, w.eps)
@@ -531,20 +604,25 @@ def oracle_run(w, units: int, ch_rms_target: float = 0.0) -> float:
     return time.perf_counter() - t0
 
 
-def tokens_per_s(w, units, seconds) -> float:
-    # one step = B*H units = B*n tokens
-    return w.n / (w.H * seconds / units)
+def tokens_per_s(w, units, seconds, rows=None) -> float:
+    """Tokens per second of a sample of `units` (batch, head) units of `rows` tokens each: one token of the
+    workload is one position of one sequence over all H heads."""
+    rows = w.n if rows is None else rows
+    return units * rows / (w.H * seconds)
 
 
 def cpu_baseline(w, target_s, ch_rms_target=0.0):
     import oracle
     threads = oracle.max_threads()
-    t1 = oracle_run(w, threads, ch_rms_target)
+    rows = sample_rows(w)
+    t1 = oracle_run(w, threads, ch_rms_target, rows)
     units = int(min(max(threads, threads * round(target_s / max(t1, 1e-3))), 4 * w.B * w.H))
-    t = oracle_run(w, units, ch_rms_target) if units != threads else t1
-    return {"value": tokens_per_s(w, units, t), "unit": "tokens/s", "cores": threads, "kind": "oracle",
-            "sample": f"{units} (batch, head) units of {w.n} tokens, fwd{'+bwd' if w.backward else ''}, "
-                      f"{t:.1f} s on {threads} threads, scaled to B*H={w.B * w.H} units per step"}
+    t = oracle_run(w, units, ch_rms_target, rows) if units != threads else t1
+    return {"value": tokens_per_s(w, units, t, rows), "unit": "tokens/s", "cores": threads, "kind": "oracle",
+            "sample": f"{units} (batch, head) units of {rows} tokens"
+                      + (f" (the first {rows} of each {w.n}-token sequence)" if rows < w.n else "")
+                      + f", fwd{'+bwd' if w.backward else ''}, {t:.1f} s on {threads} threads; tokens/s scaled "
+                        f"from the sample (value = units * rows / H / seconds)"}
 
 
 def run_reference(args, w):
@@ -553,19 +631,25 @@ def run_reference(args, w):
         return None
     import oracle
     threads = oracle.max_threads()
+    rows = sample_rows(w)
     if args.warmup > 0:
-        oracle_run(w, 1, args.ch_rms_target)
-    per = []
+        oracle_run(w, 1, args.ch_rms_target, min(rows, 256))
+    per, secs = [], []
     for _ in range(args.steps):
-        t = oracle_run(w, threads, args.ch_rms_target)
-        per.append(tokens_per_s(w, threads, t))
+        t = oracle_run(w, threads, args.ch_rms_target, rows)
+        secs.append(t)
+        per.append(tokens_per_s(w, threads, t, rows))
     value = statistics.median(per)
-    sample = f"{threads} (batch, head) units of {w.n} tokens per step on {threads} threads"
+    sample = (f"{threads} (batch, head) units of {rows} tokens per step"
+              + (f" (the first {rows} of each {w.n}-token sequence)" if rows < w.n else "")
+              + f" on {threads} threads, {statistics.median(secs):.2f} s each")
     return {"metric": METRIC, "value": value, "unit": "tokens/s", "n_gpus": world, "steps": args.steps,
             "warmup": args.warmup, "ms_per_step": w.tokens / value * 1e3, "higher_is_better": True,
+            "ms_per_step_kind": "extrapolated: the time the oracle would take for one whole step (B*H units of "
+                                "n tokens) at the sample's rate; each timed step ran the sample only",
+            "sample_seconds_per_step": statistics.median(secs),
             "scaling": "weak", "vs_baseline": None, "dtype": "f64", "data": "synthetic", "impl": "reference",
-            "config": {"workload": f"{w.name}: B={w.B} H={w.H} n={w.n} d={w.d} D={w.D}, fp64 CPU oracle"
-                                   + ch_rms_label(args),
+            "config": {"workload": workload_label(w, args.ch_rms_target) + ", fp64 CPU oracle",
                        "global_batch": w.B, "seq_len": w.n, "parallelism": "cpu"},
             "cpu_baseline": {"value": value, "unit": "tokens/s", "cores": threads, "kind": "oracle",
                              "sample": sample},

@@ -251,10 +251,28 @@ luna_status luna_selftest_wait(void *workspace, int64_t limit_ns, void *stream);
  * per device and leave their contents in it; each call clears what must start
  * at zero.  Calls whose executions overlap on the GPU (different streams, or
  * different host threads) race on the array and give undefined results: order
- * them on one stream. */
+ * them on one stream.  The cached address is that of the device's primary
+ * context: after cudaDeviceReset the array may move, and the library must not
+ * be used on that device again in the same process.
+ *
+ * A bounded device-side wait of the call that ran out sets the status word at
+ * the start of the array, as luna_attn_fwd does in its workspace (O is then
+ * undefined); the next call clears it.  luna_noalloc_scratch gives the array's
+ * address, so that luna_device_status(scratch, stream) reports the status of
+ * the last call on the device. */
 luna_status luna_attn_fwd_noalloc(const luna_attn_desc *ad, const luna_phi_desc *pd, const void *table,
                                   const void *Q, const void *K, const void *V, const int32_t *lengths, void *O,
                                   void *stream);
+
+/* Device address and size of the scratch array of luna_attn_fwd_noalloc on the
+ * current device (the same set-up as that call's first use: make the first call
+ * before any stream capture).  Allocates nothing.  The address serves
+ * luna_device_status, which reads and clears the status word of the last
+ * luna_attn_fwd_noalloc call on this device, and luna_selftest_wait; the rest of
+ * the array is the no-allocation call's scratch and must not be written while
+ * such a call may be in flight.  The paper has no counterpart.
+ * LUNA_ERR_INVALID_ARG for NULL arguments, LUNA_ERR_CUDA if the lookup fails. */
+luna_status luna_noalloc_scratch(void **scratch, size_t *bytes);
 
 /* Kernel timing (tracing aid, not needed for computation).  After
  * luna_profile_start(name), every launch of the library kernel `name` (e.g.

@@ -46,6 +46,18 @@ struct Plan {
     TcPlan tc;
 };
 
+// Fixed state-segment length of the streaming form (tuning and tests: LUNA_CAUSAL_SEG_ROWS, a multiple of
+// 128 rows).  The segment length decides the layout of the forward state that luna_attn_bwd,
+// luna_state_final and luna_attn_decode read back, so the variable is read once, when the library is
+// loaded, and every call of the process plans with the same value.
+int read_seg_rows_override() {
+    const char *env = getenv("LUNA_CAUSAL_SEG_ROWS");
+    if (!env) return 0;
+    const long v = atol(env);
+    return (v >= 128 && v % 128 == 0 && v < (1L << 24)) ? (int)v : 0;
+}
+const int g_seg_rows_override = read_seg_rows_override();
+
 struct Bump {
     size_t n = 0;
     size_t take(size_t bytes) {
@@ -86,10 +98,7 @@ luna_status make_plan(const luna_attn_desc *ad, const luna_phi_desc *pd, Plan &p
         p.nsplit_b = (int)cdiv(n, p.rps_b);
         int64_t nc = std::min<int64_t>(std::min<int64_t>(target, 64), cdiv(n, 16));
         p.seg_len = (int)round_up(cdiv(n, nc), 128);  // whole 128-row tiles (tensor-core streaming form)
-        if (const char *env = getenv("LUNA_CAUSAL_SEG_ROWS")) {  // tuning and tests: fixed segment length
-            const long v = atol(env);
-            if (v >= 128 && v % 128 == 0 && v < (1L << 24)) p.seg_len = (int)v;
-        }
+        if (g_seg_rows_override > 0) p.seg_len = g_seg_rows_override;
         p.nseg = (int)cdiv(n, p.seg_len);
     }
     const size_t f = sizeof(float);

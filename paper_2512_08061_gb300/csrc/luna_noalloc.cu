@@ -20,7 +20,9 @@ constexpr int kMaxDevices = 64;
 std::mutex g_mu;
 void *g_scratch_ptr[kMaxDevices] = {nullptr};
 
-// Device address of the scratch array on the current device (set-up on first use).
+// Device address of the scratch array on the current device (set-up on first use).  The cached address
+// belongs to the device's primary context: after cudaDeviceReset the module is loaded again and the
+// array may move, so the library must not be used on that device after a reset.
 luna_status scratch_for_current_device(void **out) {
     int dev = -1;
     if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= kMaxDevices) return LUNA_ERR_CUDA;
@@ -50,4 +52,14 @@ extern "C" luna_status luna_attn_fwd_noalloc(const luna_attn_desc *ad, const lun
     // (status word and arrival counters) on `stream` before its kernels run.
     return luna_attn_fwd(ad, pd, table, Q, K, V, lengths, O, nullptr, scratch, (size_t)LUNA_NOALLOC_SCRATCH_BYTES,
                          stream);
+}
+
+extern "C" luna_status luna_noalloc_scratch(void **scratch, size_t *bytes) {
+    if (!scratch || !bytes) return LUNA_ERR_INVALID_ARG;
+    void *p = nullptr;
+    const luna_status st = scratch_for_current_device(&p);
+    if (st != LUNA_OK) return st;
+    *scratch = p;
+    *bytes = (size_t)LUNA_NOALLOC_SCRATCH_BYTES;
+    return LUNA_OK;
 }

@@ -15,7 +15,7 @@ constexpr int kMaxRecords = 4096;
 
 struct Profiler {
     std::mutex mu;
-    bool on = false;
+    std::atomic<bool> on{false};  // read without the lock on every launch; the name is compared under it
     char name[64] = {0};
     std::vector<cudaEvent_t> ev;  // 2 per record
     int used = 0;
@@ -34,18 +34,19 @@ std::atomic<unsigned long long> g_launches{0};
 void prof_before(const char *kernel, cudaStream_t s) {
     g_launches.fetch_add(1, std::memory_order_relaxed);
     Profiler &p = prof();
-    if (!p.on || strcmp(kernel, p.name) != 0) return;
+    if (!p.on.load(std::memory_order_acquire)) return;
     std::lock_guard<std::mutex> g(p.mu);
-    if (p.used >= kMaxRecords) return;
+    if (!p.on.load(std::memory_order_relaxed) || strcmp(kernel, p.name) != 0 || p.used >= kMaxRecords) return;
     cudaEventRecord(p.ev[2 * p.used], s);
     p.open = true;
 }
 
 void prof_after(const char *kernel, cudaStream_t s) {
     Profiler &p = prof();
-    if (!p.on || strcmp(kernel, p.name) != 0) return;
+    if (!p.on.load(std::memory_order_acquire)) return;
     std::lock_guard<std::mutex> g(p.mu);
-    if (!p.open || p.used >= kMaxRecords) return;
+    if (!p.on.load(std::memory_order_relaxed) || strcmp(kernel, p.name) != 0 || !p.open || p.used >= kMaxRecords)
+        return;
     cudaEventRecord(p.ev[2 * p.used + 1], s);
     p.used++;
     p.open = false;
@@ -74,7 +75,7 @@ luna_status luna_profile_start(const char *kernel) {
     strncpy(p.name, kernel, sizeof(p.name) - 1);
     p.used = 0;
     p.open = false;
-    p.on = true;
+    p.on.store(true, std::memory_order_release);
     return LUNA_OK;
 }
 
@@ -82,7 +83,7 @@ luna_status luna_profile_stop(double *total_ms, int *launches) {
     if (!total_ms || !launches) return LUNA_ERR_INVALID_ARG;
     Profiler &p = prof();
     std::lock_guard<std::mutex> g(p.mu);
-    p.on = false;
+    p.on.store(false, std::memory_order_release);
     double tot = 0.0;
     for (int i = 0; i < p.used; ++i) {
         if (cudaEventSynchronize(p.ev[2 * i + 1]) != cudaSuccess) return LUNA_ERR_CUDA;

@@ -20,6 +20,8 @@
 //   MMA U, workers phi(Q) (bf16) and the fp32 normaliser phi.z,
 //   MMA  num = phi [S_hi; S_lo]^T,  O = num / (phi.z + eps)
 // S and W enter their products split into bf16 hi + lo parts.
+#include <atomic>
+
 #include "luna_tc_dev.cuh"
 
 namespace luna {
@@ -820,13 +822,20 @@ __global__ void __launch_bounds__(kSplitThreads) k_tile_split(AttnArgs a, int G,
     }
 }
 
+// SM count of the current device, cached per device ordinal (host threads may plan for different
+// devices at once; a racing first lookup stores the same value twice).
 int sm_count_impl() {
-    static int n = 0;
-    if (n == 0) {
-        int dev = 0;
-        if (cudaGetDevice(&dev) != cudaSuccess || cudaDeviceGetAttribute(&n, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess || n <= 0)
-            n = 148;
+    constexpr int kMaxDev = 64;
+    static std::atomic<int> cache[kMaxDev];
+    int dev = 0;
+    if (cudaGetDevice(&dev) != cudaSuccess) return 148;
+    if (dev >= 0 && dev < kMaxDev) {
+        const int c = cache[dev].load(std::memory_order_relaxed);
+        if (c > 0) return c;
     }
+    int n = 0;
+    if (cudaDeviceGetAttribute(&n, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess || n <= 0) return 148;
+    if (dev >= 0 && dev < kMaxDev) cache[dev].store(n, std::memory_order_relaxed);
     return n;
 }
 

@@ -80,6 +80,7 @@ def _load():
                               ctypes.POINTER(I64)], I),
         "luna_attn_decode": ([ad, pd, P, P, P, P, P, P, I64, P, I64, P], I),
         "luna_selftest_wait": ([P, I64, P], I),
+        "luna_noalloc_scratch": ([ctypes.POINTER(P), ctypes.POINTER(S)], I),
     }
     for name, (args, res) in sig.items():
         fn = getattr(lib, name)
@@ -92,12 +93,15 @@ _lib = _load()
 EXPORTED = ("luna_status_string", "luna_version", "luna_phi_table_size", "luna_phi_prepare", "luna_featmap",
             "luna_workspace_size", "luna_state_size", "luna_attn_fwd", "luna_attn_bwd", "luna_device_status",
             "luna_profile_start", "luna_profile_stop", "luna_launch_count", "luna_attn_fwd_noalloc",
-            "luna_state_final", "luna_attn_decode", "luna_selftest_wait")
+            "luna_state_final", "luna_attn_decode", "luna_selftest_wait", "luna_noalloc_scratch")
 
 
 def _ptr(t):
+    """Device address of a tensor, or a raw address given as an int."""
     if t is None:
         return None
+    if isinstance(t, int):
+        return ctypes.c_void_p(t)
     return ctypes.c_void_p(t.data_ptr())
 
 
@@ -205,6 +209,13 @@ def luna_attn_decode(ad, pd, table, q, k, v, o, S, S_stride, z, z_stride, stream
 
 def luna_device_status(workspace: torch.Tensor, stream=None) -> int:
     return _lib.luna_device_status(_ptr(workspace), _stream(stream))
+
+
+def luna_noalloc_scratch() -> tuple[int, int]:
+    """(device address, bytes) of the no-allocation entry point's scratch array on the current device."""
+    p, n = ctypes.c_void_p(), ctypes.c_size_t(0)
+    _check(_lib.luna_noalloc_scratch(ctypes.byref(p), ctypes.byref(n)), "luna_noalloc_scratch")
+    return p.value, n.value
 
 
 def luna_selftest_wait(workspace: torch.Tensor, limit_ns: int, stream=None) -> None:

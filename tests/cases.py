@@ -59,6 +59,55 @@ def sum_err(got, ref, abs_terms, tol) -> float:
     return float(np.max(np.where(bound > 0, err / np.where(bound > 0, bound, 1.0), np.where(err > 0, np.inf, 0.0))))
 
 
+# ---------------------------------------------------------------------------
+# guard bands (the sanitizer's out-of-bounds checks are not available): every
+# buffer the library writes in the parity tests sits between two bands of a
+# known byte pattern that must still be intact after each call
+
+GUARD_BYTES = 4096  # keeps the 256-byte alignment the library asks for
+GUARD_PATTERN = 0x5A
+
+
+def guarded_bytes(nbytes: int, device, registry: list):
+    """A uint8 device buffer of nbytes between two guard bands; the band is recorded in `registry`."""
+    import torch
+    base = torch.full((int(nbytes) + 2 * GUARD_BYTES,), GUARD_PATTERN, dtype=torch.uint8, device=device)
+    registry.append((base, int(nbytes)))
+    return base[GUARD_BYTES:GUARD_BYTES + int(nbytes)]
+
+
+def guarded_empty(shape, dtype, device, registry: list):
+    """An uninitialised-looking tensor (filled with the guard pattern) of `shape` and `dtype` between guard bands."""
+    import torch
+    n = int(np.prod(shape)) * torch.empty((), dtype=dtype).element_size()
+    return guarded_bytes(n, device, registry).view(dtype).view(tuple(shape))
+
+
+def check_guards(registry: list) -> None:
+    """Asserts that no guard band of `registry` was written."""
+    import torch
+    torch.cuda.synchronize()
+    for base, n in registry:
+        for band in (base[:GUARD_BYTES], base[GUARD_BYTES + n:]):
+            bad = torch.nonzero(band != GUARD_PATTERN)
+            assert bad.numel() == 0, f"guard band of a {n}-byte buffer written at byte {int(bad[0, 0])}"
+
+
+def run_in_child(module: str, func: str, args=(), env=None, timeout=1200) -> None:
+    """Runs tests/<module>.<func>(*args) in a fresh Python process with extra environment variables, for
+    settings the library reads once, when it is loaded; fails with the child's output if the child fails."""
+    import os
+    import subprocess
+    import sys
+    tests = os.path.dirname(os.path.abspath(__file__))
+    root = os.path.dirname(tests)
+    code = f"import sys; sys.path[:0] = [{root!r}, {tests!r}]; import {module} as m; m.{func}(*{tuple(args)!r})"
+    e = dict(os.environ)
+    e.update(env or {})
+    r = subprocess.run([sys.executable, "-c", code], env=e, capture_output=True, text=True, timeout=timeout)
+    assert r.returncode == 0, (r.stdout[-3000:] + "\n" + r.stderr[-6000:])
+
+
 def to_device(t: "synth.IOTensor"):
     import torch
     if t.io == "f32":
@@ -86,24 +135,42 @@ class Case:
 
     # ---- device side
     def luna(self, chunk=0):
+        """The library object for this case, its table, workspace and state buffers between guard bands."""
         import torch
         import paper_2512_08061_gb300.luna as L
         lu = L.Luna(self.B, self.H, self.n, self.d, self.dv, self.M, self.L, self.hidden, self.causal, self.eps,
                     torch.float32 if self.io == "f32" else torch.bfloat16, chunk, shared=self.shared,
                     ch_rms_target=self.ch_rms_target)
+        self.guards = []
+        for name in ("table", "ws", "state"):
+            setattr(lu, name, guarded_bytes(getattr(lu, name).numel(), lu.device, self.guards))
         params = {k: torch.from_numpy(v).cuda() for k, v in self.params.items()}
         lu.prepare(params)
         self.dev = {k: to_device(self.inp[k]) for k in ("Q", "K", "V", "dO") if k in self.inp}
         self.dev["lengths"] = None if self.lengths is None else torch.from_numpy(self.lengths).cuda()
+        check_guards(self.guards)
         return lu
 
     def run_fwd(self, lu, save_state=True):
         d = self.dev
-        return lu.forward(d["Q"], d["K"], d["V"], d["lengths"], save_state=save_state)
+        O = guarded_empty(tuple(d["V"].shape), d["V"].dtype, d["V"].device, self.guards)
+        out = lu.forward(d["Q"], d["K"], d["V"], d["lengths"], O=O, save_state=save_state)
+        check_guards(self.guards)
+        return out
 
     def run_bwd(self, lu, use_state=True):
+        import torch
         d = self.dev
-        return lu.backward(d["Q"], d["K"], d["V"], d["dO"], d["lengths"], use_state=use_state)
+        dev = d["Q"].device
+        fc1 = (self.hidden,) if self.shared else (self.L, self.hidden)
+        shapes = {"dQ": (tuple(d["Q"].shape), d["Q"].dtype), "dK": (tuple(d["K"].shape), d["K"].dtype),
+                  "dV": (tuple(d["V"].shape), d["V"].dtype), "dW": ((self.M, self.d), torch.float32),
+                  "db": ((self.M,), torch.float32), "dw1": (fc1, torch.float32), "db1": (fc1, torch.float32),
+                  "dw2": ((self.L, self.hidden), torch.float32), "db2": ((self.L,), torch.float32)}
+        out = {k: guarded_empty(shp, dt, dev, self.guards) for k, (shp, dt) in shapes.items()}
+        g = lu.backward(d["Q"], d["K"], d["V"], d["dO"], d["lengths"], use_state=use_state, out=out)
+        check_guards(self.guards)
+        return g
 
     # ---- oracle side
     @property

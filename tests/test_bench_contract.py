@@ -74,3 +74,33 @@ def test_algorithmic_bytes_by_hand():
     assert bench.kernel_bytes(w, ln, "chrms_stats") == 2 * 356 * row
     assert bench.kernel_bytes(w, ln, "chrms_kterm") == 2 * 356 * 3 * row
     assert bench.kernel_bytes(w, ln, "no_such_kernel") == 0.0
+
+
+def test_streaming_form_algorithmic_bytes_by_hand():
+    """The streaming-form stages count only the method's tensors they read or write:
+    B = 1, H = 2, n = 300, d = dv = 128, bf16 (a row is 256 B), no padding: 600 rows.
+    The stage that reads only another stage's rows has no algorithmic bytes."""
+    sys.path.insert(0, ROOT)
+    import dataclasses
+    import bench
+    from synth.workloads import WORKLOADS
+    w = dataclasses.replace(WORKLOADS["causal_long"], B=1, H=2, n=300)
+    row = 128 * 2
+    assert bench.kernel_bytes(w, None, "tc_causal") == 600 * 3 * row + 600 * row  # Q, K, V; O
+    assert bench.kernel_bytes(w, None, "tc_keys") == 600 * 2 * row                 # K, V
+    assert bench.kernel_bytes(w, None, "tcc_query") == 600 * 4 * row               # Q, K, V, dO
+    assert bench.kernel_bytes(w, None, "tcc_dstats") == 0.0
+    assert bench.kernel_bytes(w, None, "tcc_key") == 600 * 2 * row + 600 * row     # V, dO; dV
+    assert bench.kernel_bytes(w, None, "tc_phi_bwd") == 600 * row + 600 * row      # X; dX
+    # the whole step: read Q, K, V and write O; read Q, K, V, dO and write dQ, dK, dV
+    assert bench.step_bytes(w, None) == 600 * row * (4 + 7)
+
+
+def test_reference_arm_streaming_form_sample_is_bounded_and_labelled():
+    """The streaming-form workload's reference arm times a prefix sample of each sequence and says that its
+    per-step time is extrapolated from the sample's rate."""
+    d = _run("--impl", "reference", "--workload", "causal_long", "--steps", "1", "--warmup", "0")
+    assert d["impl"] == "reference" and d["value"] > 0
+    assert "first 4096" in d["cpu_baseline"]["sample"]
+    assert d["ms_per_step_kind"].startswith("extrapolated")
+    assert d["sample_seconds_per_step"] < 60

@@ -12,7 +12,7 @@ import pytest
 
 import oracle
 import synth
-from cases import TOL, Case, relerr, relerr_rows, sum_err, to_device, to_host
+from cases import TOL, Case, relerr, relerr_rows, run_in_child, sum_err, to_device, to_host
 
 pytestmark = pytest.mark.gpu
 
@@ -121,12 +121,16 @@ def test_forward_tensor_core_tile_loops(d, M, tiles, monkeypatch):
 
 
 @pytest.mark.parametrize("seg_rows", ["128", "384", "1280"])
-def test_forward_tensor_core_causal(seg_rows, monkeypatch):
+def test_forward_tensor_core_causal(seg_rows):
     """Streaming form through the tensor-core kernels (d = 128, M = 16): state
     segments of 1, 3 and 9 tiles (the running state carried across tiles in
     TMEM), a ragged last tile, a sequence with padding and segments that hold
-    no valid row."""
-    monkeypatch.setenv("LUNA_CAUSAL_SEG_ROWS", seg_rows)
+    no valid row.  The library reads the segment length once, when it is
+    loaded, so each length runs in a process of its own."""
+    run_in_child("test_gpu_parity", "check_forward_tensor_core_causal", env={"LUNA_CAUSAL_SEG_ROWS": seg_rows})
+
+
+def check_forward_tensor_core_causal():
     case = Case(2, 2, 1100, 128, 16, 8, "bf16", True, seed=59, qkv_scale=1.0 / math.sqrt(128),
                 lengths=[1100, 333])
     lu = case.luna()
@@ -263,7 +267,7 @@ def test_backward_tensor_core_balanced_split(d, tiles, monkeypatch):
 
 
 @pytest.mark.parametrize("d,M,causal", [(32, 8, False), (64, 8, False), (128, 16, True)])
-def test_backward_tensor_core_histogram_ranges(d, M, causal, monkeypatch):
+def test_backward_tensor_core_histogram_ranges(d, M, causal):
     """The fixed-point interval histogram of the channel-MLP gradient
     statistics when the output gradient is zero on the first 300 rows of every
     sequence (no scale until a later tile) and then grows by four orders of
@@ -271,10 +275,14 @@ def test_backward_tensor_core_histogram_ranges(d, M, causal, monkeypatch):
     scales taken from the group before it and its large values go to the
     unscaled fallback.  One work item per head (18 tiles of 128 rows), so that
     a block walks more than one group (16 tiles of 128 rows x 8 projections,
-    8 tiles of 128 x 16)."""
+    8 tiles of 128 x 16).  Runs in a process of its own with the segment length
+    set (the library reads it once, when it is loaded)."""
+    run_in_child("test_gpu_parity", "check_backward_histogram_ranges", (d, M, causal),
+                 env={"LUNA_TC_TILES_PER_SPLIT": "18", "LUNA_CAUSAL_SEG_ROWS": "2304"})
+
+
+def check_backward_histogram_ranges(d, M, causal):
     n = 2200
-    monkeypatch.setenv("LUNA_TC_TILES_PER_SPLIT", "18")
-    monkeypatch.setenv("LUNA_CAUSAL_SEG_ROWS", "2304")
     case = Case(2, 2, n, d, M, 8, "bf16", causal, seed=83, qkv_scale=1.0 / math.sqrt(d), with_grad=True)
     ramp = 10.0 ** (4.0 * np.arange(n) / n)
     ramp[:300] = 0.0
@@ -286,12 +294,16 @@ def test_backward_tensor_core_histogram_ranges(d, M, causal, monkeypatch):
 
 
 @pytest.mark.parametrize("seg_rows", ["128", "384", "1280"])
-def test_backward_tensor_core_causal(seg_rows, monkeypatch):
+def test_backward_tensor_core_causal(seg_rows):
     """Streaming-form backward through the tensor-core kernels (d = 128, M = 16):
     state segments of 2, 6 and 20 tiles of 64 rows (the running S and dS carried
     across tiles in TMEM, the reverse scan of the segment sums), ragged last
-    tiles, a sequence with padding and segments that hold no valid row."""
-    monkeypatch.setenv("LUNA_CAUSAL_SEG_ROWS", seg_rows)
+    tiles, a sequence with padding and segments that hold no valid row.  One
+    process per segment length (read once, when the library is loaded)."""
+    run_in_child("test_gpu_parity", "check_backward_tensor_core_causal", env={"LUNA_CAUSAL_SEG_ROWS": seg_rows})
+
+
+def check_backward_tensor_core_causal():
     case = Case(2, 2, 1100, 128, 16, 8, "bf16", True, seed=61, qkv_scale=1.0 / math.sqrt(128),
                 lengths=[1100, 333], with_grad=True)
     lu = case.luna()

@@ -47,6 +47,7 @@ def test_noalloc_forward_matches_workspace_forward_on_two_calls():
         got = _noalloc_forward(case, lu)
         assert np.all(np.isfinite(got))
         assert relerr(got, ref) < TOL[case.io]
+        assert relerr(got, case.oracle_fwd()) < TOL[case.io]
         for b, ln in enumerate(case.lengths):
             assert np.all(got[b, :, ln:] == 0)
 
@@ -61,3 +62,23 @@ def test_noalloc_rejects_problems_beyond_the_scratch_array():
     with pytest.raises(L.LunaError) as e:
         L.luna_attn_fwd_noalloc(ad, pd, dummy, dummy, dummy, dummy, None, dummy)
     assert e.value.status == 3  # LUNA_ERR_WORKSPACE, returned before any launch
+
+
+def test_noalloc_status_word_reports_a_timed_out_wait():
+    """The status word at the start of the scratch array is read through
+    luna_noalloc_scratch + luna_device_status: a bounded wait that ran out in
+    that array (the self-test) is reported once, and the next no-allocation
+    call clears the word and computes as before."""
+    import paper_2512_08061_gb300.luna as L
+    case = Case(2, 2, 300, 32, 8, 8, "bf16", False, seed=43, qkv_scale=1 / math.sqrt(32), lengths=[300, 77])
+    lu = case.luna()
+    first = _noalloc_forward(case, lu)
+    scratch, nbytes = L.luna_noalloc_scratch()
+    assert scratch != 0 and nbytes == L.NOALLOC_SCRATCH_BYTES
+    assert L.luna_device_status(scratch) == 0
+    L.luna_selftest_wait(scratch, 10_000_000)
+    assert L.luna_device_status(scratch) == 5  # LUNA_ERR_DEVICE_TIMEOUT
+    assert L.luna_device_status(scratch) == 0  # read once, then cleared
+    again = _noalloc_forward(case, lu)
+    assert np.array_equal(first, again)
+    assert L.luna_device_status(scratch) == 0
