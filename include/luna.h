@@ -178,6 +178,30 @@ luna_status luna_attn_bwd(const luna_attn_desc *ad, const luna_phi_desc *pd, con
                           const void *state, void *dQ, void *dK, void *dV, const luna_phi_grads *grads,
                           void *workspace, size_t ws_bytes, void *stream);
 
+/* Attention weights of query rows [row0, row0 + rows) of every (b, h), for the
+ * conversion of a softmax model (appendix, "Stage 1: attention distillation":
+ * the feature-map parameters are trained so that the attention distribution the
+ * kernel induces matches the one of the original softmax module; the paper
+ * does not fix the loss, so this call only produces the distributions).
+ *   teacher = 0: the LUNA weights, Eq. (kernel-attn) read as a weighted average
+ *       of the values,  a_ij = k(q_i, k_j) / (sum_j' k(q_i, k_j') + eps),
+ *       k(x, y) = phi(x)^T phi(y), so that O_i = sum_j a_ij v_j exactly;
+ *   teacher = 1: the softmax weights of the same queries and keys,
+ *       p_ij = exp(q_i . k_j / sqrt(d)) / sum_j' exp(q_i . k_j' / sqrt(d))
+ *       (`table` may then be NULL).
+ * The sums run over the valid keys (j <= i with ad->causal = 1).  Keys outside
+ * them, query rows at or past the valid length, and rows whose guarded sum is
+ * exactly 0 get weight 0.  Q, K as in the conventions (ad->dv and ad->chunk are
+ * ignored); A: fp32 device array (B, H, rows, n), every entry written.
+ * 0 <= row0, 0 <= rows, row0 + rows <= n, else LUNA_ERR_INVALID_ARG;
+ * pd->ch_rms_target > 0 gives LUNA_ERR_UNSUPPORTED.  No workspace: each block
+ * of 32 rows writes its raw scores and normalises them in a second pass over
+ * its own rows.  The feature map is fp32 for both io types; each row's sum
+ * is accumulated in fp64. */
+luna_status luna_attn_weights(const luna_attn_desc *ad, const luna_phi_desc *pd, const void *table, const void *Q,
+                              const void *K, const int32_t *lengths, int row0, int rows, int teacher, float *A,
+                              void *stream);
+
 /* Location of the final state of a streaming-form forward pass (ad->causal = 1)
  * inside a `state` buffer written by luna_attn_fwd: the key statistics over all
  * valid tokens of each sequence, S = sum_j phi(k_j) v_j^T and z = sum_j phi(k_j)

@@ -9,7 +9,10 @@ Parity pins (tests/test_oracle_pins.py): hand-computed feature maps
 (tests/golden/phi_hand.json), brute-force quadratic form of Eq. (kernel-attn),
 constant-channel closed form, Gram matrix PSD (Prop. 1), permutation/padding/
 linearity invariances, normalised weights summing to 1, causal = masked
-quadratic form, and central finite differences of every gradient.
+quadratic form, and central finite differences of every gradient.  The
+attention weights of the conversion stage (tests/test_oracle_weights.py): their
+product with V is the linear form's output, rows sum to den/(den+eps), constant
+channels give uniform weights, the softmax teacher against a closed form.
 """
 from __future__ import annotations
 
@@ -71,6 +74,7 @@ def lib():
             L.oracle_attn_quadratic.argtypes = [phi, _I, _I, _I, _I, _I, _D, _P, _P, _P, _P, _P]
             L.oracle_attn_bwd.argtypes = [phi, _I, _I, _I, _I, _I, _D, _P, _P, _P, _P, _P, _P, _P, _P] + [_P] * 6
             L.oracle_ch_rms.argtypes = [phi, _P, _I, _I, _I, _P, _P, _P]
+            L.oracle_attn_weights.argtypes = [phi, _I, _I, _I, _I, _D, _P, _P, _P, _I, _I, _I, _P]
             L.oracle_max_threads.restype = _I
             L.oracle_set_threads.argtypes = [_I]
             L.oracle_set_abs_terms.argtypes = [_I]
@@ -227,6 +231,22 @@ def attn_quadratic(params, Q, K, V, lengths=None, causal=False, eps=1e-6) -> np.
     lib().oracle_attn_quadratic(p.ref(), B, H, n, dv, int(bool(causal)), float(eps),
                                 Q.ctypes.data, K.ctypes.data, V.ctypes.data, lp, O.ctypes.data)
     return O
+
+
+def attn_weights(params, Q, K, lengths=None, causal=False, eps=1e-6, row0=0, rows=None, teacher=False) -> np.ndarray:
+    """Attention weights of query rows [row0, row0 + rows) of every (b, h): (B, H, rows, n).
+    teacher=False: the LUNA weights a_ij = k(q_i,k_j) / (sum_j k + eps) (O = A V);
+    teacher=True: the softmax weights exp(q_i.k_j/sqrt(d)) / sum_j exp(...) over the same keys."""
+    p = _as_params(params)
+    Q, K = _f64(Q), _f64(K)
+    B, H, n, d = Q.shape
+    rows = n - row0 if rows is None else rows
+    assert p.heads in (0, H) and K.shape == Q.shape
+    la, lp = _lens(lengths, B)
+    A = np.empty((B, H, rows, n), dtype=np.float64)
+    lib().oracle_attn_weights(p.ref(), B, H, n, int(bool(causal)), float(eps), Q.ctypes.data, K.ctypes.data, lp,
+                              int(row0), int(rows), int(bool(teacher)), A.ctypes.data)
+    return A
 
 
 def attn_bwd_abs_terms(params, Q, K, V, dO, lengths=None, causal=False, eps=1e-6) -> dict:

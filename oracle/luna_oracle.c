@@ -444,6 +444,71 @@ void oracle_attn_quadratic(const oracle_phi *p, int B, int H, int n, int dv, int
 }
 
 /* ------------------------------------------------------------------------ */
+/* attention weights of a block of query rows (conversion, stage 1)          */
+
+/* The attention distribution that the kernel induces, Eq. (kernel-attn) read
+ * as a weighted average of the values: for query rows i in [row0, row0+rows)
+ * of every (b, h),
+ *     a_ij = k(q_i, k_j) / (sum_j' k(q_i, k_j') + eps),   k(x, y) = phi(x)^T phi(y),
+ * over the valid keys j (j <= i in the streaming form), 0 for the other keys, for
+ * query rows at or past the valid length, and for a row whose guarded sum is
+ * exactly 0.  So O_i = sum_j a_ij v_j.  A is (B, H, rows, n).
+ * With `teacher` non-zero, the softmax attention that the conversion distils
+ * from instead (appendix, stage 1: the teacher is the original softmax module):
+ *     p_ij = exp(q_i . k_j / sqrt(d)) / sum_j' exp(q_i . k_j' / sqrt(d))
+ * over the same keys, with the same zero rows and columns. */
+void oracle_attn_weights(const oracle_phi *p, int B, int H, int n, int causal, double eps, const double *Q,
+                         const double *K, const int32_t *lengths, int row0, int rows, int teacher, double *A) {
+    const int D = p->M * p->L, d = p->d;
+    side_maps sm;
+    side_maps_init(&sm, p, Q, K, B, H, n, lengths);
+#pragma omp parallel for schedule(dynamic, 1)
+    for (int bh = 0; bh < B * H; ++bh) {
+        const int len = head_len(lengths, bh / H, n);
+        const double *q = Q + (size_t)bh * n * d, *k = K + (size_t)bh * n * d;
+        double *a = A + (size_t)bh * rows * n;
+        memset(a, 0, sizeof(double) * (size_t)rows * n);
+        double *pq = (double *)malloc(sizeof(double) * D);
+        double *PK = (double *)malloc(sizeof(double) * (size_t)(len > 0 ? len : 1) * D);
+        const oracle_phi vq = head_view(&sm.pq, bh % H), vk = head_view(&sm.pk, bh % H);
+        for (int j = 0; j < len; ++j) phi_row(&vk, k + (size_t)j * d, PK + (size_t)j * D);
+        for (int r = 0; r < rows; ++r) {
+            const int i = row0 + r;
+            if (i < 0 || i >= len) continue;
+            const int jmax = causal ? i + 1 : len;
+            double *ar = a + (size_t)r * n;
+            if (teacher) {
+                double mx = -INFINITY;
+                for (int j = 0; j < jmax; ++j) {
+                    double s = 0.0;
+                    for (int c = 0; c < d; ++c) s += q[(size_t)i * d + c] * k[(size_t)j * d + c];
+                    ar[j] = s / sqrt((double)d);
+                    if (ar[j] > mx) mx = ar[j];
+                }
+                double tot = 0.0;
+                for (int j = 0; j < jmax; ++j) {
+                    ar[j] = exp(ar[j] - mx);
+                    tot += ar[j];
+                }
+                for (int j = 0; j < jmax; ++j) ar[j] /= tot;
+                continue;
+            }
+            phi_row(&vq, q + (size_t)i * d, pq);
+            double den = eps;
+            for (int j = 0; j < jmax; ++j) {
+                double kij = 0.0;
+                for (int f = 0; f < D; ++f) kij += pq[f] * PK[(size_t)j * D + f];
+                ar[j] = kij;
+                den += kij;
+            }
+            for (int j = 0; j < jmax; ++j) ar[j] = den == 0.0 ? 0.0 : ar[j] / den;
+        }
+        free(pq); free(PK);
+    }
+    free(sm.st);
+}
+
+/* ------------------------------------------------------------------------ */
 /* backward                                                                  */
 
 static void attn_bwd_head(const oracle_phi *pq_, const oracle_phi *pk_, int n, int dv, int causal, double eps,

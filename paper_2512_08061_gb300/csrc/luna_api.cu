@@ -128,8 +128,10 @@ luna_status make_plan(const luna_attn_desc *ad, const luna_phi_desc *pd, Plan &p
         p.o_dSfin = w.take((size_t)BH * SD * f);
         p.o_dzfin = w.take((size_t)BH * D * f);
         // with channel normalisation, the partials of the scale term of the backward follow
-        p.o_gpart = w.take((2 * (size_t)BH * p.nsplit_b + (p.ch_target > 0.0f ? 2 * kChKBlocks : 0)) * p.gsize * f);
-        p.o_hist = w.take((size_t)p.gsize * f);
+        // parameter-gradient partials: fp32 (tensor-core kernels) or fp64 (generic kernels)
+        p.o_gpart = w.take((2 * (size_t)BH * p.nsplit_b + (p.ch_target > 0.0f ? 2 * kChKBlocks : 0)) * p.gsize *
+                           sizeof(double));
+        p.o_hist = w.take((size_t)p.gsize * sizeof(double));
         p.ws_bwd = w.n;
         p.state_bytes = (size_t)BH * (SD + D) * f;
     } else {
@@ -144,8 +146,8 @@ luna_status make_plan(const luna_attn_desc *ad, const luna_phi_desc *pd, Plan &p
         p.o_segdS = w.take((size_t)BH * ns * SD * f);
         p.o_segdz = w.take((size_t)BH * ns * D * f);
         p.o_rowstat = w.take((size_t)BH * n * 2 * f);
-        p.o_gpart = w.take(2 * (size_t)BH * ns * p.gsize * f);
-        p.o_hist = w.take((size_t)p.gsize * f);
+        p.o_gpart = w.take(2 * (size_t)BH * ns * p.gsize * sizeof(double));
+        p.o_hist = w.take((size_t)p.gsize * sizeof(double));
         p.ws_bwd = w.n;
         p.state_bytes = (size_t)BH * (ns + 1) * (SD + D) * f;
     }
@@ -355,7 +357,7 @@ luna_status luna_attn_bwd(const luna_attn_desc *ad, const luna_phi_desc *pd, con
     a.dS_part = reinterpret_cast<float *>(w + p.o_dSpart);
     a.dz_part = reinterpret_cast<float *>(w + p.o_dzpart);
     a.gpart = reinterpret_cast<float *>(w + p.o_gpart);
-    a.hist = reinterpret_cast<float *>(w + p.o_hist);
+    a.hist = reinterpret_cast<double *>(w + p.o_hist);
     if (!ad->causal) {
         a.dS_fin = reinterpret_cast<float *>(w + p.o_dSfin);
         a.dz_fin = reinterpret_cast<float *>(w + p.o_dzfin);
@@ -383,6 +385,36 @@ luna_status luna_attn_bwd(const luna_attn_desc *ad, const luna_phi_desc *pd, con
     if (p.tc.eligible && tc_inputs_ok(p.tc, Q, K, V, dO) && tc_inputs_ok(p.tc, dQ, dK, dV, nullptr))
         return cuda_status(launch_tc_bwd(p.tc, a, w, state != nullptr, s));
     return cuda_status(launch_simt_bwd(a, ad->io, state != nullptr, s));
+}
+
+luna_status luna_attn_weights(const luna_attn_desc *ad, const luna_phi_desc *pd, const void *table, const void *Q,
+                              const void *K, const int32_t *lengths, int row0, int rows, int teacher, float *A,
+                              void *stream) {
+    if (!ad) return LUNA_ERR_INVALID_ARG;
+    if (ad->B < 0 || ad->H < 0 || ad->n < 0 || ad->d < 1 || ad->dv < 1) return LUNA_ERR_INVALID_ARG;
+    if (ad->io != LUNA_F32 && ad->io != LUNA_BF16) return LUNA_ERR_INVALID_ARG;
+    if (ad->causal != 0 && ad->causal != 1) return LUNA_ERR_INVALID_ARG;
+    if (!(ad->eps >= 0.0f) || isinf(ad->eps)) return LUNA_ERR_INVALID_ARG;
+    if (teacher != 0 && teacher != 1) return LUNA_ERR_INVALID_ARG;
+    if (row0 < 0 || rows < 0 || (int64_t)row0 + rows > ad->n) return LUNA_ERR_INVALID_ARG;
+    luna_status st = check_phi(pd, ad->d);
+    if (st != LUNA_OK) return st;
+    if (pd->ch_rms_target > 0.0f) return LUNA_ERR_UNSUPPORTED;  // batch statistics: not for a block of rows
+    if (ad->n > (1 << 24) || (int64_t)ad->B * ad->H > 65535) return LUNA_ERR_UNSUPPORTED;
+    if ((int64_t)ad->B * ad->H == 0 || rows == 0 || ad->n == 0) return LUNA_OK;
+    if (!Q || !K || !A || (!teacher && !table)) return LUNA_ERR_INVALID_ARG;
+    if (table && !aligned(table, 256)) return LUNA_ERR_INVALID_ARG;
+    AttnArgs a;
+    memset(&a, 0, sizeof(a));
+    a.B = ad->B; a.H = ad->H; a.n = ad->n; a.d = ad->d; a.dv = ad->dv;
+    a.lay = table_layout(pd->M, pd->L, pd->hidden, ad->d, pd->shared_channels);
+    a.M = a.lay.M; a.L = a.lay.L; a.D = a.lay.D;
+    a.eps = ad->eps;
+    a.table = static_cast<const char *>(table);
+    a.Q = Q; a.K = K;
+    a.lengths = lengths;
+    if (weights_max_smem(a) > kMaxSmem) return LUNA_ERR_UNSUPPORTED;
+    return cuda_status(launch_weights(a, ad->io, ad->causal, row0, rows, teacher, A, static_cast<cudaStream_t>(stream)));
 }
 
 luna_status luna_state_final(const luna_attn_desc *ad, const luna_phi_desc *pd, void *state, float **S,

@@ -168,9 +168,9 @@ __global__ void __launch_bounds__(kThreads) k_causal_bwd_seg(AttnArgs a) {
         chunk_outputs(a, S, z, sPq, sA, sV, nr, sden, sO);
         __syncthreads();
         for (int r = threadIdx.x; r < nr; r += blockDim.x) {
-            float dot = 0.0f;
-            for (int c = 0; c < dv; ++c) dot = fmaf(sdO[r * dv + c], sO[r * dv + c], dot);
-            const float dd = (sden[r] != 0.0f) ? -dot / sden[r] : 0.0f;
+            double dot = 0.0;  // dden and dphi are formed in fp64 and rounded once: they cancel
+            for (int c = 0; c < dv; ++c) dot = fma((double)sdO[r * dv + c], (double)sO[r * dv + c], dot);
+            const float dd = (sden[r] != 0.0f) ? (float)(-dot / (double)sden[r]) : 0.0f;
             sdden[r] = dd;
             float *rs = a.rowstat + ((size_t)bh * a.n + t0 + r) * 2;
             rs[0] = sden[r];
@@ -212,8 +212,9 @@ __global__ void __launch_bounds__(kThreads) k_causal_dq(AttnArgs a) {
     float *sU = cv.take(kCs * M);
     int *sJ = reinterpret_cast<int *>(cv.take(kCs * M));
     float *sdU = cv.take(kCs * M);
-    float *shist = cv.take(lay.nint * lay.L * 2);
     const int bh = blockIdx.y, seg = blockIdx.x;
+    double *gp = reinterpret_cast<double *>(a.gpart) + ((size_t)bh * a.nseg + seg) * a.gsize;
+    double *shist = gp + M * d + M;  // the block's fp64 histogram, accumulated in place by L2 atomics
     const int len = head_length(a.lengths, bh / a.H, a.n);
     const int r0 = seg * a.seg_len, rend = min(a.n, r0 + a.seg_len), r1 = min(len, rend);
     IO *dQ = static_cast<IO *>(a.dQ) + (size_t)bh * a.n * d;
@@ -222,7 +223,7 @@ __global__ void __launch_bounds__(kThreads) k_causal_dq(AttnArgs a) {
     const size_t so = ((size_t)bh * (a.nseg + 1) + seg);
     for (int e = threadIdx.x; e < D * dv; e += blockDim.x) S[e] = a.seg_S[so * D * dv + e];
     for (int e = threadIdx.x; e < D; e += blockDim.x) z[e] = a.seg_z[so * D + e];
-    for (int e = threadIdx.x; e < lay.nint * lay.L * 2; e += blockDim.x) shist[e] = 0.0f;
+    for (int e = threadIdx.x; e < lay.nint * lay.L * 2; e += blockDim.x) shist[e] = 0.0;
     GradAcc g = {};
     for (int t0 = r0; t0 < r1; t0 += kCs) {
         const int nr = min(kCs, r1 - t0);
@@ -243,20 +244,20 @@ __global__ void __launch_bounds__(kThreads) k_causal_dq(AttnArgs a) {
         __syncthreads();
         for (int e = threadIdx.x; e < nr * kCs; e += blockDim.x) {
             const int r = e / kCs, j = e - r * kCs;
-            float acc = 0.0f;
+            double acc = 0.0;
             if (j <= r && j < nr) {
-                for (int c = 0; c < dv; ++c) acc = fmaf(sdO[r * dv + c], sV[j * dv + c], acc);
-                acc += sdden[r];
+                for (int c = 0; c < dv; ++c) acc = fma((double)sdO[r * dv + c], (double)sV[j * dv + c], acc);
+                acc += (double)sdden[r];
             }
-            sP[e] = acc;
+            sP[e] = (float)acc;
         }
         __syncthreads();
         for (int e = threadIdx.x; e < nr * D; e += blockDim.x) {
             const int r = e / D, f = e - r * D;
-            float acc = z[f] * sdden[r];
-            for (int c = 0; c < dv; ++c) acc = fmaf(S[f * dv + c], sdO[r * dv + c], acc);
-            for (int j = 0; j <= r; ++j) acc = fmaf(sP[r * kCs + j], sPk[j * D + f], acc);
-            sdPq[e] = acc;
+            double acc = (double)z[f] * (double)sdden[r];
+            for (int c = 0; c < dv; ++c) acc = fma((double)S[f * dv + c], (double)sdO[r * dv + c], acc);
+            for (int j = 0; j <= r; ++j) acc = fma((double)sP[r * kCs + j], (double)sPk[j * D + f], acc);
+            sdPq[e] = (float)acc;
         }
         __syncthreads();
         advance_state(S, z, sPk, sV, nr, D, dv);
@@ -264,7 +265,7 @@ __global__ void __launch_bounds__(kThreads) k_causal_dq(AttnArgs a) {
         store_dx(lay, s, sdU, nr, dQ + (size_t)t0 * d);
     }
     __syncthreads();
-    store_grad_partial(lay, g, shist, a.gpart + ((size_t)bh * a.nseg + seg) * a.gsize);
+    store_grad_partial(lay, g, gp);
 }
 
 // dK, dV: reverse sweep with the suffix state G (after the current chunk).
@@ -285,8 +286,9 @@ __global__ void __launch_bounds__(kThreads) k_causal_dkv(AttnArgs a) {
     float *sU = cv.take(kCs * M);
     int *sJ = reinterpret_cast<int *>(cv.take(kCs * M));
     float *sdU = cv.take(kCs * M);
-    float *shist = cv.take(lay.nint * lay.L * 2);
     const int bh = blockIdx.y, seg = blockIdx.x;
+    double *gp = reinterpret_cast<double *>(a.gpart) + ((size_t)a.B * a.H * a.nseg + (size_t)bh * a.nseg + seg) * a.gsize;
+    double *shist = gp + M * d + M;  // the block's fp64 histogram, accumulated in place by L2 atomics
     const int len = head_length(a.lengths, bh / a.H, a.n);
     const int r0 = seg * a.seg_len, rend = min(a.n, r0 + a.seg_len), r1 = min(len, rend);
     IO *dK = static_cast<IO *>(a.dK) + (size_t)bh * a.n * d;
@@ -297,7 +299,7 @@ __global__ void __launch_bounds__(kThreads) k_causal_dkv(AttnArgs a) {
     const size_t so = (size_t)bh * a.nseg + seg;
     for (int e = threadIdx.x; e < D * dv; e += blockDim.x) G[e] = a.seg_dS[so * D * dv + e];
     for (int e = threadIdx.x; e < D; e += blockDim.x) gz[e] = a.seg_dz[so * D + e];
-    for (int e = threadIdx.x; e < lay.nint * lay.L * 2; e += blockDim.x) shist[e] = 0.0f;
+    for (int e = threadIdx.x; e < lay.nint * lay.L * 2; e += blockDim.x) shist[e] = 0.0;
     GradAcc g = {};
     if (r1 > r0) {
         for (int t0 = r0 + ((r1 - 1 - r0) / kCs) * kCs; t0 >= r0; t0 -= kCs) {
@@ -320,12 +322,12 @@ __global__ void __launch_bounds__(kThreads) k_causal_dkv(AttnArgs a) {
             masked_scores(sPq, sPk, nr, D, sA);
             for (int e = threadIdx.x; e < nr * kCs; e += blockDim.x) {
                 const int r = e / kCs, j = e - r * kCs;
-                float acc = 0.0f;
+                double acc = 0.0;
                 if (j <= r && j < nr) {
-                    for (int c = 0; c < dv; ++c) acc = fmaf(sdO[r * dv + c], sV[j * dv + c], acc);
-                    acc += sdden[r];
+                    for (int c = 0; c < dv; ++c) acc = fma((double)sdO[r * dv + c], (double)sV[j * dv + c], acc);
+                    acc += (double)sdden[r];
                 }
-                sP[e] = acc;
+                sP[e] = (float)acc;
             }
             __syncthreads();
             for (int e = threadIdx.x; e < nr * dv; e += blockDim.x) {
@@ -337,10 +339,10 @@ __global__ void __launch_bounds__(kThreads) k_causal_dkv(AttnArgs a) {
             }
             for (int e = threadIdx.x; e < nr * D; e += blockDim.x) {
                 const int j = e / D, f = e - j * D;
-                float acc = gz[f];
-                for (int c = 0; c < dv; ++c) acc = fmaf(G[f * dv + c], sV[j * dv + c], acc);
-                for (int r = j; r < nr; ++r) acc = fmaf(sP[r * kCs + j], sPq[r * D + f], acc);
-                sdPk[e] = acc;
+                double acc = gz[f];
+                for (int c = 0; c < dv; ++c) acc = fma((double)G[f * dv + c], (double)sV[j * dv + c], acc);
+                for (int r = j; r < nr; ++r) acc = fma((double)sP[r * kCs + j], (double)sPq[r * D + f], acc);
+                sdPk[e] = (float)acc;
             }
             __syncthreads();
             // G += phi(Q_chunk)^T dnum, g += phi(Q_chunk)^T dden
@@ -360,7 +362,7 @@ __global__ void __launch_bounds__(kThreads) k_causal_dkv(AttnArgs a) {
         }
     }
     __syncthreads();
-    store_grad_partial(lay, g, shist, a.gpart + ((size_t)a.B * a.H * a.nseg + (size_t)bh * a.nseg + seg) * a.gsize);
+    store_grad_partial(lay, g, gp);
 }
 
 // ---------------------------------------------------------------------------
@@ -379,7 +381,6 @@ size_t smem_dq(const AttnArgs &a) {
     cv.take(a.D * a.dv); cv.take(a.D); cv.take(kCs * a.d); cv.take(kCs * a.d); cv.take(kCs * a.dv);
     cv.take(kCs * a.dv); cv.take(kCs * a.D); cv.take(kCs * a.D); cv.take(kCs * a.D); cv.take(kCs * kCs);
     cv.take(kCs); cv.take(kCs); cv.take(kCs * a.M); cv.take(kCs * a.M); cv.take(kCs * a.M);
-    cv.take(a.lay.nint * a.lay.L * 2);
     return cv.bytes();
 }
 size_t smem_dkv(const AttnArgs &a) { return smem_dq(a) + 4 * (size_t)r4(kCs * kCs); }
@@ -403,7 +404,9 @@ cudaError_t causal_fwd_impl(const AttnArgs &a, cudaStream_t s) {
 }
 
 template <typename IO>
-cudaError_t causal_bwd_impl(const AttnArgs &a, bool have_state, cudaStream_t s) {
+cudaError_t causal_bwd_impl(const AttnArgs &a0, bool have_state, cudaStream_t s) {
+    AttnArgs a = a0;
+    a.gpart64 = 1;  // the generic kernels write fp64 parameter-gradient partials
     cudaError_t e;
     if (!have_state && (e = seg_stats<IO>(a, s)) != cudaSuccess) return e;
     const dim3 grid(a.nseg, a.B * a.H);

@@ -222,10 +222,11 @@ __global__ void __launch_bounds__(kRed) k_chrms_kappa(AttnArgs a, const double *
 // rows fall in distinct banks), computes every projection's u, interval, channels and dU, then, with
 // the lanes over input columns, adds dU W to the rows of dQ / dK and dU^T X, column sums of dU to the
 // block's dW, db.  One parameter-gradient partial per block at gpart[(side * gridDim.x + blockIdx.x) *
-// gsize]; its interval histogram is accumulated in place by fp32 reductions in L2 (atomic adds without
-// a return value), which do not serialise like fp32 atomics in shared memory.
-template <typename IO>
-__global__ void __launch_bounds__(kKWarps * 32) k_chrms_kterm(AttnArgs a, const float *kappa, float *gpart) {
+// gsize], of the partials' type P (fp32 beside the tensor-core kernels' partials, fp64 beside the
+// generic kernels'); its interval histogram is accumulated in place by reductions in L2 (atomic adds
+// without a return value), which do not serialise like fp32 atomics in shared memory.
+template <typename IO, typename GP>
+__global__ void __launch_bounds__(kKWarps * 32) k_chrms_kterm(AttnArgs a, const float *kappa, GP *gpart) {
     extern __shared__ __align__(16) float smem[];
     const TableLayout &lay = a.lay;
     const int d = a.d, M = a.M, L = a.L, P = lay.Ppad, NH = lay.nint * L * 2;
@@ -236,23 +237,23 @@ __global__ void __launch_bounds__(kKWarps * 32) k_chrms_kterm(AttnArgs a, const 
     float *sAB = sT + r4(P);
     float *sW = sAB + r4(NH);
     float *sb = sW + r4(M * d);
-    float *sdW = sb + r4(M);
-    float *sdb = sdW + r4(M * d);
-    float *sk = sdb + r4(M);
+    double *sdW = reinterpret_cast<double *>(sb + r4(M));       // fp64 block sums of dW, db
+    double *sdb = sdW + r4(M * d);
+    float *sk = reinterpret_cast<float *>(sdb + r4(M));
     float *sx = sk + r4(kMaxL) + warp * (r4(32 * dp) + r4(32 * mp));
     float *sdu = sx + r4(32 * dp);
     const int Md = M * d;
-    float *gp = gpart + ((size_t)side * gridDim.x + blockIdx.x) * a.gsize;
-    float *ghist = gp + Md + M;
+    GP *gp = gpart + ((size_t)side * gridDim.x + blockIdx.x) * a.gsize;
+    GP *ghist = gp + Md + M;
     {
         const float *T = reinterpret_cast<const float *>(a.table + lay.off_T);
         const float *AB = reinterpret_cast<const float *>(a.table + lay.off_AB);
         const float *W = reinterpret_cast<const float *>(a.table + lay.off_W);
         const float *b = reinterpret_cast<const float *>(a.table + lay.off_b);
         for (int e = threadIdx.x; e < P; e += blockDim.x) sT[e] = T[e];
-        for (int e = threadIdx.x; e < NH; e += blockDim.x) { sAB[e] = AB[e]; ghist[e] = 0.0f; }
-        for (int e = threadIdx.x; e < M * d; e += blockDim.x) { sW[e] = W[e]; sdW[e] = 0.0f; }
-        for (int e = threadIdx.x; e < M; e += blockDim.x) { sb[e] = b[e]; sdb[e] = 0.0f; }
+        for (int e = threadIdx.x; e < NH; e += blockDim.x) { sAB[e] = AB[e]; ghist[e] = (GP)0; }
+        for (int e = threadIdx.x; e < M * d; e += blockDim.x) { sW[e] = W[e]; sdW[e] = 0.0; }
+        for (int e = threadIdx.x; e < M; e += blockDim.x) { sb[e] = b[e]; sdb[e] = 0.0; }
         if ((int)threadIdx.x < L) sk[threadIdx.x] = kappa[side * kMaxL + threadIdx.x] * (float)M;
     }
     __syncthreads();
@@ -282,15 +283,15 @@ __global__ void __launch_bounds__(kKWarps * 32) k_chrms_kterm(AttnArgs a, const 
                 for (int c = 0; c < d; ++c) u = fmaf(w[c], x[c], u);
                 const int j = interval_of(sT, P, u);
                 const float *ab = sAB + j * L * 2;
-                float *h = ghist + j * L * 2;
+                GP *h = ghist + j * L * 2;
                 for (int l = 0; l < L; ++l) {
                     const float ph = fmaxf(fmaf(ab[2 * l], u, ab[2 * l + 1]), 0.0f);
                     if (ph > 0.0f) {  // outer ReLU on
                         const float g = sk[l] * ph;
                         du = fmaf(g, ab[2 * l], du);
                         if (g != 0.0f) {
-                            atomicAdd(h + 2 * l, g);
-                            atomicAdd(h + 2 * l + 1, g * u);
+                            atomicAdd(h + 2 * l, (GP)g);
+                            atomicAdd(h + 2 * l + 1, (GP)g * (GP)u);
                         }
                     }
                 }
@@ -310,21 +311,21 @@ __global__ void __launch_bounds__(kKWarps * 32) k_chrms_kterm(AttnArgs a, const 
                 io_store(dX + (row0 + r) * d + c, cur[r] + acc);
             }
             for (int i = 0; i < M; ++i) {
-                float acc = 0.0f;
-                for (int r = 0; r < 32; ++r) acc = fmaf(sdu[r * mp + i], sx[r * dp + c], acc);
+                double acc = 0.0;
+                for (int r = 0; r < 32; ++r) acc = fma((double)sdu[r * mp + i], (double)sx[r * dp + c], acc);
                 atomicAdd(sdW + i * d + c, acc);
             }
         }
         if (lane < M) {
-            float acc = 0.0f;
-            for (int r = 0; r < 32; ++r) acc += sdu[r * mp + lane];
+            double acc = 0.0;
+            for (int r = 0; r < 32; ++r) acc += (double)sdu[r * mp + lane];
             atomicAdd(sdb + lane, acc);
         }
         __syncwarp();
     }
     __syncthreads();
-    for (int e = threadIdx.x; e < Md; e += blockDim.x) gp[e] = sdW[e];
-    for (int e = threadIdx.x; e < M; e += blockDim.x) gp[Md + e] = sdb[e];
+    for (int e = threadIdx.x; e < Md; e += blockDim.x) gp[e] = (GP)sdW[e];
+    for (int e = threadIdx.x; e < M; e += blockDim.x) gp[Md + e] = (GP)sdb[e];
 }
 
 size_t smem_stats(const AttnArgs &a) {
@@ -332,7 +333,7 @@ size_t smem_stats(const AttnArgs &a) {
 }
 size_t smem_kterm(const AttnArgs &a) {
     const int NH = a.lay.nint * a.L * 2;
-    return (size_t)(r4(a.lay.Ppad) + r4(NH) + 2 * r4(a.M * a.d) + 2 * r4(a.M) + r4(kMaxL) +
+    return (size_t)(r4(a.lay.Ppad) + r4(NH) + 3 * r4(a.M * a.d) + 3 * r4(a.M) + r4(kMaxL) +
                     kKWarps * (r4(32 * (a.d + 1)) + r4(32 * (a.M + 1)))) * 4;
 }
 
@@ -348,12 +349,13 @@ cudaError_t stats_impl(const AttnArgs &a, cudaStream_t s) {
     return cudaGetLastError();
 }
 
-template <typename IO>
-cudaError_t kterm_impl(const AttnArgs &a, float *gpart, cudaStream_t s) {
+template <typename IO, typename GP>
+cudaError_t kterm_impl(const AttnArgs &a, GP *gpart, cudaStream_t s) {
     const size_t sm = smem_kterm(a);
-    cudaError_t e = set_smem(k_chrms_kterm<IO>, sm);
+    cudaError_t e = set_smem(k_chrms_kterm<IO, GP>, sm);
     if (e != cudaSuccess) return e;
-    LUNA_LAUNCH("chrms_kterm", k_chrms_kterm<IO>, dim3(kChKBlocks, 2), kKWarps * 32, sm, s, a, a.ch_kappa, gpart);
+    LUNA_LAUNCH("chrms_kterm", (k_chrms_kterm<IO, GP>), dim3(kChKBlocks, 2), kKWarps * 32, sm, s, a, a.ch_kappa,
+                gpart);
     return cudaGetLastError();
 }
 
@@ -398,8 +400,13 @@ cudaError_t launch_chrms_backward(const AttnArgs &a, int main_parts, int *nparts
     LUNA_LAUNCH("chrms_kappa", k_chrms_kappa, 1, kRed, 0, s, a, a.ch_T, a.ch_target, a.ch_stat, a.ch_kappa);
     cudaError_t e = cudaGetLastError();
     if (e != cudaSuccess) return e;
-    float *gpart = a.gpart + (size_t)main_parts * a.gsize;
-    e = a.ch_io == LUNA_F32 ? kterm_impl<float>(a, gpart, s) : kterm_impl<__nv_bfloat16>(a, gpart, s);
+    if (a.gpart64) {
+        double *gpart = reinterpret_cast<double *>(a.gpart) + (size_t)main_parts * a.gsize;
+        e = a.ch_io == LUNA_F32 ? kterm_impl<float>(a, gpart, s) : kterm_impl<__nv_bfloat16>(a, gpart, s);
+    } else {
+        float *gpart = a.gpart + (size_t)main_parts * a.gsize;
+        e = a.ch_io == LUNA_F32 ? kterm_impl<float>(a, gpart, s) : kterm_impl<__nv_bfloat16>(a, gpart, s);
+    }
     if (e != cudaSuccess) return e;
     *nparts = main_parts + 2 * kChKBlocks;
     return cudaSuccess;

@@ -166,12 +166,14 @@ __global__ void __launch_bounds__(kThreads) k_bwd_query(AttnArgs a) {
     float *sU = cv.take(kTileB * M);
     int *sJ = reinterpret_cast<int *>(cv.take(kTileB * M));
     float *sdU = cv.take(kTileB * M);
-    float *shist = cv.take(lay.nint * lay.L * 2);
     load_phi(s, lay, a.table);
     const int bh = blockIdx.y, split = blockIdx.x;
+    const size_t slot = (size_t)bh * a.nsplit_b + split;
+    double *gp = reinterpret_cast<double *>(a.gpart) + slot * a.gsize;
+    double *shist = gp + M * d + M;  // the block's fp64 histogram, accumulated in place by L2 atomics
     for (int e = threadIdx.x; e < D * dv; e += blockDim.x) sS[e] = a.S_fin[(size_t)bh * D * dv + e];
     for (int e = threadIdx.x; e < D; e += blockDim.x) sz[e] = a.z_fin[(size_t)bh * D + e];
-    for (int e = threadIdx.x; e < lay.nint * lay.L * 2; e += blockDim.x) shist[e] = 0.0f;
+    for (int e = threadIdx.x; e < lay.nint * lay.L * 2; e += blockDim.x) shist[e] = 0.0;
 
     const int len = head_length(a.lengths, bh / a.H, a.n);
     const int r0 = split * a.rows_per_split_b;
@@ -215,9 +217,9 @@ __global__ void __launch_bounds__(kThreads) k_bwd_query(AttnArgs a) {
         }
         __syncthreads();
         for (int r = threadIdx.x; r < nr; r += blockDim.x) {
-            float dot = 0.0f;
-            for (int c = 0; c < dv; ++c) dot = fmaf(sdO[r * dv + c], sdnum[r * dv + c], dot);
-            sdden[r] = (sden[r] != 0.0f) ? -dot / sden[r] : 0.0f;
+            double dot = 0.0;  // dden and dphi are formed in fp64 and rounded once: they cancel
+            for (int c = 0; c < dv; ++c) dot = fma((double)sdO[r * dv + c], (double)sdnum[r * dv + c], dot);
+            sdden[r] = (sden[r] != 0.0f) ? (float)(-dot / (double)sden[r]) : 0.0f;
         }
         __syncthreads();
         for (int e = threadIdx.x; e < nr * dv; e += blockDim.x) {
@@ -227,9 +229,9 @@ __global__ void __launch_bounds__(kThreads) k_bwd_query(AttnArgs a) {
         __syncthreads();
         for (int e = threadIdx.x; e < nr * D; e += blockDim.x) {
             const int r = e / D, f = e - r * D;
-            float acc2 = sz[f] * sdden[r];
-            for (int c = 0; c < dv; ++c) acc2 = fmaf(sS[f * dv + c], sdnum[r * dv + c], acc2);
-            sdPhi[e] = acc2;
+            double acc2 = (double)sz[f] * (double)sdden[r];
+            for (int c = 0; c < dv; ++c) acc2 = fma((double)sS[f * dv + c], (double)sdnum[r * dv + c], acc2);
+            sdPhi[e] = (float)acc2;
         }
         __syncthreads();
         if (active) outer_accumulate(acc, zacc, true, sPhi, D, sdnum, dv, sdden, nr, f0, c0);
@@ -237,9 +239,8 @@ __global__ void __launch_bounds__(kThreads) k_bwd_query(AttnArgs a) {
         store_dx(lay, s, sdU, nr, dQ + (size_t)t0 * d);
     }
     __syncthreads();
-    const size_t slot = (size_t)bh * a.nsplit_b + split;
     store_tile(acc, zacc, active, tc, f0, c0, D, dv, a.dS_part + slot * D * dv, a.dz_part + slot * D);
-    store_grad_partial(lay, g, shist, a.gpart + slot * a.gsize);
+    store_grad_partial(lay, g, gp);
     if (last_arrival(a.counters + a.B * a.H + bh, a.nsplit_b)) {
         ordered_sum(a.dS_part + (size_t)bh * a.nsplit_b * D * dv, a.nsplit_b, D * dv, a.dS_fin + (size_t)bh * D * dv);
         ordered_sum(a.dz_part + (size_t)bh * a.nsplit_b * D, a.nsplit_b, D, a.dz_fin + (size_t)bh * D);
@@ -265,12 +266,14 @@ __global__ void __launch_bounds__(kThreads) k_bwd_key(AttnArgs a) {
     float *sU = cv.take(kTileB * M);
     int *sJ = reinterpret_cast<int *>(cv.take(kTileB * M));
     float *sdU = cv.take(kTileB * M);
-    float *shist = cv.take(lay.nint * lay.L * 2);
     load_phi(s, lay, a.table);
     const int bh = blockIdx.y, split = blockIdx.x;
+    const size_t slot = (size_t)a.B * a.H * a.nsplit_b + (size_t)bh * a.nsplit_b + split;
+    double *gp = reinterpret_cast<double *>(a.gpart) + slot * a.gsize;
+    double *shist = gp + M * d + M;  // the block's fp64 histogram, accumulated in place by L2 atomics
     for (int e = threadIdx.x; e < D * dv; e += blockDim.x) sdS[e] = a.dS_fin[(size_t)bh * D * dv + e];
     for (int e = threadIdx.x; e < D; e += blockDim.x) sdz[e] = a.dz_fin[(size_t)bh * D + e];
-    for (int e = threadIdx.x; e < lay.nint * lay.L * 2; e += blockDim.x) shist[e] = 0.0f;
+    for (int e = threadIdx.x; e < lay.nint * lay.L * 2; e += blockDim.x) shist[e] = 0.0;
 
     const int len = head_length(a.lengths, bh / a.H, a.n);
     const int r0 = split * a.rows_per_split_b;
@@ -300,17 +303,16 @@ __global__ void __launch_bounds__(kThreads) k_bwd_key(AttnArgs a) {
         }
         for (int e = threadIdx.x; e < nr * D; e += blockDim.x) {
             const int r = e / D, f = e - r * D;
-            float acc2 = sdz[f];
-            for (int c = 0; c < dv; ++c) acc2 = fmaf(sdS[f * dv + c], sV[r * dv + c], acc2);
-            sdPhi[e] = acc2;
+            double acc2 = sdz[f];
+            for (int c = 0; c < dv; ++c) acc2 = fma((double)sdS[f * dv + c], (double)sV[r * dv + c], acc2);
+            sdPhi[e] = (float)acc2;
         }
         __syncthreads();
         phi_backward_tile(lay, s, sK, nr, sPhi, sdPhi, sU, sJ, sdU, shist, g);
         store_dx(lay, s, sdU, nr, dK + (size_t)t0 * d);
     }
     __syncthreads();
-    const size_t slot = (size_t)a.B * a.H * a.nsplit_b + (size_t)bh * a.nsplit_b + split;
-    store_grad_partial(lay, g, shist, a.gpart + slot * a.gsize);
+    store_grad_partial(lay, g, gp);
 }
 
 // ---------------------------------------------------------------------------
@@ -335,41 +337,58 @@ struct CompSum {
 
 // Sum of the per-block parameter-gradient partials, in the fixed order p = 0..nparts-1
 // per element: 64 elements per block, each summed by 8 threads over consecutive
-// eighths of the partials (8 loads in flight, compensated fp32), then the eight parts
-// combined in order in fp64.
+// eighths of the partials (8 loads in flight; fp32 partials in compensated fp32,
+// fp64 partials in fp64), then the eight parts combined in order in fp64.
 constexpr int kSumElems = 64, kSumSplit = 8;
-__global__ void __launch_bounds__(kSumElems * kSumSplit) k_grad_sum(const float *gpart, int nparts, int gsize,
-                                                                    float *out) {
+template <typename P>
+__global__ void __launch_bounds__(kSumElems * kSumSplit) k_grad_sum(const P *gpart, int nparts, int gsize,
+                                                                    double *out) {
     __shared__ double part[kSumSplit][kSumElems];
     const int el = threadIdx.x % kSumElems, q = threadIdx.x / kSumElems;
     const int e = blockIdx.x * kSumElems + el;
     const int p0 = (int)((long long)q * nparts / kSumSplit), p1 = (int)((long long)(q + 1) * nparts / kSumSplit);
-    CompSum cs;
-    if (e < gsize) {
-        int p = p0;
-        for (; p + 8 <= p1; p += 8) {
-            float v[8];
+    if constexpr (sizeof(P) == 4) {
+        CompSum cs;
+        if (e < gsize) {
+            int p = p0;
+            for (; p + 8 <= p1; p += 8) {
+                float v[8];
 #pragma unroll
-            for (int k = 0; k < 8; ++k) v[k] = __ldcg(gpart + (size_t)(p + k) * gsize + e);
+                for (int k = 0; k < 8; ++k) v[k] = __ldcg(gpart + (size_t)(p + k) * gsize + e);
 #pragma unroll
-            for (int k = 0; k < 8; ++k) cs.add(v[k]);
+                for (int k = 0; k < 8; ++k) cs.add(v[k]);
+            }
+            for (; p < p1; ++p) cs.add(__ldcg(gpart + (size_t)p * gsize + e));
         }
-        for (; p < p1; ++p) cs.add(__ldcg(gpart + (size_t)p * gsize + e));
+        part[q][el] = (double)cs.s + (double)cs.c;
+    } else {
+        double t = 0.0;
+        if (e < gsize) {
+            int p = p0;
+            for (; p + 8 <= p1; p += 8) {
+                double v[8];
+#pragma unroll
+                for (int k = 0; k < 8; ++k) v[k] = __ldcg(gpart + (size_t)(p + k) * gsize + e);
+#pragma unroll
+                for (int k = 0; k < 8; ++k) t += v[k];
+            }
+            for (; p < p1; ++p) t += __ldcg(gpart + (size_t)p * gsize + e);
+        }
+        part[q][el] = t;
     }
-    part[q][el] = (double)cs.s + (double)cs.c;
     __syncthreads();
     if (q == 0 && e < gsize) {
         double t = part[0][el];
 #pragma unroll
         for (int k = 1; k < kSumSplit; ++k) t += part[k][el];
-        out[e] = (float)t;
+        out[e] = t;
     }
 }
 
 // Inclusive scan of x[0..n) into y (forward: prefix sums; backward: suffix sums), accumulated in fp64,
 // by one warp, in a fixed order: lane c sums a contiguous chunk, the chunk totals
 // are scanned across lanes, then every lane writes its chunk.
-__device__ void warp_scan(const float *x, double *y, int n, bool backward) {
+__device__ void warp_scan(const double *x, double *y, int n, bool backward) {
     const int lane = threadIdx.x & 31;
     const int chunk = (n + 31) / 32;
     const int b = lane * chunk, e = min(n, b + chunk);
@@ -393,19 +412,19 @@ __device__ void warp_scan(const float *x, double *y, int n, bool backward) {
 // channel's interval histogram.  Block L: dW and db.  With the shared-channel
 // MLP every channel reads every hidden unit: block l writes its channel's fc1
 // contributions to fc1_part ([dw1 | db1][l][k], fp64), summed by k_mlp_fc1_sum.
-__global__ void __launch_bounds__(128) k_mlp_grads(TableLayout lay, const char *table, const float *gsum,
+__global__ void __launch_bounds__(128) k_mlp_grads(TableLayout lay, const char *table, const double *gsum,
                                                    luna_phi_grads grads, double *fc1_part) {
-    __shared__ float h[2][kMaxUnits + 1];
+    __shared__ double h[2][kMaxUnits + 1];
     __shared__ double pre[2][kMaxUnits + 1], suf[2][kMaxUnits + 1];  // fp64: dw2 = w1 G1 + b1 G0 cancels
     const int Md = lay.M * lay.d, L = lay.L, hid = lay.hid, nint = lay.nint;
     const float scale = 1.0f / sqrtf((float)lay.M);
     if ((int)blockIdx.x == L) {
-        for (int e = threadIdx.x; e < Md; e += blockDim.x) grads.dW[e] = gsum[e];
-        for (int e = threadIdx.x; e < lay.M; e += blockDim.x) grads.db[e] = gsum[Md + e];
+        for (int e = threadIdx.x; e < Md; e += blockDim.x) grads.dW[e] = (float)gsum[e];
+        for (int e = threadIdx.x; e < lay.M; e += blockDim.x) grads.db[e] = (float)gsum[Md + e];
         return;
     }
     const int l = blockIdx.x;
-    const float *hist = gsum + Md + lay.M;
+    const double *hist = gsum + Md + lay.M;
     for (int j = threadIdx.x; j < nint; j += blockDim.x) {
         h[0][j] = hist[(j * L + l) * 2];
         h[1][j] = hist[(j * L + l) * 2 + 1];
@@ -475,14 +494,13 @@ size_t smem_bwd_query(const AttnArgs &a) {
     HostCarve cv; carve_phi_host(cv, a.lay);
     cv.take(a.D * a.dv); cv.take(a.D); cv.take(kTileB * a.d); cv.take(kTileB * a.dv); cv.take(kTileB * a.D);
     cv.take(kTileB * a.D); cv.take(kTileB * a.dv); cv.take(kTileB); cv.take(kTileB); cv.take(kTileB * a.M);
-    cv.take(kTileB * a.M); cv.take(kTileB * a.M); cv.take(a.lay.nint * a.lay.L * 2);
+    cv.take(kTileB * a.M);
     return cv.bytes();
 }
 size_t smem_bwd_key(const AttnArgs &a) {
     HostCarve cv; carve_phi_host(cv, a.lay);
     cv.take(a.D * a.dv); cv.take(a.D); cv.take(kTileB * a.d); cv.take(kTileB * a.dv); cv.take(kTileB * a.D);
     cv.take(kTileB * a.D); cv.take(kTileB * a.M); cv.take(kTileB * a.M); cv.take(kTileB * a.M);
-    cv.take(a.lay.nint * a.lay.L * 2);
     return cv.bytes();
 }
 
@@ -507,7 +525,9 @@ cudaError_t fwd_impl(const AttnArgs &a, cudaStream_t s) {
 }
 
 template <typename IO>
-cudaError_t bwd_impl(const AttnArgs &a, bool have_stats, cudaStream_t s) {
+cudaError_t bwd_impl(const AttnArgs &a0, bool have_stats, cudaStream_t s) {
+    AttnArgs a = a0;
+    a.gpart64 = 1;  // the generic kernels write fp64 parameter-gradient partials
     cudaError_t e;
     if (!have_stats && (e = stats_impl<IO>(a, s)) != cudaSuccess) return e;
     size_t sm = smem_bwd_query(a);
@@ -535,8 +555,12 @@ size_t simt_max_smem(const AttnArgs &a) {
 }
 
 cudaError_t launch_grad_reduce(const AttnArgs &a, int nparts, cudaStream_t s) {
-    LUNA_LAUNCH("grad_sum", k_grad_sum, (a.gsize + kSumElems - 1) / kSumElems, kSumElems * kSumSplit, 0, s, a.gpart,
-                nparts, a.gsize, a.hist);
+    const int nb = (a.gsize + kSumElems - 1) / kSumElems;
+    if (a.gpart64)
+        LUNA_LAUNCH("grad_sum", k_grad_sum<double>, nb, kSumElems * kSumSplit, 0, s,
+                    reinterpret_cast<const double *>(a.gpart), nparts, a.gsize, a.hist);
+    else
+        LUNA_LAUNCH("grad_sum", k_grad_sum<float>, nb, kSumElems * kSumSplit, 0, s, a.gpart, nparts, a.gsize, a.hist);
     cudaError_t e = cudaGetLastError();
     if (e != cudaSuccess) return e;
     // the partials have been summed: their buffer holds the shared MLP's per-channel fc1 terms

@@ -21,9 +21,11 @@ struct AttnArgs {
     // backward
     int nsplit_b, rows_per_split_b;
     float *dS_part, *dz_part, *dS_fin, *dz_fin;
-    float *gpart;                      // [2 * BH * nsplit_b][gsize] parameter-gradient partials
+    float *gpart;                      // [2 * BH * nsplit_b][gsize] parameter-gradient partials (fp32, or
+                                       // fp64 when gpart64: the generic kernels)
+    int gpart64;                       // 1: the partials are doubles
     int gsize;                         // M*d + M + nint*L*2
-    float *hist;                       // [nint][L][2] reduced histogram
+    double *hist;                      // [gsize] the partials' sum: dW, db, then the histogram [nint][L][2]
     luna_phi_grads grads;
     // causal
     int chunk, seg_len, nseg;          // state segments of seg_len rows (multiple of chunk)
@@ -78,6 +80,10 @@ cudaError_t launch_grad_reduce(const AttnArgs &a, int nparts, cudaStream_t s);
 cudaError_t launch_causal_fwd(const AttnArgs &a, luna_dtype io, bool write_state, cudaStream_t s);
 cudaError_t launch_causal_bwd(const AttnArgs &a, luna_dtype io, bool have_state, cudaStream_t s);
 size_t simt_max_smem(const AttnArgs &a);
+// attention weights of query rows [row0, row0 + rows) of every head (conversion, stage 1): A (BH, rows, n)
+cudaError_t launch_weights(const AttnArgs &a, luna_dtype io, int causal, int row0, int rows, int teacher, float *A,
+                           cudaStream_t s);
+size_t weights_max_smem(const AttnArgs &a);
 // channel RMS normalisation: statistics and scales of both sides; S, z rows times sigma (after any key
 // statistics); dS, dz rows times sigma and the per-head sums T (between the query- and key-side backward
 // kernels); the scale term of the backward (before the parameter-gradient reduction: its partials follow

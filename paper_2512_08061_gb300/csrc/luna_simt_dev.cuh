@@ -168,45 +168,48 @@ __device__ void store_tile(const float (&acc)[8][8], const float (&zacc)[8], boo
 // backward through phi for a tile: dU = sum_l dPhi * dphi/du, histogram of
 // the channel-MLP gradient statistics, then dX = dU W and dW += dU^T X.
 
+// The parameter gradients are sums over every row, projection and channel whose terms cancel (the
+// loss is nearly invariant to a common scale of the features), so the generic kernels accumulate them,
+// and the histogram, in fp64; the per-sample terms stay fp32.
 struct GradAcc {
-    float dW[16];  // entries threadIdx.x + k * blockDim.x of the M*d matrix
-    float db;      // entry threadIdx.x of b (if < M)
+    double dW[16];  // entries threadIdx.x + k * blockDim.x of the M*d matrix
+    double db;      // entry threadIdx.x of b (if < M)
 };
 
 __device__ void phi_backward_tile(const TableLayout &lay, const SmemPhi &s, const float *sX, int nr,
                                   const float *sPhi, const float *sdPhi, const float *sU, const int *sJ, float *sdU,
-                                  float *shist, GradAcc &g) {
+                                  double *shist, GradAcc &g) {
     const int M = lay.M, L = lay.L, d = lay.d, D = lay.D;
     for (int e = threadIdx.x; e < nr * M; e += blockDim.x) {
         const int r = e / M, i = e - r * M;
         const float u = sU[e];
         const int j = sJ[e];
         const float *ab = s.AB + j * L * 2;
-        float du = 0.0f;
+        double du = 0.0;
         for (int l = 0; l < L; ++l) {
             const int f = r * D + i * L + l;
             if (sPhi[f] > 0.0f) {  // outer ReLU on
-                const float gl = sdPhi[f];
-                du = fmaf(gl, ab[2 * l], du);
-                if (gl != 0.0f) {
+                const double gl = sdPhi[f];
+                du = fma(gl, (double)ab[2 * l], du);
+                if (gl != 0.0) {
                     atomicAdd(shist + (j * L + l) * 2, gl);
-                    atomicAdd(shist + (j * L + l) * 2 + 1, gl * u);
+                    atomicAdd(shist + (j * L + l) * 2 + 1, gl * (double)u);  // exact product
                 }
             }
         }
-        sdU[e] = du;
+        sdU[e] = (float)du;
     }
     __syncthreads();
     for (int k = 0; k < 16; ++k) {
         const int e = threadIdx.x + k * blockDim.x;
         if (e >= M * d) break;
         const int i = e / d, c = e - i * d;
-        float acc = g.dW[k];
-        for (int r = 0; r < nr; ++r) acc = fmaf(sdU[r * M + i], sX[r * d + c], acc);
+        double acc = g.dW[k];
+        for (int r = 0; r < nr; ++r) acc = fma((double)sdU[r * M + i], (double)sX[r * d + c], acc);
         g.dW[k] = acc;
     }
     if (threadIdx.x < M)
-        for (int r = 0; r < nr; ++r) g.db += sdU[r * M + threadIdx.x];
+        for (int r = 0; r < nr; ++r) g.db += (double)sdU[r * M + threadIdx.x];
 }
 
 template <typename IO>
@@ -220,7 +223,9 @@ __device__ void store_dx(const TableLayout &lay, const SmemPhi &s, const float *
     }
 }
 
-__device__ void store_grad_partial(const TableLayout &lay, const GradAcc &g, const float *shist, float *gp) {
+// Writes dW and db into the block's fp64 partial gp = [dW | db | histogram]; the histogram was
+// accumulated in place.
+__device__ void store_grad_partial(const TableLayout &lay, const GradAcc &g, double *gp) {
     const int Md = lay.M * lay.d;
     for (int k = 0; k < 16; ++k) {
         const int e = threadIdx.x + k * blockDim.x;
@@ -228,7 +233,6 @@ __device__ void store_grad_partial(const TableLayout &lay, const GradAcc &g, con
         gp[e] = g.dW[k];
     }
     if (threadIdx.x < lay.M) gp[Md + threadIdx.x] = g.db;
-    for (int e = threadIdx.x; e < lay.nint * lay.L * 2; e += blockDim.x) gp[Md + lay.M + e] = shist[e];
 }
 
 template <typename K>

@@ -81,6 +81,7 @@ def _load():
         "luna_attn_decode": ([ad, pd, P, P, P, P, P, P, I64, P, I64, P], I),
         "luna_selftest_wait": ([P, I64, P], I),
         "luna_noalloc_scratch": ([ctypes.POINTER(P), ctypes.POINTER(S)], I),
+        "luna_attn_weights": ([ad, pd, P, P, P, P, I, I, I, P, P], I),
     }
     for name, (args, res) in sig.items():
         fn = getattr(lib, name)
@@ -93,7 +94,8 @@ _lib = _load()
 EXPORTED = ("luna_status_string", "luna_version", "luna_phi_table_size", "luna_phi_prepare", "luna_featmap",
             "luna_workspace_size", "luna_state_size", "luna_attn_fwd", "luna_attn_bwd", "luna_device_status",
             "luna_profile_start", "luna_profile_stop", "luna_launch_count", "luna_attn_fwd_noalloc",
-            "luna_state_final", "luna_attn_decode", "luna_selftest_wait", "luna_noalloc_scratch")
+            "luna_state_final", "luna_attn_decode", "luna_selftest_wait", "luna_noalloc_scratch",
+            "luna_attn_weights")
 
 
 def _ptr(t):
@@ -189,6 +191,13 @@ def luna_attn_fwd_noalloc(ad, pd, table, Q, K, V, lengths, O, stream=None) -> No
 
 
 NOALLOC_SCRATCH_BYTES = 16 << 20
+
+
+def luna_attn_weights(ad, pd, table, Q, K, lengths, row0: int, rows: int, teacher: bool, A: torch.Tensor,
+                      stream=None) -> None:
+    _check(_lib.luna_attn_weights(ctypes.byref(ad), ctypes.byref(pd), _ptr(table), _ptr(Q), _ptr(K), _ptr(lengths),
+                                  int(row0), int(rows), int(bool(teacher)), _ptr(A), _stream(stream)),
+           "luna_attn_weights")
 
 
 def luna_state_final(ad, pd, state) -> tuple[int, int, int, int]:

@@ -41,24 +41,6 @@ def relerr_rows(got, ref) -> float:
     return float(max(np.max(np.where(zero, 0.0, err / np.where(zero, 1.0, floor))), np.max(np.where(zero, err, 0.0))))
 
 
-SUM_ULPS = 8  # fp32 parameter gradients: rounding allowance in ulps of sum |terms|
-
-
-def sum_err(got, ref, abs_terms, tol) -> float:
-    """max_i |g_i - r_i| / (tol * max(|r_i|, rms(r)) + SUM_ULPS * 2^-24 * A_i), A the sum
-    of the absolute per-sample contributions of each element: passes at <= 1.
-    A feature-map parameter gradient is a sum over every row, projection and
-    channel whose terms cancel, and an fp32 evaluation of it carries an error of
-    the order of 2^-24 * A in any order of summation."""
-    g = np.asarray(got, dtype=np.float64)
-    r = np.asarray(ref, dtype=np.float64)
-    A = np.asarray(abs_terms, dtype=np.float64)
-    rms = float(np.sqrt(np.mean(r * r))) if r.size else 0.0
-    bound = tol * np.maximum(np.abs(r), rms) + SUM_ULPS * 2.0 ** -24 * A
-    err = np.abs(g - r)
-    return float(np.max(np.where(bound > 0, err / np.where(bound > 0, bound, 1.0), np.where(err > 0, np.inf, 0.0))))
-
-
 # ---------------------------------------------------------------------------
 # guard bands (the sanitizer's out-of-bounds checks are not available): every
 # buffer the library writes in the parity tests sits between two bands of a
@@ -187,11 +169,6 @@ class Case:
         i = self.inp
         return oracle.attn_bwd(self.phi, i["Q"].value, i["K"].value, i["V"].value, i["dO"].value, self.lengths,
                                self.causal, self.eps)
-
-    def oracle_bwd_abs_terms(self):
-        i = self.inp
-        return oracle.attn_bwd_abs_terms(self.phi, i["Q"].value, i["K"].value, i["V"].value, i["dO"].value,
-                                         self.lengths, self.causal, self.eps)
 
     def smooth_rows(self, which: str) -> np.ndarray:
         """Rows whose feature map has no ReLU argument within rounding distance of

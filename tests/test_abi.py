@@ -169,3 +169,23 @@ def test_channel_rms_descriptor(L):
     dec = L.attn_desc(2, 4, 1, 32, 32, True)
     assert lib.luna_attn_decode(ctypes.byref(dec), ctypes.byref(pd1), None, None, None, None, None, None, 0, None, 0,
                                 None) == 2
+
+
+def test_attention_weights_arguments(L):
+    """luna_attn_weights checks its row window, flags and descriptors before any launch; an
+    empty window is a no-op."""
+    lib = L._lib
+    P = ctypes.c_void_p
+    pd = L.phi_desc(8, 8, 64)
+    ad = L.attn_desc(2, 2, 100, 32, 32)
+    args = (P(256), P(256), P(256), None)
+    assert lib.luna_attn_weights(ctypes.byref(ad), ctypes.byref(pd), *args, 90, 11, 0, P(256), None) == 1
+    assert lib.luna_attn_weights(ctypes.byref(ad), ctypes.byref(pd), *args, -1, 5, 0, P(256), None) == 1
+    assert lib.luna_attn_weights(ctypes.byref(ad), ctypes.byref(pd), *args, 0, 5, 2, P(256), None) == 1
+    assert lib.luna_attn_weights(ctypes.byref(ad), ctypes.byref(pd), *args, 0, 5, 0, None, None) == 1
+    assert lib.luna_attn_weights(ctypes.byref(ad), ctypes.byref(pd), None, P(256), P(256), None, 0, 5, 0, P(256),
+                                 None) == 1  # the LUNA weights need the table
+    rms = L.phi_desc(8, 8, 64, ch_rms_target=0.1)
+    assert lib.luna_attn_weights(ctypes.byref(ad), ctypes.byref(rms), *args, 0, 5, 0, P(256), None) == 2
+    assert lib.luna_attn_weights(ctypes.byref(ad), ctypes.byref(pd), None, None, None, None, 100, 0, 0, None,
+                                 None) == 0

@@ -12,7 +12,7 @@ import pytest
 
 import oracle
 import synth
-from cases import TOL, Case, relerr, relerr_rows, run_in_child, sum_err, to_device, to_host
+from cases import TOL, Case, relerr, relerr_rows, run_in_child, to_device, to_host
 
 pytestmark = pytest.mark.gpu
 
@@ -170,17 +170,29 @@ def test_backward(c):
     assert relerr(g["dV"], ref["dV"]) < tol
     for k in ("dQ", "dK", "dV"):
         assert np.all(np.isfinite(g[k]))
-    if c["io"] == "f32":  # fp32 sums over every sample: rounding bound in ulps of sum |terms|
-        A = case.oracle_bwd_abs_terms()
-        for k in ("dW", "db", "dw1", "db1", "dw2", "db2"):
-            assert sum_err(g[k], ref[k], A[k], tol) <= 1.0, k
-    else:
-        for k in ("dW", "db", "dw1", "db1", "dw2", "db2"):
-            assert relerr(g[k], ref[k]) < tol, k
+    for k in ("dW", "db", "dw1", "db1", "dw2", "db2"):
+        assert relerr(g[k], ref[k]) < tol, k
     if case.lengths is not None:
         for b, ln in enumerate(case.lengths):
             for k in ("dQ", "dK", "dV"):
                 assert np.all(g[k][b, :, ln:] == 0)
+
+
+@pytest.mark.parametrize("seed", [21, 22, 23, 24])
+@pytest.mark.parametrize("causal,d,lengths", [(False, 64, None), (False, 32, [300, 123]), (True, 32, [300, 201])])
+def test_backward_fp32_parameter_gradients(seed, causal, d, lengths):
+    """fp32 I/O: every parameter gradient within the plain 1e-4 gate on several
+    seeds.  These gradients are sums over every row, projection and channel
+    whose terms cancel to a few hundredths of a percent of their absolute sum
+    (the loss barely changes under a common scale of the features)."""
+    case = Case(len(lengths) if lengths else 1, 2, 300, d, 8, 8, "f32", causal, seed=seed,
+                qkv_scale=1.0 / math.sqrt(d), lengths=lengths, with_grad=True)
+    lu = case.luna()
+    case.run_fwd(lu)
+    g = {k: to_host(v) for k, v in case.run_bwd(lu).items()}
+    ref = case.oracle_bwd()
+    for k in ("dW", "db", "dw1", "db1", "dw2", "db2"):
+        assert relerr(g[k], ref[k]) < TOL["f32"], k
 
 
 def _check_bwd(case, g, ref, tol):
@@ -481,13 +493,8 @@ def test_shared_channel_mlp(io, d, M, causal):
     assert relerr(g["dK"][okk], rb["dK"][okk]) < TOL[io]
     assert relerr(g["dV"], rb["dV"]) < TOL[io]
     assert g["dw1"].shape == (64,) and g["db1"].shape == (64,)
-    if io == "f32":
-        A = case.oracle_bwd_abs_terms()
-        for k in ("dW", "db", "dw1", "db1", "dw2", "db2"):
-            assert sum_err(g[k], rb[k], A[k], TOL[io]) <= 1.0, k
-    else:
-        for k in ("dW", "db", "dw1", "db1", "dw2", "db2"):
-            assert relerr(g[k], rb[k]) < TOL[io], k
+    for k in ("dW", "db", "dw1", "db1", "dw2", "db2"):
+        assert relerr(g[k], rb[k]) < TOL[io], k
 
 
 def test_shared_channel_featmap():
@@ -533,18 +540,62 @@ def test_channel_rms_normalisation(io, d, M, lengths):
     okq, okk = case.smooth_rows("Q"), case.smooth_rows("K")
     assert okq.mean() > 0.9 and okk.mean() > 0.9
     rb = case.oracle_bwd()
-    A = case.oracle_bwd_abs_terms() if io == "f32" else None
     for use_state in (True, False):
         g = {k: to_host(v) for k, v in case.run_bwd(lu, use_state=use_state).items()}
         assert relerr(g["dQ"][okq], rb["dQ"][okq]) < TOL[io], use_state
         assert relerr(g["dK"][okk], rb["dK"][okk]) < TOL[io], use_state
         assert relerr(g["dV"], rb["dV"]) < TOL[io], use_state
         for k in ("dW", "db", "dw1", "db1", "dw2", "db2"):
-            if io == "f32":
-                assert sum_err(g[k], rb[k], A[k], TOL[io]) <= 1.0, (k, use_state)
-            else:
-                assert relerr(g[k], rb[k]) < TOL[io], (k, use_state)
+            assert relerr(g[k], rb[k]) < TOL[io], (k, use_state)
         if case.lengths is not None:
             for b, ln in enumerate(case.lengths):
                 for k in ("dQ", "dK", "dV"):
                     assert np.all(g[k][b, :, ln:] == 0)
+
+
+# --------------------------------------------------------------------------
+# attention weights of a block of query rows (conversion, stage 1)
+
+@pytest.mark.parametrize("teacher", [False, True])
+@pytest.mark.parametrize("io,d,M,causal,lengths,row0,rows", [
+    ("f32", 64, 8, False, [300, 177], 0, 300),
+    ("bf16", 32, 8, False, [300, 1], 37, 70),
+    ("f32", 128, 16, True, [300, 250], 100, 131),
+    ("bf16", 64, 8, True, None, 250, 50),
+])
+def test_attention_weights(io, d, M, causal, lengths, row0, rows, teacher):
+    """luna_attn_weights against the oracle's weights: LUNA's normalised kernel
+    weights (whose product with V is the attention output) and the softmax
+    teacher's, for a window of query rows with ragged 32-row blocks, padded
+    sequences (including a one-token one), causal and not; masked entries and
+    padded rows exactly zero, every row a distribution."""
+    import torch
+    import paper_2512_08061_gb300.luna as L
+    case = Case(2, 2, 300, d, M, 8, io, causal, seed=97, qkv_scale=1.0 / math.sqrt(d), lengths=lengths)
+    lu = case.luna()
+    A = torch.full((2, 2, rows, 300), float("nan"), dtype=torch.float32, device="cuda")
+    L.luna_attn_weights(lu.ad, lu.pd, lu.table, case.dev["Q"], case.dev["K"], case.dev["lengths"], row0, rows,
+                        teacher, A)
+    got = to_host(A)
+    i = case.inp
+    ref = oracle.attn_weights(case.params, i["Q"].value, i["K"].value, case.lengths, causal, case.eps, row0, rows,
+                              teacher)
+    assert np.all(np.isfinite(got))
+    assert np.array_equal(got == 0, ref == 0)  # the same masked keys and padded rows
+    assert relerr(got, ref) < TOL[io]
+    s = got.sum(-1)
+    live = ref.sum(-1) > 0
+    assert np.allclose(s[live], 1.0, atol=1e-4)
+
+
+def test_attention_weights_times_values_is_the_forward():
+    """The weights of every row times V equals luna_attn_fwd's output (fp32)."""
+    import torch
+    import paper_2512_08061_gb300.luna as L
+    case = Case(1, 2, 200, 32, 8, 8, "f32", False, seed=101, qkv_scale=1.0 / math.sqrt(32), lengths=[150])
+    lu = case.luna()
+    O = to_host(case.run_fwd(lu))
+    A = torch.empty((1, 2, 200, 200), dtype=torch.float32, device="cuda")
+    L.luna_attn_weights(lu.ad, lu.pd, lu.table, case.dev["Q"], case.dev["K"], case.dev["lengths"], 0, 200, False, A)
+    AV = to_host(A) @ case.inp["V"].value
+    assert relerr(AV, O) < 1e-4

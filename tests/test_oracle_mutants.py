@@ -68,7 +68,18 @@ SIGNED_MUTANTS = {
         "if (!p->signed_out && !(y > 0.0)) continue;", "if (!(y > 0.0)) continue;"),
 }
 
+WEIGHTS_PINS = "tests/test_oracle_weights.py"
+WEIGHTS_MUTANTS = {
+    "weights: eps dropped from the normaliser": (
+        "double den = eps;\n            for (int j = 0; j < jmax; ++j) {\n                double kij",
+        "double den = 0.0;\n            for (int j = 0; j < jmax; ++j) {\n                double kij"),
+    "weights: exclusive causal mask": (
+        "const int jmax = causal ? i + 1 : len;", "const int jmax = causal ? i : len;"),
+    "teacher: 1/sqrt(d) scale dropped": ("ar[j] = s / sqrt((double)d);", "ar[j] = s;"),
+}
+
 ALL = {**{k: (v, "tests/test_oracle_pins.py") for k, v in MUTANTS.items()},
+       **{k: (v, WEIGHTS_PINS) for k, v in WEIGHTS_MUTANTS.items()},
        **{k: (v, SIGNED_PINS) for k, v in SIGNED_MUTANTS.items()},
        **{k: (v, CH_RMS_PINS) for k, v in CH_RMS_MUTANTS.items()},
        **{k: (v, PER_HEAD_PINS) for k, v in PER_HEAD_MUTANTS.items()}}
