@@ -104,6 +104,7 @@ __global__ void __launch_bounds__(kThreads) k_causal_out(AttnArgs a) {
     float *sQ = cv.take(kCs * d), *sK = cv.take(kCs * d), *sV = cv.take(kCs * dv);
     float *sPq = cv.take(kCs * D), *sPk = cv.take(kCs * D), *sA = cv.take(kCs * kCs);
     float *sden = cv.take(kCs), *sO = cv.take(kCs * dv);
+    if (!carve_fits(cv, smem)) return;
     const int bh = blockIdx.y, seg = blockIdx.x;
     const int len = head_length(a.lengths, bh / a.H, a.n);
     const int r0 = seg * a.seg_len, rend = min(a.n, r0 + a.seg_len), r1 = min(len, rend);
@@ -143,6 +144,7 @@ __global__ void __launch_bounds__(kThreads) k_causal_bwd_seg(AttnArgs a) {
     float *sQ = cv.take(kCs * d), *sK = cv.take(kCs * d), *sV = cv.take(kCs * dv), *sdO = cv.take(kCs * dv);
     float *sPq = cv.take(kCs * D), *sPk = cv.take(kCs * D), *sA = cv.take(kCs * kCs);
     float *sden = cv.take(kCs), *sdden = cv.take(kCs), *sO = cv.take(kCs * dv);
+    if (!carve_fits(cv, smem)) return;
     const int bh = blockIdx.y, seg = blockIdx.x;
     const int len = head_length(a.lengths, bh / a.H, a.n);
     const int r0 = seg * a.seg_len, rend = min(a.n, r0 + a.seg_len), r1 = min(len, rend);
@@ -212,6 +214,7 @@ __global__ void __launch_bounds__(kThreads) k_causal_dq(AttnArgs a) {
     float *sU = cv.take(kCs * M);
     int *sJ = reinterpret_cast<int *>(cv.take(kCs * M));
     float *sdU = cv.take(kCs * M);
+    if (!carve_fits(cv, smem)) return;
     const int bh = blockIdx.y, seg = blockIdx.x;
     double *gp = reinterpret_cast<double *>(a.gpart) + ((size_t)bh * a.nseg + seg) * a.gsize;
     double *shist = gp + M * d + M;  // the block's fp64 histogram, accumulated in place by L2 atomics
@@ -286,6 +289,7 @@ __global__ void __launch_bounds__(kThreads) k_causal_dkv(AttnArgs a) {
     float *sU = cv.take(kCs * M);
     int *sJ = reinterpret_cast<int *>(cv.take(kCs * M));
     float *sdU = cv.take(kCs * M);
+    if (!carve_fits(cv, smem)) return;
     const int bh = blockIdx.y, seg = blockIdx.x;
     double *gp = reinterpret_cast<double *>(a.gpart) + ((size_t)a.B * a.H * a.nseg + (size_t)bh * a.nseg + seg) * a.gsize;
     double *shist = gp + M * d + M;  // the block's fp64 histogram, accumulated in place by L2 atomics

@@ -242,6 +242,7 @@ __global__ void __launch_bounds__(kKWarps * 32) k_chrms_kterm(AttnArgs a, const 
     float *sk = reinterpret_cast<float *>(sdb + r4(M));
     float *sx = sk + r4(kMaxL) + warp * (r4(32 * dp) + r4(32 * mp));
     float *sdu = sx + r4(32 * dp);
+    if (!carve_fits(Carve{sk + r4(kMaxL) + kKWarps * (r4(32 * dp) + r4(32 * mp))}, smem)) return;
     const int Md = M * d;
     GP *gp = gpart + ((size_t)side * gridDim.x + blockIdx.x) * a.gsize;
     GP *ghist = gp + Md + M;

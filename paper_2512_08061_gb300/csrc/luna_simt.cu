@@ -25,6 +25,7 @@ __global__ void __launch_bounds__(kThreads) k_featmap(TableLayout lay, const cha
     extern __shared__ __align__(16) float smem[];
     Carve cv{smem};
     SmemPhi s = carve_phi(cv, lay);
+    if (!carve_fits(cv, smem)) return;
     load_phi(s, lay, table);
     __syncthreads();
     const int M = lay.M, L = lay.L, d = lay.d, D = lay.D;
@@ -54,6 +55,7 @@ __global__ void __launch_bounds__(kThreads) k_keystats(AttnArgs a) {
     float *sK = cv.take(kTileK * a.d);
     float *sV = cv.take(kTileK * a.dv);
     float *sPhi = cv.take(kTileK * a.D);
+    if (!carve_fits(cv, smem)) return;
     load_phi(s, lay, a.table);
 
     const int bh = blockIdx.y, split = blockIdx.x;
@@ -118,6 +120,7 @@ __global__ void __launch_bounds__(kThreads) k_query(AttnArgs a) {
     float *sQ = cv.take(kTileQ * a.d);
     float *sPhi = cv.take(kTileQ * a.D);
     float *sden = cv.take(kTileQ);
+    if (!carve_fits(cv, smem)) return;
     load_phi(s, lay, a.table);
     for (int e = threadIdx.x; e < a.D * a.dv; e += blockDim.x) sS[e] = a.S_fin[(size_t)bh * a.D * a.dv + e];
     for (int e = threadIdx.x; e < a.D; e += blockDim.x) sz[e] = a.z_fin[(size_t)bh * a.D + e];
@@ -166,6 +169,7 @@ __global__ void __launch_bounds__(kThreads) k_bwd_query(AttnArgs a) {
     float *sU = cv.take(kTileB * M);
     int *sJ = reinterpret_cast<int *>(cv.take(kTileB * M));
     float *sdU = cv.take(kTileB * M);
+    if (!carve_fits(cv, smem)) return;
     load_phi(s, lay, a.table);
     const int bh = blockIdx.y, split = blockIdx.x;
     const size_t slot = (size_t)bh * a.nsplit_b + split;
@@ -266,6 +270,7 @@ __global__ void __launch_bounds__(kThreads) k_bwd_key(AttnArgs a) {
     float *sU = cv.take(kTileB * M);
     int *sJ = reinterpret_cast<int *>(cv.take(kTileB * M));
     float *sdU = cv.take(kTileB * M);
+    if (!carve_fits(cv, smem)) return;
     load_phi(s, lay, a.table);
     const int bh = blockIdx.y, split = blockIdx.x;
     const size_t slot = (size_t)a.B * a.H * a.nsplit_b + (size_t)bh * a.nsplit_b + split;
@@ -494,7 +499,7 @@ size_t smem_bwd_query(const AttnArgs &a) {
     HostCarve cv; carve_phi_host(cv, a.lay);
     cv.take(a.D * a.dv); cv.take(a.D); cv.take(kTileB * a.d); cv.take(kTileB * a.dv); cv.take(kTileB * a.D);
     cv.take(kTileB * a.D); cv.take(kTileB * a.dv); cv.take(kTileB); cv.take(kTileB); cv.take(kTileB * a.M);
-    cv.take(kTileB * a.M);
+    cv.take(kTileB * a.M); cv.take(kTileB * a.M);
     return cv.bytes();
 }
 size_t smem_bwd_key(const AttnArgs &a) {

@@ -23,6 +23,15 @@ struct Carve {
     }
 };
 
+// True when the arrays carved so far fit in the block's dynamic shared memory (the host sizes the
+// launch with a HostCarve of the same arrays; a kernel whose carve does not fit returns before it
+// touches shared memory, so a mismatch shows as a wrong result, not as an out-of-bounds access).
+__device__ __forceinline__ bool carve_fits(const Carve &cv, const float *base) {
+    uint32_t dyn;
+    asm volatile("mov.u32 %0, %%dynamic_smem_size;" : "=r"(dyn));
+    return (size_t)(cv.p - base) * sizeof(float) <= (size_t)dyn;
+}
+
 struct HostCarve {
     int n = 0;
     void take(int k) { n += r4(k); }

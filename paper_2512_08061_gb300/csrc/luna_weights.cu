@@ -39,6 +39,7 @@ __global__ void __launch_bounds__(kThreads) k_weights(AttnArgs a, int causal, in
     float *sPq = cv.take(kWRows * D);
     float *sK = cv.take(kWKeys * d);
     float *sPk = cv.take(kWKeys * D);
+    if (!carve_fits(cv, smem)) return;
     const int bh = blockIdx.y;
     const int len = head_length(a.lengths, bh / a.H, n);
     const int r_lo = blockIdx.x * kWRows;              // first output row of this block (relative to row0)
