@@ -76,6 +76,12 @@ typedef enum { LUNA_F32 = 0, LUNA_BF16 = 1 } luna_dtype;
  * LUNA_ERR_INVALID_ARG.  With it on, only the non-causal luna_attn_fwd /
  * luna_attn_bwd are supported (the causal form, luna_featmap and
  * luna_attn_decode give LUNA_ERR_UNSUPPORTED).
+ * signed_outputs = 1 is the listing's ScalarMLP(nonneg = False): the channel
+ * outputs are fc2(relu(fc1(u))) without the outer ReLU, so features (and kernel
+ * values) of either sign; 0 keeps the outer ReLU (the listing's default).  The
+ * table is the same for both (the flag is read from the descriptor by every
+ * call, so pass the same descriptor to all calls of one problem); with
+ * ch_rms_target > 0 it gives LUNA_ERR_UNSUPPORTED.
  * Supported: 1 <= M, 1 <= L <= 16, M*L <= 128, 1 <= hidden <= 128, L*hidden <= 512. */
 typedef struct {
     int M;               /* number of projections w_i (rows of W)       */
@@ -83,6 +89,7 @@ typedef struct {
     int hidden;          /* hidden width of each (or the shared) MLP     */
     int shared_channels; /* 0 or 1, see above                           */
     float ch_rms_target; /* channel RMS normalisation target, 0 = off   */
+    int signed_outputs;  /* 0 or 1, see above                           */
 } luna_phi_desc;
 
 /* Feature-map parameters, fp32 device arrays, row-major:

@@ -21,7 +21,9 @@ luna_status check_phi(const luna_phi_desc *pd, int d) {
     if (!pd) return LUNA_ERR_INVALID_ARG;
     if (pd->M < 1 || pd->L < 1 || pd->hidden < 1 || d < 1) return LUNA_ERR_INVALID_ARG;
     if (pd->shared_channels != 0 && pd->shared_channels != 1) return LUNA_ERR_INVALID_ARG;
+    if (pd->signed_outputs != 0 && pd->signed_outputs != 1) return LUNA_ERR_INVALID_ARG;
     if (!(pd->ch_rms_target >= 0.0f) || isinf(pd->ch_rms_target)) return LUNA_ERR_INVALID_ARG;
+    if (pd->signed_outputs && pd->ch_rms_target > 0.0f) return LUNA_ERR_UNSUPPORTED;
     if (pd->L > kMaxL || pd->M * pd->L > kMaxFeat || pd->M > 32 || pd->hidden > kMaxHidden ||
         pd->L * pd->hidden > kMaxUnits || d > kMaxD || pd->M * d > 4096)
         return LUNA_ERR_UNSUPPORTED;
@@ -81,7 +83,7 @@ luna_status make_plan(const luna_attn_desc *ad, const luna_phi_desc *pd, Plan &p
     p.ch_target = pd->ch_rms_target;
     if ((int64_t)ad->B * ad->H > (1 << 24)) return LUNA_ERR_UNSUPPORTED;
 
-    p.lay = table_layout(pd->M, pd->L, pd->hidden, ad->d, pd->shared_channels);
+    p.lay = table_layout(pd->M, pd->L, pd->hidden, ad->d, pd->shared_channels, pd->signed_outputs);
     const int BH = ad->B * ad->H, n = ad->n, D = p.lay.D, dv = ad->dv;
     p.BH = BH;
     p.gsize = pd->M * ad->d + pd->M + p.lay.nint * pd->L * 2;
@@ -247,7 +249,7 @@ luna_status luna_phi_table_size(const luna_phi_desc *pd, int d, size_t *bytes) {
     if (!bytes) return LUNA_ERR_INVALID_ARG;
     luna_status st = check_phi(pd, d);
     if (st != LUNA_OK) return st;
-    *bytes = (size_t)table_layout(pd->M, pd->L, pd->hidden, d, pd->shared_channels).bytes;
+    *bytes = (size_t)table_layout(pd->M, pd->L, pd->hidden, d, pd->shared_channels, pd->signed_outputs).bytes;
     return LUNA_OK;
 }
 
@@ -258,7 +260,7 @@ luna_status luna_phi_prepare(const luna_phi_desc *pd, int d, const luna_phi_para
     if (!params || !table || !params->W || !params->b || !params->w1 || !params->b1 || !params->w2 || !params->b2)
         return LUNA_ERR_INVALID_ARG;
     if (!aligned(table, 256)) return LUNA_ERR_INVALID_ARG;
-    TableLayout lay = table_layout(pd->M, pd->L, pd->hidden, d, pd->shared_channels);
+    TableLayout lay = table_layout(pd->M, pd->L, pd->hidden, d, pd->shared_channels, pd->signed_outputs);
     if (table_bytes < (size_t)lay.bytes) return LUNA_ERR_WORKSPACE;
     return cuda_status(launch_phi_prepare(*params, lay, table, static_cast<cudaStream_t>(stream)));
 }
@@ -271,7 +273,7 @@ luna_status luna_featmap(const luna_phi_desc *pd, int d, const void *table, cons
     if (pd->ch_rms_target > 0.0f) return LUNA_ERR_UNSUPPORTED;
     if (rows == 0) return LUNA_OK;
     if (!table || !X || !Phi) return LUNA_ERR_INVALID_ARG;
-    TableLayout lay = table_layout(pd->M, pd->L, pd->hidden, d, pd->shared_channels);
+    TableLayout lay = table_layout(pd->M, pd->L, pd->hidden, d, pd->shared_channels, pd->signed_outputs);
     return cuda_status(launch_featmap(lay, static_cast<const char *>(table), X, xtype, rows, Phi,
                                       static_cast<cudaStream_t>(stream)));
 }
@@ -407,7 +409,7 @@ luna_status luna_attn_weights(const luna_attn_desc *ad, const luna_phi_desc *pd,
     AttnArgs a;
     memset(&a, 0, sizeof(a));
     a.B = ad->B; a.H = ad->H; a.n = ad->n; a.d = ad->d; a.dv = ad->dv;
-    a.lay = table_layout(pd->M, pd->L, pd->hidden, ad->d, pd->shared_channels);
+    a.lay = table_layout(pd->M, pd->L, pd->hidden, ad->d, pd->shared_channels, pd->signed_outputs);
     a.M = a.lay.M; a.L = a.lay.L; a.D = a.lay.D;
     a.eps = ad->eps;
     a.table = static_cast<const char *>(table);
@@ -447,7 +449,7 @@ luna_status luna_attn_decode(const luna_attn_desc *ad, const luna_phi_desc *pd, 
     if (pd->ch_rms_target > 0.0f) return LUNA_ERR_UNSUPPORTED;  // a batch statistic: no single-token step
     const int64_t BH = (int64_t)ad->B * ad->H;
     if (BH > (1 << 24)) return LUNA_ERR_UNSUPPORTED;
-    const TableLayout lay = table_layout(pd->M, pd->L, pd->hidden, ad->d, pd->shared_channels);
+    const TableLayout lay = table_layout(pd->M, pd->L, pd->hidden, ad->d, pd->shared_channels, pd->signed_outputs);
     const int64_t SD = (int64_t)lay.D * ad->dv;
     if (S_stride == 0) S_stride = SD;
     if (z_stride == 0) z_stride = lay.D;

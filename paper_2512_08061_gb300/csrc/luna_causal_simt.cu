@@ -35,10 +35,11 @@ struct ChunkBufs {
 
 template <typename IO>
 __device__ void load_chunk(const AttnArgs &a, int bh, int t0, int nr, float *sQ, float *sK, float *sV, float *sdO) {
-    load_rows(sQ, static_cast<const IO *>(a.Q) + ((size_t)bh * a.n + t0) * a.d, nr * a.d);
-    load_rows(sK, static_cast<const IO *>(a.K) + ((size_t)bh * a.n + t0) * a.d, nr * a.d);
-    load_rows(sV, static_cast<const IO *>(a.V) + ((size_t)bh * a.n + t0) * a.dv, nr * a.dv);
-    if (sdO) load_rows(sdO, static_cast<const IO *>(a.dO) + ((size_t)bh * a.n + t0) * a.dv, nr * a.dv);
+    const size_t r0 = head_rows(a, bh) + t0;
+    load_rows(sQ, static_cast<const IO *>(a.Q) + r0 * a.d, nr * a.d);
+    load_rows(sK, static_cast<const IO *>(a.K) + r0 * a.d, nr * a.d);
+    load_rows(sV, static_cast<const IO *>(a.V) + r0 * a.dv, nr * a.dv);
+    if (sdO) load_rows(sdO, static_cast<const IO *>(a.dO) + r0 * a.dv, nr * a.dv);
 }
 
 // sA[r][j] = phi(q_r) . phi(k_j) for j <= r (0 above the diagonal)
@@ -108,11 +109,11 @@ __global__ void __launch_bounds__(kThreads) k_causal_out(AttnArgs a) {
     const int bh = blockIdx.y, seg = blockIdx.x;
     const int len = head_length(a.lengths, bh / a.H, a.n);
     const int r0 = seg * a.seg_len, rend = min(a.n, r0 + a.seg_len), r1 = min(len, rend);
-    IO *O = static_cast<IO *>(a.O) + (size_t)bh * a.n * dv;
+    IO *O = static_cast<IO *>(a.O) + head_rows(a, bh) * dv;
     for (int e = threadIdx.x + max(r0, len) * dv; e < rend * dv; e += blockDim.x) io_store(O + e, 0.0f);
     if (r0 >= r1) return;
     load_phi(s, lay, a.table);
-    const size_t so = ((size_t)bh * (a.nseg + 1) + seg);
+    const size_t so = head_state(a, bh) * (a.nseg + 1) + seg;
     for (int e = threadIdx.x; e < D * dv; e += blockDim.x) S[e] = a.seg_S[so * D * dv + e];
     for (int e = threadIdx.x; e < D; e += blockDim.x) z[e] = a.seg_z[so * D + e];
     for (int t0 = r0; t0 < r1; t0 += kCs) {
@@ -149,7 +150,7 @@ __global__ void __launch_bounds__(kThreads) k_causal_bwd_seg(AttnArgs a) {
     const int len = head_length(a.lengths, bh / a.H, a.n);
     const int r0 = seg * a.seg_len, rend = min(a.n, r0 + a.seg_len), r1 = min(len, rend);
     load_phi(s, lay, a.table);
-    const size_t so = ((size_t)bh * (a.nseg + 1) + seg);
+    const size_t so = head_state(a, bh) * (a.nseg + 1) + seg;
     for (int e = threadIdx.x; e < D * dv; e += blockDim.x) S[e] = a.seg_S[so * D * dv + e];
     for (int e = threadIdx.x; e < D; e += blockDim.x) z[e] = a.seg_z[so * D + e];
     const int nc = (dv + 7) / 8, nf = (D + 7) / 8;
@@ -220,10 +221,10 @@ __global__ void __launch_bounds__(kThreads) k_causal_dq(AttnArgs a) {
     double *shist = gp + M * d + M;  // the block's fp64 histogram, accumulated in place by L2 atomics
     const int len = head_length(a.lengths, bh / a.H, a.n);
     const int r0 = seg * a.seg_len, rend = min(a.n, r0 + a.seg_len), r1 = min(len, rend);
-    IO *dQ = static_cast<IO *>(a.dQ) + (size_t)bh * a.n * d;
+    IO *dQ = static_cast<IO *>(a.dQ) + head_rows(a, bh) * d;
     for (int e = threadIdx.x + max(r0, len) * d; e < rend * d; e += blockDim.x) io_store(dQ + e, 0.0f);
     load_phi(s, lay, a.table);
-    const size_t so = ((size_t)bh * (a.nseg + 1) + seg);
+    const size_t so = head_state(a, bh) * (a.nseg + 1) + seg;
     for (int e = threadIdx.x; e < D * dv; e += blockDim.x) S[e] = a.seg_S[so * D * dv + e];
     for (int e = threadIdx.x; e < D; e += blockDim.x) z[e] = a.seg_z[so * D + e];
     for (int e = threadIdx.x; e < lay.nint * lay.L * 2; e += blockDim.x) shist[e] = 0.0;
@@ -295,8 +296,8 @@ __global__ void __launch_bounds__(kThreads) k_causal_dkv(AttnArgs a) {
     double *shist = gp + M * d + M;  // the block's fp64 histogram, accumulated in place by L2 atomics
     const int len = head_length(a.lengths, bh / a.H, a.n);
     const int r0 = seg * a.seg_len, rend = min(a.n, r0 + a.seg_len), r1 = min(len, rend);
-    IO *dK = static_cast<IO *>(a.dK) + (size_t)bh * a.n * d;
-    IO *dV = static_cast<IO *>(a.dV) + (size_t)bh * a.n * dv;
+    IO *dK = static_cast<IO *>(a.dK) + head_rows(a, bh) * d;
+    IO *dV = static_cast<IO *>(a.dV) + head_rows(a, bh) * dv;
     for (int e = threadIdx.x + max(r0, len) * d; e < rend * d; e += blockDim.x) io_store(dK + e, 0.0f);
     for (int e = threadIdx.x + max(r0, len) * dv; e < rend * dv; e += blockDim.x) io_store(dV + e, 0.0f);
     load_phi(s, lay, a.table);

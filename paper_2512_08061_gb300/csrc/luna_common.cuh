@@ -38,13 +38,15 @@ __host__ __device__ inline int64_t align256(int64_t x) { return (x + 255) & ~int
 struct TableLayout {
     int M, L, hid, d, D, P, Ppad, nint;
     int shared;  // one MLP for all channels: P = hid kinks (else P = L * hid)
+    int signed_out;  // channel outputs without the outer ReLU (the listing's nonneg = False)
     int64_t off_T, off_Te, off_AB, off_W, off_b, off_rank, off_utype, off_w1, off_b1, off_w2, off_b2, bytes;
 };
 
-__host__ __device__ inline TableLayout table_layout(int M, int L, int hid, int d, int shared = 0) {
+__host__ __device__ inline TableLayout table_layout(int M, int L, int hid, int d, int shared = 0, int signed_out = 0) {
     TableLayout t;
     t.M = M; t.L = L; t.hid = hid; t.d = d; t.D = M * L;
     t.shared = shared ? 1 : 0;
+    t.signed_out = signed_out ? 1 : 0;
     t.P = shared ? hid : L * hid;
     t.Ppad = next_pow2(t.P);
     t.nint = t.P + 1;
@@ -82,6 +84,13 @@ __device__ __forceinline__ void io_store(__nv_bfloat16 *p, float v) { *p = __flo
 
 // ---------------------------------------------------------------------------
 // Feature map from the table
+
+// Lower bound of a channel output: 0 (outer ReLU, the listing's default) or -inf (signed outputs).
+// Every channel value is fmaxf(alpha u + beta, floor), and an output is active in the backward pass
+// where it is above the floor.
+__host__ __device__ __forceinline__ float channel_floor(const TableLayout &lay) {
+    return lay.signed_out ? -INFINITY : 0.0f;
+}
 
 // Number of sorted thresholds strictly below u (branch-free lower bound over a
 // power-of-two sized array whose tail is padded with +inf).

@@ -68,6 +68,7 @@ __global__ void __launch_bounds__(kDecThreads) k_decode(DecodeArgs a) {
     __syncthreads();
     // phi: interval of u in the breadth-first kink tree, then relu(alpha u + beta) per channel
     const float2 *AB = reinterpret_cast<const float2 *>(a.table + a.lay.off_AB);
+    const float fl = channel_floor(a.lay);
     for (int p = tid; p < 2 * M; p += blockDim.x) {
         const int side = p / M, m = p % M;
         const float u = su[side][m];
@@ -81,13 +82,13 @@ __global__ void __launch_bounds__(kDecThreads) k_decode(DecodeArgs a) {
             for (int k = 0; k < 4; ++k) w[k] = __ldg(ab4 + k);
 #pragma unroll
             for (int k = 0; k < 4; ++k) {
-                sphi[side][m * 8 + 2 * k] = fmaxf(fmaf(w[k].x, u, w[k].y), 0.0f);
-                sphi[side][m * 8 + 2 * k + 1] = fmaxf(fmaf(w[k].z, u, w[k].w), 0.0f);
+                sphi[side][m * 8 + 2 * k] = fmaxf(fmaf(w[k].x, u, w[k].y), fl);
+                sphi[side][m * 8 + 2 * k + 1] = fmaxf(fmaf(w[k].z, u, w[k].w), fl);
             }
         } else {
             for (int l = 0; l < L; ++l) {
                 const float2 ab = __ldg(AB + (size_t)j * L + l);
-                sphi[side][m * L + l] = fmaxf(fmaf(ab.x, u, ab.y), 0.0f);
+                sphi[side][m * L + l] = fmaxf(fmaf(ab.x, u, ab.y), fl);
             }
         }
     }

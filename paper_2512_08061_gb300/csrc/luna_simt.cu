@@ -39,7 +39,7 @@ __global__ void __launch_bounds__(kThreads) k_featmap(TableLayout lay, const cha
         const int j = interval_of(s.T, lay.Ppad, u);
         const float *ab = s.AB + j * L * 2;
         float *out = Phi + r * D + i * L;
-        for (int l = 0; l < L; ++l) out[l] = fmaxf(fmaf(ab[2 * l], u, ab[2 * l + 1]), 0.0f);
+        for (int l = 0; l < L; ++l) out[l] = fmaxf(fmaf(ab[2 * l], u, ab[2 * l + 1]), channel_floor(lay));
     }
 }
 
@@ -62,8 +62,8 @@ __global__ void __launch_bounds__(kThreads) k_keystats(AttnArgs a) {
     const int len = head_length(a.lengths, bh / a.H, a.n);
     const int r0 = split * a.rows_per_split;
     const int r1 = min(len, r0 + a.rows_per_split);
-    const IO *K = static_cast<const IO *>(a.K) + (size_t)bh * a.n * a.d;
-    const IO *V = static_cast<const IO *>(a.V) + (size_t)bh * a.n * a.dv;
+    const IO *K = static_cast<const IO *>(a.K) + head_rows(a, bh) * a.d;
+    const IO *V = static_cast<const IO *>(a.V) + head_rows(a, bh) * a.dv;
 
     const int nc = (a.dv + 7) / 8, nf = (a.D + 7) / 8;
     const bool active = threadIdx.x < nf * nc;
@@ -85,13 +85,13 @@ __global__ void __launch_bounds__(kThreads) k_keystats(AttnArgs a) {
     if (last_arrival(a.counters + bh, a.nsplit)) {
         if (a.seg_S) {  // causal: exclusive prefix at every segment start, total in slot nsplit
             exclusive_scan(a.S_part + (size_t)bh * a.nsplit * a.D * a.dv, a.nsplit, a.D * a.dv,
-                           a.seg_S + (size_t)bh * (a.nsplit + 1) * a.D * a.dv, false);
+                           a.seg_S + head_state(a, bh) * (a.nsplit + 1) * a.D * a.dv, false);
             exclusive_scan(a.z_part + (size_t)bh * a.nsplit * a.D, a.nsplit, a.D,
-                           a.seg_z + (size_t)bh * (a.nsplit + 1) * a.D, false);
+                           a.seg_z + head_state(a, bh) * (a.nsplit + 1) * a.D, false);
         } else {
             ordered_sum(a.S_part + (size_t)bh * a.nsplit * a.D * a.dv, a.nsplit, a.D * a.dv,
-                        a.S_fin + (size_t)bh * a.D * a.dv);
-            ordered_sum(a.z_part + (size_t)bh * a.nsplit * a.D, a.nsplit, a.D, a.z_fin + (size_t)bh * a.D);
+                        a.S_fin + head_state(a, bh) * a.D * a.dv);
+            ordered_sum(a.z_part + (size_t)bh * a.nsplit * a.D, a.nsplit, a.D, a.z_fin + head_state(a, bh) * a.D);
         }
         if (threadIdx.x == 0) a.counters[bh] = 0;
     }
@@ -106,7 +106,7 @@ __global__ void __launch_bounds__(kThreads) k_query(AttnArgs a) {
     const int bh = blockIdx.y;
     const int q0 = blockIdx.x * kTileQ;
     const int len = head_length(a.lengths, bh / a.H, a.n);
-    IO *O = static_cast<IO *>(a.O) + (size_t)bh * a.n * a.dv;
+    IO *O = static_cast<IO *>(a.O) + head_rows(a, bh) * a.dv;
     const int nrows = min(kTileQ, a.n - q0);
     if (q0 >= len) {  // padded rows only
         for (int e = threadIdx.x; e < nrows * a.dv; e += blockDim.x) io_store(O + (size_t)q0 * a.dv + e, 0.0f);
@@ -122,10 +122,10 @@ __global__ void __launch_bounds__(kThreads) k_query(AttnArgs a) {
     float *sden = cv.take(kTileQ);
     if (!carve_fits(cv, smem)) return;
     load_phi(s, lay, a.table);
-    for (int e = threadIdx.x; e < a.D * a.dv; e += blockDim.x) sS[e] = a.S_fin[(size_t)bh * a.D * a.dv + e];
-    for (int e = threadIdx.x; e < a.D; e += blockDim.x) sz[e] = a.z_fin[(size_t)bh * a.D + e];
+    for (int e = threadIdx.x; e < a.D * a.dv; e += blockDim.x) sS[e] = a.S_fin[head_state(a, bh) * a.D * a.dv + e];
+    for (int e = threadIdx.x; e < a.D; e += blockDim.x) sz[e] = a.z_fin[head_state(a, bh) * a.D + e];
     const int nr = min(nrows, len - q0);
-    load_rows(sQ, static_cast<const IO *>(a.Q) + ((size_t)bh * a.n + q0) * a.d, nr * a.d);
+    load_rows(sQ, static_cast<const IO *>(a.Q) + (head_rows(a, bh) + q0) * a.d, nr * a.d);
     __syncthreads();
     phi_tile(lay, s, sQ, nr, sPhi, nullptr, nullptr);
     __syncthreads();
@@ -175,17 +175,17 @@ __global__ void __launch_bounds__(kThreads) k_bwd_query(AttnArgs a) {
     const size_t slot = (size_t)bh * a.nsplit_b + split;
     double *gp = reinterpret_cast<double *>(a.gpart) + slot * a.gsize;
     double *shist = gp + M * d + M;  // the block's fp64 histogram, accumulated in place by L2 atomics
-    for (int e = threadIdx.x; e < D * dv; e += blockDim.x) sS[e] = a.S_fin[(size_t)bh * D * dv + e];
-    for (int e = threadIdx.x; e < D; e += blockDim.x) sz[e] = a.z_fin[(size_t)bh * D + e];
+    for (int e = threadIdx.x; e < D * dv; e += blockDim.x) sS[e] = a.S_fin[head_state(a, bh) * D * dv + e];
+    for (int e = threadIdx.x; e < D; e += blockDim.x) sz[e] = a.z_fin[head_state(a, bh) * D + e];
     for (int e = threadIdx.x; e < lay.nint * lay.L * 2; e += blockDim.x) shist[e] = 0.0;
 
     const int len = head_length(a.lengths, bh / a.H, a.n);
     const int r0 = split * a.rows_per_split_b;
     const int rend = min(a.n, r0 + a.rows_per_split_b);
     const int r1 = min(len, rend);
-    const IO *Q = static_cast<const IO *>(a.Q) + (size_t)bh * a.n * d;
-    const IO *dO = static_cast<const IO *>(a.dO) + (size_t)bh * a.n * dv;
-    IO *dQ = static_cast<IO *>(a.dQ) + (size_t)bh * a.n * d;
+    const IO *Q = static_cast<const IO *>(a.Q) + head_rows(a, bh) * d;
+    const IO *dO = static_cast<const IO *>(a.dO) + head_rows(a, bh) * dv;
+    IO *dQ = static_cast<IO *>(a.dQ) + head_rows(a, bh) * d;
     // padded rows of this range receive zero gradients
     for (int e = threadIdx.x + max(r0, len) * d; e < rend * d; e += blockDim.x) io_store(dQ + e, 0.0f);
 
@@ -284,10 +284,10 @@ __global__ void __launch_bounds__(kThreads) k_bwd_key(AttnArgs a) {
     const int r0 = split * a.rows_per_split_b;
     const int rend = min(a.n, r0 + a.rows_per_split_b);
     const int r1 = min(len, rend);
-    const IO *K = static_cast<const IO *>(a.K) + (size_t)bh * a.n * d;
-    const IO *V = static_cast<const IO *>(a.V) + (size_t)bh * a.n * dv;
-    IO *dK = static_cast<IO *>(a.dK) + (size_t)bh * a.n * d;
-    IO *dV = static_cast<IO *>(a.dV) + (size_t)bh * a.n * dv;
+    const IO *K = static_cast<const IO *>(a.K) + head_rows(a, bh) * d;
+    const IO *V = static_cast<const IO *>(a.V) + head_rows(a, bh) * dv;
+    IO *dK = static_cast<IO *>(a.dK) + head_rows(a, bh) * d;
+    IO *dV = static_cast<IO *>(a.dV) + head_rows(a, bh) * dv;
     for (int e = threadIdx.x + max(r0, len) * d; e < rend * d; e += blockDim.x) io_store(dK + e, 0.0f);
     for (int e = threadIdx.x + max(r0, len) * dv; e < rend * dv; e += blockDim.x) io_store(dV + e, 0.0f);
 

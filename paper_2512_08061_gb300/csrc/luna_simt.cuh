@@ -37,6 +37,10 @@ struct AttnArgs {
     void *phik, *pq2;                  // [BH][n][2D] bf16 phi(k), phi(q)/den, each as (hi | lo)
     // tensor-core work items balanced by valid tiles (non-causal, with lengths): workspace for the split
     // ([kMaxGrid + 1] block starts, [2*BH] runs), and the split in use (null: by count)
+    // per-head parameters run one sub-problem per head index h (over the B sequences): head bh of the
+    // sub-problem is head bh * hs_mul of the caller's tensors and state (base pointers already offset to
+    // head h); hs_mul = 1 otherwise
+    int hs_mul;
     int *items_ws;
     const int *split;                  // block b takes items split[b] .. split[b+1]-1
     const int *runs;                   // [2*BH]: first and last block holding an item of head bh
@@ -50,6 +54,11 @@ struct AttnArgs {
     double *ch_T;                      // [BH][L]: per-head sums of S' . dS + z' dz over each channel's rows
     float *ch_kappa;                   // [2][kMaxL]: factor of y_l in dLoss/dy_l from the scale, per side
 };
+
+// Row offset of head bh in the caller's tensors (Q, K, V, dO, O, dQ, dK, dV), and its index among the
+// caller's per-head state blocks (S, z; the streaming form's segment prefixes).
+__host__ __device__ inline size_t head_rows(const AttnArgs &a, int bh) { return (size_t)bh * a.hs_mul * a.n; }
+__host__ __device__ inline size_t head_state(const AttnArgs &a, int bh) { return (size_t)bh * a.hs_mul; }
 
 // blocks per side of the channel-statistics kernel and of the scale-term backward pass (fixed counts:
 // the sums do not depend on the device)

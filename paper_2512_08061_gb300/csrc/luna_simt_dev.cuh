@@ -75,6 +75,7 @@ __device__ void load_rows(float *dst, const IO *src, int count) {
 __device__ void phi_tile(const TableLayout &lay, const SmemPhi &s, const float *sX, int nr, float *sPhi, float *sU,
                          int *sJ) {
     const int M = lay.M, L = lay.L, d = lay.d, D = lay.D;
+    const float fl = channel_floor(lay);
     for (int e = threadIdx.x; e < nr * M; e += blockDim.x) {
         const int r = e / M, i = e - r * M;
         const float *x = sX + r * d;
@@ -84,7 +85,7 @@ __device__ void phi_tile(const TableLayout &lay, const SmemPhi &s, const float *
         const int j = interval_of(s.T, lay.Ppad, u);
         const float *ab = s.AB + j * L * 2;
         float *out = sPhi + r * D + i * L;
-        for (int l = 0; l < L; ++l) out[l] = fmaxf(fmaf(ab[2 * l], u, ab[2 * l + 1]), 0.0f);
+        for (int l = 0; l < L; ++l) out[l] = fmaxf(fmaf(ab[2 * l], u, ab[2 * l + 1]), fl);
         if (sU) { sU[e] = u; sJ[e] = j; }
     }
 }
@@ -189,6 +190,7 @@ __device__ void phi_backward_tile(const TableLayout &lay, const SmemPhi &s, cons
                                   const float *sPhi, const float *sdPhi, const float *sU, const int *sJ, float *sdU,
                                   double *shist, GradAcc &g) {
     const int M = lay.M, L = lay.L, d = lay.d, D = lay.D;
+    const float fl = channel_floor(lay);
     for (int e = threadIdx.x; e < nr * M; e += blockDim.x) {
         const int r = e / M, i = e - r * M;
         const float u = sU[e];
@@ -197,7 +199,7 @@ __device__ void phi_backward_tile(const TableLayout &lay, const SmemPhi &s, cons
         double du = 0.0;
         for (int l = 0; l < L; ++l) {
             const int f = r * D + i * L + l;
-            if (sPhi[f] > 0.0f) {  // outer ReLU on
+            if (sPhi[f] > fl) {  // outer ReLU on (always, for signed outputs)
                 const double gl = sdPhi[f];
                 du = fma(gl, (double)ab[2 * l], du);
                 if (gl != 0.0) {

@@ -88,7 +88,8 @@ struct Cfg {
 // fp32 normaliser phi . z.
 template <class C>
 __device__ __forceinline__ void phi_row_quarter(int Q, uint32_t tmem_u_row, const float *sTe, const float *sAB,
-                                                const float *sbias, bool valid, int r, uint8_t *phi, uint8_t *plo,
+                                                const float *sbias, float fl, bool valid, int r, uint8_t *phi,
+                                                uint8_t *plo,
                                                 float *zacc, const float *sz, float &den) {
     constexpr int PP = C::PP;
     float u[PP];
@@ -127,8 +128,8 @@ __device__ __forceinline__ void phi_row_quarter(int Q, uint32_t tmem_u_row, cons
 #pragma unroll
             for (int k = 0; k < 4; ++k) {
                 const float4 v = ab[ab_slot(j, k)];
-                y[2 * k] = fmaxf(fmaf(v.x, u[q], v.y), 0.0f);
-                y[2 * k + 1] = fmaxf(fmaf(v.z, u[q], v.w), 0.0f);
+                y[2 * k] = fmaxf(fmaf(v.x, u[q], v.y), fl);
+                y[2 * k + 1] = fmaxf(fmaf(v.z, u[q], v.w), fl);
             }
             if (zacc) {
 #pragma unroll
@@ -328,7 +329,7 @@ __global__ void __launch_bounds__(kThreadsTC, 1)
                     tc_fence_after();
                     uint8_t *ph = Pb + p * 2 * C::PT, *pl = ph + C::PT;
                     const bool valid = r < nvalid;
-                    phi_row_quarter<C>(Q, tbase + lrow + (g & 1) * C::NU, sTe, sAB, sbias, valid, r, ph, pl, zacc,
+                    phi_row_quarter<C>(Q, tbase + lrow + (g & 1) * C::NU, sTe, sAB, sbias, channel_floor(a.lay), valid, r, ph, pl, zacc,
                                    nullptr, dummy);
                     if (!valid && Q == 0) {  // padded rows: clear V so that no garbage enters S
                         wait_or_fail(fullv + v, (g / NV) & 1, failed, status);
@@ -421,8 +422,8 @@ __global__ void __launch_bounds__(kThreadsTC, 1)
                 if (*slast) {
                     __threadfence();
                     ordered_sum4(a.S_part + (size_t)bh * it.nchunk * C::D * C::DV, nruns, C::D * C::DV,
-                                 a.S_fin + (size_t)bh * C::D * C::DV, tid, 128);
-                    ordered_sum4(a.z_part + (size_t)bh * it.nchunk * C::D, nruns, C::D, a.z_fin + (size_t)bh * C::D,
+                                 a.S_fin + head_state(a, bh) * C::D * C::DV, tid, 128);
+                    ordered_sum4(a.z_part + (size_t)bh * it.nchunk * C::D, nruns, C::D, a.z_fin + head_state(a, bh) * C::D,
                                  tid, 128);
                     if (tid == 0) a.counters[bh] = 0;
                 }
@@ -480,7 +481,7 @@ __global__ void __launch_bounds__(kThreadsTC, 1)
     // padded rows of every item of this block produce zeros (unless the split kernel zeroed them)
     for (int item = it.begin; item < it.end && !a.padded_zeroed; ++item) {
         const ItemRange ir = item_range(a, it, item);
-        __nv_bfloat16 *O = static_cast<__nv_bfloat16 *>(a.O) + (size_t)ir.bh * a.n * C::DV;
+        __nv_bfloat16 *O = static_cast<__nv_bfloat16 *>(a.O) + head_rows(a, ir.bh) * C::DV;
         const int z0 = max(ir.r0, ir.r1);
         for (int e = tid; e < (ir.rend - z0) * C::DV / 8; e += kThreadsTC)
             reinterpret_cast<uint4 *>(O + (size_t)z0 * C::DV)[e] = make_uint4(0, 0, 0, 0);
@@ -605,7 +606,7 @@ __global__ void __launch_bounds__(kThreadsTC, 1)
                 // has passed the barrier below.
                 if (pend_g >= 0) { o_out(pend_g, pend_row, pend_dsum); pend_g = -1; }
                 named_sync<kWorkers>(1);
-                const float *Sg = a.S_fin + (size_t)ir.bh * C::D * C::DV;
+                const float *Sg = a.S_fin + head_state(a, ir.bh) * C::D * C::DV;
                 for (int e = tid; e < 2 * C::DV * C::D; e += kWorkers) {
                     const int n = e / C::D, f = e % C::D;
                     __nv_bfloat16 hi, lo;
@@ -613,7 +614,7 @@ __global__ void __launch_bounds__(kThreadsTC, 1)
                     *reinterpret_cast<__nv_bfloat16 *>(Sop + (f / 64) * (2 * C::DV * 128) + sw128_chunk(n, (f % 64) / 8) +
                                                        (f % 8) * 2) = (n < C::DV) ? hi : lo;
                 }
-                for (int e = tid; e < C::D; e += kWorkers) sz[e] = a.z_fin[(size_t)ir.bh * C::D + e];
+                for (int e = tid; e < C::D; e += kWorkers) sz[e] = a.z_fin[head_state(a, ir.bh) * C::D + e];
                 named_sync<kWorkers>(1);
                 cur_bh = ir.bh;
             }
@@ -626,7 +627,7 @@ __global__ void __launch_bounds__(kThreadsTC, 1)
                 tc_fence_after();
                 const bool valid = r < nvalid;
                 float den = 0.0f;
-                phi_row_quarter<C>(Q, tbase + lrow + (g & 1) * C::NU, sTe, sAB, sbias, valid, r, Pb + p * C::PT, nullptr,
+                phi_row_quarter<C>(Q, tbase + lrow + (g & 1) * C::NU, sTe, sAB, sbias, channel_floor(a.lay), valid, r, Pb + p * C::PT, nullptr,
                                nullptr, sz, den);
                 float *dslot = sden + (g & 1) * 512;
                 dslot[Q * 128 + r] = den;
@@ -638,7 +639,7 @@ __global__ void __launch_bounds__(kThreadsTC, 1)
                 const float dsum = dslot[r] + dslot[128 + r] + dslot[256 + r] + dslot[384 + r] + a.eps;
                 if (pend_g >= 0) o_out(pend_g, pend_row, pend_dsum);
                 pend_g = g;
-                pend_row = valid ? ir.bh * a.n + row0 + r : -1;
+                pend_row = valid ? (int)head_rows(a, ir.bh) + row0 + r : -1;
                 pend_dsum = dsum;
             }
         }
@@ -671,12 +672,13 @@ EncodeTiledFn encoder() {
 }
 
 // (width, n, BH) bf16 tensor, boxes of 64 columns x `rows` rows, 128B swizzle,
-// out-of-range elements read as zero.
-bool make_map_impl(CUtensorMap *m, const void *base, int width, int n, int BH, int rows = 128) {
+// out-of-range elements read as zero.  Head z starts hs_mul * n rows after head z - 1 (hs_mul > 1: one
+// head index of each sequence, for per-head parameters).
+bool make_map_impl(CUtensorMap *m, const void *base, int width, int n, int BH, int rows = 128, int hs_mul = 1) {
     EncodeTiledFn enc = encoder();
     if (!enc) return false;
     cuuint64_t dims[3] = {(cuuint64_t)width, (cuuint64_t)n, (cuuint64_t)BH};
-    cuuint64_t strides[2] = {(cuuint64_t)width * 2, (cuuint64_t)n * width * 2};
+    cuuint64_t strides[2] = {(cuuint64_t)width * 2, (cuuint64_t)hs_mul * n * width * 2};
     cuuint32_t box[3] = {64, (cuuint32_t)rows, 1};
     cuuint32_t es[3] = {1, 1, 1};
     return enc(m, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 3, const_cast<void *>(base), dims, strides, box, es,
@@ -728,7 +730,7 @@ __global__ void __launch_bounds__(kSplitThreads) k_tile_split(AttnArgs a, int G,
             const int len = head_length(a.lengths, bh / a.H, a.n);
             if (len >= a.n) continue;
             auto zero = [&](void *X, int w) {  // w: bf16 elements per row (a multiple of 8)
-                uint4 *p = reinterpret_cast<uint4 *>(static_cast<__nv_bfloat16 *>(X) + ((size_t)bh * a.n + len) * w);
+                uint4 *p = reinterpret_cast<uint4 *>(static_cast<__nv_bfloat16 *>(X) + (head_rows(a, bh) + len) * w);
                 const int cnt = (a.n - len) * (w / 8);
                 for (int e = threadIdx.x; e < cnt; e += blockDim.x) p[e] = make_uint4(0, 0, 0, 0);
             };
@@ -867,7 +869,8 @@ AttnArgs balanced_impl(const AttnArgs &a0, cudaStream_t s, cudaError_t *err, int
 template <class C>
 cudaError_t keys_tc(const AttnArgs &a, cudaStream_t s) {
     CUtensorMap mK, mV;
-    if (!make_map_impl(&mK, a.K, a.d, a.n, a.B * a.H) || !make_map_impl(&mV, a.V, a.dv, a.n, a.B * a.H))
+    if (!make_map_impl(&mK, a.K, a.d, a.n, a.B * a.H, 128, a.hs_mul) ||
+        !make_map_impl(&mV, a.V, a.dv, a.n, a.B * a.H, 128, a.hs_mul))
         return cudaErrorInvalidValue;
     cudaError_t e = cudaFuncSetAttribute(k_tc_keys<C>, cudaFuncAttributeMaxDynamicSharedMemorySize, C::SMEM_K);
     if (e != cudaSuccess) return e;
@@ -883,7 +886,7 @@ cudaError_t fwd_tc(const AttnArgs &a0, cudaStream_t s) {
     if ((e = keys_tc<C>(a, s)) != cudaSuccess) return e;
     if ((e = launch_chrms_scale_state(a, s)) != cudaSuccess) return e;
     CUtensorMap mQ;
-    if (!make_map_impl(&mQ, a.Q, a.d, a.n, a.B * a.H)) return cudaErrorInvalidValue;
+    if (!make_map_impl(&mQ, a.Q, a.d, a.n, a.B * a.H, 128, a.hs_mul)) return cudaErrorInvalidValue;
     e = cudaFuncSetAttribute(k_tc_query<C>, cudaFuncAttributeMaxDynamicSharedMemorySize, C::SMEM_Q);
     if (e != cudaSuccess) return e;
     LUNA_LAUNCH("tc_query", k_tc_query<C>, grid_impl(a), kThreadsTC, C::SMEM_Q, s, mQ, a, status_word(a));
@@ -904,11 +907,11 @@ int variant(const luna_attn_desc &ad, const TableLayout &lay) {
 
 }  // namespace
 
-bool tc_make_map(CUtensorMap *m, const void *base, int width, int n, int BH) {
-    return make_map_impl(m, base, width, n, BH);
+bool tc_make_map(CUtensorMap *m, const void *base, int width, int n, int BH, int hs_mul) {
+    return make_map_impl(m, base, width, n, BH, 128, hs_mul);
 }
-bool tc_make_map_rows(CUtensorMap *m, const void *base, int width, int n, int BH, int rows) {
-    return make_map_impl(m, base, width, n, BH, rows);
+bool tc_make_map_rows(CUtensorMap *m, const void *base, int width, int n, int BH, int rows, int hs_mul) {
+    return make_map_impl(m, base, width, n, BH, rows, hs_mul);
 }
 int tc_sm_count() { return sm_count_impl(); }
 AttnArgs tc_work_items(const AttnArgs &a) { return tc_items_impl(a); }

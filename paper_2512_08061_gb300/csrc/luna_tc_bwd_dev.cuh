@@ -88,16 +88,18 @@ __device__ __forceinline__ void search(const float *sTe, const float (&u)[PP], i
     for (int q = 0; q < PP; ++q) j[q] = node[q] - kEytzinger;
 }
 
-// alpha, beta of the 8 channels on interval j (swizzled table) and phi = relu(alpha u + beta).
-__device__ __forceinline__ void channel_eval(const float *sAB, int j, float u, float (&al)[8], float (&y)[8]) {
+// alpha, beta of the 8 channels on interval j (swizzled table) and phi = max(alpha u + beta, fl): the
+// outer ReLU (fl = 0) or the signed output (fl = -inf).
+__device__ __forceinline__ void channel_eval(const float *sAB, int j, float u, float fl, float (&al)[8],
+                                             float (&y)[8]) {
     const float4 *ab = reinterpret_cast<const float4 *>(sAB);
 #pragma unroll
     for (int k = 0; k < 4; ++k) {
         const float4 v = ab[ab_slot(j, k)];
         al[2 * k] = v.x;
         al[2 * k + 1] = v.z;
-        y[2 * k] = fmaxf(fmaf(v.x, u, v.y), 0.0f);
-        y[2 * k + 1] = fmaxf(fmaf(v.z, u, v.w), 0.0f);
+        y[2 * k] = fmaxf(fmaf(v.x, u, v.y), fl);
+        y[2 * k + 1] = fmaxf(fmaf(v.z, u, v.w), fl);
     }
 }
 

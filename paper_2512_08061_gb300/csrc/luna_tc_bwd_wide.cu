@@ -56,6 +56,7 @@ __global__ void __launch_bounds__(kBThreads, 1)
     k_tc_bwd_query_w(const __grid_constant__ CUtensorMap mapQ, const __grid_constant__ CUtensorMap mapdO, AttnArgs a,
                      int *status) {
     extern __shared__ uint8_t smem_raw[];
+    const float fl = channel_floor(a.lay);  // lower bound of a channel output
     uint8_t *sm = align1024(smem_raw);
     constexpr int NS = C::NSQ, NO = C::NOQ;
     constexpr uint32_t T16 = C::TILE;
@@ -119,7 +120,7 @@ __global__ void __launch_bounds__(kBThreads, 1)
     for (int e = tid; e < a.lay.nint * 16; e += blockDim.x) hpart[e] = 0.0f;
     for (int item = it.begin; item < it.end && !a.padded_zeroed; ++item) {  // padded rows: zero gradients
         const ItemRange ir = item_range(a, it, item);
-        __nv_bfloat16 *dQ = static_cast<__nv_bfloat16 *>(a.dQ) + (size_t)ir.bh * a.n * C::d;
+        __nv_bfloat16 *dQ = static_cast<__nv_bfloat16 *>(a.dQ) + head_rows(a, ir.bh) * C::d;
         const int z0 = max(ir.r0, ir.r1);
         for (int e = tid; e < (ir.rend - z0) * C::d / 8; e += blockDim.x)
             reinterpret_cast<uint4 *>(dQ + (size_t)z0 * C::d)[e] = make_uint4(0, 0, 0, 0);
@@ -275,8 +276,8 @@ __global__ void __launch_bounds__(kBThreads, 1)
             for (int i = i0; i < i1; ++i) run_tiles += item_range(a, it, i).ntiles;
             if (run_tiles > 0) {  // operands of this head: [S_hi; S_lo] rows per feature, z
                 named_sync<kBWorkers>(1);
-                stage_rows_per_feature<C>(a.S_fin + (size_t)bh * C::D * C::DV, Sop2, tid, kBWorkers);
-                for (int e = tid; e < C::D; e += kBWorkers) sz[e] = a.z_fin[(size_t)bh * C::D + e];
+                stage_rows_per_feature<C>(a.S_fin + head_state(a, bh) * C::D * C::DV, Sop2, tid, kBWorkers);
+                for (int e = tid; e < C::D; e += kBWorkers) sz[e] = a.z_fin[head_state(a, bh) * C::D + e];
                 fence_proxy_async_smem();
                 named_sync<kBWorkers>(1);
                 mbar_arrive(opready);
@@ -316,7 +317,7 @@ __global__ void __launch_bounds__(kBThreads, 1)
                     for (int q = 0; q < C::PP; ++q) {
                         const int i = H * C::PP + q;
                         float al[8], y[8];
-                        channel_eval(sAB, j[q], u[q], al, y);
+                        channel_eval(sAB, j[q], u[q], fl, al, y);
                         uint32_t ph[8], pl[8];
                         tmem_ld8(tbase + lrow + cP + 8 * i, ph);
                         tmem_ld8(tbase + lrow + cP + C::D + 8 * i, pl);
@@ -348,7 +349,7 @@ __global__ void __launch_bounds__(kBThreads, 1)
                     for (int q = 0; q < C::PP; ++q) {
                         const int i = H * C::PP + q;
                         float al[8], y[8];
-                        channel_eval(sAB, j[q], u[q], al, y);
+                        channel_eval(sAB, j[q], u[q], fl, al, y);
                         {
                             float yh[8], yl[8];
 #pragma unroll
@@ -370,7 +371,7 @@ __global__ void __launch_bounds__(kBThreads, 1)
                         for (int l = 0; l < 8; ++l) {
                             const float dphi =
                                 live ? (__uint_as_float(ph[l]) + __uint_as_float(pl[l])) * inv + sz[8 * i + l] * dden : 0.0f;
-                            const float gl = y[l] > 0.0f ? dphi : 0.0f;
+                            const float gl = y[l] > fl ? dphi : 0.0f;
                             gv[q][l] = gl;
                             du = fmaf(gl, al[l], du);
                         }
@@ -416,7 +417,7 @@ __global__ void __launch_bounds__(kBThreads, 1)
                         if (++hacc.tiles == hist_tiles<C::MP>()) hist_close(bins, hpart, a.lay.nint, hacc, tid, true, smax, warp, lane);
                     }
                     pend_g = g;
-                    pend_row = valid ? bh * a.n + row0 + r : -1;
+                    pend_row = valid ? (int)head_rows(a, bh) + row0 + r : -1;
                 }
             }
             // run epilogue (warps 0..3): dS, dz partial of this head; warp w holds features 16w..16w+15,
@@ -514,6 +515,7 @@ __global__ void __launch_bounds__(kBThreads, 1)
     k_tc_bwd_key_w(const __grid_constant__ CUtensorMap mapK, const __grid_constant__ CUtensorMap mapV, AttnArgs a,
                    int *status) {
     extern __shared__ uint8_t smem_raw[];
+    const float fl = channel_floor(a.lay);  // lower bound of a channel output
     uint8_t *sm = align1024(smem_raw);
     constexpr int NS = C::NSK;
     constexpr uint32_t T16 = C::TILE;
@@ -577,8 +579,8 @@ __global__ void __launch_bounds__(kBThreads, 1)
     for (int e = tid; e < a.lay.nint * 16; e += blockDim.x) hpart[e] = 0.0f;
     for (int item = it.begin; item < it.end && !a.padded_zeroed; ++item) {  // padded rows: zero gradients
         const ItemRange ir = item_range(a, it, item);
-        __nv_bfloat16 *dK = static_cast<__nv_bfloat16 *>(a.dK) + (size_t)ir.bh * a.n * C::d;
-        __nv_bfloat16 *dV = static_cast<__nv_bfloat16 *>(a.dV) + (size_t)ir.bh * a.n * C::DV;
+        __nv_bfloat16 *dK = static_cast<__nv_bfloat16 *>(a.dK) + head_rows(a, ir.bh) * C::d;
+        __nv_bfloat16 *dV = static_cast<__nv_bfloat16 *>(a.dV) + head_rows(a, ir.bh) * C::DV;
         const int z0 = max(ir.r0, ir.r1);
         for (int e = tid; e < (ir.rend - z0) * C::d / 8; e += blockDim.x)
             reinterpret_cast<uint4 *>(dK + (size_t)z0 * C::d)[e] = make_uint4(0, 0, 0, 0);
@@ -707,8 +709,8 @@ __global__ void __launch_bounds__(kBThreads, 1)
                 named_sync<kBWorkers>(1);
                 mbar_arrive(opready);
             }
-            __nv_bfloat16 *dK = static_cast<__nv_bfloat16 *>(a.dK) + (size_t)bh * a.n * C::d;
-            __nv_bfloat16 *dV = static_cast<__nv_bfloat16 *>(a.dV) + (size_t)bh * a.n * C::DV;
+            __nv_bfloat16 *dK = static_cast<__nv_bfloat16 *>(a.dK) + head_rows(a, bh) * C::d;
+            __nv_bfloat16 *dV = static_cast<__nv_bfloat16 *>(a.dV) + head_rows(a, bh) * C::DV;
             for (int item = i0; item < i1; ++item) {
                 const ItemRange ir = item_range(a, it, item);
                 for (int t = 0; t < ir.ntiles; ++t, ++g) {
@@ -738,7 +740,7 @@ __global__ void __launch_bounds__(kBThreads, 1)
 #pragma unroll
                     for (int q = 0; q < C::PP; ++q) {
                         float al[8], y[8];
-                        channel_eval(sAB, j[q], u[q], al, y);
+                        channel_eval(sAB, j[q], u[q], fl, al, y);
                         *reinterpret_cast<uint4 *>(phit + sw128_chunk(r, H * C::PP + q)) =
                             valid ? pack8(y) : make_uint4(0, 0, 0, 0);
                     }
@@ -755,7 +757,7 @@ __global__ void __launch_bounds__(kBThreads, 1)
                     for (int q = 0; q < C::PP; ++q) {
                         const int i = H * C::PP + q;
                         float al[8], y[8];
-                        channel_eval(sAB, j[q], u[q], al, y);
+                        channel_eval(sAB, j[q], u[q], fl, al, y);
                         uint32_t ph[8], pl[8];
                         tmem_ld8(tbase + lrow + cF + 8 * i, ph);
                         tmem_ld8(tbase + lrow + cF + C::D + 8 * i, pl);
@@ -764,7 +766,7 @@ __global__ void __launch_bounds__(kBThreads, 1)
 #pragma unroll
                         for (int l = 0; l < 8; ++l) {
                             const float dphi = __uint_as_float(ph[l]) + __uint_as_float(pl[l]) + sdz[8 * i + l];
-                            const float gl = (valid && y[l] > 0.0f) ? dphi : 0.0f;
+                            const float gl = (valid && y[l] > fl) ? dphi : 0.0f;
                             gv[q][l] = gl;
                             du = fmaf(gl, al[l], du);
                         }
@@ -872,7 +874,7 @@ __global__ void __launch_bounds__(kBThreads, 1)
 
 }  // namespace
 
-bool tc_make_map(CUtensorMap *m, const void *base, int width, int n, int BH);
+bool tc_make_map(CUtensorMap *m, const void *base, int width, int n, int BH, int hs_mul);
 
 cudaError_t launch_tc_bwd_wide(const AttnArgs &a0, bool have_stats, cudaStream_t s) {
     using C = B64;
@@ -882,8 +884,9 @@ cudaError_t launch_tc_bwd_wide(const AttnArgs &a0, bool have_stats, cudaStream_t
     const int grid = tc_grid(a);
     if (!have_stats && (e = launch_tc_stats(a, s)) != cudaSuccess) return e;
     CUtensorMap mQ, mdO, mK, mV;
-    if (!tc_make_map(&mQ, a.Q, a.d, a.n, a.B * a.H) || !tc_make_map(&mdO, a.dO, a.dv, a.n, a.B * a.H) ||
-        !tc_make_map(&mK, a.K, a.d, a.n, a.B * a.H) || !tc_make_map(&mV, a.V, a.dv, a.n, a.B * a.H))
+    if (!tc_make_map(&mQ, a.Q, a.d, a.n, a.B * a.H, a.hs_mul) ||
+        !tc_make_map(&mdO, a.dO, a.dv, a.n, a.B * a.H, a.hs_mul) ||
+        !tc_make_map(&mK, a.K, a.d, a.n, a.B * a.H, a.hs_mul) || !tc_make_map(&mV, a.V, a.dv, a.n, a.B * a.H, a.hs_mul))
         return cudaErrorInvalidValue;
     if ((e = cudaFuncSetAttribute(k_tc_bwd_query_w<C>, cudaFuncAttributeMaxDynamicSharedMemorySize, C::SMEM_Q)) !=
         cudaSuccess)

@@ -63,8 +63,8 @@ __host__ __device__ constexpr uint32_t col_uq(int g) { return (g & 1) ? cUq1 : c
 // sz, the normaliser part that the numerator's rounding matches.
 template <class C>
 __device__ __forceinline__ float phi_quarter_qk(uint32_t uq, uint32_t uk, int Qd, const float *sTe, const float *sAB,
-                                                const float *sbias, bool valid, int r, uint8_t *tq, uint8_t *tk,
-                                                const float *sz) {
+                                                const float *sbias, float fl, bool valid, int r, uint8_t *tq,
+                                                uint8_t *tk, const float *sz) {
     constexpr int PP = C::PP;
     static_assert(PP == 4, "four projections per thread");
     float u[2 * PP];
@@ -100,8 +100,8 @@ __device__ __forceinline__ float phi_quarter_qk(uint32_t uq, uint32_t uk, int Qd
 #pragma unroll
             for (int k = 0; k < 4; ++k) {
                 const float4 v = ab[ab_slot(j, k)];
-                y[2 * k] = fmaxf(fmaf(v.x, u[q], v.y), 0.0f);
-                y[2 * k + 1] = fmaxf(fmaf(v.z, u[q], v.w), 0.0f);
+                y[2 * k] = fmaxf(fmaf(v.x, u[q], v.y), fl);
+                y[2 * k + 1] = fmaxf(fmaf(v.z, u[q], v.w), fl);
             }
             w = make_uint4(pack_bf16x2(y[0], y[1]), pack_bf16x2(y[2], y[3]), pack_bf16x2(y[4], y[5]),
                            pack_bf16x2(y[6], y[7]));
@@ -173,7 +173,7 @@ __global__ void __launch_bounds__(kCThreads, 1)
     // padded rows of every item get O = 0
     for (int item = it.begin; item < it.end; ++item) {
         const ItemRange ir = item_range(a, it, item);
-        __nv_bfloat16 *O = static_cast<__nv_bfloat16 *>(a.O) + (size_t)ir.bh * a.n * C::DV;
+        __nv_bfloat16 *O = static_cast<__nv_bfloat16 *>(a.O) + head_rows(a, ir.bh) * C::DV;
         const int z0 = max(ir.r0, ir.r1);
         for (int e = tid; e < (ir.rend - z0) * C::DV / 8; e += blockDim.x)
             reinterpret_cast<uint4 *>(O + (size_t)z0 * C::DV)[e] = make_uint4(0, 0, 0, 0);
@@ -301,7 +301,7 @@ __global__ void __launch_bounds__(kCThreads, 1)
             if (ir.ntiles == 0) continue;
             // segment start: S (TMEM, fp32) and its bf16 operand from the prefix state, z from the prefix sums
             {
-                const float *Sp = a.seg_S + ((size_t)ir.bh * (a.nseg + 1) + ir.chunk) * C::D * C::DV;
+                const float *Sp = a.seg_S + (head_state(a, ir.bh) * (a.nseg + 1) + ir.chunk) * C::D * C::DV;
                 const int f = r, c0 = 32 * Qd;  // TMEM lane f (feature), columns c0 .. c0+31
                 float v[32];
 #pragma unroll
@@ -317,7 +317,7 @@ __global__ void __launch_bounds__(kCThreads, 1)
                 tmem_wait_st();
                 store_row32<C>(Sop, f, c0, v);
                 if (Qd == 0) {
-                    const float zv = __ldcg(a.seg_z + ((size_t)ir.bh * (a.nseg + 1) + ir.chunk) * C::D + f);
+                    const float zv = __ldcg(a.seg_z + (head_state(a, ir.bh) * (a.nseg + 1) + ir.chunk) * C::D + f);
                     zpre[f] = zv;
                     sz[f] = zv;
                 }
@@ -326,7 +326,7 @@ __global__ void __launch_bounds__(kCThreads, 1)
                 mbar_arrive(sready);
                 named_sync<kCWorkers>(1);  // sz of the segment start
             }
-            __nv_bfloat16 *O = static_cast<__nv_bfloat16 *>(a.O) + (size_t)ir.bh * a.n * C::DV;
+            __nv_bfloat16 *O = static_cast<__nv_bfloat16 *>(a.O) + head_rows(a, ir.bh) * C::DV;
             for (int t = 0; t < ir.ntiles; ++t, ++g) {
                 const int row0 = ir.r0 + t * 128;
                 const int nvalid = min(128, ir.r1 - row0);
@@ -336,7 +336,7 @@ __global__ void __launch_bounds__(kCThreads, 1)
                 wait_or_fail(uready, g & 1, failed, status);
                 tc_fence_after();
                 const float dq = phi_quarter_qk<C>(tbase + lrow + col_uq(g), tbase + lrow + cU + C::NU, Qd, sTe, sAB,
-                                                   sbias, valid, r, Pq, Pk, sz);
+                                                   sbias, channel_floor(a.lay), valid, r, Pq, Pk, sz);
                 tc_fence_before();
                 mbar_arrive(ufree);
                 if (!valid && Qd == 0) {  // padded key rows: clear V so that no garbage enters num or S
@@ -439,7 +439,7 @@ __global__ void __launch_bounds__(256) k_seg_scan(AttnArgs a) {
     const int e4 = blockIdx.x * blockDim.x + threadIdx.x;  // float4 position
     if ((size_t)e4 * 4 < SD) {
         const float4 *part = reinterpret_cast<const float4 *>(a.S_part + (size_t)bh * a.nseg * SD) + e4;
-        float4 *out = reinterpret_cast<float4 *>(a.seg_S + (size_t)bh * (a.nseg + 1) * SD) + e4;
+        float4 *out = reinterpret_cast<float4 *>(a.seg_S + head_state(a, bh) * (a.nseg + 1) * SD) + e4;
         float4 acc = make_float4(0.f, 0.f, 0.f, 0.f);
         for (int s = 0; s < a.nseg; ++s) {
             const float4 v = __ldcg(part + (size_t)s * (SD / 4));
@@ -451,7 +451,7 @@ __global__ void __launch_bounds__(256) k_seg_scan(AttnArgs a) {
     if (blockIdx.x == 0) {
         for (int f = threadIdx.x; f < a.D; f += blockDim.x) {
             const float *part = a.z_part + (size_t)bh * a.nseg * a.D + f;
-            float *out = a.seg_z + (size_t)bh * (a.nseg + 1) * a.D + f;
+            float *out = a.seg_z + head_state(a, bh) * (a.nseg + 1) * a.D + f;
             float acc = 0.0f;
             for (int s = 0; s < a.nseg; ++s) {
                 const float v = __ldcg(part + (size_t)s * a.D);
@@ -465,7 +465,7 @@ __global__ void __launch_bounds__(256) k_seg_scan(AttnArgs a) {
 
 }  // namespace
 
-bool tc_make_map(CUtensorMap *m, const void *base, int width, int n, int BH);
+bool tc_make_map(CUtensorMap *m, const void *base, int width, int n, int BH, int hs_mul);
 int tc_sm_count();
 
 bool tc_causal_supported(const luna_attn_desc &ad, const TableLayout &lay) {
@@ -492,8 +492,8 @@ cudaError_t launch_tc_causal_fwd(const AttnArgs &a0, cudaStream_t s) {
     if (e != cudaSuccess) return e;
     const int BH = a.B * a.H;
     CUtensorMap mQ, mK, mV;
-    if (!tc_make_map(&mQ, a.Q, a.d, a.n, BH) || !tc_make_map(&mK, a.K, a.d, a.n, BH) ||
-        !tc_make_map(&mV, a.V, a.dv, a.n, BH))
+    if (!tc_make_map(&mQ, a.Q, a.d, a.n, BH, a.hs_mul) || !tc_make_map(&mK, a.K, a.d, a.n, BH, a.hs_mul) ||
+        !tc_make_map(&mV, a.V, a.dv, a.n, BH, a.hs_mul))
         return cudaErrorInvalidValue;
     if ((e = cudaFuncSetAttribute(k_tc_causal<C>, cudaFuncAttributeMaxDynamicSharedMemorySize, C::SMEM)) != cudaSuccess)
         return e;

@@ -361,7 +361,7 @@ __global__ void __launch_bounds__(kCBThreads, 1)
             if (nt == 0) continue;
             // segment start: S (TMEM fp32 and the bf16 hi/lo operand) and z from the prefix state
             {
-                const float *Sp = a.seg_S + ((size_t)ir.bh * (a.nseg + 1) + ir.chunk) * C::D * C::DV;
+                const float *Sp = a.seg_S + (head_state(a, ir.bh) * (a.nseg + 1) + ir.chunk) * C::D * C::DV;
                 const int f = 32 * q + lane, c0 = 32 * cg;
                 float v[32];
 #pragma unroll
@@ -377,7 +377,7 @@ __global__ void __launch_bounds__(kCBThreads, 1)
                 tmem_wait_st();
                 store_state32(Sh, Sl, f, c0, v);
                 if (cg == 0) {
-                    const float zv = __ldcg(a.seg_z + ((size_t)ir.bh * (a.nseg + 1) + ir.chunk) * C::D + f);
+                    const float zv = __ldcg(a.seg_z + (head_state(a, ir.bh) * (a.nseg + 1) + ir.chunk) * C::D + f);
                     zpre[f] = zv;
                     sz[f] = zv;
                 }
@@ -386,7 +386,7 @@ __global__ void __launch_bounds__(kCBThreads, 1)
                 mbar_arrive(sopready);
                 named_sync<kCBWorkers>(1);
             }
-            const size_t hrow = (size_t)ir.bh * a.n;
+            const size_t hrow = (size_t)ir.bh * a.n;  // workspace rows (staged rows, row statistics)
             for (int t = 0; t < nt; ++t, ++g) {
                 const int row0 = ir.r0 + 64 * t;
                 const int nvalid = min(64, ir.r1 - row0);
@@ -418,6 +418,7 @@ __global__ void __launch_bounds__(kCBThreads, 1)
 #pragma unroll
                         for (int p = 0; p < 4; ++p) node[p] = 2 * node[p] + (sTe[node[p]] < u[p] ? 1 : 0);
                     const float4 *ab = reinterpret_cast<const float4 *>(sAB);
+                    const float fl = channel_floor(a.lay);
                     float yk[16];
 #pragma unroll
                     for (int p = 0; p < 4; ++p) {
@@ -425,8 +426,8 @@ __global__ void __launch_bounds__(kCBThreads, 1)
 #pragma unroll
                         for (int k = 0; k < 4; ++k) {
                             const float4 w = ab[ab_slot(jv, k)];
-                            const float y0 = valid ? fmaxf(fmaf(w.x, u[p], w.y), 0.0f) : 0.0f;
-                            const float y1 = valid ? fmaxf(fmaf(w.z, u[p], w.w), 0.0f) : 0.0f;
+                            const float y0 = valid ? fmaxf(fmaf(w.x, u[p], w.y), fl) : 0.0f;
+                            const float y1 = valid ? fmaxf(fmaf(w.z, u[p], w.w), fl) : 0.0f;
                             if (p < 2) { phq[8 * p + 2 * k] = y0; phq[8 * p + 2 * k + 1] = y1; }
                             else { yk[8 * (p - 2) + 2 * k] = y0; yk[8 * (p - 2) + 2 * k + 1] = y1; }
                         }
@@ -808,7 +809,7 @@ __global__ void __launch_bounds__(kCBThreads, 1)
     // rows beyond the sequence length receive zero dV
     for (int item = it.begin; item < it.end; ++item) {
         const ItemRange ir = item_range(a, it, item);
-        __nv_bfloat16 *dV = static_cast<__nv_bfloat16 *>(a.dV) + (size_t)ir.bh * a.n * C::DV;
+        __nv_bfloat16 *dV = static_cast<__nv_bfloat16 *>(a.dV) + head_rows(a, ir.bh) * C::DV;
         const int z0 = max(ir.r0, ir.r1);
         for (int e = tid; e < (ir.rend - z0) * C::DV / 8; e += blockDim.x)
             reinterpret_cast<uint4 *>(dV + (size_t)z0 * C::DV)[e] = make_uint4(0, 0, 0, 0);
@@ -973,7 +974,8 @@ __global__ void __launch_bounds__(kCBThreads, 1)
                 mbar_arrive(sopready);
                 named_sync<kCBWorkers>(1);
             }
-            const size_t hrow = (size_t)ir.bh * a.n;
+            const size_t hrow = (size_t)ir.bh * a.n;  // workspace rows (staged rows, row statistics)
+            const size_t urow = head_rows(a, ir.bh);  // the caller's rows (dV)
             for (int tr = 0; tr < nt; ++tr, ++g) {
                 const int t = nt - 1 - tr;
                 const int row0 = ir.r0 + 64 * t;
@@ -1039,7 +1041,7 @@ __global__ void __launch_bounds__(kCBThreads, 1)
                     half_cols<16>(x, dv, lane);
                     if (valid) {
                         uint4 *dst = reinterpret_cast<uint4 *>(static_cast<__nv_bfloat16 *>(a.dV) +
-                                                               (hrow + row0 + r) * C::DV + 16 * part);
+                                                               (urow + row0 + r) * C::DV + 16 * part);
                         dst[0] = pack8f(dv);
                         dst[1] = pack8f(dv + 8);
                     }
@@ -1093,7 +1095,7 @@ __global__ void __launch_bounds__(kCBThreads, 1)
 
 }  // namespace
 
-bool tc_make_map_rows(CUtensorMap *m, const void *base, int width, int n, int BH, int rows);
+bool tc_make_map_rows(CUtensorMap *m, const void *base, int width, int n, int BH, int rows, int hs_mul);
 int tc_sm_count();
 cudaError_t launch_tc_causal_stats(const AttnArgs &a, cudaStream_t s);
 cudaError_t launch_tc_phi_bwd(const AttnArgs &a, const void *X, const float *dphi, void *dX, int slot0, int grid,
@@ -1111,11 +1113,13 @@ cudaError_t launch_tc_causal_bwd(const AttnArgs &a0, bool have_state, cudaStream
     const int grid = items < tc_sm_count() ? items : tc_sm_count();
     int *st = reinterpret_cast<int *>(reinterpret_cast<char *>(a.counters) - 256);
     CUtensorMap mQ, mK, mV, mdO, mPk, mPq, mPq128, mdO128;
-    if (!tc_make_map_rows(&mQ, a.Q, a.d, a.n, BH, 64) || !tc_make_map_rows(&mK, a.K, a.d, a.n, BH, 64) ||
-        !tc_make_map_rows(&mV, a.V, a.dv, a.n, BH, 64) || !tc_make_map_rows(&mdO, a.dO, a.dv, a.n, BH, 64) ||
-        !tc_make_map_rows(&mPk, a.phik, 2 * C::D, a.n, BH, 64) || !tc_make_map_rows(&mPq, a.pq2, 2 * C::D, a.n, BH, 64) ||
-        !tc_make_map_rows(&mPq128, a.pq2, 2 * C::D, a.n, BH, 128) ||
-        !tc_make_map_rows(&mdO128, a.dO, a.dv, a.n, BH, 128))
+    const int hm = a.hs_mul;  // the caller's tensors; the staged rows (phi(k), phi(q)/den) are the workspace's
+    if (!tc_make_map_rows(&mQ, a.Q, a.d, a.n, BH, 64, hm) || !tc_make_map_rows(&mK, a.K, a.d, a.n, BH, 64, hm) ||
+        !tc_make_map_rows(&mV, a.V, a.dv, a.n, BH, 64, hm) || !tc_make_map_rows(&mdO, a.dO, a.dv, a.n, BH, 64, hm) ||
+        !tc_make_map_rows(&mPk, a.phik, 2 * C::D, a.n, BH, 64, 1) ||
+        !tc_make_map_rows(&mPq, a.pq2, 2 * C::D, a.n, BH, 64, 1) ||
+        !tc_make_map_rows(&mPq128, a.pq2, 2 * C::D, a.n, BH, 128, 1) ||
+        !tc_make_map_rows(&mdO128, a.dO, a.dv, a.n, BH, 128, hm))
         return cudaErrorInvalidValue;
     // 1. query side
     if ((e = cudaFuncSetAttribute(k_tcc_query<C>, cudaFuncAttributeMaxDynamicSharedMemorySize, C::SMEM_Q)) != cudaSuccess)

@@ -54,6 +54,7 @@ __global__ void __launch_bounds__(kBThreads, 1)
     k_tc_phi_bwd(const __grid_constant__ CUtensorMap mapX, AttnArgs a, const float *dphi, __nv_bfloat16 *dXg,
                  int slot0, int *status) {
     extern __shared__ uint8_t smem_raw[];
+    const float fl = channel_floor(a.lay);  // lower bound of a channel output
     uint8_t *sm = align1024(smem_raw);
     constexpr int NS = C::NS;
     constexpr uint32_t T16 = C::TILE;
@@ -104,7 +105,7 @@ __global__ void __launch_bounds__(kBThreads, 1)
     for (int e = tid; e < a.lay.nint * 16; e += blockDim.x) hpart[e] = 0.0f;
     for (int item = it.begin; item < it.end; ++item) {  // padded rows receive zero gradients
         const ItemRange ir = item_range(a, it, item);
-        __nv_bfloat16 *dX = dXg + (size_t)ir.bh * a.n * C::d;
+        __nv_bfloat16 *dX = dXg + head_rows(a, ir.bh) * C::d;
         const int z0 = max(ir.r0, ir.r1);
         for (int e = tid; e < (ir.rend - z0) * C::d / 8; e += blockDim.x)
             reinterpret_cast<uint4 *>(dX + (size_t)z0 * C::d)[e] = make_uint4(0, 0, 0, 0);
@@ -187,7 +188,7 @@ __global__ void __launch_bounds__(kBThreads, 1)
         int g = 0;
         for (int item = it.begin; item < it.end; ++item) {
             const ItemRange ir = item_range(a, it, item);
-            __nv_bfloat16 *dX = dXg + (size_t)ir.bh * a.n * C::d;
+            __nv_bfloat16 *dX = dXg + head_rows(a, ir.bh) * C::d;
             for (int t = 0; t < ir.ntiles; ++t, ++g) {
                 const int row0 = ir.r0 + t * 128;
                 const bool valid = r < min(128, ir.r1 - row0);
@@ -222,13 +223,13 @@ __global__ void __launch_bounds__(kBThreads, 1)
 #pragma unroll
                 for (int q = 0; q < C::PP; ++q) {
                     float al[8], y[8];
-                    channel_eval(sAB, j[q], u[q], al, y);
+                    channel_eval(sAB, j[q], u[q], fl, al, y);
                     const float4 p0 = pv[q][0], p1 = pv[q][1];
                     const float dv[8] = {p0.x, p0.y, p0.z, p0.w, p1.x, p1.y, p1.z, p1.w};
                     float du = 0.0f;
 #pragma unroll
                     for (int l = 0; l < 8; ++l) {
-                        const float gl = (valid && y[l] > 0.0f) ? dv[l] : 0.0f;
+                        const float gl = (valid && y[l] > fl) ? dv[l] : 0.0f;
                         gv[q][l] = gl;
                         du = fmaf(gl, al[l], du);
                     }
@@ -321,7 +322,7 @@ __global__ void __launch_bounds__(kBThreads, 1)
 
 }  // namespace
 
-bool tc_make_map(CUtensorMap *m, const void *base, int width, int n, int BH);
+bool tc_make_map(CUtensorMap *m, const void *base, int width, int n, int BH, int hs_mul);
 int tc_sm_count();
 
 // Chain rule through the feature map for X in {Q, K}: dphi (fp32, [BH][n][D]) -> dX
@@ -331,7 +332,7 @@ cudaError_t launch_tc_phi_bwd(const AttnArgs &a, const void *X, const float *dph
                               cudaStream_t s) {
     using C = P128;
     CUtensorMap mX;
-    if (!tc_make_map(&mX, X, a.d, a.n, a.B * a.H)) return cudaErrorInvalidValue;
+    if (!tc_make_map(&mX, X, a.d, a.n, a.B * a.H, a.hs_mul)) return cudaErrorInvalidValue;
     cudaError_t e = cudaFuncSetAttribute(k_tc_phi_bwd<C>, cudaFuncAttributeMaxDynamicSharedMemorySize, C::SMEM);
     if (e != cudaSuccess) return e;
     int *st = reinterpret_cast<int *>(reinterpret_cast<char *>(a.counters) - 256);

@@ -33,7 +33,7 @@ class LunaError(RuntimeError):
 
 class PhiDesc(ctypes.Structure):
     _fields_ = [("M", ctypes.c_int), ("L", ctypes.c_int), ("hidden", ctypes.c_int), ("shared_channels", ctypes.c_int),
-                ("ch_rms_target", ctypes.c_float)]
+                ("ch_rms_target", ctypes.c_float), ("signed_outputs", ctypes.c_int)]
 
 
 class PhiParams(ctypes.Structure):
@@ -124,8 +124,9 @@ def _io_code(t: torch.Tensor) -> int:
     return _DTYPES[t.dtype]
 
 
-def phi_desc(M: int, L: int, hidden: int, shared: bool = False, ch_rms_target: float = 0.0) -> PhiDesc:
-    return PhiDesc(M, L, hidden, int(bool(shared)), float(ch_rms_target))
+def phi_desc(M: int, L: int, hidden: int, shared: bool = False, ch_rms_target: float = 0.0,
+             signed: bool = False) -> PhiDesc:
+    return PhiDesc(M, L, hidden, int(bool(shared)), float(ch_rms_target), int(bool(signed)))
 
 
 def attn_desc(B, H, n, d, dv, causal=False, chunk=0, eps=1e-6, io=LUNA_BF16) -> AttnDesc:
@@ -257,8 +258,8 @@ class Luna:
     """Owns the table, workspace and state buffers of one problem shape."""
 
     def __init__(self, B, H, n, d, dv, M, L, hidden=64, causal=False, eps=1e-6, io=torch.bfloat16, chunk=0,
-                 device="cuda", shared=False, ch_rms_target=0.0):
-        self.pd = phi_desc(M, L, hidden, shared, ch_rms_target)
+                 device="cuda", shared=False, ch_rms_target=0.0, signed=False):
+        self.pd = phi_desc(M, L, hidden, shared, ch_rms_target, signed)
         self.ad = attn_desc(B, H, n, d, dv, causal, chunk, eps, _DTYPES[io])
         self.d = d
         self.device = torch.device(device)

@@ -104,12 +104,14 @@ def to_host(x) -> np.ndarray:
 
 class Case:
     def __init__(self, B, H, n, d, M, L, io, causal=False, seed=0, qkv_scale=1.0, len_range=None, hidden=64,
-                 eps=1e-6, dv=None, with_grad=False, lengths=None, shared=False, ch_rms_target=0.0):
+                 eps=1e-6, dv=None, with_grad=False, lengths=None, shared=False, ch_rms_target=0.0, signed=False,
+                 params=None):
         self.B, self.H, self.n, self.d, self.M, self.L = B, H, n, d, M, L
         self.ch_rms_target = ch_rms_target
+        self.signed = signed
         self.dv = dv or d
         self.io, self.causal, self.eps, self.hidden, self.shared = io, causal, eps, hidden, shared
-        self.params = synth.phi_params(seed, d, M, L, hidden, shared)
+        self.params = params if params is not None else synth.phi_params(seed, d, M, L, hidden, shared)
         self.inp = synth.attn_inputs(seed, B, H, n, d, self.dv, io, qkv_scale, len_range, with_grad)
         if lengths is not None:
             self.inp["lengths"] = np.asarray(lengths, dtype=np.int32)
@@ -122,7 +124,7 @@ class Case:
         import paper_2512_08061_gb300.luna as L
         lu = L.Luna(self.B, self.H, self.n, self.d, self.dv, self.M, self.L, self.hidden, self.causal, self.eps,
                     torch.float32 if self.io == "f32" else torch.bfloat16, chunk, shared=self.shared,
-                    ch_rms_target=self.ch_rms_target)
+                    ch_rms_target=self.ch_rms_target, signed=self.signed)
         self.guards = []
         for name in ("table", "ws", "state"):
             setattr(lu, name, guarded_bytes(getattr(lu, name).numel(), lu.device, self.guards))
@@ -157,8 +159,11 @@ class Case:
     # ---- oracle side
     @property
     def phi(self):
-        """The oracle's feature map: the parameters, with the channel normalisation when it is on."""
-        return oracle.PhiParams(self.params, self.ch_rms_target) if self.ch_rms_target else self.params
+        """The oracle's feature map: the parameters, with the channel normalisation and the signed
+        channel outputs when they are on."""
+        if self.ch_rms_target or self.signed:
+            return oracle.PhiParams(self.params, self.ch_rms_target, nonneg=not self.signed)
+        return self.params
 
     def oracle_fwd(self):
         i = self.inp
@@ -173,4 +178,4 @@ class Case:
     def smooth_rows(self, which: str) -> np.ndarray:
         """Rows whose feature map has no ReLU argument within rounding distance of
         its kink: there the gradient is unique at fp32 resolution."""
-        return oracle.kink_margin(self.params, self.inp[which].value) > KINK_MARGIN
+        return oracle.kink_margin(self.phi, self.inp[which].value) > KINK_MARGIN

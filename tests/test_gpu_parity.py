@@ -599,3 +599,74 @@ def test_attention_weights_times_values_is_the_forward():
     L.luna_attn_weights(lu.ad, lu.pd, lu.table, case.dev["Q"], case.dev["K"], case.dev["lengths"], 0, 200, False, A)
     AV = to_host(A) @ case.inp["V"].value
     assert relerr(AV, O) < 1e-4
+
+
+# --------------------------------------------------------------------------
+# signed channel outputs (the listing's nonneg = False)
+
+def _signed_params(seed, d, M, L=8, hidden=64, shift=0.5):
+    """Random-init parameters with fc2's bias raised by `shift`: most channel outputs positive, some
+    negative, so the kernel's row sums stay away from zero while the signed path is exercised."""
+    p = synth.phi_params(seed, d, M, L, hidden)
+    p["b2"] = (p["b2"] + np.float32(shift)).astype(np.float32)
+    return p
+
+
+@pytest.mark.parametrize("io,d,M,causal,lengths", [("bf16", 32, 8, False, [300, 177]), ("bf16", 64, 8, False, None),
+                                                   ("bf16", 128, 16, True, [300, 250]), ("f32", 32, 8, False, [300, 9]),
+                                                   ("f32", 32, 8, True, None)])
+def test_signed_channel_outputs(io, d, M, causal, lengths):
+    """Signed channel outputs (no outer ReLU) through the tensor-core kernels
+    (bf16 non-causal d = 32 and 64, the streaming form at d = 128) and the
+    generic ones (fp32, causal and not), forward and backward, against the
+    oracle's nonneg = False; some features must be negative for the case to
+    mean anything."""
+    params = _signed_params(103, d, M)
+    case = Case(2, 2, 300, d, M, 8, io, causal, seed=103, qkv_scale=1.0 / math.sqrt(d), lengths=lengths,
+                with_grad=True, signed=True, params=params)
+    phiq = oracle.featmap(case.phi, case.inp["Q"].value)
+    assert 0.01 < np.mean(phiq < 0) < 0.5
+    lu = case.luna()
+    O = to_host(case.run_fwd(lu))
+    ref = case.oracle_fwd()
+    assert (relerr_rows(O, ref) if causal else relerr(O, ref)) < TOL[io]
+    g = {k: to_host(v) for k, v in case.run_bwd(lu).items()}
+    rb = case.oracle_bwd()
+    okq, okk = case.smooth_rows("Q"), case.smooth_rows("K")
+    assert okq.mean() > 0.9 and okk.mean() > 0.9
+    assert relerr(g["dQ"][okq], rb["dQ"][okq]) < TOL[io]
+    assert relerr(g["dK"][okk], rb["dK"][okk]) < TOL[io]
+    assert relerr(g["dV"], rb["dV"]) < TOL[io]
+    for k in ("dW", "db", "dw1", "db1", "dw2", "db2"):
+        assert relerr(g[k], rb[k]) < TOL[io], k
+
+
+def test_signed_channel_featmap_and_decode():
+    """luna_featmap and the decode step with signed channel outputs."""
+    import torch
+    import paper_2512_08061_gb300.luna as L
+    d, M = 64, 8
+    params = _signed_params(107, d, M)
+    X = synth.IOTensor(synth.normal(107, "sg.X", (777, d)), "f32")
+    pd = L.phi_desc(M, 8, 64, signed=True)
+    table = L.alloc_bytes(L.luna_phi_table_size(pd, d), "cuda")
+    L.luna_phi_prepare(pd, d, {k: torch.from_numpy(v).cuda() for k, v in params.items()}, table)
+    Phi = torch.empty(777, M * 8, dtype=torch.float32, device="cuda")
+    L.luna_featmap(pd, d, table, to_device(X), Phi)
+    ref = oracle.featmap(oracle.PhiParams(params, nonneg=False), X.value)
+    assert np.mean(ref < 0) > 0.01
+    assert relerr(to_host(Phi), ref) < 1e-4
+    # one decode step after a causal prefill of 40 tokens equals the causal output of token 41
+    n = 41
+    case = Case(2, 2, n, d, M, 8, "f32", True, seed=109, qkv_scale=1.0 / math.sqrt(d), signed=True, params=params)
+    full = case.oracle_fwd()
+    pre = Case(2, 2, n - 1, d, M, 8, "f32", True, seed=109, qkv_scale=1.0 / math.sqrt(d), signed=True,
+               params=params)
+    for k in ("Q", "K", "V"):
+        pre.inp[k] = synth.IOTensor(case.inp[k].value[:, :, :n - 1], "f32")
+    lu = pre.luna()
+    pre.run_fwd(lu, save_state=True)
+    tok = {k: torch.from_numpy(np.ascontiguousarray(case.inp[k].value[:, :, n - 1]).astype(np.float32)).cuda()
+           for k in ("Q", "K", "V")}
+    o = to_host(lu.decode(tok["Q"], tok["K"], tok["V"]))
+    assert relerr(o, full[:, :, n - 1]) < 1e-4
