@@ -82,6 +82,18 @@ typedef enum { LUNA_F32 = 0, LUNA_BF16 = 1 } luna_dtype;
  * table is the same for both (the flag is read from the descriptor by every
  * call, so pass the same descriptor to all calls of one problem); with
  * ch_rms_target > 0 it gives LUNA_ERR_UNSUPPORTED.
+ * param_head_stride = 0: one parameter set serves every head (the listing's
+ * "shared ... over tokens/heads").  > 0: per-head parameters, as in the
+ * conversion of a pretrained model, where the feature map's parameters are
+ * instantiated per layer and head (appendix, conversion of BERT and ViT):
+ * `table` holds ad->H tables, head h's at table + h * param_head_stride bytes
+ * (each prepared by luna_phi_prepare from head h's parameters; the stride is
+ * at least luna_phi_table_size and a multiple of 256), and luna_attn_bwd
+ * writes each head's parameter gradients, summed over the batch only, as
+ * arrays with a leading head axis (dW [H][M][d], ..., db2 [H][L]).  The
+ * attention calls then run one sub-problem per head index (the B sequences'
+ * head h at a time).  Not with ch_rms_target > 0 (LUNA_ERR_UNSUPPORTED); for
+ * luna_featmap pass head h's table with a stride of 0.
  * Supported: 1 <= M, 1 <= L <= 16, M*L <= 128, 1 <= hidden <= 128, L*hidden <= 512. */
 typedef struct {
     int M;               /* number of projections w_i (rows of W)       */
@@ -90,6 +102,7 @@ typedef struct {
     int shared_channels; /* 0 or 1, see above                           */
     float ch_rms_target; /* channel RMS normalisation target, 0 = off   */
     int signed_outputs;  /* 0 or 1, see above                           */
+    int64_t param_head_stride; /* bytes between heads' tables, 0 = shared  */
 } luna_phi_desc;
 
 /* Feature-map parameters, fp32 device arrays, row-major:

@@ -24,6 +24,12 @@ luna_status check_phi(const luna_phi_desc *pd, int d) {
     if (pd->signed_outputs != 0 && pd->signed_outputs != 1) return LUNA_ERR_INVALID_ARG;
     if (!(pd->ch_rms_target >= 0.0f) || isinf(pd->ch_rms_target)) return LUNA_ERR_INVALID_ARG;
     if (pd->signed_outputs && pd->ch_rms_target > 0.0f) return LUNA_ERR_UNSUPPORTED;
+    if (pd->param_head_stride < 0) return LUNA_ERR_INVALID_ARG;
+    if (pd->param_head_stride) {  // one table per head, each a whole 256-byte aligned table
+        const int64_t tb = table_layout(pd->M, pd->L, pd->hidden, d, pd->shared_channels).bytes;
+        if (pd->param_head_stride < tb || pd->param_head_stride % 256 != 0) return LUNA_ERR_INVALID_ARG;
+        if (pd->ch_rms_target > 0.0f) return LUNA_ERR_UNSUPPORTED;  // batch statistics of one shared map
+    }
     if (pd->L > kMaxL || pd->M * pd->L > kMaxFeat || pd->M > 32 || pd->hidden > kMaxHidden ||
         pd->L * pd->hidden > kMaxUnits || d > kMaxD || pd->M * d > 4096)
         return LUNA_ERR_UNSUPPORTED;
@@ -178,6 +184,7 @@ AttnArgs make_args(const luna_attn_desc *ad, const Plan &p, const void *table, c
     a.M = p.lay.M; a.L = p.lay.L; a.D = p.lay.D;
     a.eps = ad->eps;
     a.lay = p.lay;
+    a.hs_mul = 1;
     a.table = static_cast<const char *>(table);
     a.Q = Q; a.K = K; a.V = V;
     a.lengths = lengths;
@@ -225,6 +232,40 @@ void point_state(const luna_attn_desc *ad, const Plan &p, AttnArgs &a, void *sta
 
 luna_status cuda_status(cudaError_t e) { return e == cudaSuccess ? LUNA_OK : LUNA_ERR_CUDA; }
 
+// Per-head parameters: the sub-problem of head index h of every sequence.  Its B heads are the caller's
+// heads (b, h): the tensors start at head h and step H heads (hs_mul = H), the state and the gradients
+// start at head h's block, and the table is head h's.  Workspace buffers are indexed by the sub-problem's
+// own head numbers, so the sub-problems run one after another on the stream.
+AttnArgs head_args(const AttnArgs &a, const luna_attn_desc *ad, const luna_phi_desc *pd, const Plan &p, int h) {
+    AttnArgs s = a;
+    const size_t eb = ad->io == LUNA_F32 ? 4 : 2;
+    const size_t oq = (size_t)h * ad->n * ad->d * eb, ov = (size_t)h * ad->n * ad->dv * eb;
+    auto at = [](const void *x, size_t o) -> const void * {
+        return x ? static_cast<const void *>(static_cast<const char *>(x) + o) : nullptr;
+    };
+    auto atw = [](void *x, size_t o) -> void * { return x ? static_cast<void *>(static_cast<char *>(x) + o) : nullptr; };
+    s.Q = at(a.Q, oq); s.K = at(a.K, oq); s.V = at(a.V, ov); s.dO = at(a.dO, ov);
+    s.O = atw(a.O, ov); s.dQ = atw(a.dQ, oq); s.dK = atw(a.dK, oq); s.dV = atw(a.dV, ov);
+    s.H = 1;
+    s.hs_mul = ad->H;
+    s.table = a.table + (size_t)h * pd->param_head_stride;
+    const size_t D = p.lay.D, SD = D * ad->dv;
+    if (!ad->causal) {
+        s.S_fin = a.S_fin + (size_t)h * SD;
+        s.z_fin = a.z_fin + (size_t)h * D;
+    } else {
+        s.seg_S = a.seg_S + (size_t)h * (p.nseg + 1) * SD;
+        s.seg_z = a.seg_z + (size_t)h * (p.nseg + 1) * D;
+    }
+    const size_t Md = (size_t)pd->M * ad->d, fc1 = pd->shared_channels ? pd->hidden : (size_t)pd->L * pd->hidden;
+    if (s.grads.dW) {
+        s.grads.dW += h * Md; s.grads.db += (size_t)h * pd->M;
+        s.grads.dw1 += h * fc1; s.grads.db1 += h * fc1;
+        s.grads.dw2 += (size_t)h * pd->L * pd->hidden; s.grads.db2 += (size_t)h * pd->L;
+    }
+    return s;
+}
+
 bool aligned(const void *p, size_t a) { return (reinterpret_cast<uintptr_t>(p) % a) == 0; }
 
 }  // namespace
@@ -271,6 +312,7 @@ luna_status luna_featmap(const luna_phi_desc *pd, int d, const void *table, cons
     if (st != LUNA_OK) return st;
     if (rows < 0 || (xtype != LUNA_F32 && xtype != LUNA_BF16)) return LUNA_ERR_INVALID_ARG;
     if (pd->ch_rms_target > 0.0f) return LUNA_ERR_UNSUPPORTED;
+    if (pd->param_head_stride) return LUNA_ERR_UNSUPPORTED;  // rows carry no head: pass that head's table
     if (rows == 0) return LUNA_OK;
     if (!table || !X || !Phi) return LUNA_ERR_INVALID_ARG;
     TableLayout lay = table_layout(pd->M, pd->L, pd->hidden, d, pd->shared_channels, pd->signed_outputs);
@@ -318,13 +360,20 @@ luna_status luna_attn_fwd(const luna_attn_desc *ad, const luna_phi_desc *pd, con
     cudaError_t e = cudaMemsetAsync(workspace, 0, p.o_counters + 2 * sizeof(int) * (size_t)p.BH, s);
     if (e != cudaSuccess) return LUNA_ERR_CUDA;
     if (a.ch_sigma && (e = launch_chrms_stats(a, ad->io, s)) != cudaSuccess) return LUNA_ERR_CUDA;
-    if (ad->causal) {
-        if (p.tc.causal_fwd && tc_inputs_ok(TcPlan{true}, Q, K, V, O)) return cuda_status(launch_tc_causal_fwd(a, s));
-        return cuda_status(launch_causal_fwd(a, ad->io, state != nullptr, s));
+    const int nsub = pd->param_head_stride ? ad->H : 1;  // per-head parameters: one sub-problem per head index
+    for (int h = 0; h < nsub; ++h) {
+        const AttnArgs b = pd->param_head_stride ? head_args(a, ad, pd, p, h) : a;
+        if (ad->causal) {
+            if (p.tc.causal_fwd && tc_inputs_ok(TcPlan{true}, b.Q, b.K, b.V, b.O)) e = launch_tc_causal_fwd(b, s);
+            else e = launch_causal_fwd(b, ad->io, state != nullptr, s);
+        } else if (p.tc.eligible && tc_inputs_ok(p.tc, b.Q, b.K, b.V, b.O)) {
+            e = launch_tc_fwd(p.tc, b, static_cast<char *>(workspace), s);
+        } else {
+            e = launch_simt_fwd(b, ad->io, s);
+        }
+        if (e != cudaSuccess) return LUNA_ERR_CUDA;
     }
-    if (p.tc.eligible && tc_inputs_ok(p.tc, Q, K, V, O))
-        return cuda_status(launch_tc_fwd(p.tc, a, static_cast<char *>(workspace), s));
-    return cuda_status(launch_simt_fwd(a, ad->io, s));
+    return LUNA_OK;
 }
 
 luna_status luna_attn_bwd(const luna_attn_desc *ad, const luna_phi_desc *pd, const void *table, const void *Q,
@@ -338,14 +387,15 @@ luna_status luna_attn_bwd(const luna_attn_desc *ad, const luna_phi_desc *pd, con
         return LUNA_ERR_INVALID_ARG;
     cudaStream_t s = static_cast<cudaStream_t>(stream);
     if (p.BH == 0 || ad->n == 0) {  // empty problem: parameter gradients are zero
-        const size_t Md = (size_t)pd->M * ad->d, P = (size_t)pd->L * pd->hidden;
-        const size_t P1 = pd->shared_channels ? (size_t)pd->hidden : P;  // fc1 entries
+        const size_t G = pd->param_head_stride ? (size_t)ad->H : 1;  // parameter sets
+        const size_t Md = G * pd->M * ad->d, P = G * pd->L * pd->hidden;
+        const size_t P1 = pd->shared_channels ? G * pd->hidden : P;  // fc1 entries
         cudaError_t e = cudaMemsetAsync(grads->dW, 0, Md * 4, s);
-        if (e == cudaSuccess) e = cudaMemsetAsync(grads->db, 0, pd->M * 4, s);
+        if (e == cudaSuccess) e = cudaMemsetAsync(grads->db, 0, G * pd->M * 4, s);
         if (e == cudaSuccess) e = cudaMemsetAsync(grads->dw1, 0, P1 * 4, s);
         if (e == cudaSuccess) e = cudaMemsetAsync(grads->db1, 0, P1 * 4, s);
         if (e == cudaSuccess) e = cudaMemsetAsync(grads->dw2, 0, P * 4, s);
-        if (e == cudaSuccess) e = cudaMemsetAsync(grads->db2, 0, pd->L * 4, s);
+        if (e == cudaSuccess) e = cudaMemsetAsync(grads->db2, 0, G * pd->L * 4, s);
         return cuda_status(e);
     }
     if (!table || !Q || !K || !V || !dO || !dQ || !dK || !dV || !workspace) return LUNA_ERR_INVALID_ARG;
@@ -375,18 +425,29 @@ luna_status luna_attn_bwd(const luna_attn_desc *ad, const luna_phi_desc *pd, con
     cudaError_t e = cudaMemsetAsync(workspace, 0, p.o_counters + 2 * sizeof(int) * (size_t)p.BH, s);
     if (e != cudaSuccess) return LUNA_ERR_CUDA;
     if (a.ch_sigma && (e = launch_chrms_stats(a, ad->io, s)) != cudaSuccess) return LUNA_ERR_CUDA;
-    if (ad->causal) {
-        if (p.tc.causal_bwd && tc_inputs_ok(TcPlan{true}, Q, K, V, dO) && tc_inputs_ok(TcPlan{true}, dQ, dK, dV, nullptr)) {
-            a.dphi = reinterpret_cast<float *>(w + p.o_dphi);
-            a.phik = w + p.o_phik;
-            a.pq2 = w + p.o_pq2;
-            return cuda_status(launch_tc_causal_bwd(a, state != nullptr, s));
-        }
-        return cuda_status(launch_causal_bwd(a, ad->io, state != nullptr, s));
+    if (ad->causal && p.tc.causal_bwd) {
+        a.dphi = reinterpret_cast<float *>(w + p.o_dphi);
+        a.phik = w + p.o_phik;
+        a.pq2 = w + p.o_pq2;
     }
-    if (p.tc.eligible && tc_inputs_ok(p.tc, Q, K, V, dO) && tc_inputs_ok(p.tc, dQ, dK, dV, nullptr))
-        return cuda_status(launch_tc_bwd(p.tc, a, w, state != nullptr, s));
-    return cuda_status(launch_simt_bwd(a, ad->io, state != nullptr, s));
+    const int nsub = pd->param_head_stride ? ad->H : 1;  // per-head parameters: one sub-problem per head index
+    for (int h = 0; h < nsub; ++h) {
+        const AttnArgs b = pd->param_head_stride ? head_args(a, ad, pd, p, h) : a;
+        if (ad->causal) {
+            if (p.tc.causal_bwd && tc_inputs_ok(TcPlan{true}, b.Q, b.K, b.V, b.dO) &&
+                tc_inputs_ok(TcPlan{true}, b.dQ, b.dK, b.dV, nullptr))
+                e = launch_tc_causal_bwd(b, state != nullptr, s);
+            else
+                e = launch_causal_bwd(b, ad->io, state != nullptr, s);
+        } else if (p.tc.eligible && tc_inputs_ok(p.tc, b.Q, b.K, b.V, b.dO) &&
+                   tc_inputs_ok(p.tc, b.dQ, b.dK, b.dV, nullptr)) {
+            e = launch_tc_bwd(p.tc, b, w, state != nullptr, s);
+        } else {
+            e = launch_simt_bwd(b, ad->io, state != nullptr, s);
+        }
+        if (e != cudaSuccess) return LUNA_ERR_CUDA;
+    }
+    return LUNA_OK;
 }
 
 luna_status luna_attn_weights(const luna_attn_desc *ad, const luna_phi_desc *pd, const void *table, const void *Q,
@@ -416,7 +477,8 @@ luna_status luna_attn_weights(const luna_attn_desc *ad, const luna_phi_desc *pd,
     a.Q = Q; a.K = K;
     a.lengths = lengths;
     if (weights_max_smem(a) > kMaxSmem) return LUNA_ERR_UNSUPPORTED;
-    return cuda_status(launch_weights(a, ad->io, ad->causal, row0, rows, teacher, A, static_cast<cudaStream_t>(stream)));
+    return cuda_status(launch_weights(a, ad->io, ad->causal, row0, rows, teacher, pd->param_head_stride, A,
+                                      static_cast<cudaStream_t>(stream)));
 }
 
 luna_status luna_state_final(const luna_attn_desc *ad, const luna_phi_desc *pd, void *state, float **S,
@@ -462,6 +524,8 @@ luna_status luna_attn_decode(const luna_attn_desc *ad, const luna_phi_desc *pd, 
     a.eps = ad->eps;
     a.lay = lay;
     a.table = static_cast<const char *>(table);
+    a.H = ad->H;
+    a.table_stride = pd->param_head_stride;
     a.q = q; a.k = k; a.v = v; a.o = o;
     a.S = S; a.z = z;
     a.S_stride = S_stride; a.z_stride = z_stride;

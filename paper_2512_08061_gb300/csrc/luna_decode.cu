@@ -46,17 +46,18 @@ __global__ void __launch_bounds__(kDecThreads) k_decode(DecodeArgs a) {
     const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
     const int64_t bh = blockIdx.x;
     const int d = a.d, dv = a.dv, M = a.M, L = a.L, D = a.D;
+    const char *table = a.table + (size_t)(bh % a.H) * a.table_stride;  // this head's table
     for (int e = tid; e < d; e += blockDim.x) {
         sx[0][e] = ld_io(static_cast<const IO *>(a.q), bh * d + e);
         sx[1][e] = ld_io(static_cast<const IO *>(a.k), bh * d + e);
     }
     for (int e = tid; e < dv; e += blockDim.x) sv[e] = ld_io(static_cast<const IO *>(a.v), bh * dv + e);
-    const float4 *Te4 = reinterpret_cast<const float4 *>(a.table + a.lay.off_Te);
+    const float4 *Te4 = reinterpret_cast<const float4 *>(table + a.lay.off_Te);
     for (int e = tid; e < kEytzinger / 4; e += blockDim.x) reinterpret_cast<float4 *>(sTe)[e] = __ldg(Te4 + e);
     __syncthreads();
     // u = W x + b for x = q, k: one warp per dot product
-    const float *W = reinterpret_cast<const float *>(a.table + a.lay.off_W);
-    const float *bias = reinterpret_cast<const float *>(a.table + a.lay.off_b);
+    const float *W = reinterpret_cast<const float *>(table + a.lay.off_W);
+    const float *bias = reinterpret_cast<const float *>(table + a.lay.off_b);
     for (int p = warp; p < 2 * M; p += blockDim.x / 32) {
         const int side = p / M, m = p % M;
         float acc = 0.0f;
@@ -67,7 +68,7 @@ __global__ void __launch_bounds__(kDecThreads) k_decode(DecodeArgs a) {
     }
     __syncthreads();
     // phi: interval of u in the breadth-first kink tree, then relu(alpha u + beta) per channel
-    const float2 *AB = reinterpret_cast<const float2 *>(a.table + a.lay.off_AB);
+    const float2 *AB = reinterpret_cast<const float2 *>(table + a.lay.off_AB);
     const float fl = channel_floor(a.lay);
     for (int p = tid; p < 2 * M; p += blockDim.x) {
         const int side = p / M, m = p % M;

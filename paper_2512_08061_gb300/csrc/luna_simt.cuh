@@ -71,6 +71,8 @@ struct DecodeArgs {
     float eps;
     TableLayout lay;
     const char *table;
+    int H;                       // heads per sequence
+    int64_t table_stride;        // bytes between heads' tables (per-head parameters), 0: one shared table
     const void *q, *k, *v;
     void *o;
     float *S, *z;
@@ -90,8 +92,8 @@ cudaError_t launch_causal_fwd(const AttnArgs &a, luna_dtype io, bool write_state
 cudaError_t launch_causal_bwd(const AttnArgs &a, luna_dtype io, bool have_state, cudaStream_t s);
 size_t simt_max_smem(const AttnArgs &a);
 // attention weights of query rows [row0, row0 + rows) of every head (conversion, stage 1): A (BH, rows, n)
-cudaError_t launch_weights(const AttnArgs &a, luna_dtype io, int causal, int row0, int rows, int teacher, float *A,
-                           cudaStream_t s);
+cudaError_t launch_weights(const AttnArgs &a, luna_dtype io, int causal, int row0, int rows, int teacher,
+                           int64_t tstride, float *A, cudaStream_t s);
 size_t weights_max_smem(const AttnArgs &a);
 // channel RMS normalisation: statistics and scales of both sides; S, z rows times sigma (after any key
 // statistics); dS, dz rows times sigma and the per-head sums T (between the query- and key-side backward

@@ -29,7 +29,8 @@ constexpr int kWKeys = 32;  // key rows per tile
 constexpr int kWLanes = kThreads / kWRows;  // threads per query row (8): keys jj, jj + 8, ...
 
 template <typename IO>
-__global__ void __launch_bounds__(kThreads) k_weights(AttnArgs a, int causal, int row0, int rows, int teacher, float *A) {
+__global__ void __launch_bounds__(kThreads) k_weights(AttnArgs a, int causal, int row0, int rows, int teacher, int64_t tstride,
+                                                                float *A) {
     extern __shared__ __align__(16) float smem[];
     Carve cv{smem};
     const TableLayout &lay = a.lay;
@@ -52,7 +53,7 @@ __global__ void __launch_bounds__(kThreads) k_weights(AttnArgs a, int causal, in
     // rows past the valid length: zeros
     for (size_t e = (size_t)nq * n + threadIdx.x; e < (size_t)nr * n; e += blockDim.x) Ab[e] = 0.0f;
     if (nq == 0) return;
-    if (!teacher) load_phi(s, lay, a.table);
+    if (!teacher) load_phi(s, lay, a.table + (size_t)(bh % a.H) * tstride);  // this head's table
     load_rows(sQ, Qh + (size_t)i_lo * d, nq * d);
     __syncthreads();
     if (!teacher) phi_tile(lay, s, sQ, nq, sPq, nullptr, nullptr);
@@ -133,12 +134,13 @@ size_t smem_weights(const AttnArgs &a) {
 }
 
 template <typename IO>
-cudaError_t weights_impl(const AttnArgs &a, int causal, int row0, int rows, int teacher, float *A, cudaStream_t s) {
+cudaError_t weights_impl(const AttnArgs &a, int causal, int row0, int rows, int teacher, int64_t tstride, float *A,
+                         cudaStream_t s) {
     const size_t sm = smem_weights(a);
     cudaError_t e = set_smem(k_weights<IO>, sm);
     if (e != cudaSuccess) return e;
     const dim3 grid((rows + kWRows - 1) / kWRows, a.B * a.H);
-    LUNA_LAUNCH("weights", k_weights<IO>, grid, kThreads, sm, s, a, causal, row0, rows, teacher, A);
+    LUNA_LAUNCH("weights", k_weights<IO>, grid, kThreads, sm, s, a, causal, row0, rows, teacher, tstride, A);
     return cudaGetLastError();
 }
 
@@ -146,10 +148,10 @@ cudaError_t weights_impl(const AttnArgs &a, int causal, int row0, int rows, int 
 
 size_t weights_max_smem(const AttnArgs &a) { return smem_weights(a); }
 
-cudaError_t launch_weights(const AttnArgs &a, luna_dtype io, int causal, int row0, int rows, int teacher, float *A,
-                           cudaStream_t s) {
-    return io == LUNA_F32 ? weights_impl<float>(a, causal, row0, rows, teacher, A, s)
-                          : weights_impl<__nv_bfloat16>(a, causal, row0, rows, teacher, A, s);
+cudaError_t launch_weights(const AttnArgs &a, luna_dtype io, int causal, int row0, int rows, int teacher,
+                           int64_t tstride, float *A, cudaStream_t s) {
+    return io == LUNA_F32 ? weights_impl<float>(a, causal, row0, rows, teacher, tstride, A, s)
+                          : weights_impl<__nv_bfloat16>(a, causal, row0, rows, teacher, tstride, A, s);
 }
 
 }  // namespace luna

@@ -33,7 +33,8 @@ class LunaError(RuntimeError):
 
 class PhiDesc(ctypes.Structure):
     _fields_ = [("M", ctypes.c_int), ("L", ctypes.c_int), ("hidden", ctypes.c_int), ("shared_channels", ctypes.c_int),
-                ("ch_rms_target", ctypes.c_float), ("signed_outputs", ctypes.c_int)]
+                ("ch_rms_target", ctypes.c_float), ("signed_outputs", ctypes.c_int),
+                ("param_head_stride", ctypes.c_int64)]
 
 
 class PhiParams(ctypes.Structure):
@@ -125,8 +126,8 @@ def _io_code(t: torch.Tensor) -> int:
 
 
 def phi_desc(M: int, L: int, hidden: int, shared: bool = False, ch_rms_target: float = 0.0,
-             signed: bool = False) -> PhiDesc:
-    return PhiDesc(M, L, hidden, int(bool(shared)), float(ch_rms_target), int(bool(signed)))
+             signed: bool = False, param_head_stride: int = 0) -> PhiDesc:
+    return PhiDesc(M, L, hidden, int(bool(shared)), float(ch_rms_target), int(bool(signed)), int(param_head_stride))
 
 
 def attn_desc(B, H, n, d, dv, causal=False, chunk=0, eps=1e-6, io=LUNA_BF16) -> AttnDesc:
@@ -258,18 +259,29 @@ class Luna:
     """Owns the table, workspace and state buffers of one problem shape."""
 
     def __init__(self, B, H, n, d, dv, M, L, hidden=64, causal=False, eps=1e-6, io=torch.bfloat16, chunk=0,
-                 device="cuda", shared=False, ch_rms_target=0.0, signed=False):
+                 device="cuda", shared=False, ch_rms_target=0.0, signed=False, per_head=False):
         self.pd = phi_desc(M, L, hidden, shared, ch_rms_target, signed)
         self.ad = attn_desc(B, H, n, d, dv, causal, chunk, eps, _DTYPES[io])
         self.d = d
         self.device = torch.device(device)
-        self.table = alloc_bytes(luna_phi_table_size(self.pd, d), self.device)
+        tb = luna_phi_table_size(self.pd, d)
+        self.heads = H if per_head else 0  # per-head parameters: one table per head, tb bytes apart
+        if per_head:
+            self.pd.param_head_stride = tb
+        self.table = alloc_bytes(tb * max(1, self.heads), self.device)
         self.ws = alloc_bytes(max(luna_workspace_size(self.ad, self.pd, False),
                                   luna_workspace_size(self.ad, self.pd, True)), self.device)
         self.state = alloc_bytes(luna_state_size(self.ad, self.pd), self.device)
 
     def prepare(self, params: dict, stream=None):
-        luna_phi_prepare(self.pd, self.d, params, self.table, stream)
+        """params: W, b, w1, b1, w2, b2 device tensors (with a leading head axis for per-head parameters)."""
+        if not self.heads:
+            luna_phi_prepare(self.pd, self.d, params, self.table, stream)
+            return
+        tb = self.pd.param_head_stride
+        for h in range(self.heads):
+            luna_phi_prepare(self.pd, self.d, {k: v[h] for k, v in params.items()}, self.table[h * tb:(h + 1) * tb],
+                             stream)
 
     def forward(self, Q, K, V, lengths=None, O=None, save_state=True, stream=None):
         if O is None:
@@ -283,10 +295,11 @@ class Luna:
             M, L, hid = self.pd.M, self.pd.L, self.pd.hidden
             f32 = dict(dtype=torch.float32, device=Q.device)
             fc1 = (hid,) if self.pd.shared_channels else (L, hid)
+            g = (self.heads,) if self.heads else ()
             out = {"dQ": torch.empty_like(Q), "dK": torch.empty_like(K), "dV": torch.empty_like(V),
-                   "dW": torch.empty(M, self.d, **f32), "db": torch.empty(M, **f32),
-                   "dw1": torch.empty(fc1, **f32), "db1": torch.empty(fc1, **f32),
-                   "dw2": torch.empty(L, hid, **f32), "db2": torch.empty(L, **f32)}
+                   "dW": torch.empty(g + (M, self.d), **f32), "db": torch.empty(g + (M,), **f32),
+                   "dw1": torch.empty(g + fc1, **f32), "db1": torch.empty(g + fc1, **f32),
+                   "dw2": torch.empty(g + (L, hid), **f32), "db2": torch.empty(g + (L,), **f32)}
         luna_attn_bwd(self.ad, self.pd, self.table, Q, K, V, dO, lengths, self.state if use_state else None,
                       out["dQ"], out["dK"], out["dV"], out, self.ws, stream)
         return out

@@ -105,12 +105,16 @@ def to_host(x) -> np.ndarray:
 class Case:
     def __init__(self, B, H, n, d, M, L, io, causal=False, seed=0, qkv_scale=1.0, len_range=None, hidden=64,
                  eps=1e-6, dv=None, with_grad=False, lengths=None, shared=False, ch_rms_target=0.0, signed=False,
-                 params=None):
+                 params=None, per_head=False):
         self.B, self.H, self.n, self.d, self.M, self.L = B, H, n, d, M, L
         self.ch_rms_target = ch_rms_target
         self.signed = signed
+        self.per_head = per_head
         self.dv = dv or d
         self.io, self.causal, self.eps, self.hidden, self.shared = io, causal, eps, hidden, shared
+        if params is None and per_head:  # one parameter set per head, each from its own seed
+            sets = [synth.phi_params(seed * 1000 + h, d, M, L, hidden, shared) for h in range(H)]
+            params = {k: np.stack([s[k] for s in sets]) for k in sets[0]}
         self.params = params if params is not None else synth.phi_params(seed, d, M, L, hidden, shared)
         self.inp = synth.attn_inputs(seed, B, H, n, d, self.dv, io, qkv_scale, len_range, with_grad)
         if lengths is not None:
@@ -124,7 +128,7 @@ class Case:
         import paper_2512_08061_gb300.luna as L
         lu = L.Luna(self.B, self.H, self.n, self.d, self.dv, self.M, self.L, self.hidden, self.causal, self.eps,
                     torch.float32 if self.io == "f32" else torch.bfloat16, chunk, shared=self.shared,
-                    ch_rms_target=self.ch_rms_target, signed=self.signed)
+                    ch_rms_target=self.ch_rms_target, signed=self.signed, per_head=self.per_head)
         self.guards = []
         for name in ("table", "ws", "state"):
             setattr(lu, name, guarded_bytes(getattr(lu, name).numel(), lu.device, self.guards))
@@ -147,10 +151,12 @@ class Case:
         d = self.dev
         dev = d["Q"].device
         fc1 = (self.hidden,) if self.shared else (self.L, self.hidden)
+        g = (self.H,) if self.per_head else ()
         shapes = {"dQ": (tuple(d["Q"].shape), d["Q"].dtype), "dK": (tuple(d["K"].shape), d["K"].dtype),
-                  "dV": (tuple(d["V"].shape), d["V"].dtype), "dW": ((self.M, self.d), torch.float32),
-                  "db": ((self.M,), torch.float32), "dw1": (fc1, torch.float32), "db1": (fc1, torch.float32),
-                  "dw2": ((self.L, self.hidden), torch.float32), "db2": ((self.L,), torch.float32)}
+                  "dV": (tuple(d["V"].shape), d["V"].dtype), "dW": (g + (self.M, self.d), torch.float32),
+                  "db": (g + (self.M,), torch.float32), "dw1": (g + fc1, torch.float32),
+                  "db1": (g + fc1, torch.float32), "dw2": (g + (self.L, self.hidden), torch.float32),
+                  "db2": (g + (self.L,), torch.float32)}
         out = {k: guarded_empty(shp, dt, dev, self.guards) for k, (shp, dt) in shapes.items()}
         g = lu.backward(d["Q"], d["K"], d["V"], d["dO"], d["lengths"], use_state=use_state, out=out)
         check_guards(self.guards)
@@ -161,7 +167,7 @@ class Case:
     def phi(self):
         """The oracle's feature map: the parameters, with the channel normalisation and the signed
         channel outputs when they are on."""
-        if self.ch_rms_target or self.signed:
+        if self.ch_rms_target or self.signed or self.per_head:
             return oracle.PhiParams(self.params, self.ch_rms_target, nonneg=not self.signed)
         return self.params
 

@@ -670,3 +670,68 @@ def test_signed_channel_featmap_and_decode():
            for k in ("Q", "K", "V")}
     o = to_host(lu.decode(tok["Q"], tok["K"], tok["V"]))
     assert relerr(o, full[:, :, n - 1]) < 1e-4
+
+
+# --------------------------------------------------------------------------
+# per-head feature-map parameters (the conversion's per-layer, per-head instantiation)
+
+@pytest.mark.parametrize("io,d,M,causal,lengths,H", [
+    ("bf16", 32, 8, False, [300, 177, 1], 3),   # tensor-core non-causal, d = 32 (LRA shape)
+    ("bf16", 64, 8, False, None, 4),            # tensor-core non-causal, d = 64 (BERT / ViT shape)
+    ("bf16", 128, 16, True, [300, 250], 2),     # tensor-core streaming form, d = 128
+    ("f32", 32, 8, False, [300, 41], 3),        # generic kernels
+    ("f32", 32, 8, True, [300, 200], 2),
+])
+def test_per_head_parameters(io, d, M, causal, lengths, H):
+    """Head h of every sequence uses its own W, b and channel MLPs: forward and
+    backward against the oracle's per-head mode, each head's parameter
+    gradients summed over the batch only, with the state saved by the forward
+    (the library runs one sub-problem per head index over strided views of the
+    caller's tensors, state and gradients)."""
+    B = len(lengths) if lengths else 2
+    case = Case(B, H, 300, d, M, 8, io, causal, seed=113, qkv_scale=1.0 / math.sqrt(d), lengths=lengths,
+                with_grad=True, per_head=True)
+    assert case.params["W"].shape == (H, M, d)
+    lu = case.luna()
+    O = to_host(case.run_fwd(lu))
+    ref = case.oracle_fwd()
+    assert (relerr_rows(O, ref) if causal else relerr(O, ref)) < TOL[io]
+    g = {k: to_host(v) for k, v in case.run_bwd(lu).items()}
+    rb = case.oracle_bwd()
+    okq, okk = case.smooth_rows("Q"), case.smooth_rows("K")
+    assert okq.mean() > 0.9 and okk.mean() > 0.9
+    assert relerr(g["dQ"][okq], rb["dQ"][okq]) < TOL[io]
+    assert relerr(g["dK"][okk], rb["dK"][okk]) < TOL[io]
+    assert relerr(g["dV"], rb["dV"]) < TOL[io]
+    for k in ("dW", "db", "dw1", "db1", "dw2", "db2"):
+        assert g[k].shape[0] == H
+        for h in range(H):
+            assert relerr(g[k][h], rb[k][h]) < TOL[io], (k, h)
+    if lengths is not None:
+        for b, ln in enumerate(lengths):
+            for k in ("dQ", "dK", "dV"):
+                assert np.all(g[k][b, :, ln:] == 0)
+
+
+def test_per_head_parameters_decode_and_weights():
+    """The decode step and the attention weights read the table of their own head."""
+    import torch
+    import paper_2512_08061_gb300.luna as L
+    d, M, H, n = 64, 8, 3, 41
+    case = Case(2, H, n, d, M, 8, "f32", True, seed=127, qkv_scale=1.0 / math.sqrt(d), per_head=True)
+    full = case.oracle_fwd()
+    pre = Case(2, H, n - 1, d, M, 8, "f32", True, seed=127, qkv_scale=1.0 / math.sqrt(d), per_head=True,
+               params=case.params)
+    for k in ("Q", "K", "V"):
+        pre.inp[k] = synth.IOTensor(case.inp[k].value[:, :, :n - 1], "f32")
+    lu = pre.luna()
+    pre.run_fwd(lu, save_state=True)
+    tok = {k: torch.from_numpy(np.ascontiguousarray(case.inp[k].value[:, :, n - 1]).astype(np.float32)).cuda()
+           for k in ("Q", "K", "V")}
+    o = to_host(lu.decode(tok["Q"], tok["K"], tok["V"]))
+    assert relerr(o, full[:, :, n - 1]) < 1e-4
+    lu2 = case.luna()
+    A = torch.empty((2, H, n, n), dtype=torch.float32, device="cuda")
+    L.luna_attn_weights(lu2.ad, lu2.pd, lu2.table, case.dev["Q"], case.dev["K"], None, 0, n, False, A)
+    ref = oracle.attn_weights(case.phi, case.inp["Q"].value, case.inp["K"].value, None, True, case.eps)
+    assert relerr(to_host(A), ref) < 1e-4
