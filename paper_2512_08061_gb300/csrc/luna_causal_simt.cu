@@ -68,25 +68,27 @@ __device__ void advance_state(float *S, float *z, const float *sPk, const float 
     }
 }
 
-// den_r = eps + phi(q_r).z + sum_{j<=r} A[r][j];  O_r = (phi(q_r) S + sum_{j<=r} A[r][j] v_j) / den_r
+// den_r = eps + phi(q_r).z + sum_{j<=r} A[r][j];  O_r = (phi(q_r) S + sum_{j<=r} A[r][j] v_j) / den_r,
+// both formed in fp64 and rounded once (the backward's gradients cancel to a small part of their terms
+// under the scale invariance of each row, so a row's rounding must stay at half an ulp)
 __device__ void chunk_outputs(const AttnArgs &a, const float *S, const float *z, const float *sPq, const float *sA,
                               const float *sV, int nr, float *sden, float *sO) {
     const int D = a.D, dv = a.dv;
     for (int r = threadIdx.x; r < nr; r += blockDim.x) {
-        float den = a.eps;
-        for (int f = 0; f < D; ++f) den = fmaf(sPq[r * D + f], z[f], den);
-        for (int j = 0; j <= r; ++j) den += sA[r * kCs + j];
-        sden[r] = den;
+        double den = a.eps;
+        for (int f = 0; f < D; ++f) den = fma((double)sPq[r * D + f], (double)z[f], den);
+        for (int j = 0; j <= r; ++j) den += (double)sA[r * kCs + j];
+        sden[r] = (float)den;
     }
     __syncthreads();
     for (int e = threadIdx.x; e < nr * dv; e += blockDim.x) {
         const int r = e / dv, c = e - r * dv;
         float o = 0.0f;
         if (sden[r] != 0.0f) {
-            float num = 0.0f;
-            for (int f = 0; f < D; ++f) num = fmaf(sPq[r * D + f], S[f * dv + c], num);
-            for (int j = 0; j <= r; ++j) num = fmaf(sA[r * kCs + j], sV[j * dv + c], num);
-            o = num / sden[r];
+            double num = 0.0;
+            for (int f = 0; f < D; ++f) num = fma((double)sPq[r * D + f], (double)S[f * dv + c], num);
+            for (int j = 0; j <= r; ++j) num = fma((double)sA[r * kCs + j], (double)sV[j * dv + c], num);
+            o = (float)(num / (double)sden[r]);
         }
         sO[e] = o;
     }

@@ -203,19 +203,22 @@ __global__ void __launch_bounds__(kThreads) k_bwd_query(AttnArgs a) {
         __syncthreads();
         phi_tile(lay, s, sQ, nr, sPhi, sU, sJ);
         __syncthreads();
+        // den and o_i are formed in fp64 and rounded once: the gradients below cancel to a small part of
+        // their terms (the loss barely changes under a common scale of phi(q_i)), so each row's rounding
+        // must stay at half an ulp
         for (int r = threadIdx.x; r < nr; r += blockDim.x) {
-            float den = a.eps;
-            for (int f = 0; f < D; ++f) den = fmaf(sPhi[r * D + f], sz[f], den);
-            sden[r] = den;
+            double den = a.eps;
+            for (int f = 0; f < D; ++f) den = fma((double)sPhi[r * D + f], (double)sz[f], den);
+            sden[r] = (float)den;
         }
         __syncthreads();
         for (int e = threadIdx.x; e < nr * dv; e += blockDim.x) {  // o_i into sdnum for now
             const int r = e / dv, c = e - r * dv;
             float o = 0.0f;
             if (sden[r] != 0.0f) {
-                float num = 0.0f;
-                for (int f = 0; f < D; ++f) num = fmaf(sPhi[r * D + f], sS[f * dv + c], num);
-                o = num / sden[r];
+                double num = 0.0;
+                for (int f = 0; f < D; ++f) num = fma((double)sPhi[r * D + f], (double)sS[f * dv + c], num);
+                o = (float)(num / (double)sden[r]);
             }
             sdnum[e] = o;
         }
@@ -228,7 +231,7 @@ __global__ void __launch_bounds__(kThreads) k_bwd_query(AttnArgs a) {
         __syncthreads();
         for (int e = threadIdx.x; e < nr * dv; e += blockDim.x) {
             const int r = e / dv;
-            sdnum[e] = (sden[r] != 0.0f) ? sdO[e] / sden[r] : 0.0f;
+            sdnum[e] = (sden[r] != 0.0f) ? (float)((double)sdO[e] / (double)sden[r]) : 0.0f;
         }
         __syncthreads();
         for (int e = threadIdx.x; e < nr * D; e += blockDim.x) {
