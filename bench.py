@@ -70,8 +70,8 @@ def parse():
     args = ap.parse_args()
     if args.ch_rms_target < 0:
         ap.error("--ch-rms-target must be >= 0")
-    if args.ch_rms_target > 0 and (WORKLOADS[args.workload].causal or WORKLOADS[args.workload].decode):
-        ap.error("--ch-rms-target: the channel normalisation is built for the non-causal form only")
+    if args.ch_rms_target > 0 and WORKLOADS[args.workload].decode:
+        ap.error("--ch-rms-target: the channel normalisation is a batch statistic, not defined for a decode step")
     args.also = [a for a in args.also.split(",") if a]
     for a in args.also:
         if a not in WORKLOADS or WORKLOADS[a].decode:

@@ -73,9 +73,12 @@ typedef enum { LUNA_F32 = 0, LUNA_BF16 = 1 } luna_dtype;
  * every valid row (rows at or past a sequence's length excluded) and every
  * projection; the backward pass includes the dependence of s_l on every
  * sample.  0 = off (the listing's default); negative, NaN or infinite is
- * LUNA_ERR_INVALID_ARG.  With it on, only the non-causal luna_attn_fwd /
- * luna_attn_bwd are supported (the causal form, luna_featmap and
- * luna_attn_decode give LUNA_ERR_UNSUPPORTED).
+ * LUNA_ERR_INVALID_ARG.  With it on, luna_attn_fwd / luna_attn_bwd support
+ * both forms (the streaming form runs on a copy of the table, in the
+ * workspace, whose channel-l coefficients are scaled by sqrt(s^q_l s^k_l));
+ * luna_featmap, luna_attn_decode and luna_attn_weights give
+ * LUNA_ERR_UNSUPPORTED (a batch statistic has no single-row or single-token
+ * form).
  * signed_outputs = 1 is the listing's ScalarMLP(nonneg = False): the channel
  * outputs are fc2(relu(fc1(u))) without the outer ReLU, so features (and kernel
  * values) of either sign; 0 keeps the outer ReLU (the listing's default).  The

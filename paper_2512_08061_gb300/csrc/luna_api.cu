@@ -50,6 +50,7 @@ struct Plan {
     size_t o_items = 0;                        // split of the tensor-core work items (non-causal)
     float ch_target = 0.0f;                    // channel RMS normalisation (non-causal; 0: off)
     size_t o_chpart = 0, o_chstat = 0, o_chsigma = 0, o_chkappa = 0, o_chT = 0;
+    size_t o_chtab = 0;                        // streaming form: the sqrt(sigma)-scaled table
     size_t ws_fwd = 0, ws_bwd = 0, state_bytes = 0;
     TcPlan tc;
 };
@@ -85,7 +86,6 @@ luna_status make_plan(const luna_attn_desc *ad, const luna_phi_desc *pd, Plan &p
     luna_status st = check_phi(pd, ad->d);
     if (st != LUNA_OK) return st;
     if (ad->dv > kMaxD || ad->n > (1 << 24)) return LUNA_ERR_UNSUPPORTED;
-    if (pd->ch_rms_target > 0.0f && ad->causal) return LUNA_ERR_UNSUPPORTED;  // non-causal form only
     p.ch_target = pd->ch_rms_target;
     if ((int64_t)ad->B * ad->H > (1 << 24)) return LUNA_ERR_UNSUPPORTED;
 
@@ -148,13 +148,23 @@ luna_status make_plan(const luna_attn_desc *ad, const luna_phi_desc *pd, Plan &p
         p.o_zpart = w.take((size_t)BH * ns * D * f);
         p.o_segS = w.take((size_t)BH * (ns + 1) * SD * f);
         p.o_segz = w.take((size_t)BH * (ns + 1) * D * f);
+        if (p.ch_target > 0.0f) {
+            p.o_chpart = w.take(2 * (size_t)kChStatBlocks * p.lay.L * f);
+            p.o_chstat = w.take(8 * (size_t)kMaxL * sizeof(double));
+            p.o_chsigma = w.take((size_t)kMaxL * f);
+            p.o_chkappa = w.take(2 * (size_t)kMaxL * f);
+            // T rows: one per block of the tensor-core chain rule or per (head, segment) of the generic one
+            p.o_chT = w.take((size_t)std::max<int64_t>(kMaxGrid, (int64_t)BH * ns) * p.lay.L * sizeof(double));
+            p.o_chtab = w.take((size_t)p.lay.bytes);
+        }
         p.ws_fwd = w.n;
         p.o_dSpart = w.take((size_t)BH * ns * SD * f);
         p.o_dzpart = w.take((size_t)BH * ns * D * f);
         p.o_segdS = w.take((size_t)BH * ns * SD * f);
         p.o_segdz = w.take((size_t)BH * ns * D * f);
         p.o_rowstat = w.take((size_t)BH * n * 2 * f);
-        p.o_gpart = w.take(2 * (size_t)BH * ns * p.gsize * sizeof(double));
+        p.o_gpart = w.take((2 * (size_t)BH * ns + (p.ch_target > 0.0f ? 2 * kChKBlocks : 0)) * p.gsize *
+                           sizeof(double));
         p.o_hist = w.take((size_t)p.gsize * sizeof(double));
         p.ws_bwd = w.n;
         p.state_bytes = (size_t)BH * (ns + 1) * (SD + D) * f;
@@ -213,6 +223,16 @@ AttnArgs make_args(const luna_attn_desc *ad, const Plan &p, const void *table, c
     } else {
         a.seg_S = reinterpret_cast<float *>(w + p.o_segS);
         a.seg_z = reinterpret_cast<float *>(w + p.o_segz);
+        if (p.ch_target > 0.0f) {
+            a.ch_target = p.ch_target;
+            a.ch_io = ad->io;
+            a.ch_causal = 1;
+            a.ch_part = reinterpret_cast<float *>(w + p.o_chpart);
+            a.ch_stat = reinterpret_cast<double *>(w + p.o_chstat);
+            a.ch_sigma = reinterpret_cast<float *>(w + p.o_chsigma);
+            a.ch_kappa = reinterpret_cast<float *>(w + p.o_chkappa);
+            a.ch_T = reinterpret_cast<double *>(w + p.o_chT);
+        }
     }
     return a;
 }
@@ -360,6 +380,11 @@ luna_status luna_attn_fwd(const luna_attn_desc *ad, const luna_phi_desc *pd, con
     cudaError_t e = cudaMemsetAsync(workspace, 0, p.o_counters + 2 * sizeof(int) * (size_t)p.BH, s);
     if (e != cudaSuccess) return LUNA_ERR_CUDA;
     if (a.ch_sigma && (e = launch_chrms_stats(a, ad->io, s)) != cudaSuccess) return LUNA_ERR_CUDA;
+    if (a.ch_causal) {  // the streaming form runs on the sqrt(sigma)-scaled table
+        if ((e = launch_chrms_table(a, static_cast<char *>(workspace) + p.o_chtab, s)) != cudaSuccess)
+            return LUNA_ERR_CUDA;
+        a.table = static_cast<const char *>(workspace) + p.o_chtab;
+    }
     const int nsub = pd->param_head_stride ? ad->H : 1;  // per-head parameters: one sub-problem per head index
     for (int h = 0; h < nsub; ++h) {
         const AttnArgs b = pd->param_head_stride ? head_args(a, ad, pd, p, h) : a;
@@ -425,6 +450,10 @@ luna_status luna_attn_bwd(const luna_attn_desc *ad, const luna_phi_desc *pd, con
     cudaError_t e = cudaMemsetAsync(workspace, 0, p.o_counters + 2 * sizeof(int) * (size_t)p.BH, s);
     if (e != cudaSuccess) return LUNA_ERR_CUDA;
     if (a.ch_sigma && (e = launch_chrms_stats(a, ad->io, s)) != cudaSuccess) return LUNA_ERR_CUDA;
+    if (a.ch_causal) {  // the streaming form runs on the sqrt(sigma)-scaled table
+        if ((e = launch_chrms_table(a, w + p.o_chtab, s)) != cudaSuccess) return LUNA_ERR_CUDA;
+        a.table = w + p.o_chtab;
+    }
     if (ad->causal && p.tc.causal_bwd) {
         a.dphi = reinterpret_cast<float *>(w + p.o_dphi);
         a.phik = w + p.o_phik;

@@ -53,18 +53,19 @@ __device__ void masked_scores(const float *sPq, const float *sPk, int nr, int D,
     }
 }
 
-// state update S += phi(K)^T V, z += sum phi(K) over the chunk rows
+// state update S += phi(K)^T V, z += sum phi(K) over the chunk rows (fp64, one rounding per chunk: the
+// running state is shared by every later row, so its rounding does not average out in the gradients)
 __device__ void advance_state(float *S, float *z, const float *sPk, const float *sV, int nr, int D, int dv) {
     for (int e = threadIdx.x; e < D * dv; e += blockDim.x) {
         const int f = e / dv, c = e - f * dv;
-        float acc = S[e];
-        for (int r = 0; r < nr; ++r) acc = fmaf(sPk[r * D + f], sV[r * dv + c], acc);
-        S[e] = acc;
+        double acc = S[e];
+        for (int r = 0; r < nr; ++r) acc = fma((double)sPk[r * D + f], (double)sV[r * dv + c], acc);
+        S[e] = (float)acc;
     }
     for (int f = threadIdx.x; f < D; f += blockDim.x) {
-        float acc = z[f];
-        for (int r = 0; r < nr; ++r) acc += sPk[r * D + f];
-        z[f] = acc;
+        double acc = z[f];
+        for (int r = 0; r < nr; ++r) acc += (double)sPk[r * D + f];
+        z[f] = (float)acc;
     }
 }
 
@@ -159,7 +160,7 @@ __global__ void __launch_bounds__(kThreads) k_causal_bwd_seg(AttnArgs a) {
     const bool active = threadIdx.x < nf * nc;
     const int tf = active ? threadIdx.x / nc : 0, tc = active ? threadIdx.x % nc : 0;
     const int f0 = tf * 8, c0 = tc * 8;
-    float acc[8][8] = {}, zacc[8] = {};
+    double acc[8][8] = {}, zacc[8] = {};
     for (int t0 = r0; t0 < r1; t0 += kCs) {
         const int nr = min(kCs, r1 - t0);
         __syncthreads();
@@ -219,6 +220,8 @@ __global__ void __launch_bounds__(kThreads) k_causal_dq(AttnArgs a) {
     float *sdU = cv.take(kCs * M);
     if (!carve_fits(cv, smem)) return;
     const int bh = blockIdx.y, seg = blockIdx.x;
+    __shared__ double sT[kMaxL];  // channel normalisation: the block's sums of phi . dphi per channel
+    if ((int)threadIdx.x < kMaxL) sT[threadIdx.x] = 0.0;
     double *gp = reinterpret_cast<double *>(a.gpart) + ((size_t)bh * a.nseg + seg) * a.gsize;
     double *shist = gp + M * d + M;  // the block's fp64 histogram, accumulated in place by L2 atomics
     const int len = head_length(a.lengths, bh / a.H, a.n);
@@ -264,6 +267,7 @@ __global__ void __launch_bounds__(kThreads) k_causal_dq(AttnArgs a) {
             for (int c = 0; c < dv; ++c) acc = fma((double)S[f * dv + c], (double)sdO[r * dv + c], acc);
             for (int j = 0; j <= r; ++j) acc = fma((double)sP[r * kCs + j], (double)sPk[j * D + f], acc);
             sdPq[e] = (float)acc;
+            if (a.ch_T) atomicAdd(sT + f % a.L, (double)sPq[e] * acc);
         }
         __syncthreads();
         advance_state(S, z, sPk, sV, nr, D, dv);
@@ -272,6 +276,7 @@ __global__ void __launch_bounds__(kThreads) k_causal_dq(AttnArgs a) {
     }
     __syncthreads();
     store_grad_partial(lay, g, gp);
+    if (a.ch_T && (int)threadIdx.x < a.L) a.ch_T[((size_t)bh * a.nseg + seg) * a.L + threadIdx.x] = sT[threadIdx.x];
 }
 
 // dK, dV: reverse sweep with the suffix state G (after the current chunk).
@@ -355,14 +360,14 @@ __global__ void __launch_bounds__(kThreads) k_causal_dkv(AttnArgs a) {
             // G += phi(Q_chunk)^T dnum, g += phi(Q_chunk)^T dden
             for (int e = threadIdx.x; e < D * dv; e += blockDim.x) {
                 const int f = e / dv, c = e - f * dv;
-                float acc = G[e];
-                for (int r = 0; r < nr; ++r) acc = fmaf(sPq[r * D + f], sdO[r * dv + c], acc);
-                G[e] = acc;
+                double acc = G[e];
+                for (int r = 0; r < nr; ++r) acc = fma((double)sPq[r * D + f], (double)sdO[r * dv + c], acc);
+                G[e] = (float)acc;
             }
             for (int f = threadIdx.x; f < D; f += blockDim.x) {
-                float acc = gz[f];
-                for (int r = 0; r < nr; ++r) acc = fmaf(sPq[r * D + f], sdden[r], acc);
-                gz[f] = acc;
+                double acc = gz[f];
+                for (int r = 0; r < nr; ++r) acc = fma((double)sPq[r * D + f], (double)sdden[r], acc);
+                gz[f] = (float)acc;
             }
             phi_backward_tile(lay, s, sK, nr, sPk, sdPk, sU, sJ, sdU, shist, g);
             store_dx(lay, s, sdU, nr, dK + (size_t)t0 * d);
@@ -429,7 +434,12 @@ cudaError_t causal_bwd_impl(const AttnArgs &a0, bool have_state, cudaStream_t s)
     if ((e = set_smem(k_causal_dkv<IO>, sm)) != cudaSuccess) return e;
     LUNA_LAUNCH("causal_dkv", k_causal_dkv<IO>, grid, kThreads, sm, s, a);
     if ((e = cudaGetLastError()) != cudaSuccess) return e;
-    return launch_grad_reduce(a, 2 * a.B * a.H * a.nseg, s);
+    int nparts = 2 * a.B * a.H * a.nseg;
+    if (a.ch_sigma) {  // the scale term of the channel normalisation (kappa from the queries' T rows)
+        a.ch_T_rows = a.B * a.H * a.nseg;
+        if ((e = launch_chrms_backward(a, nparts, &nparts, s)) != cudaSuccess) return e;
+    }
+    return launch_grad_reduce(a, nparts, s);
 }
 
 }  // namespace

@@ -23,6 +23,18 @@
 // on both sides (S', z' the scaled statistics, dS, dz before scaling): the sample
 // sums collapse onto each head's statistics.  The kappa term then runs through the
 // ordinary chain rule of the feature map as dLoss/dphi = M kappa_l phi (phi = y/sqrt(M)).
+//
+// Streaming (causal) form: the prefix states do not collapse the sample sums, so
+// both sides run on a copy of the table whose channel-l coefficients are scaled
+// by sqrt(sigma_l): phi^ = sqrt(sigma) phi on queries and keys gives the same
+// kernel value, and the streaming kernels run unchanged.  T_l is the sum over the
+// query samples of phi^ . dLoss/dphi^ on channel l (equal to the sum over the
+// normalised features, and the same for the key side, since the loss depends on
+// s^q_l and s^k_l only through their product), accumulated by the chain-rule
+// kernel of the queries.  The kappa term runs on the scaled table with kappa_l /
+// sigma_l (its dU is then that of the unscaled map), and before the channel-MLP
+// gradients the reduced interval histogram of channel l, a sum of dLoss/dphi^,
+// is multiplied by sqrt(sigma_l) to give sums of dLoss/dphi.
 #include <math.h>
 
 #include "luna_prof.cuh"
@@ -196,10 +208,11 @@ __global__ void __launch_bounds__(128) k_chrms_dstate(AttnArgs a, const float *s
 }
 
 // kappa[side*kMaxL + l] = d s_l / d rms_l * (T_l / s_l) / (N rms_l), zero where the scale is clamped
-// at 1 (target/(rms + eps) > 1) or the side has no samples.
-__global__ void __launch_bounds__(kRed) k_chrms_kappa(AttnArgs a, const double *T, float target, const double *stat,
-                                                      float *kappa) {
-    const int BH = a.B * a.H, L = a.L, warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+// at 1 (target/(rms + eps) > 1) or the side has no samples; T_l the sum of rows T[0 .. BH)[l] in order.
+// With `sigma` (the streaming form's scaled table), kappa_l / sigma_l.
+__global__ void __launch_bounds__(kRed) k_chrms_kappa(AttnArgs a, const double *T, int BH, float target,
+                                                      const double *stat, const float *sigma, float *kappa) {
+    const int L = a.L, warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     const double N = stat[3 * kMaxL];
     for (int l = warp; l < L; l += blockDim.x >> 5) {
         double v = 0.0;
@@ -211,7 +224,8 @@ __global__ void __launch_bounds__(kRed) k_chrms_kappa(AttnArgs a, const double *
                 const double s = stat[(side * 4 + 0) * kMaxL + l], rms = stat[(side * 4 + 1) * kMaxL + l];
                 const double r = stat[(side * 4 + 2) * kMaxL + l];
                 const double ds = -(double)target / ((rms + kChEps) * (rms + kChEps));  // d s / d rms, unclamped
-                kappa[side * kMaxL + l] = (N > 0.0 && r <= 1.0) ? (float)(ds * (v / s) / (N * rms)) : 0.0f;
+                const double k = (N > 0.0 && r <= 1.0) ? ds * (v / s) / (N * rms) : 0.0;
+                kappa[side * kMaxL + l] = (float)(sigma ? k / (double)sigma[l] : k);
             }
     }
 }
@@ -329,6 +343,23 @@ __global__ void __launch_bounds__(kKWarps * 32) k_chrms_kterm(AttnArgs a, const 
     for (int e = threadIdx.x; e < M; e += blockDim.x) gp[Md + e] = (GP)sdb[e];
 }
 
+// Copy of the table with every channel's (alpha, beta) scaled by sqrt(sigma_l) (streaming form).
+__global__ void k_chrms_scale_table(const float *src, float *dst, TableLayout lay, const float *sigma) {
+    const int64_t n = lay.bytes / 4, ab0 = lay.off_AB / 4, ab1 = ab0 + (int64_t)lay.nint * lay.L * 2;
+    for (int64_t e = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; e < n; e += (int64_t)gridDim.x * blockDim.x) {
+        float v = src[e];
+        if (e >= ab0 && e < ab1) v *= sqrtf(sigma[(int)(((e - ab0) >> 1) % lay.L)]);
+        dst[e] = v;
+    }
+}
+
+// Reduced interval histogram [nint][L][2] (after dW, db) of channel l times sqrt(sigma_l).
+__global__ void k_chrms_scale_hist(double *gsum, TableLayout lay, const float *sigma) {
+    double *h = gsum + (size_t)lay.M * lay.d + lay.M;
+    for (int e = blockIdx.x * blockDim.x + threadIdx.x; e < lay.nint * lay.L * 2; e += gridDim.x * blockDim.x)
+        h[e] *= sqrt((double)sigma[(e >> 1) % lay.L]);
+}
+
 size_t smem_stats(const AttnArgs &a) {
     return (size_t)(r4(a.lay.Ppad) + r4(a.lay.nint * a.lay.L * 2) + r4(a.M * a.d) + r4(a.M) + kThreads) * 4;
 }
@@ -395,10 +426,26 @@ cudaError_t launch_chrms_dstate(const AttnArgs &a, cudaStream_t s) {
     return cudaGetLastError();
 }
 
+cudaError_t launch_chrms_table(const AttnArgs &a, char *dst, cudaStream_t s) {
+    LUNA_LAUNCH("chrms_table", k_chrms_scale_table, blocks_for(a.lay.bytes / 4), 256, 0, s,
+                reinterpret_cast<const float *>(a.table), reinterpret_cast<float *>(dst), a.lay, a.ch_sigma);
+    return cudaGetLastError();
+}
+
+cudaError_t launch_chrms_hist(const AttnArgs &a, cudaStream_t s) {
+    if (!a.ch_sigma || !a.ch_causal) return cudaSuccess;
+    LUNA_LAUNCH("chrms_hist", k_chrms_scale_hist, blocks_for((int64_t)a.lay.nint * a.lay.L * 2), 256, 0, s, a.hist,
+                a.lay, a.ch_sigma);
+    return cudaGetLastError();
+}
+
 cudaError_t launch_chrms_backward(const AttnArgs &a, int main_parts, int *nparts, cudaStream_t s) {
     *nparts = main_parts;
     if (!a.ch_sigma) return cudaSuccess;
-    LUNA_LAUNCH("chrms_kappa", k_chrms_kappa, 1, kRed, 0, s, a, a.ch_T, a.ch_target, a.ch_stat, a.ch_kappa);
+    // non-causal: one T row per head; streaming form: one per block of the queries' chain-rule kernel
+    const int trows = a.ch_causal ? a.ch_T_rows : a.B * a.H;
+    LUNA_LAUNCH("chrms_kappa", k_chrms_kappa, 1, kRed, 0, s, a, a.ch_T, trows, a.ch_target, a.ch_stat,
+                a.ch_causal ? a.ch_sigma : nullptr, a.ch_kappa);
     cudaError_t e = cudaGetLastError();
     if (e != cudaSuccess) return e;
     if (a.gpart64) {

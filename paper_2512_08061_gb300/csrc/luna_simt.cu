@@ -69,7 +69,7 @@ __global__ void __launch_bounds__(kThreads) k_keystats(AttnArgs a) {
     const bool active = threadIdx.x < nf * nc;
     const int tf = active ? threadIdx.x / nc : 0, tc = active ? threadIdx.x % nc : 0;
     const int f0 = tf * 8, c0 = tc * 8;
-    float acc[8][8] = {}, zacc[8] = {};
+    double acc[8][8] = {}, zacc[8] = {};
     for (int t0 = r0; t0 < r1; t0 += kTileK) {
         const int nr = min(kTileK, r1 - t0);
         __syncthreads();
@@ -193,7 +193,7 @@ __global__ void __launch_bounds__(kThreads) k_bwd_query(AttnArgs a) {
     const bool active = threadIdx.x < nf * nc;
     const int tf = active ? threadIdx.x / nc : 0, tc = active ? threadIdx.x % nc : 0;
     const int f0 = tf * 8, c0 = tc * 8;
-    float acc[8][8] = {}, zacc[8] = {};
+    double acc[8][8] = {}, zacc[8] = {};
     GradAcc g = {};
     for (int t0 = r0; t0 < r1; t0 += kTileB) {
         const int nr = min(kTileB, r1 - t0);
@@ -571,6 +571,7 @@ cudaError_t launch_grad_reduce(const AttnArgs &a, int nparts, cudaStream_t s) {
         LUNA_LAUNCH("grad_sum", k_grad_sum<float>, nb, kSumElems * kSumSplit, 0, s, a.gpart, nparts, a.gsize, a.hist);
     cudaError_t e = cudaGetLastError();
     if (e != cudaSuccess) return e;
+    if ((e = launch_chrms_hist(a, s)) != cudaSuccess) return e;
     // the partials have been summed: their buffer holds the shared MLP's per-channel fc1 terms
     double *fc1_part = reinterpret_cast<double *>(a.gpart);
     LUNA_LAUNCH("mlp_grads", k_mlp_grads, a.lay.L + 1, 128, 0, s, a.lay, a.table, a.hist, a.grads, fc1_part);

@@ -52,7 +52,10 @@ struct AttnArgs {
     double *ch_stat;                   // [8][kMaxL]: per side s, rms, target/(rms+eps), unused; [3][0] = N
     float *ch_sigma;                   // [kMaxL]: s^q_l s^k_l
     double *ch_T;                      // [BH][L]: per-head sums of S' . dS + z' dz over each channel's rows
+                                       // (streaming form: [ch_T_rows][L] block sums of phi^ . dLoss/dphi^)
     float *ch_kappa;                   // [2][kMaxL]: factor of y_l in dLoss/dy_l from the scale, per side
+    int ch_causal;                     // streaming form: the kernels run on the sqrt(sigma)-scaled table
+    int ch_T_rows;                     // rows of ch_T written by the streaming form's chain rule
 };
 
 // Row offset of head bh in the caller's tensors (Q, K, V, dO, O, dQ, dK, dV), and its index among the
@@ -103,6 +106,10 @@ cudaError_t launch_chrms_stats(const AttnArgs &a, luna_dtype io, cudaStream_t s)
 cudaError_t launch_chrms_scale_state(const AttnArgs &a, cudaStream_t s);
 cudaError_t launch_chrms_dstate(const AttnArgs &a, cudaStream_t s);
 cudaError_t launch_chrms_backward(const AttnArgs &a, int main_parts, int *nparts, cudaStream_t s);
+// streaming form: the table with channel l's coefficients times sqrt(sigma_l) into dst (a.lay.bytes), and
+// the reduced histogram's channel l times sqrt(sigma_l) (between the partial sum and the MLP gradients)
+cudaError_t launch_chrms_table(const AttnArgs &a, char *dst, cudaStream_t s);
+cudaError_t launch_chrms_hist(const AttnArgs &a, cudaStream_t s);
 size_t chrms_max_smem(const AttnArgs &a);
 size_t causal_max_smem(const AttnArgs &a);
 

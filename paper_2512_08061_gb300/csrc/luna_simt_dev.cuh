@@ -90,25 +90,27 @@ __device__ void phi_tile(const TableLayout &lay, const SmemPhi &s, const float *
     }
 }
 
-// acc[k][m] += sum_r A[r][f0+k] * Bm[r][c0+m];  z[k] += sum_r A[r][f0+k] * (w ? w[r] : 1)
-__device__ __forceinline__ void outer_accumulate(float (&acc)[8][8], float (&zacc)[8], bool do_z, const float *sA,
+// acc[k][m] += sum_r A[r][f0+k] * Bm[r][c0+m];  z[k] += sum_r A[r][f0+k] * (w ? w[r] : 1), accumulated in fp64:
+// the statistics (S, z and dS, dz) are sums over every row of a head, and their rounding is shared by every
+// row that reads them, so it does not average out in the parameter gradients
+__device__ __forceinline__ void outer_accumulate(double (&acc)[8][8], double (&zacc)[8], bool do_z, const float *sA,
                                                  int D, const float *sB, int dv, const float *sw, int nr, int f0,
                                                  int c0) {
     for (int r = 0; r < nr; ++r) {
-        float a8[8], b8[8];
+        double a8[8], b8[8];
 #pragma unroll
         for (int k = 0; k < 8; ++k) {
-            a8[k] = (f0 + k < D) ? sA[r * D + f0 + k] : 0.0f;
-            b8[k] = (c0 + k < dv) ? sB[r * dv + c0 + k] : 0.0f;
+            a8[k] = (f0 + k < D) ? (double)sA[r * D + f0 + k] : 0.0;
+            b8[k] = (c0 + k < dv) ? (double)sB[r * dv + c0 + k] : 0.0;
         }
 #pragma unroll
         for (int k = 0; k < 8; ++k)
 #pragma unroll
-            for (int m = 0; m < 8; ++m) acc[k][m] = fmaf(a8[k], b8[m], acc[k][m]);
+            for (int m = 0; m < 8; ++m) acc[k][m] = fma(a8[k], b8[m], acc[k][m]);
         if (do_z) {
-            const float wr = sw ? sw[r] : 1.0f;
+            const double wr = sw ? (double)sw[r] : 1.0;
 #pragma unroll
-            for (int k = 0; k < 8; ++k) zacc[k] = fmaf(a8[k], wr, zacc[k]);
+            for (int k = 0; k < 8; ++k) zacc[k] = fma(a8[k], wr, zacc[k]);
         }
     }
 }
@@ -123,44 +125,44 @@ __device__ bool last_arrival(int *counter, int expected) {
     return s_flag != 0;
 }
 
-// out[e] = sum_p part[p][e] in order p = 0..nparts-1
+// out[e] = sum_p part[p][e] in order p = 0..nparts-1 (fp64, rounded once)
 __device__ void ordered_sum(const float *part, int nparts, int count, float *out) {
     for (int e = threadIdx.x; e < count; e += blockDim.x) {
-        float s = 0.0f;
+        double s = 0.0;
         for (int p0 = 0; p0 < nparts; p0 += 8) {  // eight loads in flight, added in order
             float v[8];
 #pragma unroll
             for (int k = 0; k < 8; ++k) v[k] = (p0 + k < nparts) ? __ldcg(part + (size_t)(p0 + k) * count + e) : 0.0f;
 #pragma unroll
             for (int k = 0; k < 8; ++k)
-                if (p0 + k < nparts) s += v[k];
+                if (p0 + k < nparts) s += (double)v[k];
         }
-        out[e] = s;
+        out[e] = (float)s;
     }
 }
 
 // Exclusive scan over partials in order: forward (out[p] = sum_{q<p} part[q],
-// out[nparts] = total) or reverse (out[p] = sum_{q>p} part[q]).
+// out[nparts] = total) or reverse (out[p] = sum_{q>p} part[q]); fp64 running sums, each output rounded once.
 __device__ void exclusive_scan(const float *part, int nparts, int count, float *out, bool reverse) {
     for (int e = threadIdx.x; e < count; e += blockDim.x) {
-        float s = 0.0f;
+        double s = 0.0;
         if (!reverse) {
             for (int p = 0; p < nparts; ++p) {
-                out[(size_t)p * count + e] = s;
-                s += __ldcg(part + (size_t)p * count + e);
+                out[(size_t)p * count + e] = (float)s;
+                s += (double)__ldcg(part + (size_t)p * count + e);
             }
-            out[(size_t)nparts * count + e] = s;
+            out[(size_t)nparts * count + e] = (float)s;
         } else {
             for (int p = nparts - 1; p >= 0; --p) {
-                out[(size_t)p * count + e] = s;
-                s += __ldcg(part + (size_t)p * count + e);
+                out[(size_t)p * count + e] = (float)s;
+                s += (double)__ldcg(part + (size_t)p * count + e);
             }
         }
     }
 }
 
 // Writes a (D x dv) register-tiled accumulator and its z-vector to a partial slot.
-__device__ void store_tile(const float (&acc)[8][8], const float (&zacc)[8], bool active, int tc, int f0, int c0,
+__device__ void store_tile(const double (&acc)[8][8], const double (&zacc)[8], bool active, int tc, int f0, int c0,
                            int D, int dv, float *Sp, float *zp) {
     if (!active) return;
 #pragma unroll

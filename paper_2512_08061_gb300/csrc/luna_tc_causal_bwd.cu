@@ -1099,7 +1099,7 @@ bool tc_make_map_rows(CUtensorMap *m, const void *base, int width, int n, int BH
 int tc_sm_count();
 cudaError_t launch_tc_causal_stats(const AttnArgs &a, cudaStream_t s);
 cudaError_t launch_tc_phi_bwd(const AttnArgs &a, const void *X, const float *dphi, void *dX, int slot0, int grid,
-                              cudaStream_t s);
+                              cudaStream_t s, double *tpart = nullptr);
 
 cudaError_t launch_tc_causal_bwd(const AttnArgs &a0, bool have_state, cudaStream_t s) {
     using C = K64;
@@ -1126,7 +1126,9 @@ cudaError_t launch_tc_causal_bwd(const AttnArgs &a0, bool have_state, cudaStream
         return e;
     LUNA_LAUNCH("tcc_query", k_tcc_query<C>, grid, kCBThreads, C::SMEM_Q, s, mQ, mK, mV, mdO, a, st);
     if ((e = cudaGetLastError()) != cudaSuccess) return e;
-    if ((e = launch_tc_phi_bwd(a, a.Q, a.dphi, a.dQ, 0, grid, s)) != cudaSuccess) return e;
+    // (with the channel normalisation the queries' chain rule also sums phi^ . dphi^ per channel and block)
+    if ((e = launch_tc_phi_bwd(a, a.Q, a.dphi, a.dQ, 0, grid, s, a.ch_sigma ? a.ch_T : nullptr)) != cudaSuccess)
+        return e;
     // 2, 3. segment sums of dS, dz and their suffix
     constexpr uint32_t SMEM_S = 2 * (6 * C::T16 + 4096) + 128 + 1024;
     static_assert(SMEM_S <= kSmemLimit, "shared memory budget");
@@ -1144,7 +1146,12 @@ cudaError_t launch_tc_causal_bwd(const AttnArgs &a0, bool have_state, cudaStream
     if ((e = cudaGetLastError()) != cudaSuccess) return e;
     // 5. chain rule for K, then the parameter-gradient reduction over both sides
     if ((e = launch_tc_phi_bwd(a, a.K, a.dphi, a.dK, grid, grid, s)) != cudaSuccess) return e;
-    return launch_grad_reduce(a, 2 * grid, s);
+    int nparts = 2 * grid;
+    if (a.ch_sigma) {  // the scale term of the channel normalisation (kappa from the queries' T rows)
+        a.ch_T_rows = grid;
+        if ((e = launch_chrms_backward(a, 2 * grid, &nparts, s)) != cudaSuccess) return e;
+    }
+    return launch_grad_reduce(a, nparts, s);
 }
 
 }  // namespace luna

@@ -148,9 +148,10 @@ def test_shared_channel_descriptor(L):
 
 def test_channel_rms_descriptor(L):
     """ch_rms_target: 0 is off, a positive value turns the channel normalisation on
-    (more workspace: the statistics and the partials of the scale term), negative,
-    NaN or infinite targets are rejected; the causal form, luna_featmap and
-    luna_attn_decode do not support it (all checked before any device call)."""
+    (more workspace: the statistics and the partials of the scale term; the
+    streaming form also holds the scaled table), negative, NaN or infinite targets
+    are rejected; luna_featmap and luna_attn_decode do not support it (all checked
+    before any device call)."""
     lib = L._lib
     for bad in (-0.1, float("nan"), float("inf")):
         with pytest.raises(L.LunaError) as e:
@@ -162,9 +163,10 @@ def test_channel_rms_descriptor(L):
     for bwd in (False, True):
         assert L.luna_workspace_size(ad, pd1, bwd) > L.luna_workspace_size(ad, pd0, bwd)
     assert L.luna_state_size(ad, pd1) == L.luna_state_size(ad, pd0)
-    with pytest.raises(L.LunaError) as e:
-        L.luna_workspace_size(L.attn_desc(2, 4, 1024, 128, 128, True), pd1, True)
-    assert e.value.status == 2
+    pdc0, pdc1 = L.phi_desc(16, 8, 64), L.phi_desc(16, 8, 64, ch_rms_target=0.1)
+    adc = L.attn_desc(2, 4, 1024, 128, 128, True)
+    for bwd in (False, True):
+        assert L.luna_workspace_size(adc, pdc1, bwd) > L.luna_workspace_size(adc, pdc0, bwd)
     assert lib.luna_featmap(ctypes.byref(pd1), 32, None, None, L.LUNA_F32, 1, None, None) == 2
     dec = L.attn_desc(2, 4, 1, 32, 32, True)
     assert lib.luna_attn_decode(ctypes.byref(dec), ctypes.byref(pd1), None, None, None, None, None, None, 0, None, 0,

@@ -45,14 +45,13 @@ def test_reference_arm_decode():
 
 def test_channel_rms_option():
     """--ch-rms-target runs the normalised feature map and names it in the workload;
-    the streaming-form workloads reject it before any work."""
+    the decode workload rejects it before any work."""
     d = _run("--impl", "reference", "--workload", "tiny_f32", "--steps", "1", "--warmup", "0", "--ch-rms-target",
              "0.1")
     assert d["value"] > 0 and "channel RMS normalisation target 0.1" in d["config"]["workload"]
-    for wl in ("causal_long", "decode"):
-        r = subprocess.run([sys.executable, os.path.join(ROOT, "bench.py"), "--workload", wl, "--ch-rms-target", "0.1"],
-                           cwd=ROOT, capture_output=True, text=True, timeout=120)
-        assert r.returncode == 2 and "non-causal form only" in r.stderr
+    r = subprocess.run([sys.executable, os.path.join(ROOT, "bench.py"), "--workload", "decode", "--ch-rms-target",
+                        "0.1"], cwd=ROOT, capture_output=True, text=True, timeout=120)
+    assert r.returncode == 2 and "decode step" in r.stderr
 
 
 def test_algorithmic_bytes_by_hand():
