@@ -586,15 +586,16 @@ def oracle_run(w, units: int, ch_rms_target: float = 0.0, rows: int | None = Non
     ln = None
     if w.len_range is not None:
         ln = synth.randint(w.seed, "attn.lengths", (w.B,), w.len_range[0], w.len_range[1]).astype(np.int32)
-    # (units, 1, w.n, d) has the same flat order as the first `units` heads of (B, H, n, d)
-    shape = (units, 1, w.n, w.d)
-    Q = synth.IOTensor(synth.normal(w.seed, "attn.Q", shape) * w.qkv_scale, w.io).value[:, :, :n]
-    K = synth.IOTensor(synth.normal(w.seed, "attn.K", shape) * w.qkv_scale, w.io).value[:, :, :n]
-    V = synth.IOTensor(synth.normal(w.seed, "attn.V", (units, 1, w.n, w.dv)) * w.qkv_scale, w.io).value[:, :, :n]
-    dO = (synth.IOTensor(synth.normal(w.seed, "attn.dO", (units, 1, w.n, w.dv)), w.io).value[:, :, :n]
-          if w.backward else None)
-    Q, K, V = (np.ascontiguousarray(t) for t in (Q, K, V))
-    dO = None if dO is None else np.ascontiguousarray(dO)
+    # the first `units` heads of (B, H, n, d) in flat order, their first n tokens drawn directly
+    def draw(name, width, scale):
+        idx = ((np.arange(units)[:, None, None] * w.n + np.arange(n)[None, :, None]) * width
+               + np.arange(width)[None, None, :]).ravel()
+        x = synth.normal_at(w.seed, name, idx).reshape(units, 1, n, width) * scale
+        return np.ascontiguousarray(synth.IOTensor(x, w.io).value)
+
+    Q, K = draw("attn.Q", w.d, w.qkv_scale), draw("attn.K", w.d, w.qkv_scale)
+    V = draw("attn.V", w.dv, w.qkv_scale)
+    dO = draw("attn.dO", w.dv, 1.0) if w.backward else None
     lengths = None if ln is None else np.array([min(n, ln[(u // w.H) % w.B]) for u in range(units)], dtype=np.int32)
     p = oracle.PhiParams(synth.phi_params(w.seed, w.d, w.M, w.L, w.hidden), ch_rms_target)
     t0 = time.perf_counter()

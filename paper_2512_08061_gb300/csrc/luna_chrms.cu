@@ -413,7 +413,8 @@ cudaError_t launch_chrms_stats(const AttnArgs &a, luna_dtype io, cudaStream_t s)
 }
 
 cudaError_t launch_chrms_scale_state(const AttnArgs &a, cudaStream_t s) {
-    if (!a.ch_sigma) return cudaSuccess;
+    // non-causal only: the streaming form has no S_fin, z_fin (its sigma sits in the scaled table)
+    if (!a.ch_sigma || a.ch_causal) return cudaSuccess;
     const int64_t BH = (int64_t)a.B * a.H;
     LUNA_LAUNCH("chrms_scale", k_chrms_scale_rows, blocks_for(BH * a.D * a.dv), 256, 0, s, a.S_fin, a.z_fin,
                 a.ch_sigma, BH, a.D, a.L, a.dv);
@@ -421,7 +422,7 @@ cudaError_t launch_chrms_scale_state(const AttnArgs &a, cudaStream_t s) {
 }
 
 cudaError_t launch_chrms_dstate(const AttnArgs &a, cudaStream_t s) {
-    if (!a.ch_sigma) return cudaSuccess;
+    if (!a.ch_sigma || a.ch_causal) return cudaSuccess;  // non-causal only, as above
     LUNA_LAUNCH("chrms_dstate", k_chrms_dstate, a.B * a.H, 128, 0, s, a, a.ch_sigma, a.ch_T);
     return cudaGetLastError();
 }

@@ -121,7 +121,7 @@ __device__ __forceinline__ uint4 pack8(const float (&y)[8]) {
 // interval j, the sum of g (c = 0) and of g * u (c = 1) over the samples u that
 // fall into interval j, g = dLoss/dphi on an active output.
 //
-// Shared-memory fp32 atomics are compare-and-swap loops; integer atomics are
+// Shared-memory fp32 atomics are compare-and-swap loops; int32 atomics are
 // native and about five times faster.  So the bins hold fixed-point int32 sums
 // over groups of hist_tiles() tiles, quantised with power-of-two scales 2^e such
 // that |q| < 2^kHistQBits for the scale's reference maxima of |g| and |g*u|; a
@@ -139,18 +139,9 @@ __device__ __forceinline__ uint4 pack8(const float (&y)[8]) {
 // the kernels' operands).  Large groups keep the block-wide flushes (a worker
 // barrier and a pass over every bin) rare.
 //
-// Layout in shared memory: one 64-bit word per channel and interval,
-// bins[l * kNint + j], that holds both sums: the sum of the quantised g in its
-// low 32 bits (two's complement) and the sum of the quantised g * u above them.
-// A sample adds q0 + 2^32 q1 with one 64-bit atomic instead of two 32-bit ones;
-// since every group keeps |sum q0| < 2^31, the low word read as a signed
-// integer is sum q0 exactly, and (word - sum q0) / 2^32 is sum q1.  The partial
-// in global memory is [interval][channel][g, g*u].
-__device__ __forceinline__ int hist_at(int l, int j) { return l * kNint + j; }
-
-__device__ __forceinline__ unsigned long long hist_pack(int q0, int q1) {
-    return (unsigned long long)((long long)q1 * 4294967296LL + (long long)q0);
-}
+// Layout in shared memory: bins[(c * 8 + l) * kNint + j] (lanes with different
+// intervals fall into different banks); the partial is [interval][channel][g, g*u].
+__device__ __forceinline__ int hist_at(int c, int l, int j) { return (c * 8 + l) * kNint + j; }
 
 constexpr int kHistQBits = 16;      // |q| < 2^16 per sample
 constexpr int kHistSamples = 16384;  // samples per group: 16384 * 2^16 = 2^30
@@ -219,13 +210,10 @@ __device__ __forceinline__ bool hist_open(HistAcc &h, float m0, float m1, float 
 __device__ __forceinline__ void hist_put(int *bins, float *part, int c, int l, int j, float v, float s) {
     if (v != 0.0f) {
         const float q = v * s;
-        if (fabsf(q) < (float)(1 << kHistQBits)) {
-            const int qi = __float2int_rn(q);
-            atomicAdd(reinterpret_cast<unsigned long long *>(bins) + hist_at(l, j),
-                      c == 0 ? hist_pack(qi, 0) : hist_pack(0, qi));
-        } else {
+        if (fabsf(q) < (float)(1 << kHistQBits))
+            atomicAdd(bins + hist_at(c, l, j), __float2int_rn(q));
+        else
             atomicAdd(part + ((j * 8 + l) << 1) + c, v);
-        }
     }
 }
 
@@ -274,11 +262,12 @@ __device__ __forceinline__ void hist_add(int *bins, float *part, HistAcc &h, con
         h.m1 = finite_max(h.m1, mgu);
         if (mg * s0 < kQ && mgu * s1 < kQ && du[q] - du[q] == 0.0f) {
             const float us1 = u[q] * s1;
-            unsigned long long *b64 = reinterpret_cast<unsigned long long *>(bins) + j[q];
 #pragma unroll
             for (int l = 0; l < 8; ++l)
-                if (g[q][l] != 0.0f)
-                    atomicAdd(b64 + l * kNint, hist_pack(round_scaled(g[q][l], s0), round_scaled(g[q][l], us1)));
+                if (g[q][l] != 0.0f) {
+                    atomicAdd(bins + hist_at(0, l, j[q]), round_scaled(g[q][l], s0));
+                    atomicAdd(bins + hist_at(1, l, j[q]), round_scaled(g[q][l], us1));
+                }
         } else {
             hist_add_slow(bins, part, j[q], u[q], s0, s1, g[q][0], g[q][1], g[q][2], g[q][3], g[q][4], g[q][5],
                           g[q][6], g[q][7]);
@@ -287,24 +276,19 @@ __device__ __forceinline__ void hist_add(int *bins, float *part, HistAcc &h, con
 }
 
 // Closes the group: after a worker barrier (every atomic done), adds the bins,
-// rescaled, into the partial and clears them (thread t handles words t,
+// rescaled, into the partial and clears them (thread t handles entries t,
 // t + kBWorkers, ...); with `next`, the group's block-wide maxima then give the
 // scales of the next group (unchanged if it was all zero).
 __device__ __forceinline__ void hist_close(int *bins, float *part, int nint, HistAcc &h, int t, bool next,
                                            float *smax, int warp, int lane) {
     named_sync<kBWorkers>(1);
     const float inv0 = pow2f(-h.e0), inv1 = pow2f(-h.e1);
-    unsigned long long *b64 = reinterpret_cast<unsigned long long *>(bins);
 #pragma unroll 4
-    for (int e = t; e < nint * 8; e += kBWorkers) {  // word e: channel e % 8, interval e / 8
-        const int at = hist_at(e & 7, e >> 3);
-        const unsigned long long w = b64[at];
-        b64[at] = 0ull;
-        const int q0 = (int)(unsigned)(w & 0xffffffffull);                      // sum of q0, exactly
-        const long long q1 = ((long long)w - (long long)q0) / 4294967296LL;     // sum of q1, exactly
-        float *p = part + 2 * e;  // [interval][channel][g, g*u]; L2 copy: fp32 atomics went there
-        p[0] = __ldcg(p) + (float)q0 * inv0;
-        p[1] = __ldcg(p + 1) + (float)q1 * inv1;
+    for (int e = t; e < nint * 16; e += kBWorkers) {
+        const int at = hist_at(e & 1, (e >> 1) & 7, e >> 4);
+        const int v = bins[at];
+        bins[at] = 0;
+        part[e] = __ldcg(part + e) + (float)v * ((e & 1) ? inv1 : inv0);  // L2 copy: fp32 atomics went there
     }
     if (next) hist_scales(h, h.m0, h.m1, smax, warp, lane);
     h.tiles = 0;

@@ -81,6 +81,22 @@ def normal(seed: int, name: str, shape) -> np.ndarray:
     return z[:count].reshape(shape)
 
 
+def normal_at(seed: int, name: str, idx) -> np.ndarray:
+    """Elements idx (flat indices) of the stream that `normal` draws, without drawing the others: the
+    generator is counter-based, so element e takes uniforms 2*(e // 2) and 2*(e // 2) + 1 of its
+    stream.  Equal, bit for bit, to normal(seed, name, shape).ravel()[idx]."""
+    idx = np.asarray(idx, dtype=np.int64)
+    key = stream_key(seed, name)
+    pair = (idx // 2).astype(np.uint64)
+    with np.errstate(over="ignore"):
+        a = _mix(key + (np.uint64(2) * pair + np.uint64(1)) * GOLDEN)
+        b = _mix(key + (np.uint64(2) * pair + np.uint64(2)) * GOLDEN)
+    u1 = 1.0 - (a >> np.uint64(11)).astype(np.float64) * (2.0 ** -53)
+    u2 = (b >> np.uint64(11)).astype(np.float64) * (2.0 ** -53)
+    r = np.sqrt(-2.0 * np.log(u1))
+    return np.where(idx % 2 == 0, r * np.cos(2.0 * math.pi * u2), r * np.sin(2.0 * math.pi * u2))
+
+
 def randint(seed: int, name: str, shape, lo: int, hi: int) -> np.ndarray:
     """Integers uniform on [lo, hi] inclusive."""
     count = int(np.prod(shape)) if len(shape) else 1

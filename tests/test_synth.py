@@ -88,3 +88,13 @@ def test_attn_inputs_shapes_and_lengths():
     # bf16 values: the fp64 value of every element has at most 8 significant bits
     v = inp["Q"].value
     assert np.array_equal(v, synth.bf16_bits_to_f64(synth.f32_to_bf16_bits(v.astype(np.float32))))
+
+
+def test_normal_at_equals_the_full_draw():
+    """Drawing chosen elements of a normal stream gives the same values, bit for bit, as drawing the
+    whole tensor and indexing it (odd and even positions, both ends)."""
+    full = synth.normal(9, "na.X", (7, 13, 5)).ravel()
+    idx = np.array([0, 1, 2, 3, 64, 65, 299, 453, 454, full.size - 1])
+    assert np.array_equal(synth.normal_at(9, "na.X", idx), full[idx])
+    rows = (np.arange(3)[:, None] * 65 + np.arange(5)[None, :]).ravel()
+    assert np.array_equal(synth.normal_at(9, "na.X", rows), full[rows])
