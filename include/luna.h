@@ -128,8 +128,11 @@ typedef struct {
 
 /* Problem description (Sec. 3.1: Q, K in R^{n x d}; Sec. 4: values of width d_v).
  * Supported: 1 <= d, dv <= 128; B, H, n >= 0 (an empty problem is a no-op).
- * causal = 1 selects the streaming form (sums over j <= i).  chunk is the
- * causal chunk length (0 selects 64; otherwise 16..128, multiple of 16).
+ * causal = 1 selects the streaming form (sums over j <= i).  chunk (0, or
+ * 16..128 in steps of 16, else LUNA_ERR_INVALID_ARG) is accepted for the
+ * interface and otherwise not used: the kernels choose their own tiles (128
+ * rows in the tensor-core streaming forward, 64 in its backward, 16 in the
+ * generic kernels), and results do not depend on it beyond rounding order.
  * eps >= 0 guards the row normaliser: O_i = num_i / (den_i + eps); a row
  * whose guarded normaliser is exactly 0 produces O_i = 0 and zero gradients. */
 typedef struct {
