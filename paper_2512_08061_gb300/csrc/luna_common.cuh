@@ -4,6 +4,7 @@
 #include <cuda_bf16.h>
 #include <cuda_runtime.h>
 #include <stdint.h>
+#include <string.h>
 
 #include "luna.h"
 
@@ -16,7 +17,48 @@ constexpr int kMaxFeat = 128;   // max D = M * L
 constexpr int kMaxL = 16;
 constexpr int kMaxHidden = 128;
 constexpr int kMaxUnits = 512;  // max L * hidden
-constexpr int kEytzinger = 1024; // slots of the breadth-first kink tree (1023 nodes, P <= 512)
+constexpr int kEytzinger = 1024; // floats of the interval-search block (kept at the size of a 1023-node kink tree)
+
+// Interval search block (4096 bytes, staged whole into shared memory by the tensor-core kernels):
+//   floats [0, kSearchT)        the sorted kinks, +inf from P on (at least 16 +inf sentinels)
+//   uint16 [kBuckets] after it   for each bucket of u, the number of kinks strictly below the bucket's
+//                                smallest value
+// A bucket is a range of an order-preserving integer key of u: 32 buckets per binade for
+// 2^-7 <= |u| < 2^8, one bucket for |u| < 2^-7, and the two outer buckets extended to +-inf.  The
+// interval of u (the number of kinks strictly below it) is the bucket's start plus a scan over the
+// few kinks between the bucket's lower end and u; the sentinels end every scan.
+constexpr int kSearchT = 528;
+constexpr int kBktPos0 = 3840;                 // key >> 18 of 2^-7 (biased exponent 120, 32 per binade)
+constexpr int kBktSide = 480;                  // buckets per side: 15 binades x 32
+constexpr int kBktMid = kBktSide;              // the bucket of |u| < 2^-7
+constexpr int kBktNeg0 = -kBktPos0 - kBktSide; // key >> 18 of the first negative bucket after the outer one
+constexpr int kBuckets = 2 * kBktSide + 1;
+static_assert(kSearchT * 4 + kBuckets * 2 <= kEytzinger * 4, "search block size");
+
+// Order-preserving integer key of a float (a < b iff key(a) < key(b) for non-NaN floats other than -0/+0).
+__host__ __device__ __forceinline__ int float_key(float u) {
+#ifdef __CUDA_ARCH__
+    const int bits = __float_as_int(u);
+#else
+    int bits;
+    memcpy(&bits, &u, 4);
+#endif
+    return bits ^ ((bits >> 31) & 0x7fffffff);
+}
+
+__host__ __device__ __forceinline__ int bucket_of(float u) {
+    const int kk = float_key(u) >> 18;
+    if (kk >= kBktPos0) return kBktMid + 1 + (kk - kBktPos0 < kBktSide - 1 ? kk - kBktPos0 : kBktSide - 1);
+    if (kk <= -kBktPos0 - 1) return kk - kBktNeg0 > 0 ? kk - kBktNeg0 : 0;
+    return kBktMid;
+}
+
+// Smallest key of bucket b (b = 0: no lower end).
+__host__ __device__ __forceinline__ int bucket_lo_key(int b) {
+    if (b <= kBktMid - 1) return (b + kBktNeg0) * (1 << 18);
+    if (b == kBktMid) return -kBktPos0 * (1 << 18);  // the first key above the negative buckets
+    return (kBktPos0 + (b - kBktMid - 1)) * (1 << 18);
+}
 
 __host__ __device__ inline int next_pow2(int x) {
     int p = 1;
@@ -28,8 +70,8 @@ __host__ __device__ inline int64_t align256(int64_t x) { return (x + 255) & ~int
 
 // Layout of the prepared feature-map table (byte offsets from its start).
 //   T      [Ppad]          sorted fp32 kink thresholds of all hidden units (+inf padding)
-//   Te     [1024]          the same thresholds in Eytzinger (breadth-first) order of a
-//                          complete 1023-node search tree, index 0 unused, +inf padding
+//   Te     [1024]          the interval search block (4096 bytes): the sorted kinks with +inf sentinels
+//                          and the bucket starts (see kSearchT, bucket_of)
 //   AB     [nint][L][2]    per merged interval j and channel l: (alpha, beta) / sqrt(M)
 //   W      [M][d], b [M]   projection copy
 //   rank   [P]             position of unit (l,k) (shared MLP: unit k) in the sorted kink list
@@ -99,6 +141,13 @@ __device__ __forceinline__ int interval_of(const float *T, int Ppad, float u) {
     for (int s = Ppad >> 1; s > 0; s >>= 1) pos += (T[pos + s - 1] < u) ? s : 0;
     pos += (T[pos] < u) ? 1 : 0;
     return pos;
+}
+
+// Interval of u from the search block (sT: its kinks, sB: its bucket starts).
+__device__ __forceinline__ int interval_bucketed(const float *sT, const unsigned short *sB, float u) {
+    int j = sB[bucket_of(u)];
+    while (sT[j] < u) ++j;
+    return j;
 }
 
 __device__ __forceinline__ int head_length(const int32_t *lengths, int b, int n) {

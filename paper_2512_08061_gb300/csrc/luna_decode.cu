@@ -9,7 +9,7 @@
 // fp32 state (read, update, write back) with the output accumulated on the
 // way: the state traffic bounds the step, so it is CUDA-core code that reads
 // and writes every state element once, in 16-byte accesses along the value
-// columns.  The kink tree is staged in shared memory so that the searches do
+// columns.  The interval search block is staged in shared memory so that the searches do
 // not wait on ten dependent global loads.
 #include <math.h>
 
@@ -67,15 +67,13 @@ __global__ void __launch_bounds__(kDecThreads) k_decode(DecodeArgs a) {
         if (lane == 0) su[side][m] = acc + bias[m];
     }
     __syncthreads();
-    // phi: interval of u in the breadth-first kink tree, then relu(alpha u + beta) per channel
+    // phi: interval of u from the bucketed search block, then max(alpha u + beta, floor) per channel
     const float2 *AB = reinterpret_cast<const float2 *>(table + a.lay.off_AB);
     const float fl = channel_floor(a.lay);
     for (int p = tid; p < 2 * M; p += blockDim.x) {
         const int side = p / M, m = p % M;
         const float u = su[side][m];
-        int node = 1;
-        for (int lvl = 0; lvl < 10; ++lvl) node = 2 * node + (sTe[node] < u ? 1 : 0);
-        const int j = node - kEytzinger;
+        const int j = interval_bucketed(sTe, reinterpret_cast<const unsigned short *>(sTe + kSearchT), u);
         if (L == 8) {  // the (alpha, beta) of the 8 channels as four 16-byte loads in flight
             const float4 *ab4 = reinterpret_cast<const float4 *>(AB + (size_t)j * 8);
             float4 w[4];

@@ -43,7 +43,7 @@ __device__ float down_threshold(float w, float c) {
 // per thread: warp shuffles for partners within a warp, shared memory across
 // warps; a stable total order), then computes its slice of alpha and beta,
 // eight threads per (interval, channel) entry; block 0 also writes the sorted
-// and breadth-first kink lists, each unit's rank and active side, and the
+// kink list and interval search block, each unit's rank and active side, and the
 // parameter copies.
 constexpr int kPrepThreads = kMaxUnits;                       // one thread per (padded) unit
 constexpr int kPrepSplit = 8;                                 // threads per (interval, channel) entry
@@ -119,18 +119,24 @@ __global__ void __launch_bounds__(kPrepThreads) k_phi_prepare(luna_phi_params pr
             reinterpret_cast<float *>(table + lay.off_b1)[k] = b1t[tpos];
         }
         for (int e = tid; e < L * hid; e += nt) reinterpret_cast<float *>(table + lay.off_w2)[e] = prm.w2[e];
-        // breadth-first (Eytzinger) copy: node e at depth d, position p in its level
-        // holds the in-order element (2p+1) * 2^(9-d) - 1
-        float *Te = reinterpret_cast<float *>(table + lay.off_Te);
-        for (int e = tid; e < kEytzinger; e += nt) {
-            float v = INFINITY;
-            if (e > 0) {
-                const int d = 31 - __clz(e);
-                const int idx = ((2 * (e - (1 << d)) + 1) << (9 - d)) - 1;
-                if (idx < P) v = sk[idx];
+        // interval search block: the sorted kinks with +inf sentinels, then every bucket's start (the
+        // number of kinks strictly below the bucket's smallest value, by binary search over the kinks)
+        float *Ts = reinterpret_cast<float *>(table + lay.off_Te);
+        for (int e = tid; e < kSearchT; e += nt) Ts[e] = e < P ? sk[e] : INFINITY;
+        unsigned short *Bk = reinterpret_cast<unsigned short *>(Ts + kSearchT);
+        for (int bk = tid; bk < kBuckets; bk += nt) {
+            int cnt = 0;
+            if (bk > 0) {
+                const int key = bucket_lo_key(bk);
+                const float lo = __int_as_float(key ^ ((key >> 31) & 0x7fffffff));
+                for (int step = N >> 1; step > 0; step >>= 1)  // N: power of two, +inf beyond P
+                    if (sk[cnt + step - 1] < lo) cnt += step;
+                if (sk[cnt] < lo) ++cnt;
             }
-            Te[e] = v;
+            Bk[bk] = (unsigned short)cnt;
         }
+        for (int e = kSearchT * 2 + kBuckets + tid; e < kEytzinger * 2; e += nt)
+            reinterpret_cast<unsigned short *>(Ts)[e] = 0;  // the block's unused tail
         float *W = reinterpret_cast<float *>(table + lay.off_W);
         for (int e = tid; e < lay.M * lay.d; e += nt) W[e] = prm.W[e];
         for (int e = tid; e < lay.M; e += nt) reinterpret_cast<float *>(table + lay.off_b)[e] = prm.b[e];

@@ -23,11 +23,14 @@ template <typename IO>
 __global__ void __launch_bounds__(kThreads) k_featmap(TableLayout lay, const char *table, const IO *X, int64_t rows,
                                                       float *Phi) {
     extern __shared__ __align__(16) float smem[];
+    __shared__ __align__(16) float sS[kEytzinger];  // the interval search block (the tensor-core kernels' lookup)
     Carve cv{smem};
     SmemPhi s = carve_phi(cv, lay);
     if (!carve_fits(cv, smem)) return;
     load_phi(s, lay, table);
+    for (int e = threadIdx.x; e < kEytzinger; e += blockDim.x) sS[e] = reinterpret_cast<const float *>(table + lay.off_Te)[e];
     __syncthreads();
+    const unsigned short *sB = reinterpret_cast<const unsigned short *>(sS + kSearchT);
     const int M = lay.M, L = lay.L, d = lay.d, D = lay.D;
     for (int64_t e = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; e < rows * M; e += (int64_t)gridDim.x * blockDim.x) {
         const int64_t r = e / M;
@@ -36,7 +39,7 @@ __global__ void __launch_bounds__(kThreads) k_featmap(TableLayout lay, const cha
         const float *w = s.W + i * d;
         float u = s.b[i];
         for (int c = 0; c < d; ++c) u = fmaf(w[c], io_load(x + c), u);
-        const int j = interval_of(s.T, lay.Ppad, u);
+        const int j = interval_bucketed(sS, sB, u);
         const float *ab = s.AB + j * L * 2;
         float *out = Phi + r * D + i * L;
         for (int l = 0; l < L; ++l) out[l] = fmaxf(fmaf(ab[2 * l], u, ab[2 * l + 1]), channel_floor(lay));

@@ -12,8 +12,8 @@
 //
 // Forward key pass per tile (Sec. 4, S_KV and S_K1):
 //   MMA  U = K [W_hi; W_lo]^T                      (projections -> TMEM)
-//   workers: u = U_hi + U_lo + b; interval j of u in the breadth-first kink
-//            tree; phi = relu(alpha_j u + beta_j) for the 8 channels, written
+//   workers: u = U_hi + U_lo + b; interval j of u from the bucketed search
+//            block; phi = relu(alpha_j u + beta_j) for the 8 channels, written
 //            as bf16 hi and lo tiles; z += phi in fp32 registers
 //   MMA  S += [phi_hi | phi_lo]^T V                 (MN-major operands)
 // Forward query pass (Eq. kernel-attn):
@@ -81,7 +81,7 @@ struct Cfg {
 
 // Worker: phi for projections [Q*PP, Q*PP+PP) of row r from the projection
 // columns in TMEM.  The PP interval searches run interleaved over the
-// breadth-first kink tree (count of thresholds below u = final node - 1024).
+// bucketed search block (j = the number of kinks strictly below u).
 // Writes the bf16 chunks of the phi tile (and, if plo is not null, the bf16
 // residual phi - bf16(phi) into a second tile), zeros for rows that are not
 // valid.  Optionally adds phi into zacc (fp32 feature sums) and accumulates the
@@ -107,22 +107,16 @@ __device__ __forceinline__ void phi_row_quarter(int Q, uint32_t tmem_u_row, cons
 #pragma unroll
         for (int q = 0; q < PP; ++q) u[q] = __uint_as_float(xh[q]) + __uint_as_float(xl[q]);
     }
+#pragma unroll
+    for (int q = 0; q < PP; ++q) u[q] += sbias[Q * PP + q];
     int node[PP];
-#pragma unroll
-    for (int q = 0; q < PP; ++q) {
-        u[q] += sbias[Q * PP + q];
-        node[q] = 1;
-    }
-#pragma unroll
-    for (int lvl = 0; lvl < 10; ++lvl)
-#pragma unroll
-        for (int q = 0; q < PP; ++q) node[q] = 2 * node[q] + (sTe[node[q]] < u[q] ? 1 : 0);
+    search_bucketed<PP>(sTe, u, node);
 #pragma unroll
     for (int q = 0; q < PP; ++q) {
         const int i = Q * PP + q;
         uint4 ph = make_uint4(0u, 0u, 0u, 0u), pl = make_uint4(0u, 0u, 0u, 0u);
         if (valid) {
-            const int j = node[q] - kEytzinger;
+            const int j = node[q];
             const float4 *ab = reinterpret_cast<const float4 *>(sAB);
             float y[8];
 #pragma unroll

@@ -74,18 +74,10 @@ __device__ void stage_rows_per_column(const float *Sg, uint8_t *op, int tid, int
     }
 }
 
-// Interval search for the PP projections of this thread (breadth-first kink tree).
+// Interval search for the PP projections of this thread (bucketed search block).
 template <int PP>
 __device__ __forceinline__ void search(const float *sTe, const float (&u)[PP], int (&j)[PP]) {
-    int node[PP];
-#pragma unroll
-    for (int q = 0; q < PP; ++q) node[q] = 1;
-#pragma unroll
-    for (int lvl = 0; lvl < 10; ++lvl)
-#pragma unroll
-        for (int q = 0; q < PP; ++q) node[q] = 2 * node[q] + (sTe[node[q]] < u[q] ? 1 : 0);
-#pragma unroll
-    for (int q = 0; q < PP; ++q) j[q] = node[q] - kEytzinger;
+    search_bucketed<PP>(sTe, u, j);
 }
 
 // alpha, beta of the 8 channels on interval j (swizzled table) and phi = max(alpha u + beta, fl): the

@@ -83,17 +83,12 @@ __device__ __forceinline__ float phi_quarter_qk(uint32_t uq, uint32_t uk, int Qd
         }
     }
     int node[2 * PP];
-#pragma unroll
-    for (int q = 0; q < 2 * PP; ++q) node[q] = 1;
-#pragma unroll
-    for (int lvl = 0; lvl < 10; ++lvl)
-#pragma unroll
-        for (int q = 0; q < 2 * PP; ++q) node[q] = 2 * node[q] + (sTe[node[q]] < u[q] ? 1 : 0);
+    search_bucketed<2 * PP>(sTe, u, node);
     float dot = 0.0f;
     const float4 *ab = reinterpret_cast<const float4 *>(sAB);
 #pragma unroll
     for (int q = 0; q < 2 * PP; ++q) {
-        const int i = Qd * PP + (q % PP), j = node[q] - kEytzinger;
+        const int i = Qd * PP + (q % PP), j = node[q];
         uint4 w = make_uint4(0u, 0u, 0u, 0u);
         if (valid) {
             float y[8];

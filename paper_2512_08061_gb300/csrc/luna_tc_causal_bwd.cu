@@ -412,17 +412,14 @@ __global__ void __launch_bounds__(kCBThreads, 1)
                     u[1] = uu[0][1] + uu[1][1] + sbias[m0 + 1];
                     u[2] = uu[2][0] + uu[3][0] + sbias[m0];
                     u[3] = uu[2][1] + uu[3][1] + sbias[m0 + 1];
-                    int node[4] = {1, 1, 1, 1};
-#pragma unroll
-                    for (int lvl = 0; lvl < 10; ++lvl)
-#pragma unroll
-                        for (int p = 0; p < 4; ++p) node[p] = 2 * node[p] + (sTe[node[p]] < u[p] ? 1 : 0);
+                    int node[4];
+                    search_bucketed<4>(sTe, u, node);
                     const float4 *ab = reinterpret_cast<const float4 *>(sAB);
                     const float fl = channel_floor(a.lay);
                     float yk[16];
 #pragma unroll
                     for (int p = 0; p < 4; ++p) {
-                        const int jv = node[p] - kEytzinger;
+                        const int jv = node[p];
 #pragma unroll
                         for (int k = 0; k < 4; ++k) {
                             const float4 w = ab[ab_slot(jv, k)];

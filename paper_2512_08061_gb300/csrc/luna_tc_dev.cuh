@@ -20,6 +20,22 @@ constexpr int kPpad = 512;   // merged kink list (L * hidden <= 512, L = 8)
 constexpr int kNint = 513;   // intervals
 constexpr uint32_t kTableBytes = (kEytzinger + kNint * 16 + 32) * 4;
 
+// Intervals of the PP values u (the number of kinks strictly below each) from the interval search block
+// in shared memory (sS: its sorted kinks, then its bucket starts): the bucket starts of all PP values,
+// one scan step for all of them (most buckets hold at most one kink below u), then the rest of each scan,
+// rarely more than one step more.  Exact for every non-NaN u (the sentinels end each scan).
+template <int PP>
+__device__ __forceinline__ void search_bucketed(const float *sS, const float (&u)[PP], int (&j)[PP]) {
+    const unsigned short *sB = reinterpret_cast<const unsigned short *>(sS + kSearchT);
+#pragma unroll
+    for (int q = 0; q < PP; ++q) j[q] = sB[bucket_of(u[q])];
+#pragma unroll
+    for (int q = 0; q < PP; ++q) j[q] += sS[j[q]] < u[q] ? 1 : 0;
+#pragma unroll
+    for (int q = 0; q < PP; ++q)
+        while (sS[j[q]] < u[q]) ++j[q];
+}
+
 // First 1024-byte boundary at or after p (a shared-memory array), formed by
 // pointer arithmetic on p so that the compiler still sees a shared address.
 __device__ __forceinline__ uint8_t *align1024(uint8_t *p) {
