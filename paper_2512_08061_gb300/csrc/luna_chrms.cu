@@ -30,11 +30,13 @@
 // kernel value, and the streaming kernels run unchanged.  T_l is the sum over the
 // query samples of phi^ . dLoss/dphi^ on channel l (equal to the sum over the
 // normalised features, and the same for the key side, since the loss depends on
-// s^q_l and s^k_l only through their product), accumulated by the chain-rule
-// kernel of the queries.  The kappa term runs on the scaled table with kappa_l /
-// sigma_l (its dU is then that of the unscaled map), and before the channel-MLP
-// gradients the reduced interval histogram of channel l, a sum of dLoss/dphi^,
-// is multiplied by sqrt(sigma_l) to give sums of dLoss/dphi.
+// s^q_l and s^k_l only through their product): the tensor-core query sweep sums
+// it where it forms dphi^(q), so kappa is known before either chain rule, which
+// adds M (kappa_l / sigma_l) phi^ to dLoss/dphi^ (its dU is then that of the
+// unscaled map's scale term); the generic path sums T in its query-side kernel
+// and runs the kappa pass on the scaled table with kappa_l / sigma_l.  Before
+// the channel-MLP gradients the reduced interval histogram of channel l, a sum
+// of dLoss/dphi^, is multiplied by sqrt(sigma_l) to give sums of dLoss/dphi.
 #include <math.h>
 
 #include "luna_prof.cuh"
@@ -251,8 +253,8 @@ __global__ void __launch_bounds__(kKWarps * 32) k_chrms_kterm(AttnArgs a, const 
     float *sAB = sT + r4(P);
     float *sW = sAB + r4(NH);
     float *sb = sW + r4(M * d);
-    double *sdW = reinterpret_cast<double *>(sb + r4(M));       // fp64 block sums of dW, db
-    double *sdb = sdW + r4(M * d);
+    GP *sdW = reinterpret_cast<GP *>(sb + r4(M));  // block sums of dW, db in the partials' type
+    GP *sdb = sdW + r4(M * d);
     float *sk = reinterpret_cast<float *>(sdb + r4(M));
     float *sx = sk + r4(kMaxL) + warp * (r4(32 * dp) + r4(32 * mp));
     float *sdu = sx + r4(32 * dp);
@@ -267,8 +269,8 @@ __global__ void __launch_bounds__(kKWarps * 32) k_chrms_kterm(AttnArgs a, const 
         const float *b = reinterpret_cast<const float *>(a.table + lay.off_b);
         for (int e = threadIdx.x; e < P; e += blockDim.x) sT[e] = T[e];
         for (int e = threadIdx.x; e < NH; e += blockDim.x) { sAB[e] = AB[e]; ghist[e] = (GP)0; }
-        for (int e = threadIdx.x; e < M * d; e += blockDim.x) { sW[e] = W[e]; sdW[e] = 0.0; }
-        for (int e = threadIdx.x; e < M; e += blockDim.x) { sb[e] = b[e]; sdb[e] = 0.0; }
+        for (int e = threadIdx.x; e < M * d; e += blockDim.x) { sW[e] = W[e]; sdW[e] = (GP)0; }
+        for (int e = threadIdx.x; e < M; e += blockDim.x) { sb[e] = b[e]; sdb[e] = (GP)0; }
         if ((int)threadIdx.x < L) sk[threadIdx.x] = kappa[side * kMaxL + threadIdx.x] * (float)M;
     }
     __syncthreads();
@@ -326,14 +328,14 @@ __global__ void __launch_bounds__(kKWarps * 32) k_chrms_kterm(AttnArgs a, const 
                 io_store(dX + (row0 + r) * d + c, cur[r] + acc);
             }
             for (int i = 0; i < M; ++i) {
-                double acc = 0.0;
-                for (int r = 0; r < 32; ++r) acc = fma((double)sdu[r * mp + i], (double)sx[r * dp + c], acc);
+                GP acc = (GP)0;
+                for (int r = 0; r < 32; ++r) acc = fma((GP)sdu[r * mp + i], (GP)sx[r * dp + c], acc);
                 atomicAdd(sdW + i * d + c, acc);
             }
         }
         if (lane < M) {
-            double acc = 0.0;
-            for (int r = 0; r < 32; ++r) acc += (double)sdu[r * mp + lane];
+            GP acc = (GP)0;
+            for (int r = 0; r < 32; ++r) acc += (GP)sdu[r * mp + lane];
             atomicAdd(sdb + lane, acc);
         }
         __syncwarp();
@@ -363,9 +365,10 @@ __global__ void k_chrms_scale_hist(double *gsum, TableLayout lay, const float *s
 size_t smem_stats(const AttnArgs &a) {
     return (size_t)(r4(a.lay.Ppad) + r4(a.lay.nint * a.lay.L * 2) + r4(a.M * a.d) + r4(a.M) + kThreads) * 4;
 }
-size_t smem_kterm(const AttnArgs &a) {
+// shared memory of the scale-term pass with block sums of GP (gp_words: 4-byte words per GP)
+size_t smem_kterm(const AttnArgs &a, int gp_words = 2) {
     const int NH = a.lay.nint * a.L * 2;
-    return (size_t)(r4(a.lay.Ppad) + r4(NH) + 3 * r4(a.M * a.d) + 3 * r4(a.M) + r4(kMaxL) +
+    return (size_t)(r4(a.lay.Ppad) + r4(NH) + (1 + gp_words) * (r4(a.M * a.d) + r4(a.M)) + r4(kMaxL) +
                     kKWarps * (r4(32 * (a.d + 1)) + r4(32 * (a.M + 1)))) * 4;
 }
 
@@ -383,7 +386,7 @@ cudaError_t stats_impl(const AttnArgs &a, cudaStream_t s) {
 
 template <typename IO, typename GP>
 cudaError_t kterm_impl(const AttnArgs &a, GP *gpart, cudaStream_t s) {
-    const size_t sm = smem_kterm(a);
+    const size_t sm = smem_kterm(a, (int)(sizeof(GP) / 4));
     cudaError_t e = set_smem(k_chrms_kterm<IO, GP>, sm);
     if (e != cudaSuccess) return e;
     LUNA_LAUNCH("chrms_kterm", (k_chrms_kterm<IO, GP>), dim3(kChKBlocks, 2), kKWarps * 32, sm, s, a, a.ch_kappa,
@@ -440,14 +443,18 @@ cudaError_t launch_chrms_hist(const AttnArgs &a, cudaStream_t s) {
     return cudaGetLastError();
 }
 
-cudaError_t launch_chrms_backward(const AttnArgs &a, int main_parts, int *nparts, cudaStream_t s) {
-    *nparts = main_parts;
-    if (!a.ch_sigma) return cudaSuccess;
-    // non-causal: one T row per head; streaming form: one per block of the queries' chain-rule kernel
+cudaError_t launch_chrms_kappa(const AttnArgs &a, cudaStream_t s) {
+    // non-causal: one T row per head; streaming form: one per block of the kernel that summed T
     const int trows = a.ch_causal ? a.ch_T_rows : a.B * a.H;
     LUNA_LAUNCH("chrms_kappa", k_chrms_kappa, 1, kRed, 0, s, a, a.ch_T, trows, a.ch_target, a.ch_stat,
                 a.ch_causal ? a.ch_sigma : nullptr, a.ch_kappa);
-    cudaError_t e = cudaGetLastError();
+    return cudaGetLastError();
+}
+
+cudaError_t launch_chrms_backward(const AttnArgs &a, int main_parts, int *nparts, cudaStream_t s) {
+    *nparts = main_parts;
+    if (!a.ch_sigma) return cudaSuccess;
+    cudaError_t e = launch_chrms_kappa(a, s);
     if (e != cudaSuccess) return e;
     if (a.gpart64) {
         double *gpart = reinterpret_cast<double *>(a.gpart) + (size_t)main_parts * a.gsize;

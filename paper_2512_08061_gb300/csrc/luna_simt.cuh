@@ -109,6 +109,8 @@ cudaError_t launch_chrms_backward(const AttnArgs &a, int main_parts, int *nparts
 // streaming form: the table with channel l's coefficients times sqrt(sigma_l) into dst (a.lay.bytes), and
 // the reduced histogram's channel l times sqrt(sigma_l) (between the partial sum and the MLP gradients)
 cudaError_t launch_chrms_table(const AttnArgs &a, char *dst, cudaStream_t s);
+// kappa of both sides from the T rows (the streaming form on tensor cores folds it into its chain rule)
+cudaError_t launch_chrms_kappa(const AttnArgs &a, cudaStream_t s);
 cudaError_t launch_chrms_hist(const AttnArgs &a, cudaStream_t s);
 size_t chrms_max_smem(const AttnArgs &a);
 size_t causal_max_smem(const AttnArgs &a);

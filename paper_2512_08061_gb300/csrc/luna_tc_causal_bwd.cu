@@ -161,11 +161,11 @@ __device__ __forceinline__ uint4 pack8f(const float *y) {
 // ---------------------------------------------------------------------------
 // 1. query side
 
-template <class C>
+template <class C, bool TSUM>  // TSUM: also sum phi . dphi per channel into tpart (channel normalisation)
 __global__ void __launch_bounds__(kCBThreads, 1)
     k_tcc_query(const __grid_constant__ CUtensorMap mapQ, const __grid_constant__ CUtensorMap mapK,
                 const __grid_constant__ CUtensorMap mapV, const __grid_constant__ CUtensorMap mapdO, AttnArgs a,
-                int *status) {
+                double *tpart, int *status) {
     extern __shared__ uint8_t smem_raw[];
     uint8_t *sm = align1024(smem_raw);
     constexpr uint32_t T8 = C::T8, RT = C::RT;
@@ -354,6 +354,7 @@ __global__ void __launch_bounds__(kCBThreads, 1)
         const int part = 2 * cg + h;                  // this thread's 16 features / columns: 16 * part ..
         const uint32_t lq = (uint32_t)(32 * q) << 16;  // TMEM lane base of the warp
         bool failed = false;
+        float tq[TSUM ? 8 : 1] = {};  // channel normalisation: sums of phi . dphi per channel
         int g = 0;
         for (int item = it.begin; item < it.end; ++item) {
             const ItemRange ir = item_range(a, it, item);
@@ -524,6 +525,10 @@ __global__ void __launch_bounds__(kCBThreads, 1)
                         dq[k] = live ? (pv[k] + zi[k] * ndot) * inv : 0.0f;
                         pt[k] = phq[k] * inv;
                     }
+                    if constexpr (TSUM) {  // feature 16 * part + k is channel k % 8
+#pragma unroll
+                        for (int k = 0; k < 16; ++k) tq[k & 7] = fmaf(phq[k], dq[k], tq[k & 7]);
+                    }
                     if (valid) {  // workspace rows, 32-byte aligned
                         float4 *dst = reinterpret_cast<float4 *>(a.dphi + (hrow + row0 + r) * C::D + 16 * part);
 #pragma unroll
@@ -566,6 +571,15 @@ __global__ void __launch_bounds__(kCBThreads, 1)
                     mbar_arrive(sopready);
                 }
                 named_sync<kCBWorkers>(1);  // sz, and sred free for the next tile
+            }
+        }
+        if constexpr (TSUM) {  // the block's row of T: warp sums, then fp64 adds (the launch cleared the row)
+#pragma unroll
+            for (int l = 0; l < 8; ++l) {
+                float v = tq[l];
+#pragma unroll
+                for (int o = 16; o > 0; o >>= 1) v += __shfl_xor_sync(0xffffffffu, v, o);
+                if (lane == 0) atomicAdd(tpart + (size_t)blockIdx.x * 8 + l, (double)v);
             }
         }
     }
@@ -1096,7 +1110,7 @@ bool tc_make_map_rows(CUtensorMap *m, const void *base, int width, int n, int BH
 int tc_sm_count();
 cudaError_t launch_tc_causal_stats(const AttnArgs &a, cudaStream_t s);
 cudaError_t launch_tc_phi_bwd(const AttnArgs &a, const void *X, const float *dphi, void *dX, int slot0, int grid,
-                              cudaStream_t s, double *tpart = nullptr);
+                              cudaStream_t s, const float *kfold = nullptr);
 
 cudaError_t launch_tc_causal_bwd(const AttnArgs &a0, bool have_state, cudaStream_t s) {
     using C = K64;
@@ -1119,13 +1133,26 @@ cudaError_t launch_tc_causal_bwd(const AttnArgs &a0, bool have_state, cudaStream
         !tc_make_map_rows(&mdO128, a.dO, a.dv, a.n, BH, 128, hm))
         return cudaErrorInvalidValue;
     // 1. query side
-    if ((e = cudaFuncSetAttribute(k_tcc_query<C>, cudaFuncAttributeMaxDynamicSharedMemorySize, C::SMEM_Q)) != cudaSuccess)
+    if ((e = cudaFuncSetAttribute(k_tcc_query<C, false>, cudaFuncAttributeMaxDynamicSharedMemorySize, C::SMEM_Q)) !=
+            cudaSuccess ||
+        (e = cudaFuncSetAttribute(k_tcc_query<C, true>, cudaFuncAttributeMaxDynamicSharedMemorySize, C::SMEM_Q)) !=
+            cudaSuccess)
         return e;
-    LUNA_LAUNCH("tcc_query", k_tcc_query<C>, grid, kCBThreads, C::SMEM_Q, s, mQ, mK, mV, mdO, a, st);
+    // with the channel normalisation the sweep also sums phi^ . dphi^ per channel and block (T), so that
+    // the scale term's kappa is known before either chain rule, which then adds M kappa_l phi^ to dphi^
+    double *tpart = a.ch_sigma ? a.ch_T : nullptr;
+    if (tpart && (e = cudaMemsetAsync(tpart, 0, (size_t)grid * 8 * sizeof(double), s)) != cudaSuccess) return e;
+    if (tpart)
+        LUNA_LAUNCH("tcc_query", (k_tcc_query<C, true>), grid, kCBThreads, C::SMEM_Q, s, mQ, mK, mV, mdO, a, tpart, st);
+    else
+        LUNA_LAUNCH("tcc_query", (k_tcc_query<C, false>), grid, kCBThreads, C::SMEM_Q, s, mQ, mK, mV, mdO, a, tpart, st);
     if ((e = cudaGetLastError()) != cudaSuccess) return e;
-    // (with the channel normalisation the queries' chain rule also sums phi^ . dphi^ per channel and block)
-    if ((e = launch_tc_phi_bwd(a, a.Q, a.dphi, a.dQ, 0, grid, s, a.ch_sigma ? a.ch_T : nullptr)) != cudaSuccess)
-        return e;
+    if (a.ch_sigma) {
+        a.ch_T_rows = grid;
+        if ((e = launch_chrms_kappa(a, s)) != cudaSuccess) return e;
+    }
+    const float *kq = a.ch_sigma ? a.ch_kappa : nullptr, *kk = a.ch_sigma ? a.ch_kappa + kMaxL : nullptr;
+    if ((e = launch_tc_phi_bwd(a, a.Q, a.dphi, a.dQ, 0, grid, s, kq)) != cudaSuccess) return e;
     // 2, 3. segment sums of dS, dz and their suffix
     constexpr uint32_t SMEM_S = 2 * (6 * C::T16 + 4096) + 128 + 1024;
     static_assert(SMEM_S <= kSmemLimit, "shared memory budget");
@@ -1142,13 +1169,8 @@ cudaError_t launch_tc_causal_bwd(const AttnArgs &a0, bool have_state, cudaStream
     LUNA_LAUNCH("tcc_key", k_tcc_key<C>, grid, kCBThreads, C::SMEM_K, s, mPk, mPq, mV, mdO, a, st);
     if ((e = cudaGetLastError()) != cudaSuccess) return e;
     // 5. chain rule for K, then the parameter-gradient reduction over both sides
-    if ((e = launch_tc_phi_bwd(a, a.K, a.dphi, a.dK, grid, grid, s)) != cudaSuccess) return e;
-    int nparts = 2 * grid;
-    if (a.ch_sigma) {  // the scale term of the channel normalisation (kappa from the queries' T rows)
-        a.ch_T_rows = grid;
-        if ((e = launch_chrms_backward(a, 2 * grid, &nparts, s)) != cudaSuccess) return e;
-    }
-    return launch_grad_reduce(a, nparts, s);
+    if ((e = launch_tc_phi_bwd(a, a.K, a.dphi, a.dK, grid, grid, s, kk)) != cudaSuccess) return e;
+    return launch_grad_reduce(a, 2 * grid, s);
 }
 
 }  // namespace luna

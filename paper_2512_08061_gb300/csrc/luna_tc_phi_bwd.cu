@@ -52,7 +52,7 @@ __device__ void stage_wx64(const AttnArgs &a, uint8_t *dst) {
 template <class C>
 __global__ void __launch_bounds__(kBThreads, 1)
     k_tc_phi_bwd(const __grid_constant__ CUtensorMap mapX, AttnArgs a, const float *dphi, __nv_bfloat16 *dXg,
-                 int slot0, double *tpart, int *status) {
+                 int slot0, const float *kfold, int *status) {
     extern __shared__ uint8_t smem_raw[];
     const float fl = channel_floor(a.lay);  // lower bound of a channel output
     uint8_t *sm = align1024(smem_raw);
@@ -184,9 +184,9 @@ __global__ void __launch_bounds__(kBThreads, 1)
         float db_acc[C::PP];
 #pragma unroll
         for (int q = 0; q < C::PP; ++q) db_acc[q] = 0.0f;
-        float tacc[8];  // channel normalisation: this thread's sums of phi . dphi per channel
+        float kf[8];  // channel normalisation: dphi += M kappa_l phi (the scale term, on the scaled table)
 #pragma unroll
-        for (int l = 0; l < 8; ++l) tacc[l] = 0.0f;
+        for (int l = 0; l < 8; ++l) kf[l] = kfold ? (float)C::MP * kfold[l] : 0.0f;
         HistAcc hacc;
         int g = 0;
         for (int item = it.begin; item < it.end; ++item) {
@@ -232,10 +232,9 @@ __global__ void __launch_bounds__(kBThreads, 1)
                     float du = 0.0f;
 #pragma unroll
                     for (int l = 0; l < 8; ++l) {
-                        const float gl = (valid && y[l] > fl) ? dv[l] : 0.0f;
+                        const float gl = (valid && y[l] > fl) ? fmaf(kf[l], y[l], dv[l]) : 0.0f;
                         gv[q][l] = gl;
                         du = fmaf(gl, al[l], du);
-                        if (tpart) tacc[l] = fmaf(y[l], gl, tacc[l]);
                     }
                     dU[q] = du;
                     db_acc[q] += du;
@@ -297,15 +296,6 @@ __global__ void __launch_bounds__(kBThreads, 1)
             }
         }
         if (hacc.tiles > 0) hist_close(bins, hpart, a.lay.nint, hacc, tid, false, smax, warp, lane);
-        if (tpart) {  // the block's row of T: warp sums, then fp64 adds (the launch cleared the row)
-#pragma unroll
-            for (int l = 0; l < 8; ++l) {
-                float v = tacc[l];
-#pragma unroll
-                for (int o = 16; o > 0; o >>= 1) v += __shfl_xor_sync(0xffffffffu, v, o);
-                if (lane == 0) atomicAdd(tpart + (size_t)blockIdx.x * 8 + l, (double)v);
-            }
-        }
 #pragma unroll
         for (int q = 0; q < C::PP; ++q) {
             float v = db_acc[q];
@@ -342,16 +332,15 @@ int tc_sm_count();
 // and the parameter-gradient partials of blocks slot0 .. slot0 + grid - 1.
 // Work items: a.rows_per_split rows (whole 128-row tiles) of one head.
 cudaError_t launch_tc_phi_bwd(const AttnArgs &a, const void *X, const float *dphi, void *dX, int slot0, int grid,
-                              cudaStream_t s, double *tpart) {
+                              cudaStream_t s, const float *kfold) {
     using C = P128;
     CUtensorMap mX;
     if (!tc_make_map(&mX, X, a.d, a.n, a.B * a.H, a.hs_mul)) return cudaErrorInvalidValue;
     cudaError_t e = cudaFuncSetAttribute(k_tc_phi_bwd<C>, cudaFuncAttributeMaxDynamicSharedMemorySize, C::SMEM);
     if (e != cudaSuccess) return e;
     int *st = reinterpret_cast<int *>(reinterpret_cast<char *>(a.counters) - 256);
-    if (tpart && (e = cudaMemsetAsync(tpart, 0, (size_t)grid * 8 * sizeof(double), s)) != cudaSuccess) return e;
     LUNA_LAUNCH("tc_phi_bwd", k_tc_phi_bwd<C>, grid, kBThreads, C::SMEM, s, mX, a, dphi,
-                static_cast<__nv_bfloat16 *>(dX), slot0, tpart, st);
+                static_cast<__nv_bfloat16 *>(dX), slot0, kfold, st);
     return cudaGetLastError();
 }
 
