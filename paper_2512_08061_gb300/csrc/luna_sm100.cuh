@@ -98,6 +98,16 @@ __device__ __forceinline__ void prefetch_tmap(const CUtensorMap *map) {
     asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(map)) : "memory");
 }
 
+// Brings the box that tma_load_3d(map, c0, c1, c2) would load into L2 (a hint: no shared memory, no
+// completion to wait for; the parts of the box outside the tensor are skipped as a load would fill
+// them).  A producer issues it for its next tile so that the DRAM reads overlap the current tile's work.
+__device__ __forceinline__ void tma_prefetch_3d(const CUtensorMap *map, int c0, int c1, int c2) {
+    asm volatile("cp.async.bulk.prefetch.tensor.3d.L2.global.tile [%0, {%1, %2, %3}];" ::"l"(
+                     reinterpret_cast<uint64_t>(map)),
+                 "r"(c0), "r"(c1), "r"(c2)
+                 : "memory");
+}
+
 // 3-D tiled load of box (x, y, z) at coordinates (c0, c1, c2) into shared memory.
 __device__ __forceinline__ void tma_load_3d(void *dst, const CUtensorMap *map, int c0, int c1, int c2,
                                             uint64_t *bar) {

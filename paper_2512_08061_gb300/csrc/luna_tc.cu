@@ -243,6 +243,14 @@ __global__ void __launch_bounds__(kThreadsTC, 1)
                     for (int vb = 0; vb < C::NVB; ++vb)
                         tma_load_3d(Vb + v * C::VT + vb * 16384, &mapV, vb * 64, cur.row0(), cur.g.bh, fullv + v);
                 }
+                if (g + 1 < T) {  // the next tile into L2 while this one is worked on
+                    TileCursor nx = cur;
+                    nx.next(a, it);
+                    if (lane == 0)
+                        for (int kb = 0; kb < C::KBX; ++kb) tma_prefetch_3d(&mapK, kb * 64, nx.row0(), nx.g.bh);
+                    else
+                        for (int vb = 0; vb < C::NVB; ++vb) tma_prefetch_3d(&mapV, vb * 64, nx.row0(), nx.g.bh);
+                }
             }
         }
     } else if (warp == kMmaWarp) {

@@ -640,6 +640,13 @@ __global__ void __launch_bounds__(kSThreads, 1)
                 for (int kb = 0; kb < 4; ++kb) tma_load_3d(b + kb * T16, &mapPq, kb * 64, cur.row0(), cur.g.bh, full + s);
                 for (int kb = 0; kb < 2; ++kb)
                     tma_load_3d(b + (4 + kb) * T16, &mapdO, kb * 64, cur.row0(), cur.g.bh, full + s);
+                if (g + 2 < T) {  // the tile after the next into L2 (two stages are in flight)
+                    TileCursor nx = cur;
+                    nx.next(a, it);
+                    nx.next(a, it);
+                    for (int kb = 0; kb < 4; ++kb) tma_prefetch_3d(&mapPq, kb * 64, nx.row0(), nx.g.bh);
+                    for (int kb = 0; kb < 2; ++kb) tma_prefetch_3d(&mapdO, kb * 64, nx.row0(), nx.g.bh);
+                }
             }
         }
     } else if (warp == 1) {
@@ -848,6 +855,19 @@ __global__ void __launch_bounds__(kCBThreads, 1)
                 for (int kb = 0; kb < 4; ++kb) {
                     tma_load_3d(Pk + kb * T8, &mapPk, kb * 64, r0, bh, full);
                     tma_load_3d(Pq + kb * T8, &mapPq, kb * 64, r0, bh, full);
+                }
+                if (g + 1 < T && !failed) {  // the next tile into L2 while this one is worked on
+                    Cursor64 nx = cur;
+                    nx.next(a, it);
+                    const int n0 = nx.row0(), nb = nx.g.bh;
+                    for (int kb = 0; kb < 2; ++kb) {
+                        tma_prefetch_3d(&mapV, kb * 64, n0, nb);
+                        tma_prefetch_3d(&mapdO, kb * 64, n0, nb);
+                    }
+                    for (int kb = 0; kb < 4; ++kb) {
+                        tma_prefetch_3d(&mapPk, kb * 64, n0, nb);
+                        tma_prefetch_3d(&mapPq, kb * 64, n0, nb);
+                    }
                 }
             }
         }
