@@ -50,7 +50,11 @@ class _Phi(ctypes.Structure):
     _fields_ = [("d", ctypes.c_int), ("M", ctypes.c_int), ("L", ctypes.c_int), ("hid", ctypes.c_int)] + [
         (k, ctypes.c_void_p) for k in ("W", "b", "w1", "b1", "w2", "b2")
     ] + [("shared", ctypes.c_int), ("ch_rms_target", ctypes.c_double), ("chs", ctypes.c_void_p), ("heads", ctypes.c_int),
-         ("signed_out", ctypes.c_int)]
+         ("signed_out", ctypes.c_int), ("act", ctypes.c_int), ("We", ctypes.c_void_p), ("be", ctypes.c_void_p),
+         ("coef", ctypes.c_void_p)]
+
+# hidden-unit activations of the channel MLPs, by name (the code the C oracle takes)
+ACTS = {"relu": 0, "gelu": 1, "silu": 2, "tanh": 3}
 
 
 _P = ctypes.c_void_p
@@ -73,6 +77,7 @@ def lib():
             L.oracle_attn_fwd.argtypes = [phi, _I, _I, _I, _I, _I, _D, _P, _P, _P, _P, _P]
             L.oracle_attn_quadratic.argtypes = [phi, _I, _I, _I, _I, _I, _D, _P, _P, _P, _P, _P]
             L.oracle_attn_bwd.argtypes = [phi, _I, _I, _I, _I, _I, _D, _P, _P, _P, _P, _P, _P, _P, _P] + [_P] * 6
+            L.oracle_attn_bwd_var.argtypes = [phi, _I, _I, _I, _I, _I, _D, _P, _P, _P, _P, _P, _P, _P, _P] + [_P] * 9
             L.oracle_ch_rms.argtypes = [phi, _P, _I, _I, _I, _P, _P, _P]
             L.oracle_attn_weights.argtypes = [phi, _I, _I, _I, _I, _D, _P, _P, _P, _I, _I, _I, _P]
             L.oracle_max_threads.restype = _I
@@ -83,7 +88,7 @@ def lib():
             L.oracle_phi_offset.argtypes = [_I]
             # the mirror of the C struct must have its layout
             assert L.oracle_phi_size() == ctypes.sizeof(_Phi)
-            for i, f in enumerate(("W", "shared", "ch_rms_target", "chs", "heads", "signed_out")):
+            for i, f in enumerate(("W", "shared", "ch_rms_target", "chs", "heads", "signed_out", "act", "We", "coef")):
                 assert L.oracle_phi_offset(i) == getattr(_Phi, f).offset, f
             _lib = L
     return _lib
@@ -110,10 +115,18 @@ class PhiParams:
     the channel outputs without the outer ReLU.  ch_rms_target > 0 turns on the channel RMS
     normalisation: every channel's MLP outputs are scaled by
     s_l = min(target / (rms_l + 1e-6), 1) with rms_l over the valid rows of the input
-    the feature map is applied to (the queries and the keys separately)."""
+    the feature map is applied to (the queries and the keys separately).
 
-    def __init__(self, params: dict, ch_rms_target: float = 0.0, nonneg: bool = True):
+    The ablation variants of the feature map (Sec. 5.4, Table 5) and the listing's activation:
+    act in ACTS (the hidden-unit activation of the channel MLPs; "relu" is the default);
+    params["We"] (L, d) and params["be"] (L,) add the envelope gate
+    h_l(x) = sigmoid(We_l . x + be_l) multiplying channel l of every projection;
+    params["coef"] (L,) adds the Bank+Coef coefficient c_l multiplying channel l.  These
+    combine with each other, not with per-head parameters or ch_rms."""
+
+    def __init__(self, params: dict, ch_rms_target: float = 0.0, nonneg: bool = True, act: str = "relu"):
         self.arrays = {k: _f64(params[k]) for k in ("W", "b", "w1", "b1", "w2", "b2")}
+        self.extra = {k: _f64(params[k]) for k in ("We", "be", "coef") if params.get(k) is not None}
         W = self.arrays["W"]
         self.heads = W.shape[0] if W.ndim == 3 else 0
         lead = (self.heads,) if self.heads else ()
@@ -127,9 +140,20 @@ class PhiParams:
         assert core["b2"] == (self.L,)
         if self.heads and ch_rms_target > 0:
             raise ValueError("channel normalisation with per-head parameters is not defined here")
+        self.act = act
+        self.variant = act != "relu" or bool(self.extra)
+        if self.variant and (self.heads or ch_rms_target > 0):
+            raise ValueError("the feature-map variants combine with neither per-head parameters nor ch_rms")
+        assert ("We" in self.extra) == ("be" in self.extra)
+        if "We" in self.extra:
+            assert self.extra["We"].shape == (self.L, self.d) and self.extra["be"].shape == (self.L,)
+        if "coef" in self.extra:
+            assert self.extra["coef"].shape == (self.L,)
+        ex = [self.extra[k].ctypes.data if k in self.extra else None for k in ("We", "be", "coef")]
         self.struct = _Phi(self.d, self.M, self.L, self.hid,
                            *[self.arrays[k].ctypes.data for k in ("W", "b", "w1", "b1", "w2", "b2")],
-                           int(self.shared), float(ch_rms_target), None, int(self.heads), int(not nonneg))
+                           int(self.shared), float(ch_rms_target), None, int(self.heads), int(not nonneg),
+                           ACTS[act], *ex)
         self.ch_rms_target = float(ch_rms_target)
         self.nonneg = bool(nonneg)
 
@@ -140,7 +164,7 @@ class PhiParams:
     def head(self, h: int) -> "PhiParams":
         """The parameters of head h (per-head parameters only)."""
         assert self.heads
-        return PhiParams({k: v[h] for k, v in self.arrays.items()}, nonneg=self.nonneg)
+        return PhiParams({k: v[h] for k, v in self.arrays.items()}, nonneg=self.nonneg, act=self.act)
 
     def ref(self):
         return ctypes.byref(self.struct)
@@ -259,7 +283,7 @@ def attn_bwd_abs_terms(params, Q, K, V, dO, lengths=None, causal=False, eps=1e-6
         g = attn_bwd(params, Q, K, V, dO, lengths, causal, eps)
     finally:
         lib().oracle_set_abs_terms(0)
-    return {k: g[k] for k in ("dW", "db", "dw1", "db1", "dw2", "db2")}
+    return {k: v for k, v in g.items() if k not in ("dQ", "dK", "dV")}
 
 
 def attn_bwd(params, Q, K, V, dO, lengths=None, causal=False, eps=1e-6) -> dict:
@@ -272,8 +296,10 @@ def attn_bwd(params, Q, K, V, dO, lengths=None, causal=False, eps=1e-6) -> dict:
     la, lp = _lens(lengths, B)
     out = {"dQ": np.empty(Q.shape), "dK": np.empty(K.shape), "dV": np.empty(V.shape)}
     out.update({"d" + k: np.empty(p.arrays[k].shape) for k in ("W", "b", "w1", "b1", "w2", "b2")})
-    lib().oracle_attn_bwd(p.ref(), B, H, n, dv, int(bool(causal)), float(eps),
-                          Q.ctypes.data, K.ctypes.data, V.ctypes.data, dO.ctypes.data, lp,
-                          out["dQ"].ctypes.data, out["dK"].ctypes.data, out["dV"].ctypes.data,
-                          *[out[k].ctypes.data for k in ("dW", "db", "dw1", "db1", "dw2", "db2")])
+    out.update({"d" + k: np.empty(v.shape) for k, v in p.extra.items()})
+    lib().oracle_attn_bwd_var(p.ref(), B, H, n, dv, int(bool(causal)), float(eps),
+                              Q.ctypes.data, K.ctypes.data, V.ctypes.data, dO.ctypes.data, lp,
+                              out["dQ"].ctypes.data, out["dK"].ctypes.data, out["dV"].ctypes.data,
+                              *[out[k].ctypes.data for k in ("dW", "db", "dw1", "db1", "dw2", "db2")],
+                              *[out["d" + k].ctypes.data if k in p.extra else None for k in ("We", "be", "coef")])
     return out

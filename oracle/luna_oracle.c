@@ -32,6 +32,12 @@
  *     map's parameters per layer and head, Sec. 5 / appendix): head h of every
  *     sequence uses its own W, b and channel MLPs; their gradients are summed
  *     over the batch only.
+ *   - the feature-map variants of the kernel ablation (Sec. 5.4, Table 5) and
+ *     the listing's ScalarMLP activation: a hidden-unit activation other
+ *     than ReLU (GELU in its erf form, SiLU, tanh) evaluated directly; the
+ *     envelope-gated map, channel l of every projection multiplied by the
+ *     tokenwise gate h_l(x) = sigmoid(We_l . x + be_l) in [0, 1]; and
+ *     Bank+Coef, channel l multiplied by a learned global coefficient c_l.
  *   - the listing's ch_rms channel normalisation: per call of the feature map
  *     (once over Q, once over K), every channel's MLP outputs are scaled by
  *     s_l = min(target / (rms_l + 1e-6), 1), rms_l = sqrt(mean y_l^2 + 1e-6)
@@ -68,6 +74,10 @@ typedef struct {
     const double *chs;    /* per-channel scales s_l in effect (NULL: 1); set per input by the callers */
     int heads;            /* > 0: parameters per head (arrays carry a leading head axis of this size) */
     int signed_out;       /* 1: the listing's nonneg = False (no outer ReLU); 0: its default */
+    int act;              /* hidden-unit activation: 0 ReLU (the default), 1 GELU (erf form), 2 SiLU, 3 tanh */
+    const double *We;     /* L x d envelope gate weights (NULL: no gate, h = 1) */
+    const double *be;     /* L envelope gate biases */
+    const double *coef;   /* L Bank+Coef channel coefficients (NULL: 1) */
 } oracle_phi;
 
 /* Layout of oracle_phi, checked by the Python binding against its mirror of the struct. */
@@ -80,6 +90,9 @@ size_t oracle_phi_offset(int field) {
         case 3: return offsetof(oracle_phi, chs);
         case 4: return offsetof(oracle_phi, heads);
         case 5: return offsetof(oracle_phi, signed_out);
+        case 6: return offsetof(oracle_phi, act);
+        case 7: return offsetof(oracle_phi, We);
+        case 8: return offsetof(oracle_phi, coef);
     }
     return (size_t)-1;
 }
@@ -105,9 +118,31 @@ static size_t fc1_row(const oracle_phi *p, int l) { return (size_t)(p->shared ? 
 
 typedef struct {
     double *dW, *db, *dw1, *db1, *dw2, *db2;
+    double *dWe, *dbe, *dcoef;  /* envelope and Bank+Coef parameters (NULL when the map has none) */
 } oracle_grads;
 
 static double relu(double x) { return x > 0.0 ? x : 0.0; }
+
+/* The hidden-unit activation of the channel MLPs and its derivative (ReLU'(0) = 0).
+ * GELU(a) = a Phi(a) with Phi the standard normal distribution function,
+ * SiLU(a) = a sigma(a), tanh. */
+#define ORACLE_PI 3.14159265358979323846
+static double act_f(int act, double a) {
+    switch (act) {
+        case 1: return 0.5 * a * (1.0 + erf(a / sqrt(2.0)));
+        case 2: return a / (1.0 + exp(-a));
+        case 3: return tanh(a);
+        default: return relu(a);
+    }
+}
+static double act_df(int act, double a) {
+    switch (act) {
+        case 1: return 0.5 * (1.0 + erf(a / sqrt(2.0))) + a * exp(-0.5 * a * a) / sqrt(2.0 * ORACLE_PI);
+        case 2: { const double sg = 1.0 / (1.0 + exp(-a)); return sg * (1.0 + a * (1.0 - sg)); }
+        case 3: { const double t = tanh(a); return 1.0 - t * t; }
+        default: return a > 0.0 ? 1.0 : 0.0;
+    }
+}
 
 int oracle_max_threads(void) {
 #ifdef _OPENMP
@@ -132,13 +167,13 @@ static double project(const oracle_phi *p, int i, const double *x) {
     return u;
 }
 
-/* y_l(u) = fc2(relu(fc1(u))) before the non-negativity ReLU (listing: ScalarMLP) */
+/* y_l(u) = fc2(act(fc1(u))) before the non-negativity ReLU (listing: ScalarMLP) */
 static double channel_pre(const oracle_phi *p, int l, double u) {
     const double *w1 = p->w1 + fc1_row(p, l);
     const double *b1 = p->b1 + fc1_row(p, l);
     const double *w2 = p->w2 + (size_t)l * p->hid;
     double y = p->b2[l];
-    for (int k = 0; k < p->hid; ++k) y += w2[k] * relu(w1[k] * u + b1[k]);
+    for (int k = 0; k < p->hid; ++k) y += w2[k] * act_f(p->act, w1[k] * u + b1[k]);
     return y;
 }
 
@@ -150,13 +185,25 @@ static double channel_out(const oracle_phi *p, int l, double u) {
 
 double oracle_psi(const oracle_phi *p, int l, double u) { return channel_out(p, l, u); }
 
-/* phi(x) = (1/sqrt(M)) [s_l psi_l(w_i^T x + b_i)]_{i,l},  index i*L + l (s_l = 1 without ch_rms) */
+/* The envelope gate of channel l for the row x: h_l(x) = sigmoid(We_l . x + be_l), 1 without a gate. */
+static double gate(const oracle_phi *p, int l, const double *x) {
+    if (!p->We) return 1.0;
+    double a = p->be[l];
+    for (int c = 0; c < p->d; ++c) a += p->We[(size_t)l * p->d + c] * x[c];
+    return 1.0 / (1.0 + exp(-a));
+}
+
+/* The Bank+Coef coefficient of channel l, 1 without one. */
+static double chcoef(const oracle_phi *p, int l) { return p->coef ? p->coef[l] : 1.0; }
+
+/* phi(x) = (1/sqrt(M)) [s_l h_l(x) c_l psi_l(w_i^T x + b_i)]_{i,l},  index i*L + l (s_l = 1 without
+ * ch_rms, h_l = 1 without the envelope gate, c_l = 1 without Bank+Coef) */
 static void phi_row(const oracle_phi *p, const double *x, double *out) {
     const double s = 1.0 / sqrt((double)p->M);
     for (int i = 0; i < p->M; ++i) {
         double u = project(p, i, x);
         for (int l = 0; l < p->L; ++l)
-            out[i * p->L + l] = s * (p->chs ? p->chs[l] : 1.0) * channel_out(p, l, u);
+            out[i * p->L + l] = s * (p->chs ? p->chs[l] : 1.0) * gate(p, l, x) * chcoef(p, l) * channel_out(p, l, u);
     }
 }
 
@@ -234,12 +281,12 @@ void oracle_kink_margin(const oracle_phi *p, const double *X, int64_t rows, doub
                 for (int k = 0; k < p->hid; ++k) {
                     double a = w1[k] * u + b1[k];
                     double sc = fabs(w1[k] * u) + fabs(b1[k]);
-                    if (w1[k] != 0.0 && sc > 0.0) {
+                    if (p->act == 0 && w1[k] != 0.0 && sc > 0.0) {  /* smooth activations have no kink */
                         double rel = fabs(a) / sc;
                         if (rel < m) m = rel;
                     }
-                    y += w2[k] * relu(a);
-                    ysc += fabs(w2[k] * relu(a));
+                    y += w2[k] * act_f(p->act, a);
+                    ysc += fabs(w2[k] * act_f(p->act, a));
                 }
                 if (ysc > 0.0 && !p->signed_out) {  /* the outer ReLU's kink */
                     double rel = fabs(y) / ysc;
@@ -266,19 +313,25 @@ static double term(double v) { return abs_terms ? fabs(v) : v; }
  * depends on every sample of the channel (kappa from ch_rms_kappa). */
 static void phi_rows_backward(const oracle_phi *p, const double *X, int64_t rows, const double *dPhi,
                               const double *kappa, double *dX, oracle_grads *g) {
-    const int D = p->M * p->L, d = p->d;
+    const int D = p->M * p->L, d = p->d, L = p->L;
     const double s = 1.0 / sqrt((double)p->M);
+    double *h = (double *)malloc(sizeof(double) * 2 * (size_t)L);
+    double *dE = h + L;  /* gradient with respect to e_l = h_l c_l of the row */
     for (int64_t r = 0; r < rows; ++r) {
         const double *x = X + r * d;
         double *dx = dX + r * d;
         for (int c = 0; c < d; ++c) dx[c] = 0.0;
+        for (int l = 0; l < L; ++l) { h[l] = gate(p, l, x); dE[l] = 0.0; }
         for (int i = 0; i < p->M; ++i) {
             double u = project(p, i, x);
             double du = 0.0;
-            for (int l = 0; l < p->L; ++l) {
+            for (int l = 0; l < L; ++l) {
                 double y = channel_pre(p, l, u);
+                const double dphi = dPhi[r * D + i * L + l];
+                const double cs = p->chs ? p->chs[l] : 1.0;
+                dE[l] += dphi * s * cs * (p->signed_out ? y : relu(y));
                 if (!p->signed_out && !(y > 0.0)) continue; /* outer ReLU inactive */
-                double dy = dPhi[r * D + i * p->L + l] * s;
+                double dy = dphi * s * h[l] * chcoef(p, l);
                 if (p->chs) dy = dy * p->chs[l] + (kappa ? kappa[l] * y : 0.0);
                 if (dy == 0.0) continue;
                 const double *w1 = p->w1 + fc1_row(p, l);
@@ -287,9 +340,9 @@ static void phi_rows_backward(const oracle_phi *p, const double *X, int64_t rows
                 g->db2[l] += term(dy);
                 for (int k = 0; k < p->hid; ++k) {
                     double a = w1[k] * u + b1[k];
-                    if (!(a > 0.0)) continue;
-                    g->dw2[(size_t)l * p->hid + k] += term(dy * a);
-                    double dh = dy * w2[k];
+                    if (p->act == 0 && !(a > 0.0)) continue;  /* inactive ReLU unit */
+                    g->dw2[(size_t)l * p->hid + k] += term(dy * act_f(p->act, a));
+                    double dh = dy * w2[k] * act_df(p->act, a);
                     g->dw1[fc1_row(p, l) + k] += term(dh * u);  /* shared: summed over the channels */
                     g->db1[fc1_row(p, l) + k] += term(dh);
                     du += dh * w1[k];
@@ -301,7 +354,20 @@ static void phi_rows_backward(const oracle_phi *p, const double *X, int64_t rows
                 dx[c] += du * p->W[(size_t)i * d + c];
             }
         }
+        /* e_l = h_l c_l: dc_l = dE_l h_l; through the gate, dh_l = dE_l c_l and
+         * d(We_l . x + be_l) = dh_l h_l (1 - h_l) */
+        for (int l = 0; l < L; ++l) {
+            if (p->coef) g->dcoef[l] += term(dE[l] * h[l]);
+            if (!p->We) continue;
+            const double dpre = dE[l] * chcoef(p, l) * h[l] * (1.0 - h[l]);
+            g->dbe[l] += term(dpre);
+            for (int c = 0; c < d; ++c) {
+                g->dWe[(size_t)l * d + c] += term(dpre * x[c]);
+                dx[c] += dpre * p->We[(size_t)l * d + c];
+            }
+        }
     }
+    free(h);
 }
 
 static int head_len(const int32_t *lengths, int b, int n) {
@@ -606,13 +672,22 @@ static void attn_bwd_head(const oracle_phi *pq_, const oracle_phi *pk_, int n, i
     free(PQ); free(PK); free(dPQ); free(dPK); free(dnum); free(dden); free(S); free(z); free(o);
 }
 
-void oracle_attn_bwd(const oracle_phi *p, int B, int H, int n, int dv, int causal, double eps, const double *Q,
-                     const double *K, const double *V, const double *dO, const int32_t *lengths, double *dQ,
-                     double *dK, double *dV, double *dW, double *db, double *dw1, double *db1, double *dw2,
-                     double *db2) {
+/* The gradient slots of one head's partial: [dW | db | dw1 | db1 | dw2 | db2 | dWe | dbe | dcoef]. */
+static oracle_grads grads_at(const oracle_phi *p, double *base) {
+    const size_t nW = (size_t)p->M * p->d, nb = p->M, nh = (size_t)p->L * p->hid, x = nW + nb + 3 * nh + p->L;
+    oracle_grads g = {base, base + nW, base + nW + nb, base + nW + nb + nh, base + nW + nb + 2 * nh,
+                      base + nW + nb + 3 * nh, base + x, base + x + (size_t)p->L * p->d,
+                      base + x + (size_t)p->L * p->d + p->L};
+    return g;
+}
+
+static void attn_bwd_all(const oracle_phi *p, int B, int H, int n, int dv, int causal, double eps, const double *Q,
+                         const double *K, const double *V, const double *dO, const int32_t *lengths, double *dQ,
+                         double *dK, double *dV, double *dW, double *db, double *dw1, double *db1, double *dw2,
+                         double *db2, double *dWe, double *dbe, double *dcoef) {
     const int d = p->d, M = p->M, L = p->L, hid = p->hid;
     const size_t nW = (size_t)M * d, nb = M, nh = (size_t)L * hid, nb2 = L;
-    const size_t per = nW + nb + 3 * nh + nb2;
+    const size_t per = nW + nb + 3 * nh + nb2 + (size_t)L * d + 2 * (size_t)L;
     const int BH = B * H, D = M * L;
     double *part = (double *)calloc((size_t)(BH > 0 ? BH : 1) * per, sizeof(double));
     side_maps sm;
@@ -626,9 +701,7 @@ void oracle_attn_bwd(const oracle_phi *p, int B, int H, int n, int dv, int causa
     }
 #pragma omp parallel for schedule(dynamic, 1)
     for (int bh = 0; bh < BH; ++bh) {
-        double *base = part + (size_t)bh * per;
-        oracle_grads g = {base, base + nW, base + nW + nb, base + nW + nb + nh, base + nW + nb + 2 * nh,
-                          base + nW + nb + 3 * nh};
+        oracle_grads g = grads_at(p, part + (size_t)bh * per);
         size_t qo = (size_t)bh * n * d, vo = (size_t)bh * n * dv, po = (size_t)bh * n * D;
         const oracle_phi vq = head_view(&sm.pq, bh % H), vk = head_view(&sm.pk, bh % H);
         attn_bwd_head(&vq, &vk, n, dv, causal, eps, Q + qo, K + qo, V + vo, dO + vo,
@@ -674,9 +747,7 @@ void oracle_attn_bwd(const oracle_phi *p, int B, int H, int n, int dv, int causa
         }
 #pragma omp parallel for schedule(dynamic, 1)
         for (int bh = 0; bh < BH; ++bh) {
-            double *base = part + (size_t)bh * per;
-            oracle_grads g = {base, base + nW, base + nW + nb, base + nW + nb + nh, base + nW + nb + 2 * nh,
-                              base + nW + nb + 3 * nh};
+            oracle_grads g = grads_at(p, part + (size_t)bh * per);
             const int len = head_len(lengths, bh / H, n);
             size_t qo = (size_t)bh * n * d, po = (size_t)bh * n * D;
             const oracle_phi vq = head_view(&sm.pq, bh % H), vk = head_view(&sm.pk, bh % H);
@@ -688,12 +759,14 @@ void oracle_attn_bwd(const oracle_phi *p, int B, int H, int n, int dv, int causa
     free(sm.st);
     /* ordered reduction over the heads (fc1 gradients: hid entries when the MLP is shared); with
      * per-head parameters, head h's gradients are the sum over the batch of its units b*H + h */
-    double *outs[6] = {dW, db, dw1, db1, dw2, db2};
-    const size_t n1 = p->shared ? (size_t)hid : nh;
-    size_t sizes[6] = {nW, nb, n1, n1, nh, nb2};
-    size_t offs[6] = {0, nW, nW + nb, nW + nb + nh, nW + nb + 2 * nh, nW + nb + 3 * nh};
+    double *outs[9] = {dW, db, dw1, db1, dw2, db2, dWe, dbe, dcoef};
+    const size_t n1 = p->shared ? (size_t)hid : nh, x = nW + nb + 3 * nh + nb2;
+    size_t sizes[9] = {nW, nb, n1, n1, nh, nb2, (size_t)L * d, (size_t)L, (size_t)L};
+    size_t offs[9] = {0, nW, nW + nb, nW + nb + nh, nW + nb + 2 * nh, nW + nb + 3 * nh, x, x + (size_t)L * d,
+                      x + (size_t)L * d + L};
     const int G = p->heads > 0 ? H : 1;
-    for (int t = 0; t < 6; ++t)
+    for (int t = 0; t < 9; ++t) {
+        if (!outs[t]) continue;
         for (int h = 0; h < G; ++h)
             for (size_t e = 0; e < sizes[t]; ++e) {
                 double acc = 0.0;
@@ -701,5 +774,24 @@ void oracle_attn_bwd(const oracle_phi *p, int B, int H, int n, int dv, int causa
                     if (G == 1 || bh % H == h) acc += part[(size_t)bh * per + offs[t] + e];
                 outs[t][(size_t)h * sizes[t] + e] = acc;
             }
+    }
     free(part);
+}
+
+void oracle_attn_bwd(const oracle_phi *p, int B, int H, int n, int dv, int causal, double eps, const double *Q,
+                     const double *K, const double *V, const double *dO, const int32_t *lengths, double *dQ,
+                     double *dK, double *dV, double *dW, double *db, double *dw1, double *db1, double *dw2,
+                     double *db2) {
+    attn_bwd_all(p, B, H, n, dv, causal, eps, Q, K, V, dO, lengths, dQ, dK, dV, dW, db, dw1, db1, dw2, db2, NULL,
+                 NULL, NULL);
+}
+
+/* oracle_attn_bwd with the gradients of the envelope gate (dWe: L x d, dbe: L) and of the Bank+Coef
+ * coefficients (dcoef: L); each may be NULL when the map has no such parameters. */
+void oracle_attn_bwd_var(const oracle_phi *p, int B, int H, int n, int dv, int causal, double eps, const double *Q,
+                         const double *K, const double *V, const double *dO, const int32_t *lengths, double *dQ,
+                         double *dK, double *dV, double *dW, double *db, double *dw1, double *db1, double *dw2,
+                         double *db2, double *dWe, double *dbe, double *dcoef) {
+    attn_bwd_all(p, B, H, n, dv, causal, eps, Q, K, V, dO, lengths, dQ, dK, dV, dW, db, dw1, db1, dw2, db2, dWe,
+                 dbe, dcoef);
 }

@@ -20,14 +20,15 @@ MUTANTS = {
     "wrong sign of d(den)": ("dden[i] = -dot / den;", "dden[i] = dot / den;"),
     "exclusive causal mask": ("int jmax = causal ? i + 1 : len;", "int jmax = causal ? i : len;"),
     "fc2 weight gradient without activation": (
-        "g->dw2[(size_t)l * p->hid + k] += term(dy * a);", "g->dw2[(size_t)l * p->hid + k] += term(dy);"),
+        "g->dw2[(size_t)l * p->hid + k] += term(dy * act_f(p->act, a));",
+        "g->dw2[(size_t)l * p->hid + k] += term(dy);"),
     "eps dropped from the linear form": (
         "double den = eps;\n        for (int f = 0; f < D; ++f) den += phq[f] * z[f];",
         "double den = 0;\n        for (int f = 0; f < D; ++f) den += phq[f] * z[f];"),
     "transposed state index": (
         "for (int f = 0; f < D; ++f) num += phq[f] * S[(size_t)f * dv + c];",
         "for (int f = 0; f < D; ++f) num += phq[f] * S[(size_t)c * D + f];"),
-    "inner ReLU mask dropped in backward": ("if (!(a > 0.0)) continue;\n                    g->dw2", "g->dw2"),
+    "inner ReLU mask inverted in backward": ("if (p->act == 0 && !(a > 0.0)) continue;", "if (p->act == 0 && a > 0.0) continue;"),
     "shared fc1 read per channel": ("return (size_t)(p->shared ? 0 : l) * p->hid;", "return (size_t)l * p->hid;"),
     "shared fc1 gradient not summed over channels": (
         "g->dw1[fc1_row(p, l) + k] += term(dh * u);", "g->dw1[(size_t)l * p->hid + k] += term(dh * u);"),
@@ -68,6 +69,26 @@ SIGNED_MUTANTS = {
         "if (!p->signed_out && !(y > 0.0)) continue;", "if (!(y > 0.0)) continue;"),
 }
 
+VARIANT_PINS = "tests/test_oracle_variants.py"
+VARIANT_MUTANTS = {
+    "GELU: tanh-free form with a wrong argument": (
+        "case 1: return 0.5 * a * (1.0 + erf(a / sqrt(2.0)));", "case 1: return 0.5 * a * (1.0 + erf(a));"),
+    "GELU derivative without the density term": (
+        " + a * exp(-0.5 * a * a) / sqrt(2.0 * ORACLE_PI);", ";"),
+    "SiLU derivative taken as the logistic function": ("return sg * (1.0 + a * (1.0 - sg));", "return sg;"),
+    "tanh derivative with the wrong sign": ("return 1.0 - t * t;", "return 1.0 + t * t;"),
+    "envelope gate without its bias": ("double a = p->be[l];", "double a = 0.0;"),
+    "envelope gate derivative without h (1 - h)": (
+        "const double dpre = dE[l] * chcoef(p, l) * h[l] * (1.0 - h[l]);", "const double dpre = dE[l] * chcoef(p, l);"),
+    "envelope gradient does not reach dX": ("dx[c] += dpre * p->We[(size_t)l * d + c];", ""),
+    "coefficient gradient without the gate": (
+        "if (p->coef) g->dcoef[l] += term(dE[l] * h[l]);", "if (p->coef) g->dcoef[l] += term(dE[l]);"),
+    "coefficient missing from the feature": (
+        "* gate(p, l, x) * chcoef(p, l) * channel_out", "* gate(p, l, x) * channel_out"),
+    "coefficient missing from the chain rule into the MLP": (
+        "double dy = dphi * s * h[l] * chcoef(p, l);", "double dy = dphi * s * h[l];"),
+}
+
 WEIGHTS_PINS = "tests/test_oracle_weights.py"
 WEIGHTS_MUTANTS = {
     "weights: eps dropped from the normaliser": (
@@ -80,6 +101,7 @@ WEIGHTS_MUTANTS = {
 
 ALL = {**{k: (v, "tests/test_oracle_pins.py") for k, v in MUTANTS.items()},
        **{k: (v, WEIGHTS_PINS) for k, v in WEIGHTS_MUTANTS.items()},
+       **{k: (v, VARIANT_PINS) for k, v in VARIANT_MUTANTS.items()},
        **{k: (v, SIGNED_PINS) for k, v in SIGNED_MUTANTS.items()},
        **{k: (v, CH_RMS_PINS) for k, v in CH_RMS_MUTANTS.items()},
        **{k: (v, PER_HEAD_PINS) for k, v in PER_HEAD_MUTANTS.items()}}
