@@ -62,6 +62,13 @@ typedef enum {
 
 typedef enum { LUNA_F32 = 0, LUNA_BF16 = 1 } luna_dtype;
 
+/* Hidden-unit activation of the channel MLPs (the listing's ScalarMLP `act`):
+ * ReLU is the listing's default and the only one with the exact
+ * piecewise-linear table; the others are evaluated directly.
+ * GELU(a) = a Phi(a) (Phi: the standard normal distribution function, the erf
+ * form), SiLU(a) = a / (1 + e^-a), tanh. */
+typedef enum { LUNA_ACT_RELU = 0, LUNA_ACT_GELU = 1, LUNA_ACT_SILU = 2, LUNA_ACT_TANH = 3 } luna_act;
+
 /* Shape of the feature map (Eq. phi-def-scalarenv; listing defaults hidden = 64).
  * shared_channels = 0: one scalar MLP per channel (the listing's default);
  * 1: one scalar MLP with L outputs serves all channels (the listing's
@@ -97,6 +104,26 @@ typedef enum { LUNA_F32 = 0, LUNA_BF16 = 1 } luna_dtype;
  * attention calls then run one sub-problem per head index (the B sequences'
  * head h at a time).  Not with ch_rms_target > 0 (LUNA_ERR_UNSUPPORTED); for
  * luna_featmap pass head h's table with a stride of 0.
+ * Feature-map variants (the kernel ablation of Sec. 5.4, Table 5; each 0 = off,
+ * the paper's default "no gate" map psi):
+ *   act (a luna_act): the channel MLPs' hidden activation.  Not ReLU: every
+ *     (row, projection) evaluates the L channel MLPs unit by unit, and the
+ *     backward pass sums the MLP parameter gradients sample by sample (the
+ *     interval histogram needs a piecewise-linear MLP).
+ *   envelope = 1: the envelope-gated map phi(x) = h(x) (.) psi(x), channel l
+ *     of every projection multiplied by the tokenwise gate
+ *     h_l(x) = sigmoid(We_l . x + be_l) in (0, 1) (We, be in luna_phi_params;
+ *     their gradients dWe, dbe in luna_phi_grads).
+ *   bank_coef = 1: Bank+Coef, channel l of every projection multiplied by a
+ *     learned global coefficient c_l (coef; gradient dcoef): an input-agnostic
+ *     reweighting of the bank of channel functions that keeps the feature
+ *     dimension M*L (a negative c_l gives features of either sign).
+ *   They combine with each other and with shared_channels and signed_outputs;
+ *   any of them runs the attention calls on the generic (CUDA-core) kernels and
+ *   gives LUNA_ERR_UNSUPPORTED with ch_rms_target > 0, with param_head_stride,
+ *   and in luna_attn_decode and luna_attn_weights.  The
+ *   table holds the gate and coefficient parameters, so pass the same
+ *   descriptor to every call of one problem.
  * Supported: 1 <= M, 1 <= L <= 16, M*L <= 128, 1 <= hidden <= 128, L*hidden <= 512. */
 typedef struct {
     int M;               /* number of projections w_i (rows of W)       */
@@ -106,6 +133,9 @@ typedef struct {
     float ch_rms_target; /* channel RMS normalisation target, 0 = off   */
     int signed_outputs;  /* 0 or 1, see above                           */
     int64_t param_head_stride; /* bytes between heads' tables, 0 = shared  */
+    int act;             /* luna_act of the channel MLPs' hidden units   */
+    int envelope;        /* 0 or 1: envelope-gated map, see above        */
+    int bank_coef;       /* 0 or 1: Bank+Coef channel coefficients       */
 } luna_phi_desc;
 
 /* Feature-map parameters, fp32 device arrays, row-major:
@@ -114,16 +144,21 @@ typedef struct {
  * w1[l][k], b1[l][k] are fc1 of channel l (Linear(1, hidden)); w2[l][k], b2[l]
  * are its fc2 (Linear(hidden, 1)), or row l of the shared fc2. The same
  * parameters serve queries and keys and are shared by all heads (listing:
- * "shared ... over tokens/heads"). */
+ * "shared ... over tokens/heads").  The variants' parameters: We [L][d], be [L]
+ * (envelope gate; read only with envelope = 1) and coef [L] (read only with
+ * bank_coef = 1); NULL when their variant is off. */
 typedef struct {
     const float *W, *b, *w1, *b1, *w2, *b2;
+    const float *We, *be, *coef;
 } luna_phi_params;
 
 /* Gradients of the feature-map parameters, fp32 device arrays with the shapes
  * of luna_phi_params (dw1, db1 of [hidden] with shared_channels).  They are
- * OVERWRITTEN (not accumulated) by luna_attn_bwd. */
+ * OVERWRITTEN (not accumulated) by luna_attn_bwd.  dWe, dbe (envelope = 1) and
+ * dcoef (bank_coef = 1) are required with their variant and ignored without. */
 typedef struct {
     float *dW, *db, *dw1, *db1, *dw2, *db2;
+    float *dWe, *dbe, *dcoef;
 } luna_phi_grads;
 
 /* Problem description (Sec. 3.1: Q, K in R^{n x d}; Sec. 4: values of width d_v).
@@ -158,6 +193,9 @@ luna_status luna_phi_table_size(const luna_phi_desc *pd, int d, size_t *bytes);
  * psi_l(u) = relu(alpha_{l,j} u + beta_{l,j}) on interval j.  Kinks are
  * placed at the exact fp32 thresholds of fma(w1, u, b1) > 0, so the interval
  * decides every hidden unit exactly as an fp32 evaluation of fc1 would.
+ * With a non-ReLU act the table still holds the parameters (the calls
+ * evaluate the MLPs from them) and the piecewise form is not used; with
+ * envelope or bank_coef it also holds We, be or coef.
  * `table` is a device buffer of at least luna_phi_table_size bytes, 256-byte
  * aligned; it must not be modified while a call that reads it is in flight.
  * Parameters must be finite. */

@@ -26,15 +26,28 @@ luna_status check_phi(const luna_phi_desc *pd, int d) {
     if (pd->signed_outputs && pd->ch_rms_target > 0.0f) return LUNA_ERR_UNSUPPORTED;
     if (pd->param_head_stride < 0) return LUNA_ERR_INVALID_ARG;
     if (pd->param_head_stride) {  // one table per head, each a whole 256-byte aligned table
-        const int64_t tb = table_layout(pd->M, pd->L, pd->hidden, d, pd->shared_channels).bytes;
+        const int64_t tb = table_layout(pd->M, pd->L, pd->hidden, d, pd->shared_channels).bytes;  // no variants here
         if (pd->param_head_stride < tb || pd->param_head_stride % 256 != 0) return LUNA_ERR_INVALID_ARG;
         if (pd->ch_rms_target > 0.0f) return LUNA_ERR_UNSUPPORTED;  // batch statistics of one shared map
     }
+    if (pd->act < LUNA_ACT_RELU || pd->act > LUNA_ACT_TANH) return LUNA_ERR_INVALID_ARG;
+    if ((pd->envelope != 0 && pd->envelope != 1) || (pd->bank_coef != 0 && pd->bank_coef != 1))
+        return LUNA_ERR_INVALID_ARG;
+    if ((pd->act || pd->envelope || pd->bank_coef) && (pd->ch_rms_target > 0.0f || pd->param_head_stride))
+        return LUNA_ERR_UNSUPPORTED;
     if (pd->L > kMaxL || pd->M * pd->L > kMaxFeat || pd->M > 32 || pd->hidden > kMaxHidden ||
         pd->L * pd->hidden > kMaxUnits || d > kMaxD || pd->M * d > 4096)
         return LUNA_ERR_UNSUPPORTED;
     return LUNA_OK;
 }
+
+// Layout of the table of a descriptor (input width d).
+TableLayout phi_layout(const luna_phi_desc *pd, int d) {
+    return table_layout(pd->M, pd->L, pd->hidden, d, pd->shared_channels, pd->signed_outputs, pd->act, pd->envelope,
+                        pd->bank_coef);
+}
+
+bool phi_variant(const luna_phi_desc *pd) { return pd->act || pd->envelope || pd->bank_coef; }
 
 struct Plan {
     TableLayout lay;
@@ -89,10 +102,10 @@ luna_status make_plan(const luna_attn_desc *ad, const luna_phi_desc *pd, Plan &p
     p.ch_target = pd->ch_rms_target;
     if ((int64_t)ad->B * ad->H > (1 << 24)) return LUNA_ERR_UNSUPPORTED;
 
-    p.lay = table_layout(pd->M, pd->L, pd->hidden, ad->d, pd->shared_channels, pd->signed_outputs);
+    p.lay = phi_layout(pd, ad->d);
     const int BH = ad->B * ad->H, n = ad->n, D = p.lay.D, dv = ad->dv;
     p.BH = BH;
-    p.gsize = pd->M * ad->d + pd->M + p.lay.nint * pd->L * 2;
+    p.gsize = grad_words(p.lay);
     if (BH == 0 || n == 0) return LUNA_OK;
     // splits depend only on the descriptor, so workspace sizes are reproducible
     {
@@ -310,7 +323,7 @@ luna_status luna_phi_table_size(const luna_phi_desc *pd, int d, size_t *bytes) {
     if (!bytes) return LUNA_ERR_INVALID_ARG;
     luna_status st = check_phi(pd, d);
     if (st != LUNA_OK) return st;
-    *bytes = (size_t)table_layout(pd->M, pd->L, pd->hidden, d, pd->shared_channels, pd->signed_outputs).bytes;
+    *bytes = (size_t)phi_layout(pd, d).bytes;
     return LUNA_OK;
 }
 
@@ -320,8 +333,9 @@ luna_status luna_phi_prepare(const luna_phi_desc *pd, int d, const luna_phi_para
     if (st != LUNA_OK) return st;
     if (!params || !table || !params->W || !params->b || !params->w1 || !params->b1 || !params->w2 || !params->b2)
         return LUNA_ERR_INVALID_ARG;
+    if ((pd->envelope && (!params->We || !params->be)) || (pd->bank_coef && !params->coef)) return LUNA_ERR_INVALID_ARG;
     if (!aligned(table, 256)) return LUNA_ERR_INVALID_ARG;
-    TableLayout lay = table_layout(pd->M, pd->L, pd->hidden, d, pd->shared_channels, pd->signed_outputs);
+    TableLayout lay = phi_layout(pd, d);
     if (table_bytes < (size_t)lay.bytes) return LUNA_ERR_WORKSPACE;
     return cuda_status(launch_phi_prepare(*params, lay, table, static_cast<cudaStream_t>(stream)));
 }
@@ -335,7 +349,7 @@ luna_status luna_featmap(const luna_phi_desc *pd, int d, const void *table, cons
     if (pd->param_head_stride) return LUNA_ERR_UNSUPPORTED;  // rows carry no head: pass that head's table
     if (rows == 0) return LUNA_OK;
     if (!table || !X || !Phi) return LUNA_ERR_INVALID_ARG;
-    TableLayout lay = table_layout(pd->M, pd->L, pd->hidden, d, pd->shared_channels, pd->signed_outputs);
+    TableLayout lay = phi_layout(pd, d);
     return cuda_status(launch_featmap(lay, static_cast<const char *>(table), X, xtype, rows, Phi,
                                       static_cast<cudaStream_t>(stream)));
 }
@@ -410,6 +424,7 @@ luna_status luna_attn_bwd(const luna_attn_desc *ad, const luna_phi_desc *pd, con
     if (st != LUNA_OK) return st;
     if (!grads || !grads->dW || !grads->db || !grads->dw1 || !grads->db1 || !grads->dw2 || !grads->db2)
         return LUNA_ERR_INVALID_ARG;
+    if ((pd->envelope && (!grads->dWe || !grads->dbe)) || (pd->bank_coef && !grads->dcoef)) return LUNA_ERR_INVALID_ARG;
     cudaStream_t s = static_cast<cudaStream_t>(stream);
     if (p.BH == 0 || ad->n == 0) {  // empty problem: parameter gradients are zero
         const size_t G = pd->param_head_stride ? (size_t)ad->H : 1;  // parameter sets
@@ -421,6 +436,9 @@ luna_status luna_attn_bwd(const luna_attn_desc *ad, const luna_phi_desc *pd, con
         if (e == cudaSuccess) e = cudaMemsetAsync(grads->db1, 0, P1 * 4, s);
         if (e == cudaSuccess) e = cudaMemsetAsync(grads->dw2, 0, P * 4, s);
         if (e == cudaSuccess) e = cudaMemsetAsync(grads->db2, 0, G * pd->L * 4, s);
+        if (e == cudaSuccess && pd->envelope) e = cudaMemsetAsync(grads->dWe, 0, (size_t)pd->L * ad->d * 4, s);
+        if (e == cudaSuccess && pd->envelope) e = cudaMemsetAsync(grads->dbe, 0, (size_t)pd->L * 4, s);
+        if (e == cudaSuccess && pd->bank_coef) e = cudaMemsetAsync(grads->dcoef, 0, (size_t)pd->L * 4, s);
         return cuda_status(e);
     }
     if (!table || !Q || !K || !V || !dO || !dQ || !dK || !dV || !workspace) return LUNA_ERR_INVALID_ARG;
@@ -492,6 +510,7 @@ luna_status luna_attn_weights(const luna_attn_desc *ad, const luna_phi_desc *pd,
     luna_status st = check_phi(pd, ad->d);
     if (st != LUNA_OK) return st;
     if (pd->ch_rms_target > 0.0f) return LUNA_ERR_UNSUPPORTED;  // batch statistics: not for a block of rows
+    if (phi_variant(pd)) return LUNA_ERR_UNSUPPORTED;
     if (ad->n > (1 << 24) || (int64_t)ad->B * ad->H > 65535) return LUNA_ERR_UNSUPPORTED;
     if ((int64_t)ad->B * ad->H == 0 || rows == 0 || ad->n == 0) return LUNA_OK;
     if (!Q || !K || !A || (!teacher && !table)) return LUNA_ERR_INVALID_ARG;
@@ -499,7 +518,7 @@ luna_status luna_attn_weights(const luna_attn_desc *ad, const luna_phi_desc *pd,
     AttnArgs a;
     memset(&a, 0, sizeof(a));
     a.B = ad->B; a.H = ad->H; a.n = ad->n; a.d = ad->d; a.dv = ad->dv;
-    a.lay = table_layout(pd->M, pd->L, pd->hidden, ad->d, pd->shared_channels, pd->signed_outputs);
+    a.lay = phi_layout(pd, ad->d);
     a.M = a.lay.M; a.L = a.lay.L; a.D = a.lay.D;
     a.eps = ad->eps;
     a.table = static_cast<const char *>(table);
@@ -538,9 +557,10 @@ luna_status luna_attn_decode(const luna_attn_desc *ad, const luna_phi_desc *pd, 
     if (st != LUNA_OK) return st;
     if (ad->dv > kMaxD) return LUNA_ERR_UNSUPPORTED;
     if (pd->ch_rms_target > 0.0f) return LUNA_ERR_UNSUPPORTED;  // a batch statistic: no single-token step
+    if (phi_variant(pd)) return LUNA_ERR_UNSUPPORTED;
     const int64_t BH = (int64_t)ad->B * ad->H;
     if (BH > (1 << 24)) return LUNA_ERR_UNSUPPORTED;
-    const TableLayout lay = table_layout(pd->M, pd->L, pd->hidden, ad->d, pd->shared_channels, pd->signed_outputs);
+    const TableLayout lay = phi_layout(pd, ad->d);
     const int64_t SD = (int64_t)lay.D * ad->dv;
     if (S_stride == 0) S_stride = SD;
     if (z_stride == 0) z_stride = lay.D;

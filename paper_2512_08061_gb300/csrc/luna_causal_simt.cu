@@ -232,7 +232,7 @@ __global__ void __launch_bounds__(kThreads) k_causal_dq(AttnArgs a) {
     const size_t so = head_state(a, bh) * (a.nseg + 1) + seg;
     for (int e = threadIdx.x; e < D * dv; e += blockDim.x) S[e] = a.seg_S[so * D * dv + e];
     for (int e = threadIdx.x; e < D; e += blockDim.x) z[e] = a.seg_z[so * D + e];
-    for (int e = threadIdx.x; e < lay.nint * lay.L * 2; e += blockDim.x) shist[e] = 0.0;
+    for (int e = threadIdx.x; e < mlp_words(lay) + var_words(lay); e += blockDim.x) shist[e] = 0.0;
     GradAcc g = {};
     for (int t0 = r0; t0 < r1; t0 += kCs) {
         const int nr = min(kCs, r1 - t0);
@@ -271,7 +271,7 @@ __global__ void __launch_bounds__(kThreads) k_causal_dq(AttnArgs a) {
         }
         __syncthreads();
         advance_state(S, z, sPk, sV, nr, D, dv);
-        phi_backward_tile(lay, s, sQ, nr, sPq, sdPq, sU, sJ, sdU, shist, g);
+        phi_backward_tile(lay, s, sQ, nr, sPq, sdPq, sU, sJ, sdU, shist, shist + mlp_words(lay), g);
         store_dx(lay, s, sdU, nr, dQ + (size_t)t0 * d);
     }
     __syncthreads();
@@ -311,7 +311,7 @@ __global__ void __launch_bounds__(kThreads) k_causal_dkv(AttnArgs a) {
     const size_t so = (size_t)bh * a.nseg + seg;
     for (int e = threadIdx.x; e < D * dv; e += blockDim.x) G[e] = a.seg_dS[so * D * dv + e];
     for (int e = threadIdx.x; e < D; e += blockDim.x) gz[e] = a.seg_dz[so * D + e];
-    for (int e = threadIdx.x; e < lay.nint * lay.L * 2; e += blockDim.x) shist[e] = 0.0;
+    for (int e = threadIdx.x; e < mlp_words(lay) + var_words(lay); e += blockDim.x) shist[e] = 0.0;
     GradAcc g = {};
     if (r1 > r0) {
         for (int t0 = r0 + ((r1 - 1 - r0) / kCs) * kCs; t0 >= r0; t0 -= kCs) {
@@ -369,7 +369,7 @@ __global__ void __launch_bounds__(kThreads) k_causal_dkv(AttnArgs a) {
                 for (int r = 0; r < nr; ++r) acc = fma((double)sPq[r * D + f], (double)sdden[r], acc);
                 gz[f] = (float)acc;
             }
-            phi_backward_tile(lay, s, sK, nr, sPk, sdPk, sU, sJ, sdU, shist, g);
+            phi_backward_tile(lay, s, sK, nr, sPk, sdPk, sU, sJ, sdU, shist, shist + mlp_words(lay), g);
             store_dx(lay, s, sdU, nr, dK + (size_t)t0 * d);
         }
     }

@@ -76,19 +76,29 @@ __host__ __device__ inline int64_t align256(int64_t x) { return (x + 255) & ~int
 //   W      [M][d], b [M]   projection copy
 //   rank   [P]             position of unit (l,k) (shared MLP: unit k) in the sorted kink list
 //   utype  [P]             +1: unit active iff u > T[rank] ; -1: active iff u <= T[rank]
-//   w1, b1 [P], w2 [L*hid], b2 [L]  channel-MLP parameter copy (used by the gradient reduction)
+//   w1, b1 [P], w2 [L*hid], b2 [L]  channel-MLP parameter copy (used by the gradient reduction and,
+//                                    with a non-ReLU activation, by the direct evaluation)
+//   We [L][d], be [L]  envelope gate (envelope variant only), coef [L] (Bank+Coef variant only)
 struct TableLayout {
     int M, L, hid, d, D, P, Ppad, nint;
     int shared;  // one MLP for all channels: P = hid kinks (else P = L * hid)
     int signed_out;  // channel outputs without the outer ReLU (the listing's nonneg = False)
+    int act;     // hidden-unit activation (luna_act): not ReLU = direct evaluation, no table lookup
+    int env;     // envelope gate h_l(x) = sigmoid(We_l . x + be_l) on channel l
+    int coef;    // Bank+Coef coefficient c_l on channel l
     int64_t off_T, off_Te, off_AB, off_W, off_b, off_rank, off_utype, off_w1, off_b1, off_w2, off_b2, bytes;
+    int64_t off_We, off_be, off_coef;
 };
 
-__host__ __device__ inline TableLayout table_layout(int M, int L, int hid, int d, int shared = 0, int signed_out = 0) {
+__host__ __device__ inline TableLayout table_layout(int M, int L, int hid, int d, int shared = 0, int signed_out = 0,
+                                                    int act = 0, int env = 0, int coef = 0) {
     TableLayout t;
     t.M = M; t.L = L; t.hid = hid; t.d = d; t.D = M * L;
     t.shared = shared ? 1 : 0;
     t.signed_out = signed_out ? 1 : 0;
+    t.act = act;
+    t.env = env ? 1 : 0;
+    t.coef = coef ? 1 : 0;
     t.P = shared ? hid : L * hid;
     t.Ppad = next_pow2(t.P);
     t.nint = t.P + 1;
@@ -104,8 +114,28 @@ __host__ __device__ inline TableLayout table_layout(int M, int L, int hid, int d
     t.off_b1 = o;    o = align16(o + 4 * (int64_t)t.P);
     t.off_w2 = o;    o = align16(o + 4 * (int64_t)L * hid);
     t.off_b2 = o;    o = align16(o + 4 * (int64_t)L);
+    t.off_We = o;    o = align16(o + (t.env ? 4 * (int64_t)L * d : 0));
+    t.off_be = o;    o = align16(o + (t.env ? 4 * (int64_t)L : 0));
+    t.off_coef = o;  o = align16(o + (t.coef ? 4 * (int64_t)L : 0));
     t.bytes = align256(o);
     return t;
+}
+
+// One of the feature-map variants (a non-ReLU activation, the envelope gate, Bank+Coef): generic kernels only.
+__host__ __device__ __forceinline__ bool lay_variant(const TableLayout &lay) { return lay.act || lay.env || lay.coef; }
+
+// Parameter-gradient partial of a block: [dW (M*d) | db (M) | MLP region | variant region].  The MLP region
+// holds the interval histogram [nint][L][2] (ReLU), or with another activation the MLP gradients themselves
+// [dw2 (L*hid) | dw1 (P) | db1 (P) | db2 (L)]; the variant region [dWe (L*d) | dbe (L)] (envelope) then
+// [dcoef (L)] (Bank+Coef).
+__host__ __device__ __forceinline__ int mlp_words(const TableLayout &lay) {
+    return lay.act ? lay.L * lay.hid + 2 * lay.P + lay.L : lay.nint * lay.L * 2;
+}
+__host__ __device__ __forceinline__ int var_words(const TableLayout &lay) {
+    return (lay.env ? lay.L * lay.d + lay.L : 0) + (lay.coef ? lay.L : 0);
+}
+__host__ __device__ __forceinline__ int grad_words(const TableLayout &lay) {
+    return lay.M * lay.d + lay.M + mlp_words(lay) + var_words(lay);
 }
 
 struct TableHeader {

@@ -141,6 +141,12 @@ __global__ void __launch_bounds__(kPrepThreads) k_phi_prepare(luna_phi_params pr
         for (int e = tid; e < lay.M * lay.d; e += nt) W[e] = prm.W[e];
         for (int e = tid; e < lay.M; e += nt) reinterpret_cast<float *>(table + lay.off_b)[e] = prm.b[e];
         for (int e = tid; e < L; e += nt) reinterpret_cast<float *>(table + lay.off_b2)[e] = prm.b2[e];
+        if (lay.env) {  // envelope gate
+            for (int e = tid; e < L * lay.d; e += nt) reinterpret_cast<float *>(table + lay.off_We)[e] = prm.We[e];
+            for (int e = tid; e < L; e += nt) reinterpret_cast<float *>(table + lay.off_be)[e] = prm.be[e];
+        }
+        if (lay.coef)  // Bank+Coef coefficients
+            for (int e = tid; e < L; e += nt) reinterpret_cast<float *>(table + lay.off_coef)[e] = prm.coef[e];
         if (tid == 0) {
             TableHeader *h = reinterpret_cast<TableHeader *>(table);
             h->magic = kTableMagic; h->version = kTableVersion;

@@ -46,6 +46,29 @@ __global__ void __launch_bounds__(kThreads) k_featmap(TableLayout lay, const cha
     }
 }
 
+// The feature map of the variants (a non-ReLU activation, the envelope gate, Bank+Coef): blocks walk tiles of
+// kPhiRows rows through the generic tile helper.
+template <typename IO>
+__global__ void __launch_bounds__(kThreads) k_featmap_var(TableLayout lay, const char *table, const IO *X,
+                                                          int64_t rows, float *Phi) {
+    extern __shared__ __align__(16) float smem[];
+    Carve cv{smem};
+    SmemPhi s = carve_phi(cv, lay);
+    float *sX = cv.take(kPhiRows * lay.d);
+    float *sPhi = cv.take(kPhiRows * lay.D);
+    if (!carve_fits(cv, smem)) return;
+    load_phi(s, lay, table);
+    for (int64_t t0 = (int64_t)blockIdx.x * kPhiRows; t0 < rows; t0 += (int64_t)gridDim.x * kPhiRows) {
+        const int nr = (int)(rows - t0 < kPhiRows ? rows - t0 : kPhiRows);
+        __syncthreads();
+        load_rows(sX, X + t0 * lay.d, nr * lay.d);
+        __syncthreads();
+        phi_tile(lay, s, sX, nr, sPhi, nullptr, nullptr);
+        __syncthreads();
+        for (int e = threadIdx.x; e < nr * lay.D; e += blockDim.x) Phi[t0 * lay.D + e] = sPhi[e];
+    }
+}
+
 // ---------------------------------------------------------------------------
 // key statistics S = sum_j phi(k_j) v_j^T, z = sum_j phi(k_j)   (Sec. 4: S_KV, S_K1)
 
@@ -180,7 +203,7 @@ __global__ void __launch_bounds__(kThreads) k_bwd_query(AttnArgs a) {
     double *shist = gp + M * d + M;  // the block's fp64 histogram, accumulated in place by L2 atomics
     for (int e = threadIdx.x; e < D * dv; e += blockDim.x) sS[e] = a.S_fin[head_state(a, bh) * D * dv + e];
     for (int e = threadIdx.x; e < D; e += blockDim.x) sz[e] = a.z_fin[head_state(a, bh) * D + e];
-    for (int e = threadIdx.x; e < lay.nint * lay.L * 2; e += blockDim.x) shist[e] = 0.0;
+    for (int e = threadIdx.x; e < mlp_words(lay) + var_words(lay); e += blockDim.x) shist[e] = 0.0;
 
     const int len = head_length(a.lengths, bh / a.H, a.n);
     const int r0 = split * a.rows_per_split_b;
@@ -245,7 +268,7 @@ __global__ void __launch_bounds__(kThreads) k_bwd_query(AttnArgs a) {
         }
         __syncthreads();
         if (active) outer_accumulate(acc, zacc, true, sPhi, D, sdnum, dv, sdden, nr, f0, c0);
-        phi_backward_tile(lay, s, sQ, nr, sPhi, sdPhi, sU, sJ, sdU, shist, g);
+        phi_backward_tile(lay, s, sQ, nr, sPhi, sdPhi, sU, sJ, sdU, shist, shist + mlp_words(lay), g);
         store_dx(lay, s, sdU, nr, dQ + (size_t)t0 * d);
     }
     __syncthreads();
@@ -284,7 +307,7 @@ __global__ void __launch_bounds__(kThreads) k_bwd_key(AttnArgs a) {
     double *shist = gp + M * d + M;  // the block's fp64 histogram, accumulated in place by L2 atomics
     for (int e = threadIdx.x; e < D * dv; e += blockDim.x) sdS[e] = a.dS_fin[(size_t)bh * D * dv + e];
     for (int e = threadIdx.x; e < D; e += blockDim.x) sdz[e] = a.dz_fin[(size_t)bh * D + e];
-    for (int e = threadIdx.x; e < lay.nint * lay.L * 2; e += blockDim.x) shist[e] = 0.0;
+    for (int e = threadIdx.x; e < mlp_words(lay) + var_words(lay); e += blockDim.x) shist[e] = 0.0;
 
     const int len = head_length(a.lengths, bh / a.H, a.n);
     const int r0 = split * a.rows_per_split_b;
@@ -319,7 +342,7 @@ __global__ void __launch_bounds__(kThreads) k_bwd_key(AttnArgs a) {
             sdPhi[e] = (float)acc2;
         }
         __syncthreads();
-        phi_backward_tile(lay, s, sK, nr, sPhi, sdPhi, sU, sJ, sdU, shist, g);
+        phi_backward_tile(lay, s, sK, nr, sPhi, sdPhi, sU, sJ, sdU, shist, shist + mlp_words(lay), g);
         store_dx(lay, s, sdU, nr, dK + (size_t)t0 * d);
     }
     __syncthreads();
@@ -423,6 +446,9 @@ __device__ void warp_scan(const double *x, double *y, int n, bool backward) {
 // channel's interval histogram.  Block L: dW and db.  With the shared-channel
 // MLP every channel reads every hidden unit: block l writes its channel's fc1
 // contributions to fc1_part ([dw1 | db1][l][k], fp64), summed by k_mlp_fc1_sum.
+// With a non-ReLU activation the partials already hold the MLP gradients
+// (summed unit by unit): block l copies channel l's, block 0 the shared fc1's.
+// Block L also writes the gate's and the coefficients' gradients.
 __global__ void __launch_bounds__(128) k_mlp_grads(TableLayout lay, const char *table, const double *gsum,
                                                    luna_phi_grads grads, double *fc1_part) {
     __shared__ double h[2][kMaxUnits + 1];
@@ -432,10 +458,31 @@ __global__ void __launch_bounds__(128) k_mlp_grads(TableLayout lay, const char *
     if ((int)blockIdx.x == L) {
         for (int e = threadIdx.x; e < Md; e += blockDim.x) grads.dW[e] = (float)gsum[e];
         for (int e = threadIdx.x; e < lay.M; e += blockDim.x) grads.db[e] = (float)gsum[Md + e];
+        const double *gv = gsum + Md + lay.M + mlp_words(lay);  // [dWe | dbe] [dcoef]
+        if (lay.env) {
+            for (int e = threadIdx.x; e < L * lay.d; e += blockDim.x) grads.dWe[e] = (float)gv[e];
+            for (int e = threadIdx.x; e < L; e += blockDim.x) grads.dbe[e] = (float)gv[L * lay.d + e];
+            gv += L * lay.d + L;
+        }
+        if (lay.coef)
+            for (int e = threadIdx.x; e < L; e += blockDim.x) grads.dcoef[e] = (float)gv[e];
         return;
     }
     const int l = blockIdx.x;
     const double *hist = gsum + Md + lay.M;
+    if (lay.act) {  // [dw2 (L*hid) | dw1 (P) | db1 (P) | db2 (L)]
+        const int P = lay.P;
+        for (int k = threadIdx.x; k < hid; k += blockDim.x) grads.dw2[l * hid + k] = (float)hist[l * hid + k];
+        if (!lay.shared || l == 0) {
+            const int u0 = lay.shared ? 0 : l * hid;
+            for (int k = threadIdx.x; k < hid; k += blockDim.x) {
+                grads.dw1[u0 + k] = (float)hist[L * hid + u0 + k];
+                grads.db1[u0 + k] = (float)hist[L * hid + P + u0 + k];
+            }
+        }
+        if (threadIdx.x == 0) grads.db2[l] = (float)hist[L * hid + 2 * P + l];
+        return;
+    }
     for (int j = threadIdx.x; j < nint; j += blockDim.x) {
         h[0][j] = hist[(j * L + l) * 2];
         h[1][j] = hist[(j * L + l) * 2 + 1];
@@ -578,13 +625,30 @@ cudaError_t launch_grad_reduce(const AttnArgs &a, int nparts, cudaStream_t s) {
     // the partials have been summed: their buffer holds the shared MLP's per-channel fc1 terms
     double *fc1_part = reinterpret_cast<double *>(a.gpart);
     LUNA_LAUNCH("mlp_grads", k_mlp_grads, a.lay.L + 1, 128, 0, s, a.lay, a.table, a.hist, a.grads, fc1_part);
-    if ((e = cudaGetLastError()) != cudaSuccess || !a.lay.shared) return e;
+    if ((e = cudaGetLastError()) != cudaSuccess || !a.lay.shared || a.lay.act) return e;
     LUNA_LAUNCH("mlp_fc1_sum", k_mlp_fc1_sum, 1, 128, 0, s, a.lay, fc1_part, a.grads);
     return cudaGetLastError();
 }
 
 cudaError_t launch_featmap(const TableLayout &lay, const char *table, const void *X, luna_dtype xt, int64_t rows,
                            float *Phi, cudaStream_t s) {
+    if (lay_variant(lay)) {
+        HostCarve cv; carve_phi_host(cv, lay);
+        cv.take(kPhiRows * lay.d); cv.take(kPhiRows * lay.D);
+        const size_t sm = cv.bytes();
+        const int64_t tiles = (rows + kPhiRows - 1) / kPhiRows;
+        const int blocks = (int)(tiles < 4096 ? (tiles > 0 ? tiles : 1) : 4096);
+        cudaError_t e;
+        if (xt == LUNA_F32) {
+            if ((e = set_smem(k_featmap_var<float>, sm)) != cudaSuccess) return e;
+            k_featmap_var<float><<<blocks, kThreads, sm, s>>>(lay, table, static_cast<const float *>(X), rows, Phi);
+        } else {
+            if ((e = set_smem(k_featmap_var<__nv_bfloat16>, sm)) != cudaSuccess) return e;
+            k_featmap_var<__nv_bfloat16><<<blocks, kThreads, sm, s>>>(lay, table, static_cast<const __nv_bfloat16 *>(X),
+                                                                      rows, Phi);
+        }
+        return cudaGetLastError();
+    }
     HostCarve cv; carve_phi_host(cv, lay);
     const size_t sm = cv.bytes();
     int64_t work = rows * lay.M;

@@ -924,6 +924,7 @@ int tc_grid(const AttnArgs &items) { return grid_impl(items); }
 
 TcPlan tc_plan(const luna_attn_desc &ad, const TableLayout &lay) {
     TcPlan p;
+    if (lay_variant(lay)) return p;  // the feature-map variants run on the generic kernels
     p.variant = variant(ad, lay);
     p.eligible = p.variant >= 0 && encoder() != nullptr;
     p.bwd = p.eligible && tc_bwd_supported(ad, lay);

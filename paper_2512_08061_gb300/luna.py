@@ -34,15 +34,21 @@ class LunaError(RuntimeError):
 class PhiDesc(ctypes.Structure):
     _fields_ = [("M", ctypes.c_int), ("L", ctypes.c_int), ("hidden", ctypes.c_int), ("shared_channels", ctypes.c_int),
                 ("ch_rms_target", ctypes.c_float), ("signed_outputs", ctypes.c_int),
-                ("param_head_stride", ctypes.c_int64)]
+                ("param_head_stride", ctypes.c_int64), ("act", ctypes.c_int), ("envelope", ctypes.c_int),
+                ("bank_coef", ctypes.c_int)]
+
+
+PARAM_KEYS = ("W", "b", "w1", "b1", "w2", "b2", "We", "be", "coef")
+GRAD_KEYS = tuple("d" + k for k in PARAM_KEYS)
+ACTS = {"relu": 0, "gelu": 1, "silu": 2, "tanh": 3}  # luna_act
 
 
 class PhiParams(ctypes.Structure):
-    _fields_ = [(k, ctypes.c_void_p) for k in ("W", "b", "w1", "b1", "w2", "b2")]
+    _fields_ = [(k, ctypes.c_void_p) for k in PARAM_KEYS]
 
 
 class PhiGrads(ctypes.Structure):
-    _fields_ = [(k, ctypes.c_void_p) for k in ("dW", "db", "dw1", "db1", "dw2", "db2")]
+    _fields_ = [(k, ctypes.c_void_p) for k in GRAD_KEYS]
 
 
 class AttnDesc(ctypes.Structure):
@@ -126,8 +132,10 @@ def _io_code(t: torch.Tensor) -> int:
 
 
 def phi_desc(M: int, L: int, hidden: int, shared: bool = False, ch_rms_target: float = 0.0,
-             signed: bool = False, param_head_stride: int = 0) -> PhiDesc:
-    return PhiDesc(M, L, hidden, int(bool(shared)), float(ch_rms_target), int(bool(signed)), int(param_head_stride))
+             signed: bool = False, param_head_stride: int = 0, act: str = "relu", envelope: bool = False,
+             bank_coef: bool = False) -> PhiDesc:
+    return PhiDesc(M, L, hidden, int(bool(shared)), float(ch_rms_target), int(bool(signed)), int(param_head_stride),
+                   ACTS[act], int(bool(envelope)), int(bool(bank_coef)))
 
 
 def attn_desc(B, H, n, d, dv, causal=False, chunk=0, eps=1e-6, io=LUNA_BF16) -> AttnDesc:
@@ -149,7 +157,7 @@ def luna_phi_table_size(pd: PhiDesc, d: int) -> int:
 
 
 def luna_phi_prepare(pd: PhiDesc, d: int, params: dict, table: torch.Tensor, stream=None) -> None:
-    pp = PhiParams(*[_ptr(params[k]) for k in ("W", "b", "w1", "b1", "w2", "b2")])
+    pp = PhiParams(*[_ptr(params.get(k)) for k in PARAM_KEYS])
     _check(_lib.luna_phi_prepare(ctypes.byref(pd), d, ctypes.byref(pp), _ptr(table), table.numel() * table.element_size(),
                                  _stream(stream)), "luna_phi_prepare")
 
@@ -180,7 +188,7 @@ def luna_attn_fwd(ad, pd, table, Q, K, V, lengths, O, state, workspace, stream=N
 
 
 def luna_attn_bwd(ad, pd, table, Q, K, V, dO, lengths, state, dQ, dK, dV, grads: dict, workspace, stream=None) -> None:
-    pg = PhiGrads(*[_ptr(grads[k]) for k in ("dW", "db", "dw1", "db1", "dw2", "db2")])
+    pg = PhiGrads(*[_ptr(grads.get(k)) for k in GRAD_KEYS])
     _check(_lib.luna_attn_bwd(ctypes.byref(ad), ctypes.byref(pd), _ptr(table), _ptr(Q), _ptr(K), _ptr(V), _ptr(dO),
                               _ptr(lengths), _ptr(state), _ptr(dQ), _ptr(dK), _ptr(dV), ctypes.byref(pg),
                               _ptr(workspace), workspace.numel() * workspace.element_size(), _stream(stream)),
@@ -259,8 +267,9 @@ class Luna:
     """Owns the table, workspace and state buffers of one problem shape."""
 
     def __init__(self, B, H, n, d, dv, M, L, hidden=64, causal=False, eps=1e-6, io=torch.bfloat16, chunk=0,
-                 device="cuda", shared=False, ch_rms_target=0.0, signed=False, per_head=False):
-        self.pd = phi_desc(M, L, hidden, shared, ch_rms_target, signed)
+                 device="cuda", shared=False, ch_rms_target=0.0, signed=False, per_head=False, act="relu",
+                 envelope=False, bank_coef=False):
+        self.pd = phi_desc(M, L, hidden, shared, ch_rms_target, signed, 0, act, envelope, bank_coef)
         self.ad = attn_desc(B, H, n, d, dv, causal, chunk, eps, _DTYPES[io])
         self.d = d
         self.device = torch.device(device)
@@ -274,7 +283,8 @@ class Luna:
         self.state = alloc_bytes(luna_state_size(self.ad, self.pd), self.device)
 
     def prepare(self, params: dict, stream=None):
-        """params: W, b, w1, b1, w2, b2 device tensors (with a leading head axis for per-head parameters)."""
+        """params: W, b, w1, b1, w2, b2 device tensors (with a leading head axis for per-head parameters),
+        and We, be (envelope) or coef (Bank+Coef) with those variants."""
         if not self.heads:
             luna_phi_prepare(self.pd, self.d, params, self.table, stream)
             return
@@ -300,6 +310,10 @@ class Luna:
                    "dW": torch.empty(g + (M, self.d), **f32), "db": torch.empty(g + (M,), **f32),
                    "dw1": torch.empty(g + fc1, **f32), "db1": torch.empty(g + fc1, **f32),
                    "dw2": torch.empty(g + (L, hid), **f32), "db2": torch.empty(g + (L,), **f32)}
+            if self.pd.envelope:
+                out.update(dWe=torch.empty((L, self.d), **f32), dbe=torch.empty((L,), **f32))
+            if self.pd.bank_coef:
+                out["dcoef"] = torch.empty((L,), **f32)
         luna_attn_bwd(self.ad, self.pd, self.table, Q, K, V, dO, lengths, self.state if use_state else None,
                       out["dQ"], out["dK"], out["dV"], out, self.ws, stream)
         return out

@@ -1,6 +1,8 @@
 """Helpers for the GPU parity tests: seeded cases, device transfer, error metric."""
 from __future__ import annotations
 
+import math
+
 import numpy as np
 
 import oracle
@@ -105,8 +107,9 @@ def to_host(x) -> np.ndarray:
 class Case:
     def __init__(self, B, H, n, d, M, L, io, causal=False, seed=0, qkv_scale=1.0, len_range=None, hidden=64,
                  eps=1e-6, dv=None, with_grad=False, lengths=None, shared=False, ch_rms_target=0.0, signed=False,
-                 params=None, per_head=False):
+                 params=None, per_head=False, act="relu", envelope=False, bank_coef=False):
         self.B, self.H, self.n, self.d, self.M, self.L = B, H, n, d, M, L
+        self.act, self.envelope, self.bank_coef = act, envelope, bank_coef
         self.ch_rms_target = ch_rms_target
         self.signed = signed
         self.per_head = per_head
@@ -116,6 +119,14 @@ class Case:
             sets = [synth.phi_params(seed * 1000 + h, d, M, L, hidden, shared) for h in range(H)]
             params = {k: np.stack([s[k] for s in sets]) for k in sets[0]}
         self.params = params if params is not None else synth.phi_params(seed, d, M, L, hidden, shared)
+        if envelope and "We" not in self.params:  # gate pre-activations We_l . x of standard deviation 2
+            w_scale = 2.0 / (qkv_scale * math.sqrt(d))
+            self.params = {**self.params,
+                           "We": (synth.normal(seed, "case.We", (L, d)) * w_scale).astype(np.float32),
+                           "be": synth.normal(seed, "case.be", (L,)).astype(np.float32)}
+        if bank_coef and "coef" not in self.params:  # coefficients in [0.25, ~3): kernel values stay positive
+            self.params = {**self.params,
+                           "coef": (0.25 + np.abs(synth.normal(seed, "case.coef", (L,)))).astype(np.float32)}
         self.inp = synth.attn_inputs(seed, B, H, n, d, self.dv, io, qkv_scale, len_range, with_grad)
         if lengths is not None:
             self.inp["lengths"] = np.asarray(lengths, dtype=np.int32)
@@ -128,7 +139,8 @@ class Case:
         import paper_2512_08061_gb300.luna as L
         lu = L.Luna(self.B, self.H, self.n, self.d, self.dv, self.M, self.L, self.hidden, self.causal, self.eps,
                     torch.float32 if self.io == "f32" else torch.bfloat16, chunk, shared=self.shared,
-                    ch_rms_target=self.ch_rms_target, signed=self.signed, per_head=self.per_head)
+                    ch_rms_target=self.ch_rms_target, signed=self.signed, per_head=self.per_head, act=self.act,
+                    envelope=self.envelope, bank_coef=self.bank_coef)
         self.guards = []
         for name in ("table", "ws", "state"):
             setattr(lu, name, guarded_bytes(getattr(lu, name).numel(), lu.device, self.guards))
@@ -157,6 +169,10 @@ class Case:
                   "db": (g + (self.M,), torch.float32), "dw1": (g + fc1, torch.float32),
                   "db1": (g + fc1, torch.float32), "dw2": (g + (self.L, self.hidden), torch.float32),
                   "db2": (g + (self.L,), torch.float32)}
+        if self.envelope:
+            shapes.update(dWe=((self.L, self.d), torch.float32), dbe=((self.L,), torch.float32))
+        if self.bank_coef:
+            shapes["dcoef"] = ((self.L,), torch.float32)
         out = {k: guarded_empty(shp, dt, dev, self.guards) for k, (shp, dt) in shapes.items()}
         g = lu.backward(d["Q"], d["K"], d["V"], d["dO"], d["lengths"], use_state=use_state, out=out)
         check_guards(self.guards)
@@ -167,9 +183,13 @@ class Case:
     def phi(self):
         """The oracle's feature map: the parameters, with the channel normalisation and the signed
         channel outputs when they are on."""
-        if self.ch_rms_target or self.signed or self.per_head:
-            return oracle.PhiParams(self.params, self.ch_rms_target, nonneg=not self.signed)
+        if self.ch_rms_target or self.signed or self.per_head or self.variant:
+            return oracle.PhiParams(self.params, self.ch_rms_target, nonneg=not self.signed, act=self.act)
         return self.params
+
+    @property
+    def variant(self) -> bool:
+        return self.act != "relu" or self.envelope or self.bank_coef
 
     def oracle_fwd(self):
         i = self.inp

@@ -191,3 +191,48 @@ def test_attention_weights_arguments(L):
     assert lib.luna_attn_weights(ctypes.byref(ad), ctypes.byref(rms), *args, 0, 5, 0, P(256), None) == 2
     assert lib.luna_attn_weights(ctypes.byref(ad), ctypes.byref(pd), None, None, None, None, 100, 0, 0, None,
                                  None) == 0
+
+
+def test_variant_descriptors(L):
+    """The feature-map variants: act in 0..3 and the envelope / bank_coef flags in {0, 1}
+    (else LUNA_ERR_INVALID_ARG); the gate's and the coefficients' parameters enlarge the
+    table; the variants do not combine with ch_rms or per-head parameters, and
+    luna_attn_weights / luna_attn_decode do not support them (all before any launch);
+    luna_phi_prepare and luna_attn_bwd require the variants' parameter and gradient
+    pointers."""
+    lib = L._lib
+    P = ctypes.c_void_p
+    for kw in ({"act": 4}, {"act": -1}, {"envelope": 2}, {"bank_coef": 3}):
+        pd = L.phi_desc(8, 8, 64)
+        for k, v in kw.items():
+            setattr(pd, k, v)
+        with pytest.raises(L.LunaError) as e:
+            L.luna_phi_table_size(pd, 32)
+        assert e.value.status == 1, kw
+    base = L.luna_phi_table_size(L.phi_desc(8, 8, 64), 32)
+    assert L.luna_phi_table_size(L.phi_desc(8, 8, 64, act="gelu"), 32) == base
+    assert L.luna_phi_table_size(L.phi_desc(8, 8, 64, envelope=True), 32) >= base + 4 * 8 * 32
+    assert L.luna_phi_table_size(L.phi_desc(8, 8, 64, bank_coef=True), 32) >= base  # 8 floats: may fit the padding
+    for kw in ({"act": "tanh"}, {"envelope": True}, {"bank_coef": True}):
+        with pytest.raises(L.LunaError) as e:
+            L.luna_phi_table_size(L.phi_desc(8, 8, 64, ch_rms_target=0.1, **kw), 32)
+        assert e.value.status == 2, kw
+        with pytest.raises(L.LunaError) as e:
+            L.luna_phi_table_size(L.phi_desc(8, 8, 64, param_head_stride=1 << 20, **kw), 32)
+        assert e.value.status == 2, kw
+        pd = L.phi_desc(8, 8, 64, **kw)
+        ad = L.attn_desc(2, 2, 100, 32, 32)
+        assert lib.luna_attn_weights(ctypes.byref(ad), ctypes.byref(pd), P(256), P(256), P(256), None, 0, 5, 0,
+                                     P(256), None) == 2
+        dec = L.attn_desc(2, 4, 1, 32, 32, True)
+        assert lib.luna_attn_decode(ctypes.byref(dec), ctypes.byref(pd), None, None, None, None, None, None, 0, None,
+                                    0, None) == 2
+        assert L.luna_workspace_size(ad, pd, True) >= L.luna_workspace_size(ad, pd, False) > 0
+    # prepare without the gate's parameters, backward without its gradients: argument errors
+    pd = L.phi_desc(8, 8, 64, envelope=True)
+    pp = L.PhiParams(*([P(256)] * 6 + [None, None, None]))
+    assert lib.luna_phi_prepare(ctypes.byref(pd), 32, ctypes.byref(pp), P(256), 1 << 20, None) == 1
+    ad = L.attn_desc(2, 2, 64, 32, 32)
+    pg = L.PhiGrads(*([P(256)] * 6 + [None, None, None]))
+    assert lib.luna_attn_bwd(ctypes.byref(ad), ctypes.byref(pd), P(256), P(256), P(256), P(256), P(256), None, None,
+                             P(256), P(256), P(256), ctypes.byref(pg), P(256), 1 << 30, None) == 1

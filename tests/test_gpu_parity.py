@@ -12,7 +12,8 @@ import pytest
 
 import oracle
 import synth
-from cases import TOL, Case, relerr, relerr_rows, run_in_child, to_device, to_host
+from cases import (TOL, Case, check_guards, guarded_bytes, guarded_empty, relerr, relerr_rows, run_in_child, to_device,
+                   to_host)
 
 pytestmark = pytest.mark.gpu
 
@@ -739,3 +740,69 @@ def test_per_head_parameters_decode_and_weights():
     L.luna_attn_weights(lu2.ad, lu2.pd, lu2.table, case.dev["Q"], case.dev["K"], None, 0, n, False, A)
     ref = oracle.attn_weights(case.phi, case.inp["Q"].value, case.inp["K"].value, None, True, case.eps)
     assert relerr(to_host(A), ref) < 1e-4
+
+
+# the feature-map variants: (activation, envelope gate, Bank+Coef, shared-channel MLP)
+VARIANTS = {
+    "gelu": ("gelu", False, False, False),
+    "silu": ("silu", False, False, False),
+    "tanh": ("tanh", False, False, False),
+    "tanh-shared": ("tanh", False, False, True),
+    "envelope": ("relu", True, False, False),
+    "coef": ("relu", False, True, False),
+    "gelu+envelope+coef": ("gelu", True, True, False),
+}
+
+
+@pytest.mark.parametrize("io,causal", [("f32", False), ("f32", True), ("bf16", False), ("bf16", True)])
+@pytest.mark.parametrize("name", sorted(VARIANTS))
+def test_feature_map_variants(name, io, causal):
+    """The kernel ablation's feature maps (Sec. 5.4, Table 5) and the channel MLPs' activation on the
+    generic kernels, forward and backward (every parameter gradient, the gate's and the coefficients'
+    included), against the oracle: direct evaluation of GELU / SiLU / tanh MLPs, the envelope gate
+    sigmoid(We x + be) and the Bank+Coef coefficients; ragged lengths over several 16- and 32-row
+    tiles."""
+    act, env, coef, shared = VARIANTS[name]
+    d, M = 32, 8
+    seed = 300 + sorted(VARIANTS).index(name)
+    case = Case(2, 2, 150, d, M, 8, io, causal, seed=seed, qkv_scale=1.0 / math.sqrt(d), lengths=[150, 71],
+                with_grad=True, shared=shared, act=act, envelope=env, bank_coef=coef)
+    phiq = oracle.featmap(case.phi, case.inp["Q"].value)
+    assert np.mean(phiq > 0) > 0.1  # the map is not dead
+    lu = case.luna()
+    O = to_host(case.run_fwd(lu))
+    ref = case.oracle_fwd()
+    assert (relerr_rows(O, ref) if causal else relerr(O, ref)) < TOL[io]
+    g = {k: to_host(v) for k, v in case.run_bwd(lu).items()}
+    rb = case.oracle_bwd()
+    okq, okk = case.smooth_rows("Q"), case.smooth_rows("K")
+    assert okq.mean() > 0.9 and okk.mean() > 0.9
+    assert relerr(g["dQ"][okq], rb["dQ"][okq]) < TOL[io]
+    assert relerr(g["dK"][okk], rb["dK"][okk]) < TOL[io]
+    assert relerr(g["dV"], rb["dV"]) < TOL[io]
+    keys = ["dW", "db", "dw1", "db1", "dw2", "db2"] + (["dWe", "dbe"] if env else []) + (["dcoef"] if coef else [])
+    for k in keys:
+        assert relerr(g[k], rb[k]) < TOL[io], k
+
+
+@pytest.mark.parametrize("name", sorted(VARIANTS))
+def test_feature_map_variants_featmap(name):
+    """luna_featmap of every variant, fp32 and bf16 rows, against the oracle's feature map."""
+    import torch
+    import paper_2512_08061_gb300.luna as L
+    act, env, coef, shared = VARIANTS[name]
+    d, M = 64, 8
+    seed = 320 + sorted(VARIANTS).index(name)
+    case = Case(1, 1, 8, d, M, 8, "f32", seed=seed, qkv_scale=1.0 / math.sqrt(d), shared=shared, act=act,
+                envelope=env, bank_coef=coef)
+    pd = L.phi_desc(M, 8, 64, shared, act=act, envelope=env, bank_coef=coef)
+    guards = []
+    table = guarded_bytes(L.luna_phi_table_size(pd, d), "cuda", guards)
+    L.luna_phi_prepare(pd, d, {k: torch.from_numpy(v).cuda() for k, v in case.params.items()}, table)
+    for io in ("f32", "bf16"):
+        X = synth.IOTensor(synth.normal(seed, "var.X", (333, d)) / math.sqrt(d), io)
+        Phi = guarded_empty((333, M * 8), torch.float32, "cuda", guards)
+        L.luna_featmap(pd, d, table, to_device(X), Phi)
+        check_guards(guards)
+        ref = oracle.featmap(case.phi, X.value)
+        assert relerr(to_host(Phi), ref) < 1e-4, io
