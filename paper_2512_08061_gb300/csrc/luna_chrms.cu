@@ -66,61 +66,86 @@ __device__ double block_sum(double v, double *sh) {
 }
 
 // Sum of phi^2 per channel over the valid rows and every projection of one side (blockIdx.y: 0 = Q,
-// 1 = K): one thread per (row, projection) item in a grid-stride loop, no block barriers in the loop;
-// block partials at part[(side * gridDim.x + blockIdx.x) * L + l].  W sits transposed in shared
-// memory (WT[c][i]), so the lanes of a row, which differ in i, read consecutive words.
+// 1 = K): one thread per row in a grid-stride loop, all M projections of the row in registers, no block
+// barriers in the loop; block partials at part[(side * gridDim.x + blockIdx.x) * L + l].  W sits
+// transposed in shared memory, padded to kStatMP columns (WT[c][i]): every lane of a warp reads the same
+// four-word group at once (a broadcast), so the projections cost one shared load per four FMAs.  Each u_i
+// is the fp32 chain b_i + sum_c W_ic x_c in order of c; the interval comes from the bucketed search block.
+constexpr int kStatMP = 32;  // projections held per row (M <= 32)
 template <typename IO, bool VEC>
 __global__ void __launch_bounds__(kThreads) k_chrms_stats(AttnArgs a, float *part) {
     extern __shared__ __align__(16) float smem[];
     const TableLayout &lay = a.lay;
-    const int d = a.d, M = a.M, L = a.L, P = lay.Ppad;
-    float *sT = smem;
-    float *sAB = sT + r4(P);
-    float *sWT = sAB + r4(lay.nint * L * 2);
-    float *sb = sWT + r4(M * d);
-    float *sred = sb + r4(M);
+    const int d = a.d, M = a.M, L = a.L;
+    float *sS = smem;                          // the interval search block
+    float *sAB = sS + kEytzinger;
+    float *sWT = sAB + r4(lay.nint * L * 2);   // [d][kStatMP]
+    float *sb = sWT + d * kStatMP;             // [kStatMP]
+    float *sred = sb + kStatMP;
     {
-        const float *T = reinterpret_cast<const float *>(a.table + lay.off_T);
+        const float *S = reinterpret_cast<const float *>(a.table + lay.off_Te);
         const float *AB = reinterpret_cast<const float *>(a.table + lay.off_AB);
         const float *W = reinterpret_cast<const float *>(a.table + lay.off_W);
         const float *b = reinterpret_cast<const float *>(a.table + lay.off_b);
-        for (int e = threadIdx.x; e < P; e += blockDim.x) sT[e] = T[e];
+        for (int e = threadIdx.x; e < kEytzinger; e += blockDim.x) sS[e] = S[e];
         for (int e = threadIdx.x; e < lay.nint * L * 2; e += blockDim.x) sAB[e] = AB[e];
-        for (int e = threadIdx.x; e < M * d; e += blockDim.x) sWT[(e % d) * M + e / d] = W[e];
-        for (int e = threadIdx.x; e < M; e += blockDim.x) sb[e] = b[e];
+        for (int e = threadIdx.x; e < d * kStatMP; e += blockDim.x) {
+            const int c = e / kStatMP, i = e - c * kStatMP;
+            sWT[e] = i < M ? W[i * d + c] : 0.0f;
+        }
+        for (int e = threadIdx.x; e < kStatMP; e += blockDim.x) sb[e] = e < M ? b[e] : 0.0f;
     }
     __syncthreads();
+    const unsigned short *sB = reinterpret_cast<const unsigned short *>(sS + kSearchT);
     const int side = blockIdx.y;
     const IO *X = static_cast<const IO *>(side ? a.K : a.Q);
-    const int64_t items = (int64_t)a.B * a.H * a.n * M;
+    const int64_t rows = (int64_t)a.B * a.H * a.n;
     float acc[kMaxL];
 #pragma unroll
     for (int l = 0; l < kMaxL; ++l) acc[l] = 0.0f;
-    for (int64_t e = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; e < items; e += (int64_t)gridDim.x * blockDim.x) {
-        const int64_t row = e / M;
-        const int i = (int)(e - row * M);
+    // the projections of one input column: u_i += W_ic x_c for the groups of four with a live projection
+    auto column = [&](float (&u)[kStatMP], int c, float xc) {
+        const float4 *w = reinterpret_cast<const float4 *>(sWT + c * kStatMP);
+#pragma unroll
+        for (int q = 0; q < kStatMP / 4; ++q)
+            if (4 * q < M) {
+                const float4 ww = w[q];
+                u[4 * q] = fmaf(ww.x, xc, u[4 * q]);
+                u[4 * q + 1] = fmaf(ww.y, xc, u[4 * q + 1]);
+                u[4 * q + 2] = fmaf(ww.z, xc, u[4 * q + 2]);
+                u[4 * q + 3] = fmaf(ww.w, xc, u[4 * q + 3]);
+            }
+    };
+    for (int64_t row = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; row < rows;
+         row += (int64_t)gridDim.x * blockDim.x) {
         const int64_t bh = row / a.n;
         if ((int)(row - bh * a.n) >= head_length(a.lengths, (int)(bh / a.H), a.n)) continue;
         const IO *x = X + row * d;
-        float u = sb[i];
+        float u[kStatMP];
+#pragma unroll
+        for (int i = 0; i < kStatMP; ++i) u[i] = sb[i];
         if (VEC) {  // 16-byte loads: 8 bf16 or 4 fp32 values
             constexpr int V = 16 / sizeof(IO);
             for (int c0 = 0; c0 < d; c0 += V) {
                 const uint4 raw = __ldg(reinterpret_cast<const uint4 *>(x + c0));
                 const IO *v = reinterpret_cast<const IO *>(&raw);
 #pragma unroll
-                for (int k = 0; k < V; ++k) u = fmaf(sWT[(c0 + k) * M + i], io_load(v + k), u);
+                for (int k = 0; k < V; ++k) column(u, c0 + k, io_load(v + k));
             }
         } else {
-            for (int c = 0; c < d; ++c) u = fmaf(sWT[c * M + i], io_load(x + c), u);
+            for (int c = 0; c < d; ++c) column(u, c, io_load(x + c));
         }
-        const float *ab = sAB + interval_of(sT, P, u) * L * 2;
 #pragma unroll
-        for (int l = 0; l < kMaxL; ++l)
-            if (l < L) {
-                const float y = fmaxf(fmaf(ab[2 * l], u, ab[2 * l + 1]), 0.0f);
-                acc[l] = fmaf(y, y, acc[l]);
-            }
+        for (int i = 0; i < kStatMP; ++i) {
+            if (i >= M) break;
+            const float *ab = sAB + interval_bucketed(sS, sB, u[i]) * L * 2;
+#pragma unroll
+            for (int l = 0; l < kMaxL; ++l)
+                if (l < L) {
+                    const float y = fmaxf(fmaf(ab[2 * l], u[i], ab[2 * l + 1]), 0.0f);
+                    acc[l] = fmaf(y, y, acc[l]);
+                }
+        }
     }
 #pragma unroll
     for (int l = 0; l < kMaxL; ++l) {
@@ -363,7 +388,7 @@ __global__ void k_chrms_scale_hist(double *gsum, TableLayout lay, const float *s
 }
 
 size_t smem_stats(const AttnArgs &a) {
-    return (size_t)(r4(a.lay.Ppad) + r4(a.lay.nint * a.lay.L * 2) + r4(a.M * a.d) + r4(a.M) + kThreads) * 4;
+    return (size_t)(kEytzinger + r4(a.lay.nint * a.lay.L * 2) + a.d * kStatMP + kStatMP + kThreads) * 4;
 }
 // shared memory of the scale-term pass with block sums of GP (gp_words: 4-byte words per GP)
 size_t smem_kterm(const AttnArgs &a, int gp_words = 2) {

@@ -636,7 +636,7 @@ __global__ void __launch_bounds__(kThreadsTC, 1)
                 fence_proxy_async_smem();
                 tc_fence_before();
                 mbar_arrive(phiready + p);
-                named_sync<kWorkers>(1);  // all four parts of every row's normaliser are written
+                quarter_sync(warp);  // all four parts of this quarter's rows' normalisers are written
                 // read now: the slot is written again two tiles on, after the next tile's barrier
                 const float dsum = dslot[r] + dslot[128 + r] + dslot[256 + r] + dslot[384 + r] + a.eps;
                 if (pend_g >= 0) o_out(pend_g, pend_row, pend_dsum);

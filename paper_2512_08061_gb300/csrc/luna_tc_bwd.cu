@@ -337,7 +337,7 @@ __global__ void __launch_bounds__(kBThreads, 1)
                     float *rs = sred + (g & 1) * (C::SRED / 2);
                     rs[H * 128 + r] = denp;
                     rs[kBRowThreads * 128 + H * 128 + r] = dotp;
-                    named_sync<kBWorkers>(1);
+                    quarter_sync(warp);  // the parts of this quarter's rows
                     float den = a.eps, dotn = 0.0f;  // dotn = (dO.O) * den; parts added in a fixed order
 #pragma unroll
                     for (int h = 0; h < kBRowThreads; ++h) {

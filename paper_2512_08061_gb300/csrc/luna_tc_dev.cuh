@@ -73,6 +73,12 @@ __device__ __forceinline__ void named_sync(int id) {
     asm volatile("bar.sync %0, %1;" ::"r"(id), "r"(N) : "memory");
 }
 
+// Barrier of the four worker warps w, w + 4, w + 8, w + 12 that share TMEM lane quarter w % 4 (the threads
+// of the same rows): named barriers 3..6, so that the quarters of a tile run independently.
+__device__ __forceinline__ void quarter_sync(int warp) {
+    asm volatile("bar.sync %0, 128;" ::"r"(3 + (warp & 3)) : "memory");
+}
+
 // Adds a byte offset to the start-address field of a shared-memory descriptor.
 __device__ __forceinline__ uint64_t dadd(uint64_t desc, uint32_t bytes) { return desc + (bytes >> 4); }
 
