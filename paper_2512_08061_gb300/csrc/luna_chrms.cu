@@ -79,16 +79,15 @@ __global__ void __launch_bounds__(kThreads) k_chrms_stats(AttnArgs a, float *par
     const int d = a.d, M = a.M, L = a.L;
     float *sS = smem;                          // the interval search block
     float *sAB = sS + kEytzinger;
-    float *sWT = sAB + r4(lay.nint * L * 2);   // [d][kStatMP]
+    float *sWT = sAB + r4(lay.nint * ab_stride(lay));  // [d][kStatMP]
     float *sb = sWT + d * kStatMP;             // [kStatMP]
     float *sred = sb + kStatMP;
     {
         const float *S = reinterpret_cast<const float *>(a.table + lay.off_Te);
-        const float *AB = reinterpret_cast<const float *>(a.table + lay.off_AB);
         const float *W = reinterpret_cast<const float *>(a.table + lay.off_W);
         const float *b = reinterpret_cast<const float *>(a.table + lay.off_b);
         for (int e = threadIdx.x; e < kEytzinger; e += blockDim.x) sS[e] = S[e];
-        for (int e = threadIdx.x; e < lay.nint * L * 2; e += blockDim.x) sAB[e] = AB[e];
+        copy_ab(sAB, lay, a.table);
         for (int e = threadIdx.x; e < d * kStatMP; e += blockDim.x) {
             const int c = e / kStatMP, i = e - c * kStatMP;
             sWT[e] = i < M ? W[i * d + c] : 0.0f;
@@ -138,11 +137,12 @@ __global__ void __launch_bounds__(kThreads) k_chrms_stats(AttnArgs a, float *par
 #pragma unroll
         for (int i = 0; i < kStatMP; ++i) {
             if (i >= M) break;
-            const float *ab = sAB + interval_bucketed(sS, sB, u[i]) * L * 2;
+            const float *ab = sAB + interval_bucketed(sS, sB, u[i]) * ab_stride(lay);
 #pragma unroll
             for (int l = 0; l < kMaxL; ++l)
                 if (l < L) {
-                    const float y = fmaxf(fmaf(ab[2 * l], u[i], ab[2 * l + 1]), 0.0f);
+                    const float2 p = ab_pair(ab, l);
+                    const float y = fmaxf(fmaf(p.x, u[i], p.y), 0.0f);
                     acc[l] = fmaf(y, y, acc[l]);
                 }
         }
@@ -276,7 +276,7 @@ __global__ void __launch_bounds__(kKWarps * 32) k_chrms_kterm(AttnArgs a, const 
     const int side = blockIdx.y;
     float *sT = smem;
     float *sAB = sT + r4(P);
-    float *sW = sAB + r4(NH);
+    float *sW = sAB + r4(lay.nint * ab_stride(lay));
     float *sb = sW + r4(M * d);
     GP *sdW = reinterpret_cast<GP *>(sb + r4(M));  // block sums of dW, db in the partials' type
     GP *sdb = sdW + r4(M * d);
@@ -289,11 +289,11 @@ __global__ void __launch_bounds__(kKWarps * 32) k_chrms_kterm(AttnArgs a, const 
     GP *ghist = gp + Md + M;
     {
         const float *T = reinterpret_cast<const float *>(a.table + lay.off_T);
-        const float *AB = reinterpret_cast<const float *>(a.table + lay.off_AB);
         const float *W = reinterpret_cast<const float *>(a.table + lay.off_W);
         const float *b = reinterpret_cast<const float *>(a.table + lay.off_b);
         for (int e = threadIdx.x; e < P; e += blockDim.x) sT[e] = T[e];
-        for (int e = threadIdx.x; e < NH; e += blockDim.x) { sAB[e] = AB[e]; ghist[e] = (GP)0; }
+        copy_ab(sAB, lay, a.table);
+        for (int e = threadIdx.x; e < NH; e += blockDim.x) ghist[e] = (GP)0;
         for (int e = threadIdx.x; e < M * d; e += blockDim.x) { sW[e] = W[e]; sdW[e] = (GP)0; }
         for (int e = threadIdx.x; e < M; e += blockDim.x) { sb[e] = b[e]; sdb[e] = (GP)0; }
         if ((int)threadIdx.x < L) sk[threadIdx.x] = kappa[side * kMaxL + threadIdx.x] * (float)M;
@@ -324,13 +324,14 @@ __global__ void __launch_bounds__(kKWarps * 32) k_chrms_kterm(AttnArgs a, const 
                 float u = sb[i];
                 for (int c = 0; c < d; ++c) u = fmaf(w[c], x[c], u);
                 const int j = interval_of(sT, P, u);
-                const float *ab = sAB + j * L * 2;
+                const float *ab = sAB + j * ab_stride(lay);
                 GP *h = ghist + j * L * 2;
                 for (int l = 0; l < L; ++l) {
-                    const float ph = fmaxf(fmaf(ab[2 * l], u, ab[2 * l + 1]), 0.0f);
+                    const float2 p = ab_pair(ab, l);
+                    const float ph = fmaxf(fmaf(p.x, u, p.y), 0.0f);
                     if (ph > 0.0f) {  // outer ReLU on
                         const float g = sk[l] * ph;
-                        du = fmaf(g, ab[2 * l], du);
+                        du = fmaf(g, p.x, du);
                         if (g != 0.0f) {
                             atomicAdd(h + 2 * l, (GP)g);
                             atomicAdd(h + 2 * l + 1, (GP)g * (GP)u);
@@ -388,12 +389,11 @@ __global__ void k_chrms_scale_hist(double *gsum, TableLayout lay, const float *s
 }
 
 size_t smem_stats(const AttnArgs &a) {
-    return (size_t)(kEytzinger + r4(a.lay.nint * a.lay.L * 2) + a.d * kStatMP + kStatMP + kThreads) * 4;
+    return (size_t)(kEytzinger + r4(a.lay.nint * ab_stride(a.lay)) + a.d * kStatMP + kStatMP + kThreads) * 4;
 }
 // shared memory of the scale-term pass with block sums of GP (gp_words: 4-byte words per GP)
 size_t smem_kterm(const AttnArgs &a, int gp_words = 2) {
-    const int NH = a.lay.nint * a.L * 2;
-    return (size_t)(r4(a.lay.Ppad) + r4(NH) + (1 + gp_words) * (r4(a.M * a.d) + r4(a.M)) + r4(kMaxL) +
+    return (size_t)(r4(a.lay.Ppad) + r4(a.lay.nint * ab_stride(a.lay)) + (1 + gp_words) * (r4(a.M * a.d) + r4(a.M)) + r4(kMaxL) +
                     kKWarps * (r4(32 * (a.d + 1)) + r4(32 * (a.M + 1)))) * 4;
 }
 

@@ -121,6 +121,11 @@ __host__ __device__ inline TableLayout table_layout(int M, int L, int hid, int d
     return t;
 }
 
+// Words per interval of the (alpha, beta) table in shared memory (generic kernels): 2L + 2 instead of 2L,
+// so that the entries of lanes at random intervals start in 16 different 8-byte bank pairs (a 64-byte
+// stride at L = 8 would put every entry in one of two) and each (alpha, beta) pair is one aligned 8-byte load.
+__host__ __device__ __forceinline__ int ab_stride(const TableLayout &lay) { return 2 * lay.L + 2; }
+
 // One of the feature-map variants (a non-ReLU activation, the envelope gate, Bank+Coef): generic kernels only.
 __host__ __device__ __forceinline__ bool lay_variant(const TableLayout &lay) { return lay.act || lay.env || lay.coef; }
 

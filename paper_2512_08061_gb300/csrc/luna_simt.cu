@@ -40,9 +40,12 @@ __global__ void __launch_bounds__(kThreads) k_featmap(TableLayout lay, const cha
         float u = s.b[i];
         for (int c = 0; c < d; ++c) u = fmaf(w[c], io_load(x + c), u);
         const int j = interval_bucketed(sS, sB, u);
-        const float *ab = s.AB + j * L * 2;
+        const float *ab = s.AB + j * ab_stride(lay);
         float *out = Phi + r * D + i * L;
-        for (int l = 0; l < L; ++l) out[l] = fmaxf(fmaf(ab[2 * l], u, ab[2 * l + 1]), channel_floor(lay));
+        for (int l = 0; l < L; ++l) {
+            const float2 p = ab_pair(ab, l);
+            out[l] = fmaxf(fmaf(p.x, u, p.y), channel_floor(lay));
+        }
     }
 }
 

@@ -54,7 +54,7 @@ __device__ SmemPhi carve_phi(Carve &cv, const TableLayout &lay) {
     SmemPhi s = {};
     if (!lay.act) {
         s.T = cv.take(lay.Ppad);
-        s.AB = cv.take(lay.nint * lay.L * 2);
+        s.AB = cv.take(lay.nint * ab_stride(lay));
     }
     s.W = cv.take(lay.M * lay.d);
     s.b = cv.take(lay.M);
@@ -69,13 +69,23 @@ __device__ SmemPhi carve_phi(Carve &cv, const TableLayout &lay) {
     return s;
 }
 void carve_phi_host(HostCarve &cv, const TableLayout &lay) {
-    if (!lay.act) { cv.take(lay.Ppad); cv.take(lay.nint * lay.L * 2); }
+    if (!lay.act) { cv.take(lay.Ppad); cv.take(lay.nint * ab_stride(lay)); }
     cv.take(lay.M * lay.d); cv.take(lay.M);
     if (lay.act) { cv.take(lay.P); cv.take(lay.P); cv.take(lay.L * lay.hid); cv.take(lay.L); }
     if (lay.env) { cv.take(lay.L * lay.d); cv.take(lay.L); }
     if (lay.coef) cv.take(lay.L);
     if (lay.env || lay.coef) { cv.take(kPhiRows * lay.L); cv.take(kPhiRows * lay.L); cv.take(kPhiRows * lay.L); }
 }
+
+// The (alpha, beta) table into shared memory at ab_stride(lay) words per interval.
+__device__ void copy_ab(float *dst, const TableLayout &lay, const char *table) {
+    const float *src = reinterpret_cast<const float *>(table + lay.off_AB);
+    const int w = 2 * lay.L, st = ab_stride(lay);
+    for (int e = threadIdx.x; e < lay.nint * w; e += blockDim.x) dst[(e / w) * st + e % w] = src[e];
+}
+
+// (alpha, beta) of channel l in the entry of one interval.
+__device__ __forceinline__ float2 ab_pair(const float *entry, int l) { return reinterpret_cast<const float2 *>(entry)[l]; }
 
 __device__ void load_phi(const SmemPhi &s, const TableLayout &lay, const char *table) {
     auto copy = [&](float *dst, int64_t off, int count) {
@@ -84,7 +94,7 @@ __device__ void load_phi(const SmemPhi &s, const TableLayout &lay, const char *t
     };
     if (!lay.act) {
         copy(s.T, lay.off_T, lay.Ppad);
-        copy(s.AB, lay.off_AB, lay.nint * lay.L * 2);
+        copy_ab(s.AB, lay, table);
     }
     copy(s.W, lay.off_W, lay.M * lay.d);
     copy(s.b, lay.off_b, lay.M);
@@ -147,8 +157,8 @@ __device__ __forceinline__ float channel_direct(const TableLayout &lay, const Sm
 __device__ __forceinline__ float channel_value(const TableLayout &lay, const SmemPhi &s, float u, int j, int l,
                                                float fl) {
     if (lay.act) return fmaxf(phi_scale(lay) * channel_direct(lay, s, l, u, nullptr), fl);
-    const float *ab = s.AB + j * lay.L * 2;
-    return fmaxf(fmaf(ab[2 * l], u, ab[2 * l + 1]), fl);
+    const float2 ab = ab_pair(s.AB + j * ab_stride(lay), l);
+    return fmaxf(fmaf(ab.x, u, ab.y), fl);
 }
 
 // Per-row factors of the variants for rows [0, nr) of sX: H = h_l(x) = sigmoid(We_l . x + be_l) (1 without the
@@ -197,8 +207,11 @@ __device__ void phi_tile(const TableLayout &lay, const SmemPhi &s, const float *
         int j = 0;
         if (!lay.act) {
             j = interval_of(s.T, lay.Ppad, u);
-            const float *ab = s.AB + j * L * 2;
-            for (int l = 0; l < L; ++l) out[l] = fmaxf(fmaf(ab[2 * l], u, ab[2 * l + 1]), fl);
+            const float *ab = s.AB + j * ab_stride(lay);
+            for (int l = 0; l < L; ++l) {
+                const float2 p = ab_pair(ab, l);
+                out[l] = fmaxf(fmaf(p.x, u, p.y), fl);
+            }
         } else {
             for (int l = 0; l < L; ++l) out[l] = fmaxf(sc * channel_direct(lay, s, l, u, nullptr), fl);
         }
@@ -334,13 +347,14 @@ __device__ void phi_backward_tile(const TableLayout &lay, const SmemPhi &s, cons
         double du = 0.0;
         if (!lay.act) {
             const int j = sJ[e];
-            const float *ab = s.AB + j * L * 2;
+            const float *ab = s.AB + j * ab_stride(lay);
             for (int l = 0; l < L; ++l) {
                 const int f = r * D + i * L + l;
-                const bool on = ev ? fmaf(ab[2 * l], u, ab[2 * l + 1]) > fl : sPhi[f] > fl;
+                const float2 p = ab_pair(ab, l);
+                const bool on = ev ? fmaf(p.x, u, p.y) > fl : sPhi[f] > fl;
                 if (on) {  // outer ReLU on (always, for signed outputs)
                     const double gl = ev ? (double)sdPhi[f] * (double)s.E[r * L + l] : (double)sdPhi[f];
-                    du = fma(gl, (double)ab[2 * l], du);
+                    du = fma(gl, (double)p.x, du);
                     if (gl != 0.0) {
                         atomicAdd(shist + (j * L + l) * 2, gl);
                         atomicAdd(shist + (j * L + l) * 2 + 1, gl * (double)u);  // exact product
