@@ -216,6 +216,12 @@ __global__ void __launch_bounds__(kBThreads, 1)
                 wait_or_fail(gready + (g & 1), (g >> 1) & 1, failed, status);
                 if (g >= 1) wait_or_fail(dqfree, (g - 1) & 1, failed, status);
                 tc_fence_after();
+                // dQ = G W first, its barrier committed at once: the workers read it out during the next tile
+                constexpr uint32_t idQ = idesc_bf16(128, C::d, false, false);
+#pragma unroll
+                for (int k = 0; k < 2; ++k)
+                    mma_bf16_ss(tbase + cQ, dadd(dO0, o * T16 + 64 + 32 * k), dadd(dWx, 32 * k), idQ, k != 0);
+                mma_commit(dqready);
                 // [phi/den hi, lo]^T G: dS (cols 0..31) and dz (cols 56, 57) of every feature, once as hi, once as lo
                 constexpr uint32_t idG = idesc_bf16(128, 64, true, true);
 #pragma unroll
@@ -228,11 +234,6 @@ __global__ void __launch_bounds__(kBThreads, 1)
                 for (int k = 0; k < 8; ++k)
                     mma_bf16_ss(tbase + cW, dadd(dS0, s * 3 * T16 + 2 * T16 + 2048 * k),
                                 dadd(dO0, o * T16 + 64 + 2048 * k), idW, (g > 0 || k > 0) ? 1u : 0u);
-                constexpr uint32_t idQ = idesc_bf16(128, C::d, false, false);
-#pragma unroll
-                for (int k = 0; k < 2; ++k)
-                    mma_bf16_ss(tbase + cQ, dadd(dO0, o * T16 + 64 + 32 * k), dadd(dWx, 32 * k), idQ, k != 0);
-                mma_commit(dqready);
                 mma_commit(ofree + o);
                 mma_commit(sfree + s);
                 ++tile_in_run;
@@ -684,12 +685,12 @@ __global__ void __launch_bounds__(kBThreads, 1)
 #pragma unroll
                 for (int k = 0; k < 2; ++k)
                     mma_bf16_ss(tbase + cK, dadd(dG, 32 * k), dadd(dWx, 32 * k), idK, k != 0);
+                mma_commit(dkready);  // before the dW^T products: the workers read dK out during the next tile
                 constexpr uint32_t idW = idesc_bf16(64, 16, true, true);
 #pragma unroll
                 for (int k = 0; k < 8; ++k)
                     mma_bf16_ss(tbase + cW, dadd(dS0, s * 2 * T16 + T16 + 2048 * k), dadd(dG, 2048 * k), idW,
                                 (g > 0 || k > 0) ? 1u : 0u);
-                mma_commit(dkready);
                 mma_commit(gfree);
                 mma_commit(sfree + s);
                 if (next_new_run) { wait_or_fail(opready, op_phase++ & 1, failed, status); fmma(g + 1); }

@@ -202,6 +202,11 @@ __global__ void __launch_bounds__(kBThreads, 1)
                 wait_or_fail(gready, g & 1, failed, status);
                 if (g >= 1) wait_or_fail(dqfree, (g - 1) & 1, failed, status);
                 tc_fence_after();
+                // dQ = [dU_hi | dU_lo | dU_hi | 0] W first, its barrier committed at once
+                constexpr uint32_t idQ = idesc_bf16(128, C::d, false, false);
+#pragma unroll
+                for (int k = 0; k < 2; ++k) mma_bf16_ss(tbase + cQ, dadd(dG, 32 * k), dadd(dWx, 32 * k), idQ, k != 0);
+                mma_commit(dqready);
                 const uint32_t acc = (tile_in_run > 0) ? 1u : 0u;
                 // dS += [phi/den hi, lo]^T dO ;  dz += [phi/den hi, lo]^T G (columns 32..47)
                 constexpr uint32_t idS = idesc_bf16(128, C::DV, true, true);
@@ -219,11 +224,6 @@ __global__ void __launch_bounds__(kBThreads, 1)
                 for (int k = 0; k < 8; ++k)
                     mma_bf16_ss(tbase + cW, dadd(dQt, s * T16 + 2048 * k), dadd(dG, 2048 * k), idW,
                                 (g > 0 || k > 0) ? 1u : 0u);
-                // dQ = [dU_hi | dU_lo | dU_hi | 0] W
-                constexpr uint32_t idQ = idesc_bf16(128, C::d, false, false);
-#pragma unroll
-                for (int k = 0; k < 2; ++k) mma_bf16_ss(tbase + cQ, dadd(dG, 32 * k), dadd(dWx, 32 * k), idQ, k != 0);
-                mma_commit(dqready);
                 mma_commit(ofree + o);
                 mma_commit(qfree + s);
                 ++tile_in_run;
@@ -666,12 +666,12 @@ __global__ void __launch_bounds__(kBThreads, 1)
                 constexpr uint32_t idK = idesc_bf16(128, C::d, false, false);
 #pragma unroll
                 for (int k = 0; k < 2; ++k) mma_bf16_ss(tbase + cK, dadd(dG, 32 * k), dadd(dWx, 32 * k), idK, k != 0);
+                mma_commit(dkready);  // before the dW^T products: the workers read dK out sooner
                 constexpr uint32_t idW = idesc_bf16(64, 16, true, true);
 #pragma unroll
                 for (int k = 0; k < 8; ++k)
                     mma_bf16_ss(tbase + cW, dadd(dS0, s * 2 * T16 + T16 + 2048 * k), dadd(dG, 2048 * k), idW,
                                 (g > 0 || k > 0) ? 1u : 0u);
-                mma_commit(dkready);
                 mma_commit(gfree);
                 mma_commit(sfree + s);
                 // the workers have read dphi(g) (before gready): dphi of the next tile

@@ -163,12 +163,12 @@ __global__ void __launch_bounds__(kBThreads, 1)
                 constexpr uint32_t idX = idesc_bf16(128, C::d, false, false);
 #pragma unroll
                 for (int k = 0; k < 4; ++k) mma_bf16_ss(tbase + cX, dadd(dGk, 32 * k), dadd(dWx, 32 * k), idX, k != 0);
+                mma_commit(dxready);  // before the dW^T products: the workers wait for dX only
                 constexpr uint32_t idW = idesc_bf16(128, 2 * C::MP, true, true);
 #pragma unroll
                 for (int k = 0; k < 8; ++k)
                     mma_bf16_ss(tbase + cW, dadd(dXm, s * C::XT + 2048 * k), dadd(dGm, 2048 * k), idW,
                                 (g > 0 || k > 0) ? 1u : 0u);
-                mma_commit(dxready);
                 mma_commit(gfree);
                 mma_commit(xfree + s);
                 if (g + 2 < T) proj(g + 2);  // the workers read U(g) before gready
