@@ -806,3 +806,25 @@ def test_feature_map_variants_featmap(name):
         check_guards(guards)
         ref = oracle.featmap(case.phi, X.value)
         assert relerr(to_host(Phi), ref) < 1e-4, io
+
+
+@pytest.mark.parametrize("causal", [False, True])
+def test_feature_map_variants_many_blocks(causal):
+    """Every variant at once on a longer ragged problem: many work splits per head, so the
+    gate's, the coefficients' and the directly summed MLP gradients are reduced over many
+    block partials (fp32 I/O, the plain 1e-4 gate)."""
+    d, M = 32, 8
+    case = Case(2, 3, 1100, d, M, 8, "f32", causal, seed=340, qkv_scale=1.0 / math.sqrt(d), lengths=[1100, 613],
+                with_grad=True, act="silu", envelope=True, bank_coef=True)
+    lu = case.luna()
+    O = to_host(case.run_fwd(lu))
+    ref = case.oracle_fwd()
+    assert (relerr_rows(O, ref) if causal else relerr(O, ref)) < TOL["f32"]
+    g = {k: to_host(v) for k, v in case.run_bwd(lu).items()}
+    rb = case.oracle_bwd()
+    okq, okk = case.smooth_rows("Q"), case.smooth_rows("K")
+    assert relerr(g["dQ"][okq], rb["dQ"][okq]) < TOL["f32"]
+    assert relerr(g["dK"][okk], rb["dK"][okk]) < TOL["f32"]
+    assert relerr(g["dV"], rb["dV"]) < TOL["f32"]
+    for k in ("dW", "db", "dw1", "db1", "dw2", "db2", "dWe", "dbe", "dcoef"):
+        assert relerr(g[k], rb[k]) < TOL["f32"], k
