@@ -431,7 +431,18 @@ size_t chrms_max_smem(const AttnArgs &a) {
     return x > y ? x : y;
 }
 
+bool tc_chstats_supported(const AttnArgs &a, luna_dtype io);
+cudaError_t launch_tc_chstats(const AttnArgs &a, float *part, int max_parts, int *nparts, cudaStream_t s);
+
 cudaError_t launch_chrms_stats(const AttnArgs &a, luna_dtype io, cudaStream_t s) {
+    if (tc_chstats_supported(a, io)) {  // the projections on tensor cores (luna_tc_chstats.cu)
+        int nparts = 0;
+        cudaError_t e = launch_tc_chstats(a, a.ch_part, kChStatBlocks, &nparts, s);
+        if (e != cudaSuccess) return e;
+        LUNA_LAUNCH("chrms_scales", k_chrms_scales, 1, kRed, 0, s, a, a.ch_part, nparts, a.ch_target, a.ch_stat,
+                    a.ch_sigma);
+        return cudaGetLastError();
+    }
     // 16-byte row loads when every row starts on a 16-byte boundary
     const size_t rb = (size_t)a.d * (io == LUNA_F32 ? 4 : 2);
     const bool vec = rb % 16 == 0 && (reinterpret_cast<uintptr_t>(a.Q) & 15) == 0 &&
