@@ -146,6 +146,7 @@ def kernel_bytes(w, lengths, kernel: str) -> float:
         # channel normalisation, both sides per launch: the statistics read every valid row of Q and K;
         # the scale-term pass reads them and reads and writes the same rows of dQ and dK
         "chrms_stats": 2 * valid * rd,
+        "tc_chstats": 2 * valid * rd,             # the same statistics with the projections on tensor cores
         "chrms_kterm": 2 * valid * 3 * rd,
     }
     # the tensor-core kernels move the same tensors as their generic counterparts
@@ -373,7 +374,8 @@ def measure_workload(args, w, dev, world, steps, ch_rms_target=0.0, with_e2e=Tru
     kernels = ["phi_prepare", "keystats", "query", "bwd_query", "bwd_key", "grad_sum", "mlp_grads",
                "causal_out", "causal_bwd_seg", "causal_dq", "causal_dkv"] + L.TC_KERNELS
     if ch_rms_target > 0:
-        kernels += ["chrms_stats", "chrms_scales", "chrms_scale", "chrms_dstate", "chrms_kappa", "chrms_kterm"]
+        kernels += ["chrms_stats", "tc_chstats", "chrms_scales", "chrms_scale", "chrms_dstate", "chrms_kappa",
+                    "chrms_kterm"]
     per_kernel = {}
     for k in kernels:
         L.luna_profile_start(k)
