@@ -148,6 +148,7 @@ def kernel_bytes(w, lengths, kernel: str) -> float:
         "chrms_stats": 2 * valid * rd,
         "tc_chstats": 2 * valid * rd,             # the same statistics with the projections on tensor cores
         "chrms_kterm": 2 * valid * 3 * rd,
+        "tc_kterm": 2 * valid * 3 * rd,           # the same scale term on tensor cores
     }
     # the tensor-core kernels move the same tensors as their generic counterparts
     for tc, generic in (("tc_keys", "keystats"), ("tc_query", "query"), ("tc_bwd_query", "bwd_query"),
@@ -375,7 +376,7 @@ def measure_workload(args, w, dev, world, steps, ch_rms_target=0.0, with_e2e=Tru
                "causal_out", "causal_bwd_seg", "causal_dq", "causal_dkv"] + L.TC_KERNELS
     if ch_rms_target > 0:
         kernels += ["chrms_stats", "tc_chstats", "chrms_scales", "chrms_scale", "chrms_dstate", "chrms_kappa",
-                    "chrms_kterm"]
+                    "chrms_kterm", "tc_kterm"]
     per_kernel = {}
     for k in kernels:
         L.luna_profile_start(k)

@@ -487,11 +487,21 @@ cudaError_t launch_chrms_kappa(const AttnArgs &a, cudaStream_t s) {
     return cudaGetLastError();
 }
 
+bool tc_kterm_supported(const AttnArgs &a);
+cudaError_t launch_tc_kterm(const AttnArgs &a, float *gpart, int max_parts, int *nparts, cudaStream_t s);
+
 cudaError_t launch_chrms_backward(const AttnArgs &a, int main_parts, int *nparts, cudaStream_t s) {
     *nparts = main_parts;
     if (!a.ch_sigma) return cudaSuccess;
     cudaError_t e = launch_chrms_kappa(a, s);
     if (e != cudaSuccess) return e;
+    if (tc_kterm_supported(a)) {  // the scale term on tensor cores (luna_tc_kterm.cu)
+        int np = 0;
+        if ((e = launch_tc_kterm(a, a.gpart + (size_t)main_parts * a.gsize, kChKBlocks, &np, s)) != cudaSuccess)
+            return e;
+        *nparts = main_parts + 2 * np;
+        return cudaSuccess;
+    }
     if (a.gpart64) {
         double *gpart = reinterpret_cast<double *>(a.gpart) + (size_t)main_parts * a.gsize;
         e = a.ch_io == LUNA_F32 ? kterm_impl<float>(a, gpart, s) : kterm_impl<__nv_bfloat16>(a, gpart, s);

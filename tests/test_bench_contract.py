@@ -71,6 +71,7 @@ def test_algorithmic_bytes_by_hand():
     assert bench.kernel_bytes(w, ln, "tc_bwd_query") == 356 * 2 * row + 512 * row + 2 * 16896
     assert bench.kernel_bytes(w, ln, "tc_bwd_key") == 356 * 2 * row + 512 * 2 * row + 16896
     assert bench.kernel_bytes(w, ln, "chrms_stats") == bench.kernel_bytes(w, ln, "tc_chstats") == 2 * 356 * row
+    assert bench.kernel_bytes(w, ln, "tc_kterm") == bench.kernel_bytes(w, ln, "chrms_kterm")
     assert bench.kernel_bytes(w, ln, "chrms_kterm") == 2 * 356 * 3 * row
     assert bench.kernel_bytes(w, ln, "no_such_kernel") == 0.0
 
