@@ -558,6 +558,30 @@ def test_channel_rms_normalisation(io, d, M, lengths, causal):
                     assert np.all(g[k][b, :, ln:] == 0)
 
 
+@pytest.mark.parametrize("d", [32, 64])
+def test_channel_rms_normalisation_many_tiles(d):
+    """The non-causal channel normalisation on the tensor-core statistics and scale-term passes with
+    more tiles than blocks (each block of a side takes several, some none) and ragged lengths that
+    end inside a tile; the scale term adds into dQ and dK, whose padded rows must stay zero."""
+    case = Case(3, 4, 1400, d, 8, 8, "bf16", False, seed=93, qkv_scale=1.0 / math.sqrt(d), lengths=[1400, 1029, 130],
+                with_grad=True)
+    case.ch_rms_target = _median_channel_rms(case)
+    lu = case.luna()
+    O = to_host(case.run_fwd(lu))
+    assert relerr(O, case.oracle_fwd()) < TOL["bf16"]
+    okq, okk = case.smooth_rows("Q"), case.smooth_rows("K")
+    rb = case.oracle_bwd()
+    g = {k: to_host(v) for k, v in case.run_bwd(lu).items()}
+    assert relerr(g["dQ"][okq], rb["dQ"][okq]) < TOL["bf16"]
+    assert relerr(g["dK"][okk], rb["dK"][okk]) < TOL["bf16"]
+    assert relerr(g["dV"], rb["dV"]) < TOL["bf16"]
+    for k in ("dW", "db", "dw1", "db1", "dw2", "db2"):
+        assert relerr(g[k], rb[k]) < TOL["bf16"], k
+    for b, ln in enumerate(case.lengths):
+        for k in ("dQ", "dK", "dV"):
+            assert np.all(g[k][b, :, ln:] == 0)
+
+
 # --------------------------------------------------------------------------
 # attention weights of a block of query rows (conversion, stage 1)
 
