@@ -53,6 +53,34 @@ __device__ __forceinline__ bool pair_less(float ta, int ka, float tb, int kb) {
     return ta < tb || (ta == tb && ka < kb);
 }
 
+// Bitonic sort of the first 2^LOGN (threshold, unit) pairs over the threads of the block, one pair per
+// thread (warp shuffles for partners within a warp, shared memory across warps; a stable total order),
+// fully unrolled for the size.  Positions at or past 2^LOGN sort among themselves.
+template <int LOGN>
+__device__ __forceinline__ void bitonic_sort(float &key, int &idx, float *sk, int *si, int tid) {
+#pragma unroll
+    for (int size = 2; size <= (1 << LOGN); size <<= 1) {
+#pragma unroll
+        for (int stride = size >> 1; stride > 0; stride >>= 1) {
+            float pk;
+            int pi;
+            if (stride >= 32) {
+                sk[tid] = key; si[tid] = idx;
+                __syncthreads();
+                pk = sk[tid ^ stride]; pi = si[tid ^ stride];
+                __syncthreads();
+            } else {
+                pk = __shfl_xor_sync(0xffffffffu, key, stride);
+                pi = __shfl_xor_sync(0xffffffffu, idx, stride);
+            }
+            // the lower position of a pair keeps the smaller element in an ascending
+            // run (the larger in a descending one); elements are distinct
+            const bool keep_min = ((tid & stride) == 0) == ((tid & size) == 0);
+            if (pair_less(pk, pi, key, idx) == keep_min) { key = pk; idx = pi; }
+        }
+    }
+}
+
 // Position of input unit `unit` (fc1 index: l*hid + k, or k when shared) in the
 // per-unit arrays, which are kept in [k][l] order (k only when shared).
 __device__ __forceinline__ int unit_pos(const TableLayout &lay, int unit) {
@@ -79,25 +107,18 @@ __global__ void __launch_bounds__(kPrepThreads) k_phi_prepare(luna_phi_params pr
         w1t[tpos] = w; b1t[tpos] = c; tyt[tpos] = ty;
     }
     for (int e = tid; e < L * hid; e += nt) w2t[(e % hid) * L + e / hid] = prm.w2[e];  // w2[l][k]
-    // bitonic sort of the first N elements (positions >= N sort among themselves)
-    for (int size = 2; size <= N; size <<= 1) {
-        for (int stride = size >> 1; stride > 0; stride >>= 1) {
-            float pk;
-            int pi;
-            if (stride >= 32) {
-                sk[tid] = key; si[tid] = idx;
-                __syncthreads();
-                pk = sk[tid ^ stride]; pi = si[tid ^ stride];
-                __syncthreads();
-            } else {
-                pk = __shfl_xor_sync(0xffffffffu, key, stride);
-                pi = __shfl_xor_sync(0xffffffffu, idx, stride);
-            }
-            // the lower position of a pair keeps the smaller element in an ascending
-            // run (the larger in a descending one); elements are distinct
-            const bool keep_min = ((tid & stride) == 0) == ((tid & size) == 0);
-            if (pair_less(pk, pi, key, idx) == keep_min) { key = pk; idx = pi; }
-        }
+    // bitonic sort of the first N elements (N a power of two, at most kMaxUnits = 512)
+    switch (N) {
+        case 2: bitonic_sort<1>(key, idx, sk, si, tid); break;
+        case 4: bitonic_sort<2>(key, idx, sk, si, tid); break;
+        case 8: bitonic_sort<3>(key, idx, sk, si, tid); break;
+        case 16: bitonic_sort<4>(key, idx, sk, si, tid); break;
+        case 32: bitonic_sort<5>(key, idx, sk, si, tid); break;
+        case 64: bitonic_sort<6>(key, idx, sk, si, tid); break;
+        case 128: bitonic_sort<7>(key, idx, sk, si, tid); break;
+        case 256: bitonic_sort<8>(key, idx, sk, si, tid); break;
+        case 512: bitonic_sort<9>(key, idx, sk, si, tid); break;
+        default: break;  // N = 1: nothing to sort
     }
     sk[tid] = key;
     si[tid] = idx;
