@@ -561,10 +561,11 @@ def test_channel_rms_normalisation(io, d, M, lengths, causal):
 @pytest.mark.parametrize("d", [32, 64])
 def test_channel_rms_normalisation_many_tiles(d):
     """The non-causal channel normalisation on the tensor-core statistics and scale-term passes with
-    more tiles than blocks (each block of a side takes several, some none) and ragged lengths that
-    end inside a tile; the scale term adds into dQ and dK, whose padded rows must stay zero."""
-    case = Case(3, 4, 1400, d, 8, 8, "bf16", False, seed=93, qkv_scale=1.0 / math.sqrt(d), lengths=[1400, 1029, 130],
-                with_grad=True)
+    more tiles than blocks (each block of a side takes several, some none), ragged lengths that end
+    inside a tile and an empty sequence; the scale term adds into dQ and dK, whose padded rows must
+    stay zero."""
+    case = Case(4, 4, 1400, d, 8, 8, "bf16", False, seed=93, qkv_scale=1.0 / math.sqrt(d),
+                lengths=[1400, 1029, 0, 130], with_grad=True)
     case.ch_rms_target = _median_channel_rms(case)
     lu = case.luna()
     O = to_host(case.run_fwd(lu))
