@@ -9,6 +9,8 @@
 // histograms of the channel-MLP parameters.
 #include <math.h>
 
+#include <type_traits>
+
 #include "luna_prof.cuh"
 #include "luna_simt_dev.cuh"
 
@@ -372,47 +374,38 @@ struct CompSum {
     }
 };
 
-// Sum of the per-block parameter-gradient partials, in the fixed order p = 0..nparts-1
-// per element: 64 elements per block, each summed by 8 threads over consecutive
-// eighths of the partials (8 loads in flight; fp32 partials in compensated fp32,
-// fp64 partials in fp64), then the eight parts combined in order in fp64.
-constexpr int kSumElems = 64, kSumSplit = 8;
+// Sum of the per-block parameter-gradient partials, in a fixed order per
+// element: 16 elements per block, each summed by 32 threads over consecutive
+// 32nds of the partials (fp32 partials in compensated fp32, fp64 partials in
+// fp64), then the 32 parts combined in order in fp64.  A thread issues up to 16
+// loads before its first add, so that a few hundred partials (the persistent
+// kernels' count) cost one round of memory latency.
+constexpr int kSumElems = 16, kSumSplit = 32, kSumBatch = 16;
 template <typename P>
 __global__ void __launch_bounds__(kSumElems * kSumSplit) k_grad_sum(const P *gpart, int nparts, int gsize,
                                                                     double *out) {
     __shared__ double part[kSumSplit][kSumElems];
+    grid_dependency_sync();
     const int el = threadIdx.x % kSumElems, q = threadIdx.x / kSumElems;
     const int e = blockIdx.x * kSumElems + el;
     const int p0 = (int)((long long)q * nparts / kSumSplit), p1 = (int)((long long)(q + 1) * nparts / kSumSplit);
-    if constexpr (sizeof(P) == 4) {
-        CompSum cs;
-        if (e < gsize) {
-            int p = p0;
-            for (; p + 8 <= p1; p += 8) {
-                float v[8];
+    using Acc = typename std::conditional<sizeof(P) == 4, CompSum, double>::type;
+    Acc acc{};
+    if (e < gsize) {
+        for (int p = p0; p < p1; p += kSumBatch) {
+            P v[kSumBatch];
 #pragma unroll
-                for (int k = 0; k < 8; ++k) v[k] = __ldcg(gpart + (size_t)(p + k) * gsize + e);
+            for (int k = 0; k < kSumBatch; ++k) v[k] = p + k < p1 ? __ldcg(gpart + (size_t)(p + k) * gsize + e) : P(0);
 #pragma unroll
-                for (int k = 0; k < 8; ++k) cs.add(v[k]);
+            for (int k = 0; k < kSumBatch; ++k) {
+                if (p + k >= p1) break;
+                if constexpr (sizeof(P) == 4) acc.add(v[k]);
+                else acc += v[k];
             }
-            for (; p < p1; ++p) cs.add(__ldcg(gpart + (size_t)p * gsize + e));
         }
-        part[q][el] = (double)cs.s + (double)cs.c;
-    } else {
-        double t = 0.0;
-        if (e < gsize) {
-            int p = p0;
-            for (; p + 8 <= p1; p += 8) {
-                double v[8];
-#pragma unroll
-                for (int k = 0; k < 8; ++k) v[k] = __ldcg(gpart + (size_t)(p + k) * gsize + e);
-#pragma unroll
-                for (int k = 0; k < 8; ++k) t += v[k];
-            }
-            for (; p < p1; ++p) t += __ldcg(gpart + (size_t)p * gsize + e);
-        }
-        part[q][el] = t;
     }
+    if constexpr (sizeof(P) == 4) part[q][el] = (double)acc.s + (double)acc.c;
+    else part[q][el] = acc;
     __syncthreads();
     if (q == 0 && e < gsize) {
         double t = part[0][el];
@@ -458,6 +451,25 @@ __global__ void __launch_bounds__(128) k_mlp_grads(TableLayout lay, const char *
     __shared__ double pre[2][kMaxUnits + 1], suf[2][kMaxUnits + 1];  // fp64: dw2 = w1 G1 + b1 G0 cancels
     const int Md = lay.M * lay.d, L = lay.L, hid = lay.hid, nint = lay.nint;
     const float scale = 1.0f / sqrtf((float)lay.M);
+    const int *rank = reinterpret_cast<const int *>(table + lay.off_rank);
+    const int *utype = reinterpret_cast<const int *>(table + lay.off_utype);
+    const float *w1 = reinterpret_cast<const float *>(table + lay.off_w1);
+    const float *b1 = reinterpret_cast<const float *>(table + lay.off_b1);
+    const float *w2 = reinterpret_cast<const float *>(table + lay.off_w2);
+    // The first hidden unit of each thread comes from the parameter table, which no kernel of the
+    // backward call writes: it is read before the wait for the histogram.
+    const bool hist_block = (int)blockIdx.x < L && !lay.act;
+    int r_first = 0, t_first = 0;
+    float w1_first = 0.0f, b1_first = 0.0f, w2_first = 0.0f;
+    if (hist_block && (int)threadIdx.x < hid) {
+        const int u = lay.shared ? threadIdx.x : blockIdx.x * hid + threadIdx.x, uw = blockIdx.x * hid + threadIdx.x;
+        r_first = rank[u];
+        t_first = utype[u];
+        w1_first = w1[u];
+        b1_first = b1[u];
+        w2_first = w2[uw];
+    }
+    grid_dependency_sync();
     if ((int)blockIdx.x == L) {
         for (int e = threadIdx.x; e < Md; e += blockDim.x) grads.dW[e] = (float)gsum[e];
         for (int e = threadIdx.x; e < lay.M; e += blockDim.x) grads.db[e] = (float)gsum[Md + e];
@@ -486,33 +498,43 @@ __global__ void __launch_bounds__(128) k_mlp_grads(TableLayout lay, const char *
         if (threadIdx.x == 0) grads.db2[l] = (float)hist[L * hid + 2 * P + l];
         return;
     }
-    for (int j = threadIdx.x; j < nint; j += blockDim.x) {
-        h[0][j] = hist[(j * L + l) * 2];
-        h[1][j] = hist[(j * L + l) * 2 + 1];
+    {  // the channel's histogram: every load issued before the first store
+        constexpr int kLd = (kMaxUnits + 1 + 127) / 128;
+        double v0[kLd], v1[kLd];
+#pragma unroll
+        for (int k = 0; k < kLd; ++k) {
+            const int j = threadIdx.x + 128 * k;
+            v0[k] = j < nint ? hist[(j * L + l) * 2] : 0.0;
+            v1[k] = j < nint ? hist[(j * L + l) * 2 + 1] : 0.0;
+        }
+#pragma unroll
+        for (int k = 0; k < kLd; ++k) {
+            const int j = threadIdx.x + 128 * k;
+            if (j < nint) { h[0][j] = v0[k]; h[1][j] = v1[k]; }
+        }
     }
     __syncthreads();
     const int warp = threadIdx.x >> 5;  // warps 0, 1: prefix of m0, m1; warps 2, 3: suffix
     warp_scan(h[warp & 1], (warp < 2 ? pre : suf)[warp & 1], nint, warp >= 2);
     __syncthreads();
-    const int *rank = reinterpret_cast<const int *>(table + lay.off_rank);
-    const int *utype = reinterpret_cast<const int *>(table + lay.off_utype);
-    const float *w1 = reinterpret_cast<const float *>(table + lay.off_w1);
-    const float *b1 = reinterpret_cast<const float *>(table + lay.off_b1);
-    const float *w2 = reinterpret_cast<const float *>(table + lay.off_w2);
     for (int k = threadIdx.x; k < hid; k += blockDim.x) {
         const int u = lay.shared ? k : l * hid + k;  // the unit: its kink and fc1
         const int uw = l * hid + k;                  // fc2 weight (l, k)
-        const int r = rank[u];
+        const bool first = k == (int)threadIdx.x;
+        const int r = first ? r_first : rank[u];
+        const bool above = (first ? t_first : utype[u]) > 0;
+        const double w1u = first ? w1_first : w1[u], b1u = first ? b1_first : b1[u];
+        const double w2u = first ? w2_first : w2[uw];
         double G0, G1;
-        if (utype[u] > 0) {  // active on intervals j > r
+        if (above) {  // active on intervals j > r
             G0 = r + 1 < nint ? suf[0][r + 1] : 0.0;
             G1 = r + 1 < nint ? suf[1][r + 1] : 0.0;
-        } else {             // active on intervals j <= r
+        } else {      // active on intervals j <= r
             G0 = pre[0][r];
             G1 = pre[1][r];
         }
-        grads.dw2[uw] = (float)(((double)w1[u] * G1 + (double)b1[u] * G0) * (double)scale);
-        const double c1 = (double)w2[uw] * G1 * (double)scale, c0 = (double)w2[uw] * G0 * (double)scale;
+        grads.dw2[uw] = (float)((w1u * G1 + b1u * G0) * (double)scale);
+        const double c1 = w2u * G1 * (double)scale, c0 = w2u * G0 * (double)scale;
         if (lay.shared) {
             fc1_part[(size_t)l * hid + k] = c1;
             fc1_part[(size_t)(L + l) * hid + k] = c0;
@@ -526,6 +548,7 @@ __global__ void __launch_bounds__(128) k_mlp_grads(TableLayout lay, const char *
 
 // Shared-channel MLP: dw1[k], db1[k] = sums over the channels (in order) of their contributions.
 __global__ void __launch_bounds__(128) k_mlp_fc1_sum(TableLayout lay, const double *fc1_part, luna_phi_grads grads) {
+    grid_dependency_sync();
     const int L = lay.L, hid = lay.hid;
     for (int k = threadIdx.x; k < hid; k += blockDim.x) {
         double a = 0.0, b = 0.0;
@@ -617,19 +640,23 @@ size_t simt_max_smem(const AttnArgs &a) {
 
 cudaError_t launch_grad_reduce(const AttnArgs &a, int nparts, cudaStream_t s) {
     const int nb = (a.gsize + kSumElems - 1) / kSumElems;
+    const bool dep = !a.ch_sigma;
     if (a.gpart64)
-        LUNA_LAUNCH("grad_sum", k_grad_sum<double>, nb, kSumElems * kSumSplit, 0, s,
-                    reinterpret_cast<const double *>(a.gpart), nparts, a.gsize, a.hist);
+        LUNA_LAUNCH_DEP("grad_sum", dep, k_grad_sum<double>, nb, kSumElems * kSumSplit, 0, s,
+                        reinterpret_cast<const double *>(a.gpart), nparts, a.gsize, a.hist);
     else
-        LUNA_LAUNCH("grad_sum", k_grad_sum<float>, nb, kSumElems * kSumSplit, 0, s, a.gpart, nparts, a.gsize, a.hist);
+        LUNA_LAUNCH_DEP("grad_sum", dep, k_grad_sum<float>, nb, kSumElems * kSumSplit, 0, s,
+                        static_cast<const float *>(a.gpart), nparts, a.gsize, a.hist);
     cudaError_t e = cudaGetLastError();
     if (e != cudaSuccess) return e;
     if ((e = launch_chrms_hist(a, s)) != cudaSuccess) return e;
     // the partials have been summed: their buffer holds the shared MLP's per-channel fc1 terms
     double *fc1_part = reinterpret_cast<double *>(a.gpart);
-    LUNA_LAUNCH("mlp_grads", k_mlp_grads, a.lay.L + 1, 128, 0, s, a.lay, a.table, a.hist, a.grads, fc1_part);
+    LUNA_LAUNCH_DEP("mlp_grads", dep, k_mlp_grads, a.lay.L + 1, 128, 0, s, a.lay, a.table,
+                    static_cast<const double *>(a.hist), a.grads, fc1_part);
     if ((e = cudaGetLastError()) != cudaSuccess || !a.lay.shared || a.lay.act) return e;
-    LUNA_LAUNCH("mlp_fc1_sum", k_mlp_fc1_sum, 1, 128, 0, s, a.lay, fc1_part, a.grads);
+    LUNA_LAUNCH_DEP("mlp_fc1_sum", dep, k_mlp_fc1_sum, 1, 128, 0, s, a.lay, static_cast<const double *>(fc1_part),
+                    a.grads);
     return cudaGetLastError();
 }
 

@@ -203,7 +203,6 @@ __global__ void __launch_bounds__(kThreadsTC, 1)
     int *slast = reinterpret_cast<int *>(tslot + 1);
 
     const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
-    const Items it(a);
     const bool per_item = a.seg_S != nullptr;
 
     if (tid == 0) {
@@ -216,6 +215,8 @@ __global__ void __launch_bounds__(kThreadsTC, 1)
     }
     if (warp == 0) { tmem_alloc(tslot, C::TMEM_K); tmem_relinquish(); }
     stage_phi_table<C>(a, sTe, sAB, sbias, Wop);
+    grid_dependency_sync();  // the work split and the counters are read from here on
+    const Items it(a);
     fence_proxy_async_smem();
     tc_fence_before();
     __syncthreads();
@@ -469,7 +470,6 @@ __global__ void __launch_bounds__(kThreadsTC, 1)
     uint32_t *tslot = reinterpret_cast<uint32_t *>(numfree + NN);
 
     const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
-    const Items it(a);
 
     if (tid == 0) {
         for (int i = 0; i < NX; ++i) { mbar_init(fullx + i, 1); mbar_init(xfree + i, 1); }
@@ -480,6 +480,8 @@ __global__ void __launch_bounds__(kThreadsTC, 1)
     }
     if (warp == 0) { tmem_alloc(tslot, C::TMEM_Q); tmem_relinquish(); }
     stage_phi_table<C>(a, sTe, sAB, sbias, Wop);
+    grid_dependency_sync();  // the key statistics and the work split are read from here on
+    const Items it(a);
     // padded rows of every item of this block produce zeros (unless the split kernel zeroed them)
     for (int item = it.begin; item < it.end && !a.padded_zeroed; ++item) {
         const ItemRange ir = item_range(a, it, item);
@@ -726,6 +728,7 @@ constexpr int kSplitItems = 12 * 1024;
 // Blocks 1.. of the launch zero the rows past each sequence's length of the outputs in zmask (1: O, 2: dQ,
 // 4: dK, 8: dV), head by head with the whole GPU's store bandwidth, so that the persistent kernels skip it.
 __global__ void __launch_bounds__(kSplitThreads) k_tile_split(AttnArgs a, int G, int zmask) {
+    grid_dependency_sync();
     if (blockIdx.x > 0) {
         const int Z = gridDim.x - 1;
         for (int bh = blockIdx.x - 1; bh < a.B * a.H; bh += Z) {
@@ -860,7 +863,7 @@ AttnArgs balanced_impl(const AttnArgs &a0, cudaStream_t s, cudaError_t *err, int
         (*err = cudaFuncSetAttribute(k_tile_split, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem)) != cudaSuccess)
         return a;
     const int zblocks = zmask ? std::min(a.B * a.H, sm_count_impl()) : 0;
-    LUNA_LAUNCH("tile_split", k_tile_split, 1 + zblocks, kSplitThreads, smem, s, a, G, zmask);
+    LUNA_LAUNCH_DEP("tile_split", !a.ch_sigma, k_tile_split, 1 + zblocks, kSplitThreads, smem, s, a, G, zmask);
     if ((*err = cudaGetLastError()) != cudaSuccess) return a;
     a.split = a.items_ws;
     a.runs = a.split + kMaxGrid + 1;
@@ -876,7 +879,7 @@ cudaError_t keys_tc(const AttnArgs &a, cudaStream_t s) {
         return cudaErrorInvalidValue;
     cudaError_t e = cudaFuncSetAttribute(k_tc_keys<C>, cudaFuncAttributeMaxDynamicSharedMemorySize, C::SMEM_K);
     if (e != cudaSuccess) return e;
-    LUNA_LAUNCH("tc_keys", k_tc_keys<C>, grid_impl(a), kThreadsTC, C::SMEM_K, s, mK, mV, a, status_word(a));
+    LUNA_LAUNCH_DEP("tc_keys", !a.ch_sigma, k_tc_keys<C>, grid_impl(a), kThreadsTC, C::SMEM_K, s, mK, mV, a, status_word(a));
     return cudaGetLastError();
 }
 
@@ -891,7 +894,7 @@ cudaError_t fwd_tc(const AttnArgs &a0, cudaStream_t s) {
     if (!make_map_impl(&mQ, a.Q, a.d, a.n, a.B * a.H, 128, a.hs_mul)) return cudaErrorInvalidValue;
     e = cudaFuncSetAttribute(k_tc_query<C>, cudaFuncAttributeMaxDynamicSharedMemorySize, C::SMEM_Q);
     if (e != cudaSuccess) return e;
-    LUNA_LAUNCH("tc_query", k_tc_query<C>, grid_impl(a), kThreadsTC, C::SMEM_Q, s, mQ, a, status_word(a));
+    LUNA_LAUNCH_DEP("tc_query", !a.ch_sigma, k_tc_query<C>, grid_impl(a), kThreadsTC, C::SMEM_Q, s, mQ, a, status_word(a));
     return cudaGetLastError();
 }
 

@@ -153,7 +153,6 @@ __global__ void __launch_bounds__(kCThreads, 1)
     uint32_t *tslot = reinterpret_cast<uint32_t *>(bars + 11);
 
     const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
-    const Items it(a);
 
     if (tid == 0) {
         mbar_init(fullx, 1); mbar_init(xfree, 1); mbar_init(fullv, 1); mbar_init(vfree, 1);
@@ -165,6 +164,8 @@ __global__ void __launch_bounds__(kCThreads, 1)
     stage_phi_table<C>(a, sTe, sAB, sbias, Wop);
     for (int e = tid; e < (int)(C::ONES / 4); e += blockDim.x)
         reinterpret_cast<uint32_t *>(Ones)[e] = 0x3F803F80u;  // bf16 1.0 pairs
+    grid_dependency_sync();  // the segment prefixes are read, O written from here on
+    const Items it(a);
     // padded rows of every item get O = 0
     for (int item = it.begin; item < it.end; ++item) {
         const ItemRange ir = item_range(a, it, item);
@@ -429,6 +430,7 @@ __global__ void __launch_bounds__(kCThreads, 1)
 // Exclusive prefix of the segment statistics at every segment start, total last:
 // seg_S[bh][s] = sum_{s' < s} S_part[bh][s'] (s = 0 .. nseg), in segment order.
 __global__ void __launch_bounds__(256) k_seg_scan(AttnArgs a) {
+    grid_dependency_sync();
     const int bh = blockIdx.y;
     const size_t SD = (size_t)a.D * a.dv;
     const int e4 = blockIdx.x * blockDim.x + threadIdx.x;  // float4 position
@@ -474,7 +476,7 @@ cudaError_t launch_tc_causal_stats(const AttnArgs &a0, cudaStream_t s) {
     cudaError_t e = launch_tc_keys_items(a, s);
     if (e != cudaSuccess) return e;
     const size_t SD4 = (size_t)a.D * a.dv / 4;
-    LUNA_LAUNCH("seg_scan", k_seg_scan, dim3((unsigned)((SD4 + 255) / 256), a.B * a.H), 256, 0, s, a);
+    LUNA_LAUNCH_DEP("seg_scan", !a.ch_sigma, k_seg_scan, dim3((unsigned)((SD4 + 255) / 256), a.B * a.H), 256, 0, s, a);
     return cudaGetLastError();
 }
 
@@ -495,7 +497,7 @@ cudaError_t launch_tc_causal_fwd(const AttnArgs &a0, cudaStream_t s) {
     const int items = BH * a.nsplit;
     const int grid = items < tc_sm_count() ? items : tc_sm_count();
     int *st = reinterpret_cast<int *>(reinterpret_cast<char *>(a.counters) - 256);
-    LUNA_LAUNCH("tc_causal", k_tc_causal<C>, grid, kCThreads, C::SMEM, s, mQ, mK, mV, a, st);
+    LUNA_LAUNCH_DEP("tc_causal", !a.ch_sigma, k_tc_causal<C>, grid, kCThreads, C::SMEM, s, mQ, mK, mV, a, st);
     return cudaGetLastError();
 }
 
