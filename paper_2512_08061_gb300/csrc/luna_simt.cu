@@ -9,8 +9,6 @@
 // histograms of the channel-MLP parameters.
 #include <math.h>
 
-#include <type_traits>
-
 #include "luna_prof.cuh"
 #include "luna_simt_dev.cuh"
 
@@ -374,13 +372,11 @@ struct CompSum {
     }
 };
 
-// Sum of the per-block parameter-gradient partials, in a fixed order per
-// element: 16 elements per block, each summed by 32 threads over consecutive
-// 32nds of the partials (fp32 partials in compensated fp32, fp64 partials in
-// fp64), then the 32 parts combined in order in fp64.  A thread issues up to 16
-// loads before its first add, so that a few hundred partials (the persistent
-// kernels' count) cost one round of memory latency.
-constexpr int kSumElems = 16, kSumSplit = 32, kSumBatch = 16;
+// Sum of the per-block parameter-gradient partials, in the fixed order p = 0..nparts-1
+// per element: 64 elements per block, each summed by 8 threads over consecutive
+// eighths of the partials (8 loads in flight; fp32 partials in compensated fp32,
+// fp64 partials in fp64), then the eight parts combined in order in fp64.
+constexpr int kSumElems = 64, kSumSplit = 8;
 template <typename P>
 __global__ void __launch_bounds__(kSumElems * kSumSplit) k_grad_sum(const P *gpart, int nparts, int gsize,
                                                                     double *out) {
@@ -389,23 +385,35 @@ __global__ void __launch_bounds__(kSumElems * kSumSplit) k_grad_sum(const P *gpa
     const int el = threadIdx.x % kSumElems, q = threadIdx.x / kSumElems;
     const int e = blockIdx.x * kSumElems + el;
     const int p0 = (int)((long long)q * nparts / kSumSplit), p1 = (int)((long long)(q + 1) * nparts / kSumSplit);
-    using Acc = typename std::conditional<sizeof(P) == 4, CompSum, double>::type;
-    Acc acc{};
-    if (e < gsize) {
-        for (int p = p0; p < p1; p += kSumBatch) {
-            P v[kSumBatch];
+    if constexpr (sizeof(P) == 4) {
+        CompSum cs;
+        if (e < gsize) {
+            int p = p0;
+            for (; p + 8 <= p1; p += 8) {
+                float v[8];
 #pragma unroll
-            for (int k = 0; k < kSumBatch; ++k) v[k] = p + k < p1 ? __ldcg(gpart + (size_t)(p + k) * gsize + e) : P(0);
+                for (int k = 0; k < 8; ++k) v[k] = __ldcg(gpart + (size_t)(p + k) * gsize + e);
 #pragma unroll
-            for (int k = 0; k < kSumBatch; ++k) {
-                if (p + k >= p1) break;
-                if constexpr (sizeof(P) == 4) acc.add(v[k]);
-                else acc += v[k];
+                for (int k = 0; k < 8; ++k) cs.add(v[k]);
             }
+            for (; p < p1; ++p) cs.add(__ldcg(gpart + (size_t)p * gsize + e));
         }
+        part[q][el] = (double)cs.s + (double)cs.c;
+    } else {
+        double t = 0.0;
+        if (e < gsize) {
+            int p = p0;
+            for (; p + 8 <= p1; p += 8) {
+                double v[8];
+#pragma unroll
+                for (int k = 0; k < 8; ++k) v[k] = __ldcg(gpart + (size_t)(p + k) * gsize + e);
+#pragma unroll
+                for (int k = 0; k < 8; ++k) t += v[k];
+            }
+            for (; p < p1; ++p) t += __ldcg(gpart + (size_t)p * gsize + e);
+        }
+        part[q][el] = t;
     }
-    if constexpr (sizeof(P) == 4) part[q][el] = (double)acc.s + (double)acc.c;
-    else part[q][el] = acc;
     __syncthreads();
     if (q == 0 && e < gsize) {
         double t = part[0][el];

@@ -105,6 +105,7 @@ __global__ void __launch_bounds__(kBThreads, 1)
     static_assert((2 * NS + 2 * NO + 15) * 8 + 8 <= kBarBytes, "barrier area");
 
     const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+    const Items it(a);
     // TMEM: U [2 x 32] | P [2 x 128] | acc [2 x 64] | dQ [32] | dW^T (M = 64) [16]
     constexpr uint32_t cU = 0, cP = 64, cA = 320, cQ = 448, cW = 480;
 
@@ -127,8 +128,6 @@ __global__ void __launch_bounds__(kBThreads, 1)
     stage_wx<C>(a, Wop, 4);
     for (int e = tid; e < kNint * 16; e += blockDim.x) bins[e] = 0;
     for (int e = tid; e < C::MP * C::d + 16; e += blockDim.x) sdW[e] = 0.0f;
-    grid_dependency_sync();  // global memory is read and written from here on
-    const Items it(a);
     float *hpart = a.gpart + (size_t)blockIdx.x * a.gsize + C::MP * a.d + C::MP;  // histogram part of the partial
     for (int e = tid; e < a.lay.nint * 16; e += blockDim.x) hpart[e] = 0.0f;
     // padded rows of every item produce zero gradients (unless the split kernel zeroed them)
@@ -565,6 +564,7 @@ __global__ void __launch_bounds__(kBThreads, 1)
     static_assert((2 * NS + 2 * NV + 17) * 8 + 4 <= kBarBytes, "barrier area");
 
     const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+    const Items it(a);
     // TMEM: U [2 x 32] | dphi [2 x 128] | dV [2 x 64] | dK [32] | dW (M = 64) [16]
     constexpr uint32_t cU = 0, cF = 64, cV = 320, cK = 448, cW = 480;
 
@@ -588,8 +588,6 @@ __global__ void __launch_bounds__(kBThreads, 1)
     stage_wx<C>(a, Wop, 4);
     for (int e = tid; e < kNint * 16; e += blockDim.x) bins[e] = 0;
     for (int e = tid; e < C::MP * C::d + 16; e += blockDim.x) sdW[e] = 0.0f;
-    grid_dependency_sync();  // global memory is read and written from here on
-    const Items it(a);
     float *hpart = a.gpart + (size_t)(gridDim.x + blockIdx.x) * a.gsize + C::MP * a.d + C::MP;
     for (int e = tid; e < a.lay.nint * 16; e += blockDim.x) hpart[e] = 0.0f;
     for (int e = tid; e < (int)(T16 / 16); e += blockDim.x) reinterpret_cast<uint4 *>(Gt)[e] = make_uint4(0, 0, 0, 0);
@@ -922,10 +920,10 @@ cudaError_t bwd_tc(const AttnArgs &a0, bool have_stats, cudaStream_t s) {
         cudaSuccess)
         return e;
     int *st = reinterpret_cast<int *>(reinterpret_cast<char *>(a.counters) - 256);
-    LUNA_LAUNCH_DEP("tc_bwd_query", !a.ch_sigma, k_tc_bwd_query<C>, grid, kBThreads, C::SMEM_Q, s, mQ, mdO, a, st);
+    LUNA_LAUNCH("tc_bwd_query", k_tc_bwd_query<C>, grid, kBThreads, C::SMEM_Q, s, mQ, mdO, a, st);
     if ((e = cudaGetLastError()) != cudaSuccess) return e;
     if ((e = launch_chrms_dstate(a, s)) != cudaSuccess) return e;
-    LUNA_LAUNCH_DEP("tc_bwd_key", !a.ch_sigma, k_tc_bwd_key<C>, grid, kBThreads, C::SMEM_K, s, mK, mV, a, st);
+    LUNA_LAUNCH("tc_bwd_key", k_tc_bwd_key<C>, grid, kBThreads, C::SMEM_K, s, mK, mV, a, st);
     if ((e = cudaGetLastError()) != cudaSuccess) return e;
     int nparts = 0;
     if ((e = launch_chrms_backward(a, 2 * grid, &nparts, s)) != cudaSuccess) return e;

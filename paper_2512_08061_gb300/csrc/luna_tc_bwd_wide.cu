@@ -95,6 +95,7 @@ __global__ void __launch_bounds__(kBThreads, 1)
     static_assert((2 * NS + 2 * NO + 13) * 8 + 8 <= kBarBytes, "barrier area");
 
     const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+    const Items it(a);
     // TMEM: U [2 x 32] | P [128] | dS [2 x 64] | dz [2 x 16] | dQ [64] | dW^T (M = 64) [16]
     constexpr uint32_t cU = 0, cP = 64, cA = 192, cZ = 320, cQ = 352, cW = 416;
 
@@ -115,8 +116,6 @@ __global__ void __launch_bounds__(kBThreads, 1)
     for (int e = tid; e < kNint * 16; e += blockDim.x) bins[e] = 0;
     for (int e = tid; e < C::MP * C::d + 16; e += blockDim.x) sdW[e] = 0.0f;
     for (int e = tid; e < (int)(T16 / 16); e += blockDim.x) reinterpret_cast<uint4 *>(Gt)[e] = make_uint4(0, 0, 0, 0);
-    grid_dependency_sync();  // global memory is read and written from here on
-    const Items it(a);
     float *hpart = a.gpart + (size_t)blockIdx.x * a.gsize + C::MP * a.d + C::MP;
     for (int e = tid; e < a.lay.nint * 16; e += blockDim.x) hpart[e] = 0.0f;
     for (int item = it.begin; item < it.end && !a.padded_zeroed; ++item) {  // padded rows: zero gradients
@@ -555,6 +554,7 @@ __global__ void __launch_bounds__(kBThreads, 1)
     static_assert((2 * NS + 16) * 8 + 4 <= kBarBytes, "barrier area");
 
     const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+    const Items it(a);
     // TMEM: U [2 x 32] | dphi [128] | dV [128] | dK [64] | dW (M = 64) [16]
     constexpr uint32_t cU = 0, cF = 64, cV = 192, cK = 320, cW = 384;
 
@@ -575,8 +575,6 @@ __global__ void __launch_bounds__(kBThreads, 1)
     for (int e = tid; e < kNint * 16; e += blockDim.x) bins[e] = 0;
     for (int e = tid; e < C::MP * C::d + 16; e += blockDim.x) sdW[e] = 0.0f;
     for (int e = tid; e < (int)(T16 / 16); e += blockDim.x) reinterpret_cast<uint4 *>(Gt)[e] = make_uint4(0, 0, 0, 0);
-    grid_dependency_sync();  // global memory is read and written from here on
-    const Items it(a);
     float *hpart = a.gpart + (size_t)(gridDim.x + blockIdx.x) * a.gsize + C::MP * a.d + C::MP;
     for (int e = tid; e < a.lay.nint * 16; e += blockDim.x) hpart[e] = 0.0f;
     for (int item = it.begin; item < it.end && !a.padded_zeroed; ++item) {  // padded rows: zero gradients
@@ -897,10 +895,10 @@ cudaError_t launch_tc_bwd_wide(const AttnArgs &a0, bool have_stats, cudaStream_t
         cudaSuccess)
         return e;
     int *st = reinterpret_cast<int *>(reinterpret_cast<char *>(a.counters) - 256);
-    LUNA_LAUNCH_DEP("tc_bwd_query", !a.ch_sigma, k_tc_bwd_query_w<C>, grid, kBThreads, C::SMEM_Q, s, mQ, mdO, a, st);
+    LUNA_LAUNCH("tc_bwd_query", k_tc_bwd_query_w<C>, grid, kBThreads, C::SMEM_Q, s, mQ, mdO, a, st);
     if ((e = cudaGetLastError()) != cudaSuccess) return e;
     if ((e = launch_chrms_dstate(a, s)) != cudaSuccess) return e;
-    LUNA_LAUNCH_DEP("tc_bwd_key", !a.ch_sigma, k_tc_bwd_key_w<C>, grid, kBThreads, C::SMEM_K, s, mK, mV, a, st);
+    LUNA_LAUNCH("tc_bwd_key", k_tc_bwd_key_w<C>, grid, kBThreads, C::SMEM_K, s, mK, mV, a, st);
     if ((e = cudaGetLastError()) != cudaSuccess) return e;
     int nparts = 0;
     if ((e = launch_chrms_backward(a, 2 * grid, &nparts, s)) != cudaSuccess) return e;
